@@ -1,0 +1,105 @@
+"""Seeded synthetic inputs shared by the tests, the benchmark and the smoke check.
+
+This module only draws random numbers and lays them out; it holds none of the
+mixing layer's arithmetic (no partner rule, no products, no sums), so that the
+device path and the CPU oracle can be fed identical inputs without sharing
+any code that computes the method.
+
+Recipes (the paper's corpora are not available; these stand in for their
+shapes, which is all the mixing cost depends on):
+
+* activations x ~ N(0, 1);
+* weights W_self, W_nbr ~ N(0, 1/d) for the tiny check and N(0, 1/(2d)) for
+  the timed stacks (keeps the activation scale steady over 16 layers);
+* bias ~ N(0, 0.1^2);
+* character-LM ids: Zipf(1.1) over a byte vocabulary of 256 (rank r has
+  probability proportional to r^-1.1, rank r is byte r-1), embedded through
+  an N(0, 1) table [256, d];
+* reachability ids: uniform over 16 symbols, embedded through [16, d].
+
+All host draws use numpy's PCG64 with an explicit seed.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+
+import numpy as np
+
+
+def rng(seed: int) -> np.random.Generator:
+    return np.random.Generator(np.random.PCG64(seed))
+
+
+def normal(shape, seed: int, std: float = 1.0) -> np.ndarray:
+    return (rng(seed).standard_normal(shape) * std).astype(np.float32)
+
+
+def zipf_ids(B: int, n: int, seed: int, vocab: int = 256, alpha: float = 1.1) -> np.ndarray:
+    ranks = np.arange(1, vocab + 1, dtype=np.float64)
+    p = ranks ** (-alpha)
+    p /= p.sum()
+    return rng(seed).choice(vocab, size=(B, n), p=p).astype(np.int64)
+
+
+def uniform_ids(B: int, n: int, seed: int, vocab: int = 16) -> np.ndarray:
+    return rng(seed).integers(0, vocab, size=(B, n)).astype(np.int64)
+
+
+def embed(ids: np.ndarray, table: np.ndarray) -> np.ndarray:
+    """Row lookup table[ids] (input preparation, not part of the mixing path)."""
+    return table[ids]
+
+
+@dataclass
+class Problem:
+    """Seeded inputs of a stack of L mixing layers (float32, not yet rounded)."""
+    x: np.ndarray          # [B, n, d]
+    W_self: np.ndarray     # [L, d, d]  (d_out, d_in)
+    W_nbr: np.ndarray      # [L, d, d]
+    bias: np.ndarray       # [L, d]
+    dy: np.ndarray         # [B, n, d]  upstream gradient for backward checks
+    z: np.ndarray = field(default=None)  # [L, B, n, d] pre-activations for layer-level bwd checks
+
+
+def problem(B: int, n: int, d: int, L: int = 1, seed: int = 0, w_std: float | None = None,
+            bias_std: float = 0.1, x_ids: str | None = None) -> Problem:
+    """Draw one seeded problem.  ``x_ids`` selects token-id inputs
+    ("zipf256" or "uniform16") embedded through an N(0,1) table instead of
+    x ~ N(0,1)."""
+    if w_std is None:
+        w_std = (1.0 / d) ** 0.5
+    if x_ids == "zipf256":
+        ids = zipf_ids(B, n, seed + 11)
+        x = embed(ids, normal((256, d), seed + 12))
+    elif x_ids == "uniform16":
+        ids = uniform_ids(B, n, seed + 11)
+        x = embed(ids, normal((16, d), seed + 12))
+    else:
+        x = normal((B, n, d), seed + 1)
+    return Problem(
+        x=np.ascontiguousarray(x, dtype=np.float32),
+        W_self=normal((L, d, d), seed + 2, w_std),
+        W_nbr=normal((L, d, d), seed + 3, w_std),
+        bias=normal((L, d), seed + 4, bias_std),
+        dy=normal((B, n, d), seed + 5),
+        z=normal((L, B, n, d), seed + 6),
+    )
+
+
+def to_bf16_exact(a: np.ndarray):
+    """Round a float32 array to bfloat16 (torch's conversion, ties to even)
+    and return (bf16 torch tensor on CPU, float64 numpy copy of its exact
+    values).  The oracle consumes the float64 copy so both sides see the
+    same numbers."""
+    import torch
+    t = torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(torch.bfloat16)
+    return t, t.to(torch.float64).numpy()
+
+
+# The workloads, by what they are.  Used by the benchmark and the tests.
+WORKLOADS = {
+    "tiny_n16_d32": dict(n=16, d=32, L=4, B=4, causal=False, w_std=(1 / 32) ** 0.5),
+    "reach_n64_d128": dict(n=64, d=128, L=6, B=256, causal=False, x_ids="uniform16"),
+    "charlm_w64_d512": dict(n=64, d=512, L=16, B=64, causal=True, x_ids="zipf256"),
+    "charlm_w256_d512": dict(n=256, d=512, L=16, B=64, causal=True, x_ids="zipf256"),
+}
