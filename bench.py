@@ -1,0 +1,488 @@
+#!/usr/bin/env python
+"""Throughput of the rotated-hypercube mixing stack on GB300, forward + backward.
+
+One step = hcw_stack_fwd + hcw_stack_bwd over one batch of the char-LM
+window-256 workload: B = 64 sequences of n = 256 positions, d = 512,
+16 rotated causal layers (dimensions 0..7 twice), residual, ReLU, bias, with
+per-layer weight gradients (Sec. 3.1 wiring, Eq. (1) maps).  Inputs are
+synthetic (Zipf(1.1) byte ids embedded to d; see paper_2609_18145_gb300.synth)
+and resident in HBM when the timed region starts; L2 is flushed (a 256 MiB
+write) before every timed step, outside the timed events.
+
+Prints ONE JSON line (rank 0).  --impl reference times the fp64 CPU oracle
+instead (the reference arm of this build: there is no reference code).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+  torchrun --nproc-per-node N bench.py --gpus N ...   (N independent replicas)
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "HypercubeMix fwd+bwd tokens/s at n=256,d=512 bf16; % of roofline"
+WORKLOAD = "charlm_w256_d512"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+L2_FLUSH_BYTES = 256 << 20
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return p, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def workload():
+    from paper_2609_18145_gb300 import synth
+    w = dict(synth.WORKLOADS[WORKLOAD])
+    w["flags"] = 1 | 2 | 4          # causal, residual, ReLU
+    return w
+
+
+def step_flops(B, n, d, L):
+    """Algorithmic flops of one fwd+bwd step (causal): per token and layer
+    3d^2 forward (half the positions use both maps), 3d^2 input gradient,
+    3d^2 weight gradients (flop = 2 MAC)."""
+    return 9.0 * d * d * B * n * L
+
+
+class ClockSampler:
+    """nvidia-smi sampled every 200 ms while a timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, local_rank: int):
+        vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+        ids = [v.strip() for v in vis.split(",")] if vis else []
+        self.gpu = ids[local_rank] if local_rank < len(ids) else str(local_rank)
+        self.proc = None
+        self.file = None
+
+    def __enter__(self):
+        try:
+            self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.FIELDS,
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.file, stderr=subprocess.DEVNULL)
+        except (OSError, ValueError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if self.proc is None or self.file is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.file.flush()
+        rows = []
+        with open(self.file.name) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.file.name)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+
+        def num(v):
+            try:
+                return float(v)
+            except ValueError:
+                return None
+
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        mx = [num(r[2]) for r in rows if num(r[2]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i] == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons,
+                "samples": len(rows)}
+
+
+def kernel_source_sha():
+    h = hashlib.sha256()
+    for f in ("hcw_tc.cu", "hcw_ptx.cuh", "hcw_api.cu"):
+        with open(os.path.join(ROOT, "paper_2609_18145_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(kernel: str):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, or None
+    when the kernel sources changed since those counters were taken."""
+    path = os.path.join(ROOT, "profiles", "dram_traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except (OSError, ValueError):
+        return None
+    e = rec.get(kernel)
+    if not e or e.get("src_sha") != kernel_source_sha():
+        return None
+    return e.get("bytes_per_launch")
+
+
+# ---------------------------------------------------------------- oracle timing
+
+def time_oracle(w, seconds_target: float, seed: int = 0, max_seqs: int = 64):
+    """Time the fp64 oracle's stack forward + backward on a bounded sample of
+    the workload (whole sequences); returns (tokens/s, seconds, sequences, threads)."""
+    from oracle import oracle as O
+    from paper_2609_18145_gb300 import synth
+    n, d, L = w["n"], w["d"], w["L"]
+
+    def run(seqs):
+        pr = synth.problem(seqs, n, d, L=L, seed=seed, w_std=(1 / (2 * d)) ** 0.5,
+                           x_ids="zipf256")
+        _, x = synth.to_bf16_exact(pr.x)
+        _, Ws = synth.to_bf16_exact(pr.W_self)
+        _, Wn = synth.to_bf16_exact(pr.W_nbr)
+        _, dy = synth.to_bf16_exact(pr.dy)
+        t0 = time.perf_counter()
+        _, acts, zs = O.stack_fwd(x, Ws, Wn, pr.bias.astype(np.float64), 0, L, -1, w["flags"],
+                                  round_bf16=True)
+        O.stack_bwd(acts, zs, dy, Ws, Wn, 0, L, -1, w["flags"], round_bf16=True)
+        return time.perf_counter() - t0
+
+    t1 = run(1)
+    seqs = 1
+    total = t1
+    if t1 < seconds_target:
+        seqs = int(min(max_seqs, max(1, round(seconds_target / max(t1, 1e-3)))))
+        if seqs > 1:
+            total = run(seqs)
+    return seqs * n / total, total, seqs, O.num_threads()
+
+
+# ---------------------------------------------------------------- reference arm
+
+def run_reference(args):
+    from paper_2609_18145_gb300 import replicas
+    rank, _, world = replicas.env_world()
+    if rank != 0:
+        return 0
+    w = workload()
+    n, d, L = w["n"], w["d"], w["L"]
+    from oracle import oracle as O
+    from paper_2609_18145_gb300 import synth
+    # one bounded sample per step: whole sequences, sized to about 2 s of CPU work
+    _, t1, seqs, threads = time_oracle(w, 2.0, max_seqs=8)
+    pr = synth.problem(seqs, n, d, L=L, seed=0, w_std=(1 / (2 * d)) ** 0.5, x_ids="zipf256")
+    _, x = synth.to_bf16_exact(pr.x)
+    _, Ws = synth.to_bf16_exact(pr.W_self)
+    _, Wn = synth.to_bf16_exact(pr.W_nbr)
+    _, dy = synth.to_bf16_exact(pr.dy)
+    bias = pr.bias.astype(np.float64)
+
+    def step():
+        _, acts, zs = O.stack_fwd(x, Ws, Wn, bias, 0, L, -1, w["flags"], round_bf16=True)
+        O.stack_bwd(acts, zs, dy, Ws, Wn, 0, L, -1, w["flags"], round_bf16=True)
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    el = time.perf_counter() - t0
+    tokens = seqs * n
+    value = tokens * args.steps / el
+    sample = "%d sequence(s) of n=%d (of the 64-sequence batch) per step, 16 layers fwd+bwd" % (
+        seqs, n)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * el / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "n": n, "d": d, "layers": L, "batch": w["B"],
+                   "sample_sequences_per_step": seqs, "causal": True, "residual": True,
+                   "act": "relu", "bias": True},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads,
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------- our arm
+
+def run_ours(args):
+    import torch
+
+    from paper_2609_18145_gb300 import hcw as H
+    from paper_2609_18145_gb300 import replicas, synth
+
+    rank, local_rank, world = replicas.env_world()
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU (the compute path has no CPU fallback)")
+    torch.cuda.set_device(local_rank)
+    replicas.init("nccl")
+    dev = torch.device("cuda", local_rank)
+    H.lib()
+
+    w = workload()
+    B, n, d, L, flags = w["B"], w["n"], w["d"], w["L"], w["flags"]
+    tokens = B * n
+    peaks, peak_src = load_peaks()
+
+    # ---- inputs: weights shared by all replicas, activations per rank
+    wstd = (1 / (2 * d)) ** 0.5
+    pw = synth.problem(1, n, d, L=L, seed=0, w_std=wstd)
+    px = synth.problem(B, n, d, L=1, seed=replicas.batch_seed(0, rank), x_ids="zipf256")
+    x = torch.from_numpy(px.x).to(torch.bfloat16).to(dev)
+    dy = torch.from_numpy(px.dy).to(torch.bfloat16).to(dev)
+    Ws = torch.from_numpy(pw.W_self).to(torch.bfloat16).to(dev)
+    Wn = torch.from_numpy(pw.W_nbr).to(torch.bfloat16).to(dev)
+    bias = torch.from_numpy(pw.bias).to(dev)
+    act_shape = (L - 1, B, n, d)
+    y = torch.empty_like(x)
+    acts = torch.empty(act_shape, dtype=torch.bfloat16, device=dev)
+    zs = torch.empty((L, B, n, d), dtype=torch.bfloat16, device=dev)
+    dx = torch.empty_like(x)
+    gWs = torch.empty((L, d, d), dtype=torch.float32, device=dev)
+    gWn = torch.empty((L, d, d), dtype=torch.float32, device=dev)
+    gb = torch.empty((L, d), dtype=torch.float32, device=dev)
+    ws = torch.empty(H.hcw_stack_workspace_bytes(B, n, d, H.HCW_BF16, flags), dtype=torch.uint8,
+                     device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(xin, dyin):
+        H.hcw_stack_fwd(xin, Ws, Wn, bias, 0, -1, flags, y=y, acts=acts, zs=zs)
+        H.hcw_stack_bwd(xin, acts, zs, dyin, Ws, Wn, 0, -1, flags, dx=dx, dW_self=gWs,
+                        dW_nbr=gWn, dbias=gb, workspace=ws)
+
+    for _ in range(args.warmup):
+        step(x, dy)
+    if H.hcw_sync_status() != H.HCW_OK:
+        raise SystemExit("device error during warm-up")
+
+    # ---- timed region: K steps, device time by CUDA events, L2 flushed before each
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    replicas.barrier()
+    torch.cuda.synchronize()
+    launches0 = H.hcw_launch_count()
+    with ClockSampler(local_rank) as clk:
+        for i in range(args.steps):
+            flush.fill_(i & 0xFF)
+            starts[i].record(stream)
+            step(x, dy)
+            ends[i].record(stream)
+        torch.cuda.synchronize()
+    launches = H.hcw_launch_count() - launches0
+    replicas.barrier()
+    if H.hcw_sync_status() != H.HCW_OK:
+        raise SystemExit("device error during the timed region")
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    ms_local = sum(step_ms) / len(step_ms)
+    ms = replicas.max_over_ranks(ms_local, dev)
+    value = world * tokens / (ms * 1e-3)
+    clocks = clk.summary()
+
+    # ---- per-kernel device time (each kernel kind launched alone, same inputs)
+    def time_calls(fn, reps):
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(reps)]
+        for i in range(reps):
+            flush.fill_(i & 0xFF)
+            evs[i][0].record(stream)
+            fn(i)
+            evs[i][1].record(stream)
+        torch.cuda.synchronize()
+        return sum(a.elapsed_time(b) for a, b in evs) / reps
+
+    dz = dy   # a layer's pre-activation gradient has the activations' shape and scale
+    fwd_ms = time_calls(lambda i: H.hcw_layer_fwd(x, Ws[i % L], Wn[i % L], bias[i % L], i % L,
+                                                  -1, flags, y=y, z_save=zs[0]), 2 * L)
+    dx_ms = time_calls(lambda i: H.hcw_layer_bwd_data(dz, dy, Ws[i % L], Wn[i % L], i % L, -1,
+                                                      flags, dx=dx), 2 * L)
+    wws = torch.empty(H.hcw_layer_bwd_weight_workspace_bytes(B, n, d, H.HCW_BF16, flags),
+                      dtype=torch.uint8, device=dev)
+    dw_ms = time_calls(lambda i: H.hcw_layer_bwd_weight(x, dz, i % L, -1, flags,
+                                                        dW_self=gWs[0], dW_nbr=gWn[0],
+                                                        want_dbias=False, workspace=wws), 2 * L)
+    layer_flops = 3.0 * d * d * tokens          # per kernel launch (causal)
+    kernels = {"hcw_tc_kernel<FWD,256>": fwd_ms, "hcw_tc_kernel<DX,256>": dx_ms,
+               "dW (hcw_tc_kernel<DW,256> + split reduce)": dw_ms}
+    dominant = max(kernels, key=kernels.get)
+    dom_ms = kernels[dominant]
+    peak = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
+    achieved = layer_flops / (dom_ms * 1e-3) / 1e12
+    step_tflops = step_flops(B, n, d, L) / (ms * 1e-3) / 1e12
+    peak_sus = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    traffic = recorded_traffic(dominant)
+
+    # ---- end to end through the public API with host buffers
+    x_h = torch.empty(x.shape, dtype=x.dtype, pin_memory=True)
+    dy_h = torch.empty(dy.shape, dtype=dy.dtype, pin_memory=True)
+    x_h.copy_(x)
+    dy_h.copy_(dy)
+    gWs_h = torch.empty(gWs.shape, dtype=gWs.dtype, pin_memory=True)
+    gWn_h = torch.empty(gWn.shape, dtype=gWn.dtype, pin_memory=True)
+    gb_h = torch.empty(gb.shape, dtype=gb.dtype, pin_memory=True)
+    x_d = torch.empty_like(x)
+    dy_d = torch.empty_like(dy)
+    h2d = x_h.numel() * x_h.element_size() + dy_h.numel() * dy_h.element_size()
+    d2h = sum(t.numel() * t.element_size() for t in (gWs_h, gWn_h, gb_h))
+    e2e_steps = max(3, args.steps // 2)
+    replicas.barrier()
+    torch.cuda.synchronize()
+    e_start = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
+    e_end = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
+    for i in range(e2e_steps):
+        flush.fill_(i & 0xFF)
+        e_start[i].record(stream)
+        x_d.copy_(x_h, non_blocking=True)
+        dy_d.copy_(dy_h, non_blocking=True)
+        step(x_d, dy_d)
+        gWs_h.copy_(gWs, non_blocking=True)
+        gWn_h.copy_(gWn, non_blocking=True)
+        gb_h.copy_(gb, non_blocking=True)
+        e_end[i].record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = replicas.max_over_ranks(
+        sum(a.elapsed_time(b) for a, b in zip(e_start, e_end)) / e2e_steps, dev)
+    e2e_value = world * tokens / (e2e_ms * 1e-3)
+
+    # ---- the oracle on the host cores, bounded sample (rank 0, N = 1 only)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        v, secs, seqs, threads = time_oracle(w, 10.0)
+        cpu = {"value": v, "unit": "tokens/s", "cores": threads, "kind": "oracle",
+               "sample": "%d of the 64 sequences (n=256), 16 layers fwd+bwd, fp64, %.1f s"
+                         % (seqs, secs)}
+
+    replicas.barrier()
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic",
+            "config": {"workload": WORKLOAD, "n": n, "d": d, "layers": L, "batch": B,
+                       "tokens_per_step_per_gpu": tokens, "causal": True, "residual": True,
+                       "act": "relu", "bias": True,
+                       "l2": "flushed before every timed step (256 MiB write, untimed)",
+                       "parallelism": "replicas" if world > 1 else "single"},
+            "roofline": {"bound": "tensor", "kernel": dominant, "achieved": achieved,
+                         "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                         "traffic": traffic, "peak_source": peak_src + " bf16 burst",
+                         "flops_per_launch": layer_flops, "avg_launch_ms": dom_ms,
+                         "kernel_ms": kernels},
+            "step_roofline": {"achieved": step_tflops, "peak": peak_sus, "unit": "TFLOP/s",
+                              "frac": step_tflops / peak_sus,
+                              "peak_source": peak_src + " bf16 sustained",
+                              "flops_per_step": step_flops(B, n, d, L)},
+            "cpu_baseline": cpu,
+            "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
+            "gpu_launches": launches,
+            "clocks": clocks,
+        }
+        print(json.dumps(line), flush=True)
+    replicas.finish()
+    return 0
+
+
+def run_kernel_only(args):
+    """Launch one kernel kind alone (for profiler captures): the layer
+    forward, input-gradient or weight-gradient pass of the workload's shape
+    with --batch sequences, --warmup untimed and --steps timed launches."""
+    import torch
+
+    from paper_2609_18145_gb300 import hcw as H
+    from paper_2609_18145_gb300 import synth
+
+    w = workload()
+    B, n, d, flags = args.batch, w["n"], w["d"], w["flags"]
+    dev = torch.device("cuda", 0)
+    H.lib()
+    pr = synth.problem(B, n, d, L=1, seed=0, w_std=(1 / (2 * d)) ** 0.5, x_ids="zipf256")
+    x = torch.from_numpy(pr.x).to(torch.bfloat16).to(dev)
+    dz = torch.from_numpy(pr.dy).to(torch.bfloat16).to(dev)
+    Ws = torch.from_numpy(pr.W_self[0]).to(torch.bfloat16).to(dev)
+    Wn = torch.from_numpy(pr.W_nbr[0]).to(torch.bfloat16).to(dev)
+    bias = torch.from_numpy(pr.bias[0]).to(dev)
+    y = torch.empty_like(x)
+    z = torch.empty_like(x)
+    gWs = torch.empty((d, d), dtype=torch.float32, device=dev)
+    gWn = torch.empty_like(gWs)
+    wws = torch.empty(max(1, H.hcw_layer_bwd_weight_workspace_bytes(B, n, d, H.HCW_BF16, flags)),
+                      dtype=torch.uint8, device=dev)
+    layer = 3
+    if args.kernel == "fwd":
+        fn = lambda: H.hcw_layer_fwd(x, Ws, Wn, bias, layer, -1, flags, y=y, z_save=z)
+    elif args.kernel == "dx":
+        fn = lambda: H.hcw_layer_bwd_data(dz, dz, Ws, Wn, layer, -1, flags, dx=y)
+    else:
+        fn = lambda: H.hcw_layer_bwd_weight(x, dz, layer, -1, flags, dW_self=gWs, dW_nbr=gWn,
+                                            want_dbias=False, workspace=wws)
+    for _ in range(args.warmup):
+        fn()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(args.steps):
+        fn()
+    b.record()
+    torch.cuda.synchronize()
+    if H.hcw_sync_status() != H.HCW_OK:
+        raise SystemExit("device error")
+    ms = a.elapsed_time(b) / args.steps
+    print(json.dumps({"kernel": args.kernel, "batch": B, "n": n, "d": d, "avg_ms": ms,
+                      "tflops": 3.0 * d * d * B * n / (ms * 1e-3) / 1e12}), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--no-cpu-baseline", action="store_true",
+                    help="skip timing the CPU oracle (it is only timed at N = 1 anyway)")
+    ap.add_argument("--kernel", choices=("fwd", "dx", "dw"),
+                    help="launch only this kernel kind (profiler captures); no JSON bench line")
+    ap.add_argument("--batch", type=int, default=64, help="sequences for --kernel runs")
+    args = ap.parse_args()
+    if args.kernel:
+        return run_kernel_only(args)
+    if args.warmup < 3:
+        ap.error("--warmup must be at least 3")
+    if args.steps < 1:
+        ap.error("--steps must be at least 1")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

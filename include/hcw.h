@@ -1,0 +1,210 @@
+/*
+ * hcw.h -- C ABI of the rotated-hypercube mixing layer on GB300 (sm_103a).
+ *
+ * Method (arXiv 2609.18145, "Reaching Every Position Without Searching"):
+ *   Sec. 3.1  positions i = 0..n-1 of a sample (n = 2^b) are vertices of a
+ *             b-cube; layer l links i with its partner p(i) = i XOR 2^s,
+ *             s = l mod b.  Causal rule: only the earlier endpoint is kept,
+ *             so i receives from p(i) iff bit s of i is set (p(i) = i - 2^s).
+ *   Eq. (1)   y_i = W_self x_i + W_off x_{i-k}: two d x d linear maps, no
+ *             input-dependent routing.  W_off is called W_nbr here.
+ *   Sec. 3.3  stacks: "rot" (s = l mod b) and the "fixed" control (one
+ *             dimension at every layer, selected by dim_override >= 0).
+ *
+ * Conventions for every entry point
+ *   - Matrices act on column vectors as in Eq. (1) and are stored row-major
+ *     as W[o][k] (d_out x d_in), i.e. z[i][o] = sum_k W[o][k] x[i][k].
+ *   - Activations are [B][n][d] row-major (d contiguous), samples
+ *     independent (no link crosses a sample).
+ *   - Optional epilogue (the paper states none; flags select it):
+ *       z = W_self x_i + m_i W_nbr x_{p(i)} + bias,  y = act(z) + (RESIDUAL ? x_i : 0)
+ *     with act = identity, or ReLU (ReLU'(0) = 0) under HCW_ACT_RELU.
+ *   - dtype HCW_BF16: x, W, y, z, dy, dx are bf16; products accumulate in
+ *     fp32; stored activations are rounded to bf16 (nearest, ties to even).
+ *     Needs d % 64 == 0.  dtype HCW_F32: all of those are fp32 (any d >= 1).
+ *     bias, dW_self, dW_nbr and dbias are always fp32.
+ *   - Pointers are device pointers unless stated; all must be 16-byte
+ *     aligned.  The caller owns every buffer; the library allocates no
+ *     device memory.  Outputs are overwritten, never accumulated into.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t passed as void*,
+ *     NULL = legacy default stream).  The return value reports argument
+ *     validation and launch errors.  A kernel that gives up on a bounded
+ *     wait records HCW_ERR_TIMEOUT in a per-device error word, read (and
+ *     cleared) by hcw_sync_status.
+ *   - n must be a power of two >= 2; B >= 0 (B = 0 does nothing); a
+ *     violated requirement returns a non-zero hcw_status and launches
+ *     nothing.
+ */
+#ifndef HCW_H
+#define HCW_H
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    HCW_OK = 0,
+    HCW_ERR_INVALID_ARG = 1,   /* bad size, NULL required pointer, bad flag or dimension */
+    HCW_ERR_UNSUPPORTED = 2,   /* valid request this build does not handle (e.g. bf16 with d % 64) */
+    HCW_ERR_ALIGNMENT = 3,     /* a pointer is not 16-byte aligned */
+    HCW_ERR_ALIASING = 4,      /* an output overlaps an input it must not overlap */
+    HCW_ERR_CUDA = 5,          /* a CUDA runtime/driver call failed */
+    HCW_ERR_TIMEOUT = 6,       /* a kernel gave up on a bounded wait (see hcw_sync_status) */
+    HCW_ERR_WORKSPACE = 7      /* workspace NULL or smaller than hcw_workspace_bytes */
+} hcw_status;
+
+typedef enum { HCW_BF16 = 0, HCW_F32 = 1 } hcw_dtype;
+
+#define HCW_CAUSAL   1u   /* Sec. 3.1 causal rule: receive only from the earlier endpoint */
+#define HCW_RESIDUAL 2u   /* y = act(z) + x */
+#define HCW_ACT_RELU 4u   /* act = ReLU (else identity, which is Eq. (1) itself) */
+
+/* Library version (major * 10000 + minor * 100 + patch). */
+int hcw_version(void);
+
+/* Human-readable name of a status code.  Never NULL. */
+const char* hcw_status_string(int status);
+
+/*
+ * Partner table of one layer, computed on the HOST (Sec. 3.1).
+ *   partner[i] = i XOR 2^s if position i receives at this layer, else -1,
+ *   for i = 0..n-1; s = layer mod log2 n, or dim_override if >= 0.
+ *   partner: host array of n ints, written.
+ * Returns HCW_ERR_INVALID_ARG for n not a power of two >= 2, dim_override >= log2 n,
+ * layer < 0 or partner NULL.
+ */
+int hcw_partner_table(int layer, int dim_override, int n, unsigned flags, int* partner);
+
+/*
+ * The same table computed by the device index code that the kernels use,
+ * written to device memory partner_dev[n] (int32) on `stream`.
+ */
+int hcw_partner_table_device(int layer, int dim_override, int n, unsigned flags,
+                             int* partner_dev, void* stream);
+
+/*
+ * One mixing layer forward (Sec. 3.1 wiring, Eq. (1) maps, epilogue above).
+ *   x       [B][n][d]  input (dtype)
+ *   W_self  [d][d]     W[o][k] (dtype)
+ *   W_nbr   [d][d]     W[o][k] (dtype)
+ *   bias    [d] fp32 or NULL (no bias)
+ *   layer   layer index l >= 0 (dimension s = l mod log2 n)
+ *   dim_override  -1 for the rotated rule, else the fixed dimension s
+ *   y       [B][n][d]  output (dtype); must not overlap x, W, bias or z_save
+ *   z_save  [B][n][d]  pre-activation z (dtype) or NULL; needed by
+ *                      hcw_layer_bwd when HCW_ACT_RELU is set
+ */
+int hcw_layer_fwd(const void* x, const void* W_self, const void* W_nbr, const float* bias,
+                  int layer, int dim_override, int B, int n, int d, int dtype, unsigned flags,
+                  void* y, void* z_save, void* stream);
+
+/*
+ * Bytes of device workspace hcw_layer_bwd / hcw_stack_bwd need for these
+ * sizes and flags (0 is possible).  Depends on the device's SM count, so
+ * query it with the target device current.
+ */
+size_t hcw_workspace_bytes(int B, int n, int d, int dtype, unsigned flags);
+
+/*
+ * One mixing layer backward (the chain rule through the forward above):
+ *   dz = dy * act'(z)
+ *   dx_i = W_self^T dz_i + m_{p(i)} W_nbr^T dz_{p(i)} + (RESIDUAL ? dy_i : 0)
+ *          -- a gather, since p is an involution: no atomics
+ *   dW_self = sum_i dz_i x_i^T, dW_nbr = sum_i m_i dz_i x_{p(i)}^T, dbias = sum_i dz_i
+ *   x, dy   [B][n][d] (dtype); z_save [B][n][d] (dtype), required iff HCW_ACT_RELU
+ *   dx      [B][n][d] (dtype) output; must not overlap any input
+ *   dW_self, dW_nbr  [d][d] fp32 outputs (same W[o][k] layout as the weights)
+ *   dbias   [d] fp32 output or NULL
+ *   workspace/ws_bytes  device scratch of at least hcw_workspace_bytes(...)
+ *   bytes (NULL allowed when that is 0); contents need not be initialised.
+ * dW sums are reduced in a fixed order: results are deterministic.
+ */
+int hcw_layer_bwd(const void* x, const void* z_save, const void* dy,
+                  const void* W_self, const void* W_nbr,
+                  int layer, int dim_override, int B, int n, int d, int dtype, unsigned flags,
+                  void* dx, float* dW_self, float* dW_nbr, float* dbias,
+                  void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * The two halves of hcw_layer_bwd, for callers that schedule them
+ * separately (e.g. the weight gradient on a second stream).
+ *
+ * hcw_layer_bwd_data: dx_i = W_self^T dz_i + m_{p(i)} W_nbr^T dz_{p(i)}
+ *                            + (RESIDUAL ? dy_i : 0)
+ *   dz [B][n][d] (dtype): gradient at the pre-activation, dy * act'(z)
+ *   dy [B][n][d] (dtype): gradient at the output, read only under
+ *                         HCW_RESIDUAL (may be NULL otherwise)
+ *   dx [B][n][d] (dtype) output.  One kernel launch; no workspace.
+ *
+ * hcw_layer_bwd_weight: dW_self = sum_i dz_i x_i^T,
+ *   dW_nbr = sum_i m_i dz_i x_{p(i)}^T, dbias = sum_i dz_i (if not NULL).
+ *   workspace of at least hcw_layer_bwd_weight_workspace_bytes(...) bytes.
+ *   Deterministic (fixed-order reductions).
+ */
+int hcw_layer_bwd_data(const void* dz, const void* dy, const void* W_self, const void* W_nbr,
+                       int layer, int dim_override, int B, int n, int d, int dtype,
+                       unsigned flags, void* dx, void* stream);
+
+size_t hcw_layer_bwd_weight_workspace_bytes(int B, int n, int d, int dtype, unsigned flags);
+
+int hcw_layer_bwd_weight(const void* x, const void* dz, int layer, int dim_override, int B,
+                         int n, int d, int dtype, unsigned flags, float* dW_self,
+                         float* dW_nbr, float* dbias, void* workspace, size_t ws_bytes,
+                         void* stream);
+
+/*
+ * Stack of L layers (Sec. 3.3 "rot": layer l uses s = (layer0 + l) mod log2 n,
+ * or dim_override for every layer).
+ *   W_self, W_nbr  [L][d][d]; bias [L][d] fp32 or NULL
+ *   y      [B][n][d] output of the last layer
+ *   acts   [L-1][B][n][d] outputs of layers 0..L-2 (= inputs of layers
+ *          1..L-1), written; required when L > 1 (kept for the backward)
+ *   zs     [L][B][n][d] pre-activations, written, or NULL
+ */
+int hcw_stack_fwd(const void* x, const void* W_self, const void* W_nbr, const float* bias,
+                  int layer0, int L, int dim_override, int B, int n, int d, int dtype,
+                  unsigned flags, void* y, void* acts, void* zs, void* stream);
+
+/*
+ * Backward of hcw_stack_fwd, layers L-1 down to 0.
+ *   x, acts, zs as given to / written by hcw_stack_fwd (zs required iff
+ *   HCW_ACT_RELU); dy [B][n][d] gradient of y.
+ *   dx [B][n][d] gradient of x (output); dW_self, dW_nbr [L][d][d] and
+ *   dbias [L][d] (or NULL) fp32 outputs.
+ *   workspace: at least hcw_workspace_bytes(...) + 2 * B*n*d*sizeof(dtype)
+ *   bytes (two gradient buffers between layers).
+ */
+int hcw_stack_bwd(const void* x, const void* acts, const void* zs, const void* dy,
+                  const void* W_self, const void* W_nbr, int layer0, int L, int dim_override,
+                  int B, int n, int d, int dtype, unsigned flags,
+                  void* dx, float* dW_self, float* dW_nbr, float* dbias,
+                  void* workspace, size_t ws_bytes, void* stream);
+
+/* Workspace bytes hcw_stack_bwd needs. */
+size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags);
+
+/* Number of kernels this library has launched in this process (all devices). */
+unsigned long long hcw_launch_count(void);
+
+/*
+ * Synchronise `stream`, then read and clear the current device's error
+ * word.  Returns HCW_ERR_TIMEOUT if a kernel gave up on a bounded wait since
+ * the last call, HCW_ERR_CUDA if the synchronisation failed, else HCW_OK.
+ */
+int hcw_sync_status(void* stream);
+
+/*
+ * Self-test of the bounded-wait path the kernels use: launches one CTA that
+ * waits on an mbarrier nothing ever arrives on.  After timeout_ns
+ * nanoseconds (1e3 .. 1e10) it records HCW_ERR_TIMEOUT in the error word and
+ * exits normally, leaving the context usable.  Follow with hcw_sync_status.
+ */
+int hcw_selftest_wait(long long timeout_ns, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HCW_H */

@@ -1,0 +1,695 @@
+// hcw_api.cu -- the C ABI of include/hcw.h: argument validation, TMA tensor
+// maps, work decomposition and launches.  No device memory is allocated
+// here; every buffer is the caller's.
+#include <stdio.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <atomic>
+#include <mutex>
+
+#include "hcw.h"
+#include "hcw_internal.h"
+
+namespace hcw {
+namespace {
+
+constexpr unsigned kAllFlags = HCW_CAUSAL | HCW_RESIDUAL | HCW_ACT_RELU;
+constexpr unsigned long long kDefaultTimeoutNs = 2000000000ull;   // 2 s per wait
+
+int log2_exact(long long n) {
+    if (n < 2 || (n & (n - 1))) return -1;
+    int b = 0;
+    while ((1ll << b) < n) ++b;
+    return b;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bool overlaps(const void* a, size_t na, const void* b, size_t nb) {
+    if (!a || !b || na == 0 || nb == 0) return false;
+    const uintptr_t x = reinterpret_cast<uintptr_t>(a), y = reinterpret_cast<uintptr_t>(b);
+    return x < y + nb && y < x + na;
+}
+
+size_t elem_size(int dtype) { return dtype == HCW_F32 ? 4 : 2; }
+
+int sm_count() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
+        return 148;
+    return n;
+}
+
+// ------------------------------------------------------------ tensor maps
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    });
+    return fn;
+}
+
+// Token-major activations [B*n][d] bf16 viewed as (d, lo = k, bit = 2, HI),
+// box (64 features, box_lo, 1, box_hi), 128-byte swizzle.
+bool map_rows(CUtensorMap* m, const void* base, long long tokens, int d, int k, int box_rows) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    const int box_lo = k < box_rows ? k : box_rows;
+    const int box_hi = box_rows / box_lo;
+    const long long HI = tokens / (2ll * k);
+    cuuint64_t dims[4] = {(cuuint64_t)d, (cuuint64_t)k, 2, (cuuint64_t)HI};
+    cuuint64_t strides[3] = {(cuuint64_t)d * 2, (cuuint64_t)k * d * 2, (cuuint64_t)2 * k * d * 2};
+    cuuint32_t box[4] = {64, (cuuint32_t)box_lo, 1, (cuuint32_t)box_hi};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides,
+               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Weights W[o][k] bf16 [d][d], box (64 k, box_o), 128-byte swizzle.
+bool map_weight(CUtensorMap* m, const void* base, int d, int box_o) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)d};
+    cuuint64_t strides[1] = {(cuuint64_t)d * 2};
+    cuuint32_t box[2] = {64, (cuuint32_t)box_o};
+    cuuint32_t estr[2] = {1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int pick_bn(int d) { return d % 256 == 0 ? 256 : d % 128 == 0 ? 128 : 64; }
+
+// ------------------------------------------------------------ validation
+struct Shape {
+    int B, n, d, b, s;
+    long long tokens;
+    size_t act_bytes;
+};
+
+int check_shape(int layer, int dim_override, int B, int n, int d, int dtype, unsigned flags,
+                Shape* sh) {
+    if (dtype != HCW_BF16 && dtype != HCW_F32) return HCW_ERR_INVALID_ARG;
+    if (flags & ~kAllFlags) return HCW_ERR_INVALID_ARG;
+    const int b = log2_exact(n);
+    if (b < 1 || n > (1 << 30)) return HCW_ERR_INVALID_ARG;
+    if (B < 0 || d < 1 || layer < 0) return HCW_ERR_INVALID_ARG;
+    if (dim_override < -1 || dim_override >= b) return HCW_ERR_INVALID_ARG;
+    const long long tokens = (long long)B * n;
+    if (tokens > (1ll << 31) - 1) return HCW_ERR_UNSUPPORTED;
+    if (dtype == HCW_BF16 && (d % 64 != 0 || d > 16384)) return HCW_ERR_UNSUPPORTED;
+    sh->B = B;
+    sh->n = n;
+    sh->d = d;
+    sh->b = b;
+    sh->s = dim_override >= 0 ? dim_override : layer % b;
+    sh->tokens = tokens;
+    sh->act_bytes = (size_t)tokens * d * elem_size(dtype);
+    return HCW_OK;
+}
+
+// ------------------------------------------------------------ bf16 sizes
+struct WPlan {
+    int n_ot, n_nt, qb, nkb_self, nkb_nbr, kb_per_unit, splits_self, splits_nbr, splits_max,
+        units;
+};
+
+WPlan plan_dw(long long tokens, int d, unsigned flags) {
+    WPlan w;
+    const int BN = pick_bn(d);
+    const long long Mh = tokens / 2;
+    w.n_ot = (d + 127) / 128;
+    w.n_nt = d / BN;
+    w.qb = (int)((Mh + 63) / 64);
+    w.nkb_self = 2 * w.qb;
+    w.nkb_nbr = (flags & HCW_CAUSAL) ? w.qb : 2 * w.qb;
+    const int tiles = w.n_ot * w.n_nt;
+    const long long total_kb = (long long)tiles * (w.nkb_self + w.nkb_nbr);
+    const int sms = sm_count();
+    // about one unit per SM, at least 4 token blocks (256 tokens) per unit
+    long long kpu = (total_kb + sms - 1) / sms;
+    if (kpu < 4) kpu = 4;
+    w.kb_per_unit = (int)kpu;
+    w.splits_self = (int)((w.nkb_self + kpu - 1) / kpu);
+    w.splits_nbr = (int)((w.nkb_nbr + kpu - 1) / kpu);
+    if (w.splits_self < 1) w.splits_self = 1;
+    if (w.splits_nbr < 1) w.splits_nbr = 1;
+    w.splits_max = w.splits_self > w.splits_nbr ? w.splits_self : w.splits_nbr;
+    w.units = tiles * (w.splits_self + w.splits_nbr);
+    return w;
+}
+
+// Workspace of the weight gradient (bf16: dW split partials, both dtypes:
+// column-sum partials of dbias) and of the full layer backward, which adds
+// the masked gradient dz = dy * act'(z) in front when an activation is used:
+//   [dz (ReLU only)][dW partials (bf16, more than one split)][colsum partials]
+struct WsLayout {
+    size_t dz_off, dz_bytes, w_off, part_bytes, col_off, col_bytes, w_bytes, total;
+};
+
+size_t align256(size_t v) { return (v + 255) & ~(size_t)255; }
+
+WsLayout ws_layout(long long tokens, int d, int dtype, unsigned flags) {
+    WsLayout l;
+    const size_t es = elem_size(dtype);
+    l.dz_off = 0;
+    l.dz_bytes = (flags & HCW_ACT_RELU) ? align256((size_t)tokens * d * es) : 0;
+    l.w_off = l.dz_off + l.dz_bytes;
+    if (dtype == HCW_BF16 && tokens > 0) {
+        WPlan w = plan_dw(tokens, d, flags);
+        l.part_bytes = (w.splits_max > 1) ? align256((size_t)2 * w.splits_max * d * d * 4) : 0;
+    } else {
+        l.part_bytes = 0;
+    }
+    l.col_off = l.part_bytes;   // relative to w_off
+    l.col_bytes = align256(colsum_workspace_bytes(tokens, d));
+    l.w_bytes = l.part_bytes + l.col_bytes;
+    l.total = l.w_off + l.w_bytes;
+    return l;
+}
+
+unsigned long long g_timeout_ns = kDefaultTimeoutNs;
+std::atomic<unsigned long long> g_launches{0};
+
+int cuda_status(cudaError_t e) { return e == cudaSuccess ? HCW_OK : HCW_ERR_CUDA; }
+
+// Count `kernels` launches if the launch call succeeded.
+int launched(cudaError_t e, int kernels) {
+    if (e != cudaSuccess) return HCW_ERR_CUDA;
+    g_launches.fetch_add((unsigned long long)kernels, std::memory_order_relaxed);
+    return HCW_OK;
+}
+
+// ------------------------------------------------------------ layer internals
+int fwd_bf16(const Shape& sh, const void* x, const void* Ws, const void* Wn, const float* bias,
+             unsigned flags, void* y, void* z, cudaStream_t st) {
+    const int d = sh.d, BN = pick_bn(d), k = 1 << sh.s;
+    CUtensorMap tA, tB0, tB1;
+    if (!map_rows(&tA, x, sh.tokens, d, k, 128) || !map_weight(&tB0, Ws, d, BN) ||
+        !map_weight(&tB1, Wn, d, BN))
+        return HCW_ERR_CUDA;
+    TcParams p;
+    memset(&p, 0, sizeof(p));
+    p.d = d;
+    p.k = k;
+    p.Mh = (int)(sh.tokens / 2);
+    p.nK = d / 64;
+    p.n_rb = (p.Mh + 127) / 128;
+    p.n_nt = d / BN;
+    if (flags & HCW_CAUSAL) {
+        // Sec. 3.1: positions with bit s set receive (K = 2d), the others do not (K = d)
+        p.n_full = 1;
+        p.full_bit0 = 1;
+        p.half_bit = 0;
+    } else {
+        p.n_full = 2;
+        p.full_bit0 = 0;
+        p.full_bit1 = 1;
+        p.half_bit = -1;
+    }
+    p.n_units = p.n_rb * p.n_nt * 2;
+    p.flags = flags;
+    p.bias = bias;
+    p.resid = static_cast<const __nv_bfloat16*>(x);
+    p.out = static_cast<__nv_bfloat16*>(y);
+    p.zout = static_cast<__nv_bfloat16*>(z);
+    p.timeout_ns = g_timeout_ns;
+    const int sms = sm_count();
+    const int grid = p.n_units < sms ? p.n_units : sms;
+    return launched(launch_tc(MODE_FWD, BN, tA, tB0, tB1, p, grid, st), 1);
+}
+
+// dx: a row gathers dz from its partner exactly when the partner received from it
+int dx_bf16(const Shape& sh, const void* dz, const void* dy, const void* Ws, const void* Wn,
+            unsigned flags, void* dx, cudaStream_t st) {
+    const int d = sh.d, BN = pick_bn(d), k = 1 << sh.s;
+    CUtensorMap tA, tB0, tB1;
+    if (!map_rows(&tA, dz, sh.tokens, d, k, 128) || !map_weight(&tB0, Ws, d, 64) ||
+        !map_weight(&tB1, Wn, d, 64))
+        return HCW_ERR_CUDA;
+    TcParams p;
+    memset(&p, 0, sizeof(p));
+    p.d = d;
+    p.k = k;
+    p.Mh = (int)(sh.tokens / 2);
+    p.nK = d / 64;
+    p.n_rb = (p.Mh + 127) / 128;
+    p.n_nt = d / BN;
+    if (flags & HCW_CAUSAL) {
+        p.n_full = 1;
+        p.full_bit0 = 0;   // bit-0 rows: their partner (bit 1) received from them
+        p.half_bit = 1;
+    } else {
+        p.n_full = 2;
+        p.full_bit0 = 0;
+        p.full_bit1 = 1;
+        p.half_bit = -1;
+    }
+    p.n_units = p.n_rb * p.n_nt * 2;
+    p.flags = flags & HCW_RESIDUAL;
+    p.resid = static_cast<const __nv_bfloat16*>(dy);
+    p.out = static_cast<__nv_bfloat16*>(dx);
+    p.timeout_ns = g_timeout_ns;
+    const int sms = sm_count();
+    const int grid = p.n_units < sms ? p.n_units : sms;
+    return launched(launch_tc(MODE_DX, BN, tA, tB0, tB1, p, grid, st), 1);
+}
+
+// dW: token-contracted, split over token blocks, fixed-order reduction; dbias
+// by a deterministic two-pass column sum.  wws: weight workspace.
+int dw_bf16(const Shape& sh, const void* x, const void* dz, unsigned flags, float* dWs,
+            float* dWn, float* dbias, uint8_t* wws, cudaStream_t st) {
+    const int d = sh.d, BN = pick_bn(d), k = 1 << sh.s;
+    const WsLayout lay = ws_layout(sh.tokens, d, HCW_BF16, flags);
+    const WPlan w = plan_dw(sh.tokens, d, flags);
+    CUtensorMap tA, tB0;
+    if (!map_rows(&tA, dz, sh.tokens, d, k, 64) || !map_rows(&tB0, x, sh.tokens, d, k, 64))
+        return HCW_ERR_CUDA;
+    TcParams p;
+    memset(&p, 0, sizeof(p));
+    p.d = d;
+    p.k = k;
+    p.Mh = (int)(sh.tokens / 2);
+    p.n_nt = w.n_nt;
+    p.n_ot = w.n_ot;
+    p.qb = w.qb;
+    p.nkb_self = w.nkb_self;
+    p.nkb_nbr = w.nkb_nbr;
+    p.kb_per_unit = w.kb_per_unit;
+    p.splits_self = w.splits_self;
+    p.splits_nbr = w.splits_nbr;
+    p.splits_max = w.splits_max;
+    p.causal = (flags & HCW_CAUSAL) ? 1 : 0;
+    p.n_units = w.units;
+    p.dw_self = dWs;
+    p.dw_nbr = dWn;
+    p.dw_partial = reinterpret_cast<float*>(wws);
+    p.timeout_ns = g_timeout_ns;
+    const int sms = sm_count();
+    const int grid = p.n_units < sms ? p.n_units : sms;
+    int rc = launched(launch_tc(MODE_DW, BN, tA, tB0, tB0, p, grid, st), 1);
+    if (rc) return rc;
+    if (w.splits_max > 1) {
+        rc = launched(launch_splitk_reduce(p.dw_partial, w.splits_max, w.splits_self,
+                                           w.splits_nbr, d, dWs, dWn, st),
+                      1);
+        if (rc) return rc;
+    }
+    if (dbias)
+        return launched(launch_colsum_bf16(static_cast<const __nv_bfloat16*>(dz), sh.tokens, d,
+                                           reinterpret_cast<float*>(wws + lay.col_off), dbias,
+                                           st),
+                        2);
+    return HCW_OK;
+}
+
+int fwd_f32(const Shape& sh, const void* x, const void* Ws, const void* Wn, const float* bias,
+            unsigned flags, void* y, void* z, cudaStream_t st) {
+    return launched(launch_f32_fwd(static_cast<const float*>(x), static_cast<const float*>(Ws),
+                                   static_cast<const float*>(Wn), bias, sh.s, sh.B, sh.n, sh.d,
+                                   flags, static_cast<float*>(y), static_cast<float*>(z), st),
+                    1);
+}
+
+int dx_f32(const Shape& sh, const void* dz, const void* dy, const void* Ws, const void* Wn,
+           unsigned flags, void* dx, cudaStream_t st) {
+    return launched(launch_f32_dx(static_cast<const float*>(dz), static_cast<const float*>(dy),
+                                  static_cast<const float*>(Ws), static_cast<const float*>(Wn),
+                                  sh.s, sh.B, sh.n, sh.d, flags, static_cast<float*>(dx), st),
+                    1);
+}
+
+int dw_f32(const Shape& sh, const void* x, const void* dz, unsigned flags, float* dWs,
+           float* dWn, float* dbias, uint8_t* wws, cudaStream_t st) {
+    const WsLayout lay = ws_layout(sh.tokens, sh.d, HCW_F32, flags);
+    int rc = launched(launch_f32_dw(static_cast<const float*>(x), static_cast<const float*>(dz),
+                                    sh.s, sh.B, sh.n, sh.d, flags, dWs, dWn, st),
+                      1);
+    if (rc || !dbias) return rc;
+    return launched(launch_colsum_f32(static_cast<const float*>(dz), sh.tokens, sh.d,
+                                      reinterpret_cast<float*>(wws + lay.col_off), dbias, st),
+                    2);
+}
+
+int layer_fwd_impl(const Shape& sh, int dtype, const void* x, const void* Ws, const void* Wn,
+                   const float* bias, unsigned flags, void* y, void* z, cudaStream_t st) {
+    if (sh.tokens == 0) return HCW_OK;
+    return dtype == HCW_BF16 ? fwd_bf16(sh, x, Ws, Wn, bias, flags, y, z, st)
+                             : fwd_f32(sh, x, Ws, Wn, bias, flags, y, z, st);
+}
+
+int zero_weight_grads(const Shape& sh, float* dWs, float* dWn, float* dbias, cudaStream_t st) {
+    // empty batch: the sums over no tokens are zero
+    const size_t wbytes = (size_t)sh.d * sh.d * sizeof(float);
+    cudaError_t e = cudaMemsetAsync(dWs, 0, wbytes, st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(dWn, 0, wbytes, st);
+    if (e == cudaSuccess && dbias) e = cudaMemsetAsync(dbias, 0, sh.d * sizeof(float), st);
+    return cuda_status(e);
+}
+
+int layer_dx_impl(const Shape& sh, int dtype, const void* dz, const void* dy, const void* Ws,
+                  const void* Wn, unsigned flags, void* dx, cudaStream_t st) {
+    if (sh.tokens == 0) return HCW_OK;
+    return dtype == HCW_BF16 ? dx_bf16(sh, dz, dy, Ws, Wn, flags, dx, st)
+                             : dx_f32(sh, dz, dy, Ws, Wn, flags, dx, st);
+}
+
+int layer_dw_impl(const Shape& sh, int dtype, const void* x, const void* dz, unsigned flags,
+                  float* dWs, float* dWn, float* dbias, uint8_t* wws, cudaStream_t st) {
+    if (sh.tokens == 0) return zero_weight_grads(sh, dWs, dWn, dbias, st);
+    return dtype == HCW_BF16 ? dw_bf16(sh, x, dz, flags, dWs, dWn, dbias, wws, st)
+                             : dw_f32(sh, x, dz, flags, dWs, dWn, dbias, wws, st);
+}
+
+int layer_bwd_impl(const Shape& sh, int dtype, const void* x, const void* z, const void* dy,
+                   const void* Ws, const void* Wn, unsigned flags, void* dx, float* dWs,
+                   float* dWn, float* dbias, void* ws, cudaStream_t st) {
+    if (sh.tokens == 0) return zero_weight_grads(sh, dWs, dWn, dbias, st);
+    const WsLayout lay = ws_layout(sh.tokens, sh.d, dtype, flags);
+    uint8_t* wsb = static_cast<uint8_t*>(ws);
+    const void* dz = dy;
+    int rc;
+    if (flags & HCW_ACT_RELU) {
+        void* dzw = wsb + lay.dz_off;
+        const size_t count = (size_t)sh.tokens * sh.d;
+        rc = launched(dtype == HCW_BF16
+                          ? launch_relu_grad_bf16(static_cast<const __nv_bfloat16*>(dy),
+                                                  static_cast<const __nv_bfloat16*>(z),
+                                                  static_cast<__nv_bfloat16*>(dzw), count, st)
+                          : launch_relu_grad_f32(static_cast<const float*>(dy),
+                                                 static_cast<const float*>(z),
+                                                 static_cast<float*>(dzw), count, st),
+                      1);
+        if (rc) return rc;
+        dz = dzw;
+    }
+    rc = layer_dx_impl(sh, dtype, dz, dy, Ws, Wn, flags, dx, st);
+    if (rc) return rc;
+    return layer_dw_impl(sh, dtype, x, dz, flags, dWs, dWn, dbias, wsb + lay.w_off, st);
+}
+
+int check_fwd_ptrs(const Shape& sh, int dtype, const void* x, const void* Ws, const void* Wn,
+                   const float* bias, void* y, void* z) {
+    if (!x || !Ws || !Wn || !y) return HCW_ERR_INVALID_ARG;
+    if (!aligned16(x) || !aligned16(Ws) || !aligned16(Wn) || !aligned16(y) ||
+        (bias && !aligned16(bias)) || (z && !aligned16(z)))
+        return HCW_ERR_ALIGNMENT;
+    const size_t wb = (size_t)sh.d * sh.d * elem_size(dtype);
+    if (overlaps(y, sh.act_bytes, x, sh.act_bytes) || overlaps(y, sh.act_bytes, Ws, wb) ||
+        overlaps(y, sh.act_bytes, Wn, wb) || overlaps(y, sh.act_bytes, bias, sh.d * 4) ||
+        overlaps(y, sh.act_bytes, z, sh.act_bytes) || overlaps(z, sh.act_bytes, x, sh.act_bytes))
+        return HCW_ERR_ALIASING;
+    return HCW_OK;
+}
+
+int check_bwd_ptrs(const Shape& sh, int dtype, unsigned flags, const void* x, const void* z,
+                   const void* dy, const void* Ws, const void* Wn, void* dx, float* dWs,
+                   float* dWn, float* dbias) {
+    if (!x || !dy || !Ws || !Wn || !dx || !dWs || !dWn) return HCW_ERR_INVALID_ARG;
+    if ((flags & HCW_ACT_RELU) && !z) return HCW_ERR_INVALID_ARG;
+    const void* ptrs[] = {x, z, dy, Ws, Wn, dx, dWs, dWn, dbias};
+    for (const void* q : ptrs)
+        if (q && !aligned16(q)) return HCW_ERR_ALIGNMENT;
+    const size_t ab = sh.act_bytes, wb = (size_t)sh.d * sh.d * elem_size(dtype);
+    const size_t gb = (size_t)sh.d * sh.d * 4;
+    if (overlaps(dx, ab, x, ab) || overlaps(dx, ab, dy, ab) || overlaps(dx, ab, z, ab) ||
+        overlaps(dx, ab, Ws, wb) || overlaps(dx, ab, Wn, wb) || overlaps(dWs, gb, dWn, gb) ||
+        overlaps(dx, ab, dWs, gb) || overlaps(dx, ab, dWn, gb) ||
+        overlaps(dbias, sh.d * 4, dWs, gb) || overlaps(dbias, sh.d * 4, dWn, gb))
+        return HCW_ERR_ALIASING;
+    return HCW_OK;
+}
+
+}  // namespace
+}  // namespace hcw
+
+using namespace hcw;
+
+extern "C" {
+
+int hcw_version(void) { return 100; }
+
+const char* hcw_status_string(int s) {
+    switch (s) {
+        case HCW_OK: return "HCW_OK";
+        case HCW_ERR_INVALID_ARG: return "HCW_ERR_INVALID_ARG";
+        case HCW_ERR_UNSUPPORTED: return "HCW_ERR_UNSUPPORTED";
+        case HCW_ERR_ALIGNMENT: return "HCW_ERR_ALIGNMENT";
+        case HCW_ERR_ALIASING: return "HCW_ERR_ALIASING";
+        case HCW_ERR_CUDA: return "HCW_ERR_CUDA";
+        case HCW_ERR_TIMEOUT: return "HCW_ERR_TIMEOUT";
+        case HCW_ERR_WORKSPACE: return "HCW_ERR_WORKSPACE";
+        default: return "HCW_ERR_UNKNOWN";
+    }
+}
+
+int hcw_partner_table(int layer, int dim_override, int n, unsigned flags, int* partner) {
+    const int b = log2_exact(n);
+    if (b < 1 || layer < 0 || dim_override < -1 || dim_override >= b || !partner ||
+        (flags & ~kAllFlags))
+        return HCW_ERR_INVALID_ARG;
+    const int s = dim_override >= 0 ? dim_override : layer % b;
+    for (int i = 0; i < n; ++i) {
+        const int p = i ^ (1 << s);
+        const bool recv = !(flags & HCW_CAUSAL) || ((i >> s) & 1);
+        partner[i] = recv ? p : -1;
+    }
+    return HCW_OK;
+}
+
+int hcw_partner_table_device(int layer, int dim_override, int n, unsigned flags,
+                             int* partner_dev, void* stream) {
+    const int b = log2_exact(n);
+    if (b < 1 || layer < 0 || dim_override < -1 || dim_override >= b || !partner_dev ||
+        (flags & ~kAllFlags))
+        return HCW_ERR_INVALID_ARG;
+    if (!aligned16(partner_dev)) return HCW_ERR_ALIGNMENT;
+    const int s = dim_override >= 0 ? dim_override : layer % b;
+    return launched(launch_partner_table(s, n, flags, partner_dev, (cudaStream_t)stream), 1);
+}
+
+int hcw_layer_fwd(const void* x, const void* W_self, const void* W_nbr, const float* bias,
+                  int layer, int dim_override, int B, int n, int d, int dtype, unsigned flags,
+                  void* y, void* z_save, void* stream) {
+    Shape sh;
+    int rc = check_shape(layer, dim_override, B, n, d, dtype, flags, &sh);
+    if (rc) return rc;
+    if (sh.tokens == 0) return HCW_OK;   // empty batch: nothing to compute
+    rc = check_fwd_ptrs(sh, dtype, x, W_self, W_nbr, bias, y, z_save);
+    if (rc) return rc;
+    return layer_fwd_impl(sh, dtype, x, W_self, W_nbr, bias, flags, y, z_save,
+                          (cudaStream_t)stream);
+}
+
+size_t hcw_workspace_bytes(int B, int n, int d, int dtype, unsigned flags) {
+    Shape sh;
+    if (check_shape(0, -1, B, n, d, dtype, flags, &sh)) return 0;
+    return ws_layout(sh.tokens, d, dtype, flags).total;
+}
+
+int hcw_layer_bwd(const void* x, const void* z_save, const void* dy, const void* W_self,
+                  const void* W_nbr, int layer, int dim_override, int B, int n, int d, int dtype,
+                  unsigned flags, void* dx, float* dW_self, float* dW_nbr, float* dbias,
+                  void* workspace, size_t ws_bytes, void* stream) {
+    Shape sh;
+    int rc = check_shape(layer, dim_override, B, n, d, dtype, flags, &sh);
+    if (rc) return rc;
+    if (sh.tokens == 0) {
+        // empty batch: only the weight gradients (sums over no tokens, zero) are written
+        if (!dW_self || !dW_nbr) return HCW_ERR_INVALID_ARG;
+        return layer_bwd_impl(sh, dtype, x, z_save, dy, W_self, W_nbr, flags, dx, dW_self,
+                              dW_nbr, dbias, workspace, (cudaStream_t)stream);
+    }
+    rc = check_bwd_ptrs(sh, dtype, flags, x, z_save, dy, W_self, W_nbr, dx, dW_self, dW_nbr,
+                        dbias);
+    if (rc) return rc;
+    const size_t need = ws_layout(sh.tokens, d, dtype, flags).total;
+    if (ws_bytes < need || (need && !workspace)) return HCW_ERR_WORKSPACE;
+    if (workspace && !aligned16(workspace)) return HCW_ERR_ALIGNMENT;
+    if (overlaps(workspace, ws_bytes, dx, sh.act_bytes) ||
+        overlaps(workspace, ws_bytes, dy, sh.act_bytes) ||
+        overlaps(workspace, ws_bytes, x, sh.act_bytes))
+        return HCW_ERR_ALIASING;
+    return layer_bwd_impl(sh, dtype, x, z_save, dy, W_self, W_nbr, flags, dx, dW_self, dW_nbr,
+                          dbias, workspace, (cudaStream_t)stream);
+}
+
+int hcw_layer_bwd_data(const void* dz, const void* dy, const void* W_self, const void* W_nbr,
+                       int layer, int dim_override, int B, int n, int d, int dtype,
+                       unsigned flags, void* dx, void* stream) {
+    Shape sh;
+    int rc = check_shape(layer, dim_override, B, n, d, dtype, flags, &sh);
+    if (rc) return rc;
+    if (sh.tokens == 0) return HCW_OK;
+    if (!dz || !W_self || !W_nbr || !dx || ((flags & HCW_RESIDUAL) && !dy))
+        return HCW_ERR_INVALID_ARG;
+    const void* ptrs[] = {dz, dy, W_self, W_nbr, dx};
+    for (const void* q : ptrs)
+        if (q && !aligned16(q)) return HCW_ERR_ALIGNMENT;
+    const size_t ab = sh.act_bytes, wb = (size_t)d * d * elem_size(dtype);
+    if (overlaps(dx, ab, dz, ab) || overlaps(dx, ab, dy, ab) || overlaps(dx, ab, W_self, wb) ||
+        overlaps(dx, ab, W_nbr, wb))
+        return HCW_ERR_ALIASING;
+    return layer_dx_impl(sh, dtype, dz, dy, W_self, W_nbr, flags, dx, (cudaStream_t)stream);
+}
+
+size_t hcw_layer_bwd_weight_workspace_bytes(int B, int n, int d, int dtype, unsigned flags) {
+    Shape sh;
+    if (check_shape(0, -1, B, n, d, dtype, flags, &sh)) return 0;
+    return ws_layout(sh.tokens, d, dtype, flags).w_bytes;
+}
+
+int hcw_layer_bwd_weight(const void* x, const void* dz, int layer, int dim_override, int B,
+                         int n, int d, int dtype, unsigned flags, float* dW_self,
+                         float* dW_nbr, float* dbias, void* workspace, size_t ws_bytes,
+                         void* stream) {
+    Shape sh;
+    int rc = check_shape(layer, dim_override, B, n, d, dtype, flags, &sh);
+    if (rc) return rc;
+    if (!dW_self || !dW_nbr) return HCW_ERR_INVALID_ARG;
+    const void* ptrs[] = {x, dz, dW_self, dW_nbr, dbias, workspace};
+    for (const void* q : ptrs)
+        if (q && !aligned16(q)) return HCW_ERR_ALIGNMENT;
+    if (sh.tokens > 0 && (!x || !dz)) return HCW_ERR_INVALID_ARG;
+    const size_t need = ws_layout(sh.tokens, d, dtype, flags).w_bytes;
+    if (sh.tokens > 0 && (ws_bytes < need || (need && !workspace))) return HCW_ERR_WORKSPACE;
+    const size_t ab = sh.act_bytes, gb = (size_t)d * d * 4;
+    if (overlaps(dW_self, gb, dW_nbr, gb) || overlaps(dbias, (size_t)d * 4, dW_self, gb) ||
+        overlaps(dbias, (size_t)d * 4, dW_nbr, gb) || overlaps(workspace, ws_bytes, x, ab) ||
+        overlaps(workspace, ws_bytes, dz, ab) || overlaps(workspace, ws_bytes, dW_self, gb) ||
+        overlaps(workspace, ws_bytes, dW_nbr, gb) || overlaps(dW_self, gb, x, ab) ||
+        overlaps(dW_nbr, gb, x, ab) || overlaps(dW_self, gb, dz, ab) ||
+        overlaps(dW_nbr, gb, dz, ab))
+        return HCW_ERR_ALIASING;
+    return layer_dw_impl(sh, dtype, x, dz, flags, dW_self, dW_nbr, dbias,
+                         static_cast<uint8_t*>(workspace), (cudaStream_t)stream);
+}
+
+int hcw_stack_fwd(const void* x, const void* W_self, const void* W_nbr, const float* bias,
+                  int layer0, int L, int dim_override, int B, int n, int d, int dtype,
+                  unsigned flags, void* y, void* acts, void* zs, void* stream) {
+    Shape sh;
+    if (L < 1) return HCW_ERR_INVALID_ARG;
+    int rc = check_shape(layer0, dim_override, B, n, d, dtype, flags, &sh);
+    if (rc) return rc;
+    if (sh.tokens == 0) return HCW_OK;
+    if (L > 1 && !acts) return HCW_ERR_INVALID_ARG;
+    if ((acts && !aligned16(acts)) || (zs && !aligned16(zs))) return HCW_ERR_ALIGNMENT;
+    const size_t ab = sh.act_bytes, wb = (size_t)d * d * elem_size(dtype);
+    rc = check_fwd_ptrs(sh, dtype, x, W_self, W_nbr, bias, y, nullptr);
+    if (rc) return rc;
+    const size_t acts_b = (size_t)(L - 1) * ab, zs_b = (size_t)L * ab;
+    if (overlaps(acts, acts_b, x, ab) || overlaps(acts, acts_b, y, ab) ||
+        overlaps(zs, zs_b, x, ab) || overlaps(zs, zs_b, y, ab) ||
+        overlaps(zs, zs_b, acts, acts_b) || overlaps(acts, acts_b, W_self, L * wb) ||
+        overlaps(acts, acts_b, W_nbr, L * wb))
+        return HCW_ERR_ALIASING;
+    cudaStream_t st = (cudaStream_t)stream;
+    const uint8_t* xin = static_cast<const uint8_t*>(x);
+    for (int l = 0; l < L; ++l) {
+        Shape shl = sh;
+        shl.s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
+        const uint8_t* in = l == 0 ? xin : static_cast<const uint8_t*>(acts) + (size_t)(l - 1) * ab;
+        void* out = l == L - 1 ? y : static_cast<uint8_t*>(acts) + (size_t)l * ab;
+        void* z = zs ? static_cast<uint8_t*>(zs) + (size_t)l * ab : nullptr;
+        rc = layer_fwd_impl(shl, dtype, in, static_cast<const uint8_t*>(W_self) + l * wb,
+                            static_cast<const uint8_t*>(W_nbr) + l * wb,
+                            bias ? bias + (size_t)l * d : nullptr, flags, out, z, st);
+        if (rc) return rc;
+    }
+    return HCW_OK;
+}
+
+size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags) {
+    Shape sh;
+    if (check_shape(0, -1, B, n, d, dtype, flags, &sh)) return 0;
+    return ws_layout(sh.tokens, d, dtype, flags).total + 2 * align256(sh.act_bytes);
+}
+
+int hcw_stack_bwd(const void* x, const void* acts, const void* zs, const void* dy,
+                  const void* W_self, const void* W_nbr, int layer0, int L, int dim_override,
+                  int B, int n, int d, int dtype, unsigned flags, void* dx, float* dW_self,
+                  float* dW_nbr, float* dbias, void* workspace, size_t ws_bytes, void* stream) {
+    Shape sh;
+    if (L < 1) return HCW_ERR_INVALID_ARG;
+    int rc = check_shape(layer0, dim_override, B, n, d, dtype, flags, &sh);
+    if (rc) return rc;
+    if (sh.tokens == 0) {
+        if (!dW_self || !dW_nbr) return HCW_ERR_INVALID_ARG;
+        cudaStream_t st0 = (cudaStream_t)stream;
+        const size_t gbytes = (size_t)L * d * d * sizeof(float);
+        cudaError_t e = cudaMemsetAsync(dW_self, 0, gbytes, st0);
+        if (e == cudaSuccess) e = cudaMemsetAsync(dW_nbr, 0, gbytes, st0);
+        if (e == cudaSuccess && dbias) e = cudaMemsetAsync(dbias, 0, (size_t)L * d * 4, st0);
+        return cuda_status(e);
+    }
+    if ((L > 1 && !acts) || ((flags & HCW_ACT_RELU) && !zs)) return HCW_ERR_INVALID_ARG;
+    rc = check_bwd_ptrs(sh, dtype, flags, x, zs, dy, W_self, W_nbr, dx, dW_self, dW_nbr, dbias);
+    if (rc) return rc;
+    if ((acts && !aligned16(acts))) return HCW_ERR_ALIGNMENT;
+    const size_t ab = sh.act_bytes, wb = (size_t)d * d * elem_size(dtype);
+    const size_t gb = (size_t)d * d * 4;
+    const size_t need = hcw_stack_workspace_bytes(B, n, d, dtype, flags);
+    if (ws_bytes < need || !workspace) return HCW_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return HCW_ERR_ALIGNMENT;
+    if (overlaps(workspace, ws_bytes, dx, ab) || overlaps(workspace, ws_bytes, dy, ab) ||
+        overlaps(workspace, ws_bytes, x, ab) ||
+        overlaps(workspace, ws_bytes, acts, (size_t)(L > 1 ? L - 1 : 0) * ab) ||
+        overlaps(workspace, ws_bytes, zs, zs ? (size_t)L * ab : 0) ||
+        overlaps(dW_self, (size_t)L * gb, dW_nbr, (size_t)L * gb) ||
+        overlaps(dx, ab, acts, (size_t)(L > 1 ? L - 1 : 0) * ab))
+        return HCW_ERR_ALIASING;
+    cudaStream_t st = (cudaStream_t)stream;
+    uint8_t* wsb = static_cast<uint8_t*>(workspace);
+    uint8_t* g[2] = {wsb, wsb + align256(ab)};
+    void* lws = wsb + 2 * align256(ab);
+    const void* cur = dy;
+    for (int l = L - 1; l >= 0; --l) {
+        Shape shl = sh;
+        shl.s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
+        const void* in = l == 0 ? x : static_cast<const uint8_t*>(acts) + (size_t)(l - 1) * ab;
+        const void* z = zs ? static_cast<const uint8_t*>(zs) + (size_t)l * ab : nullptr;
+        void* out = l == 0 ? dx : g[l & 1];
+        rc = layer_bwd_impl(shl, dtype, in, z, cur, static_cast<const uint8_t*>(W_self) + l * wb,
+                            static_cast<const uint8_t*>(W_nbr) + l * wb, flags, out,
+                            dW_self + (size_t)l * d * d, dW_nbr + (size_t)l * d * d,
+                            dbias ? dbias + (size_t)l * d : nullptr, lws, st);
+        if (rc) return rc;
+        cur = out;
+    }
+    return HCW_OK;
+}
+
+unsigned long long hcw_launch_count(void) { return g_launches.load(); }
+
+int hcw_sync_status(void* stream) {
+    if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return HCW_ERR_CUDA;
+    int word = 0;
+    if (error_word_read_clear(&word) != cudaSuccess) return HCW_ERR_CUDA;
+    if (word) return word == HCW_ERR_TIMEOUT ? HCW_ERR_TIMEOUT : HCW_ERR_CUDA;
+    return HCW_OK;
+}
+
+int hcw_selftest_wait(long long timeout_ns, void* stream) {
+    if (timeout_ns < 1000 || timeout_ns > 10000000000ll) return HCW_ERR_INVALID_ARG;
+    return launched(launch_wait_selftest((unsigned long long)timeout_ns, (cudaStream_t)stream),
+                    1);
+}
+
+}  // extern "C"

@@ -1,0 +1,93 @@
+// hcw_internal.h -- launch interfaces shared by the translation units of
+// libhcw (not part of the public ABI, which is include/hcw.h).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace hcw {
+
+enum TcMode { MODE_FWD = 0, MODE_DX = 1, MODE_DW = 2 };
+
+// Work description of one tensor-core launch (see hcw_tc.cu for the unit
+// decomposition).  Row indices are "compressed": for a fixed value beta of
+// bit s, q = HI * k + lo enumerates the Mh = B*n/2 positions whose bit s is
+// beta; the position (within the flattened [B*n] token axis) is
+// HI * 2k + beta * k + lo.
+struct TcParams {
+    int d;          // feature width
+    int k;          // 2^s, the link distance of this layer
+    int Mh;         // positions per value of bit s: B * n / 2
+    int nK;         // d / 64: K-steps per part (FWD, DX)
+    // FWD / DX units
+    int n_rb;       // ceil(Mh / 128) row blocks per bit value
+    int n_nt;       // d / BN output column tiles
+    int n_full;     // number of bit values whose rows take both parts (1 or 2)
+    int full_bit0;  // bit value of the first full group
+    int full_bit1;  // bit value of the second full group (if n_full == 2)
+    int half_bit;   // bit value of the rows that take only the self part, -1 if none
+    // DW units
+    int n_ot;       // ceil(d / 128) output row tiles (o)
+    int qb;         // ceil(Mh / 64) token blocks per bit value
+    int nkb_self;   // token blocks of the self part: 2 * qb
+    int nkb_nbr;    // token blocks of the partner part: qb (causal) or 2 * qb
+    int kb_per_unit;
+    int splits_self;
+    int splits_nbr;
+    int causal;
+    int n_units;
+    // epilogue
+    unsigned flags;
+    const float* bias;            // FWD
+    const __nv_bfloat16* resid;   // FWD: x; DX: dy
+    __nv_bfloat16* out;           // FWD: y; DX: dx
+    __nv_bfloat16* zout;          // FWD: z (may be null)
+    float* dw_self;               // DW destination when splits_self == 1
+    float* dw_nbr;                // DW destination when splits_nbr == 1
+    float* dw_partial;            // DW partials [2][splits_max][d][d]
+    int splits_max;
+    unsigned long long timeout_ns;
+};
+
+// Launch one tensor-core pass.  tmA / tmB0 / tmB1 as documented in hcw_tc.cu.
+cudaError_t launch_tc(int mode, int BN, const CUtensorMap& tmA, const CUtensorMap& tmB0,
+                      const CUtensorMap& tmB1, const TcParams& p, int grid,
+                      cudaStream_t stream);
+
+// Dynamic shared memory the tensor-core kernel uses for this N tile.
+size_t tc_smem_bytes(int BN);
+int tc_stages(int BN);
+
+// ---- SIMT kernels (hcw_simt.cu) ----
+cudaError_t launch_f32_fwd(const float* x, const float* Ws, const float* Wn, const float* bias,
+                           int s, int B, int n, int d, unsigned flags, float* y, float* z,
+                           cudaStream_t st);
+cudaError_t launch_f32_dx(const float* dz, const float* dy, const float* Ws, const float* Wn,
+                          int s, int B, int n, int d, unsigned flags, float* dx,
+                          cudaStream_t st);
+cudaError_t launch_f32_dw(const float* x, const float* dz, int s, int B, int n, int d,
+                          unsigned flags, float* dWs, float* dWn, cudaStream_t st);
+// dz = dy * (z > 0), elementwise over count elements (T = float or bf16)
+cudaError_t launch_relu_grad_f32(const float* dy, const float* z, float* dz, size_t count,
+                                 cudaStream_t st);
+cudaError_t launch_relu_grad_bf16(const __nv_bfloat16* dy, const __nv_bfloat16* z,
+                                  __nv_bfloat16* dz, size_t count, cudaStream_t st);
+// dbias[o] = sum_t dz[t][o], deterministic two-pass column sum.
+size_t colsum_workspace_bytes(long long rows, int d);
+cudaError_t launch_colsum_f32(const float* dz, long long rows, int d, float* partial,
+                              float* out, cudaStream_t st);
+cudaError_t launch_colsum_bf16(const __nv_bfloat16* dz, long long rows, int d, float* partial,
+                               float* out, cudaStream_t st);
+// out_w[o][k] = sum_{s < splits_w} partial[w][s][o][k] for w in {self, nbr}
+cudaError_t launch_splitk_reduce(const float* partial, int splits_max, int splits_self,
+                                 int splits_nbr, int d, float* dWs, float* dWn,
+                                 cudaStream_t st);
+cudaError_t launch_partner_table(int s, int n, unsigned flags, int* out, cudaStream_t st);
+cudaError_t launch_wait_selftest(unsigned long long timeout_ns, cudaStream_t st);
+// Read the current device's error word and reset it to 0 (synchronous).
+cudaError_t error_word_read_clear(int* word);
+
+}  // namespace hcw

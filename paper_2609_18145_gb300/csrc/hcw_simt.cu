@@ -1,0 +1,345 @@
+// hcw_simt.cu -- CUDA-core kernels of libhcw:
+//   * the fp32 path of the layer (forward, input gradient, weight gradient),
+//     tiled FFMA with fp32 accumulation, for callers that need fp32 accuracy;
+//   * the elementwise / reduction helpers of the bf16 path: ReLU gradient
+//     mask, deterministic column sums (dbias), split-K reduction of dW;
+//   * the device partner table (same index code as the kernels).
+//
+// Index rules (Sec. 3.1): partner p(i) = i XOR 2^s inside each sample;
+// causal: i receives from p(i) iff bit s of i is set.
+#include "hcw_internal.h"
+
+namespace hcw {
+
+namespace {
+
+__device__ __forceinline__ int partner_of(int i, int s) { return i ^ (1 << s); }
+
+__device__ __forceinline__ bool receives(int i, int s, unsigned flags) {
+    return !(flags & 1u) || ((i >> s) & 1);
+}
+
+constexpr int T = 32;   // tile edge of the fp32 kernels
+
+// z[r][o] = sum_k Ws[o][k] x[r][k] + m_r sum_k Wn[o][k] x[p(r)][k] + bias[o]
+// Block: 32 rows x 32 outputs, 32 x 8 threads, 4 outputs per thread.
+__global__ void f32_fwd_kernel(const float* __restrict__ x, const float* __restrict__ Ws,
+                               const float* __restrict__ Wn, const float* __restrict__ bias,
+                               int s, int n, int d, long long rows, unsigned flags,
+                               float* __restrict__ y, float* __restrict__ z) {
+    __shared__ float xs[T][T + 1], xp[T][T + 1], ws[T][T + 1], wn[T][T + 1];
+    const long long r0 = (long long)blockIdx.y * T;
+    const int o0 = blockIdx.x * T;
+    const int tx = threadIdx.x, ty = threadIdx.y;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int k0 = 0; k0 < d; k0 += T) {
+        for (int rr = ty; rr < T; rr += 8) {
+            const long long r = r0 + rr;
+            const int k = k0 + tx;
+            float a = 0.f, b = 0.f;
+            if (r < rows && k < d) {
+                const int i = (int)(r % n);
+                const long long rp = r - i + partner_of(i, s);
+                a = x[r * d + k];
+                b = receives(i, s, flags) ? x[rp * d + k] : 0.f;
+            }
+            xs[rr][tx] = a;
+            xp[rr][tx] = b;
+            const int o = o0 + rr;
+            ws[rr][tx] = (o < d && k < d) ? Ws[(long long)o * d + k] : 0.f;
+            wn[rr][tx] = (o < d && k < d) ? Wn[(long long)o * d + k] : 0.f;
+        }
+        __syncthreads();
+#pragma unroll 8
+        for (int kk = 0; kk < T; ++kk) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int rr = ty + 8 * q;
+                acc[q] = fmaf(xs[rr][kk], ws[tx][kk], acc[q]);
+                acc[q] = fmaf(xp[rr][kk], wn[tx][kk], acc[q]);
+            }
+        }
+        __syncthreads();
+    }
+    const int o = o0 + tx;
+    if (o >= d) return;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const long long r = r0 + ty + 8 * q;
+        if (r >= rows) continue;
+        float v = acc[q] + (bias ? bias[o] : 0.f);
+        if (z) z[r * d + o] = v;
+        if (flags & 4u) v = v > 0.f ? v : 0.f;
+        if (flags & 2u) v += x[r * d + o];
+        y[r * d + o] = v;
+    }
+}
+
+// dx[r][k] = sum_o dz[r][o] Ws[o][k] + m_{p(r)} sum_o dz[p(r)][o] Wn[o][k] (+ dy[r][k])
+__global__ void f32_dx_kernel(const float* __restrict__ dz, const float* __restrict__ dy,
+                              const float* __restrict__ Ws, const float* __restrict__ Wn, int s,
+                              int n, int d, long long rows, unsigned flags,
+                              float* __restrict__ dx) {
+    __shared__ float gs[T][T + 1], gp[T][T + 1], ws[T][T + 1], wn[T][T + 1];
+    const long long r0 = (long long)blockIdx.y * T;
+    const int k0 = blockIdx.x * T;
+    const int tx = threadIdx.x, ty = threadIdx.y;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int o0 = 0; o0 < d; o0 += T) {
+        for (int rr = ty; rr < T; rr += 8) {
+            const long long r = r0 + rr;
+            const int o = o0 + tx;
+            float a = 0.f, b = 0.f;
+            if (r < rows && o < d) {
+                const int i = (int)(r % n);
+                const int pi = partner_of(i, s);
+                const long long rp = r - i + pi;
+                a = dz[r * d + o];
+                b = receives(pi, s, flags) ? dz[rp * d + o] : 0.f;
+            }
+            gs[rr][tx] = a;
+            gp[rr][tx] = b;
+            const int oo = o0 + rr, k = k0 + tx;
+            ws[rr][tx] = (oo < d && k < d) ? Ws[(long long)oo * d + k] : 0.f;
+            wn[rr][tx] = (oo < d && k < d) ? Wn[(long long)oo * d + k] : 0.f;
+        }
+        __syncthreads();
+#pragma unroll 8
+        for (int oo = 0; oo < T; ++oo) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int rr = ty + 8 * q;
+                acc[q] = fmaf(gs[rr][oo], ws[oo][tx], acc[q]);
+                acc[q] = fmaf(gp[rr][oo], wn[oo][tx], acc[q]);
+            }
+        }
+        __syncthreads();
+    }
+    const int k = k0 + tx;
+    if (k >= d) return;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const long long r = r0 + ty + 8 * q;
+        if (r >= rows) continue;
+        float v = acc[q];
+        if (flags & 2u) v += dy[r * d + k];
+        dx[r * d + k] = v;
+    }
+}
+
+// dWs[o][k] = sum_r dz[r][o] x[r][k];  dWn[o][k] = sum_r m_r dz[r][o] x[p(r)][k]
+// Block: 32 o x 32 k; the token loop is sequential (fixed order).
+__global__ void f32_dw_kernel(const float* __restrict__ x, const float* __restrict__ dz, int s,
+                              int n, int d, long long rows, unsigned flags,
+                              float* __restrict__ dWs, float* __restrict__ dWn) {
+    __shared__ float gz[T][T + 1], xs[T][T + 1], xp[T][T + 1];
+    const int o0 = blockIdx.y * T, k0 = blockIdx.x * T;
+    const int tx = threadIdx.x, ty = threadIdx.y;
+    float as[4] = {0.f, 0.f, 0.f, 0.f}, an[4] = {0.f, 0.f, 0.f, 0.f};
+    for (long long r0 = 0; r0 < rows; r0 += T) {
+        for (int rr = ty; rr < T; rr += 8) {
+            const long long r = r0 + rr;
+            float g = 0.f, a = 0.f, b = 0.f;
+            if (r < rows) {
+                const int i = (int)(r % n);
+                const long long rp = r - i + partner_of(i, s);
+                if (o0 + tx < d) g = dz[r * d + o0 + tx];
+                if (k0 + tx < d) {
+                    a = x[r * d + k0 + tx];
+                    b = receives(i, s, flags) ? x[rp * d + k0 + tx] : 0.f;
+                }
+            }
+            gz[rr][tx] = g;
+            xs[rr][tx] = a;
+            xp[rr][tx] = b;
+        }
+        __syncthreads();
+#pragma unroll 8
+        for (int rr = 0; rr < T; ++rr) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const float g = gz[rr][ty + 8 * q];
+                as[q] = fmaf(g, xs[rr][tx], as[q]);
+                an[q] = fmaf(g, xp[rr][tx], an[q]);
+            }
+        }
+        __syncthreads();
+    }
+    const int k = k0 + tx;
+    if (k >= d) return;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int o = o0 + ty + 8 * q;
+        if (o >= d) continue;
+        dWs[(long long)o * d + k] = as[q];
+        dWn[(long long)o * d + k] = an[q];
+    }
+}
+
+template <typename V>
+__device__ __forceinline__ float to_f(V v);
+template <>
+__device__ __forceinline__ float to_f<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ float to_f<__nv_bfloat16>(__nv_bfloat16 v) {
+    return __bfloat162float(v);
+}
+
+template <typename V>
+__global__ void relu_grad_kernel(const V* __restrict__ dy, const V* __restrict__ z,
+                                 V* __restrict__ dz, size_t count) {
+    const V zero = V(0.f);
+    for (size_t t = (size_t)blockIdx.x * blockDim.x + threadIdx.x; t < count;
+         t += (size_t)gridDim.x * blockDim.x)
+        dz[t] = to_f(z[t]) > 0.f ? dy[t] : zero;
+}
+
+constexpr int kColRows = 256;   // rows per partial of the column sum
+
+// partial[c][o] = sum_{r in chunk c} dz[r][o]  (block: 32 columns x 8 row lanes)
+template <typename V>
+__global__ void colsum_partial_kernel(const V* __restrict__ dz, long long rows, int d,
+                                      float* __restrict__ partial) {
+    __shared__ float red[8][33];
+    const int o = blockIdx.x * 32 + threadIdx.x;
+    const long long r0 = (long long)blockIdx.y * kColRows;
+    const long long r1 = min(rows, r0 + kColRows);
+    float acc = 0.f;
+    if (o < d)
+        for (long long r = r0 + threadIdx.y; r < r1; r += 8) acc += to_f(dz[r * d + o]);
+    red[threadIdx.y][threadIdx.x] = acc;
+    __syncthreads();
+    if (threadIdx.y == 0 && o < d) {
+        float s = 0.f;
+        for (int q = 0; q < 8; ++q) s += red[q][threadIdx.x];
+        partial[(long long)blockIdx.y * d + o] = s;
+    }
+}
+
+__global__ void colsum_final_kernel(const float* __restrict__ partial, int chunks, int d,
+                                    float* __restrict__ out) {
+    const int o = blockIdx.x * blockDim.x + threadIdx.x;
+    if (o >= d) return;
+    float s = 0.f;
+    for (int c = 0; c < chunks; ++c) s += partial[(long long)c * d + o];
+    out[o] = s;
+}
+
+__global__ void splitk_reduce_kernel(const float* __restrict__ partial, int splits_max,
+                                     int splits_self, int splits_nbr, int d,
+                                     float* __restrict__ dWs, float* __restrict__ dWn) {
+    const size_t dd = (size_t)d * d;
+    const size_t total4 = dd / 4;
+    for (size_t t = (size_t)blockIdx.x * blockDim.x + threadIdx.x; t < 2 * total4;
+         t += (size_t)gridDim.x * blockDim.x) {
+        const int which = t >= total4;
+        const size_t e4 = t - which * total4;
+        const int S = which ? splits_nbr : splits_self;
+        if (S <= 1) continue;   // written directly by the GEMM
+        const float4* src = reinterpret_cast<const float4*>(partial + (size_t)which * splits_max * dd);
+        float4 a = src[e4];
+        for (int sp = 1; sp < S; ++sp) {
+            float4 b = src[(size_t)sp * total4 + e4];
+            a.x += b.x;
+            a.y += b.y;
+            a.z += b.z;
+            a.w += b.w;
+        }
+        reinterpret_cast<float4*>(which ? dWn : dWs)[e4] = a;
+    }
+}
+
+__global__ void partner_table_kernel(int s, int n, unsigned flags, int* out) {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < n) out[i] = receives(i, s, flags) ? partner_of(i, s) : -1;
+}
+
+inline int blocks_for(size_t count, int threads, int cap = 152 * 16) {
+    size_t b = (count + threads - 1) / threads;
+    return (int)(b < (size_t)cap ? (b == 0 ? 1 : b) : cap);
+}
+
+}  // namespace
+
+cudaError_t launch_f32_fwd(const float* x, const float* Ws, const float* Wn, const float* bias,
+                           int s, int B, int n, int d, unsigned flags, float* y, float* z,
+                           cudaStream_t st) {
+    const long long rows = (long long)B * n;
+    dim3 grid((d + T - 1) / T, (unsigned)((rows + T - 1) / T));
+    f32_fwd_kernel<<<grid, dim3(T, 8), 0, st>>>(x, Ws, Wn, bias, s, n, d, rows, flags, y, z);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_f32_dx(const float* dz, const float* dy, const float* Ws, const float* Wn,
+                          int s, int B, int n, int d, unsigned flags, float* dx,
+                          cudaStream_t st) {
+    const long long rows = (long long)B * n;
+    dim3 grid((d + T - 1) / T, (unsigned)((rows + T - 1) / T));
+    f32_dx_kernel<<<grid, dim3(T, 8), 0, st>>>(dz, dy, Ws, Wn, s, n, d, rows, flags, dx);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_f32_dw(const float* x, const float* dz, int s, int B, int n, int d,
+                          unsigned flags, float* dWs, float* dWn, cudaStream_t st) {
+    const long long rows = (long long)B * n;
+    dim3 grid((d + T - 1) / T, (d + T - 1) / T);
+    f32_dw_kernel<<<grid, dim3(T, 8), 0, st>>>(x, dz, s, n, d, rows, flags, dWs, dWn);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_relu_grad_f32(const float* dy, const float* z, float* dz, size_t count,
+                                 cudaStream_t st) {
+    relu_grad_kernel<float><<<blocks_for(count, 256), 256, 0, st>>>(dy, z, dz, count);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_relu_grad_bf16(const __nv_bfloat16* dy, const __nv_bfloat16* z,
+                                  __nv_bfloat16* dz, size_t count, cudaStream_t st) {
+    relu_grad_kernel<__nv_bfloat16><<<blocks_for(count, 256), 256, 0, st>>>(dy, z, dz, count);
+    return cudaGetLastError();
+}
+
+size_t colsum_workspace_bytes(long long rows, int d) {
+    const long long chunks = (rows + kColRows - 1) / kColRows;
+    return (size_t)(chunks < 1 ? 1 : chunks) * (size_t)d * sizeof(float);
+}
+
+template <typename V>
+static cudaError_t colsum(const V* dz, long long rows, int d, float* partial, float* out,
+                          cudaStream_t st) {
+    const long long chunks = (rows + kColRows - 1) / kColRows;
+    if (chunks == 0) {
+        cudaError_t e = cudaMemsetAsync(out, 0, (size_t)d * sizeof(float), st);
+        return e;
+    }
+    dim3 grid((d + 31) / 32, (unsigned)chunks);
+    colsum_partial_kernel<V><<<grid, dim3(32, 8), 0, st>>>(dz, rows, d, partial);
+    colsum_final_kernel<<<(d + 127) / 128, 128, 0, st>>>(partial, (int)chunks, d, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_colsum_f32(const float* dz, long long rows, int d, float* partial,
+                              float* out, cudaStream_t st) {
+    return colsum<float>(dz, rows, d, partial, out, st);
+}
+
+cudaError_t launch_colsum_bf16(const __nv_bfloat16* dz, long long rows, int d, float* partial,
+                               float* out, cudaStream_t st) {
+    return colsum<__nv_bfloat16>(dz, rows, d, partial, out, st);
+}
+
+cudaError_t launch_splitk_reduce(const float* partial, int splits_max, int splits_self,
+                                 int splits_nbr, int d, float* dWs, float* dWn,
+                                 cudaStream_t st) {
+    const size_t total4 = (size_t)d * d / 4;
+    splitk_reduce_kernel<<<blocks_for(2 * total4, 256), 256, 0, st>>>(
+        partial, splits_max, splits_self, splits_nbr, d, dWs, dWn);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_partner_table(int s, int n, unsigned flags, int* out, cudaStream_t st) {
+    partner_table_kernel<<<(n + 255) / 256, 256, 0, st>>>(s, n, flags, out);
+    return cudaGetLastError();
+}
+
+}  // namespace hcw

@@ -1,0 +1,291 @@
+"""Thin ctypes binding of libhcw (include/hcw.h), same names as the C ABI.
+
+Argument marshalling only: every step of the mixing path runs in the CUDA
+kernels of libhcw.  torch supplies device memory and the current stream.
+There is no fallback: if libhcw.so is missing or a call fails, an exception
+is raised.
+
+Layouts (Sec. 3.1 wiring, Eq. (1) maps): activations [B, n, d] contiguous;
+weights [d_out, d_in] acting on column vectors (stacks: [L, d, d]); bias and
+weight gradients fp32.  dtype follows x: torch.bfloat16 -> HCW_BF16,
+torch.float32 -> HCW_F32.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+HCW_OK = 0
+HCW_ERR_INVALID_ARG = 1
+HCW_ERR_UNSUPPORTED = 2
+HCW_ERR_ALIGNMENT = 3
+HCW_ERR_ALIASING = 4
+HCW_ERR_CUDA = 5
+HCW_ERR_TIMEOUT = 6
+HCW_ERR_WORKSPACE = 7
+
+HCW_BF16 = 0
+HCW_F32 = 1
+
+HCW_CAUSAL = 1
+HCW_RESIDUAL = 2
+HCW_ACT_RELU = 4
+
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libhcw.so")
+
+_lock = threading.Lock()
+_lib = None
+
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+_U = ctypes.c_uint
+_SZ = ctypes.c_size_t
+_LL = ctypes.c_longlong
+
+_SIGNATURES = {
+    "hcw_version": ([], _I),
+    "hcw_status_string": ([_I], ctypes.c_char_p),
+    "hcw_partner_table": ([_I, _I, _I, _U, _P], _I),
+    "hcw_partner_table_device": ([_I, _I, _I, _U, _P, _P], _I),
+    "hcw_layer_fwd": ([_P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P], _I),
+    "hcw_workspace_bytes": ([_I, _I, _I, _I, _U], _SZ),
+    "hcw_layer_bwd": ([_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P, _P,
+                       _SZ, _P], _I),
+    "hcw_layer_bwd_data": ([_P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _U, _P, _P], _I),
+    "hcw_layer_bwd_weight_workspace_bytes": ([_I, _I, _I, _I, _U], _SZ),
+    "hcw_layer_bwd_weight": ([_P, _P, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P, _SZ, _P], _I),
+    "hcw_launch_count": ([], ctypes.c_ulonglong),
+    "hcw_stack_fwd": ([_P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P], _I),
+    "hcw_stack_workspace_bytes": ([_I, _I, _I, _I, _U], _SZ),
+    "hcw_stack_bwd": ([_P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P,
+                       _P, _P, _SZ, _P], _I),
+    "hcw_sync_status": ([_P], _I),
+    "hcw_selftest_wait": ([_LL, _P], _I),
+}
+
+EXPORTED = tuple(_SIGNATURES)
+
+
+class HcwError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__("%s failed: %s (%d)" % (what, status_string(status), status))
+
+
+def lib() -> ctypes.CDLL:
+    """Load libhcw.so (built in-tree by build()); raise if it is missing."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise RuntimeError(
+                    "libhcw.so not found at %s: run __graft_entry__.build() (or "
+                    "python -m paper_2609_18145_gb300._build) first" % LIB_PATH)
+            L = ctypes.CDLL(LIB_PATH)
+            for name, (args, res) in _SIGNATURES.items():
+                f = getattr(L, name)
+                f.argtypes = args
+                f.restype = res
+            _lib = L
+    return _lib
+
+
+def status_string(status: int) -> str:
+    return lib().hcw_status_string(status).decode()
+
+
+def _check(rc: int, what: str):
+    if rc != HCW_OK:
+        raise HcwError(rc, what)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return HCW_BF16
+    if t.dtype == torch.float32:
+        return HCW_F32
+    raise TypeError("activations must be bfloat16 or float32, got %s" % t.dtype)
+
+
+def _dev(*ts):
+    for t in ts:
+        if t is None:
+            continue
+        if not t.is_cuda:
+            raise ValueError("all tensors must be CUDA tensors")
+        if not t.is_contiguous():
+            raise ValueError("all tensors must be contiguous")
+
+
+def hcw_version() -> int:
+    return lib().hcw_version()
+
+
+def hcw_partner_table(layer: int, n: int, flags: int = 0, dim_override: int = -1):
+    """Host partner table: list of n ints (-1 where the position does not receive)."""
+    buf = (ctypes.c_int * n)()
+    _check(lib().hcw_partner_table(layer, dim_override, n, flags, buf), "hcw_partner_table")
+    return list(buf)
+
+
+def hcw_partner_table_device(layer: int, n: int, flags: int = 0, dim_override: int = -1,
+                             device=None, stream=None) -> torch.Tensor:
+    out = torch.empty(n, dtype=torch.int32, device=device or "cuda")
+    _check(lib().hcw_partner_table_device(layer, dim_override, n, flags, _ptr(out),
+                                          _stream(stream)), "hcw_partner_table_device")
+    return out
+
+
+def hcw_layer_fwd(x, W_self, W_nbr, bias=None, layer: int = 0, dim_override: int = -1,
+                  flags: int = 0, y=None, z_save=None, want_z: bool = False, stream=None):
+    """One layer forward; returns y (and z_save if want_z or given)."""
+    _dev(x, W_self, W_nbr, bias, y, z_save)
+    B, n, d = x.shape
+    if y is None:
+        y = torch.empty_like(x)
+    if want_z and z_save is None:
+        z_save = torch.empty_like(x)
+    _check(lib().hcw_layer_fwd(_ptr(x), _ptr(W_self), _ptr(W_nbr), _ptr(bias), layer,
+                               dim_override, B, n, d, _dtype_code(x), flags, _ptr(y),
+                               _ptr(z_save), _stream(stream)), "hcw_layer_fwd")
+    return (y, z_save) if z_save is not None else y
+
+
+def hcw_workspace_bytes(B: int, n: int, d: int, dtype: int, flags: int) -> int:
+    return int(lib().hcw_workspace_bytes(B, n, d, dtype, flags))
+
+
+def hcw_stack_workspace_bytes(B: int, n: int, d: int, dtype: int, flags: int) -> int:
+    return int(lib().hcw_stack_workspace_bytes(B, n, d, dtype, flags))
+
+
+def _workspace(nbytes, device, workspace):
+    if workspace is not None:
+        return workspace
+    return torch.empty(max(nbytes, 1), dtype=torch.uint8, device=device)
+
+
+def hcw_layer_bwd(x, z_save, dy, W_self, W_nbr, layer: int = 0, dim_override: int = -1,
+                  flags: int = 0, dx=None, dW_self=None, dW_nbr=None, dbias=None,
+                  want_dbias: bool = True, workspace=None, stream=None):
+    """One layer backward; returns (dx, dW_self, dW_nbr, dbias)."""
+    _dev(x, z_save, dy, W_self, W_nbr, dx, dW_self, dW_nbr, dbias, workspace)
+    B, n, d = x.shape
+    dt = _dtype_code(x)
+    f32 = dict(dtype=torch.float32, device=x.device)
+    dx = torch.empty_like(x) if dx is None else dx
+    dW_self = torch.empty(d, d, **f32) if dW_self is None else dW_self
+    dW_nbr = torch.empty(d, d, **f32) if dW_nbr is None else dW_nbr
+    if dbias is None and want_dbias:
+        dbias = torch.empty(d, **f32)
+    need = hcw_workspace_bytes(B, n, d, dt, flags)
+    ws = _workspace(need, x.device, workspace)
+    _check(lib().hcw_layer_bwd(_ptr(x), _ptr(z_save), _ptr(dy), _ptr(W_self), _ptr(W_nbr),
+                               layer, dim_override, B, n, d, dt, flags, _ptr(dx),
+                               _ptr(dW_self), _ptr(dW_nbr), _ptr(dbias), _ptr(ws),
+                               ws.numel(), _stream(stream)), "hcw_layer_bwd")
+    return dx, dW_self, dW_nbr, dbias
+
+
+def hcw_layer_bwd_data(dz, dy, W_self, W_nbr, layer: int = 0, dim_override: int = -1,
+                       flags: int = 0, dx=None, stream=None):
+    """Input gradient of one layer from dz = dy * act'(z); returns dx."""
+    _dev(dz, dy, W_self, W_nbr, dx)
+    B, n, d = dz.shape
+    dx = torch.empty_like(dz) if dx is None else dx
+    _check(lib().hcw_layer_bwd_data(_ptr(dz), _ptr(dy), _ptr(W_self), _ptr(W_nbr), layer,
+                                    dim_override, B, n, d, _dtype_code(dz), flags, _ptr(dx),
+                                    _stream(stream)), "hcw_layer_bwd_data")
+    return dx
+
+
+def hcw_layer_bwd_weight_workspace_bytes(B: int, n: int, d: int, dtype: int, flags: int) -> int:
+    return int(lib().hcw_layer_bwd_weight_workspace_bytes(B, n, d, dtype, flags))
+
+
+def hcw_layer_bwd_weight(x, dz, layer: int = 0, dim_override: int = -1, flags: int = 0,
+                         dW_self=None, dW_nbr=None, dbias=None, want_dbias: bool = True,
+                         workspace=None, stream=None):
+    """Weight gradients of one layer; returns (dW_self, dW_nbr, dbias)."""
+    _dev(x, dz, dW_self, dW_nbr, dbias, workspace)
+    B, n, d = x.shape
+    dt = _dtype_code(x)
+    f32 = dict(dtype=torch.float32, device=x.device)
+    dW_self = torch.empty(d, d, **f32) if dW_self is None else dW_self
+    dW_nbr = torch.empty(d, d, **f32) if dW_nbr is None else dW_nbr
+    if dbias is None and want_dbias:
+        dbias = torch.empty(d, **f32)
+    ws = _workspace(hcw_layer_bwd_weight_workspace_bytes(B, n, d, dt, flags), x.device,
+                    workspace)
+    _check(lib().hcw_layer_bwd_weight(_ptr(x), _ptr(dz), layer, dim_override, B, n, d, dt, flags,
+                                      _ptr(dW_self), _ptr(dW_nbr), _ptr(dbias), _ptr(ws),
+                                      ws.numel(), _stream(stream)), "hcw_layer_bwd_weight")
+    return dW_self, dW_nbr, dbias
+
+
+def hcw_launch_count() -> int:
+    """Kernels launched by libhcw in this process so far."""
+    return int(lib().hcw_launch_count())
+
+
+def hcw_stack_fwd(x, W_self, W_nbr, bias=None, layer0: int = 0, dim_override: int = -1,
+                  flags: int = 0, y=None, acts=None, zs=None, want_z: bool = False,
+                  stream=None):
+    """Stack forward over L = W_self.shape[0] layers; returns (y, acts, zs)."""
+    _dev(x, W_self, W_nbr, bias, y, acts, zs)
+    B, n, d = x.shape
+    L = W_self.shape[0]
+    y = torch.empty_like(x) if y is None else y
+    if acts is None and L > 1:
+        acts = torch.empty((L - 1, B, n, d), dtype=x.dtype, device=x.device)
+    if zs is None and want_z:
+        zs = torch.empty((L, B, n, d), dtype=x.dtype, device=x.device)
+    _check(lib().hcw_stack_fwd(_ptr(x), _ptr(W_self), _ptr(W_nbr), _ptr(bias), layer0, L,
+                               dim_override, B, n, d, _dtype_code(x), flags, _ptr(y),
+                               _ptr(acts), _ptr(zs), _stream(stream)), "hcw_stack_fwd")
+    return y, acts, zs
+
+
+def hcw_stack_bwd(x, acts, zs, dy, W_self, W_nbr, layer0: int = 0, dim_override: int = -1,
+                  flags: int = 0, dx=None, dW_self=None, dW_nbr=None, dbias=None,
+                  want_dbias: bool = True, workspace=None, stream=None):
+    """Stack backward; returns (dx, dW_self[L], dW_nbr[L], dbias[L])."""
+    _dev(x, acts, zs, dy, W_self, W_nbr, dx, dW_self, dW_nbr, dbias, workspace)
+    B, n, d = x.shape
+    L = W_self.shape[0]
+    dt = _dtype_code(x)
+    f32 = dict(dtype=torch.float32, device=x.device)
+    dx = torch.empty_like(x) if dx is None else dx
+    dW_self = torch.empty(L, d, d, **f32) if dW_self is None else dW_self
+    dW_nbr = torch.empty(L, d, d, **f32) if dW_nbr is None else dW_nbr
+    if dbias is None and want_dbias:
+        dbias = torch.empty(L, d, **f32)
+    need = hcw_stack_workspace_bytes(B, n, d, dt, flags)
+    ws = _workspace(need, x.device, workspace)
+    _check(lib().hcw_stack_bwd(_ptr(x), _ptr(acts), _ptr(zs), _ptr(dy), _ptr(W_self),
+                               _ptr(W_nbr), layer0, L, dim_override, B, n, d, dt, flags,
+                               _ptr(dx), _ptr(dW_self), _ptr(dW_nbr), _ptr(dbias), _ptr(ws),
+                               ws.numel(), _stream(stream)), "hcw_stack_bwd")
+    return dx, dW_self, dW_nbr, dbias
+
+
+def hcw_sync_status(stream=None) -> int:
+    """Synchronise the stream and return (and clear) the device error status."""
+    return int(lib().hcw_sync_status(_stream(stream)))
+
+
+def hcw_selftest_wait(timeout_ns: int, stream=None):
+    _check(lib().hcw_selftest_wait(int(timeout_ns), _stream(stream)), "hcw_selftest_wait")

@@ -1,0 +1,140 @@
+"""The C-ABI library: it loads without a GPU, exports every entry point that
+include/hcw.h declares, and its host-side logic (partner tables, argument
+validation) behaves as documented.  No call here launches a kernel."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from paper_2609_18145_gb300 import _build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def hcw():
+    _build.build()
+    from paper_2609_18145_gb300 import hcw as H
+    H.lib()
+    return H
+
+
+def declared_symbols():
+    text = open(os.path.join(ROOT, "include", "hcw.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(hcw_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_header_declares_the_path():
+    syms = declared_symbols()
+    for name in ("hcw_layer_fwd", "hcw_layer_bwd", "hcw_stack_fwd", "hcw_stack_bwd",
+                 "hcw_workspace_bytes", "hcw_partner_table", "hcw_status_string"):
+        assert name in syms
+
+
+def test_library_exports_every_declared_symbol(hcw):
+    lib = ctypes.CDLL(hcw.LIB_PATH)
+    missing = [s for s in declared_symbols() if not hasattr(lib, s)]
+    assert not missing, missing
+    assert sorted(hcw.EXPORTED) == declared_symbols()
+
+
+def test_version_and_status_strings(hcw):
+    assert hcw.hcw_version() >= 100
+    assert hcw.status_string(0) == "HCW_OK"
+    assert hcw.status_string(6) == "HCW_ERR_TIMEOUT"
+    assert hcw.status_string(99) == "HCW_ERR_UNKNOWN"
+
+
+@pytest.mark.parametrize("n", [2, 4, 16, 64, 256, 65536])
+@pytest.mark.parametrize("flags", [0, 1])
+def test_host_partner_table_matches_oracle(hcw, n, flags):
+    b = n.bit_length() - 1
+    for layer in list(range(2 * b)) + [1000]:
+        got = np.array(hcw.hcw_partner_table(layer, n, flags))
+        ref = O.partner_table(layer, -1, n, flags)
+        assert np.array_equal(got, ref)
+    for dim in range(b):
+        got = np.array(hcw.hcw_partner_table(3, n, flags, dim_override=dim))
+        assert np.array_equal(got, O.partner_table(3, dim, n, flags))
+
+
+def test_host_partner_table_rejects(hcw):
+    L = hcw.lib()
+    buf = (ctypes.c_int * 64)()
+    assert L.hcw_partner_table(0, -1, 48, 0, buf) == hcw.HCW_ERR_INVALID_ARG
+    assert L.hcw_partner_table(0, 6, 64, 0, buf) == hcw.HCW_ERR_INVALID_ARG
+    assert L.hcw_partner_table(-1, -1, 64, 0, buf) == hcw.HCW_ERR_INVALID_ARG
+    assert L.hcw_partner_table(0, -1, 64, 0, None) == hcw.HCW_ERR_INVALID_ARG
+    assert L.hcw_partner_table(0, -1, 64, 64, buf) == hcw.HCW_ERR_INVALID_ARG
+
+
+def _fwd(hcw, x, ws, wn, bias, layer, dim, B, n, d, dt, flags, y, z):
+    P = ctypes.c_void_p
+    return hcw.lib().hcw_layer_fwd(P(x), P(ws), P(wn), P(bias), layer, dim, B, n, d, dt, flags,
+                                   P(y), P(z), None)
+
+
+def test_forward_validation_codes(hcw):
+    # fake, never dereferenced addresses: validation returns before any launch
+    X, WS, WN, Y = 0x100000, 0x200000, 0x300000, 0x400000
+    ok = dict(layer=0, dim=-1, B=4, n=16, d=64, dt=hcw.HCW_BF16, flags=0)
+
+    def call(**kw):
+        a = dict(ok, **kw)
+        return _fwd(hcw, a.get("x", X), a.get("ws", WS), a.get("wn", WN), a.get("bias"),
+                    a["layer"], a["dim"], a["B"], a["n"], a["d"], a["dt"], a["flags"],
+                    a.get("y", Y), a.get("z"))
+
+    assert call(n=48) == hcw.HCW_ERR_INVALID_ARG          # n not a power of two
+    assert call(n=1) == hcw.HCW_ERR_INVALID_ARG
+    assert call(B=-1) == hcw.HCW_ERR_INVALID_ARG
+    assert call(layer=-2) == hcw.HCW_ERR_INVALID_ARG
+    assert call(dim=4) == hcw.HCW_ERR_INVALID_ARG          # log2 16 = 4 dimensions: 0..3
+    assert call(flags=8) == hcw.HCW_ERR_INVALID_ARG
+    assert call(dt=7) == hcw.HCW_ERR_INVALID_ARG
+    assert call(d=96) == hcw.HCW_ERR_UNSUPPORTED          # bf16 needs d % 64 == 0
+    assert call(x=0) == hcw.HCW_ERR_INVALID_ARG
+    assert call(y=0) == hcw.HCW_ERR_INVALID_ARG
+    assert call(x=X + 8) == hcw.HCW_ERR_ALIGNMENT
+    assert call(bias=WS + 4) == hcw.HCW_ERR_ALIGNMENT
+    assert call(y=X + 1024) == hcw.HCW_ERR_ALIASING       # y overlaps x
+    assert call(z=Y) == hcw.HCW_ERR_ALIASING              # z overlaps y
+    assert call(B=0) == hcw.HCW_OK                         # empty batch: nothing to do
+
+
+def test_backward_validation_codes(hcw):
+    P = ctypes.c_void_p
+    L = hcw.lib()
+    X, DY, WS, WN, DX, GS, GN = (0x100000 * k for k in range(1, 8))
+    args = dict(x=X, z=None, dy=DY, ws=WS, wn=WN, layer=0, dim=-1, B=4, n=16, d=32,
+                dt=hcw.HCW_F32, flags=0, dx=DX, gs=GS, gn=GN, gb=None, w=None, wsb=0)
+
+    def call(**kw):
+        a = dict(args, **kw)
+        return L.hcw_layer_bwd(P(a["x"]), P(a["z"]), P(a["dy"]), P(a["ws"]), P(a["wn"]),
+                               a["layer"], a["dim"], a["B"], a["n"], a["d"], a["dt"], a["flags"],
+                               P(a["dx"]), P(a["gs"]), P(a["gn"]), P(a["gb"]), P(a["w"]),
+                               a["wsb"], None)
+
+    need = hcw.hcw_workspace_bytes(4, 16, 32, hcw.HCW_F32, 0)
+    assert need > 0
+    assert call() == hcw.HCW_ERR_WORKSPACE
+    assert call(w=0x900000, wsb=need - 1) == hcw.HCW_ERR_WORKSPACE
+    assert call(flags=hcw.HCW_ACT_RELU, w=0x900000, wsb=1 << 30) == hcw.HCW_ERR_INVALID_ARG
+    assert call(dx=X, w=0x9000000, wsb=need) == hcw.HCW_ERR_ALIASING
+    assert call(gn=GS, w=0x9000000, wsb=need) == hcw.HCW_ERR_ALIASING
+    assert call(dx=DX + 4, w=0x9000000, wsb=need) == hcw.HCW_ERR_ALIGNMENT
+    assert call(d=0) == hcw.HCW_ERR_INVALID_ARG
+
+
+def test_workspace_sizes_f32(hcw):
+    a = hcw.hcw_workspace_bytes(64, 256, 512, hcw.HCW_F32, 0)
+    b = hcw.hcw_workspace_bytes(64, 256, 512, hcw.HCW_F32, hcw.HCW_ACT_RELU)
+    assert b - a >= 64 * 256 * 512 * 4            # the masked gradient dz
+    s = hcw.hcw_stack_workspace_bytes(64, 256, 512, hcw.HCW_F32, 0)
+    assert s >= a + 2 * 64 * 256 * 512 * 4        # two gradient buffers between layers
+    assert hcw.hcw_workspace_bytes(4, 48, 64, hcw.HCW_F32, 0) == 0   # invalid n

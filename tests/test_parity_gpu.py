@@ -1,0 +1,325 @@
+"""Parity of the CUDA path (through the C ABI) with the fp64 oracle.
+
+Tolerances (relative error = max|gpu - ref| / max|ref| per tensor):
+  fp32 path 1e-5, bf16 path 2e-2 against the oracle's bf16-storage mode
+  (the oracle rounds every stored activation to bf16, as the device does);
+  partner tables bit-exact.
+Inputs are the seeded generators of paper_2609_18145_gb300.synth; the bf16
+cases hand the oracle the exact bf16 values the device sees.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as O
+from paper_2609_18145_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+TOL_F32 = 1e-5
+TOL_BF16 = 2e-2
+CAUSAL, RESIDUAL, RELU = 1, 2, 4
+
+
+@pytest.fixture(scope="module")
+def H():
+    from paper_2609_18145_gb300 import hcw
+    hcw.lib()
+    return hcw
+
+
+def rel(got, ref):
+    got = np.asarray(got, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    assert got.shape == ref.shape
+    assert np.isfinite(got).all()
+    return float(np.abs(got - ref).max() / max(np.abs(ref).max(), 1e-30))
+
+
+def dev(a, dtype):
+    """numpy float32 -> (device tensor of dtype, float64 numpy of its exact values)."""
+    if dtype == torch.bfloat16:
+        t, a64 = synth.to_bf16_exact(a)
+        return t.cuda(), a64
+    t = torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32))
+    return t.cuda(), t.double().numpy()
+
+
+def host(t):
+    return t.float().cpu().double().numpy()
+
+
+# ---------------------------------------------------------------- index code
+
+@pytest.mark.parametrize("n", [2, 8, 64, 256, 65536])
+@pytest.mark.parametrize("flags", [0, CAUSAL])
+def test_device_partner_table_bit_exact(H, n, flags):
+    b = n.bit_length() - 1
+    for layer in range(2 * b + 1):
+        got = H.hcw_partner_table_device(layer, n, flags).cpu().numpy()
+        assert np.array_equal(got, O.partner_table(layer, -1, n, flags))
+    got = H.hcw_partner_table_device(5, n, flags, dim_override=b - 1).cpu().numpy()
+    assert np.array_equal(got, O.partner_table(5, b - 1, n, flags))
+
+
+# ---------------------------------------------------------------- single layer
+
+LAYER_CASES_F32 = [
+    # B, n, d, layer, dim_override
+    (4, 16, 32, 0, -1), (4, 16, 32, 3, -1), (3, 8, 20, 2, -1), (2, 64, 96, 5, -1),
+    (1, 2, 33, 0, -1), (4, 16, 32, 9, 1),
+]
+LAYER_CASES_BF16 = [
+    (8, 16, 64, 0, -1),       # k = 1, one ragged row block
+    (3, 16, 64, 2, -1),       # 24 rows per bit value (ragged)
+    (2, 2, 64, 0, -1),        # n = 2, a single position per bit value and sample
+    (16, 64, 128, 5, -1),     # k = 32
+    (4, 256, 512, 7, -1),     # k = 128 (the 128-row box along lo)
+    (4, 256, 512, 3, -1),     # k = 8
+    (2, 64, 192, 4, -1),      # d = 192: 64-wide column tiles, ragged 128-row o tiles in dW
+    (1, 4096, 64, 11, -1),    # k = 2048 > 128
+    (5, 32, 256, 1, 0),       # fixed-dimension control, odd B
+]
+FLAG_SETS = [0, CAUSAL, CAUSAL | RESIDUAL, RESIDUAL | RELU, CAUSAL | RESIDUAL | RELU]
+
+
+@pytest.mark.parametrize("flags", FLAG_SETS)
+@pytest.mark.parametrize("case", LAYER_CASES_F32 + LAYER_CASES_BF16)
+def test_layer_forward(H, case, flags):
+    B, n, d, layer, dim = case
+    dtype = torch.float32 if case in LAYER_CASES_F32 else torch.bfloat16
+    pr = synth.problem(B, n, d, L=1, seed=B * 1000 + n + d + layer)
+    x, x64 = dev(pr.x, dtype)
+    Ws, Ws64 = dev(pr.W_self[0], dtype)
+    Wn, Wn64 = dev(pr.W_nbr[0], dtype)
+    bias = torch.from_numpy(pr.bias[0]).cuda()
+    y, z = H.hcw_layer_fwd(x, Ws, Wn, bias, layer, dim, flags, want_z=True)
+    torch.cuda.synchronize()
+    rb = dtype == torch.bfloat16
+    yr, zr = O.layer_fwd(x64, Ws64, Wn64, pr.bias[0].astype(np.float64), layer, dim, flags,
+                         round_bf16=rb, want_z=True)
+    tol = TOL_BF16 if rb else TOL_F32
+    assert rel(host(y), yr) <= tol
+    assert rel(host(z), zr) <= tol
+
+
+@pytest.mark.parametrize("flags", FLAG_SETS)
+@pytest.mark.parametrize("case", LAYER_CASES_F32 + LAYER_CASES_BF16)
+def test_layer_backward(H, case, flags):
+    B, n, d, layer, dim = case
+    dtype = torch.float32 if case in LAYER_CASES_F32 else torch.bfloat16
+    pr = synth.problem(B, n, d, L=1, seed=B * 1000 + n + d + layer + 7)
+    x, x64 = dev(pr.x, dtype)
+    z, z64 = dev(pr.z[0], dtype)            # a given pre-activation: same ReLU mask on both sides
+    dy, dy64 = dev(pr.dy, dtype)
+    Ws, Ws64 = dev(pr.W_self[0], dtype)
+    Wn, Wn64 = dev(pr.W_nbr[0], dtype)
+    dx, gWs, gWn, gb = H.hcw_layer_bwd(x, z, dy, Ws, Wn, layer, dim, flags)
+    torch.cuda.synchronize()
+    rb = dtype == torch.bfloat16
+    rdx, rWs, rWn, rb_ = O.layer_bwd(x64, z64, dy64, Ws64, Wn64, layer, dim, flags,
+                                     round_bf16=rb)
+    tol = TOL_BF16 if rb else TOL_F32
+    assert rel(host(dx), rdx) <= tol
+    assert rel(host(gWs), rWs) <= (1e-5 if not rb else 1e-4)
+    assert rel(host(gWn), rWn) <= (1e-5 if not rb else 1e-4)
+    assert rel(host(gb), rb_) <= (1e-5 if not rb else 1e-4)
+
+
+def test_backward_is_deterministic(H):
+    pr = synth.problem(8, 256, 512, L=1, seed=3)
+    x, _ = dev(pr.x, torch.bfloat16)
+    dy, _ = dev(pr.dy, torch.bfloat16)
+    Ws, _ = dev(pr.W_self[0], torch.bfloat16)
+    Wn, _ = dev(pr.W_nbr[0], torch.bfloat16)
+    a = H.hcw_layer_bwd(x, None, dy, Ws, Wn, 4, -1, CAUSAL | RESIDUAL)
+    b = H.hcw_layer_bwd(x, None, dy, Ws, Wn, 4, -1, CAUSAL | RESIDUAL)
+    for u, v in zip(a, b):
+        assert torch.equal(u, v)
+
+
+def test_empty_batch(H):
+    x = torch.empty(0, 16, 64, dtype=torch.bfloat16, device="cuda")
+    W = torch.zeros(64, 64, dtype=torch.bfloat16, device="cuda")
+    y = H.hcw_layer_fwd(x, W, W, None, 0)
+    assert y.shape == x.shape
+    dx, gWs, gWn, gb = H.hcw_layer_bwd(x, None, x, W, W, 0)
+    torch.cuda.synchronize()
+    assert float(gWs.abs().sum()) == 0.0 and float(gWn.abs().sum()) == 0.0
+    assert float(gb.abs().sum()) == 0.0
+
+
+# ---------------------------------------------------------------- stacks
+
+def run_stack(H, pr, dtype, L, flags, layer0=0, dim=-1):
+    """Forward: device stack vs oracle stack on the same inputs.  Backward: the
+    device stack backward is fed the oracle's saved layer inputs and
+    pre-activations (bf16-exact in bf16 mode), so that both sides take the
+    same ReLU decisions; near-zero pre-activations would otherwise be decided
+    differently by two forwards that differ by rounding, and both answers are
+    valid.  Returns (device, oracle) tuples (y, acts, dx, dW_self, dW_nbr, dbias)."""
+    x, x64 = dev(pr.x, dtype)
+    Ws, Ws64 = dev(pr.W_self, dtype)
+    Wn, Wn64 = dev(pr.W_nbr, dtype)
+    bias = torch.from_numpy(pr.bias).cuda()
+    dy, dy64 = dev(pr.dy, dtype)
+    y, acts, zs = H.hcw_stack_fwd(x, Ws, Wn, bias, layer0, dim, flags, want_z=True)
+    rb = dtype == torch.bfloat16
+    ry, racts, rzs = O.stack_fwd(x64, Ws64, Wn64, pr.bias.astype(np.float64), layer0, L, dim,
+                                 flags, round_bf16=rb)
+    o_acts = torch.from_numpy(racts[1:]).to(dtype).cuda() if L > 1 else None
+    o_zs = torch.from_numpy(rzs).to(dtype).cuda()
+    dx, gWs, gWn, gb = H.hcw_stack_bwd(x, o_acts, o_zs, dy, Ws, Wn, layer0, dim, flags)
+    torch.cuda.synchronize()
+    rdx, rWs, rWn, rgb = O.stack_bwd(racts, rzs, dy64, Ws64, Wn64, layer0, L, dim, flags,
+                                     round_bf16=rb)
+    dev_acts = host(acts) if L > 1 else np.zeros((0,) + pr.x.shape)
+    return ((host(y), dev_acts, host(dx), host(gWs), host(gWn), host(gb)),
+            (ry, racts[1:], rdx, rWs, rWn, rgb))
+
+
+WHAT = ("y", "acts", "dx", "dW_self", "dW_nbr", "dbias")
+
+
+STACK_CASES = [
+    # name, dtype, B, n, d, L, flags, w_std
+    ("tiny_n16_d32_f32", torch.float32, 4, 16, 32, 4, 0, None),
+    ("tiny_n16_d32_f32_causal_res_relu", torch.float32, 4, 16, 32, 4,
+     CAUSAL | RESIDUAL | RELU, None),
+    ("tiny_n16_d64_bf16", torch.bfloat16, 4, 16, 64, 4, 0, None),
+    ("n16_d64_bf16_8layers_causal_res", torch.bfloat16, 6, 16, 64, 8, CAUSAL | RESIDUAL,
+     (1 / 128) ** 0.5),
+    ("n64_d128_bf16_causal_res_relu", torch.bfloat16, 8, 64, 128, 6, CAUSAL | RESIDUAL | RELU,
+     (1 / 256) ** 0.5),
+    ("n256_d512_bf16_causal_res_relu", torch.bfloat16, 2, 256, 512, 16,
+     CAUSAL | RESIDUAL | RELU, (1 / 1024) ** 0.5),
+]
+
+
+@pytest.mark.parametrize("case", STACK_CASES, ids=lambda c: c[0])
+def test_stack_forward_backward(H, case):
+    name, dtype, B, n, d, L, flags, w_std = case
+    pr = synth.problem(B, n, d, L=L, seed=11, w_std=w_std)
+    got, ref = run_stack(H, pr, dtype, L, flags)
+    tol = TOL_BF16 if dtype == torch.bfloat16 else TOL_F32
+    for g, r, what in zip(got, ref, WHAT):
+        if g.size:
+            assert rel(g, r) <= tol, (name, what, rel(g, r))
+
+
+def test_stack_fixed_dimension_control(H):
+    pr = synth.problem(16, 64, 128, L=6, seed=5, w_std=(1 / 256) ** 0.5)
+    got, ref = run_stack(H, pr, torch.bfloat16, 6, 0, dim=0)
+    for g, r, what in zip(got, ref, WHAT):
+        assert rel(g, r) <= TOL_BF16, what
+
+
+def test_reach_workload_full_size(H):
+    # n = 64, d = 128, six rotated layers, batch 256, non-causal, embedded uniform-16 ids
+    w = synth.WORKLOADS["reach_n64_d128"]
+    pr = synth.problem(w["B"], w["n"], w["d"], L=w["L"], seed=0, w_std=(1 / 256) ** 0.5,
+                       x_ids="uniform16")
+    got, ref = run_stack(H, pr, torch.bfloat16, w["L"], 0)
+    for g, r, what in zip(got, ref, WHAT):
+        assert rel(g, r) <= TOL_BF16, what
+
+
+def test_charlm_w256_full_launch_sampled(H):
+    """The timed workload (B = 64, n = 256, d = 512, 16 causal layers, residual,
+    ReLU, bias) in its full launch configuration; the oracle recomputes two
+    sampled sequences.  Forward: the device's rows of those sequences against
+    the oracle.  Backward: the upstream gradient is zero outside them and the
+    device backward sees the oracle's saved activations for them (same ReLU
+    decisions), so its weight gradients over the whole batch must equal the
+    oracle's over the two sequences, and dx must vanish elsewhere."""
+    w = synth.WORKLOADS["charlm_w256_d512"]
+    B, n, d, L = w["B"], w["n"], w["d"], w["L"]
+    flags = CAUSAL | RESIDUAL | RELU
+    pr = synth.problem(B, n, d, L=L, seed=0, w_std=(1 / (2 * d)) ** 0.5, x_ids="zipf256")
+    picks = [5, 42]
+    mask = np.zeros((B, 1, 1), dtype=np.float32)
+    mask[picks] = 1.0
+    pr.dy = pr.dy * mask
+    x, x64 = dev(pr.x, torch.bfloat16)
+    Ws, Ws64 = dev(pr.W_self, torch.bfloat16)
+    Wn, Wn64 = dev(pr.W_nbr, torch.bfloat16)
+    bias = torch.from_numpy(pr.bias).cuda()
+    dy, dy64 = dev(pr.dy, torch.bfloat16)
+    y, acts, zs = H.hcw_stack_fwd(x, Ws, Wn, bias, 0, -1, flags, want_z=True)
+    ry, racts, rzs = O.stack_fwd(x64[picks], Ws64, Wn64, pr.bias.astype(np.float64), 0, L, -1,
+                                 flags, round_bf16=True)
+    assert rel(host(y)[picks], ry) <= TOL_BF16
+    assert rel(host(acts)[:, picks], racts[1:]) <= TOL_BF16
+    acts[:, picks] = torch.from_numpy(racts[1:]).to(torch.bfloat16).cuda()
+    zs[:, picks] = torch.from_numpy(rzs).to(torch.bfloat16).cuda()
+    dx, gWs, gWn, gb = H.hcw_stack_bwd(x, acts, zs, dy, Ws, Wn, 0, -1, flags)
+    torch.cuda.synchronize()
+    rdx, rWs, rWn, rgb = O.stack_bwd(racts, rzs, dy64[picks], Ws64, Wn64, 0, L, -1, flags,
+                                     round_bf16=True)
+    hdx = host(dx)
+    assert rel(hdx[picks], rdx) <= TOL_BF16
+    others = np.setdiff1d(np.arange(B), picks)
+    assert np.abs(hdx[others]).max() == 0.0
+    assert rel(host(gWs), rWs) <= TOL_BF16
+    assert rel(host(gWn), rWn) <= TOL_BF16
+    assert rel(host(gb), rgb) <= TOL_BF16
+
+
+def test_stack_backward_is_the_chain_of_layer_backwards(H):
+    """hcw_stack_bwd on its own saved activations equals hcw_layer_bwd applied
+    layer by layer from the top (bit-exact): the stack plumbing adds nothing."""
+    flags = CAUSAL | RESIDUAL | RELU
+    B, n, d, L = 4, 256, 512, 5
+    pr = synth.problem(B, n, d, L=L, seed=4, w_std=(1 / (2 * d)) ** 0.5)
+    x, _ = dev(pr.x, torch.bfloat16)
+    Ws, _ = dev(pr.W_self, torch.bfloat16)
+    Wn, _ = dev(pr.W_nbr, torch.bfloat16)
+    dy, _ = dev(pr.dy, torch.bfloat16)
+    bias = torch.from_numpy(pr.bias).cuda()
+    y, acts, zs = H.hcw_stack_fwd(x, Ws, Wn, bias, 3, -1, flags, want_z=True)
+    dx, gWs, gWn, gb = H.hcw_stack_bwd(x, acts, zs, dy, Ws, Wn, 3, -1, flags)
+    g = dy
+    for l in range(L - 1, -1, -1):
+        inp = x if l == 0 else acts[l - 1]
+        g, a, b, c = H.hcw_layer_bwd(inp, zs[l], g, Ws[l], Wn[l], 3 + l, -1, flags)
+        assert torch.equal(a, gWs[l]) and torch.equal(b, gWn[l]) and torch.equal(c, gb[l])
+    assert torch.equal(g, dx)
+
+
+def test_split_backward_matches_fused(H):
+    flags = CAUSAL | RESIDUAL
+    pr = synth.problem(8, 64, 256, L=1, seed=9)
+    x, _ = dev(pr.x, torch.bfloat16)
+    dy, _ = dev(pr.dy, torch.bfloat16)
+    Ws, _ = dev(pr.W_self[0], torch.bfloat16)
+    Wn, _ = dev(pr.W_nbr[0], torch.bfloat16)
+    dx, gWs, gWn, gb = H.hcw_layer_bwd(x, None, dy, Ws, Wn, 2, -1, flags)
+    dx2 = H.hcw_layer_bwd_data(dy, dy, Ws, Wn, 2, -1, flags)
+    a, b, c = H.hcw_layer_bwd_weight(x, dy, 2, -1, flags)
+    assert torch.equal(dx, dx2) and torch.equal(gWs, a) and torch.equal(gWn, b)
+    assert torch.equal(gb, c)
+
+
+def test_launch_counter_counts_kernels(H):
+    pr = synth.problem(2, 16, 64, L=1, seed=1)
+    x, _ = dev(pr.x, torch.bfloat16)
+    W, _ = dev(pr.W_self[0], torch.bfloat16)
+    c0 = H.hcw_launch_count()
+    H.hcw_layer_fwd(x, W, W, None, 0)
+    assert H.hcw_launch_count() == c0 + 1
+
+
+# ---------------------------------------------------------------- bounded waits
+
+def test_bounded_wait_reports_timeout_and_context_survives(H):
+    assert H.hcw_sync_status() == H.HCW_OK
+    H.hcw_selftest_wait(200_000_000)           # nothing arrives: gives up after 0.2 s
+    assert H.hcw_sync_status() == H.HCW_ERR_TIMEOUT
+    assert H.hcw_sync_status() == H.HCW_OK     # the word was cleared
+    pr = synth.problem(4, 16, 64, L=1, seed=1)
+    x, x64 = dev(pr.x, torch.bfloat16)
+    W, W64 = dev(pr.W_self[0], torch.bfloat16)
+    y = H.hcw_layer_fwd(x, W, W, None, 1, -1, CAUSAL)
+    torch.cuda.synchronize()
+    yr = O.layer_fwd(x64, W64, W64, None, 1, -1, CAUSAL, round_bf16=True)
+    assert rel(host(y), yr) <= TOL_BF16
