@@ -142,9 +142,11 @@ WPlan plan_dw(long long tokens, int d, unsigned flags) {
     const int tiles = w.n_ot * w.n_nt;
     const long long total_kb = (long long)tiles * (w.nkb_self + w.nkb_nbr);
     const int sms = sm_count();
-    // about one unit per SM, at least 4 token blocks (256 tokens) per unit
+    // the fewest token blocks per unit (at least 4, i.e. 256 tokens) whose
+    // units still fit in one wave of persistent CTAs: makespan = kpu blocks
     long long kpu = (total_kb + sms - 1) / sms;
     if (kpu < 4) kpu = 4;
+    while (tiles * ((w.nkb_self + kpu - 1) / kpu + (w.nkb_nbr + kpu - 1) / kpu) > sms) ++kpu;
     w.kb_per_unit = (int)kpu;
     w.splits_self = (int)((w.nkb_self + kpu - 1) / kpu);
     w.splits_nbr = (int)((w.nkb_nbr + kpu - 1) / kpu);
@@ -208,6 +210,7 @@ int fwd_bf16(const Shape& sh, const void* x, const void* Ws, const void* Wn, con
     memset(&p, 0, sizeof(p));
     p.d = d;
     p.k = k;
+    p.s = sh.s;
     p.Mh = (int)(sh.tokens / 2);
     p.nK = d / 64;
     p.n_rb = (p.Mh + 127) / 128;
@@ -237,7 +240,8 @@ int fwd_bf16(const Shape& sh, const void* x, const void* Ws, const void* Wn, con
 
 // dx: a row gathers dz from its partner exactly when the partner received from it
 int dx_bf16(const Shape& sh, const void* dz, const void* dy, const void* Ws, const void* Wn,
-            unsigned flags, void* dx, cudaStream_t st) {
+            unsigned flags, void* dx, cudaStream_t st, const void* zprev = nullptr,
+            void* dz_out = nullptr) {
     const int d = sh.d, BN = pick_bn(d), k = 1 << sh.s;
     CUtensorMap tA, tB0, tB1;
     if (!map_rows(&tA, dz, sh.tokens, d, k, 128) || !map_weight(&tB0, Ws, d, 64) ||
@@ -247,6 +251,7 @@ int dx_bf16(const Shape& sh, const void* dz, const void* dy, const void* Ws, con
     memset(&p, 0, sizeof(p));
     p.d = d;
     p.k = k;
+    p.s = sh.s;
     p.Mh = (int)(sh.tokens / 2);
     p.nK = d / 64;
     p.n_rb = (p.Mh + 127) / 128;
@@ -265,6 +270,8 @@ int dx_bf16(const Shape& sh, const void* dz, const void* dy, const void* Ws, con
     p.flags = flags & HCW_RESIDUAL;
     p.resid = static_cast<const __nv_bfloat16*>(dy);
     p.out = static_cast<__nv_bfloat16*>(dx);
+    p.zprev = static_cast<const __nv_bfloat16*>(zprev);
+    p.dz_out = static_cast<__nv_bfloat16*>(dz_out);
     p.timeout_ns = g_timeout_ns;
     const int sms = sm_count();
     const int grid = p.n_units < sms ? p.n_units : sms;
@@ -285,6 +292,7 @@ int dw_bf16(const Shape& sh, const void* x, const void* dz, unsigned flags, floa
     memset(&p, 0, sizeof(p));
     p.d = d;
     p.k = k;
+    p.s = sh.s;
     p.Mh = (int)(sh.tokens / 2);
     p.n_nt = w.n_nt;
     p.n_ot = w.n_ot;
@@ -619,7 +627,9 @@ int hcw_stack_fwd(const void* x, const void* W_self, const void* W_nbr, const fl
 size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags) {
     Shape sh;
     if (check_shape(0, -1, B, n, d, dtype, flags, &sh)) return 0;
-    return ws_layout(sh.tokens, d, dtype, flags).total + 2 * align256(sh.act_bytes);
+    // two output-gradient buffers, two pre-activation-gradient buffers, and
+    // the weight-gradient workspace of one layer
+    return ws_layout(sh.tokens, d, dtype, flags).w_bytes + 4 * align256(sh.act_bytes);
 }
 
 int hcw_stack_bwd(const void* x, const void* acts, const void* zs, const void* dy,
@@ -657,21 +667,67 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* zs, const void* d
         return HCW_ERR_ALIASING;
     cudaStream_t st = (cudaStream_t)stream;
     uint8_t* wsb = static_cast<uint8_t*>(workspace);
-    uint8_t* g[2] = {wsb, wsb + align256(ab)};
-    void* lws = wsb + 2 * align256(ab);
-    const void* cur = dy;
+    const size_t ab256 = align256(ab);
+    uint8_t* g[2] = {wsb, wsb + ab256};                    // output gradients
+    uint8_t* gz[2] = {wsb + 2 * ab256, wsb + 3 * ab256};   // pre-activation gradients
+    uint8_t* wws = wsb + 4 * ab256;                        // weight-gradient workspace
+    const bool relu = (flags & HCW_ACT_RELU) != 0;
+    const bool resid = (flags & HCW_RESIDUAL) != 0;
+    auto layer_ptr = [&](const void* base, int l) {
+        return static_cast<const uint8_t*>(base) + (size_t)l * ab;
+    };
+    // gradient at the output (cur_g) and at the pre-activation (cur_dz) of layer l
+    const void* cur_g = dy;
+    const void* cur_dz = dy;
+    if (relu) {
+        rc = launched(dtype == HCW_BF16
+                          ? launch_relu_grad_bf16(static_cast<const __nv_bfloat16*>(dy),
+                                                  reinterpret_cast<const __nv_bfloat16*>(
+                                                      layer_ptr(zs, L - 1)),
+                                                  reinterpret_cast<__nv_bfloat16*>(gz[(L - 1) & 1]),
+                                                  (size_t)sh.tokens * d, st)
+                          : launch_relu_grad_f32(static_cast<const float*>(dy),
+                                                 reinterpret_cast<const float*>(layer_ptr(zs, L - 1)),
+                                                 reinterpret_cast<float*>(gz[(L - 1) & 1]),
+                                                 (size_t)sh.tokens * d, st),
+                      1);
+        if (rc) return rc;
+        cur_dz = gz[(L - 1) & 1];
+    }
     for (int l = L - 1; l >= 0; --l) {
         Shape shl = sh;
         shl.s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
-        const void* in = l == 0 ? x : static_cast<const uint8_t*>(acts) + (size_t)(l - 1) * ab;
-        const void* z = zs ? static_cast<const uint8_t*>(zs) + (size_t)l * ab : nullptr;
-        void* out = l == 0 ? dx : g[l & 1];
-        rc = layer_bwd_impl(shl, dtype, in, z, cur, static_cast<const uint8_t*>(W_self) + l * wb,
-                            static_cast<const uint8_t*>(W_nbr) + l * wb, flags, out,
-                            dW_self + (size_t)l * d * d, dW_nbr + (size_t)l * d * d,
-                            dbias ? dbias + (size_t)l * d : nullptr, lws, st);
+        const void* in = l == 0 ? x : layer_ptr(acts, l - 1);
+        const void* Wsl = static_cast<const uint8_t*>(W_self) + l * wb;
+        const void* Wnl = static_cast<const uint8_t*>(W_nbr) + l * wb;
+        void* out_g = l == 0 ? dx : ((resid || !relu) ? (void*)g[l & 1] : nullptr);
+        void* next_dz = nullptr;
+        if (l > 0 && relu) {
+            next_dz = gz[(l - 1) & 1];
+            if (dtype == HCW_BF16) {
+                // the input gradient kernel also applies the ReLU gradient of layer l-1
+                rc = dx_bf16(shl, cur_dz, cur_g, Wsl, Wnl, flags, out_g, st, layer_ptr(zs, l - 1),
+                             next_dz);
+            } else {
+                rc = layer_dx_impl(shl, dtype, cur_dz, cur_g, Wsl, Wnl, flags, g[l & 1], st);
+                if (!rc)
+                    rc = launched(launch_relu_grad_f32(static_cast<const float*>((const void*)g[l & 1]),
+                                                       reinterpret_cast<const float*>(layer_ptr(zs, l - 1)),
+                                                       reinterpret_cast<float*>(next_dz),
+                                                       (size_t)sh.tokens * d, st),
+                                  1);
+                out_g = g[l & 1];
+            }
+        } else {
+            rc = layer_dx_impl(shl, dtype, cur_dz, cur_g, Wsl, Wnl, flags, out_g, st);
+        }
         if (rc) return rc;
-        cur = out;
+        rc = layer_dw_impl(shl, dtype, in, cur_dz, flags, dW_self + (size_t)l * d * d,
+                           dW_nbr + (size_t)l * d * d, dbias ? dbias + (size_t)l * d : nullptr,
+                           wws, st);
+        if (rc) return rc;
+        cur_g = out_g;
+        cur_dz = relu ? next_dz : out_g;
     }
     return HCW_OK;
 }

@@ -20,6 +20,7 @@ enum TcMode { MODE_FWD = 0, MODE_DX = 1, MODE_DW = 2 };
 struct TcParams {
     int d;          // feature width
     int k;          // 2^s, the link distance of this layer
+    int s;          // cube dimension of this layer
     int Mh;         // positions per value of bit s: B * n / 2
     int nK;         // d / 64: K-steps per part (FWD, DX)
     // FWD / DX units
@@ -43,8 +44,10 @@ struct TcParams {
     unsigned flags;
     const float* bias;            // FWD
     const __nv_bfloat16* resid;   // FWD: x; DX: dy
-    __nv_bfloat16* out;           // FWD: y; DX: dx
+    __nv_bfloat16* out;           // FWD: y; DX: dx (may be null when dz_out is set)
     __nv_bfloat16* zout;          // FWD: z (may be null)
+    const __nv_bfloat16* zprev;   // DX: pre-activation of the layer below (fused ReLU grad)
+    __nv_bfloat16* dz_out;        // DX: its gradient dz = dx * (zprev > 0), or null
     float* dw_self;               // DW destination when splits_self == 1
     float* dw_nbr;                // DW destination when splits_nbr == 1
     float* dw_partial;            // DW partials [2][splits_max][d][d]

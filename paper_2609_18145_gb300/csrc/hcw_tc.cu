@@ -45,15 +45,17 @@ namespace hcw {
 
 namespace {
 
-constexpr int kThreads = 192;
+constexpr int kEpiWarps = 8;                       // two per TMEM lane quarter
+constexpr int kThreads = 64 + 32 * kEpiWarps;      // producer, MMA, epilogue warps
 constexpr int kBlockM = 128;
 constexpr int kBlockK = 64;                        // bf16 elements per 128-byte row
 constexpr int kABytes = kBlockM * kBlockK * 2;     // 16 KB
-constexpr int kSmemBudget = 200 * 1024;
+constexpr int kRingBytes = 192 * 1024;             // TMA stage ring
+constexpr int kEpiBufBytes = 4096;                 // per epilogue warp: 32 rows x 128 B
 
 __host__ __device__ constexpr int stage_bytes(int BN) { return kABytes + BN * kBlockK * 2; }
 __host__ __device__ constexpr int num_stages(int BN) {
-    return (kSmemBudget / stage_bytes(BN)) > 8 ? 8 : (kSmemBudget / stage_bytes(BN));
+    return (kRingBytes / stage_bytes(BN)) > 8 ? 8 : (kRingBytes / stage_bytes(BN));
 }
 
 struct __align__(8) Barriers {
@@ -69,7 +71,7 @@ struct __align__(8) Barriers {
 template <int BN>
 __host__ __device__ constexpr size_t smem_total() {
     return 1024 /* alignment slack */ + (size_t)num_stages(BN) * stage_bytes(BN) +
-           sizeof(Barriers);
+           (size_t)kEpiWarps * kEpiBufBytes + sizeof(Barriers);
 }
 
 // FWD/DX unit -> (row bit beta, row block t, column tile j, number of K steps)
@@ -123,34 +125,68 @@ __device__ __forceinline__ WUnit decode_w_unit(const TcParams& p, int u) {
     return w;
 }
 
-__device__ __forceinline__ void store_bf16x32(__nv_bfloat16* dst, const float (&v)[32]) {
-    uint4* d4 = reinterpret_cast<uint4*>(dst);
+// ---- epilogue staging ------------------------------------------------------
+// Each epilogue warp owns 32 accumulator rows (one per lane, as tcgen05.ld
+// delivers them) and moves them through a private 4 KB shared buffer so that
+// global loads and stores are whole-line and coalesced.  Rows are 16-byte
+// pieces XOR-swizzled by row so that both the row-wise accesses (a lane per
+// row) and the line-wise accesses (lanes along a row) are conflict-free.
+//   bf16 chunk: 32 rows x 32 values = 32 x 64 B, piece m of row r at word
+//               16 r + 4 (m ^ ((r >> 1) & 3))
+//   fp32 chunk: 32 rows x 32 values = 32 x 128 B, piece m of row r at word
+//               32 r + 4 (m ^ (r & 7))
+__device__ __forceinline__ uint32_t* bf16_piece(uint32_t* buf, int r, int m) {
+    return buf + 16 * r + 4 * (m ^ ((r >> 1) & 3));
+}
+__device__ __forceinline__ uint32_t* f32_piece(uint32_t* buf, int r, int m) {
+    return buf + 32 * r + 4 * (m ^ (r & 7));
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<uint32_t*>(&h);
+}
+
+__device__ __forceinline__ float2 unpack_bf16x2(uint32_t w) {
+    __nv_bfloat162 h = *reinterpret_cast<__nv_bfloat162*>(&w);
+    return __bfloat1622float2(h);
+}
+
+// Lane `lane` writes its row (32 bf16 given as 16 packed words) into the buffer.
+__device__ __forceinline__ void stage_row_bf16(uint32_t* buf, int lane, const uint32_t (&w)[16]) {
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        uint32_t w[4];
+    for (int m = 0; m < 4; ++m)
+        *reinterpret_cast<uint4*>(bf16_piece(buf, lane, m)) =
+            make_uint4(w[4 * m], w[4 * m + 1], w[4 * m + 2], w[4 * m + 3]);
+}
+
+__device__ __forceinline__ void read_row_bf16(const uint32_t* buf, int lane, uint32_t (&w)[16]) {
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            __nv_bfloat162 h = __floats2bfloat162_rn(v[q * 8 + 2 * e], v[q * 8 + 2 * e + 1]);
-            w[e] = *reinterpret_cast<uint32_t*>(&h);
-        }
-        d4[q] = make_uint4(w[0], w[1], w[2], w[3]);
+    for (int m = 0; m < 4; ++m) {
+        uint4 u = *reinterpret_cast<const uint4*>(bf16_piece(const_cast<uint32_t*>(buf), lane, m));
+        w[4 * m] = u.x;
+        w[4 * m + 1] = u.y;
+        w[4 * m + 2] = u.z;
+        w[4 * m + 3] = u.w;
     }
 }
 
-__device__ __forceinline__ void add_bf16x32(const __nv_bfloat16* src, float (&v)[32]) {
-    const uint4* s4 = reinterpret_cast<const uint4*>(src);
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        uint4 u = __ldg(s4 + q);
-        uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            __nv_bfloat162 h = *reinterpret_cast<__nv_bfloat162*>(&w[e]);
-            float2 f = __bfloat1622float2(h);
-            v[q * 8 + 2 * e] += f.x;
-            v[q * 8 + 2 * e + 1] += f.y;
-        }
-    }
+// Line-wise mapping of a bf16 chunk: iteration it (0..3), lane -> row
+// 8 it + lane / 4, piece lane % 4 (16 bytes of the row's 64).
+__device__ __forceinline__ int line_row_bf16(int it, int lane) { return 8 * it + (lane >> 2); }
+
+// Wait for this thread's tcgen05.ld and tie the destination registers to the
+// wait so the compiler cannot read them earlier.
+__device__ __forceinline__ void tmem_ld_wait_regs(uint32_t (&r)[32]) {
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
+                   "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]),
+                   "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]),
+                   "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
+                   "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]),
+                   "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+                 :
+                 : "memory");
 }
 
 // Wait that only gives up on time (used to drain in-flight work after an
@@ -187,7 +223,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-    Barriers* bars = reinterpret_cast<Barriers*>(smem + (size_t)STAGES * SB);
+    uint8_t* epi_smem = smem + (size_t)STAGES * SB;
+    Barriers* bars =
+        reinterpret_cast<Barriers*>(epi_smem + (size_t)kEpiWarps * kEpiBufBytes);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -202,7 +240,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&bars->tfull[a], 1);
-            mbar_init(&bars->tempty[a], 4);
+            mbar_init(&bars->tempty[a], kEpiWarps);
         }
         mbar_init(&bars->drain, 1);
         bars->abort = 0;
@@ -371,8 +409,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else {
         // ------------------------------------------------------------ epilogue
-        const int quarter = warp & 3;                 // TMEM lanes 32*quarter .. +31
-        const int row = quarter * 32 + lane;          // accumulator row of this thread
+        // Warp e (0..7) drains TMEM lane quarter warp % 4 (rows 32 q .. 32 q + 31
+        // of the tile) and column half e / 4, in chunks of 32 columns.
+        const int e = warp - 2;
+        const int quarter = warp & 3;
+        const int half = e >> 2;
+        constexpr int NCH = BN / 64;                  // chunks per column half
+        uint32_t* buf = reinterpret_cast<uint32_t*>(epi_smem + (size_t)e * kEpiBufBytes);
         int acc = 0;
         uint32_t acc_phase = 0;
         for (int u = blockIdx.x; u < p.n_units; u += gridDim.x) {
@@ -382,74 +425,165 @@ __global__ void __launch_bounds__(kThreads, 1)
             ok = __shfl_sync(0xffffffffu, ok, 0);
             if (!ok) break;
             tc_fence_after();
-            const uint32_t t_row = tmem_base + ((uint32_t)(quarter * 32) << 16) +
-                                   (uint32_t)(acc * BN);
+            const uint32_t t_base = tmem_base + ((uint32_t)(quarter * 32) << 16) +
+                                    (uint32_t)(acc * BN + half * (BN / 2));
             if (MODE != MODE_DW) {
                 const RowUnit r = decode_row_unit(p, u);
-                const int q = r.t * kBlockM + row;
-                const bool valid = q < p.Mh;
-                const int lo = q % p.k, hi = q / p.k;
-                const size_t token = (size_t)hi * (2 * (size_t)p.k) + (size_t)r.beta * p.k + lo;
-                const size_t base = token * (size_t)p.d;
+                // tokens of this warp's 32 rows, as seen by the line-wise lanes
+                // (row 8 it + lane / 4 for it = 0..3); -1 marks rows past the end
+                long long tok_line[4];
+#pragma unroll
+                for (int it = 0; it < 4; ++it) {
+                    const int q = r.t * kBlockM + quarter * 32 + line_row_bf16(it, lane);
+                    tok_line[it] = q < p.Mh ? ((long long)(q >> p.s) << (p.s + 1)) +
+                                                  ((long long)r.beta << p.s) + (q & (p.k - 1))
+                                            : -1;
+                }
+                const int col_half = r.j * BN + half * (BN / 2);
+                const bool has_res = (p.flags & 2u) != 0;
+                const bool has_zp = MODE == MODE_DX && p.dz_out != nullptr;
+                uint4 res_g[4], zp_g[4];
+                auto load_lines = [&](const __nv_bfloat16* src, int c, uint4 (&g)[4]) {
+#pragma unroll
+                    for (int it = 0; it < 4; ++it) {
+                        g[it] = make_uint4(0, 0, 0, 0);
+                        if (tok_line[it] >= 0)
+                            g[it] = __ldg(reinterpret_cast<const uint4*>(
+                                src + tok_line[it] * p.d + col_half + c * 32 + 8 * (lane & 3)));
+                    }
+                };
+                // line-wise registers -> per-row words (through the buffer)
+                auto to_rows = [&](const uint4 (&g)[4], uint32_t (&w)[16]) {
+#pragma unroll
+                    for (int it = 0; it < 4; ++it)
+                        *reinterpret_cast<uint4*>(
+                            bf16_piece(buf, line_row_bf16(it, lane), lane & 3)) = g[it];
+                    __syncwarp();
+                    read_row_bf16(buf, lane, w);
+                    __syncwarp();
+                };
+                // per-row words -> coalesced line stores (through the buffer)
+                auto store_rows = [&](__nv_bfloat16* dst, int c, const uint32_t (&w)[16]) {
+                    stage_row_bf16(buf, lane, w);
+                    __syncwarp();
+#pragma unroll
+                    for (int it = 0; it < 4; ++it) {
+                        const uint4 v = *reinterpret_cast<const uint4*>(
+                            bf16_piece(buf, line_row_bf16(it, lane), lane & 3));
+                        if (tok_line[it] >= 0)
+                            *reinterpret_cast<uint4*>(dst + tok_line[it] * p.d + col_half +
+                                                      c * 32 + 8 * (lane & 3)) = v;
+                    }
+                    __syncwarp();
+                };
+                if (has_res) load_lines(p.resid, 0, res_g);
+                if (has_zp) load_lines(p.zprev, 0, zp_g);
 #pragma unroll 1
-                for (int c = 0; c < BN / 32; ++c) {
+                for (int c = 0; c < NCH; ++c) {
                     uint32_t raw[32];
-                    tmem_ld_32x32b_x32(t_row + c * 32, raw);
-                    tmem_ld_wait();
-                    if (!valid) continue;
-                    const int col0 = r.j * BN + c * 32;
+                    tmem_ld_32x32b_x32(t_base + c * 32, raw);
+                    tmem_ld_wait_regs(raw);
+                    if (c == NCH - 1) {
+                        // the accumulator is drained: hand it back to the MMA warp
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&bars->tempty[acc]);
+                    }
+                    uint32_t res_w[16], zp_w[16];
+                    if (has_res) to_rows(res_g, res_w);
+                    if (has_zp) to_rows(zp_g, zp_w);
+                    if (c + 1 < NCH) {   // prefetch the next chunk's inputs
+                        if (has_res) load_lines(p.resid, c + 1, res_g);
+                        if (has_zp) load_lines(p.zprev, c + 1, zp_g);
+                    }
                     float v[32];
 #pragma unroll
-                    for (int e = 0; e < 32; ++e) v[e] = __uint_as_float(raw[e]);
+                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(raw[i]);
+                    uint32_t w[16];
                     if (MODE == MODE_FWD) {
                         if (p.bias) {
-                            const float4* b4 = reinterpret_cast<const float4*>(p.bias + col0);
+                            const float4* b4 =
+                                reinterpret_cast<const float4*>(p.bias + col_half + c * 32);
 #pragma unroll
-                            for (int e = 0; e < 8; ++e) {
-                                float4 b = __ldg(b4 + e);
-                                v[4 * e] += b.x;
-                                v[4 * e + 1] += b.y;
-                                v[4 * e + 2] += b.z;
-                                v[4 * e + 3] += b.w;
+                            for (int i = 0; i < 8; ++i) {
+                                const float4 bb = __ldg(b4 + i);
+                                v[4 * i] += bb.x;
+                                v[4 * i + 1] += bb.y;
+                                v[4 * i + 2] += bb.z;
+                                v[4 * i + 3] += bb.w;
                             }
                         }
-                        if (p.zout) store_bf16x32(p.zout + base + col0, v);
+                        if (p.zout) {
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) w[i] = pack_bf16x2(v[2 * i], v[2 * i + 1]);
+                            store_rows(p.zout, c, w);
+                        }
                         if (p.flags & 4u) {
 #pragma unroll
-                            for (int e = 0; e < 32; ++e) v[e] = v[e] > 0.f ? v[e] : 0.f;
+                            for (int i = 0; i < 32; ++i) v[i] = v[i] > 0.f ? v[i] : 0.f;
                         }
                     }
-                    if (p.flags & 2u) add_bf16x32(p.resid + base + col0, v);
-                    store_bf16x32(p.out + base + col0, v);
+                    if (has_res) {
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            const float2 f = unpack_bf16x2(res_w[i]);
+                            v[2 * i] += f.x;
+                            v[2 * i + 1] += f.y;
+                        }
+                    }
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) w[i] = pack_bf16x2(v[2 * i], v[2 * i + 1]);
+                    if (p.out) store_rows(p.out, c, w);
+                    if (has_zp) {
+                        // fused ReLU gradient of the layer below: dz = g * (z > 0)
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            const float2 zz = unpack_bf16x2(zp_w[i]);
+                            const uint32_t lo = zz.x > 0.f ? (w[i] & 0xFFFFu) : 0u;
+                            const uint32_t hi = zz.y > 0.f ? (w[i] & 0xFFFF0000u) : 0u;
+                            w[i] = lo | hi;
+                        }
+                        store_rows(p.dz_out, c, w);
+                    }
                 }
             } else {
                 const WUnit w = decode_w_unit(p, u);
-                const int o = w.ot * kBlockM + row;
                 const int S = w.which ? p.splits_nbr : p.splits_self;
-                float* dst;
+                float* dst_base;
                 if (S == 1)
-                    dst = (w.which ? p.dw_nbr : p.dw_self) + (size_t)o * p.d;
+                    dst_base = w.which ? p.dw_nbr : p.dw_self;
                 else
-                    dst = p.dw_partial +
-                          (((size_t)w.which * p.splits_max + w.split) * p.d + o) * (size_t)p.d;
+                    dst_base = p.dw_partial + ((size_t)w.which * p.splits_max + w.split) *
+                                                  (size_t)p.d * p.d;
+                const int o0 = w.ot * kBlockM + quarter * 32;
+                const int col_half = w.nt * BN + half * (BN / 2);
 #pragma unroll 1
-                for (int c = 0; c < BN / 32; ++c) {
+                for (int c = 0; c < NCH; ++c) {
                     uint32_t raw[32];
-                    tmem_ld_32x32b_x32(t_row + c * 32, raw);
-                    tmem_ld_wait();
-                    if (o >= p.d) continue;
-                    float4* d4 = reinterpret_cast<float4*>(dst + w.nt * BN + c * 32);
+                    tmem_ld_32x32b_x32(t_base + c * 32, raw);
+                    tmem_ld_wait_regs(raw);
+                    if (c == NCH - 1) {
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&bars->tempty[acc]);
+                    }
 #pragma unroll
-                    for (int e = 0; e < 8; ++e)
-                        d4[e] = make_float4(__uint_as_float(raw[4 * e]),
-                                            __uint_as_float(raw[4 * e + 1]),
-                                            __uint_as_float(raw[4 * e + 2]),
-                                            __uint_as_float(raw[4 * e + 3]));
+                    for (int m = 0; m < 8; ++m)
+                        *reinterpret_cast<uint4*>(f32_piece(buf, lane, m)) =
+                            make_uint4(raw[4 * m], raw[4 * m + 1], raw[4 * m + 2], raw[4 * m + 3]);
+                    __syncwarp();
+#pragma unroll
+                    for (int it = 0; it < 8; ++it) {
+                        const int rr = 4 * it + (lane >> 3);
+                        const uint4 v =
+                            *reinterpret_cast<const uint4*>(f32_piece(buf, rr, lane & 7));
+                        if (o0 + rr < p.d)
+                            *reinterpret_cast<uint4*>(dst_base + (size_t)(o0 + rr) * p.d +
+                                                      col_half + c * 32 + 4 * (lane & 7)) = v;
+                    }
+                    __syncwarp();
                 }
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&bars->tempty[acc]);
             acc ^= 1;
             if (acc == 0) acc_phase ^= 1;
         }
