@@ -146,7 +146,12 @@ WPlan plan_dw(long long tokens, int d, unsigned flags) {
     // units still fit in one wave of persistent CTAs: makespan = kpu blocks
     long long kpu = (total_kb + sms - 1) / sms;
     if (kpu < 4) kpu = 4;
-    while (tiles * ((w.nkb_self + kpu - 1) / kpu + (w.nkb_nbr + kpu - 1) / kpu) > sms) ++kpu;
+    // (once kpu covers every block of both parts there is one split each and
+    // the count cannot drop further, even if the tiles alone exceed the SMs)
+    const long long kpu_max = w.nkb_self > w.nkb_nbr ? w.nkb_self : w.nkb_nbr;
+    while (kpu < kpu_max &&
+           tiles * ((w.nkb_self + kpu - 1) / kpu + (w.nkb_nbr + kpu - 1) / kpu) > sms)
+        ++kpu;
     w.kb_per_unit = (int)kpu;
     w.splits_self = (int)((w.nkb_self + kpu - 1) / kpu);
     w.splits_nbr = (int)((w.nkb_nbr + kpu - 1) / kpu);
@@ -749,3 +754,4 @@ int hcw_selftest_wait(long long timeout_ns, void* stream) {
 }
 
 }  // extern "C"
+

@@ -138,3 +138,12 @@ def test_workspace_sizes_f32(hcw):
     s = hcw.hcw_stack_workspace_bytes(64, 256, 512, hcw.HCW_F32, 0)
     assert s >= a + 2 * 64 * 256 * 512 * 4        # two gradient buffers between layers
     assert hcw.hcw_workspace_bytes(4, 48, 64, hcw.HCW_F32, 0) == 0   # invalid n
+
+
+@pytest.mark.timeout(60)
+def test_workspace_query_terminates_for_wide_layers(hcw):
+    # more output tiles than SMs: the split search must stop at one split per part
+    for d in (2048, 4096, 8192):
+        a = hcw.hcw_layer_bwd_weight_workspace_bytes(1 << 20, 4, d, hcw.HCW_BF16, 0)
+        b = hcw.hcw_workspace_bytes(1 << 20, 4, d, hcw.HCW_BF16, hcw.HCW_CAUSAL)
+        assert a > 0 and b > 0
