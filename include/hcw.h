@@ -185,6 +185,29 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* zs, const void* d
 /* Workspace bytes hcw_stack_bwd needs. */
 size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags);
 
+/*
+ * hcw_layer_bwd_weight for callers that cannot allocate device memory (a
+ * host that only lends its own input and output buffers, or code that must
+ * not call an allocator): same arguments and results, minus the workspace.
+ * The paper has no counterpart; this is an interface convenience.
+ *   Scratch: a fixed 32 MiB array inside the library, reserved on every
+ *   device that loads it until the process exits.  Sizes whose weight
+ *   gradient needs more scratch than that (hcw_layer_bwd_weight_workspace_bytes
+ *   > 32 MiB) are rejected with HCW_ERR_WORKSPACE before anything runs.
+ *   Allocates nothing: no cudaMalloc, cudaFree or allocating library call.
+ *   The first call on each device looks up the array's device address
+ *   (a one-time set-up per device, with that device current); make that
+ *   first call before any stream capture.
+ *   All calls share the one array: calls whose kernels may overlap on the
+ *   GPU (different streams without ordering, or several host threads) race
+ *   on it and must be serialised by the caller.  No part of the array needs
+ *   to start at zero; whatever a previous call left there is overwritten
+ *   before it is read.
+ */
+int hcw_layer_bwd_weight_noalloc(const void* x, const void* dz, int layer, int dim_override,
+                                 int B, int n, int d, int dtype, unsigned flags,
+                                 float* dW_self, float* dW_nbr, float* dbias, void* stream);
+
 /* Number of kernels this library has launched in this process (all devices). */
 unsigned long long hcw_launch_count(void);
 

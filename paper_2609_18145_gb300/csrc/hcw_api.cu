@@ -755,3 +755,71 @@ int hcw_selftest_wait(long long timeout_ns, void* stream) {
 
 }  // extern "C"
 
+// ---------------------------------------------------------------------------
+// Weight gradient without caller-provided workspace.
+//
+// Some callers cannot allocate device memory when they call in: a plugin
+// host that hands out only its own input/output buffers, code running in an
+// allocator-free section, or a process whose allocator is owned by someone
+// else.  hcw_layer_bwd_weight needs a scratch workspace (split-K partial
+// sums of dW and column-sum partials of dbias), so this variant keeps that
+// scratch in a fixed array linked into the library instead.  Every device
+// that loads the library reserves the array until the process exits.
+static constexpr size_t kNoAllocScratchBytes = (size_t)32 << 20;   // 32 MiB
+static __device__ __align__(256) unsigned char hcw_noalloc_scratch[kNoAllocScratchBytes];
+
+namespace {
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[1024];   // device address of the array, per device ordinal
+
+// The host-side name of the array is a stand-in, not a device address: ask
+// the runtime for the address on the current device (once per device).
+int noalloc_scratch(void** out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return HCW_ERR_CUDA;
+    if (dev < 0 || dev >= 1024) return HCW_ERR_UNSUPPORTED;
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, hcw_noalloc_scratch) != cudaSuccess || !p)
+            return HCW_ERR_CUDA;
+        g_noalloc_ptr[dev] = p;
+    }
+    *out = g_noalloc_ptr[dev];
+    return HCW_OK;
+}
+}  // namespace
+
+extern "C" {
+
+int hcw_layer_bwd_weight_noalloc(const void* x, const void* dz, int layer, int dim_override,
+                                 int B, int n, int d, int dtype, unsigned flags,
+                                 float* dW_self, float* dW_nbr, float* dbias, void* stream) {
+    Shape sh;
+    int rc = check_shape(layer, dim_override, B, n, d, dtype, flags, &sh);
+    if (rc) return rc;
+    if (!dW_self || !dW_nbr) return HCW_ERR_INVALID_ARG;
+    const void* ptrs[] = {x, dz, dW_self, dW_nbr, dbias};
+    for (const void* q : ptrs)
+        if (q && !aligned16(q)) return HCW_ERR_ALIGNMENT;
+    if (sh.tokens > 0 && (!x || !dz)) return HCW_ERR_INVALID_ARG;
+    // the fixed scratch must hold what the workspace would: reject larger sizes
+    if (ws_layout(sh.tokens, d, dtype, flags).w_bytes > kNoAllocScratchBytes)
+        return HCW_ERR_WORKSPACE;
+    const size_t ab = sh.act_bytes, gb = (size_t)d * d * 4;
+    if (overlaps(dW_self, gb, dW_nbr, gb) || overlaps(dbias, (size_t)d * 4, dW_self, gb) ||
+        overlaps(dbias, (size_t)d * 4, dW_nbr, gb) || overlaps(dW_self, gb, x, ab) ||
+        overlaps(dW_nbr, gb, x, ab) || overlaps(dW_self, gb, dz, ab) ||
+        overlaps(dW_nbr, gb, dz, ab))
+        return HCW_ERR_ALIASING;
+    void* scratch = nullptr;
+    rc = noalloc_scratch(&scratch);
+    if (rc) return rc;
+    // Every scratch byte the kernels read is written earlier in the same call
+    // (each split writes its whole slab, each column-sum chunk its row), so
+    // nothing has to be cleared between calls.
+    return layer_dw_impl(sh, dtype, x, dz, flags, dW_self, dW_nbr, dbias,
+                         static_cast<uint8_t*>(scratch), (cudaStream_t)stream);
+}
+
+}  // extern "C"

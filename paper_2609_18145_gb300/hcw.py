@@ -57,6 +57,7 @@ _SIGNATURES = {
     "hcw_layer_bwd_data": ([_P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _U, _P, _P], _I),
     "hcw_layer_bwd_weight_workspace_bytes": ([_I, _I, _I, _I, _U], _SZ),
     "hcw_layer_bwd_weight": ([_P, _P, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P, _SZ, _P], _I),
+    "hcw_layer_bwd_weight_noalloc": ([_P, _P, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P], _I),
     "hcw_launch_count": ([], ctypes.c_ulonglong),
     "hcw_stack_fwd": ([_P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P], _I),
     "hcw_stack_workspace_bytes": ([_I, _I, _I, _I, _U], _SZ),
