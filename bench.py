@@ -263,7 +263,7 @@ def run_ours(args):
     act_shape = (L - 1, B, n, d)
     y = torch.empty_like(x)
     acts = torch.empty(act_shape, dtype=torch.bfloat16, device=dev)
-    zs = torch.empty((L, B, n, d), dtype=torch.bfloat16, device=dev)
+    masks = torch.empty((L, B, n, d // 32), dtype=torch.int32, device=dev)
     dx = torch.empty_like(x)
     gWs = torch.empty((L, d, d), dtype=torch.float32, device=dev)
     gWn = torch.empty((L, d, d), dtype=torch.float32, device=dev)
@@ -273,13 +273,39 @@ def run_ours(args):
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
 
-    def step(xin, dyin):
-        H.hcw_stack_fwd(xin, Ws, Wn, bias, 0, -1, flags, y=y, acts=acts, zs=zs)
-        H.hcw_stack_bwd(xin, acts, zs, dyin, Ws, Wn, 0, -1, flags, dx=dx, dW_self=gWs,
+    def step_calls(xin, dyin):
+        H.hcw_stack_fwd(xin, Ws, Wn, bias, 0, -1, flags, y=y, acts=acts, masks=masks)
+        H.hcw_stack_bwd(xin, acts, masks, dyin, Ws, Wn, 0, -1, flags, dx=dx, dW_self=gWs,
                         dW_nbr=gWn, dbias=gb, workspace=ws)
+
+    def capture(xin, dyin):
+        # the step's launches, recorded once and replayed: no host work per step
+        g = torch.cuda.CUDAGraph()
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):
+            step_calls(xin, dyin)          # first call on this stream: one-time set-up
+            with torch.cuda.graph(g, stream=side):
+                step_calls(xin, dyin)
+        torch.cuda.current_stream().wait_stream(side)
+        return g
+
+    for _ in range(args.warmup):
+        step_calls(x, dy)
+    graph = capture(x, dy) if not args.no_graph else None
+    step_launches = H.hcw_launch_count()
+    step_calls(x, dy)
+    step_launches = H.hcw_launch_count() - step_launches
+
+    def step(xin, dyin):
+        if graph is not None and xin is x:
+            graph.replay()
+        else:
+            step_calls(xin, dyin)
 
     for _ in range(args.warmup):
         step(x, dy)
+    torch.cuda.synchronize()
     if H.hcw_sync_status() != H.HCW_OK:
         raise SystemExit("device error during warm-up")
 
@@ -297,6 +323,8 @@ def run_ours(args):
             ends[i].record(stream)
         torch.cuda.synchronize()
     launches = H.hcw_launch_count() - launches0
+    if graph is not None:
+        launches = step_launches * args.steps     # graph replays launch the captured kernels
     replicas.barrier()
     if H.hcw_sync_status() != H.HCW_OK:
         raise SystemExit("device error during the timed region")
@@ -319,8 +347,9 @@ def run_ours(args):
         return sum(a.elapsed_time(b) for a, b in evs) / reps
 
     dz = dy   # a layer's pre-activation gradient has the activations' shape and scale
-    fwd_ms = time_calls(lambda i: H.hcw_layer_fwd(x, Ws[i % L], Wn[i % L], bias[i % L], i % L,
-                                                  -1, flags, y=y, z_save=zs[0]), 2 * L)
+    fwd_ms = time_calls(lambda i: H.hcw_stack_fwd(x, Ws[i % L:i % L + 1], Wn[i % L:i % L + 1],
+                                                  bias[i % L:i % L + 1], i % L, -1, flags, y=y,
+                                                  masks=masks[:1]), 2 * L)
     dx_ms = time_calls(lambda i: H.hcw_layer_bwd_data(dz, dy, Ws[i % L], Wn[i % L], i % L, -1,
                                                       flags, dx=dx), 2 * L)
     wws = torch.empty(H.hcw_layer_bwd_weight_workspace_bytes(B, n, d, H.HCW_BF16, flags),
@@ -347,11 +376,12 @@ def run_ours(args):
     gWs_h = torch.empty(gWs.shape, dtype=gWs.dtype, pin_memory=True)
     gWn_h = torch.empty(gWn.shape, dtype=gWn.dtype, pin_memory=True)
     gb_h = torch.empty(gb.shape, dtype=gb.dtype, pin_memory=True)
-    x_d = torch.empty_like(x)
-    dy_d = torch.empty_like(dy)
+    x_d = x.clone()
+    dy_d = dy.clone()
     h2d = x_h.numel() * x_h.element_size() + dy_h.numel() * dy_h.element_size()
     d2h = sum(t.numel() * t.element_size() for t in (gWs_h, gWn_h, gb_h))
     e2e_steps = max(3, args.steps // 2)
+    e2e_graph = capture(x_d, dy_d) if not args.no_graph else None
     replicas.barrier()
     torch.cuda.synchronize()
     e_start = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
@@ -361,7 +391,10 @@ def run_ours(args):
         e_start[i].record(stream)
         x_d.copy_(x_h, non_blocking=True)
         dy_d.copy_(dy_h, non_blocking=True)
-        step(x_d, dy_d)
+        if e2e_graph is not None:
+            e2e_graph.replay()
+        else:
+            step_calls(x_d, dy_d)
         gWs_h.copy_(gWs, non_blocking=True)
         gWn_h.copy_(gWn, non_blocking=True)
         gb_h.copy_(gb, non_blocking=True)
@@ -390,7 +423,8 @@ def run_ours(args):
                        "tokens_per_step_per_gpu": tokens, "causal": True, "residual": True,
                        "act": "relu", "bias": True,
                        "l2": "flushed before every timed step (256 MiB write, untimed)",
-                       "parallelism": "replicas" if world > 1 else "single"},
+                       "parallelism": "replicas" if world > 1 else "single",
+                       "launch": "host calls" if args.no_graph else "CUDA graph of the step's calls"},
             "roofline": {"bound": "tensor", "kernel": dominant, "achieved": achieved,
                          "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                          "traffic": traffic, "peak_source": peak_src + " bf16 burst",
@@ -467,6 +501,9 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--no-graph", action="store_true",
+                    help="issue every step's launches from the host instead of replaying a "
+                         "CUDA graph of them")
     ap.add_argument("--no-cpu-baseline", action="store_true",
                     help="skip timing the CPU oracle (it is only timed at N = 1 anyway)")
     ap.add_argument("--kernel", choices=("fwd", "dx", "dw"),

@@ -161,22 +161,28 @@ int hcw_layer_bwd_weight(const void* x, const void* dz, int layer, int dim_overr
  *   y      [B][n][d] output of the last layer
  *   acts   [L-1][B][n][d] outputs of layers 0..L-2 (= inputs of layers
  *          1..L-1), written; required when L > 1 (kept for the backward)
- *   zs     [L][B][n][d] pre-activations, written, or NULL
+ *   masks  with HCW_ACT_RELU: [L][B][n][ceil(d/32)] uint32 words, written:
+ *          bit (o % 32) of word o/32 of token t is (z[t][o] > 0) -- the
+ *          one bit per activation that the ReLU backward needs (d/8 bytes
+ *          per token instead of the pre-activation itself); may be NULL
+ *          when no backward follows.  Ignored without HCW_ACT_RELU.
  */
 int hcw_stack_fwd(const void* x, const void* W_self, const void* W_nbr, const float* bias,
                   int layer0, int L, int dim_override, int B, int n, int d, int dtype,
-                  unsigned flags, void* y, void* acts, void* zs, void* stream);
+                  unsigned flags, void* y, void* acts, void* masks, void* stream);
 
 /*
  * Backward of hcw_stack_fwd, layers L-1 down to 0.
- *   x, acts, zs as given to / written by hcw_stack_fwd (zs required iff
- *   HCW_ACT_RELU); dy [B][n][d] gradient of y.
+ *   x, acts, masks as given to / written by hcw_stack_fwd (masks required
+ *   iff HCW_ACT_RELU); dy [B][n][d] gradient of y.
  *   dx [B][n][d] gradient of x (output); dW_self, dW_nbr [L][d][d] and
  *   dbias [L][d] (or NULL) fp32 outputs.
- *   workspace: at least hcw_workspace_bytes(...) + 2 * B*n*d*sizeof(dtype)
- *   bytes (two gradient buffers between layers).
+ *   workspace: at least hcw_stack_workspace_bytes(...) bytes.
+ * With HCW_ACT_RELU the input-gradient pass of layer l also applies the
+ * ReLU gradient of layer l-1 (bf16), so no separate elementwise pass runs
+ * between layers.
  */
-int hcw_stack_bwd(const void* x, const void* acts, const void* zs, const void* dy,
+int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void* dy,
                   const void* W_self, const void* W_nbr, int layer0, int L, int dim_override,
                   int B, int n, int d, int dtype, unsigned flags,
                   void* dx, float* dW_self, float* dW_nbr, float* dbias,

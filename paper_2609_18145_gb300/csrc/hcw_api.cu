@@ -63,19 +63,23 @@ EncodeTiledFn encode_fn() {
 }
 
 // Token-major activations [B*n][d] bf16 viewed as (d, lo = k, bit = 2, HI),
-// box (64 features, box_lo, 1, box_hi), 128-byte swizzle.
-bool map_rows(CUtensorMap* m, const void* base, long long tokens, int d, int k, int box_rows) {
+// box (inner features, box_lo, 1, box_hi) with box_lo * box_hi = box_rows
+// positions sharing bit s; the 128-byte swizzle for 64-feature (128-byte)
+// boxes, the 64-byte swizzle for 32-feature ones.
+bool map_rows(CUtensorMap* m, const void* base, long long tokens, int d, int k, int box_rows,
+              int inner = 64) {
     EncodeTiledFn enc = encode_fn();
-    if (!enc) return false;
+    if (!enc || !base) return false;
     const int box_lo = k < box_rows ? k : box_rows;
     const int box_hi = box_rows / box_lo;
     const long long HI = tokens / (2ll * k);
     cuuint64_t dims[4] = {(cuuint64_t)d, (cuuint64_t)k, 2, (cuuint64_t)HI};
     cuuint64_t strides[3] = {(cuuint64_t)d * 2, (cuuint64_t)k * d * 2, (cuuint64_t)2 * k * d * 2};
-    cuuint32_t box[4] = {64, (cuuint32_t)box_lo, 1, (cuuint32_t)box_hi};
+    cuuint32_t box[4] = {(cuuint32_t)inner, (cuuint32_t)box_lo, 1, (cuuint32_t)box_hi};
     cuuint32_t estr[4] = {1, 1, 1, 1};
     return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides,
-               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               inner == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
                CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -83,12 +87,27 @@ bool map_rows(CUtensorMap* m, const void* base, long long tokens, int d, int k, 
 // Weights W[o][k] bf16 [d][d], box (64 k, box_o), 128-byte swizzle.
 bool map_weight(CUtensorMap* m, const void* base, int d, int box_o) {
     EncodeTiledFn enc = encode_fn();
-    if (!enc) return false;
+    if (!enc || !base) return false;
     cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)d};
     cuuint64_t strides[1] = {(cuuint64_t)d * 2};
     cuuint32_t box[2] = {64, (cuuint32_t)box_o};
     cuuint32_t estr[2] = {1, 1};
     return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides,
+               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// fp32 matrix [rows][d], box (32 columns, 32 rows), 128-byte swizzle: the
+// patches the weight-gradient epilogue stores.
+bool map_f32_patches(CUtensorMap* m, const void* base, long long rows, int d) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc || !base) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)d * 4};
+    cuuint32_t box[2] = {32, 32};
+    cuuint32_t estr[2] = {1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(base), dims, strides,
                box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
@@ -123,6 +142,9 @@ int check_shape(int layer, int dim_override, int B, int n, int d, int dtype, uns
     sh->act_bytes = (size_t)tokens * d * elem_size(dtype);
     return HCW_OK;
 }
+
+// Bytes of one layer's ReLU mask: ceil(d/32) 32-bit words per token.
+size_t mask_bytes(const Shape& sh) { return (size_t)sh.tokens * ((sh.d + 31) / 32) * 4; }
 
 // ------------------------------------------------------------ bf16 sizes
 struct WPlan {
@@ -205,12 +227,16 @@ int launched(cudaError_t e, int kernels) {
 
 // ------------------------------------------------------------ layer internals
 int fwd_bf16(const Shape& sh, const void* x, const void* Ws, const void* Wn, const float* bias,
-             unsigned flags, void* y, void* z, cudaStream_t st) {
+             unsigned flags, void* y, void* z, uint32_t* mask, cudaStream_t st) {
     const int d = sh.d, BN = pick_bn(d), k = 1 << sh.s;
-    CUtensorMap tA, tB0, tB1;
-    if (!map_rows(&tA, x, sh.tokens, d, k, 128) || !map_weight(&tB0, Ws, d, BN) ||
-        !map_weight(&tB1, Wn, d, BN))
+    // patch width of the epilogue: 64 columns, or 32 for 64-wide tiles
+    const int pw = BN >= 128 ? 64 : 32;
+    CUtensorMap maps[6];
+    if (!map_rows(&maps[0], x, sh.tokens, d, k, 128) || !map_weight(&maps[1], Ws, d, BN) ||
+        !map_weight(&maps[2], Wn, d, BN) || !map_rows(&maps[3], x, sh.tokens, d, k, 32, pw) ||
+        !map_rows(&maps[4], y, sh.tokens, d, k, 32, pw))
         return HCW_ERR_CUDA;
+    maps[5] = maps[4];   // unused by the forward
     TcParams p;
     memset(&p, 0, sizeof(p));
     p.d = d;
@@ -234,23 +260,28 @@ int fwd_bf16(const Shape& sh, const void* x, const void* Ws, const void* Wn, con
     p.n_units = p.n_rb * p.n_nt * 2;
     p.flags = flags;
     p.bias = bias;
-    p.resid = static_cast<const __nv_bfloat16*>(x);
     p.out = static_cast<__nv_bfloat16*>(y);
     p.zout = static_cast<__nv_bfloat16*>(z);
+    p.mout = mask;
     p.timeout_ns = g_timeout_ns;
     const int sms = sm_count();
     const int grid = p.n_units < sms ? p.n_units : sms;
-    return launched(launch_tc(MODE_FWD, BN, tA, tB0, tB1, p, grid, st), 1);
+    return launched(launch_tc(MODE_FWD, BN, maps, p, grid, st), 1);
 }
 
 // dx: a row gathers dz from its partner exactly when the partner received from it
 int dx_bf16(const Shape& sh, const void* dz, const void* dy, const void* Ws, const void* Wn,
-            unsigned flags, void* dx, cudaStream_t st, const void* zprev = nullptr,
+            unsigned flags, void* dx, cudaStream_t st, const uint32_t* mprev = nullptr,
             void* dz_out = nullptr) {
     const int d = sh.d, BN = pick_bn(d), k = 1 << sh.s;
-    CUtensorMap tA, tB0, tB1;
-    if (!map_rows(&tA, dz, sh.tokens, d, k, 128) || !map_weight(&tB0, Ws, d, 64) ||
-        !map_weight(&tB1, Wn, d, 64))
+    const int pw = BN >= 128 ? 64 : 32;
+    CUtensorMap maps[6];
+    // maps of absent operands get a valid stand-in address; the kernel never uses them
+    const void* res = (flags & HCW_RESIDUAL) ? dy : dz;
+    if (!map_rows(&maps[0], dz, sh.tokens, d, k, 128) || !map_weight(&maps[1], Ws, d, 64) ||
+        !map_weight(&maps[2], Wn, d, 64) || !map_rows(&maps[3], res, sh.tokens, d, k, 32, pw) ||
+        !map_rows(&maps[4], dx ? dx : dz_out, sh.tokens, d, k, 32, pw) ||
+        !map_rows(&maps[5], dz_out ? dz_out : dx, sh.tokens, d, k, 32, pw))
         return HCW_ERR_CUDA;
     TcParams p;
     memset(&p, 0, sizeof(p));
@@ -273,14 +304,13 @@ int dx_bf16(const Shape& sh, const void* dz, const void* dy, const void* Ws, con
     }
     p.n_units = p.n_rb * p.n_nt * 2;
     p.flags = flags & HCW_RESIDUAL;
-    p.resid = static_cast<const __nv_bfloat16*>(dy);
     p.out = static_cast<__nv_bfloat16*>(dx);
-    p.zprev = static_cast<const __nv_bfloat16*>(zprev);
+    p.mprev = mprev;
     p.dz_out = static_cast<__nv_bfloat16*>(dz_out);
     p.timeout_ns = g_timeout_ns;
     const int sms = sm_count();
     const int grid = p.n_units < sms ? p.n_units : sms;
-    return launched(launch_tc(MODE_DX, BN, tA, tB0, tB1, p, grid, st), 1);
+    return launched(launch_tc(MODE_DX, BN, maps, p, grid, st), 1);
 }
 
 // dW: token-contracted, split over token blocks, fixed-order reduction; dbias
@@ -290,9 +320,14 @@ int dw_bf16(const Shape& sh, const void* x, const void* dz, unsigned flags, floa
     const int d = sh.d, BN = pick_bn(d), k = 1 << sh.s;
     const WsLayout lay = ws_layout(sh.tokens, d, HCW_BF16, flags);
     const WPlan w = plan_dw(sh.tokens, d, flags);
-    CUtensorMap tA, tB0;
-    if (!map_rows(&tA, dz, sh.tokens, d, k, 64) || !map_rows(&tB0, x, sh.tokens, d, k, 64))
+    CUtensorMap maps[6];
+    float* part = reinterpret_cast<float*>(wws);
+    if (!map_rows(&maps[0], dz, sh.tokens, d, k, 64) || !map_rows(&maps[1], x, sh.tokens, d, k, 64) ||
+        !map_f32_patches(&maps[3], w.splits_max > 1 ? (const void*)part : (const void*)dWs,
+                         w.splits_max > 1 ? 2ll * w.splits_max * d : d, d) ||
+        !map_f32_patches(&maps[4], dWs, d, d) || !map_f32_patches(&maps[5], dWn, d, d))
         return HCW_ERR_CUDA;
+    maps[2] = maps[1];   // unused by the weight gradient
     TcParams p;
     memset(&p, 0, sizeof(p));
     p.d = d;
@@ -312,11 +347,11 @@ int dw_bf16(const Shape& sh, const void* x, const void* dz, unsigned flags, floa
     p.n_units = w.units;
     p.dw_self = dWs;
     p.dw_nbr = dWn;
-    p.dw_partial = reinterpret_cast<float*>(wws);
+    p.dw_partial = part;
     p.timeout_ns = g_timeout_ns;
     const int sms = sm_count();
     const int grid = p.n_units < sms ? p.n_units : sms;
-    int rc = launched(launch_tc(MODE_DW, BN, tA, tB0, tB0, p, grid, st), 1);
+    int rc = launched(launch_tc(MODE_DW, BN, maps, p, grid, st), 1);
     if (rc) return rc;
     if (w.splits_max > 1) {
         rc = launched(launch_splitk_reduce(p.dw_partial, w.splits_max, w.splits_self,
@@ -333,10 +368,11 @@ int dw_bf16(const Shape& sh, const void* x, const void* dz, unsigned flags, floa
 }
 
 int fwd_f32(const Shape& sh, const void* x, const void* Ws, const void* Wn, const float* bias,
-            unsigned flags, void* y, void* z, cudaStream_t st) {
+            unsigned flags, void* y, void* z, uint32_t* mask, cudaStream_t st) {
     return launched(launch_f32_fwd(static_cast<const float*>(x), static_cast<const float*>(Ws),
                                    static_cast<const float*>(Wn), bias, sh.s, sh.B, sh.n, sh.d,
-                                   flags, static_cast<float*>(y), static_cast<float*>(z), st),
+                                   flags, static_cast<float*>(y), static_cast<float*>(z), mask,
+                                   st),
                     1);
 }
 
@@ -361,10 +397,11 @@ int dw_f32(const Shape& sh, const void* x, const void* dz, unsigned flags, float
 }
 
 int layer_fwd_impl(const Shape& sh, int dtype, const void* x, const void* Ws, const void* Wn,
-                   const float* bias, unsigned flags, void* y, void* z, cudaStream_t st) {
+                   const float* bias, unsigned flags, void* y, void* z, cudaStream_t st,
+                   uint32_t* mask = nullptr) {
     if (sh.tokens == 0) return HCW_OK;
-    return dtype == HCW_BF16 ? fwd_bf16(sh, x, Ws, Wn, bias, flags, y, z, st)
-                             : fwd_f32(sh, x, Ws, Wn, bias, flags, y, z, st);
+    return dtype == HCW_BF16 ? fwd_bf16(sh, x, Ws, Wn, bias, flags, y, z, mask, st)
+                             : fwd_f32(sh, x, Ws, Wn, bias, flags, y, z, mask, st);
 }
 
 int zero_weight_grads(const Shape& sh, float* dWs, float* dWn, float* dbias, cudaStream_t st) {
@@ -596,34 +633,38 @@ int hcw_layer_bwd_weight(const void* x, const void* dz, int layer, int dim_overr
 
 int hcw_stack_fwd(const void* x, const void* W_self, const void* W_nbr, const float* bias,
                   int layer0, int L, int dim_override, int B, int n, int d, int dtype,
-                  unsigned flags, void* y, void* acts, void* zs, void* stream) {
+                  unsigned flags, void* y, void* acts, void* masks, void* stream) {
     Shape sh;
     if (L < 1) return HCW_ERR_INVALID_ARG;
     int rc = check_shape(layer0, dim_override, B, n, d, dtype, flags, &sh);
     if (rc) return rc;
     if (sh.tokens == 0) return HCW_OK;
     if (L > 1 && !acts) return HCW_ERR_INVALID_ARG;
-    if ((acts && !aligned16(acts)) || (zs && !aligned16(zs))) return HCW_ERR_ALIGNMENT;
+    if ((acts && !aligned16(acts)) || (masks && !aligned16(masks))) return HCW_ERR_ALIGNMENT;
     const size_t ab = sh.act_bytes, wb = (size_t)d * d * elem_size(dtype);
+    const size_t mb = mask_bytes(sh);
     rc = check_fwd_ptrs(sh, dtype, x, W_self, W_nbr, bias, y, nullptr);
     if (rc) return rc;
-    const size_t acts_b = (size_t)(L - 1) * ab, zs_b = (size_t)L * ab;
+    const size_t acts_b = (size_t)(L - 1) * ab, m_b = (size_t)L * mb;
     if (overlaps(acts, acts_b, x, ab) || overlaps(acts, acts_b, y, ab) ||
-        overlaps(zs, zs_b, x, ab) || overlaps(zs, zs_b, y, ab) ||
-        overlaps(zs, zs_b, acts, acts_b) || overlaps(acts, acts_b, W_self, L * wb) ||
+        overlaps(masks, m_b, x, ab) || overlaps(masks, m_b, y, ab) ||
+        overlaps(masks, m_b, acts, acts_b) || overlaps(acts, acts_b, W_self, L * wb) ||
         overlaps(acts, acts_b, W_nbr, L * wb))
         return HCW_ERR_ALIASING;
     cudaStream_t st = (cudaStream_t)stream;
     const uint8_t* xin = static_cast<const uint8_t*>(x);
+    const bool want_mask = masks && (flags & HCW_ACT_RELU);
     for (int l = 0; l < L; ++l) {
         Shape shl = sh;
         shl.s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
         const uint8_t* in = l == 0 ? xin : static_cast<const uint8_t*>(acts) + (size_t)(l - 1) * ab;
         void* out = l == L - 1 ? y : static_cast<uint8_t*>(acts) + (size_t)l * ab;
-        void* z = zs ? static_cast<uint8_t*>(zs) + (size_t)l * ab : nullptr;
+        uint32_t* m = want_mask
+                          ? reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(masks) + (size_t)l * mb)
+                          : nullptr;
         rc = layer_fwd_impl(shl, dtype, in, static_cast<const uint8_t*>(W_self) + l * wb,
                             static_cast<const uint8_t*>(W_nbr) + l * wb,
-                            bias ? bias + (size_t)l * d : nullptr, flags, out, z, st);
+                            bias ? bias + (size_t)l * d : nullptr, flags, out, nullptr, st, m);
         if (rc) return rc;
     }
     return HCW_OK;
@@ -637,7 +678,7 @@ size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags)
     return ws_layout(sh.tokens, d, dtype, flags).w_bytes + 4 * align256(sh.act_bytes);
 }
 
-int hcw_stack_bwd(const void* x, const void* acts, const void* zs, const void* dy,
+int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void* dy,
                   const void* W_self, const void* W_nbr, int layer0, int L, int dim_override,
                   int B, int n, int d, int dtype, unsigned flags, void* dx, float* dW_self,
                   float* dW_nbr, float* dbias, void* workspace, size_t ws_bytes, void* stream) {
@@ -654,21 +695,24 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* zs, const void* d
         if (e == cudaSuccess && dbias) e = cudaMemsetAsync(dbias, 0, (size_t)L * d * 4, st0);
         return cuda_status(e);
     }
-    if ((L > 1 && !acts) || ((flags & HCW_ACT_RELU) && !zs)) return HCW_ERR_INVALID_ARG;
-    rc = check_bwd_ptrs(sh, dtype, flags, x, zs, dy, W_self, W_nbr, dx, dW_self, dW_nbr, dbias);
+    const bool relu = (flags & HCW_ACT_RELU) != 0;
+    const bool resid = (flags & HCW_RESIDUAL) != 0;
+    if ((L > 1 && !acts) || (relu && !masks)) return HCW_ERR_INVALID_ARG;
+    rc = check_bwd_ptrs(sh, dtype, flags & ~HCW_ACT_RELU, x, nullptr, dy, W_self, W_nbr, dx,
+                        dW_self, dW_nbr, dbias);
     if (rc) return rc;
-    if ((acts && !aligned16(acts))) return HCW_ERR_ALIGNMENT;
+    if ((acts && !aligned16(acts)) || (masks && !aligned16(masks))) return HCW_ERR_ALIGNMENT;
     const size_t ab = sh.act_bytes, wb = (size_t)d * d * elem_size(dtype);
-    const size_t gb = (size_t)d * d * 4;
+    const size_t gb = (size_t)d * d * 4, mb = mask_bytes(sh);
     const size_t need = hcw_stack_workspace_bytes(B, n, d, dtype, flags);
     if (ws_bytes < need || !workspace) return HCW_ERR_WORKSPACE;
     if (!aligned16(workspace)) return HCW_ERR_ALIGNMENT;
+    const size_t acts_b = (size_t)(L > 1 ? L - 1 : 0) * ab;
     if (overlaps(workspace, ws_bytes, dx, ab) || overlaps(workspace, ws_bytes, dy, ab) ||
-        overlaps(workspace, ws_bytes, x, ab) ||
-        overlaps(workspace, ws_bytes, acts, (size_t)(L > 1 ? L - 1 : 0) * ab) ||
-        overlaps(workspace, ws_bytes, zs, zs ? (size_t)L * ab : 0) ||
-        overlaps(dW_self, (size_t)L * gb, dW_nbr, (size_t)L * gb) ||
-        overlaps(dx, ab, acts, (size_t)(L > 1 ? L - 1 : 0) * ab))
+        overlaps(workspace, ws_bytes, x, ab) || overlaps(workspace, ws_bytes, acts, acts_b) ||
+        overlaps(workspace, ws_bytes, masks, relu ? (size_t)L * mb : 0) ||
+        overlaps(dW_self, (size_t)L * gb, dW_nbr, (size_t)L * gb) || overlaps(dx, ab, acts, acts_b) ||
+        overlaps(dx, ab, masks, relu ? (size_t)L * mb : 0))
         return HCW_ERR_ALIASING;
     cudaStream_t st = (cudaStream_t)stream;
     uint8_t* wsb = static_cast<uint8_t*>(workspace);
@@ -676,25 +720,23 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* zs, const void* d
     uint8_t* g[2] = {wsb, wsb + ab256};                    // output gradients
     uint8_t* gz[2] = {wsb + 2 * ab256, wsb + 3 * ab256};   // pre-activation gradients
     uint8_t* wws = wsb + 4 * ab256;                        // weight-gradient workspace
-    const bool relu = (flags & HCW_ACT_RELU) != 0;
-    const bool resid = (flags & HCW_RESIDUAL) != 0;
-    auto layer_ptr = [&](const void* base, int l) {
-        return static_cast<const uint8_t*>(base) + (size_t)l * ab;
+    auto act_ptr = [&](int l) { return static_cast<const uint8_t*>(acts) + (size_t)l * ab; };
+    auto mask_ptr = [&](int l) {
+        return reinterpret_cast<const uint32_t*>(static_cast<const uint8_t*>(masks) +
+                                                 (size_t)l * mb);
     };
     // gradient at the output (cur_g) and at the pre-activation (cur_dz) of layer l
     const void* cur_g = dy;
     const void* cur_dz = dy;
     if (relu) {
         rc = launched(dtype == HCW_BF16
-                          ? launch_relu_grad_bf16(static_cast<const __nv_bfloat16*>(dy),
-                                                  reinterpret_cast<const __nv_bfloat16*>(
-                                                      layer_ptr(zs, L - 1)),
-                                                  reinterpret_cast<__nv_bfloat16*>(gz[(L - 1) & 1]),
-                                                  (size_t)sh.tokens * d, st)
-                          : launch_relu_grad_f32(static_cast<const float*>(dy),
-                                                 reinterpret_cast<const float*>(layer_ptr(zs, L - 1)),
-                                                 reinterpret_cast<float*>(gz[(L - 1) & 1]),
-                                                 (size_t)sh.tokens * d, st),
+                          ? launch_relu_grad_mask_bf16(static_cast<const __nv_bfloat16*>(dy),
+                                                       mask_ptr(L - 1),
+                                                       reinterpret_cast<__nv_bfloat16*>(gz[(L - 1) & 1]),
+                                                       sh.tokens, d, st)
+                          : launch_relu_grad_mask_f32(static_cast<const float*>(dy), mask_ptr(L - 1),
+                                                      reinterpret_cast<float*>(gz[(L - 1) & 1]),
+                                                      sh.tokens, d, st),
                       1);
         if (rc) return rc;
         cur_dz = gz[(L - 1) & 1];
@@ -702,7 +744,7 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* zs, const void* d
     for (int l = L - 1; l >= 0; --l) {
         Shape shl = sh;
         shl.s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
-        const void* in = l == 0 ? x : layer_ptr(acts, l - 1);
+        const void* in = l == 0 ? x : act_ptr(l - 1);
         const void* Wsl = static_cast<const uint8_t*>(W_self) + l * wb;
         const void* Wnl = static_cast<const uint8_t*>(W_nbr) + l * wb;
         void* out_g = l == 0 ? dx : ((resid || !relu) ? (void*)g[l & 1] : nullptr);
@@ -710,18 +752,18 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* zs, const void* d
         if (l > 0 && relu) {
             next_dz = gz[(l - 1) & 1];
             if (dtype == HCW_BF16) {
-                // the input gradient kernel also applies the ReLU gradient of layer l-1
-                rc = dx_bf16(shl, cur_dz, cur_g, Wsl, Wnl, flags, out_g, st, layer_ptr(zs, l - 1),
+                // the input-gradient kernel also applies the ReLU gradient of layer l-1
+                rc = dx_bf16(shl, cur_dz, cur_g, Wsl, Wnl, flags, out_g, st, mask_ptr(l - 1),
                              next_dz);
             } else {
-                rc = layer_dx_impl(shl, dtype, cur_dz, cur_g, Wsl, Wnl, flags, g[l & 1], st);
-                if (!rc)
-                    rc = launched(launch_relu_grad_f32(static_cast<const float*>((const void*)g[l & 1]),
-                                                       reinterpret_cast<const float*>(layer_ptr(zs, l - 1)),
-                                                       reinterpret_cast<float*>(next_dz),
-                                                       (size_t)sh.tokens * d, st),
-                                  1);
                 out_g = g[l & 1];
+                rc = layer_dx_impl(shl, dtype, cur_dz, cur_g, Wsl, Wnl, flags, out_g, st);
+                if (!rc)
+                    rc = launched(launch_relu_grad_mask_f32(static_cast<const float*>(out_g),
+                                                            mask_ptr(l - 1),
+                                                            static_cast<float*>(next_dz),
+                                                            sh.tokens, d, st),
+                                  1);
             }
         } else {
             rc = layer_dx_impl(shl, dtype, cur_dz, cur_g, Wsl, Wnl, flags, out_g, st);

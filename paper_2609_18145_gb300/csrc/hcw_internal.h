@@ -43,11 +43,11 @@ struct TcParams {
     // epilogue
     unsigned flags;
     const float* bias;            // FWD
-    const __nv_bfloat16* resid;   // FWD: x; DX: dy
     __nv_bfloat16* out;           // FWD: y; DX: dx (may be null when dz_out is set)
     __nv_bfloat16* zout;          // FWD: z (may be null)
-    const __nv_bfloat16* zprev;   // DX: pre-activation of the layer below (fused ReLU grad)
-    __nv_bfloat16* dz_out;        // DX: its gradient dz = dx * (zprev > 0), or null
+    uint32_t* mout;               // FWD: ReLU mask words [tokens][d/32], bit e = (z > 0), or null
+    const uint32_t* mprev;        // DX: ReLU mask words of the layer below (fused ReLU grad)
+    __nv_bfloat16* dz_out;        // DX: that layer's gradient dz = dx * mask, or null
     float* dw_self;               // DW destination when splits_self == 1
     float* dw_nbr;                // DW destination when splits_nbr == 1
     float* dw_partial;            // DW partials [2][splits_max][d][d]
@@ -55,9 +55,9 @@ struct TcParams {
     unsigned long long timeout_ns;
 };
 
-// Launch one tensor-core pass.  tmA / tmB0 / tmB1 as documented in hcw_tc.cu.
-cudaError_t launch_tc(int mode, int BN, const CUtensorMap& tmA, const CUtensorMap& tmB0,
-                      const CUtensorMap& tmB1, const TcParams& p, int grid,
+// Launch one tensor-core pass.  maps[0..5] = tmA, tmB0, tmB1, tmE0, tmE1, tmE2
+// as documented at hcw_tc_kernel in hcw_tc.cu.
+cudaError_t launch_tc(int mode, int BN, const CUtensorMap* maps, const TcParams& p, int grid,
                       cudaStream_t stream);
 
 // Dynamic shared memory the tensor-core kernel uses for this N tile.
@@ -67,7 +67,13 @@ int tc_stages(int BN);
 // ---- SIMT kernels (hcw_simt.cu) ----
 cudaError_t launch_f32_fwd(const float* x, const float* Ws, const float* Wn, const float* bias,
                            int s, int B, int n, int d, unsigned flags, float* y, float* z,
-                           cudaStream_t st);
+                           uint32_t* mout, cudaStream_t st);
+// dz = dy where the ReLU mask bit is set, else 0 (masks [rows][ceil(d/32)] words)
+cudaError_t launch_relu_grad_mask_f32(const float* dy, const uint32_t* mask, float* dz,
+                                      long long rows, int d, cudaStream_t st);
+cudaError_t launch_relu_grad_mask_bf16(const __nv_bfloat16* dy, const uint32_t* mask,
+                                       __nv_bfloat16* dz, long long rows, int d,
+                                       cudaStream_t st);
 cudaError_t launch_f32_dx(const float* dz, const float* dy, const float* Ws, const float* Wn,
                           int s, int B, int n, int d, unsigned flags, float* dx,
                           cudaStream_t st);

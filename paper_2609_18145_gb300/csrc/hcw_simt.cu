@@ -23,10 +23,12 @@ constexpr int T = 32;   // tile edge of the fp32 kernels
 
 // z[r][o] = sum_k Ws[o][k] x[r][k] + m_r sum_k Wn[o][k] x[p(r)][k] + bias[o]
 // Block: 32 rows x 32 outputs, 32 x 8 threads, 4 outputs per thread.
+// mout (optional): ReLU mask words [rows][ceil(d/32)], bit o%32 of word o/32 = (z > 0).
 __global__ void f32_fwd_kernel(const float* __restrict__ x, const float* __restrict__ Ws,
                                const float* __restrict__ Wn, const float* __restrict__ bias,
                                int s, int n, int d, long long rows, unsigned flags,
-                               float* __restrict__ y, float* __restrict__ z) {
+                               float* __restrict__ y, float* __restrict__ z,
+                               uint32_t* __restrict__ mout) {
     __shared__ float xs[T][T + 1], xp[T][T + 1], ws[T][T + 1], wn[T][T + 1];
     const long long r0 = (long long)blockIdx.y * T;
     const int o0 = blockIdx.x * T;
@@ -62,12 +64,18 @@ __global__ void f32_fwd_kernel(const float* __restrict__ x, const float* __restr
         __syncthreads();
     }
     const int o = o0 + tx;
-    if (o >= d) return;
+    const int wpr = (d + 31) >> 5;
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
         const long long r = r0 + ty + 8 * q;
-        if (r >= rows) continue;
-        float v = acc[q] + (bias ? bias[o] : 0.f);
+        const bool ok = r < rows && o < d;
+        float v = ok ? acc[q] + (bias ? bias[o] : 0.f) : 0.f;
+        if (mout) {
+            // the warp covers the 32 columns of one mask word of row r
+            const unsigned bits = __ballot_sync(0xffffffffu, ok && v > 0.f);
+            if (tx == 0 && r < rows) mout[r * wpr + (o0 >> 5)] = bits;
+        }
+        if (!ok) continue;
         if (z) z[r * d + o] = v;
         if (flags & 4u) v = v > 0.f ? v : 0.f;
         if (flags & 2u) v += x[r * d + o];
@@ -194,6 +202,21 @@ __global__ void relu_grad_kernel(const V* __restrict__ dy, const V* __restrict__
         dz[t] = to_f(z[t]) > 0.f ? dy[t] : zero;
 }
 
+// dz[t][o] = mask bit (t, o) ? dy[t][o] : 0, masks as written by the forward.
+template <typename V>
+__global__ void relu_grad_mask_kernel(const V* __restrict__ dy, const uint32_t* __restrict__ mask,
+                                      V* __restrict__ dz, long long rows, int d) {
+    const int wpr = (d + 31) >> 5;
+    const size_t count = (size_t)rows * d;
+    const V zero = V(0.f);
+    for (size_t t = (size_t)blockIdx.x * blockDim.x + threadIdx.x; t < count;
+         t += (size_t)gridDim.x * blockDim.x) {
+        const size_t r = t / d;
+        const int o = (int)(t - r * d);
+        dz[t] = (mask[r * wpr + (o >> 5)] >> (o & 31)) & 1u ? dy[t] : zero;
+    }
+}
+
 constexpr int kColRows = 256;   // rows per partial of the column sum
 
 // partial[c][o] = sum_{r in chunk c} dz[r][o]  (block: 32 columns x 8 row lanes)
@@ -263,10 +286,26 @@ inline int blocks_for(size_t count, int threads, int cap = 152 * 16) {
 
 cudaError_t launch_f32_fwd(const float* x, const float* Ws, const float* Wn, const float* bias,
                            int s, int B, int n, int d, unsigned flags, float* y, float* z,
-                           cudaStream_t st) {
+                           uint32_t* mout, cudaStream_t st) {
     const long long rows = (long long)B * n;
     dim3 grid((d + T - 1) / T, (unsigned)((rows + T - 1) / T));
-    f32_fwd_kernel<<<grid, dim3(T, 8), 0, st>>>(x, Ws, Wn, bias, s, n, d, rows, flags, y, z);
+    f32_fwd_kernel<<<grid, dim3(T, 8), 0, st>>>(x, Ws, Wn, bias, s, n, d, rows, flags, y, z,
+                                                 mout);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_relu_grad_mask_f32(const float* dy, const uint32_t* mask, float* dz,
+                                      long long rows, int d, cudaStream_t st) {
+    relu_grad_mask_kernel<float><<<blocks_for((size_t)rows * d, 256), 256, 0, st>>>(dy, mask, dz,
+                                                                                  rows, d);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_relu_grad_mask_bf16(const __nv_bfloat16* dy, const uint32_t* mask,
+                                       __nv_bfloat16* dz, long long rows, int d,
+                                       cudaStream_t st) {
+    relu_grad_mask_kernel<__nv_bfloat16>
+        <<<blocks_for((size_t)rows * d, 256), 256, 0, st>>>(dy, mask, dz, rows, d);
     return cudaGetLastError();
 }
 

@@ -32,12 +32,19 @@
 // partials are reduced in a fixed order by a separate kernel
 // (deterministic).
 //
-// Roles (192 threads): warp 0 issues TMA loads into a STAGES-deep ring of
-// shared-memory stages; warp 1 owns TMEM (2 x BN fp32 columns, a double
-// buffered accumulator) and issues tcgen05.mma; warps 2..5 drain the
-// accumulator through tcgen05.ld, apply the epilogue and store.  Every wait
-// is bounded (hcw_ptx.cuh); a CTA that gives up records HCW_ERR_TIMEOUT,
-// drains its in-flight copies and MMAs, frees TMEM and returns.
+// Roles (320 threads): warp 0 issues TMA loads into a ring of shared-memory
+// stages; warp 1 owns TMEM (2 x BN fp32 columns, a double-buffered
+// accumulator) and issues tcgen05.mma; warps 2..9 drain the accumulator
+// through tcgen05.ld (two warps per TMEM lane quarter, one per column half).
+// All epilogue I/O goes through TMA: each epilogue warp has two 4 KB
+// buffers; the residual rows of its 32 x 64 patch are TMA-loaded into a
+// buffer before the accumulator is ready, each lane overwrites its own row
+// in place with the result, and a TMA store writes the patch back.  Every
+// wait is bounded (hcw_ptx.cuh); a CTA that gives up records
+// HCW_ERR_TIMEOUT, drains its in-flight copies and MMAs, frees TMEM and
+// returns.
+#include <atomic>
+
 #include "hcw_internal.h"
 #include "hcw_ptx.cuh"
 
@@ -50,8 +57,9 @@ constexpr int kThreads = 64 + 32 * kEpiWarps;      // producer, MMA, epilogue wa
 constexpr int kBlockM = 128;
 constexpr int kBlockK = 64;                        // bf16 elements per 128-byte row
 constexpr int kABytes = kBlockM * kBlockK * 2;     // 16 KB
-constexpr int kRingBytes = 192 * 1024;             // TMA stage ring
-constexpr int kEpiBufBytes = 4096;                 // per epilogue warp: 32 rows x 128 B
+constexpr int kRingBytes = 144 * 1024;             // TMA stage ring
+constexpr int kEpiBufBytes = 4096;                 // one epilogue patch: 32 rows x 128 B
+constexpr int kEpiBufs = 2;                        // per epilogue warp
 
 __host__ __device__ constexpr int stage_bytes(int BN) { return kABytes + BN * kBlockK * 2; }
 __host__ __device__ constexpr int num_stages(int BN) {
@@ -64,6 +72,7 @@ struct __align__(8) Barriers {
     uint64_t tfull[2];
     uint64_t tempty[2];
     uint64_t drain;
+    uint64_t epi_load[kEpiWarps][kEpiBufs];       // residual patch landed in a buffer
     uint32_t tmem_base;
     int abort;
 };
@@ -71,7 +80,8 @@ struct __align__(8) Barriers {
 template <int BN>
 __host__ __device__ constexpr size_t smem_total() {
     return 1024 /* alignment slack */ + (size_t)num_stages(BN) * stage_bytes(BN) +
-           (size_t)kEpiWarps * kEpiBufBytes + sizeof(Barriers);
+           (size_t)kEpiWarps * kEpiBufs * kEpiBufBytes + (size_t)kEpiWarps * (BN / 2) * 4 +
+           sizeof(Barriers);
 }
 
 // FWD/DX unit -> (row bit beta, row block t, column tile j, number of K steps)
@@ -125,23 +135,6 @@ __device__ __forceinline__ WUnit decode_w_unit(const TcParams& p, int u) {
     return w;
 }
 
-// ---- epilogue staging ------------------------------------------------------
-// Each epilogue warp owns 32 accumulator rows (one per lane, as tcgen05.ld
-// delivers them) and moves them through a private 4 KB shared buffer so that
-// global loads and stores are whole-line and coalesced.  Rows are 16-byte
-// pieces XOR-swizzled by row so that both the row-wise accesses (a lane per
-// row) and the line-wise accesses (lanes along a row) are conflict-free.
-//   bf16 chunk: 32 rows x 32 values = 32 x 64 B, piece m of row r at word
-//               16 r + 4 (m ^ ((r >> 1) & 3))
-//   fp32 chunk: 32 rows x 32 values = 32 x 128 B, piece m of row r at word
-//               32 r + 4 (m ^ (r & 7))
-__device__ __forceinline__ uint32_t* bf16_piece(uint32_t* buf, int r, int m) {
-    return buf + 16 * r + 4 * (m ^ ((r >> 1) & 3));
-}
-__device__ __forceinline__ uint32_t* f32_piece(uint32_t* buf, int r, int m) {
-    return buf + 32 * r + 4 * (m ^ (r & 7));
-}
-
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
     __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
     return *reinterpret_cast<uint32_t*>(&h);
@@ -152,28 +145,16 @@ __device__ __forceinline__ float2 unpack_bf16x2(uint32_t w) {
     return __bfloat1622float2(h);
 }
 
-// Lane `lane` writes its row (32 bf16 given as 16 packed words) into the buffer.
-__device__ __forceinline__ void stage_row_bf16(uint32_t* buf, int lane, const uint32_t (&w)[16]) {
-#pragma unroll
-    for (int m = 0; m < 4; ++m)
-        *reinterpret_cast<uint4*>(bf16_piece(buf, lane, m)) =
-            make_uint4(w[4 * m], w[4 * m + 1], w[4 * m + 2], w[4 * m + 3]);
+// 16-byte piece m of patch row r in an epilogue buffer, in the layout of the
+// TMA box that fills / drains it: 128-byte rows with the 128-byte swizzle
+// (piece m ^ (r & 7)), or 64-byte rows with the 64-byte swizzle
+// (piece m ^ ((r >> 1) & 3)).  Either way the lanes of a warp, one row
+// each, touch distinct banks.
+template <int ROW_BYTES>
+__device__ __forceinline__ uint4* patch_piece(uint8_t* buf, int r, int m) {
+    if (ROW_BYTES == 128) return reinterpret_cast<uint4*>(buf + r * 128 + ((m ^ (r & 7)) << 4));
+    return reinterpret_cast<uint4*>(buf + r * 64 + ((m ^ ((r >> 1) & 3)) << 4));
 }
-
-__device__ __forceinline__ void read_row_bf16(const uint32_t* buf, int lane, uint32_t (&w)[16]) {
-#pragma unroll
-    for (int m = 0; m < 4; ++m) {
-        uint4 u = *reinterpret_cast<const uint4*>(bf16_piece(const_cast<uint32_t*>(buf), lane, m));
-        w[4 * m] = u.x;
-        w[4 * m + 1] = u.y;
-        w[4 * m + 2] = u.z;
-        w[4 * m + 3] = u.w;
-    }
-}
-
-// Line-wise mapping of a bf16 chunk: iteration it (0..3), lane -> row
-// 8 it + lane / 4, piece lane % 4 (16 bytes of the row's 64).
-__device__ __forceinline__ int line_row_bf16(int it, int lane) { return 8 * it + (lane >> 2); }
 
 // Wait for this thread's tcgen05.ld and tie the destination registers to the
 // wait so the compiler cannot read them earlier.
@@ -202,30 +183,40 @@ __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity,
 
 }  // namespace
 
-// tmA : FWD x, DX dz: 4-D rows map, box (64, lo_box, 1, hi_box), 128 rows.
-//       DW dz: same map shape with 64-token boxes.
-// tmB0: FWD W_self [o][k] 2-D, box (64 k, BN o)   (K-major B)
-//       DX  W_self [o][k] 2-D, box (64 k, 64 o)   (MN-major B, BN/64 boxes)
-//       DW  x 4-D rows map with 64-token boxes    (MN-major B, BN/64 boxes)
-// tmB1: FWD/DX W_nbr like tmB0; DW unused.
+// Mainloop maps:
+//   tmA : FWD x, DX dz: 4-D rows map, box (64, lo_box, 1, hi_box) = 128 rows.
+//         DW dz: the same view with 64-row boxes.
+//   tmB0: FWD W_self [o][k] 2-D, box (64 k, BN o)   (K-major B)
+//         DX  W_self [o][k] 2-D, box (64 k, 64 o)   (MN-major B, BN/64 boxes)
+//         DW  x rows, 64-row boxes                  (MN-major B, BN/64 boxes)
+//   tmB1: FWD/DX W_nbr like tmB0; DW unused.
+// Epilogue maps (32-row patches, inner box = one patch row):
+//   tmE0: FWD x / DX dy rows (residual, loaded);  DW: dW split partials [2*S*d][d] fp32
+//   tmE1: FWD y / DX dx rows (stored);             DW: dW_self [d][d] fp32
+//   tmE2: DX dz rows of the layer below (stored);  DW: dW_nbr  [d][d] fp32
 template <int MODE, int BN>
 __global__ void __launch_bounds__(kThreads, 1)
     hcw_tc_kernel(const __grid_constant__ CUtensorMap tmA,
                   const __grid_constant__ CUtensorMap tmB0,
-                  const __grid_constant__ CUtensorMap tmB1, const TcParams p) {
+                  const __grid_constant__ CUtensorMap tmB1,
+                  const __grid_constant__ CUtensorMap tmE0,
+                  const __grid_constant__ CUtensorMap tmE1,
+                  const __grid_constant__ CUtensorMap tmE2, const TcParams p) {
     constexpr int STAGES = num_stages(BN);
     constexpr int SB = stage_bytes(BN);
     constexpr int B_BYTES = BN * kBlockK * 2;
     constexpr uint32_t TMEM_COLS = 2 * BN;
     constexpr uint32_t IDESC = idesc_bf16_f32(kBlockM, BN, MODE == MODE_DW ? 1 : 0,
                                               MODE == MODE_FWD ? 0 : 1);
+    constexpr int HALF = BN / 2;                       // columns per epilogue warp
 
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-    uint8_t* epi_smem = smem + (size_t)STAGES * SB;
-    Barriers* bars =
-        reinterpret_cast<Barriers*>(epi_smem + (size_t)kEpiWarps * kEpiBufBytes);
+    uint8_t* epi_smem = smem + (size_t)STAGES * SB;               // 1024-aligned
+    float* bias_smem =
+        reinterpret_cast<float*>(epi_smem + (size_t)kEpiWarps * kEpiBufs * kEpiBufBytes);
+    Barriers* bars = reinterpret_cast<Barriers*>(bias_smem + kEpiWarps * HALF);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -242,6 +233,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&bars->tfull[a], 1);
             mbar_init(&bars->tempty[a], kEpiWarps);
         }
+        for (int e = 0; e < kEpiWarps; ++e)
+            for (int b = 0; b < kEpiBufs; ++b) mbar_init(&bars->epi_load[e][b], 1);
         mbar_init(&bars->drain, 1);
         bars->abort = 0;
         fence_mbar_init();
@@ -410,183 +403,260 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else {
         // ------------------------------------------------------------ epilogue
         // Warp e (0..7) drains TMEM lane quarter warp % 4 (rows 32 q .. 32 q + 31
-        // of the tile) and column half e / 4, in chunks of 32 columns.
+        // of the tile) and column half e / 4, in patches of 32 rows x SW columns.
         const int e = warp - 2;
         const int quarter = warp & 3;
         const int half = e >> 2;
-        constexpr int NCH = BN / 64;                  // chunks per column half
-        uint32_t* buf = reinterpret_cast<uint32_t*>(epi_smem + (size_t)e * kEpiBufBytes);
+        uint8_t* bufs = epi_smem + (size_t)e * kEpiBufs * kEpiBufBytes;
+        float* wbias = bias_smem + e * HALF;
+        uint32_t ld_phase[kEpiBufs] = {0, 0};
         int acc = 0;
         uint32_t acc_phase = 0;
-        for (int u = blockIdx.x; u < p.n_units; u += gridDim.x) {
-            // one lane waits, the warp follows its verdict (tcgen05.ld is warp-wide)
-            int ok = 1;
-            if (lane == 0) ok = mbar_wait(&bars->tfull[acc], acc_phase, abort, tmo);
-            ok = __shfl_sync(0xffffffffu, ok, 0);
-            if (!ok) break;
-            tc_fence_after();
-            const uint32_t t_base = tmem_base + ((uint32_t)(quarter * 32) << 16) +
-                                    (uint32_t)(acc * BN + half * (BN / 2));
+        bool alive = true;
+        // every lane observes the barrier; the warp proceeds only if all did
+        // (tcgen05.ld and the patch accesses are warp-wide)
+        auto wait_bar = [&](uint64_t* bar, uint32_t parity) -> bool {
+            const bool ok = mbar_wait(bar, parity, abort, tmo);
+            return __all_sync(0xffffffffu, ok) != 0;
+        };
+        auto wait_acc = [&]() -> bool {
+            const bool ok = wait_bar(&bars->tfull[acc], acc_phase);
+            if (ok) tc_fence_after();
+            return ok;
+        };
+        auto load_acc = [&](uint32_t col, uint32_t (&raw)[32]) {
+            __syncwarp();   // tcgen05.ld is .sync.aligned: the whole warp, converged
+            tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(quarter * 32) << 16) +
+                                   (uint32_t)(acc * BN + half * HALF) + col,
+                               raw);
+            tmem_ld_wait_regs(raw);
+        };
+        auto release_acc = [&]() {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&bars->tempty[acc]);
+        };
+        // make this warp's shared-memory writes visible to TMA, then store
+        auto publish = [&]() {
+            fence_proxy_async_smem();
+            __syncwarp();
+        };
+        for (int u = blockIdx.x; u < p.n_units && alive; u += gridDim.x) {
             if (MODE != MODE_DW) {
+                constexpr int SW = HALF >= 64 ? 64 : HALF;     // patch width (columns)
+                constexpr int RB = SW * 2;                     // patch row bytes
+                constexpr int NSC = HALF / SW;                 // patches per warp (<= 2)
+                constexpr int SUB = SW / 32;                   // 32-column sub-chunks per patch
+                static_assert(NSC <= kEpiBufs, "one buffer per patch");
                 const RowUnit r = decode_row_unit(p, u);
-                // tokens of this warp's 32 rows, as seen by the line-wise lanes
-                // (row 8 it + lane / 4 for it = 0..3); -1 marks rows past the end
-                long long tok_line[4];
+                const int qw = r.t * kBlockM + quarter * 32;   // first compressed row of the warp
+                const int lo_w = qw & (p.k - 1), hi_w = qw >> p.s;
+                const int q_row = qw + lane;
+                const int tok_row = q_row < p.Mh ? ((q_row >> p.s) << (p.s + 1)) +
+                                                       (r.beta << p.s) + (q_row & (p.k - 1))
+                                                 : -1;
+                const int col_half = r.j * BN + half * HALF;
+                // a patch entirely past the end (ragged tail) loads and stores nothing
+                const bool inside = qw < p.Mh;
+                const bool has_res = (p.flags & 2u) != 0 && inside;
+                const bool fwd = MODE == MODE_FWD;
+                const bool has_mprev = MODE == MODE_DX && p.mprev != nullptr;
+                const int wpr = p.d >> 5;
+                // every earlier store has finished reading the buffers: refill them
+                if (lane == 0) bulk_wait_read<0>();
+                __syncwarp();
+                if (has_res && lane == 0) {
 #pragma unroll
-                for (int it = 0; it < 4; ++it) {
-                    const int q = r.t * kBlockM + quarter * 32 + line_row_bf16(it, lane);
-                    tok_line[it] = q < p.Mh ? ((long long)(q >> p.s) << (p.s + 1)) +
-                                                  ((long long)r.beta << p.s) + (q & (p.k - 1))
-                                            : -1;
+                    for (int sc = 0; sc < NSC; ++sc) {
+                        mbar_arrive_expect_tx(&bars->epi_load[e][sc], 32 * RB);
+                        tma_load_4d(bufs + sc * kEpiBufBytes, &tmE0, &bars->epi_load[e][sc],
+                                    col_half + sc * SW, lo_w, r.beta, hi_w);
+                    }
                 }
-                const int col_half = r.j * BN + half * (BN / 2);
-                const bool has_res = (p.flags & 2u) != 0;
-                const bool has_zp = MODE == MODE_DX && p.dz_out != nullptr;
-                uint4 res_g[4], zp_g[4];
-                auto load_lines = [&](const __nv_bfloat16* src, int c, uint4 (&g)[4]) {
+                uint32_t mp[HALF / 32];
 #pragma unroll
-                    for (int it = 0; it < 4; ++it) {
-                        g[it] = make_uint4(0, 0, 0, 0);
-                        if (tok_line[it] >= 0)
-                            g[it] = __ldg(reinterpret_cast<const uint4*>(
-                                src + tok_line[it] * p.d + col_half + c * 32 + 8 * (lane & 3)));
-                    }
-                };
-                // line-wise registers -> per-row words (through the buffer)
-                auto to_rows = [&](const uint4 (&g)[4], uint32_t (&w)[16]) {
-#pragma unroll
-                    for (int it = 0; it < 4; ++it)
-                        *reinterpret_cast<uint4*>(
-                            bf16_piece(buf, line_row_bf16(it, lane), lane & 3)) = g[it];
+                for (int c = 0; c < HALF / 32; ++c)
+                    mp[c] = (has_mprev && tok_row >= 0)
+                                ? __ldg(p.mprev + (size_t)tok_row * wpr + (col_half >> 5) + c)
+                                : 0u;
+                if (fwd) {
+                    // this warp's bias slice, read back as warp-wide broadcasts
+                    for (int c = lane; c < HALF; c += 32)
+                        wbias[c] = p.bias ? __ldg(p.bias + col_half + c) : 0.f;
                     __syncwarp();
-                    read_row_bf16(buf, lane, w);
-                    __syncwarp();
-                };
-                // per-row words -> coalesced line stores (through the buffer)
-                auto store_rows = [&](__nv_bfloat16* dst, int c, const uint32_t (&w)[16]) {
-                    stage_row_bf16(buf, lane, w);
-                    __syncwarp();
-#pragma unroll
-                    for (int it = 0; it < 4; ++it) {
-                        const uint4 v = *reinterpret_cast<const uint4*>(
-                            bf16_piece(buf, line_row_bf16(it, lane), lane & 3));
-                        if (tok_line[it] >= 0)
-                            *reinterpret_cast<uint4*>(dst + tok_line[it] * p.d + col_half +
-                                                      c * 32 + 8 * (lane & 3)) = v;
-                    }
-                    __syncwarp();
-                };
-                if (has_res) load_lines(p.resid, 0, res_g);
-                if (has_zp) load_lines(p.zprev, 0, zp_g);
+                }
+                if (!wait_acc()) {
+                    alive = false;
+                    break;
+                }
+                // FWD z (layer API only): the pre-activation, row-wise stores; every
+                // lane joins the warp-wide TMEM loads, rows past the end skip the store
+                if (fwd && p.zout) {
 #pragma unroll 1
-                for (int c = 0; c < NCH; ++c) {
-                    uint32_t raw[32];
-                    tmem_ld_32x32b_x32(t_base + c * 32, raw);
-                    tmem_ld_wait_regs(raw);
-                    if (c == NCH - 1) {
-                        // the accumulator is drained: hand it back to the MMA warp
-                        tc_fence_before();
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive(&bars->tempty[acc]);
-                    }
-                    uint32_t res_w[16], zp_w[16];
-                    if (has_res) to_rows(res_g, res_w);
-                    if (has_zp) to_rows(zp_g, zp_w);
-                    if (c + 1 < NCH) {   // prefetch the next chunk's inputs
-                        if (has_res) load_lines(p.resid, c + 1, res_g);
-                        if (has_zp) load_lines(p.zprev, c + 1, zp_g);
-                    }
-                    float v[32];
+                    for (int c = 0; c < HALF / 32; ++c) {
+                        uint32_t raw[32];
+                        load_acc(c * 32, raw);
+                        if (tok_row >= 0) {
+                            uint4* dst = reinterpret_cast<uint4*>(p.zout + (size_t)tok_row * p.d +
+                                                                  col_half + c * 32);
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(raw[i]);
-                    uint32_t w[16];
-                    if (MODE == MODE_FWD) {
-                        if (p.bias) {
-                            const float4* b4 =
-                                reinterpret_cast<const float4*>(p.bias + col_half + c * 32);
+                            for (int m = 0; m < 4; ++m) {
+                                uint32_t w[4];
+#pragma unroll
+                                for (int i = 0; i < 4; ++i) {
+                                    const int e2 = 8 * m + 2 * i;
+                                    w[i] = pack_bf16x2(
+                                        __uint_as_float(raw[e2]) + wbias[c * 32 + e2],
+                                        __uint_as_float(raw[e2 + 1]) + wbias[c * 32 + e2 + 1]);
+                                }
+                                dst[m] = make_uint4(w[0], w[1], w[2], w[3]);
+                            }
+                        }
+                    }
+                }
+#pragma unroll
+                for (int sc = 0; sc < NSC; ++sc) {
+                    uint8_t* buf = bufs + sc * kEpiBufBytes;
+                    if (has_res) {
+                        const bool okl = wait_bar(&bars->epi_load[e][sc], ld_phase[sc]);
+                        ld_phase[sc] ^= 1;
+                        if (!okl) {
+                            alive = false;
+                            break;
+                        }
+                    }
+                    uint32_t gw[SUB][16];
+#pragma unroll
+                    for (int h = 0; h < SUB; ++h) {
+                        uint32_t raw[32];
+                        load_acc(sc * SW + h * 32, raw);
+                        if (sc == NSC - 1 && h == SUB - 1) release_acc();
+                        float v[32];
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(raw[i]);
+                        if (fwd) {
+                            const float4* b4 = reinterpret_cast<const float4*>(wbias + sc * SW + h * 32);
 #pragma unroll
                             for (int i = 0; i < 8; ++i) {
-                                const float4 bb = __ldg(b4 + i);
+                                const float4 bb = b4[i];
                                 v[4 * i] += bb.x;
                                 v[4 * i + 1] += bb.y;
                                 v[4 * i + 2] += bb.z;
                                 v[4 * i + 3] += bb.w;
                             }
-                        }
-                        if (p.zout) {
+                            if (p.mout) {
+                                uint32_t bits = 0;
 #pragma unroll
-                            for (int i = 0; i < 16; ++i) w[i] = pack_bf16x2(v[2 * i], v[2 * i + 1]);
-                            store_rows(p.zout, c, w);
-                        }
-                        if (p.flags & 4u) {
+                                for (int i = 0; i < 32; ++i) bits |= (v[i] > 0.f ? 1u : 0u) << i;
+                                if (tok_row >= 0)
+                                    p.mout[(size_t)tok_row * wpr + ((col_half + sc * SW) >> 5) + h] =
+                                        bits;
+                            }
+                            if (p.flags & 4u) {
 #pragma unroll
-                            for (int i = 0; i < 32; ++i) v[i] = v[i] > 0.f ? v[i] : 0.f;
+                                for (int i = 0; i < 32; ++i) v[i] = v[i] > 0.f ? v[i] : 0.f;
+                            }
+                        }
+                        if (has_res) {
+#pragma unroll
+                            for (int m = 0; m < 4; ++m) {
+                                const uint4 q4 = *patch_piece<RB>(buf, lane, 4 * h + m);
+                                const uint32_t rw[4] = {q4.x, q4.y, q4.z, q4.w};
+#pragma unroll
+                                for (int i = 0; i < 4; ++i) {
+                                    const float2 f = unpack_bf16x2(rw[i]);
+                                    v[8 * m + 2 * i] += f.x;
+                                    v[8 * m + 2 * i + 1] += f.y;
+                                }
+                            }
+                        }
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) gw[h][i] = pack_bf16x2(v[2 * i], v[2 * i + 1]);
+                    }
+                    // the patch: y (FWD) or dx (DX), written over the residual rows
+                    if (p.out) {
+#pragma unroll
+                        for (int h = 0; h < SUB; ++h)
+#pragma unroll
+                            for (int m = 0; m < 4; ++m)
+                                *patch_piece<RB>(buf, lane, 4 * h + m) =
+                                    make_uint4(gw[h][4 * m], gw[h][4 * m + 1], gw[h][4 * m + 2],
+                                               gw[h][4 * m + 3]);
+                        publish();
+                        if (lane == 0 && inside) {
+                            tma_store_4d(&tmE1, buf, col_half + sc * SW, lo_w, r.beta, hi_w);
+                            bulk_commit();
                         }
                     }
-                    if (has_res) {
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) {
-                            const float2 f = unpack_bf16x2(res_w[i]);
-                            v[2 * i] += f.x;
-                            v[2 * i + 1] += f.y;
+                    if (has_mprev) {
+                        // fused ReLU gradient of the layer below: dz = dx * mask
+                        if (p.out) {
+                            if (lane == 0) bulk_wait_read<0>();
+                            __syncwarp();
                         }
-                    }
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) w[i] = pack_bf16x2(v[2 * i], v[2 * i + 1]);
-                    if (p.out) store_rows(p.out, c, w);
-                    if (has_zp) {
-                        // fused ReLU gradient of the layer below: dz = g * (z > 0)
+                        for (int h = 0; h < SUB; ++h) {
+                            const uint32_t mw = mp[(sc * SW >> 5) + h];
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) {
-                            const float2 zz = unpack_bf16x2(zp_w[i]);
-                            const uint32_t lo = zz.x > 0.f ? (w[i] & 0xFFFFu) : 0u;
-                            const uint32_t hi = zz.y > 0.f ? (w[i] & 0xFFFF0000u) : 0u;
-                            w[i] = lo | hi;
+                            for (int m = 0; m < 4; ++m) {
+                                uint32_t w4[4];
+#pragma unroll
+                                for (int i = 0; i < 4; ++i) {
+                                    const int b = 8 * m + 2 * i;
+                                    const uint32_t keep = ((mw >> b) & 1u ? 0x0000FFFFu : 0u) |
+                                                          ((mw >> (b + 1)) & 1u ? 0xFFFF0000u : 0u);
+                                    w4[i] = gw[h][4 * m + i] & keep;
+                                }
+                                *patch_piece<RB>(buf, lane, 4 * h + m) =
+                                    make_uint4(w4[0], w4[1], w4[2], w4[3]);
+                            }
                         }
-                        store_rows(p.dz_out, c, w);
+                        publish();
+                        if (lane == 0 && inside) {
+                            tma_store_4d(&tmE2, buf, col_half + sc * SW, lo_w, r.beta, hi_w);
+                            bulk_commit();
+                        }
                     }
                 }
             } else {
                 const WUnit w = decode_w_unit(p, u);
+                if (!wait_acc()) {
+                    alive = false;
+                    break;
+                }
                 const int S = w.which ? p.splits_nbr : p.splits_self;
-                float* dst_base;
-                if (S == 1)
-                    dst_base = w.which ? p.dw_nbr : p.dw_self;
-                else
-                    dst_base = p.dw_partial + ((size_t)w.which * p.splits_max + w.split) *
-                                                  (size_t)p.d * p.d;
-                const int o0 = w.ot * kBlockM + quarter * 32;
-                const int col_half = w.nt * BN + half * (BN / 2);
+                const CUtensorMap* map = S > 1 ? &tmE0 : (w.which ? &tmE2 : &tmE1);
+                const int row0 = (S > 1 ? (w.which * p.splits_max + w.split) * p.d : 0) +
+                                 w.ot * kBlockM + quarter * 32;
+                const int col_half = w.nt * BN + half * HALF;
 #pragma unroll 1
-                for (int c = 0; c < NCH; ++c) {
+                for (int c = 0; c < HALF / 32; ++c) {
+                    uint8_t* buf = bufs + (c & 1) * kEpiBufBytes;
                     uint32_t raw[32];
-                    tmem_ld_32x32b_x32(t_base + c * 32, raw);
-                    tmem_ld_wait_regs(raw);
-                    if (c == NCH - 1) {
-                        tc_fence_before();
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive(&bars->tempty[acc]);
-                    }
+                    load_acc(c * 32, raw);
+                    if (c == HALF / 32 - 1) release_acc();
+                    // the buffer's previous store (two chunks ago) must have been read
+                    if (lane == 0) bulk_wait_read<1>();
+                    __syncwarp();
 #pragma unroll
                     for (int m = 0; m < 8; ++m)
-                        *reinterpret_cast<uint4*>(f32_piece(buf, lane, m)) =
+                        *patch_piece<128>(buf, lane, m) =
                             make_uint4(raw[4 * m], raw[4 * m + 1], raw[4 * m + 2], raw[4 * m + 3]);
-                    __syncwarp();
-#pragma unroll
-                    for (int it = 0; it < 8; ++it) {
-                        const int rr = 4 * it + (lane >> 3);
-                        const uint4 v =
-                            *reinterpret_cast<const uint4*>(f32_piece(buf, rr, lane & 7));
-                        if (o0 + rr < p.d)
-                            *reinterpret_cast<uint4*>(dst_base + (size_t)(o0 + rr) * p.d +
-                                                      col_half + c * 32 + 4 * (lane & 7)) = v;
+                    publish();
+                    // d is a multiple of 64, so a warp's 32 rows are all inside or all
+                    // past the end (ragged o tile); the latter are not stored
+                    if (lane == 0 && w.ot * kBlockM + quarter * 32 < p.d) {
+                        tma_store_2d(map, buf, col_half + c * 32, row0);
+                        bulk_commit();
                     }
-                    __syncwarp();
                 }
             }
             acc ^= 1;
             if (acc == 0) acc_phase ^= 1;
         }
+        // every store of this warp has landed before the CTA exits
+        if (lane == 0) bulk_wait<0>();
+        __syncwarp();
     }
 
     tc_fence_before();
@@ -599,21 +669,31 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 template <int MODE, int BN>
-static cudaError_t launch_one(const CUtensorMap& a, const CUtensorMap& b0, const CUtensorMap& b1,
-                              const TcParams& p, int grid, cudaStream_t st) {
+static cudaError_t launch_one(const CUtensorMap* maps, const TcParams& p, int grid,
+                              cudaStream_t st) {
     constexpr size_t smem = smem_total<BN>();
+    static_assert(smem <= 232448, "shared memory budget");
     auto kern = hcw_tc_kernel<MODE, BN>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)smem);
+    // the shared-memory opt-in is a per-device function attribute: set it once per device
+    static std::atomic<uint64_t> configured[4] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    kern<<<grid, kThreads, smem, st>>>(a, b0, b1, p);
+    const uint64_t bit = 1ull << (dev & 63);
+    std::atomic<uint64_t>& word = configured[(dev >> 6) & 3];
+    if (dev >= 256 || !(word.load(std::memory_order_acquire) & bit)) {
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        if (dev < 256) word.fetch_or(bit, std::memory_order_acq_rel);
+    }
+    kern<<<grid, kThreads, smem, st>>>(maps[0], maps[1], maps[2], maps[3], maps[4], maps[5], p);
     return cudaGetLastError();
 }
 
-cudaError_t launch_tc(int mode, int BN, const CUtensorMap& a, const CUtensorMap& b0,
-                      const CUtensorMap& b1, const TcParams& p, int grid, cudaStream_t st) {
+cudaError_t launch_tc(int mode, int BN, const CUtensorMap* maps, const TcParams& p, int grid,
+                      cudaStream_t st) {
 #define HCW_TC_CASE(M, N) \
-    if (mode == M && BN == N) return launch_one<M, N>(a, b0, b1, p, grid, st);
+    if (mode == M && BN == N) return launch_one<M, N>(maps, p, grid, st);
     HCW_TC_CASE(MODE_FWD, 256)
     HCW_TC_CASE(MODE_FWD, 128)
     HCW_TC_CASE(MODE_FWD, 64)

@@ -243,28 +243,32 @@ def hcw_launch_count() -> int:
 
 
 def hcw_stack_fwd(x, W_self, W_nbr, bias=None, layer0: int = 0, dim_override: int = -1,
-                  flags: int = 0, y=None, acts=None, zs=None, want_z: bool = False,
+                  flags: int = 0, y=None, acts=None, masks=None, want_masks: bool = None,
                   stream=None):
-    """Stack forward over L = W_self.shape[0] layers; returns (y, acts, zs)."""
-    _dev(x, W_self, W_nbr, bias, y, acts, zs)
+    """Stack forward over L = W_self.shape[0] layers; returns (y, acts, masks).
+    masks (ReLU only) are int32 words [L, B, n, ceil(d/32)], bit o%32 of word
+    o/32 = (z > 0); allocated when the stack uses ReLU unless want_masks=False."""
+    _dev(x, W_self, W_nbr, bias, y, acts, masks)
     B, n, d = x.shape
     L = W_self.shape[0]
     y = torch.empty_like(x) if y is None else y
     if acts is None and L > 1:
         acts = torch.empty((L - 1, B, n, d), dtype=x.dtype, device=x.device)
-    if zs is None and want_z:
-        zs = torch.empty((L, B, n, d), dtype=x.dtype, device=x.device)
+    if want_masks is None:
+        want_masks = bool(flags & HCW_ACT_RELU)
+    if masks is None and want_masks:
+        masks = torch.empty((L, B, n, (d + 31) // 32), dtype=torch.int32, device=x.device)
     _check(lib().hcw_stack_fwd(_ptr(x), _ptr(W_self), _ptr(W_nbr), _ptr(bias), layer0, L,
                                dim_override, B, n, d, _dtype_code(x), flags, _ptr(y),
-                               _ptr(acts), _ptr(zs), _stream(stream)), "hcw_stack_fwd")
-    return y, acts, zs
+                               _ptr(acts), _ptr(masks), _stream(stream)), "hcw_stack_fwd")
+    return y, acts, masks
 
 
-def hcw_stack_bwd(x, acts, zs, dy, W_self, W_nbr, layer0: int = 0, dim_override: int = -1,
+def hcw_stack_bwd(x, acts, masks, dy, W_self, W_nbr, layer0: int = 0, dim_override: int = -1,
                   flags: int = 0, dx=None, dW_self=None, dW_nbr=None, dbias=None,
                   want_dbias: bool = True, workspace=None, stream=None):
     """Stack backward; returns (dx, dW_self[L], dW_nbr[L], dbias[L])."""
-    _dev(x, acts, zs, dy, W_self, W_nbr, dx, dW_self, dW_nbr, dbias, workspace)
+    _dev(x, acts, masks, dy, W_self, W_nbr, dx, dW_self, dW_nbr, dbias, workspace)
     B, n, d = x.shape
     L = W_self.shape[0]
     dt = _dtype_code(x)
@@ -276,7 +280,7 @@ def hcw_stack_bwd(x, acts, zs, dy, W_self, W_nbr, layer0: int = 0, dim_override:
         dbias = torch.empty(L, d, **f32)
     need = hcw_stack_workspace_bytes(B, n, d, dt, flags)
     ws = _workspace(need, x.device, workspace)
-    _check(lib().hcw_stack_bwd(_ptr(x), _ptr(acts), _ptr(zs), _ptr(dy), _ptr(W_self),
+    _check(lib().hcw_stack_bwd(_ptr(x), _ptr(acts), _ptr(masks), _ptr(dy), _ptr(W_self),
                                _ptr(W_nbr), layer0, L, dim_override, B, n, d, dt, flags,
                                _ptr(dx), _ptr(dW_self), _ptr(dW_nbr), _ptr(dbias), _ptr(ws),
                                ws.numel(), _stream(stream)), "hcw_stack_bwd")

@@ -49,6 +49,18 @@ def host(t):
     return t.float().cpu().double().numpy()
 
 
+def masks_from_z(z):
+    """ReLU masks in the stack's format from pre-activations z [..., d]:
+    int32 words [..., ceil(d/32)], bit o % 32 of word o // 32 = (z[..., o] > 0)."""
+    z = np.asarray(z)
+    d = z.shape[-1]
+    wpr = (d + 31) // 32
+    bits = np.zeros(z.shape[:-1] + (wpr * 32,), dtype=np.uint64)
+    bits[..., :d] = z > 0
+    words = (bits.reshape(z.shape[:-1] + (wpr, 32)) << np.arange(32, dtype=np.uint64)).sum(-1)
+    return torch.from_numpy(words.astype(np.uint32).view(np.int32))
+
+
 # ---------------------------------------------------------------- index code
 
 @pytest.mark.parametrize("n", [2, 8, 64, 256, 65536])
@@ -126,6 +138,32 @@ def test_layer_backward(H, case, flags):
     assert rel(host(gb), rb_) <= (1e-5 if not rb else 1e-4)
 
 
+@pytest.mark.parametrize("flags", [CAUSAL | RESIDUAL | RELU, RESIDUAL])
+def test_many_tiles_per_cta(H, flags):
+    """B = 256 sequences of n = 256 at d = 512 give 1024 forward / input-gradient
+    tiles, several per persistent CTA: every TMEM accumulator is reused, which
+    the smaller cases never do.  Checked on sampled sequences against the oracle."""
+    B, n, d, layer = 256, 256, 512, 6
+    pr = synth.problem(B, n, d, L=1, seed=21, w_std=(1 / (2 * d)) ** 0.5)
+    x, x64 = dev(pr.x, torch.bfloat16)
+    Ws, Ws64 = dev(pr.W_self[0], torch.bfloat16)
+    Wn, Wn64 = dev(pr.W_nbr[0], torch.bfloat16)
+    dy, dy64 = dev(pr.dy, torch.bfloat16)
+    z, z64 = dev(pr.z[0], torch.bfloat16)
+    bias = torch.from_numpy(pr.bias[0]).cuda()
+    y, zs = H.hcw_layer_fwd(x, Ws, Wn, bias, layer, -1, flags, want_z=True)
+    dx = H.hcw_layer_bwd_data(dy, dy, Ws, Wn, layer, -1, flags)
+    assert H.hcw_sync_status() == H.HCW_OK
+    picks = [0, 77, 128, 255]
+    yr, zr = O.layer_fwd(x64[picks], Ws64, Wn64, pr.bias[0].astype(np.float64), layer, -1, flags,
+                         round_bf16=True, want_z=True)
+    assert rel(host(y)[picks], yr) <= TOL_BF16
+    assert rel(host(zs)[picks], zr) <= TOL_BF16
+    rdx, _, _, _ = O.layer_bwd(x64[picks], z64[picks], dy64[picks], Ws64, Wn64, layer, -1,
+                               flags & ~RELU, round_bf16=True)
+    assert rel(host(dx)[picks], rdx) <= TOL_BF16
+
+
 def test_backward_is_deterministic(H):
     pr = synth.problem(8, 256, 512, L=1, seed=3)
     x, _ = dev(pr.x, torch.bfloat16)
@@ -163,13 +201,13 @@ def run_stack(H, pr, dtype, L, flags, layer0=0, dim=-1):
     Wn, Wn64 = dev(pr.W_nbr, dtype)
     bias = torch.from_numpy(pr.bias).cuda()
     dy, dy64 = dev(pr.dy, dtype)
-    y, acts, zs = H.hcw_stack_fwd(x, Ws, Wn, bias, layer0, dim, flags, want_z=True)
+    y, acts, masks = H.hcw_stack_fwd(x, Ws, Wn, bias, layer0, dim, flags)
     rb = dtype == torch.bfloat16
     ry, racts, rzs = O.stack_fwd(x64, Ws64, Wn64, pr.bias.astype(np.float64), layer0, L, dim,
                                  flags, round_bf16=rb)
     o_acts = torch.from_numpy(racts[1:]).to(dtype).cuda() if L > 1 else None
-    o_zs = torch.from_numpy(rzs).to(dtype).cuda()
-    dx, gWs, gWn, gb = H.hcw_stack_bwd(x, o_acts, o_zs, dy, Ws, Wn, layer0, dim, flags)
+    o_masks = masks_from_z(rzs).cuda() if flags & RELU else None
+    dx, gWs, gWn, gb = H.hcw_stack_bwd(x, o_acts, o_masks, dy, Ws, Wn, layer0, dim, flags)
     torch.cuda.synchronize()
     rdx, rWs, rWn, rgb = O.stack_bwd(racts, rzs, dy64, Ws64, Wn64, layer0, L, dim, flags,
                                      round_bf16=rb)
@@ -245,14 +283,14 @@ def test_charlm_w256_full_launch_sampled(H):
     Wn, Wn64 = dev(pr.W_nbr, torch.bfloat16)
     bias = torch.from_numpy(pr.bias).cuda()
     dy, dy64 = dev(pr.dy, torch.bfloat16)
-    y, acts, zs = H.hcw_stack_fwd(x, Ws, Wn, bias, 0, -1, flags, want_z=True)
+    y, acts, masks = H.hcw_stack_fwd(x, Ws, Wn, bias, 0, -1, flags)
     ry, racts, rzs = O.stack_fwd(x64[picks], Ws64, Wn64, pr.bias.astype(np.float64), 0, L, -1,
                                  flags, round_bf16=True)
     assert rel(host(y)[picks], ry) <= TOL_BF16
     assert rel(host(acts)[:, picks], racts[1:]) <= TOL_BF16
     acts[:, picks] = torch.from_numpy(racts[1:]).to(torch.bfloat16).cuda()
-    zs[:, picks] = torch.from_numpy(rzs).to(torch.bfloat16).cuda()
-    dx, gWs, gWn, gb = H.hcw_stack_bwd(x, acts, zs, dy, Ws, Wn, 0, -1, flags)
+    masks[:, picks] = masks_from_z(rzs).cuda()
+    dx, gWs, gWn, gb = H.hcw_stack_bwd(x, acts, masks, dy, Ws, Wn, 0, -1, flags)
     torch.cuda.synchronize()
     rdx, rWs, rWn, rgb = O.stack_bwd(racts, rzs, dy64[picks], Ws64, Wn64, 0, L, -1, flags,
                                      round_bf16=True)
@@ -266,24 +304,34 @@ def test_charlm_w256_full_launch_sampled(H):
 
 
 def test_stack_backward_is_the_chain_of_layer_backwards(H):
-    """hcw_stack_bwd on its own saved activations equals hcw_layer_bwd applied
-    layer by layer from the top (bit-exact): the stack plumbing adds nothing."""
-    flags = CAUSAL | RESIDUAL | RELU
-    B, n, d, L = 4, 256, 512, 5
-    pr = synth.problem(B, n, d, L=L, seed=4, w_std=(1 / (2 * d)) ** 0.5)
-    x, _ = dev(pr.x, torch.bfloat16)
-    Ws, _ = dev(pr.W_self, torch.bfloat16)
-    Wn, _ = dev(pr.W_nbr, torch.bfloat16)
-    dy, _ = dev(pr.dy, torch.bfloat16)
-    bias = torch.from_numpy(pr.bias).cuda()
-    y, acts, zs = H.hcw_stack_fwd(x, Ws, Wn, bias, 3, -1, flags, want_z=True)
-    dx, gWs, gWn, gb = H.hcw_stack_bwd(x, acts, zs, dy, Ws, Wn, 3, -1, flags)
-    g = dy
-    for l in range(L - 1, -1, -1):
-        inp = x if l == 0 else acts[l - 1]
-        g, a, b, c = H.hcw_layer_bwd(inp, zs[l], g, Ws[l], Wn[l], 3 + l, -1, flags)
-        assert torch.equal(a, gWs[l]) and torch.equal(b, gWn[l]) and torch.equal(c, gb[l])
-    assert torch.equal(g, dx)
+    """The stack's forward equals hcw_layer_fwd layer by layer and its ReLU masks
+    are exactly (z > 0) of those layers; hcw_stack_bwd on its own saved state
+    equals hcw_layer_bwd applied layer by layer from the top (all bit-exact):
+    the stack plumbing and the fused ReLU gradient add nothing."""
+    for flags in (CAUSAL | RESIDUAL | RELU, CAUSAL | RELU, RESIDUAL):
+        B, n, d, L = 4, 256, 512, 5
+        pr = synth.problem(B, n, d, L=L, seed=4, w_std=(1 / (2 * d)) ** 0.5)
+        x, _ = dev(pr.x, torch.bfloat16)
+        Ws, _ = dev(pr.W_self, torch.bfloat16)
+        Wn, _ = dev(pr.W_nbr, torch.bfloat16)
+        dy, _ = dev(pr.dy, torch.bfloat16)
+        bias = torch.from_numpy(pr.bias).cuda()
+        y, acts, masks = H.hcw_stack_fwd(x, Ws, Wn, bias, 3, -1, flags)
+        dx, gWs, gWn, gb = H.hcw_stack_bwd(x, acts, masks, dy, Ws, Wn, 3, -1, flags)
+        inp, zs = x, []
+        for l in range(L):
+            out, z = H.hcw_layer_fwd(inp, Ws[l], Wn[l], bias[l], 3 + l, -1, flags, want_z=True)
+            assert torch.equal(out, acts[l] if l < L - 1 else y)
+            if flags & RELU:
+                assert torch.equal(masks_from_z(host(z)).cuda(), masks[l])
+            zs.append(z)
+            inp = out
+        g = dy
+        for l in range(L - 1, -1, -1):
+            inp = x if l == 0 else acts[l - 1]
+            g, a, b, c = H.hcw_layer_bwd(inp, zs[l], g, Ws[l], Wn[l], 3 + l, -1, flags)
+            assert torch.equal(a, gWs[l]) and torch.equal(b, gWn[l]) and torch.equal(c, gb[l])
+        assert torch.equal(g, dx)
 
 
 def test_split_backward_matches_fused(H):
