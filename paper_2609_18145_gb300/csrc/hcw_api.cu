@@ -7,6 +7,7 @@
 
 #include <atomic>
 #include <mutex>
+#include <vector>
 
 #include "hcw.h"
 #include "hcw_internal.h"
@@ -16,6 +17,7 @@ namespace {
 
 constexpr unsigned kAllFlags = HCW_CAUSAL | HCW_RESIDUAL | HCW_ACT_RELU;
 constexpr unsigned long long kDefaultTimeoutNs = 2000000000ull;   // 2 s per wait
+constexpr int kStackSlots = 3;   // pre-activation-gradient slots of the stack backward
 
 int log2_exact(long long n) {
     if (n < 2 || (n & (n - 1))) return -1;
@@ -222,6 +224,37 @@ int cuda_status(cudaError_t e) { return e == cudaSuccess ? HCW_OK : HCW_ERR_CUDA
 int launched(cudaError_t e, int kernels) {
     if (e != cudaSuccess) return HCW_ERR_CUDA;
     g_launches.fetch_add((unsigned long long)kernels, std::memory_order_relaxed);
+    return HCW_OK;
+}
+
+// ------------------------------------------------------------ side stream
+// hcw_stack_bwd runs the weight gradients on a second stream, forked from and
+// joined back to the caller's stream with events, so that they fill the SMs
+// the input-gradient chain leaves idle.  One side stream and an event pool per
+// device, created on first use and kept for the process; the enqueue sequence
+// is serialised across host threads because the events are shared.
+struct SideStream {
+    cudaStream_t stream = nullptr;
+    std::vector<cudaEvent_t> events;
+};
+std::mutex g_side_mu;
+SideStream g_side[64];
+
+// Called with g_side_mu held.  Returns HCW_OK and the device's side stream with
+// at least n events.
+int side_stream(int n, SideStream** out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return HCW_ERR_CUDA;
+    if (dev < 0 || dev >= 64) return HCW_ERR_UNSUPPORTED;
+    SideStream& ss = g_side[dev];
+    if (!ss.stream && cudaStreamCreateWithFlags(&ss.stream, cudaStreamNonBlocking) != cudaSuccess)
+        return HCW_ERR_CUDA;
+    while ((int)ss.events.size() < n) {
+        cudaEvent_t e;
+        if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return HCW_ERR_CUDA;
+        ss.events.push_back(e);
+    }
+    *out = &ss;
     return HCW_OK;
 }
 
@@ -673,9 +706,12 @@ int hcw_stack_fwd(const void* x, const void* W_self, const void* W_nbr, const fl
 size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags) {
     Shape sh;
     if (check_shape(0, -1, B, n, d, dtype, flags, &sh)) return 0;
-    // two output-gradient buffers, two pre-activation-gradient buffers, and
-    // the weight-gradient workspace of one layer
-    return ws_layout(sh.tokens, d, dtype, flags).w_bytes + 4 * align256(sh.act_bytes);
+    // two output-gradient buffers, kStackSlots pre-activation-gradient slots
+    // (rotated so that a weight gradient on the side stream keeps its input
+    // while the input-gradient chain moves on), and the weight-gradient
+    // workspace the side stream reuses layer after layer
+    return ws_layout(sh.tokens, d, dtype, flags).w_bytes +
+           (2 + kStackSlots) * align256(sh.act_bytes);
 }
 
 int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void* dy,
@@ -717,66 +753,95 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void
     cudaStream_t st = (cudaStream_t)stream;
     uint8_t* wsb = static_cast<uint8_t*>(workspace);
     const size_t ab256 = align256(ab);
-    uint8_t* g[2] = {wsb, wsb + ab256};                    // output gradients
-    uint8_t* gz[2] = {wsb + 2 * ab256, wsb + 3 * ab256};   // pre-activation gradients
-    uint8_t* wws = wsb + 4 * ab256;                        // weight-gradient workspace
+    uint8_t* g[2] = {wsb, wsb + ab256};     // output gradients (residual terms)
+    uint8_t* slot[kStackSlots];             // pre-activation gradients dz_m in slot m % 3
+    for (int i = 0; i < kStackSlots; ++i) slot[i] = wsb + (2 + i) * ab256;
+    uint8_t* wws = wsb + (2 + kStackSlots) * ab256;   // weight-gradient workspace
     auto act_ptr = [&](int l) { return static_cast<const uint8_t*>(acts) + (size_t)l * ab; };
     auto mask_ptr = [&](int l) {
         return reinterpret_cast<const uint32_t*>(static_cast<const uint8_t*>(masks) +
                                                  (size_t)l * mb);
     };
+    std::lock_guard<std::mutex> lock(g_side_mu);
+    SideStream* ss = nullptr;
+    rc = side_stream(2 * L + 1, &ss);
+    if (rc) return rc;
+    cudaEvent_t* ev_ready = ss->events.data();       // dz_l written (main stream)
+    cudaEvent_t* ev_done = ev_ready + L;             // weight gradient of layer l done (side)
+    cudaEvent_t ev_fork = ev_ready[2 * L];
+    cudaStream_t side = ss->stream;
+    auto cu = [](cudaError_t e) { return e == cudaSuccess ? (int)HCW_OK : (int)HCW_ERR_CUDA; };
+    // the side stream starts after everything the caller queued before this call
+    if ((rc = cu(cudaEventRecord(ev_fork, st)))) return rc;
+    if ((rc = cu(cudaStreamWaitEvent(side, ev_fork, 0)))) return rc;
     // gradient at the output (cur_g) and at the pre-activation (cur_dz) of layer l
     const void* cur_g = dy;
     const void* cur_dz = dy;
     if (relu) {
+        void* dz_top = slot[(L - 1) % kStackSlots];
         rc = launched(dtype == HCW_BF16
                           ? launch_relu_grad_mask_bf16(static_cast<const __nv_bfloat16*>(dy),
                                                        mask_ptr(L - 1),
-                                                       reinterpret_cast<__nv_bfloat16*>(gz[(L - 1) & 1]),
+                                                       static_cast<__nv_bfloat16*>(dz_top),
                                                        sh.tokens, d, st)
                           : launch_relu_grad_mask_f32(static_cast<const float*>(dy), mask_ptr(L - 1),
-                                                      reinterpret_cast<float*>(gz[(L - 1) & 1]),
-                                                      sh.tokens, d, st),
+                                                      static_cast<float*>(dz_top), sh.tokens, d, st),
                       1);
         if (rc) return rc;
-        cur_dz = gz[(L - 1) & 1];
+        cur_dz = dz_top;
     }
+    if ((rc = cu(cudaEventRecord(ev_ready[L - 1], st)))) return rc;
     for (int l = L - 1; l >= 0; --l) {
         Shape shl = sh;
         shl.s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
         const void* in = l == 0 ? x : act_ptr(l - 1);
         const void* Wsl = static_cast<const uint8_t*>(W_self) + l * wb;
         const void* Wnl = static_cast<const uint8_t*>(W_nbr) + l * wb;
-        void* out_g = l == 0 ? dx : ((resid || !relu) ? (void*)g[l & 1] : nullptr);
-        void* next_dz = nullptr;
-        if (l > 0 && relu) {
-            next_dz = gz[(l - 1) & 1];
-            if (dtype == HCW_BF16) {
-                // the input-gradient kernel also applies the ReLU gradient of layer l-1
-                rc = dx_bf16(shl, cur_dz, cur_g, Wsl, Wnl, flags, out_g, st, mask_ptr(l - 1),
-                             next_dz);
-            } else {
-                out_g = g[l & 1];
-                rc = layer_dx_impl(shl, dtype, cur_dz, cur_g, Wsl, Wnl, flags, out_g, st);
-                if (!rc)
-                    rc = launched(launch_relu_grad_mask_f32(static_cast<const float*>(out_g),
-                                                            mask_ptr(l - 1),
-                                                            static_cast<float*>(next_dz),
-                                                            sh.tokens, d, st),
-                                  1);
-            }
-        } else {
-            rc = layer_dx_impl(shl, dtype, cur_dz, cur_g, Wsl, Wnl, flags, out_g, st);
-        }
-        if (rc) return rc;
+        // weight gradient of layer l on the side stream, once dz_l exists
+        if ((rc = cu(cudaStreamWaitEvent(side, ev_ready[l], 0)))) return rc;
         rc = layer_dw_impl(shl, dtype, in, cur_dz, flags, dW_self + (size_t)l * d * d,
                            dW_nbr + (size_t)l * d * d, dbias ? dbias + (size_t)l * d : nullptr,
-                           wws, st);
+                           wws, side);
         if (rc) return rc;
+        if ((rc = cu(cudaEventRecord(ev_done[l], side)))) return rc;
+        // input gradient of layer l on the caller's stream
+        if (l == 0) {
+            rc = layer_dx_impl(shl, dtype, cur_dz, cur_g, Wsl, Wnl, flags, dx, st);
+            if (rc) return rc;
+            break;
+        }
+        // dz_{l-1} goes to slot (l-1) % 3, last used by dz_{l+2}: its weight
+        // gradient must be done with it
+        uint8_t* dst = slot[(l - 1) % kStackSlots];
+        if (l + 2 <= L - 1 && (rc = cu(cudaStreamWaitEvent(st, ev_done[l + 2], 0)))) return rc;
+        void* out_g;
+        void* next_dz;
+        if (!relu) {
+            out_g = dst;       // without an activation dz = g
+            next_dz = dst;
+            rc = layer_dx_impl(shl, dtype, cur_dz, cur_g, Wsl, Wnl, flags, out_g, st);
+        } else if (dtype == HCW_BF16) {
+            // the input-gradient kernel also applies the ReLU gradient of layer l-1
+            out_g = resid ? (void*)g[l & 1] : nullptr;
+            next_dz = dst;
+            rc = dx_bf16(shl, cur_dz, cur_g, Wsl, Wnl, flags, out_g, st, mask_ptr(l - 1), next_dz);
+        } else {
+            out_g = g[l & 1];
+            next_dz = dst;
+            rc = layer_dx_impl(shl, dtype, cur_dz, cur_g, Wsl, Wnl, flags, out_g, st);
+            if (!rc)
+                rc = launched(launch_relu_grad_mask_f32(static_cast<const float*>(out_g),
+                                                        mask_ptr(l - 1), static_cast<float*>(next_dz),
+                                                        sh.tokens, d, st),
+                              1);
+        }
+        if (rc) return rc;
+        if ((rc = cu(cudaEventRecord(ev_ready[l - 1], st)))) return rc;
         cur_g = out_g;
-        cur_dz = relu ? next_dz : out_g;
+        cur_dz = next_dz;
     }
-    return HCW_OK;
+    // join: the caller's stream waits for the last weight gradient
+    return cu(cudaStreamWaitEvent(st, ev_done[0], 0));
 }
 
 unsigned long long hcw_launch_count(void) { return g_launches.load(); }
