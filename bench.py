@@ -270,11 +270,14 @@ def run_ours(args):
     gb = torch.empty((L, d), dtype=torch.float32, device=dev)
     ws = torch.empty(H.hcw_stack_workspace_bytes(B, n, d, H.HCW_BF16, flags), dtype=torch.uint8,
                      device=dev)
+    fws = torch.empty(max(1, H.hcw_stack_fwd_workspace_bytes(B, n, d, H.HCW_BF16, flags, L)),
+                      dtype=torch.uint8, device=dev)
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
 
     def step_calls(xin, dyin):
-        H.hcw_stack_fwd(xin, Ws, Wn, bias, 0, -1, flags, y=y, acts=acts, masks=masks)
+        H.hcw_stack_fwd(xin, Ws, Wn, bias, 0, -1, flags, y=y, acts=acts, masks=masks,
+                        workspace=fws)
         H.hcw_stack_bwd(xin, acts, masks, dyin, Ws, Wn, 0, -1, flags, dx=dx, dW_self=gWs,
                         dW_nbr=gWn, dbias=gb, workspace=ws)
 
@@ -349,7 +352,7 @@ def run_ours(args):
     dz = dy   # a layer's pre-activation gradient has the activations' shape and scale
     fwd_ms = time_calls(lambda i: H.hcw_stack_fwd(x, Ws[i % L:i % L + 1], Wn[i % L:i % L + 1],
                                                   bias[i % L:i % L + 1], i % L, -1, flags, y=y,
-                                                  masks=masks[:1]), 2 * L)
+                                                  masks=masks[:1], workspace=fws), 2 * L)
     dx_ms = time_calls(lambda i: H.hcw_layer_bwd_data(dz, dy, Ws[i % L], Wn[i % L], i % L, -1,
                                                       flags, dx=dx), 2 * L)
     wws = torch.empty(H.hcw_layer_bwd_weight_workspace_bytes(B, n, d, H.HCW_BF16, flags),
@@ -357,6 +360,12 @@ def run_ours(args):
     dw_ms = time_calls(lambda i: H.hcw_layer_bwd_weight(x, dz, i % L, -1, flags,
                                                         dW_self=gWs[0], dW_nbr=gWn[0],
                                                         want_dbias=False, workspace=wws), 2 * L)
+    # the two halves of the step as the step runs them
+    stack_fwd_ms = time_calls(lambda i: H.hcw_stack_fwd(x, Ws, Wn, bias, 0, -1, flags, y=y,
+                                                        acts=acts, masks=masks, workspace=fws), 3)
+    stack_bwd_ms = time_calls(lambda i: H.hcw_stack_bwd(x, acts, masks, dy, Ws, Wn, 0, -1, flags,
+                                                        dx=dx, dW_self=gWs, dW_nbr=gWn, dbias=gb,
+                                                        workspace=ws), 3)
     layer_flops = 3.0 * d * d * tokens          # per kernel launch (causal)
     kernels = {"hcw_tc_kernel<FWD,256>": fwd_ms, "hcw_tc_kernel<DX,256>": dx_ms,
                "dW (hcw_tc_kernel<DW,256> + split reduce)": dw_ms}
@@ -429,7 +438,8 @@ def run_ours(args):
                          "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                          "traffic": traffic, "peak_source": peak_src + " bf16 burst",
                          "flops_per_launch": layer_flops, "avg_launch_ms": dom_ms,
-                         "kernel_ms": kernels},
+                         "kernel_ms": kernels, "stack_fwd_ms": stack_fwd_ms,
+                         "stack_bwd_ms": stack_bwd_ms},
             "step_roofline": {"achieved": step_tflops, "peak": peak_sus, "unit": "TFLOP/s",
                               "frac": step_tflops / peak_sus,
                               "peak_source": peak_src + " bf16 sustained",

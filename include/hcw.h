@@ -166,10 +166,19 @@ int hcw_layer_bwd_weight(const void* x, const void* dz, int layer, int dim_overr
  *          one bit per activation that the ReLU backward needs (d/8 bytes
  *          per token instead of the pre-activation itself); may be NULL
  *          when no backward follows.  Ignored without HCW_ACT_RELU.
+ *   workspace/ws_bytes  at least hcw_stack_fwd_workspace_bytes(...) bytes of
+ *          device scratch (NULL allowed when that is 0).
+ * bf16: runs of up to 16 layers go in one persistent launch; a tile of
+ * layer l starts as soon as the rows it reads (its own and its partners')
+ * have been written by layer l-1, tracked per 128-token chunk.
  */
 int hcw_stack_fwd(const void* x, const void* W_self, const void* W_nbr, const float* bias,
                   int layer0, int L, int dim_override, int B, int n, int d, int dtype,
-                  unsigned flags, void* y, void* acts, void* masks, void* stream);
+                  unsigned flags, void* y, void* acts, void* masks, void* workspace,
+                  size_t ws_bytes, void* stream);
+
+/* Workspace bytes hcw_stack_fwd needs for these sizes and L layers (0 is possible). */
+size_t hcw_stack_fwd_workspace_bytes(int B, int n, int d, int dtype, unsigned flags, int L);
 
 /*
  * Backward of hcw_stack_fwd, layers L-1 down to 0.

@@ -259,31 +259,21 @@ int side_stream(int n, SideStream** out) {
 }
 
 // ------------------------------------------------------------ layer internals
-int fwd_bf16(const Shape& sh, const void* x, const void* Ws, const void* Wn, const float* bias,
-             unsigned flags, void* y, void* z, uint32_t* mask, cudaStream_t st) {
-    const int d = sh.d, BN = pick_bn(d), k = 1 << sh.s;
-    // patch width of the epilogue: 64 columns, or 32 for 64-wide tiles
-    const int pw = BN >= 128 ? 64 : 32;
-    CUtensorMap maps[6];
-    if (!map_rows(&maps[0], x, sh.tokens, d, k, 128) || !map_weight(&maps[1], Ws, d, BN) ||
-        !map_weight(&maps[2], Wn, d, BN) || !map_rows(&maps[3], x, sh.tokens, d, k, 32, pw) ||
-        !map_rows(&maps[4], y, sh.tokens, d, k, 32, pw))
-        return HCW_ERR_CUDA;
-    maps[5] = maps[4];   // unused by the forward
-    TcParams p;
-    memset(&p, 0, sizeof(p));
+// Row-unit geometry of a forward (or input-gradient) pass: which bit value's
+// rows take both parts.  Sec. 3.1 causal rule: in the forward, positions with
+// bit s set receive (K = 2d) and the others do not (K = d); in the input
+// gradient it is the mirror image (a bit-0 row takes dz from its partner).
+void row_unit_params(TcParams& p, const Shape& sh, int BN, unsigned flags, bool backward) {
+    const int d = sh.d;
     p.d = d;
-    p.k = k;
-    p.s = sh.s;
     p.Mh = (int)(sh.tokens / 2);
     p.nK = d / 64;
     p.n_rb = (p.Mh + 127) / 128;
     p.n_nt = d / BN;
     if (flags & HCW_CAUSAL) {
-        // Sec. 3.1: positions with bit s set receive (K = 2d), the others do not (K = d)
         p.n_full = 1;
-        p.full_bit0 = 1;
-        p.half_bit = 0;
+        p.full_bit0 = backward ? 0 : 1;
+        p.half_bit = backward ? 1 : 0;
     } else {
         p.n_full = 2;
         p.full_bit0 = 0;
@@ -291,15 +281,74 @@ int fwd_bf16(const Shape& sh, const void* x, const void* Ws, const void* Wn, con
         p.half_bit = -1;
     }
     p.n_units = p.n_rb * p.n_nt * 2;
-    p.flags = flags;
-    p.bias = bias;
-    p.out = static_cast<__nv_bfloat16*>(y);
-    p.zout = static_cast<__nv_bfloat16*>(z);
-    p.mout = mask;
     p.timeout_ns = g_timeout_ns;
+}
+
+// The five forward maps of one layer: x rows (128-row boxes), W_self, W_nbr,
+// x rows (32-row residual patches), y rows (32-row output patches).
+bool fwd_maps(CUtensorMap* m, const Shape& sh, int s, const void* x, const void* Ws,
+              const void* Wn, const void* y) {
+    const int d = sh.d, BN = pick_bn(d), k = 1 << s;
+    const int pw = BN >= 128 ? 64 : 32;   // epilogue patch width: 64 columns, 32 for narrow tiles
+    if (!map_rows(&m[0], x, sh.tokens, d, k, 128) || !map_weight(&m[1], Ws, d, BN) ||
+        !map_weight(&m[2], Wn, d, BN) || !map_rows(&m[3], x, sh.tokens, d, k, 32, pw) ||
+        !map_rows(&m[4], y, sh.tokens, d, k, 32, pw))
+        return false;
+    m[5] = m[4];   // unused by the forward
+    return true;
+}
+
+int fwd_bf16(const Shape& sh, const void* x, const void* Ws, const void* Wn, const float* bias,
+             unsigned flags, void* y, void* z, uint32_t* mask, cudaStream_t st) {
+    const int BN = pick_bn(sh.d);
+    TcLaunch<1> L;
+    memset(&L, 0, sizeof(L));
+    if (!fwd_maps(L.maps[0], sh, sh.s, x, Ws, Wn, y)) return HCW_ERR_CUDA;
+    L.layer[0] = {sh.s, 1 << sh.s, bias, mask, static_cast<__nv_bfloat16*>(z)};
+    row_unit_params(L.p, sh, BN, flags, false);
+    L.p.flags = flags;
+    L.n_layers = 1;
     const int sms = sm_count();
-    const int grid = p.n_units < sms ? p.n_units : sms;
-    return launched(launch_tc(MODE_FWD, BN, maps, p, grid, st), 1);
+    const int grid = L.p.n_units < sms ? L.p.n_units : sms;
+    return launched(launch_tc(MODE_FWD, BN, L, grid, st), 1);
+}
+
+// Completion counters of a stacked-forward launch: one int per layer of the
+// group and 128-token chunk.
+size_t stack_counter_bytes(long long tokens, int L) {
+    const int layers = L < kMaxStackLayers ? L : kMaxStackLayers;
+    return align256((size_t)layers * (size_t)((tokens + 127) / 128) * sizeof(int));
+}
+
+// Layers [l0, l0 + n) of a bf16 stack in one persistent launch.  in_ptr(l),
+// out_ptr(l), mask_ptr(l) give each layer's input, output and mask.
+template <class In, class Out, class Mask>
+int stack_fwd_group(const Shape& sh, int l0, int n, int layer0, int dim_override,
+                    const uint8_t* Ws, const uint8_t* Wn, const float* bias, unsigned flags,
+                    In in_ptr, Out out_ptr, Mask mask_ptr, int* counters, cudaStream_t st) {
+    const int d = sh.d, BN = pick_bn(d);
+    const size_t wb = (size_t)d * d * 2;
+    static thread_local TcLaunch<kMaxStackLayers> L;
+    memset(&L, 0, sizeof(L));
+    for (int i = 0; i < n; ++i) {
+        const int l = l0 + i;
+        const int s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
+        if (!fwd_maps(L.maps[i], sh, s, in_ptr(l), Ws + l * wb, Wn + l * wb, out_ptr(l)))
+            return HCW_ERR_CUDA;
+        L.layer[i] = {s, 1 << s, bias ? bias + (size_t)l * d : nullptr, mask_ptr(l), nullptr};
+    }
+    row_unit_params(L.p, sh, BN, flags, false);
+    L.p.flags = flags;
+    L.n_layers = n;
+    L.counters = counters;
+    L.n_chunks = (int)((sh.tokens + 127) / 128);
+    L.tokens = (int)sh.tokens;
+    cudaError_t e = cudaMemsetAsync(counters, 0, (size_t)n * L.n_chunks * sizeof(int), st);
+    if (e != cudaSuccess) return HCW_ERR_CUDA;
+    const int sms = sm_count();
+    const int total = L.p.n_units * n;
+    const int grid = total < sms ? total : sms;
+    return launched(launch_tc_stack_fwd(BN, L, grid, st), 1);
 }
 
 // dx: a row gathers dz from its partner exactly when the partner received from it
@@ -308,7 +357,9 @@ int dx_bf16(const Shape& sh, const void* dz, const void* dy, const void* Ws, con
             void* dz_out = nullptr) {
     const int d = sh.d, BN = pick_bn(d), k = 1 << sh.s;
     const int pw = BN >= 128 ? 64 : 32;
-    CUtensorMap maps[6];
+    TcLaunch<1> L;
+    memset(&L, 0, sizeof(L));
+    CUtensorMap* maps = L.maps[0];
     // maps of absent operands get a valid stand-in address; the kernel never uses them
     const void* res = (flags & HCW_RESIDUAL) ? dy : dz;
     if (!map_rows(&maps[0], dz, sh.tokens, d, k, 128) || !map_weight(&maps[1], Ws, d, 64) ||
@@ -316,34 +367,16 @@ int dx_bf16(const Shape& sh, const void* dz, const void* dy, const void* Ws, con
         !map_rows(&maps[4], dx ? dx : dz_out, sh.tokens, d, k, 32, pw) ||
         !map_rows(&maps[5], dz_out ? dz_out : dx, sh.tokens, d, k, 32, pw))
         return HCW_ERR_CUDA;
-    TcParams p;
-    memset(&p, 0, sizeof(p));
-    p.d = d;
-    p.k = k;
-    p.s = sh.s;
-    p.Mh = (int)(sh.tokens / 2);
-    p.nK = d / 64;
-    p.n_rb = (p.Mh + 127) / 128;
-    p.n_nt = d / BN;
-    if (flags & HCW_CAUSAL) {
-        p.n_full = 1;
-        p.full_bit0 = 0;   // bit-0 rows: their partner (bit 1) received from them
-        p.half_bit = 1;
-    } else {
-        p.n_full = 2;
-        p.full_bit0 = 0;
-        p.full_bit1 = 1;
-        p.half_bit = -1;
-    }
-    p.n_units = p.n_rb * p.n_nt * 2;
-    p.flags = flags & HCW_RESIDUAL;
-    p.out = static_cast<__nv_bfloat16*>(dx);
-    p.mprev = mprev;
-    p.dz_out = static_cast<__nv_bfloat16*>(dz_out);
-    p.timeout_ns = g_timeout_ns;
+    L.layer[0] = {sh.s, k, nullptr, nullptr, nullptr};
+    row_unit_params(L.p, sh, BN, flags, true);
+    L.p.flags = flags & HCW_RESIDUAL;
+    L.p.out = static_cast<__nv_bfloat16*>(dx);
+    L.p.mprev = mprev;
+    L.p.dz_out = static_cast<__nv_bfloat16*>(dz_out);
+    L.n_layers = 1;
     const int sms = sm_count();
-    const int grid = p.n_units < sms ? p.n_units : sms;
-    return launched(launch_tc(MODE_DX, BN, maps, p, grid, st), 1);
+    const int grid = L.p.n_units < sms ? L.p.n_units : sms;
+    return launched(launch_tc(MODE_DX, BN, L, grid, st), 1);
 }
 
 // dW: token-contracted, split over token blocks, fixed-order reduction; dbias
@@ -353,7 +386,9 @@ int dw_bf16(const Shape& sh, const void* x, const void* dz, unsigned flags, floa
     const int d = sh.d, BN = pick_bn(d), k = 1 << sh.s;
     const WsLayout lay = ws_layout(sh.tokens, d, HCW_BF16, flags);
     const WPlan w = plan_dw(sh.tokens, d, flags);
-    CUtensorMap maps[6];
+    TcLaunch<1> L;
+    memset(&L, 0, sizeof(L));
+    CUtensorMap* maps = L.maps[0];
     float* part = reinterpret_cast<float*>(wws);
     if (!map_rows(&maps[0], dz, sh.tokens, d, k, 64) || !map_rows(&maps[1], x, sh.tokens, d, k, 64) ||
         !map_f32_patches(&maps[3], w.splits_max > 1 ? (const void*)part : (const void*)dWs,
@@ -361,11 +396,9 @@ int dw_bf16(const Shape& sh, const void* x, const void* dz, unsigned flags, floa
         !map_f32_patches(&maps[4], dWs, d, d) || !map_f32_patches(&maps[5], dWn, d, d))
         return HCW_ERR_CUDA;
     maps[2] = maps[1];   // unused by the weight gradient
-    TcParams p;
-    memset(&p, 0, sizeof(p));
+    L.layer[0] = {sh.s, k, nullptr, nullptr, nullptr};
+    TcParams& p = L.p;
     p.d = d;
-    p.k = k;
-    p.s = sh.s;
     p.Mh = (int)(sh.tokens / 2);
     p.n_nt = w.n_nt;
     p.n_ot = w.n_ot;
@@ -382,9 +415,10 @@ int dw_bf16(const Shape& sh, const void* x, const void* dz, unsigned flags, floa
     p.dw_nbr = dWn;
     p.dw_partial = part;
     p.timeout_ns = g_timeout_ns;
+    L.n_layers = 1;
     const int sms = sm_count();
     const int grid = p.n_units < sms ? p.n_units : sms;
-    int rc = launched(launch_tc(MODE_DW, BN, maps, p, grid, st), 1);
+    int rc = launched(launch_tc(MODE_DW, BN, L, grid, st), 1);
     if (rc) return rc;
     if (w.splits_max > 1) {
         rc = launched(launch_splitk_reduce(p.dw_partial, w.splits_max, w.splits_self,
@@ -664,40 +698,70 @@ int hcw_layer_bwd_weight(const void* x, const void* dz, int layer, int dim_overr
                          static_cast<uint8_t*>(workspace), (cudaStream_t)stream);
 }
 
+size_t hcw_stack_fwd_workspace_bytes(int B, int n, int d, int dtype, unsigned flags, int L) {
+    Shape sh;
+    if (L < 1 || check_shape(0, -1, B, n, d, dtype, flags, &sh)) return 0;
+    return dtype == HCW_BF16 && sh.tokens > 0 ? stack_counter_bytes(sh.tokens, L) : 0;
+}
+
 int hcw_stack_fwd(const void* x, const void* W_self, const void* W_nbr, const float* bias,
                   int layer0, int L, int dim_override, int B, int n, int d, int dtype,
-                  unsigned flags, void* y, void* acts, void* masks, void* stream) {
+                  unsigned flags, void* y, void* acts, void* masks, void* workspace,
+                  size_t ws_bytes, void* stream) {
     Shape sh;
     if (L < 1) return HCW_ERR_INVALID_ARG;
     int rc = check_shape(layer0, dim_override, B, n, d, dtype, flags, &sh);
     if (rc) return rc;
     if (sh.tokens == 0) return HCW_OK;
     if (L > 1 && !acts) return HCW_ERR_INVALID_ARG;
-    if ((acts && !aligned16(acts)) || (masks && !aligned16(masks))) return HCW_ERR_ALIGNMENT;
+    if ((acts && !aligned16(acts)) || (masks && !aligned16(masks)) ||
+        (workspace && !aligned16(workspace)))
+        return HCW_ERR_ALIGNMENT;
     const size_t ab = sh.act_bytes, wb = (size_t)d * d * elem_size(dtype);
     const size_t mb = mask_bytes(sh);
+    const size_t need = hcw_stack_fwd_workspace_bytes(B, n, d, dtype, flags, L);
+    if (ws_bytes < need || (need && !workspace)) return HCW_ERR_WORKSPACE;
     rc = check_fwd_ptrs(sh, dtype, x, W_self, W_nbr, bias, y, nullptr);
     if (rc) return rc;
     const size_t acts_b = (size_t)(L - 1) * ab, m_b = (size_t)L * mb;
     if (overlaps(acts, acts_b, x, ab) || overlaps(acts, acts_b, y, ab) ||
         overlaps(masks, m_b, x, ab) || overlaps(masks, m_b, y, ab) ||
         overlaps(masks, m_b, acts, acts_b) || overlaps(acts, acts_b, W_self, L * wb) ||
-        overlaps(acts, acts_b, W_nbr, L * wb))
+        overlaps(acts, acts_b, W_nbr, L * wb) || overlaps(workspace, need, x, ab) ||
+        overlaps(workspace, need, y, ab) || overlaps(workspace, need, acts, acts_b) ||
+        overlaps(workspace, need, masks, m_b))
         return HCW_ERR_ALIASING;
     cudaStream_t st = (cudaStream_t)stream;
-    const uint8_t* xin = static_cast<const uint8_t*>(x);
     const bool want_mask = masks && (flags & HCW_ACT_RELU);
+    auto in_ptr = [&](int l) -> const void* {
+        return l == 0 ? x : static_cast<const uint8_t*>(acts) + (size_t)(l - 1) * ab;
+    };
+    auto out_ptr = [&](int l) -> void* {
+        return l == L - 1 ? y : static_cast<uint8_t*>(acts) + (size_t)l * ab;
+    };
+    auto mask_ptr = [&](int l) -> uint32_t* {
+        return want_mask ? reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(masks) + (size_t)l * mb)
+                         : nullptr;
+    };
+    if (dtype == HCW_BF16) {
+        // up to kMaxStackLayers layers per persistent launch
+        for (int l0 = 0; l0 < L; l0 += kMaxStackLayers) {
+            const int cnt = L - l0 < kMaxStackLayers ? L - l0 : kMaxStackLayers;
+            rc = stack_fwd_group(sh, l0, cnt, layer0, dim_override,
+                                 static_cast<const uint8_t*>(W_self),
+                                 static_cast<const uint8_t*>(W_nbr), bias, flags, in_ptr, out_ptr,
+                                 mask_ptr, static_cast<int*>(workspace), st);
+            if (rc) return rc;
+        }
+        return HCW_OK;
+    }
     for (int l = 0; l < L; ++l) {
         Shape shl = sh;
         shl.s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
-        const uint8_t* in = l == 0 ? xin : static_cast<const uint8_t*>(acts) + (size_t)(l - 1) * ab;
-        void* out = l == L - 1 ? y : static_cast<uint8_t*>(acts) + (size_t)l * ab;
-        uint32_t* m = want_mask
-                          ? reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(masks) + (size_t)l * mb)
-                          : nullptr;
-        rc = layer_fwd_impl(shl, dtype, in, static_cast<const uint8_t*>(W_self) + l * wb,
+        rc = layer_fwd_impl(shl, dtype, in_ptr(l), static_cast<const uint8_t*>(W_self) + l * wb,
                             static_cast<const uint8_t*>(W_nbr) + l * wb,
-                            bias ? bias + (size_t)l * d : nullptr, flags, out, nullptr, st, m);
+                            bias ? bias + (size_t)l * d : nullptr, flags, out_ptr(l), nullptr, st,
+                            mask_ptr(l));
         if (rc) return rc;
     }
     return HCW_OK;

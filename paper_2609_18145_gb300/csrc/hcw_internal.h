@@ -19,8 +19,6 @@ enum TcMode { MODE_FWD = 0, MODE_DX = 1, MODE_DW = 2 };
 // HI * 2k + beta * k + lo.
 struct TcParams {
     int d;          // feature width
-    int k;          // 2^s, the link distance of this layer
-    int s;          // cube dimension of this layer
     int Mh;         // positions per value of bit s: B * n / 2
     int nK;         // d / 64: K-steps per part (FWD, DX)
     // FWD / DX units
@@ -39,13 +37,10 @@ struct TcParams {
     int splits_self;
     int splits_nbr;
     int causal;
-    int n_units;
+    int n_units;    // units of one layer
     // epilogue
     unsigned flags;
-    const float* bias;            // FWD
-    __nv_bfloat16* out;           // FWD: y; DX: dx (may be null when dz_out is set)
-    __nv_bfloat16* zout;          // FWD: z (may be null)
-    uint32_t* mout;               // FWD: ReLU mask words [tokens][d/32], bit e = (z > 0), or null
+    __nv_bfloat16* out;           // DX: dx (may be null when dz_out is set)
     const uint32_t* mprev;        // DX: ReLU mask words of the layer below (fused ReLU grad)
     __nv_bfloat16* dz_out;        // DX: that layer's gradient dz = dx * mask, or null
     float* dw_self;               // DW destination when splits_self == 1
@@ -55,10 +50,38 @@ struct TcParams {
     unsigned long long timeout_ns;
 };
 
-// Launch one tensor-core pass.  maps[0..5] = tmA, tmB0, tmB1, tmE0, tmE1, tmE2
-// as documented at hcw_tc_kernel in hcw_tc.cu.
-cudaError_t launch_tc(int mode, int BN, const CUtensorMap* maps, const TcParams& p, int grid,
-                      cudaStream_t stream);
+// The per-layer part of a launch.  A forward launch may cover a run of
+// layers (the stacked forward); every other launch covers one layer.
+struct TcLayer {
+    int s;                        // cube dimension
+    int k;                        // 2^s
+    const float* bias;            // FWD bias or null
+    uint32_t* mout;               // FWD: ReLU mask words [tokens][d/32], bit e = (z > 0), or null
+    __nv_bfloat16* zout;          // FWD: bf16 pre-activation (layer API), or null
+};
+
+constexpr int kMaxStackLayers = 16;   // layers per stacked-forward launch
+
+// maps[l][0..5] = tmA, tmB0, tmB1, tmE0, tmE1, tmE2 of layer l, as documented
+// at hcw_tc_kernel in hcw_tc.cu.
+template <int NL>
+struct TcLaunch {
+    CUtensorMap maps[NL][6];
+    TcLayer layer[NL];
+    TcParams p;
+    int n_layers;
+    // stacked forward: completion counters [n_layers][n_chunks] (zeroed before
+    // the launch), one per layer and 128-token chunk, counting output elements
+    int* counters;
+    int n_chunks;
+    int tokens;
+};
+
+// Launch one tensor-core pass (one layer).
+cudaError_t launch_tc(int mode, int BN, const TcLaunch<1>& L, int grid, cudaStream_t stream);
+// Launch the stacked forward over L.n_layers consecutive layers.
+cudaError_t launch_tc_stack_fwd(int BN, const TcLaunch<kMaxStackLayers>& L, int grid,
+                                cudaStream_t stream);
 
 // Dynamic shared memory the tensor-core kernel uses for this N tile.
 size_t tc_smem_bytes(int BN);

@@ -75,6 +75,7 @@ struct __align__(8) Barriers {
     uint64_t epi_load[kEpiWarps][kEpiBufs];       // residual patch landed in a buffer
     uint32_t tmem_base;
     int abort;
+    int dep_unit;   // the producer has seen the inputs of this CTA's units up to this ordinal
 };
 
 template <int BN>
@@ -89,22 +90,31 @@ struct RowUnit {
     int beta, t, j, steps;
 };
 
-__device__ __forceinline__ RowUnit decode_row_unit(const TcParams& p, int u) {
+__device__ __forceinline__ RowUnit decode_row_unit(const TcParams& p, int u, bool stacked) {
     RowUnit r;
     const int per_bit = p.n_rb * p.n_nt;
-    int rem;
-    if (u < p.n_full * per_bit) {
-        const int g = u / per_bit;
+    int g, rem;
+    if (!stacked) {
+        // one layer: the long (two-part) units first, then the short ones
+        g = u / per_bit;
         rem = u - g * per_bit;
+        r.t = rem / p.n_nt;
+        r.j = rem - r.t * p.n_nt;
+    } else {
+        // a run of layers: row block by row block, so that the next layer's
+        // first blocks find their inputs early
+        r.t = u / (2 * p.n_nt);
+        rem = u - r.t * 2 * p.n_nt;
+        g = rem / p.n_nt;
+        r.j = rem - g * p.n_nt;
+    }
+    if (g < p.n_full) {
         r.beta = g == 0 ? p.full_bit0 : p.full_bit1;
         r.steps = 2 * p.nK;
     } else {
-        rem = u - p.n_full * per_bit;
         r.beta = p.half_bit;
         r.steps = p.nK;
     }
-    r.t = rem / p.n_nt;
-    r.j = rem - r.t * p.n_nt;
     return r;
 }
 
@@ -170,6 +180,46 @@ __device__ __forceinline__ void tmem_ld_wait_regs(uint32_t (&r)[32]) {
                  : "memory");
 }
 
+__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
+    int v;
+    asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void fence_proxy_async_global() {
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+__device__ __forceinline__ int ld_acquire_cta_shared(const int* p) {
+    int v;
+    asm volatile("ld.acquire.cta.shared::cta.b32 %0, [%1];" : "=r"(v) : "r"(smem_u32(p)) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ void st_release_cta_shared(int* p, int v) {
+    asm volatile("st.release.cta.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(p)), "r"(v) : "memory");
+}
+
+// Bounded wait until *ctr >= target (a counter other CTAs raise), with
+// acquire semantics; records a timeout like mbar_wait.
+__device__ __forceinline__ bool wait_counter(const int* ctr, int target, volatile int* abort,
+                                             uint64_t timeout_ns) {
+    if (ld_acquire_gpu(ctr) >= target) return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t it = 1;; ++it) {
+        __nanosleep(64);
+        if (ld_acquire_gpu(ctr) >= target) return true;
+        if ((it & 15u) == 0) {
+            if (*abort) return false;
+            if (globaltimer_ns() - t0 > timeout_ns) {
+                atomicExch(&g_error_word, kErrTimeout);
+                *abort = 1;
+                return false;
+            }
+        }
+    }
+}
+
 // Wait that only gives up on time (used to drain in-flight work after an
 // abort, when the abort flag is already set).
 __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity,
@@ -183,25 +233,30 @@ __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity,
 
 }  // namespace
 
-// Mainloop maps:
-//   tmA : FWD x, DX dz: 4-D rows map, box (64, lo_box, 1, hi_box) = 128 rows.
-//         DW dz: the same view with 64-row boxes.
-//   tmB0: FWD W_self [o][k] 2-D, box (64 k, BN o)   (K-major B)
-//         DX  W_self [o][k] 2-D, box (64 k, 64 o)   (MN-major B, BN/64 boxes)
-//         DW  x rows, 64-row boxes                  (MN-major B, BN/64 boxes)
-//   tmB1: FWD/DX W_nbr like tmB0; DW unused.
-// Epilogue maps (32-row patches, inner box = one patch row):
-//   tmE0: FWD x / DX dy rows (residual, loaded);  DW: dW split partials [2*S*d][d] fp32
-//   tmE1: FWD y / DX dx rows (stored);             DW: dW_self [d][d] fp32
-//   tmE2: DX dz rows of the layer below (stored);  DW: dW_nbr  [d][d] fp32
-template <int MODE, int BN>
+// Maps of layer l (L.maps[l][i]):
+//   0 tmA : FWD x, DX dz: 4-D rows map, box (64, lo_box, 1, hi_box) = 128 rows.
+//           DW dz: the same view with 64-row boxes.
+//   1 tmB0: FWD W_self [o][k] 2-D, box (64 k, BN o)   (K-major B)
+//           DX  W_self [o][k] 2-D, box (64 k, 64 o)   (MN-major B, BN/64 boxes)
+//           DW  x rows, 64-row boxes                  (MN-major B, BN/64 boxes)
+//   2 tmB1: FWD/DX W_nbr like tmB0; DW unused.
+//   3 tmE0: FWD x / DX dy rows (residual patches, loaded); DW dW partials [2*S*d][d] fp32
+//   4 tmE1: FWD y / DX dx rows (patches stored);           DW dW_self [d][d] fp32
+//   5 tmE2: DX dz rows of the layer below (stored);        DW dW_nbr  [d][d] fp32
+// Patch maps have 32-row boxes whose inner extent is one patch row.
+//
+// A stacked forward launch (NL > 1) covers L.n_layers consecutive layers;
+// unit u belongs to layer u / units_per_layer and the units are ordered
+// layer by layer and, within a layer, row block by row block.  The input
+// rows of a unit of layer l > 0 are outputs of layer l - 1: before loading
+// them the producer waits until the completion counters of the 128-token
+// chunks they lie in show every element written (each epilogue warp adds the
+// elements of a patch once its TMA stores have landed).  All earlier units
+// of the launch have smaller indices and each CTA takes its units in order,
+// so the lowest unfinished unit can always proceed.
+template <int MODE, int BN, int NL>
 __global__ void __launch_bounds__(kThreads, 1)
-    hcw_tc_kernel(const __grid_constant__ CUtensorMap tmA,
-                  const __grid_constant__ CUtensorMap tmB0,
-                  const __grid_constant__ CUtensorMap tmB1,
-                  const __grid_constant__ CUtensorMap tmE0,
-                  const __grid_constant__ CUtensorMap tmE1,
-                  const __grid_constant__ CUtensorMap tmE2, const TcParams p) {
+    hcw_tc_kernel(const __grid_constant__ TcLaunch<NL> L) {
     constexpr int STAGES = num_stages(BN);
     constexpr int SB = stage_bytes(BN);
     constexpr int B_BYTES = BN * kBlockK * 2;
@@ -209,6 +264,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr uint32_t IDESC = idesc_bf16_f32(kBlockM, BN, MODE == MODE_DW ? 1 : 0,
                                               MODE == MODE_FWD ? 0 : 1);
     constexpr int HALF = BN / 2;                       // columns per epilogue warp
+    constexpr bool STACKED = NL > 1;
+    const TcParams& p = L.p;
+    const int upl = p.n_units;                          // units per layer
+    const int n_units = upl * L.n_layers;
 
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>(
@@ -222,9 +281,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
-        tma_prefetch_desc(&tmA);
-        tma_prefetch_desc(&tmB0);
-        if (MODE != MODE_DW) tma_prefetch_desc(&tmB1);
+        for (int l = 0; l < L.n_layers && l < NL; ++l)
+            for (int i = 0; i < 6; ++i) tma_prefetch_desc(&L.maps[l][i]);
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&bars->full[s], 1);
             mbar_init(&bars->empty[s], 1);
@@ -237,6 +295,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int b = 0; b < kEpiBufs; ++b) mbar_init(&bars->epi_load[e][b], 1);
         mbar_init(&bars->drain, 1);
         bars->abort = 0;
+        bars->dep_unit = -1;
         fence_mbar_init();
     }
     if (warp == 1) {
@@ -257,11 +316,32 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t phase = 0;
             uint32_t issued_mask = 0, issued_phase = 0;
             bool ok = true;
-            for (int u = blockIdx.x; u < p.n_units && ok; u += gridDim.x) {
+            int ordinal = 0;
+            for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x, ++ordinal) {
+                const int l = STACKED ? u / upl : 0;
+                const int ul = STACKED ? u - l * upl : u;
+                const TcLayer& ly = L.layer[l];
+                const CUtensorMap* mA = &L.maps[l][0];
                 if (MODE != MODE_DW) {
-                    const RowUnit r = decode_row_unit(p, u);
+                    const RowUnit r = decode_row_unit(p, ul, STACKED);
                     const int q0 = r.t * kBlockM;
-                    const int lo0 = q0 % p.k, hi0 = q0 / p.k;
+                    const int lo0 = q0 & (ly.k - 1), hi0 = q0 >> ly.s;
+                    if (STACKED && l > 0) {
+                        // the unit's rows and their partners: two 128-token chunks
+                        const int tok_a = (hi0 << (ly.s + 1)) + lo0;
+                        const int ca = tok_a >> 7;
+                        const int cb = ly.k >= kBlockM ? ((tok_a + ly.k) >> 7) : ca + 1;
+                        const int* ctr = L.counters + (size_t)(l - 1) * L.n_chunks;
+                        const int cs[2] = {ca, cb};
+                        for (int i = 0; i < 2 && ok; ++i) {
+                            if (cs[i] >= L.n_chunks) continue;
+                            const int rows = min(128, L.tokens - (cs[i] << 7));
+                            ok = wait_counter(ctr + cs[i], rows * p.d, abort, tmo);
+                        }
+                        if (!ok) break;
+                        fence_proxy_async_global();
+                    }
+                    st_release_cta_shared(&bars->dep_unit, ordinal);
                     for (int ks = 0; ks < r.steps; ++ks) {
                         if (!mbar_wait(&bars->empty[stage], phase ^ 1, abort, tmo)) {
                             ok = false;
@@ -275,8 +355,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const int part = ks >= p.nK;
                         const int kk = part ? ks - p.nK : ks;
                         const int bitA = part ? 1 - r.beta : r.beta;
-                        tma_load_4d(sA, &tmA, &bars->full[stage], kk * kBlockK, lo0, bitA, hi0);
-                        const CUtensorMap* mb = part ? &tmB1 : &tmB0;
+                        tma_load_4d(sA, mA, &bars->full[stage], kk * kBlockK, lo0, bitA, hi0);
+                        const CUtensorMap* mb = &L.maps[l][part ? 2 : 1];
                         if (MODE == MODE_FWD) {
                             tma_load_2d(sB, mb, &bars->full[stage], kk * kBlockK, r.j * BN);
                         } else {
@@ -291,7 +371,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                     }
                 } else {
-                    const WUnit w = decode_w_unit(p, u);
+                    const WUnit w = decode_w_unit(p, ul);
+                    st_release_cta_shared(&bars->dep_unit, ordinal);
                     for (int kb = w.kb0; kb < w.kb1; ++kb) {
                         if (!mbar_wait(&bars->empty[stage], phase ^ 1, abort, tmo)) {
                             ok = false;
@@ -312,18 +393,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                             bB = 1 - bA;
                         }
                         const int q0 = qb * 64;
-                        const int lo0 = q0 % p.k, hi0 = q0 / p.k;
+                        const int lo0 = q0 & (ly.k - 1), hi0 = q0 >> ly.s;
                         uint8_t* sA = smem + (size_t)stage * SB;
                         uint8_t* sB = sA + kABytes;
                         mbar_arrive_expect_tx(&bars->full[stage], kABytes + B_BYTES);
                         issued_mask |= 1u << stage;
                         issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
-                        tma_load_4d(sA, &tmA, &bars->full[stage], w.ot * kBlockM, lo0, bA, hi0);
-                        tma_load_4d(sA + 8192, &tmA, &bars->full[stage], w.ot * kBlockM + 64, lo0,
+                        tma_load_4d(sA, mA, &bars->full[stage], w.ot * kBlockM, lo0, bA, hi0);
+                        tma_load_4d(sA + 8192, mA, &bars->full[stage], w.ot * kBlockM + 64, lo0,
                                     bA, hi0);
 #pragma unroll
                         for (int jj = 0; jj < BN / 64; ++jj)
-                            tma_load_4d(sB + jj * 8192, &tmB0, &bars->full[stage],
+                            tma_load_4d(sB + jj * 8192, &L.maps[l][1], &bars->full[stage],
                                         w.nt * BN + jj * 64, lo0, bB, hi0);
                         if (++stage == STAGES) {
                             stage = 0;
@@ -347,12 +428,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             int acc = 0;
             uint32_t acc_phase = 0;
             bool ok = true, any = false;
-            for (int u = blockIdx.x; u < p.n_units && ok; u += gridDim.x) {
+            for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+                const int ul = STACKED ? u % upl : u;
                 int steps;
                 if (MODE != MODE_DW) {
-                    steps = decode_row_unit(p, u).steps;
+                    steps = decode_row_unit(p, ul, STACKED).steps;
                 } else {
-                    const WUnit w = decode_w_unit(p, u);
+                    const WUnit w = decode_w_unit(p, ul);
                     steps = w.kb1 - w.kb0;
                 }
                 if (!mbar_wait(&bars->tempty[acc], acc_phase ^ 1, abort, tmo)) {
@@ -413,6 +495,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         int acc = 0;
         uint32_t acc_phase = 0;
         bool alive = true;
+        int ordinal = 0;
         // every lane observes the barrier; the warp proceeds only if all did
         // (tcgen05.ld and the patch accesses are warp-wide)
         auto wait_bar = [&](uint64_t* bar, uint32_t parity) -> bool {
@@ -441,19 +524,37 @@ __global__ void __launch_bounds__(kThreads, 1)
             fence_proxy_async_smem();
             __syncwarp();
         };
-        for (int u = blockIdx.x; u < p.n_units && alive; u += gridDim.x) {
+        // the producer has checked this unit's inputs (lane 0 waits, bounded)
+        auto wait_inputs = [&](int ord) -> bool {
+            int ok = 1;
+            if (lane == 0) {
+                const uint64_t t0 = globaltimer_ns();
+                while (ld_acquire_cta_shared(&bars->dep_unit) < ord) {
+                    if (*abort || globaltimer_ns() - t0 > tmo) {
+                        ok = 0;
+                        break;
+                    }
+                }
+                if (ok) fence_proxy_async_global();
+            }
+            return __shfl_sync(0xffffffffu, ok, 0) != 0;
+        };
+        for (int u = blockIdx.x; u < n_units && alive; u += gridDim.x, ++ordinal) {
+            const int l = STACKED ? u / upl : 0;
+            const int ul = STACKED ? u - l * upl : u;
+            const TcLayer& ly = L.layer[l];
             if (MODE != MODE_DW) {
                 constexpr int SW = HALF >= 64 ? 64 : HALF;     // patch width (columns)
                 constexpr int RB = SW * 2;                     // patch row bytes
                 constexpr int NSC = HALF / SW;                 // patches per warp (<= 2)
                 constexpr int SUB = SW / 32;                   // 32-column sub-chunks per patch
                 static_assert(NSC <= kEpiBufs, "one buffer per patch");
-                const RowUnit r = decode_row_unit(p, u);
+                const RowUnit r = decode_row_unit(p, ul, STACKED);
                 const int qw = r.t * kBlockM + quarter * 32;   // first compressed row of the warp
-                const int lo_w = qw & (p.k - 1), hi_w = qw >> p.s;
+                const int lo_w = qw & (ly.k - 1), hi_w = qw >> ly.s;
                 const int q_row = qw + lane;
-                const int tok_row = q_row < p.Mh ? ((q_row >> p.s) << (p.s + 1)) +
-                                                       (r.beta << p.s) + (q_row & (p.k - 1))
+                const int tok_row = q_row < p.Mh ? ((q_row >> ly.s) << (ly.s + 1)) +
+                                                       (r.beta << ly.s) + (q_row & (ly.k - 1))
                                                  : -1;
                 const int col_half = r.j * BN + half * HALF;
                 // a patch entirely past the end (ragged tail) loads and stores nothing
@@ -461,15 +562,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const bool has_res = (p.flags & 2u) != 0 && inside;
                 const bool fwd = MODE == MODE_FWD;
                 const bool has_mprev = MODE == MODE_DX && p.mprev != nullptr;
+                const CUtensorMap* mE0 = &L.maps[l][3];
+                const CUtensorMap* mE1 = &L.maps[l][4];
+                const CUtensorMap* mE2 = &L.maps[l][5];
                 const int wpr = p.d >> 5;
                 // every earlier store has finished reading the buffers: refill them
                 if (lane == 0) bulk_wait_read<0>();
                 __syncwarp();
+                if (!wait_inputs(ordinal)) {
+                    alive = false;
+                    break;
+                }
                 if (has_res && lane == 0) {
 #pragma unroll
                     for (int sc = 0; sc < NSC; ++sc) {
                         mbar_arrive_expect_tx(&bars->epi_load[e][sc], 32 * RB);
-                        tma_load_4d(bufs + sc * kEpiBufBytes, &tmE0, &bars->epi_load[e][sc],
+                        tma_load_4d(bufs + sc * kEpiBufBytes, mE0, &bars->epi_load[e][sc],
                                     col_half + sc * SW, lo_w, r.beta, hi_w);
                     }
                 }
@@ -482,7 +590,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (fwd) {
                     // this warp's bias slice, read back as warp-wide broadcasts
                     for (int c = lane; c < HALF; c += 32)
-                        wbias[c] = p.bias ? __ldg(p.bias + col_half + c) : 0.f;
+                        wbias[c] = ly.bias ? __ldg(ly.bias + col_half + c) : 0.f;
                     __syncwarp();
                 }
                 if (!wait_acc()) {
@@ -491,13 +599,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 // FWD z (layer API only): the pre-activation, row-wise stores; every
                 // lane joins the warp-wide TMEM loads, rows past the end skip the store
-                if (fwd && p.zout) {
+                if (fwd && ly.zout) {
 #pragma unroll 1
                     for (int c = 0; c < HALF / 32; ++c) {
                         uint32_t raw[32];
                         load_acc(c * 32, raw);
                         if (tok_row >= 0) {
-                            uint4* dst = reinterpret_cast<uint4*>(p.zout + (size_t)tok_row * p.d +
+                            uint4* dst = reinterpret_cast<uint4*>(ly.zout + (size_t)tok_row * p.d +
                                                                   col_half + c * 32);
 #pragma unroll
                             for (int m = 0; m < 4; ++m) {
@@ -544,12 +652,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 v[4 * i + 2] += bb.z;
                                 v[4 * i + 3] += bb.w;
                             }
-                            if (p.mout) {
+                            if (ly.mout) {
                                 uint32_t bits = 0;
 #pragma unroll
                                 for (int i = 0; i < 32; ++i) bits |= (v[i] > 0.f ? 1u : 0u) << i;
                                 if (tok_row >= 0)
-                                    p.mout[(size_t)tok_row * wpr + ((col_half + sc * SW) >> 5) + h] =
+                                    ly.mout[(size_t)tok_row * wpr + ((col_half + sc * SW) >> 5) + h] =
                                         bits;
                             }
                             if (p.flags & 4u) {
@@ -574,7 +682,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (int i = 0; i < 16; ++i) gw[h][i] = pack_bf16x2(v[2 * i], v[2 * i + 1]);
                     }
                     // the patch: y (FWD) or dx (DX), written over the residual rows
-                    if (p.out) {
+                    if (fwd || p.out) {
 #pragma unroll
                         for (int h = 0; h < SUB; ++h)
 #pragma unroll
@@ -584,7 +692,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                gw[h][4 * m + 3]);
                         publish();
                         if (lane == 0 && inside) {
-                            tma_store_4d(&tmE1, buf, col_half + sc * SW, lo_w, r.beta, hi_w);
+                            tma_store_4d(mE1, buf, col_half + sc * SW, lo_w, r.beta, hi_w);
                             bulk_commit();
                         }
                     }
@@ -613,19 +721,33 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                         publish();
                         if (lane == 0 && inside) {
-                            tma_store_4d(&tmE2, buf, col_half + sc * SW, lo_w, r.beta, hi_w);
+                            tma_store_4d(mE2, buf, col_half + sc * SW, lo_w, r.beta, hi_w);
                             bulk_commit();
                         }
                     }
                 }
+                if (STACKED && alive && l + 1 < L.n_layers) {
+                    // publish the finished patch to the next layer's units: its stores
+                    // have landed, then count its elements in the chunk it lies in
+                    if (lane == 0 && inside) {
+                        bulk_wait<0>();
+                        fence_proxy_async_global();
+                        __threadfence();
+                        const int rows = min(32, p.Mh - qw);
+                        const int tok0 = ((qw >> ly.s) << (ly.s + 1)) + (r.beta << ly.s) +
+                                         (qw & (ly.k - 1));
+                        atomicAdd(L.counters + (size_t)l * L.n_chunks + (tok0 >> 7), rows * HALF);
+                    }
+                    __syncwarp();
+                }
             } else {
-                const WUnit w = decode_w_unit(p, u);
+                const WUnit w = decode_w_unit(p, ul);
                 if (!wait_acc()) {
                     alive = false;
                     break;
                 }
                 const int S = w.which ? p.splits_nbr : p.splits_self;
-                const CUtensorMap* map = S > 1 ? &tmE0 : (w.which ? &tmE2 : &tmE1);
+                const CUtensorMap* map = &L.maps[l][S > 1 ? 3 : (w.which ? 5 : 4)];
                 const int row0 = (S > 1 ? (w.which * p.splits_max + w.split) * p.d : 0) +
                                  w.ot * kBlockM + quarter * 32;
                 const int col_half = w.nt * BN + half * HALF;
@@ -668,12 +790,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
-template <int MODE, int BN>
-static cudaError_t launch_one(const CUtensorMap* maps, const TcParams& p, int grid,
-                              cudaStream_t st) {
+template <int MODE, int BN, int NL>
+static cudaError_t launch_one(const TcLaunch<NL>& L, int grid, cudaStream_t st) {
     constexpr size_t smem = smem_total<BN>();
     static_assert(smem <= 232448, "shared memory budget");
-    auto kern = hcw_tc_kernel<MODE, BN>;
+    auto kern = hcw_tc_kernel<MODE, BN, NL>;
     // the shared-memory opt-in is a per-device function attribute: set it once per device
     static std::atomic<uint64_t> configured[4] = {};
     int dev = 0;
@@ -686,14 +807,13 @@ static cudaError_t launch_one(const CUtensorMap* maps, const TcParams& p, int gr
         if (e != cudaSuccess) return e;
         if (dev < 256) word.fetch_or(bit, std::memory_order_acq_rel);
     }
-    kern<<<grid, kThreads, smem, st>>>(maps[0], maps[1], maps[2], maps[3], maps[4], maps[5], p);
+    kern<<<grid, kThreads, smem, st>>>(L);
     return cudaGetLastError();
 }
 
-cudaError_t launch_tc(int mode, int BN, const CUtensorMap* maps, const TcParams& p, int grid,
-                      cudaStream_t st) {
+cudaError_t launch_tc(int mode, int BN, const TcLaunch<1>& L, int grid, cudaStream_t st) {
 #define HCW_TC_CASE(M, N) \
-    if (mode == M && BN == N) return launch_one<M, N>(maps, p, grid, st);
+    if (mode == M && BN == N) return launch_one<M, N, 1>(L, grid, st);
     HCW_TC_CASE(MODE_FWD, 256)
     HCW_TC_CASE(MODE_FWD, 128)
     HCW_TC_CASE(MODE_FWD, 64)
@@ -704,6 +824,14 @@ cudaError_t launch_tc(int mode, int BN, const CUtensorMap* maps, const TcParams&
     HCW_TC_CASE(MODE_DW, 128)
     HCW_TC_CASE(MODE_DW, 64)
 #undef HCW_TC_CASE
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_tc_stack_fwd(int BN, const TcLaunch<kMaxStackLayers>& L, int grid,
+                                cudaStream_t st) {
+    if (BN == 256) return launch_one<MODE_FWD, 256, kMaxStackLayers>(L, grid, st);
+    if (BN == 128) return launch_one<MODE_FWD, 128, kMaxStackLayers>(L, grid, st);
+    if (BN == 64) return launch_one<MODE_FWD, 64, kMaxStackLayers>(L, grid, st);
     return cudaErrorInvalidValue;
 }
 

@@ -59,7 +59,9 @@ _SIGNATURES = {
     "hcw_layer_bwd_weight": ([_P, _P, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P, _SZ, _P], _I),
     "hcw_layer_bwd_weight_noalloc": ([_P, _P, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P], _I),
     "hcw_launch_count": ([], ctypes.c_ulonglong),
-    "hcw_stack_fwd": ([_P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P], _I),
+    "hcw_stack_fwd": ([_P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P, _SZ,
+                       _P], _I),
+    "hcw_stack_fwd_workspace_bytes": ([_I, _I, _I, _I, _U, _I], _SZ),
     "hcw_stack_workspace_bytes": ([_I, _I, _I, _I, _U], _SZ),
     "hcw_stack_bwd": ([_P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P,
                        _P, _P, _SZ, _P], _I),
@@ -242,15 +244,20 @@ def hcw_launch_count() -> int:
     return int(lib().hcw_launch_count())
 
 
+def hcw_stack_fwd_workspace_bytes(B: int, n: int, d: int, dtype: int, flags: int, L: int) -> int:
+    return int(lib().hcw_stack_fwd_workspace_bytes(B, n, d, dtype, flags, L))
+
+
 def hcw_stack_fwd(x, W_self, W_nbr, bias=None, layer0: int = 0, dim_override: int = -1,
                   flags: int = 0, y=None, acts=None, masks=None, want_masks: bool = None,
-                  stream=None):
+                  workspace=None, stream=None):
     """Stack forward over L = W_self.shape[0] layers; returns (y, acts, masks).
     masks (ReLU only) are int32 words [L, B, n, ceil(d/32)], bit o%32 of word
     o/32 = (z > 0); allocated when the stack uses ReLU unless want_masks=False."""
-    _dev(x, W_self, W_nbr, bias, y, acts, masks)
+    _dev(x, W_self, W_nbr, bias, y, acts, masks, workspace)
     B, n, d = x.shape
     L = W_self.shape[0]
+    dt = _dtype_code(x)
     y = torch.empty_like(x) if y is None else y
     if acts is None and L > 1:
         acts = torch.empty((L - 1, B, n, d), dtype=x.dtype, device=x.device)
@@ -258,9 +265,11 @@ def hcw_stack_fwd(x, W_self, W_nbr, bias=None, layer0: int = 0, dim_override: in
         want_masks = bool(flags & HCW_ACT_RELU)
     if masks is None and want_masks:
         masks = torch.empty((L, B, n, (d + 31) // 32), dtype=torch.int32, device=x.device)
+    ws = _workspace(hcw_stack_fwd_workspace_bytes(B, n, d, dt, flags, L), x.device, workspace)
     _check(lib().hcw_stack_fwd(_ptr(x), _ptr(W_self), _ptr(W_nbr), _ptr(bias), layer0, L,
-                               dim_override, B, n, d, _dtype_code(x), flags, _ptr(y),
-                               _ptr(acts), _ptr(masks), _stream(stream)), "hcw_stack_fwd")
+                               dim_override, B, n, d, dt, flags, _ptr(y), _ptr(acts),
+                               _ptr(masks), _ptr(ws), ws.numel(), _stream(stream)),
+           "hcw_stack_fwd")
     return y, acts, masks
 
 
