@@ -268,7 +268,7 @@ def run_ours(args):
     gWs = torch.empty((L, d, d), dtype=torch.float32, device=dev)
     gWn = torch.empty((L, d, d), dtype=torch.float32, device=dev)
     gb = torch.empty((L, d), dtype=torch.float32, device=dev)
-    ws = torch.empty(H.hcw_stack_workspace_bytes(B, n, d, H.HCW_BF16, flags), dtype=torch.uint8,
+    ws = torch.empty(H.hcw_stack_workspace_bytes(B, n, d, H.HCW_BF16, flags, L), dtype=torch.uint8,
                      device=dev)
     fws = torch.empty(max(1, H.hcw_stack_fwd_workspace_bytes(B, n, d, H.HCW_BF16, flags, L)),
                       dtype=torch.uint8, device=dev)

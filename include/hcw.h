@@ -187,9 +187,12 @@ size_t hcw_stack_fwd_workspace_bytes(int B, int n, int d, int dtype, unsigned fl
  *   dx [B][n][d] gradient of x (output); dW_self, dW_nbr [L][d][d] and
  *   dbias [L][d] (or NULL) fp32 outputs.
  *   workspace: at least hcw_stack_workspace_bytes(...) bytes.
- * With HCW_ACT_RELU the input-gradient pass of layer l also applies the
- * ReLU gradient of layer l-1 (bf16), so no separate elementwise pass runs
- * between layers.
+ * bf16: the input gradients of runs of up to 16 layers go in one persistent
+ * launch (top down, a tile starting as soon as the rows it reads are
+ * written), whose kernel also applies the ReLU gradient of the layer below;
+ * then one launch computes the weight gradients of up to 16 layers (whole
+ * token range per tile, no split reduction) and one batched pass the bias
+ * gradients.  The workspace keeps every layer's dz.
  */
 int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void* dy,
                   const void* W_self, const void* W_nbr, int layer0, int L, int dim_override,
@@ -197,8 +200,8 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void
                   void* dx, float* dW_self, float* dW_nbr, float* dbias,
                   void* workspace, size_t ws_bytes, void* stream);
 
-/* Workspace bytes hcw_stack_bwd needs. */
-size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags);
+/* Workspace bytes hcw_stack_bwd needs for L layers. */
+size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags, int L);
 
 /*
  * hcw_layer_bwd_weight for callers that cannot allocate device memory (a

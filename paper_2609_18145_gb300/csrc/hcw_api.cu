@@ -7,7 +7,6 @@
 
 #include <atomic>
 #include <mutex>
-#include <vector>
 
 #include "hcw.h"
 #include "hcw_internal.h"
@@ -17,7 +16,6 @@ namespace {
 
 constexpr unsigned kAllFlags = HCW_CAUSAL | HCW_RESIDUAL | HCW_ACT_RELU;
 constexpr unsigned long long kDefaultTimeoutNs = 2000000000ull;   // 2 s per wait
-constexpr int kStackSlots = 3;   // pre-activation-gradient slots of the stack backward
 
 int log2_exact(long long n) {
     if (n < 2 || (n & (n - 1))) return -1;
@@ -227,37 +225,6 @@ int launched(cudaError_t e, int kernels) {
     return HCW_OK;
 }
 
-// ------------------------------------------------------------ side stream
-// hcw_stack_bwd runs the weight gradients on a second stream, forked from and
-// joined back to the caller's stream with events, so that they fill the SMs
-// the input-gradient chain leaves idle.  One side stream and an event pool per
-// device, created on first use and kept for the process; the enqueue sequence
-// is serialised across host threads because the events are shared.
-struct SideStream {
-    cudaStream_t stream = nullptr;
-    std::vector<cudaEvent_t> events;
-};
-std::mutex g_side_mu;
-SideStream g_side[64];
-
-// Called with g_side_mu held.  Returns HCW_OK and the device's side stream with
-// at least n events.
-int side_stream(int n, SideStream** out) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return HCW_ERR_CUDA;
-    if (dev < 0 || dev >= 64) return HCW_ERR_UNSUPPORTED;
-    SideStream& ss = g_side[dev];
-    if (!ss.stream && cudaStreamCreateWithFlags(&ss.stream, cudaStreamNonBlocking) != cudaSuccess)
-        return HCW_ERR_CUDA;
-    while ((int)ss.events.size() < n) {
-        cudaEvent_t e;
-        if (cudaEventCreateWithFlags(&e, cudaEventDisableTiming) != cudaSuccess) return HCW_ERR_CUDA;
-        ss.events.push_back(e);
-    }
-    *out = &ss;
-    return HCW_OK;
-}
-
 // ------------------------------------------------------------ layer internals
 // Row-unit geometry of a forward (or input-gradient) pass: which bit value's
 // rows take both parts.  Sec. 3.1 causal rule: in the forward, positions with
@@ -304,7 +271,7 @@ int fwd_bf16(const Shape& sh, const void* x, const void* Ws, const void* Wn, con
     TcLaunch<1> L;
     memset(&L, 0, sizeof(L));
     if (!fwd_maps(L.maps[0], sh, sh.s, x, Ws, Wn, y)) return HCW_ERR_CUDA;
-    L.layer[0] = {sh.s, 1 << sh.s, bias, mask, static_cast<__nv_bfloat16*>(z)};
+    L.layer[0] = {sh.s, 1 << sh.s, bias, mask, static_cast<__nv_bfloat16*>(z), true, nullptr, false};
     row_unit_params(L.p, sh, BN, flags, false);
     L.p.flags = flags;
     L.n_layers = 1;
@@ -335,7 +302,8 @@ int stack_fwd_group(const Shape& sh, int l0, int n, int layer0, int dim_override
         const int s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
         if (!fwd_maps(L.maps[i], sh, s, in_ptr(l), Ws + l * wb, Wn + l * wb, out_ptr(l)))
             return HCW_ERR_CUDA;
-        L.layer[i] = {s, 1 << s, bias ? bias + (size_t)l * d : nullptr, mask_ptr(l), nullptr};
+        L.layer[i] = {s, 1 << s, bias ? bias + (size_t)l * d : nullptr, mask_ptr(l), nullptr,
+                      true, nullptr, false};
     }
     row_unit_params(L.p, sh, BN, flags, false);
     L.p.flags = flags;
@@ -348,7 +316,7 @@ int stack_fwd_group(const Shape& sh, int l0, int n, int layer0, int dim_override
     const int sms = sm_count();
     const int total = L.p.n_units * n;
     const int grid = total < sms ? total : sms;
-    return launched(launch_tc_stack_fwd(BN, L, grid, st), 1);
+    return launched(launch_tc_stack(MODE_FWD, BN, L, grid, st), 1);
 }
 
 // dx: a row gathers dz from its partner exactly when the partner received from it
@@ -367,12 +335,9 @@ int dx_bf16(const Shape& sh, const void* dz, const void* dy, const void* Ws, con
         !map_rows(&maps[4], dx ? dx : dz_out, sh.tokens, d, k, 32, pw) ||
         !map_rows(&maps[5], dz_out ? dz_out : dx, sh.tokens, d, k, 32, pw))
         return HCW_ERR_CUDA;
-    L.layer[0] = {sh.s, k, nullptr, nullptr, nullptr};
+    L.layer[0] = {sh.s, k, nullptr, nullptr, nullptr, dx != nullptr, mprev, dz_out != nullptr};
     row_unit_params(L.p, sh, BN, flags, true);
     L.p.flags = flags & HCW_RESIDUAL;
-    L.p.out = static_cast<__nv_bfloat16*>(dx);
-    L.p.mprev = mprev;
-    L.p.dz_out = static_cast<__nv_bfloat16*>(dz_out);
     L.n_layers = 1;
     const int sms = sm_count();
     const int grid = L.p.n_units < sms ? L.p.n_units : sms;
@@ -396,7 +361,7 @@ int dw_bf16(const Shape& sh, const void* x, const void* dz, unsigned flags, floa
         !map_f32_patches(&maps[4], dWs, d, d) || !map_f32_patches(&maps[5], dWn, d, d))
         return HCW_ERR_CUDA;
     maps[2] = maps[1];   // unused by the weight gradient
-    L.layer[0] = {sh.s, k, nullptr, nullptr, nullptr};
+    L.layer[0] = {sh.s, k, nullptr, nullptr, nullptr, false, nullptr, false};
     TcParams& p = L.p;
     p.d = d;
     p.Mh = (int)(sh.tokens / 2);
@@ -411,9 +376,6 @@ int dw_bf16(const Shape& sh, const void* x, const void* dz, unsigned flags, floa
     p.splits_max = w.splits_max;
     p.causal = (flags & HCW_CAUSAL) ? 1 : 0;
     p.n_units = w.units;
-    p.dw_self = dWs;
-    p.dw_nbr = dWn;
-    p.dw_partial = part;
     p.timeout_ns = g_timeout_ns;
     L.n_layers = 1;
     const int sms = sm_count();
@@ -421,7 +383,7 @@ int dw_bf16(const Shape& sh, const void* x, const void* dz, unsigned flags, floa
     int rc = launched(launch_tc(MODE_DW, BN, L, grid, st), 1);
     if (rc) return rc;
     if (w.splits_max > 1) {
-        rc = launched(launch_splitk_reduce(p.dw_partial, w.splits_max, w.splits_self,
+        rc = launched(launch_splitk_reduce(part, w.splits_max, w.splits_self,
                                            w.splits_nbr, d, dWs, dWn, st),
                       1);
         if (rc) return rc;
@@ -519,6 +481,260 @@ int layer_bwd_impl(const Shape& sh, int dtype, const void* x, const void* z, con
     rc = layer_dx_impl(sh, dtype, dz, dy, Ws, Wn, flags, dx, st);
     if (rc) return rc;
     return layer_dw_impl(sh, dtype, x, dz, flags, dWs, dWn, dbias, wsb + lay.w_off, st);
+}
+
+// ------------------------------------------------------------ stack backward
+// Workspace of hcw_stack_bwd.
+//   bf16: dz of every layer [L] (+ the output gradient g of every layer with
+//   ReLU and residual), completion counters of the stacked input-gradient
+//   launch, the weight-gradient workspace (used only when the layers are run
+//   one by one), column-sum partials of every layer's dbias.
+//   fp32: two output-gradient and two dz buffers, the weight-gradient workspace.
+struct StackBwdLayout {
+    size_t dz_off, g_off, ctr_off, w_off, col_off, total;
+};
+
+StackBwdLayout stack_bwd_layout(const Shape& sh, int dtype, unsigned flags, int L) {
+    StackBwdLayout l;
+    const size_t a = align256(sh.act_bytes);
+    const WsLayout w = ws_layout(sh.tokens, sh.d, dtype, flags);
+    if (dtype == HCW_BF16) {
+        const bool keep_g = (flags & HCW_ACT_RELU) && (flags & HCW_RESIDUAL);
+        l.dz_off = 0;
+        l.g_off = (size_t)L * a;
+        l.ctr_off = l.g_off + (keep_g ? (size_t)L * a : 0);
+        l.w_off = l.ctr_off + stack_counter_bytes(sh.tokens, L);
+        l.col_off = l.w_off + w.w_bytes;
+        l.total = l.col_off + (size_t)L * align256(colsum_workspace_bytes(sh.tokens, sh.d));
+    } else {
+        l.dz_off = 0;
+        l.g_off = 2 * a;
+        l.ctr_off = l.w_off = 4 * a;
+        l.col_off = l.w_off;
+        l.total = l.w_off + w.w_bytes;
+    }
+    return l;
+}
+
+struct StackBwdArgs {
+    const void* x;
+    const void* acts;
+    const void* masks;
+    const void* dy;
+    const uint8_t* Ws;
+    const uint8_t* Wn;
+    int layer0, L, dim_override;
+    unsigned flags;
+    void* dx;
+    float* dWs;
+    float* dWn;
+    float* dbias;
+    uint8_t* ws;
+};
+
+int layer_dim(const Shape& sh, const StackBwdArgs& a, int l) {
+    return a.dim_override >= 0 ? a.dim_override : (a.layer0 + l) % sh.b;
+}
+
+// bf16: the relu gradient of the top layer, one stacked input-gradient
+// launch per run of <= 16 layers (top down; the ReLU gradient of the layer
+// below fused in), then one weight-gradient launch over all layers and one
+// batched column sum for the biases.
+int stack_bwd_bf16(const Shape& sh, const StackBwdArgs& a, const StackBwdLayout& lay,
+                   cudaStream_t st) {
+    const int d = sh.d, BN = pick_bn(d), L = a.L;
+    const bool relu = (a.flags & HCW_ACT_RELU) != 0;
+    const bool resid = (a.flags & HCW_RESIDUAL) != 0;
+    const size_t ab = sh.act_bytes, a256 = align256(ab), wb = (size_t)d * d * 2;
+    const size_t mb = mask_bytes(sh);
+    auto dz = [&](int l) -> void* { return a.ws + lay.dz_off + (size_t)l * a256; };
+    auto gbuf = [&](int l) -> void* { return a.ws + lay.g_off + (size_t)l * a256; };
+    auto act = [&](int l) -> const void* {
+        return l == 0 ? a.x : static_cast<const uint8_t*>(a.acts) + (size_t)(l - 1) * ab;
+    };
+    auto mask = [&](int l) {
+        return reinterpret_cast<const uint32_t*>(static_cast<const uint8_t*>(a.masks) +
+                                                 (size_t)l * mb);
+    };
+    // output gradient g_l of layer l (the residual term of its input gradient)
+    auto g = [&](int l) -> const void* {
+        if (l == L - 1) return a.dy;
+        return (relu && resid) ? gbuf(l) : dz(l);
+    };
+    int rc;
+    // dz of the top layer
+    if (relu) {
+        rc = launched(launch_relu_grad_mask_bf16(static_cast<const __nv_bfloat16*>(a.dy),
+                                                 mask(L - 1), static_cast<__nv_bfloat16*>(dz(L - 1)),
+                                                 sh.tokens, d, st),
+                      1);
+    } else {
+        rc = cuda_status(cudaMemcpyAsync(dz(L - 1), a.dy, ab, cudaMemcpyDeviceToDevice, st));
+    }
+    if (rc) return rc;
+    // input gradients, top down
+    int* counters = reinterpret_cast<int*>(a.ws + lay.ctr_off);
+    const int n_chunks = (int)((sh.tokens + 127) / 128);
+    static thread_local TcLaunch<kMaxStackLayers> T;
+    for (int top = L - 1; top >= 0; top -= kMaxStackLayers) {
+        const int cnt = top + 1 < kMaxStackLayers ? top + 1 : kMaxStackLayers;
+        memset(&T, 0, sizeof(T));
+        const int pw = BN >= 128 ? 64 : 32;
+        for (int i = 0; i < cnt; ++i) {
+            const int l = top - i;
+            const int s = layer_dim(sh, a, l);
+            const int k = 1 << s;
+            // stores: g_{l-1} (map 4) and dz_{l-1} (map 5); at l = 0 the stack's dx
+            void* out = l == 0 ? a.dx : (relu ? (resid ? gbuf(l - 1) : nullptr) : dz(l - 1));
+            void* dzo = (l > 0 && relu) ? dz(l - 1) : nullptr;
+            CUtensorMap* m = T.maps[i];
+            const void* res = resid ? g(l) : dz(l);
+            if (!map_rows(&m[0], dz(l), sh.tokens, d, k, 128) ||
+                !map_weight(&m[1], a.Ws + l * wb, d, 64) || !map_weight(&m[2], a.Wn + l * wb, d, 64) ||
+                !map_rows(&m[3], res, sh.tokens, d, k, 32, pw) ||
+                !map_rows(&m[4], out ? out : dzo, sh.tokens, d, k, 32, pw) ||
+                !map_rows(&m[5], dzo ? dzo : out, sh.tokens, d, k, 32, pw))
+                return HCW_ERR_CUDA;
+            T.layer[i] = {s, k, nullptr, nullptr, nullptr, out != nullptr,
+                          dzo ? mask(l - 1) : nullptr, dzo != nullptr};
+        }
+        row_unit_params(T.p, sh, BN, a.flags, true);
+        T.p.flags = a.flags & HCW_RESIDUAL;
+        T.n_layers = cnt;
+        T.counters = counters;
+        T.n_chunks = n_chunks;
+        T.tokens = (int)sh.tokens;
+        if (cudaMemsetAsync(counters, 0, (size_t)cnt * n_chunks * sizeof(int), st) != cudaSuccess)
+            return HCW_ERR_CUDA;
+        const int sms = sm_count();
+        const int total = T.p.n_units * cnt;
+        rc = launched(launch_tc_stack(MODE_DX, BN, T, total < sms ? total : sms, st), 1);
+        if (rc) return rc;
+    }
+    // weight gradients: runs of up to 16 independent layers in one launch,
+    // whole token range per tile; too few tiles to fill the GPU -> per layer
+    const WPlan w1 = plan_dw(sh.tokens, d, a.flags);
+    const int tiles = w1.n_ot * w1.n_nt;
+    const int sms = sm_count();
+    for (int l0 = 0; l0 < L; l0 += kMaxStackLayers) {
+        const int cnt = L - l0 < kMaxStackLayers ? L - l0 : kMaxStackLayers;
+        if (cnt * tiles * 2 < sms) {
+            for (int l = l0; l < l0 + cnt; ++l) {
+                Shape shl = sh;
+                shl.s = layer_dim(sh, a, l);
+                rc = dw_bf16(shl, act(l), dz(l), a.flags, a.dWs + (size_t)l * d * d,
+                             a.dWn + (size_t)l * d * d, nullptr, a.ws + lay.w_off, st);
+                if (rc) return rc;
+            }
+            continue;
+        }
+        memset(&T, 0, sizeof(T));
+        for (int i = 0; i < cnt; ++i) {
+            const int l = l0 + i;
+            const int s = layer_dim(sh, a, l);
+            const int k = 1 << s;
+            CUtensorMap* m = T.maps[i];
+            if (!map_rows(&m[0], dz(l), sh.tokens, d, k, 64) ||
+                !map_rows(&m[1], act(l), sh.tokens, d, k, 64) ||
+                !map_f32_patches(&m[4], a.dWs + (size_t)l * d * d, d, d) ||
+                !map_f32_patches(&m[5], a.dWn + (size_t)l * d * d, d, d))
+                return HCW_ERR_CUDA;
+            m[2] = m[1];
+            m[3] = m[4];
+            T.layer[i] = {s, k, nullptr, nullptr, nullptr, false, nullptr, false};
+        }
+        TcParams& p = T.p;
+        memset(&p, 0, sizeof(p));
+        p.d = d;
+        p.Mh = (int)(sh.tokens / 2);
+        p.n_nt = w1.n_nt;
+        p.n_ot = w1.n_ot;
+        p.qb = w1.qb;
+        p.nkb_self = w1.nkb_self;
+        p.nkb_nbr = w1.nkb_nbr;
+        p.kb_per_unit = w1.nkb_self > w1.nkb_nbr ? w1.nkb_self : w1.nkb_nbr;
+        p.splits_self = 1;
+        p.splits_nbr = 1;
+        p.splits_max = 1;
+        p.causal = (a.flags & HCW_CAUSAL) ? 1 : 0;
+        p.n_units = tiles * 2;
+        p.timeout_ns = g_timeout_ns;
+        T.n_layers = cnt;
+        const int total = p.n_units * cnt;
+        rc = launched(launch_tc_stack(MODE_DW, BN, T, total < sms ? total : sms, st), 1);
+        if (rc) return rc;
+    }
+    // bias gradients of every layer: one batched column sum (the dz buffers
+    // are contiguous when the activation size is a multiple of 256 bytes)
+    if (a.dbias && a256 != ab) {
+        for (int l = 0; l < L; ++l) {
+            rc = launched(launch_colsum_bf16(static_cast<const __nv_bfloat16*>(dz(l)), sh.tokens, d,
+                                             reinterpret_cast<float*>(a.ws + lay.col_off),
+                                             a.dbias + (size_t)l * d, st),
+                          2);
+            if (rc) return rc;
+        }
+        return HCW_OK;
+    }
+    if (a.dbias)
+        return launched(launch_colsum_bf16_batched(static_cast<const __nv_bfloat16*>(dz(0)), L,
+                                                   sh.tokens, d,
+                                                   reinterpret_cast<float*>(a.ws + lay.col_off),
+                                                   a.dbias, st),
+                        2);
+    return HCW_OK;
+}
+
+// fp32: layer by layer (the correctness path).
+int stack_bwd_f32(const Shape& sh, const StackBwdArgs& a, const StackBwdLayout& lay,
+                  cudaStream_t st) {
+    const int d = sh.d, L = a.L;
+    const bool relu = (a.flags & HCW_ACT_RELU) != 0;
+    const size_t ab = sh.act_bytes, a256 = align256(ab), wb = (size_t)d * d * 4;
+    const size_t mb = mask_bytes(sh);
+    uint8_t* g[2] = {a.ws + lay.g_off, a.ws + lay.g_off + a256};
+    uint8_t* dzb[2] = {a.ws, a.ws + a256};
+    auto mask = [&](int l) {
+        return reinterpret_cast<const uint32_t*>(static_cast<const uint8_t*>(a.masks) +
+                                                 (size_t)l * mb);
+    };
+    const void* cur_g = a.dy;
+    const void* cur_dz = a.dy;
+    int rc;
+    if (relu) {
+        rc = launched(launch_relu_grad_mask_f32(static_cast<const float*>(a.dy), mask(L - 1),
+                                                reinterpret_cast<float*>(dzb[(L - 1) & 1]),
+                                                sh.tokens, d, st),
+                      1);
+        if (rc) return rc;
+        cur_dz = dzb[(L - 1) & 1];
+    }
+    for (int l = L - 1; l >= 0; --l) {
+        Shape shl = sh;
+        shl.s = layer_dim(sh, a, l);
+        const void* in = l == 0 ? a.x : static_cast<const uint8_t*>(a.acts) + (size_t)(l - 1) * ab;
+        rc = layer_dw_impl(shl, HCW_F32, in, cur_dz, a.flags, a.dWs + (size_t)l * d * d,
+                           a.dWn + (size_t)l * d * d, a.dbias ? a.dbias + (size_t)l * d : nullptr,
+                           a.ws + lay.w_off, st);
+        if (rc) return rc;
+        void* out_g = l == 0 ? a.dx : (void*)g[l & 1];
+        rc = layer_dx_impl(shl, HCW_F32, cur_dz, cur_g, a.Ws + l * wb, a.Wn + l * wb, a.flags,
+                           out_g, st);
+        if (rc) return rc;
+        if (l == 0) break;
+        const void* next_dz = out_g;
+        if (relu) {
+            rc = launched(launch_relu_grad_mask_f32(static_cast<const float*>(out_g), mask(l - 1),
+                                                    reinterpret_cast<float*>(dzb[(l - 1) & 1]),
+                                                    sh.tokens, d, st),
+                          1);
+            if (rc) return rc;
+            next_dz = dzb[(l - 1) & 1];
+        }
+        cur_g = out_g;
+        cur_dz = next_dz;
+    }
+    return HCW_OK;
 }
 
 int check_fwd_ptrs(const Shape& sh, int dtype, const void* x, const void* Ws, const void* Wn,
@@ -767,15 +983,10 @@ int hcw_stack_fwd(const void* x, const void* W_self, const void* W_nbr, const fl
     return HCW_OK;
 }
 
-size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags) {
+size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags, int L) {
     Shape sh;
-    if (check_shape(0, -1, B, n, d, dtype, flags, &sh)) return 0;
-    // two output-gradient buffers, kStackSlots pre-activation-gradient slots
-    // (rotated so that a weight gradient on the side stream keeps its input
-    // while the input-gradient chain moves on), and the weight-gradient
-    // workspace the side stream reuses layer after layer
-    return ws_layout(sh.tokens, d, dtype, flags).w_bytes +
-           (2 + kStackSlots) * align256(sh.act_bytes);
+    if (L < 1 || check_shape(0, -1, B, n, d, dtype, flags, &sh)) return 0;
+    return stack_bwd_layout(sh, dtype, flags, L).total;
 }
 
 int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void* dy,
@@ -796,16 +1007,14 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void
         return cuda_status(e);
     }
     const bool relu = (flags & HCW_ACT_RELU) != 0;
-    const bool resid = (flags & HCW_RESIDUAL) != 0;
     if ((L > 1 && !acts) || (relu && !masks)) return HCW_ERR_INVALID_ARG;
     rc = check_bwd_ptrs(sh, dtype, flags & ~HCW_ACT_RELU, x, nullptr, dy, W_self, W_nbr, dx,
                         dW_self, dW_nbr, dbias);
     if (rc) return rc;
     if ((acts && !aligned16(acts)) || (masks && !aligned16(masks))) return HCW_ERR_ALIGNMENT;
-    const size_t ab = sh.act_bytes, wb = (size_t)d * d * elem_size(dtype);
-    const size_t gb = (size_t)d * d * 4, mb = mask_bytes(sh);
-    const size_t need = hcw_stack_workspace_bytes(B, n, d, dtype, flags);
-    if (ws_bytes < need || !workspace) return HCW_ERR_WORKSPACE;
+    const size_t ab = sh.act_bytes, gb = (size_t)d * d * 4, mb = mask_bytes(sh);
+    const StackBwdLayout lay = stack_bwd_layout(sh, dtype, flags, L);
+    if (ws_bytes < lay.total || !workspace) return HCW_ERR_WORKSPACE;
     if (!aligned16(workspace)) return HCW_ERR_ALIGNMENT;
     const size_t acts_b = (size_t)(L > 1 ? L - 1 : 0) * ab;
     if (overlaps(workspace, ws_bytes, dx, ab) || overlaps(workspace, ws_bytes, dy, ab) ||
@@ -814,98 +1023,24 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void
         overlaps(dW_self, (size_t)L * gb, dW_nbr, (size_t)L * gb) || overlaps(dx, ab, acts, acts_b) ||
         overlaps(dx, ab, masks, relu ? (size_t)L * mb : 0))
         return HCW_ERR_ALIASING;
-    cudaStream_t st = (cudaStream_t)stream;
-    uint8_t* wsb = static_cast<uint8_t*>(workspace);
-    const size_t ab256 = align256(ab);
-    uint8_t* g[2] = {wsb, wsb + ab256};     // output gradients (residual terms)
-    uint8_t* slot[kStackSlots];             // pre-activation gradients dz_m in slot m % 3
-    for (int i = 0; i < kStackSlots; ++i) slot[i] = wsb + (2 + i) * ab256;
-    uint8_t* wws = wsb + (2 + kStackSlots) * ab256;   // weight-gradient workspace
-    auto act_ptr = [&](int l) { return static_cast<const uint8_t*>(acts) + (size_t)l * ab; };
-    auto mask_ptr = [&](int l) {
-        return reinterpret_cast<const uint32_t*>(static_cast<const uint8_t*>(masks) +
-                                                 (size_t)l * mb);
-    };
-    std::lock_guard<std::mutex> lock(g_side_mu);
-    SideStream* ss = nullptr;
-    rc = side_stream(2 * L + 1, &ss);
-    if (rc) return rc;
-    cudaEvent_t* ev_ready = ss->events.data();       // dz_l written (main stream)
-    cudaEvent_t* ev_done = ev_ready + L;             // weight gradient of layer l done (side)
-    cudaEvent_t ev_fork = ev_ready[2 * L];
-    cudaStream_t side = ss->stream;
-    auto cu = [](cudaError_t e) { return e == cudaSuccess ? (int)HCW_OK : (int)HCW_ERR_CUDA; };
-    // the side stream starts after everything the caller queued before this call
-    if ((rc = cu(cudaEventRecord(ev_fork, st)))) return rc;
-    if ((rc = cu(cudaStreamWaitEvent(side, ev_fork, 0)))) return rc;
-    // gradient at the output (cur_g) and at the pre-activation (cur_dz) of layer l
-    const void* cur_g = dy;
-    const void* cur_dz = dy;
-    if (relu) {
-        void* dz_top = slot[(L - 1) % kStackSlots];
-        rc = launched(dtype == HCW_BF16
-                          ? launch_relu_grad_mask_bf16(static_cast<const __nv_bfloat16*>(dy),
-                                                       mask_ptr(L - 1),
-                                                       static_cast<__nv_bfloat16*>(dz_top),
-                                                       sh.tokens, d, st)
-                          : launch_relu_grad_mask_f32(static_cast<const float*>(dy), mask_ptr(L - 1),
-                                                      static_cast<float*>(dz_top), sh.tokens, d, st),
-                      1);
-        if (rc) return rc;
-        cur_dz = dz_top;
-    }
-    if ((rc = cu(cudaEventRecord(ev_ready[L - 1], st)))) return rc;
-    for (int l = L - 1; l >= 0; --l) {
-        Shape shl = sh;
-        shl.s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
-        const void* in = l == 0 ? x : act_ptr(l - 1);
-        const void* Wsl = static_cast<const uint8_t*>(W_self) + l * wb;
-        const void* Wnl = static_cast<const uint8_t*>(W_nbr) + l * wb;
-        // weight gradient of layer l on the side stream, once dz_l exists
-        if ((rc = cu(cudaStreamWaitEvent(side, ev_ready[l], 0)))) return rc;
-        rc = layer_dw_impl(shl, dtype, in, cur_dz, flags, dW_self + (size_t)l * d * d,
-                           dW_nbr + (size_t)l * d * d, dbias ? dbias + (size_t)l * d : nullptr,
-                           wws, side);
-        if (rc) return rc;
-        if ((rc = cu(cudaEventRecord(ev_done[l], side)))) return rc;
-        // input gradient of layer l on the caller's stream
-        if (l == 0) {
-            rc = layer_dx_impl(shl, dtype, cur_dz, cur_g, Wsl, Wnl, flags, dx, st);
-            if (rc) return rc;
-            break;
-        }
-        // dz_{l-1} goes to slot (l-1) % 3, last used by dz_{l+2}: its weight
-        // gradient must be done with it
-        uint8_t* dst = slot[(l - 1) % kStackSlots];
-        if (l + 2 <= L - 1 && (rc = cu(cudaStreamWaitEvent(st, ev_done[l + 2], 0)))) return rc;
-        void* out_g;
-        void* next_dz;
-        if (!relu) {
-            out_g = dst;       // without an activation dz = g
-            next_dz = dst;
-            rc = layer_dx_impl(shl, dtype, cur_dz, cur_g, Wsl, Wnl, flags, out_g, st);
-        } else if (dtype == HCW_BF16) {
-            // the input-gradient kernel also applies the ReLU gradient of layer l-1
-            out_g = resid ? (void*)g[l & 1] : nullptr;
-            next_dz = dst;
-            rc = dx_bf16(shl, cur_dz, cur_g, Wsl, Wnl, flags, out_g, st, mask_ptr(l - 1), next_dz);
-        } else {
-            out_g = g[l & 1];
-            next_dz = dst;
-            rc = layer_dx_impl(shl, dtype, cur_dz, cur_g, Wsl, Wnl, flags, out_g, st);
-            if (!rc)
-                rc = launched(launch_relu_grad_mask_f32(static_cast<const float*>(out_g),
-                                                        mask_ptr(l - 1), static_cast<float*>(next_dz),
-                                                        sh.tokens, d, st),
-                              1);
-        }
-        if (rc) return rc;
-        if ((rc = cu(cudaEventRecord(ev_ready[l - 1], st)))) return rc;
-        cur_g = out_g;
-        cur_dz = next_dz;
-    }
-    // join: the caller's stream waits for the last weight gradient
-    return cu(cudaStreamWaitEvent(st, ev_done[0], 0));
+    StackBwdArgs a;
+    a.x = x;
+    a.acts = acts;
+    a.masks = masks;
+    a.dy = dy;
+    a.Ws = static_cast<const uint8_t*>(W_self);
+    a.Wn = static_cast<const uint8_t*>(W_nbr);
+    a.layer0 = layer0;
+    a.L = L;
+    a.dim_override = dim_override;
+    a.flags = flags;
+    a.dx = dx;
+    a.dWs = dW_self;
+    a.dWn = dW_nbr;
+    a.dbias = dbias;
+    a.ws = static_cast<uint8_t*>(workspace);
+    return dtype == HCW_BF16 ? stack_bwd_bf16(sh, a, lay, (cudaStream_t)stream)
+                             : stack_bwd_f32(sh, a, lay, (cudaStream_t)stream);
 }
 
 unsigned long long hcw_launch_count(void) { return g_launches.load(); }

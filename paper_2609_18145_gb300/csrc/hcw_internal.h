@@ -40,12 +40,6 @@ struct TcParams {
     int n_units;    // units of one layer
     // epilogue
     unsigned flags;
-    __nv_bfloat16* out;           // DX: dx (may be null when dz_out is set)
-    const uint32_t* mprev;        // DX: ReLU mask words of the layer below (fused ReLU grad)
-    __nv_bfloat16* dz_out;        // DX: that layer's gradient dz = dx * mask, or null
-    float* dw_self;               // DW destination when splits_self == 1
-    float* dw_nbr;                // DW destination when splits_nbr == 1
-    float* dw_partial;            // DW partials [2][splits_max][d][d]
     int splits_max;
     unsigned long long timeout_ns;
 };
@@ -58,6 +52,9 @@ struct TcLayer {
     const float* bias;            // FWD bias or null
     uint32_t* mout;               // FWD: ReLU mask words [tokens][d/32], bit e = (z > 0), or null
     __nv_bfloat16* zout;          // FWD: bf16 pre-activation (layer API), or null
+    bool out;                     // DX: the input gradient dx is stored (map 4)
+    const uint32_t* mprev;        // DX: ReLU mask words of the layer below (fused ReLU grad)
+    bool dz_out;                  // DX: dz of the layer below = dx * mask is stored (map 5)
 };
 
 constexpr int kMaxStackLayers = 16;   // layers per stacked-forward launch
@@ -79,9 +76,11 @@ struct TcLaunch {
 
 // Launch one tensor-core pass (one layer).
 cudaError_t launch_tc(int mode, int BN, const TcLaunch<1>& L, int grid, cudaStream_t stream);
-// Launch the stacked forward over L.n_layers consecutive layers.
-cudaError_t launch_tc_stack_fwd(int BN, const TcLaunch<kMaxStackLayers>& L, int grid,
-                                cudaStream_t stream);
+// Launch a run of layers: MODE_FWD (layers in order) or MODE_DX (layers from
+// the top down) with chunk-level dependencies, or MODE_DW (independent
+// layers, the long self-part units of every layer first).
+cudaError_t launch_tc_stack(int mode, int BN, const TcLaunch<kMaxStackLayers>& L, int grid,
+                            cudaStream_t stream);
 
 // Dynamic shared memory the tensor-core kernel uses for this N tile.
 size_t tc_smem_bytes(int BN);
@@ -113,6 +112,10 @@ cudaError_t launch_colsum_f32(const float* dz, long long rows, int d, float* par
                               float* out, cudaStream_t st);
 cudaError_t launch_colsum_bf16(const __nv_bfloat16* dz, long long rows, int d, float* partial,
                                float* out, cudaStream_t st);
+// The same for `batch` consecutive [rows][d] matrices: out [batch][d], partial
+// batch * colsum_workspace_bytes(rows, d).
+cudaError_t launch_colsum_bf16_batched(const __nv_bfloat16* dz, int batch, long long rows, int d,
+                                       float* partial, float* out, cudaStream_t st);
 // out_w[o][k] = sum_{s < splits_w} partial[w][s][o][k] for w in {self, nbr}
 cudaError_t launch_splitk_reduce(const float* partial, int splits_max, int splits_self,
                                  int splits_nbr, int d, float* dWs, float* dWn,

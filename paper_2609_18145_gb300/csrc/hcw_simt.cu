@@ -224,6 +224,9 @@ template <typename V>
 __global__ void colsum_partial_kernel(const V* __restrict__ dz, long long rows, int d,
                                       float* __restrict__ partial) {
     __shared__ float red[8][33];
+    // blockIdx.z selects one of several equally shaped matrices (layers)
+    dz += (size_t)blockIdx.z * rows * d;
+    partial += (size_t)blockIdx.z * gridDim.y * d;
     const int o = blockIdx.x * 32 + threadIdx.x;
     const long long r0 = (long long)blockIdx.y * kColRows;
     const long long r1 = min(rows, r0 + kColRows);
@@ -242,6 +245,8 @@ __global__ void colsum_partial_kernel(const V* __restrict__ dz, long long rows, 
 __global__ void colsum_final_kernel(const float* __restrict__ partial, int chunks, int d,
                                     float* __restrict__ out) {
     const int o = blockIdx.x * blockDim.x + threadIdx.x;
+    partial += (size_t)blockIdx.y * chunks * d;
+    out += (size_t)blockIdx.y * d;
     if (o >= d) return;
     float s = 0.f;
     for (int c = 0; c < chunks; ++c) s += partial[(long long)c * d + o];
@@ -345,16 +350,21 @@ size_t colsum_workspace_bytes(long long rows, int d) {
 
 template <typename V>
 static cudaError_t colsum(const V* dz, long long rows, int d, float* partial, float* out,
-                          cudaStream_t st) {
+                          cudaStream_t st, int batch = 1) {
     const long long chunks = (rows + kColRows - 1) / kColRows;
     if (chunks == 0) {
-        cudaError_t e = cudaMemsetAsync(out, 0, (size_t)d * sizeof(float), st);
+        cudaError_t e = cudaMemsetAsync(out, 0, (size_t)batch * d * sizeof(float), st);
         return e;
     }
-    dim3 grid((d + 31) / 32, (unsigned)chunks);
+    dim3 grid((d + 31) / 32, (unsigned)chunks, (unsigned)batch);
     colsum_partial_kernel<V><<<grid, dim3(32, 8), 0, st>>>(dz, rows, d, partial);
-    colsum_final_kernel<<<(d + 127) / 128, 128, 0, st>>>(partial, (int)chunks, d, out);
+    colsum_final_kernel<<<dim3((d + 127) / 128, batch), 128, 0, st>>>(partial, (int)chunks, d, out);
     return cudaGetLastError();
+}
+
+cudaError_t launch_colsum_bf16_batched(const __nv_bfloat16* dz, int batch, long long rows, int d,
+                                       float* partial, float* out, cudaStream_t st) {
+    return colsum<__nv_bfloat16>(dz, rows, d, partial, out, st, batch);
 }
 
 cudaError_t launch_colsum_f32(const float* dz, long long rows, int d, float* partial,

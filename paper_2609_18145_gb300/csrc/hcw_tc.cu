@@ -145,6 +145,30 @@ __device__ __forceinline__ WUnit decode_w_unit(const TcParams& p, int u) {
     return w;
 }
 
+// Weight-gradient unit u of a launch.  One layer: decode_w_unit.  A run of
+// independent layers: every layer's self-part units first (the long ones),
+// then the partner-part units, layer-major inside each group.
+__device__ __forceinline__ WUnit decode_w_any(const TcParams& p, int u, bool stacked,
+                                              int n_layers, int& layer) {
+    if (!stacked) {
+        layer = 0;
+        return decode_w_unit(p, u);
+    }
+    const int tiles = p.n_ot * p.n_nt;
+    const int self_pl = tiles * p.splits_self;
+    const int nbr_pl = tiles * p.splits_nbr;
+    int local;
+    if (u < n_layers * self_pl) {
+        layer = u / self_pl;
+        local = u - layer * self_pl;
+    } else {
+        const int v = u - n_layers * self_pl;
+        layer = v / nbr_pl;
+        local = self_pl + (v - layer * nbr_pl);
+    }
+    return decode_w_unit(p, local);
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
     __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
     return *reinterpret_cast<uint32_t*>(&h);
@@ -318,8 +342,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             bool ok = true;
             int ordinal = 0;
             for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x, ++ordinal) {
-                const int l = STACKED ? u / upl : 0;
+                int l = STACKED ? u / upl : 0;
                 const int ul = STACKED ? u - l * upl : u;
+                WUnit w{};
+                if (MODE == MODE_DW) w = decode_w_any(p, u, STACKED, L.n_layers, l);
                 const TcLayer& ly = L.layer[l];
                 const CUtensorMap* mA = &L.maps[l][0];
                 if (MODE != MODE_DW) {
@@ -371,7 +397,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                     }
                 } else {
-                    const WUnit w = decode_w_unit(p, ul);
                     st_release_cta_shared(&bars->dep_unit, ordinal);
                     for (int kb = w.kb0; kb < w.kb1; ++kb) {
                         if (!mbar_wait(&bars->empty[stage], phase ^ 1, abort, tmo)) {
@@ -434,7 +459,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (MODE != MODE_DW) {
                     steps = decode_row_unit(p, ul, STACKED).steps;
                 } else {
-                    const WUnit w = decode_w_unit(p, ul);
+                    int lw;
+                    const WUnit w = decode_w_any(p, u, STACKED, L.n_layers, lw);
                     steps = w.kb1 - w.kb0;
                 }
                 if (!mbar_wait(&bars->tempty[acc], acc_phase ^ 1, abort, tmo)) {
@@ -540,8 +566,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             return __shfl_sync(0xffffffffu, ok, 0) != 0;
         };
         for (int u = blockIdx.x; u < n_units && alive; u += gridDim.x, ++ordinal) {
-            const int l = STACKED ? u / upl : 0;
+            int l = STACKED ? u / upl : 0;
             const int ul = STACKED ? u - l * upl : u;
+            WUnit wu{};
+            if (MODE == MODE_DW) wu = decode_w_any(p, u, STACKED, L.n_layers, l);
             const TcLayer& ly = L.layer[l];
             if (MODE != MODE_DW) {
                 constexpr int SW = HALF >= 64 ? 64 : HALF;     // patch width (columns)
@@ -561,7 +589,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const bool inside = qw < p.Mh;
                 const bool has_res = (p.flags & 2u) != 0 && inside;
                 const bool fwd = MODE == MODE_FWD;
-                const bool has_mprev = MODE == MODE_DX && p.mprev != nullptr;
+                const bool has_mprev = MODE == MODE_DX && ly.mprev != nullptr && ly.dz_out;
                 const CUtensorMap* mE0 = &L.maps[l][3];
                 const CUtensorMap* mE1 = &L.maps[l][4];
                 const CUtensorMap* mE2 = &L.maps[l][5];
@@ -585,7 +613,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int c = 0; c < HALF / 32; ++c)
                     mp[c] = (has_mprev && tok_row >= 0)
-                                ? __ldg(p.mprev + (size_t)tok_row * wpr + (col_half >> 5) + c)
+                                ? __ldg(ly.mprev + (size_t)tok_row * wpr + (col_half >> 5) + c)
                                 : 0u;
                 if (fwd) {
                     // this warp's bias slice, read back as warp-wide broadcasts
@@ -682,7 +710,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (int i = 0; i < 16; ++i) gw[h][i] = pack_bf16x2(v[2 * i], v[2 * i + 1]);
                     }
                     // the patch: y (FWD) or dx (DX), written over the residual rows
-                    if (fwd || p.out) {
+                    if (fwd || ly.out) {
 #pragma unroll
                         for (int h = 0; h < SUB; ++h)
 #pragma unroll
@@ -698,7 +726,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     if (has_mprev) {
                         // fused ReLU gradient of the layer below: dz = dx * mask
-                        if (p.out) {
+                        if (ly.out) {
                             if (lane == 0) bulk_wait_read<0>();
                             __syncwarp();
                         }
@@ -741,7 +769,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     __syncwarp();
                 }
             } else {
-                const WUnit w = decode_w_unit(p, ul);
+                const WUnit& w = wu;
                 if (!wait_acc()) {
                     alive = false;
                     break;
@@ -827,11 +855,20 @@ cudaError_t launch_tc(int mode, int BN, const TcLaunch<1>& L, int grid, cudaStre
     return cudaErrorInvalidValue;
 }
 
-cudaError_t launch_tc_stack_fwd(int BN, const TcLaunch<kMaxStackLayers>& L, int grid,
-                                cudaStream_t st) {
-    if (BN == 256) return launch_one<MODE_FWD, 256, kMaxStackLayers>(L, grid, st);
-    if (BN == 128) return launch_one<MODE_FWD, 128, kMaxStackLayers>(L, grid, st);
-    if (BN == 64) return launch_one<MODE_FWD, 64, kMaxStackLayers>(L, grid, st);
+cudaError_t launch_tc_stack(int mode, int BN, const TcLaunch<kMaxStackLayers>& L, int grid,
+                            cudaStream_t st) {
+#define HCW_TC_STACK_CASE(M, N) \
+    if (mode == M && BN == N) return launch_one<M, N, kMaxStackLayers>(L, grid, st);
+    HCW_TC_STACK_CASE(MODE_FWD, 256)
+    HCW_TC_STACK_CASE(MODE_FWD, 128)
+    HCW_TC_STACK_CASE(MODE_FWD, 64)
+    HCW_TC_STACK_CASE(MODE_DX, 256)
+    HCW_TC_STACK_CASE(MODE_DX, 128)
+    HCW_TC_STACK_CASE(MODE_DX, 64)
+    HCW_TC_STACK_CASE(MODE_DW, 256)
+    HCW_TC_STACK_CASE(MODE_DW, 128)
+    HCW_TC_STACK_CASE(MODE_DW, 64)
+#undef HCW_TC_STACK_CASE
     return cudaErrorInvalidValue;
 }
 

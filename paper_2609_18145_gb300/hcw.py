@@ -62,7 +62,7 @@ _SIGNATURES = {
     "hcw_stack_fwd": ([_P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P, _SZ,
                        _P], _I),
     "hcw_stack_fwd_workspace_bytes": ([_I, _I, _I, _I, _U, _I], _SZ),
-    "hcw_stack_workspace_bytes": ([_I, _I, _I, _I, _U], _SZ),
+    "hcw_stack_workspace_bytes": ([_I, _I, _I, _I, _U, _I], _SZ),
     "hcw_stack_bwd": ([_P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P,
                        _P, _P, _SZ, _P], _I),
     "hcw_sync_status": ([_P], _I),
@@ -171,8 +171,8 @@ def hcw_workspace_bytes(B: int, n: int, d: int, dtype: int, flags: int) -> int:
     return int(lib().hcw_workspace_bytes(B, n, d, dtype, flags))
 
 
-def hcw_stack_workspace_bytes(B: int, n: int, d: int, dtype: int, flags: int) -> int:
-    return int(lib().hcw_stack_workspace_bytes(B, n, d, dtype, flags))
+def hcw_stack_workspace_bytes(B: int, n: int, d: int, dtype: int, flags: int, L: int) -> int:
+    return int(lib().hcw_stack_workspace_bytes(B, n, d, dtype, flags, L))
 
 
 def _workspace(nbytes, device, workspace):
@@ -287,7 +287,7 @@ def hcw_stack_bwd(x, acts, masks, dy, W_self, W_nbr, layer0: int = 0, dim_overri
     dW_nbr = torch.empty(L, d, d, **f32) if dW_nbr is None else dW_nbr
     if dbias is None and want_dbias:
         dbias = torch.empty(L, d, **f32)
-    need = hcw_stack_workspace_bytes(B, n, d, dt, flags)
+    need = hcw_stack_workspace_bytes(B, n, d, dt, flags, L)
     ws = _workspace(need, x.device, workspace)
     _check(lib().hcw_stack_bwd(_ptr(x), _ptr(acts), _ptr(masks), _ptr(dy), _ptr(W_self),
                                _ptr(W_nbr), layer0, L, dim_override, B, n, d, dt, flags,

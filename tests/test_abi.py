@@ -135,8 +135,8 @@ def test_workspace_sizes_f32(hcw):
     a = hcw.hcw_workspace_bytes(64, 256, 512, hcw.HCW_F32, 0)
     b = hcw.hcw_workspace_bytes(64, 256, 512, hcw.HCW_F32, hcw.HCW_ACT_RELU)
     assert b - a >= 64 * 256 * 512 * 4            # the masked gradient dz
-    s = hcw.hcw_stack_workspace_bytes(64, 256, 512, hcw.HCW_F32, 0)
-    assert s >= a + 2 * 64 * 256 * 512 * 4        # two gradient buffers between layers
+    s = hcw.hcw_stack_workspace_bytes(64, 256, 512, hcw.HCW_F32, 0, 16)
+    assert s >= a + 2 * 64 * 256 * 512 * 4        # gradient buffers between layers
     assert hcw.hcw_workspace_bytes(4, 48, 64, hcw.HCW_F32, 0) == 0   # invalid n
 
 
