@@ -481,7 +481,30 @@ def run_kernel_only(args):
     wws = torch.empty(max(1, H.hcw_layer_bwd_weight_workspace_bytes(B, n, d, H.HCW_BF16, flags)),
                       dtype=torch.uint8, device=dev)
     layer = 3
-    if args.kernel == "fwd":
+    if args.kernel == "step":
+        # one whole step (stack forward + stack backward) of --batch sequences
+        L = w["L"]
+        ps = synth.problem(1, n, d, L=L, seed=0, w_std=(1 / (2 * d)) ** 0.5)
+        SWs = torch.from_numpy(ps.W_self).to(torch.bfloat16).to(dev)
+        SWn = torch.from_numpy(ps.W_nbr).to(torch.bfloat16).to(dev)
+        Sb = torch.from_numpy(ps.bias).to(dev)
+        acts = torch.empty((L - 1, B, n, d), dtype=torch.bfloat16, device=dev)
+        masks = torch.empty((L, B, n, d // 32), dtype=torch.int32, device=dev)
+        sWs = torch.empty((L, d, d), dtype=torch.float32, device=dev)
+        sWn = torch.empty_like(sWs)
+        sb = torch.empty((L, d), dtype=torch.float32, device=dev)
+        dxs = torch.empty_like(x)
+        ws = torch.empty(H.hcw_stack_workspace_bytes(B, n, d, H.HCW_BF16, flags, L),
+                         dtype=torch.uint8, device=dev)
+        fws = torch.empty(max(1, H.hcw_stack_fwd_workspace_bytes(B, n, d, H.HCW_BF16, flags, L)),
+                          dtype=torch.uint8, device=dev)
+
+        def fn():
+            H.hcw_stack_fwd(x, SWs, SWn, Sb, 0, -1, flags, y=y, acts=acts, masks=masks,
+                            workspace=fws)
+            H.hcw_stack_bwd(x, acts, masks, dz, SWs, SWn, 0, -1, flags, dx=dxs, dW_self=sWs,
+                            dW_nbr=sWn, dbias=sb, workspace=ws)
+    elif args.kernel == "fwd":
         fn = lambda: H.hcw_layer_fwd(x, Ws, Wn, bias, layer, -1, flags, y=y, z_save=z)
     elif args.kernel == "dx":
         fn = lambda: H.hcw_layer_bwd_data(dz, dz, Ws, Wn, layer, -1, flags, dx=y)
@@ -500,8 +523,9 @@ def run_kernel_only(args):
     if H.hcw_sync_status() != H.HCW_OK:
         raise SystemExit("device error")
     ms = a.elapsed_time(b) / args.steps
+    flops = step_flops(B, n, d, w["L"]) if args.kernel == "step" else 3.0 * d * d * B * n
     print(json.dumps({"kernel": args.kernel, "batch": B, "n": n, "d": d, "avg_ms": ms,
-                      "tflops": 3.0 * d * d * B * n / (ms * 1e-3) / 1e12}), flush=True)
+                      "tflops": flops / (ms * 1e-3) / 1e12}), flush=True)
     return 0
 
 
@@ -516,8 +540,9 @@ def main():
                          "CUDA graph of them")
     ap.add_argument("--no-cpu-baseline", action="store_true",
                     help="skip timing the CPU oracle (it is only timed at N = 1 anyway)")
-    ap.add_argument("--kernel", choices=("fwd", "dx", "dw"),
-                    help="launch only this kernel kind (profiler captures); no JSON bench line")
+    ap.add_argument("--kernel", choices=("fwd", "dx", "dw", "step"),
+                    help="launch only this kernel kind, or one whole step of --batch "
+                         "sequences (profiler captures); no JSON bench line")
     ap.add_argument("--batch", type=int, default=64, help="sequences for --kernel runs")
     args = ap.parse_args()
     if args.kernel:

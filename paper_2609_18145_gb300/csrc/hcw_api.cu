@@ -256,7 +256,7 @@ void row_unit_params(TcParams& p, const Shape& sh, int BN, unsigned flags, bool 
 bool fwd_maps(CUtensorMap* m, const Shape& sh, int s, const void* x, const void* Ws,
               const void* Wn, const void* y) {
     const int d = sh.d, BN = pick_bn(d), k = 1 << s;
-    const int pw = BN >= 128 ? 64 : 32;   // epilogue patch width: 64 columns, 32 for narrow tiles
+    const int pw = epi_patch_cols(BN);
     if (!map_rows(&m[0], x, sh.tokens, d, k, 128) || !map_weight(&m[1], Ws, d, BN) ||
         !map_weight(&m[2], Wn, d, BN) || !map_rows(&m[3], x, sh.tokens, d, k, 32, pw) ||
         !map_rows(&m[4], y, sh.tokens, d, k, 32, pw))
@@ -284,7 +284,8 @@ int fwd_bf16(const Shape& sh, const void* x, const void* Ws, const void* Wn, con
 // group and 128-token chunk.
 size_t stack_counter_bytes(long long tokens, int L) {
     const int layers = L < kMaxStackLayers ? L : kMaxStackLayers;
-    return align256((size_t)layers * (size_t)((tokens + 127) / 128) * sizeof(int));
+    // per (layer, 128-token chunk) completion counters, then the unit counter
+    return align256((size_t)layers * (size_t)((tokens + 127) / 128) * sizeof(int) + 16);
 }
 
 // Layers [l0, l0 + n) of a bf16 stack in one persistent launch.  in_ptr(l),
@@ -311,7 +312,8 @@ int stack_fwd_group(const Shape& sh, int l0, int n, int layer0, int dim_override
     L.counters = counters;
     L.n_chunks = (int)((sh.tokens + 127) / 128);
     L.tokens = (int)sh.tokens;
-    cudaError_t e = cudaMemsetAsync(counters, 0, (size_t)n * L.n_chunks * sizeof(int), st);
+    L.sched = counters + (size_t)n * L.n_chunks;
+    cudaError_t e = cudaMemsetAsync(counters, 0, ((size_t)n * L.n_chunks + 1) * sizeof(int), st);
     if (e != cudaSuccess) return HCW_ERR_CUDA;
     const int sms = sm_count();
     const int total = L.p.n_units * n;
@@ -324,7 +326,7 @@ int dx_bf16(const Shape& sh, const void* dz, const void* dy, const void* Ws, con
             unsigned flags, void* dx, cudaStream_t st, const uint32_t* mprev = nullptr,
             void* dz_out = nullptr) {
     const int d = sh.d, BN = pick_bn(d), k = 1 << sh.s;
-    const int pw = BN >= 128 ? 64 : 32;
+    const int pw = epi_patch_cols(BN);
     TcLaunch<1> L;
     memset(&L, 0, sizeof(L));
     CUtensorMap* maps = L.maps[0];
@@ -579,7 +581,7 @@ int stack_bwd_bf16(const Shape& sh, const StackBwdArgs& a, const StackBwdLayout&
     for (int top = L - 1; top >= 0; top -= kMaxStackLayers) {
         const int cnt = top + 1 < kMaxStackLayers ? top + 1 : kMaxStackLayers;
         memset(&T, 0, sizeof(T));
-        const int pw = BN >= 128 ? 64 : 32;
+        const int pw = epi_patch_cols(BN);
         for (int i = 0; i < cnt; ++i) {
             const int l = top - i;
             const int s = layer_dim(sh, a, l);
@@ -604,7 +606,9 @@ int stack_bwd_bf16(const Shape& sh, const StackBwdArgs& a, const StackBwdLayout&
         T.counters = counters;
         T.n_chunks = n_chunks;
         T.tokens = (int)sh.tokens;
-        if (cudaMemsetAsync(counters, 0, (size_t)cnt * n_chunks * sizeof(int), st) != cudaSuccess)
+        T.sched = counters + (size_t)cnt * n_chunks;
+        if (cudaMemsetAsync(counters, 0, ((size_t)cnt * n_chunks + 1) * sizeof(int), st) !=
+            cudaSuccess)
             return HCW_ERR_CUDA;
         const int sms = sm_count();
         const int total = T.p.n_units * cnt;
@@ -660,6 +664,8 @@ int stack_bwd_bf16(const Shape& sh, const StackBwdArgs& a, const StackBwdLayout&
         p.n_units = tiles * 2;
         p.timeout_ns = g_timeout_ns;
         T.n_layers = cnt;
+        T.sched = counters;
+        if (cudaMemsetAsync(counters, 0, sizeof(int), st) != cudaSuccess) return HCW_ERR_CUDA;
         const int total = p.n_units * cnt;
         rc = launched(launch_tc_stack(MODE_DW, BN, T, total < sms ? total : sms, st), 1);
         if (rc) return rc;

@@ -57,6 +57,10 @@ struct TcLayer {
     bool dz_out;                  // DX: dz of the layer below = dx * mask is stored (map 5)
 };
 
+// Columns of one epilogue patch (the inner extent of the 32-row residual and
+// output boxes of the row kernels): 64 for 256-column tiles, else 32.
+constexpr int epi_patch_cols(int BN) { return BN >= 256 ? 64 : 32; }
+
 constexpr int kMaxStackLayers = 16;   // layers per stacked-forward launch
 
 // maps[l][0..5] = tmA, tmB0, tmB1, tmE0, tmE1, tmE2 of layer l, as documented
@@ -72,6 +76,7 @@ struct TcLaunch {
     int* counters;
     int n_chunks;
     int tokens;
+    int* sched;   // stacked launches: next unit to hand out (zeroed per launch), or null
 };
 
 // Launch one tensor-core pass (one layer).

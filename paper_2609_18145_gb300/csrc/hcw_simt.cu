@@ -202,43 +202,109 @@ __global__ void relu_grad_kernel(const V* __restrict__ dy, const V* __restrict__
         dz[t] = to_f(z[t]) > 0.f ? dy[t] : zero;
 }
 
-// dz[t][o] = mask bit (t, o) ? dy[t][o] : 0, masks as written by the forward.
-template <typename V>
-__global__ void relu_grad_mask_kernel(const V* __restrict__ dy, const uint32_t* __restrict__ mask,
-                                      V* __restrict__ dz, long long rows, int d) {
+// dz[t][o] = mask bit (t, o) ? dy[t][o] : 0, masks as written by the forward
+// (any d: rows of ceil(d / 32) mask words).
+__global__ void relu_grad_mask_f32_kernel(const float* __restrict__ dy,
+                                          const uint32_t* __restrict__ mask,
+                                          float* __restrict__ dz, long long rows, int d) {
     const int wpr = (d + 31) >> 5;
     const size_t count = (size_t)rows * d;
-    const V zero = V(0.f);
     for (size_t t = (size_t)blockIdx.x * blockDim.x + threadIdx.x; t < count;
          t += (size_t)gridDim.x * blockDim.x) {
         const size_t r = t / d;
         const int o = (int)(t - r * d);
-        dz[t] = (mask[r * wpr + (o >> 5)] >> (o & 31)) & 1u ? dy[t] : zero;
+        dz[t] = (mask[r * wpr + (o >> 5)] >> (o & 31)) & 1u ? dy[t] : 0.f;
+    }
+}
+
+// The same for bf16 rows (d a multiple of 64): one thread per 16 bytes of a
+// row, so a group never straddles a mask word.
+template <typename V>
+__global__ void relu_grad_mask_kernel(const V* __restrict__ dy, const uint32_t* __restrict__ mask,
+                                      V* __restrict__ dz, long long rows, int d) {
+    constexpr int VEC = 16 / sizeof(V);
+    const int wpr = d >> 5;
+    const int gpr = d / VEC;   // groups per row
+    const size_t count = (size_t)rows * gpr;
+    for (size_t t = (size_t)blockIdx.x * blockDim.x + threadIdx.x; t < count;
+         t += (size_t)gridDim.x * blockDim.x) {
+        const size_t r = t / gpr;
+        const int o = (int)(t - r * gpr) * VEC;
+        const uint32_t bits = (mask[r * wpr + (o >> 5)] >> (o & 31)) & ((1u << VEC) - 1u);
+        uint4 v = reinterpret_cast<const uint4*>(dy)[t];
+        uint32_t w[4] = {v.x, v.y, v.z, v.w};
+        if (VEC == 8) {
+#pragma unroll
+            for (int i = 0; i < 4; ++i)
+                w[i] &= ((bits >> (2 * i)) & 1u ? 0x0000FFFFu : 0u) |
+                        ((bits >> (2 * i + 1)) & 1u ? 0xFFFF0000u : 0u);
+        } else {
+#pragma unroll
+            for (int i = 0; i < 4; ++i) w[i] = (bits >> i) & 1u ? w[i] : 0u;
+        }
+        reinterpret_cast<uint4*>(dz)[t] = make_uint4(w[0], w[1], w[2], w[3]);
     }
 }
 
 constexpr int kColRows = 256;   // rows per partial of the column sum
 
-// partial[c][o] = sum_{r in chunk c} dz[r][o]  (block: 32 columns x 8 row lanes)
-template <typename V>
-__global__ void colsum_partial_kernel(const V* __restrict__ dz, long long rows, int d,
-                                      float* __restrict__ partial) {
+// partial[c][o] = sum_{r in chunk c} dz[r][o] for any d (block: 32 columns x
+// 8 row lanes).
+__global__ void colsum_partial_f32_kernel(const float* __restrict__ dz, long long rows, int d,
+                                          float* __restrict__ partial) {
     __shared__ float red[8][33];
-    // blockIdx.z selects one of several equally shaped matrices (layers)
-    dz += (size_t)blockIdx.z * rows * d;
-    partial += (size_t)blockIdx.z * gridDim.y * d;
     const int o = blockIdx.x * 32 + threadIdx.x;
     const long long r0 = (long long)blockIdx.y * kColRows;
     const long long r1 = min(rows, r0 + kColRows);
     float acc = 0.f;
     if (o < d)
-        for (long long r = r0 + threadIdx.y; r < r1; r += 8) acc += to_f(dz[r * d + o]);
+        for (long long r = r0 + threadIdx.y; r < r1; r += 8) acc += dz[r * d + o];
     red[threadIdx.y][threadIdx.x] = acc;
     __syncthreads();
     if (threadIdx.y == 0 && o < d) {
         float s = 0.f;
         for (int q = 0; q < 8; ++q) s += red[q][threadIdx.x];
         partial[(long long)blockIdx.y * d + o] = s;
+    }
+}
+
+// The same for bf16 rows (d a multiple of 64), 16-byte loads.  Block: 64
+// column groups of 16 bytes x 4 row lanes; each thread sums its group over every 4th row of
+// the chunk, then the 4 row lanes are added in a fixed order.
+template <typename V>
+__global__ void colsum_partial_kernel(const V* __restrict__ dz, long long rows, int d,
+                                      float* __restrict__ partial) {
+    constexpr int VEC = 16 / sizeof(V);
+    __shared__ float red[4][64][VEC + 1];
+    // blockIdx.z selects one of several equally shaped matrices (layers)
+    dz += (size_t)blockIdx.z * rows * d;
+    partial += (size_t)blockIdx.z * gridDim.y * d;
+    const int gpr = d / VEC;
+    const int g = blockIdx.x * 64 + threadIdx.x;
+    const long long r0 = (long long)blockIdx.y * kColRows;
+    const long long r1 = min(rows, r0 + kColRows);
+    float acc[VEC];
+#pragma unroll
+    for (int i = 0; i < VEC; ++i) acc[i] = 0.f;
+    if (g < gpr) {
+        const uint4* src = reinterpret_cast<const uint4*>(dz) + g;
+        for (long long r = r0 + threadIdx.y; r < r1; r += 4) {
+            const uint4 q = src[(size_t)r * gpr];
+            const V* e = reinterpret_cast<const V*>(&q);
+#pragma unroll
+            for (int i = 0; i < VEC; ++i) acc[i] += to_f(e[i]);
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < VEC; ++i) red[threadIdx.y][threadIdx.x][i] = acc[i];
+    __syncthreads();
+    if (threadIdx.y == 0 && g < gpr) {
+#pragma unroll
+        for (int i = 0; i < VEC; ++i) {
+            const float s = ((red[0][threadIdx.x][i] + red[1][threadIdx.x][i]) +
+                             red[2][threadIdx.x][i]) + red[3][threadIdx.x][i];
+            partial[(long long)blockIdx.y * d + (long long)g * VEC + i] = s;
+        }
     }
 }
 
@@ -301,8 +367,8 @@ cudaError_t launch_f32_fwd(const float* x, const float* Ws, const float* Wn, con
 
 cudaError_t launch_relu_grad_mask_f32(const float* dy, const uint32_t* mask, float* dz,
                                       long long rows, int d, cudaStream_t st) {
-    relu_grad_mask_kernel<float><<<blocks_for((size_t)rows * d, 256), 256, 0, st>>>(dy, mask, dz,
-                                                                                  rows, d);
+    relu_grad_mask_f32_kernel<<<blocks_for((size_t)rows * d, 256), 256, 0, st>>>(dy, mask, dz,
+                                                                              rows, d);
     return cudaGetLastError();
 }
 
@@ -310,7 +376,7 @@ cudaError_t launch_relu_grad_mask_bf16(const __nv_bfloat16* dy, const uint32_t* 
                                        __nv_bfloat16* dz, long long rows, int d,
                                        cudaStream_t st) {
     relu_grad_mask_kernel<__nv_bfloat16>
-        <<<blocks_for((size_t)rows * d, 256), 256, 0, st>>>(dy, mask, dz, rows, d);
+        <<<blocks_for((size_t)rows * d / 8, 256), 256, 0, st>>>(dy, mask, dz, rows, d);
     return cudaGetLastError();
 }
 
@@ -356,8 +422,14 @@ static cudaError_t colsum(const V* dz, long long rows, int d, float* partial, fl
         cudaError_t e = cudaMemsetAsync(out, 0, (size_t)batch * d * sizeof(float), st);
         return e;
     }
-    dim3 grid((d + 31) / 32, (unsigned)chunks, (unsigned)batch);
-    colsum_partial_kernel<V><<<grid, dim3(32, 8), 0, st>>>(dz, rows, d, partial);
+    if (sizeof(V) == 4) {
+        colsum_partial_f32_kernel<<<dim3((d + 31) / 32, (unsigned)chunks, 1), dim3(32, 8), 0, st>>>(
+            reinterpret_cast<const float*>(dz), rows, d, partial);
+    } else {
+        constexpr int VEC = 16 / sizeof(V);
+        dim3 grid((d / VEC + 63) / 64, (unsigned)chunks, (unsigned)batch);
+        colsum_partial_kernel<V><<<grid, dim3(64, 4), 0, st>>>(dz, rows, d, partial);
+    }
     colsum_final_kernel<<<dim3((d + 127) / 128, batch), 128, 0, st>>>(partial, (int)chunks, d, out);
     return cudaGetLastError();
 }

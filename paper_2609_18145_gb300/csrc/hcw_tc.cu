@@ -32,14 +32,17 @@
 // partials are reduced in a fixed order by a separate kernel
 // (deterministic).
 //
-// Roles (320 threads): warp 0 issues TMA loads into a ring of shared-memory
-// stages; warp 1 owns TMEM (2 x BN fp32 columns, a double-buffered
-// accumulator) and issues tcgen05.mma; warps 2..9 drain the accumulator
-// through tcgen05.ld (two warps per TMEM lane quarter, one per column half).
-// All epilogue I/O goes through TMA: each epilogue warp has two 4 KB
-// buffers; the residual rows of its 32 x 64 patch are TMA-loaded into a
-// buffer before the accumulator is ready, each lane overwrites its own row
-// in place with the result, and a TMA store writes the patch back.  Every
+// Roles: warp 0 issues TMA loads into a ring of shared-memory stages; warp 1
+// owns TMEM (2 x BN fp32 columns, a double-buffered accumulator) and issues
+// tcgen05.mma; the other warps drain the accumulator through tcgen05.ld:
+// sixteen of them for tiles of 128 or 256 columns (four per TMEM lane
+// quarter, each a 32-row patch of BN/4 columns), eight for narrower tiles.
+// The epilogue is latency-bound (TMEM loads, residual loads, store
+// completion), so the warps per scheduler matter more than the work per
+// warp.  All epilogue I/O goes through TMA: each epilogue warp has one 4 KB
+// buffer; the residual rows of its patch are TMA-loaded into it before the
+// accumulator is ready, each lane overwrites its own row in place with the
+// result, and a TMA store writes the patch back.  Every
 // wait is bounded (hcw_ptx.cuh); a CTA that gives up records
 // HCW_ERR_TIMEOUT, drains its in-flight copies and MMAs, frees TMEM and
 // returns.
@@ -52,14 +55,19 @@ namespace hcw {
 
 namespace {
 
-constexpr int kEpiWarps = 8;                       // two per TMEM lane quarter
-constexpr int kThreads = 64 + 32 * kEpiWarps;      // producer, MMA, epilogue warps
+constexpr int kMaxEpiWarps = 16;
+constexpr int kUnitQ = 8;                          // claimed units in flight per CTA
 constexpr int kBlockM = 128;
 constexpr int kBlockK = 64;                        // bf16 elements per 128-byte row
 constexpr int kABytes = kBlockM * kBlockK * 2;     // 16 KB
 constexpr int kRingBytes = 144 * 1024;             // TMA stage ring
-constexpr int kEpiBufBytes = 4096;                 // one epilogue patch: 32 rows x 128 B
-constexpr int kEpiBufs = 2;                        // per epilogue warp
+constexpr int kEpiBufBytes = 4096;                 // one epilogue patch: 32 rows x <= 128 B
+
+// epilogue warps (a multiple of 4: one group per TMEM lane quarter), threads,
+// and columns of the patch each epilogue warp drains
+__host__ __device__ constexpr int epi_warps(int BN) { return BN >= 128 ? 16 : 8; }
+__host__ __device__ constexpr int cta_threads(int BN) { return 64 + 32 * epi_warps(BN); }
+__host__ __device__ constexpr int warp_cols(int BN) { return BN / (epi_warps(BN) / 4); }
 
 __host__ __device__ constexpr int stage_bytes(int BN) { return kABytes + BN * kBlockK * 2; }
 __host__ __device__ constexpr int num_stages(int BN) {
@@ -72,16 +80,19 @@ struct __align__(8) Barriers {
     uint64_t tfull[2];
     uint64_t tempty[2];
     uint64_t drain;
-    uint64_t epi_load[kEpiWarps][kEpiBufs];       // residual patch landed in a buffer
+    uint64_t epi_load[kMaxEpiWarps];              // residual patch landed in a warp's buffer
     uint32_t tmem_base;
     int abort;
     int dep_unit;   // the producer has seen the inputs of this CTA's units up to this ordinal
+    int unit_q[kUnitQ];   // dynamic scheduling: unit claimed for ordinal o, in slot o % kUnitQ
+    int q_pub;            // highest ordinal published in unit_q
+    int q_read;           // slot reads so far (the MMA thread and every epilogue warp)
 };
 
 template <int BN>
 __host__ __device__ constexpr size_t smem_total() {
     return 1024 /* alignment slack */ + (size_t)num_stages(BN) * stage_bytes(BN) +
-           (size_t)kEpiWarps * kEpiBufs * kEpiBufBytes + (size_t)kEpiWarps * (BN / 2) * 4 +
+           (size_t)epi_warps(BN) * kEpiBufBytes + (size_t)epi_warps(BN) * warp_cols(BN) * 4 +
            sizeof(Barriers);
 }
 
@@ -244,6 +255,25 @@ __device__ __forceinline__ bool wait_counter(const int* ctr, int target, volatil
     }
 }
 
+// Bounded wait until the shared counter *p >= target (acquire); records a
+// timeout like mbar_wait.
+__device__ __forceinline__ bool wait_shared_geq(const int* p, int target, volatile int* abort,
+                                                uint64_t timeout_ns) {
+    if (ld_acquire_cta_shared(p) >= target) return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t it = 1;; ++it) {
+        if (ld_acquire_cta_shared(p) >= target) return true;
+        if ((it & 63u) == 0) {
+            if (*abort) return false;
+            if (globaltimer_ns() - t0 > timeout_ns) {
+                atomicExch(&g_error_word, kErrTimeout);
+                *abort = 1;
+                return false;
+            }
+        }
+    }
+}
+
 // Wait that only gives up on time (used to drain in-flight work after an
 // abort, when the abort flag is already set).
 __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity,
@@ -279,7 +309,7 @@ __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity,
 // of the launch have smaller indices and each CTA takes its units in order,
 // so the lowest unfinished unit can always proceed.
 template <int MODE, int BN, int NL>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(cta_threads(BN), 1)
     hcw_tc_kernel(const __grid_constant__ TcLaunch<NL> L) {
     constexpr int STAGES = num_stages(BN);
     constexpr int SB = stage_bytes(BN);
@@ -287,7 +317,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     constexpr uint32_t TMEM_COLS = 2 * BN;
     constexpr uint32_t IDESC = idesc_bf16_f32(kBlockM, BN, MODE == MODE_DW ? 1 : 0,
                                               MODE == MODE_FWD ? 0 : 1);
-    constexpr int HALF = BN / 2;                       // columns per epilogue warp
+    constexpr int EW = epi_warps(BN);
+    constexpr int WCOLS = warp_cols(BN);               // columns per epilogue warp
+    static_assert(EW <= kMaxEpiWarps && WCOLS % 32 == 0 && WCOLS <= 64, "epilogue split");
     constexpr bool STACKED = NL > 1;
     const TcParams& p = L.p;
     const int upl = p.n_units;                          // units per layer
@@ -297,9 +329,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     uint8_t* epi_smem = smem + (size_t)STAGES * SB;               // 1024-aligned
-    float* bias_smem =
-        reinterpret_cast<float*>(epi_smem + (size_t)kEpiWarps * kEpiBufs * kEpiBufBytes);
-    Barriers* bars = reinterpret_cast<Barriers*>(bias_smem + kEpiWarps * HALF);
+    float* bias_smem = reinterpret_cast<float*>(epi_smem + (size_t)EW * kEpiBufBytes);
+    Barriers* bars = reinterpret_cast<Barriers*>(bias_smem + EW * WCOLS);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -313,13 +344,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&bars->tfull[a], 1);
-            mbar_init(&bars->tempty[a], kEpiWarps);
+            mbar_init(&bars->tempty[a], EW);
         }
-        for (int e = 0; e < kEpiWarps; ++e)
-            for (int b = 0; b < kEpiBufs; ++b) mbar_init(&bars->epi_load[e][b], 1);
+        for (int e = 0; e < EW; ++e) mbar_init(&bars->epi_load[e], 1);
         mbar_init(&bars->drain, 1);
         bars->abort = 0;
         bars->dep_unit = -1;
+        bars->q_pub = -1;
+        bars->q_read = 0;
         fence_mbar_init();
     }
     if (warp == 1) {
@@ -332,6 +364,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem_base = bars->tmem_base;
     volatile int* abort = &bars->abort;
     const uint64_t tmo = p.timeout_ns;
+    // Stacked launches hand out units dynamically, in increasing order, from a
+    // global counter: CTAs that draw short units take more of them, so no CTA
+    // runs far behind the others and stalls the next layer's units.  The
+    // producer claims a unit and publishes it in a shared slot; the MMA thread
+    // and the epilogue warps read it by ordinal.  Otherwise CTA b takes units
+    // b, b + grid, b + 2 grid, ...
+    const bool dyn = STACKED && L.sched != nullptr;
+    auto consume_unit = [&](int ord) -> int {   // -1: no more units, -2: aborted
+        if (!dyn) {
+            const int u = (int)blockIdx.x + ord * (int)gridDim.x;
+            return u < n_units ? u : -1;
+        }
+        if (!wait_shared_geq(&bars->q_pub, ord, abort, tmo)) return -2;
+        const int u = *reinterpret_cast<volatile int*>(&bars->unit_q[ord % kUnitQ]);
+        __threadfence_block();
+        atomicAdd(&bars->q_read, 1);
+        return u;
+    };
 
     if (warp == 0) {
         // ------------------------------------------------------------ producer
@@ -340,8 +390,25 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t phase = 0;
             uint32_t issued_mask = 0, issued_phase = 0;
             bool ok = true;
-            int ordinal = 0;
-            for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x, ++ordinal) {
+            for (int ordinal = 0; ok; ++ordinal) {
+                int u;
+                if (dyn) {
+                    u = atomicAdd(L.sched, 1);
+                    if (u >= n_units) u = -1;
+                    // the slot's previous unit has been read by every consumer
+                    if (ordinal >= kUnitQ &&
+                        !wait_shared_geq(&bars->q_read, (ordinal - kUnitQ + 1) * (EW + 1), abort,
+                                         tmo)) {
+                        ok = false;
+                        break;
+                    }
+                    bars->unit_q[ordinal % kUnitQ] = u;
+                    st_release_cta_shared(&bars->q_pub, ordinal);
+                } else {
+                    u = (int)blockIdx.x + ordinal * (int)gridDim.x;
+                    if (u >= n_units) u = -1;
+                }
+                if (u < 0) break;
                 int l = STACKED ? u / upl : 0;
                 const int ul = STACKED ? u - l * upl : u;
                 WUnit w{};
@@ -453,7 +520,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             int acc = 0;
             uint32_t acc_phase = 0;
             bool ok = true, any = false;
-            for (int u = blockIdx.x; u < n_units && ok; u += gridDim.x) {
+            for (int ord = 0; ok; ++ord) {
+                const int u = consume_unit(ord);
+                if (u == -2) {
+                    ok = false;
+                    break;
+                }
+                if (u < 0) break;
                 const int ul = STACKED ? u % upl : u;
                 int steps;
                 if (MODE != MODE_DW) {
@@ -510,14 +583,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else {
         // ------------------------------------------------------------ epilogue
-        // Warp e (0..7) drains TMEM lane quarter warp % 4 (rows 32 q .. 32 q + 31
-        // of the tile) and column half e / 4, in patches of 32 rows x SW columns.
+        // Warp e drains TMEM lane quarter warp % 4 (rows 32 q .. 32 q + 31 of the
+        // tile) and column slice e / 4 (WCOLS columns): one patch per tile.
         const int e = warp - 2;
         const int quarter = warp & 3;
-        const int half = e >> 2;
-        uint8_t* bufs = epi_smem + (size_t)e * kEpiBufs * kEpiBufBytes;
-        float* wbias = bias_smem + e * HALF;
-        uint32_t ld_phase[kEpiBufs] = {0, 0};
+        const int cslice = e >> 2;
+        uint8_t* buf = epi_smem + (size_t)e * kEpiBufBytes;
+        float* wbias = bias_smem + e * WCOLS;
+        uint32_t ld_phase = 0;
         int acc = 0;
         uint32_t acc_phase = 0;
         bool alive = true;
@@ -536,7 +609,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         auto load_acc = [&](uint32_t col, uint32_t (&raw)[32]) {
             __syncwarp();   // tcgen05.ld is .sync.aligned: the whole warp, converged
             tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(quarter * 32) << 16) +
-                                   (uint32_t)(acc * BN + half * HALF) + col,
+                                   (uint32_t)(acc * BN + cslice * WCOLS) + col,
                                raw);
             tmem_ld_wait_regs(raw);
         };
@@ -565,18 +638,23 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             return __shfl_sync(0xffffffffu, ok, 0) != 0;
         };
-        for (int u = blockIdx.x; u < n_units && alive; u += gridDim.x, ++ordinal) {
+        for (; alive; ++ordinal) {
+            int u = 0;
+            if (lane == 0) u = consume_unit(ordinal);
+            u = __shfl_sync(0xffffffffu, u, 0);
+            if (u == -2) {
+                alive = false;
+                break;
+            }
+            if (u < 0) break;
             int l = STACKED ? u / upl : 0;
             const int ul = STACKED ? u - l * upl : u;
             WUnit wu{};
             if (MODE == MODE_DW) wu = decode_w_any(p, u, STACKED, L.n_layers, l);
             const TcLayer& ly = L.layer[l];
             if (MODE != MODE_DW) {
-                constexpr int SW = HALF >= 64 ? 64 : HALF;     // patch width (columns)
-                constexpr int RB = SW * 2;                     // patch row bytes
-                constexpr int NSC = HALF / SW;                 // patches per warp (<= 2)
-                constexpr int SUB = SW / 32;                   // 32-column sub-chunks per patch
-                static_assert(NSC <= kEpiBufs, "one buffer per patch");
+                constexpr int RB = WCOLS * 2;                  // patch row bytes (128 or 64)
+                constexpr int SUB = WCOLS / 32;                // 32-column sub-chunks per patch
                 const RowUnit r = decode_row_unit(p, ul, STACKED);
                 const int qw = r.t * kBlockM + quarter * 32;   // first compressed row of the warp
                 const int lo_w = qw & (ly.k - 1), hi_w = qw >> ly.s;
@@ -584,7 +662,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int tok_row = q_row < p.Mh ? ((q_row >> ly.s) << (ly.s + 1)) +
                                                        (r.beta << ly.s) + (q_row & (ly.k - 1))
                                                  : -1;
-                const int col_half = r.j * BN + half * HALF;
+                const int col0 = r.j * BN + cslice * WCOLS;
                 // a patch entirely past the end (ragged tail) loads and stores nothing
                 const bool inside = qw < p.Mh;
                 const bool has_res = (p.flags & 2u) != 0 && inside;
@@ -594,7 +672,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const CUtensorMap* mE1 = &L.maps[l][4];
                 const CUtensorMap* mE2 = &L.maps[l][5];
                 const int wpr = p.d >> 5;
-                // every earlier store has finished reading the buffers: refill them
+                // every earlier store has finished reading the buffer: refill it
                 if (lane == 0) bulk_wait_read<0>();
                 __syncwarp();
                 if (!wait_inputs(ordinal)) {
@@ -602,23 +680,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                     break;
                 }
                 if (has_res && lane == 0) {
-#pragma unroll
-                    for (int sc = 0; sc < NSC; ++sc) {
-                        mbar_arrive_expect_tx(&bars->epi_load[e][sc], 32 * RB);
-                        tma_load_4d(bufs + sc * kEpiBufBytes, mE0, &bars->epi_load[e][sc],
-                                    col_half + sc * SW, lo_w, r.beta, hi_w);
-                    }
+                    mbar_arrive_expect_tx(&bars->epi_load[e], 32 * RB);
+                    tma_load_4d(buf, mE0, &bars->epi_load[e], col0, lo_w, r.beta, hi_w);
                 }
-                uint32_t mp[HALF / 32];
+                uint32_t mp[SUB];
 #pragma unroll
-                for (int c = 0; c < HALF / 32; ++c)
-                    mp[c] = (has_mprev && tok_row >= 0)
-                                ? __ldg(ly.mprev + (size_t)tok_row * wpr + (col_half >> 5) + c)
+                for (int h = 0; h < SUB; ++h)
+                    mp[h] = (has_mprev && tok_row >= 0)
+                                ? __ldg(ly.mprev + (size_t)tok_row * wpr + (col0 >> 5) + h)
                                 : 0u;
                 if (fwd) {
                     // this warp's bias slice, read back as warp-wide broadcasts
-                    for (int c = lane; c < HALF; c += 32)
-                        wbias[c] = ly.bias ? __ldg(ly.bias + col_half + c) : 0.f;
+                    for (int c = lane; c < WCOLS; c += 32)
+                        wbias[c] = ly.bias ? __ldg(ly.bias + col0 + c) : 0.f;
                     __syncwarp();
                 }
                 if (!wait_acc()) {
@@ -629,12 +703,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // lane joins the warp-wide TMEM loads, rows past the end skip the store
                 if (fwd && ly.zout) {
 #pragma unroll 1
-                    for (int c = 0; c < HALF / 32; ++c) {
+                    for (int h = 0; h < SUB; ++h) {
                         uint32_t raw[32];
-                        load_acc(c * 32, raw);
+                        load_acc(h * 32, raw);
                         if (tok_row >= 0) {
                             uint4* dst = reinterpret_cast<uint4*>(ly.zout + (size_t)tok_row * p.d +
-                                                                  col_half + c * 32);
+                                                                  col0 + h * 32);
 #pragma unroll
                             for (int m = 0; m < 4; ++m) {
                                 uint32_t w[4];
@@ -642,116 +716,113 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 for (int i = 0; i < 4; ++i) {
                                     const int e2 = 8 * m + 2 * i;
                                     w[i] = pack_bf16x2(
-                                        __uint_as_float(raw[e2]) + wbias[c * 32 + e2],
-                                        __uint_as_float(raw[e2 + 1]) + wbias[c * 32 + e2 + 1]);
+                                        __uint_as_float(raw[e2]) + wbias[h * 32 + e2],
+                                        __uint_as_float(raw[e2 + 1]) + wbias[h * 32 + e2 + 1]);
                                 }
                                 dst[m] = make_uint4(w[0], w[1], w[2], w[3]);
                             }
                         }
                     }
                 }
+                if (has_res) {
+                    const bool okl = wait_bar(&bars->epi_load[e], ld_phase);
+                    ld_phase ^= 1;
+                    if (!okl) {
+                        alive = false;
+                        break;
+                    }
+                }
+                const bool write_out = fwd || ly.out;
+                uint32_t gw[SUB][16];
 #pragma unroll
-                for (int sc = 0; sc < NSC; ++sc) {
-                    uint8_t* buf = bufs + sc * kEpiBufBytes;
-                    if (has_res) {
-                        const bool okl = wait_bar(&bars->epi_load[e][sc], ld_phase[sc]);
-                        ld_phase[sc] ^= 1;
-                        if (!okl) {
-                            alive = false;
-                            break;
+                for (int h = 0; h < SUB; ++h) {
+                    uint32_t raw[32];
+                    load_acc(h * 32, raw);
+                    if (h == SUB - 1) release_acc();
+                    float v[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(raw[i]);
+                    if (fwd) {
+                        const float4* b4 = reinterpret_cast<const float4*>(wbias + h * 32);
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const float4 bb = b4[i];
+                            v[4 * i] += bb.x;
+                            v[4 * i + 1] += bb.y;
+                            v[4 * i + 2] += bb.z;
+                            v[4 * i + 3] += bb.w;
+                        }
+                        if (ly.mout) {
+                            uint32_t bits = 0;
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) bits |= (v[i] > 0.f ? 1u : 0u) << i;
+                            if (tok_row >= 0)
+                                ly.mout[(size_t)tok_row * wpr + (col0 >> 5) + h] = bits;
+                        }
+                        if (p.flags & 4u) {
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) v[i] = v[i] > 0.f ? v[i] : 0.f;
                         }
                     }
-                    uint32_t gw[SUB][16];
+                    if (has_res) {
+#pragma unroll
+                        for (int m = 0; m < 4; ++m) {
+                            const uint4 q4 = *patch_piece<RB>(buf, lane, 4 * h + m);
+                            const uint32_t rw[4] = {q4.x, q4.y, q4.z, q4.w};
+#pragma unroll
+                            for (int i = 0; i < 4; ++i) {
+                                const float2 f = unpack_bf16x2(rw[i]);
+                                v[8 * m + 2 * i] += f.x;
+                                v[8 * m + 2 * i + 1] += f.y;
+                            }
+                        }
+                    }
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) gw[h][i] = pack_bf16x2(v[2 * i], v[2 * i + 1]);
+                    // the lane's own row, the pieces just read: safe to overwrite now
+                    if (write_out) {
+#pragma unroll
+                        for (int m = 0; m < 4; ++m)
+                            *patch_piece<RB>(buf, lane, 4 * h + m) =
+                                make_uint4(gw[h][4 * m], gw[h][4 * m + 1], gw[h][4 * m + 2],
+                                           gw[h][4 * m + 3]);
+                    }
+                }
+                // the patch: y (FWD) or dx (DX), written over the residual rows
+                if (write_out) {
+                    publish();
+                    if (lane == 0 && inside) {
+                        tma_store_4d(mE1, buf, col0, lo_w, r.beta, hi_w);
+                        bulk_commit();
+                    }
+                }
+                if (has_mprev) {
+                    // fused ReLU gradient of the layer below: dz = dx * mask
+                    if (write_out) {
+                        if (lane == 0) bulk_wait_read<0>();
+                        __syncwarp();
+                    }
 #pragma unroll
                     for (int h = 0; h < SUB; ++h) {
-                        uint32_t raw[32];
-                        load_acc(sc * SW + h * 32, raw);
-                        if (sc == NSC - 1 && h == SUB - 1) release_acc();
-                        float v[32];
+                        const uint32_t mw = mp[h];
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(raw[i]);
-                        if (fwd) {
-                            const float4* b4 = reinterpret_cast<const float4*>(wbias + sc * SW + h * 32);
+                        for (int m = 0; m < 4; ++m) {
+                            uint32_t w4[4];
 #pragma unroll
-                            for (int i = 0; i < 8; ++i) {
-                                const float4 bb = b4[i];
-                                v[4 * i] += bb.x;
-                                v[4 * i + 1] += bb.y;
-                                v[4 * i + 2] += bb.z;
-                                v[4 * i + 3] += bb.w;
+                            for (int i = 0; i < 4; ++i) {
+                                const int b = 8 * m + 2 * i;
+                                const uint32_t keep = ((mw >> b) & 1u ? 0x0000FFFFu : 0u) |
+                                                      ((mw >> (b + 1)) & 1u ? 0xFFFF0000u : 0u);
+                                w4[i] = gw[h][4 * m + i] & keep;
                             }
-                            if (ly.mout) {
-                                uint32_t bits = 0;
-#pragma unroll
-                                for (int i = 0; i < 32; ++i) bits |= (v[i] > 0.f ? 1u : 0u) << i;
-                                if (tok_row >= 0)
-                                    ly.mout[(size_t)tok_row * wpr + ((col_half + sc * SW) >> 5) + h] =
-                                        bits;
-                            }
-                            if (p.flags & 4u) {
-#pragma unroll
-                                for (int i = 0; i < 32; ++i) v[i] = v[i] > 0.f ? v[i] : 0.f;
-                            }
-                        }
-                        if (has_res) {
-#pragma unroll
-                            for (int m = 0; m < 4; ++m) {
-                                const uint4 q4 = *patch_piece<RB>(buf, lane, 4 * h + m);
-                                const uint32_t rw[4] = {q4.x, q4.y, q4.z, q4.w};
-#pragma unroll
-                                for (int i = 0; i < 4; ++i) {
-                                    const float2 f = unpack_bf16x2(rw[i]);
-                                    v[8 * m + 2 * i] += f.x;
-                                    v[8 * m + 2 * i + 1] += f.y;
-                                }
-                            }
-                        }
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) gw[h][i] = pack_bf16x2(v[2 * i], v[2 * i + 1]);
-                    }
-                    // the patch: y (FWD) or dx (DX), written over the residual rows
-                    if (fwd || ly.out) {
-#pragma unroll
-                        for (int h = 0; h < SUB; ++h)
-#pragma unroll
-                            for (int m = 0; m < 4; ++m)
-                                *patch_piece<RB>(buf, lane, 4 * h + m) =
-                                    make_uint4(gw[h][4 * m], gw[h][4 * m + 1], gw[h][4 * m + 2],
-                                               gw[h][4 * m + 3]);
-                        publish();
-                        if (lane == 0 && inside) {
-                            tma_store_4d(mE1, buf, col_half + sc * SW, lo_w, r.beta, hi_w);
-                            bulk_commit();
+                            *patch_piece<RB>(buf, lane, 4 * h + m) =
+                                make_uint4(w4[0], w4[1], w4[2], w4[3]);
                         }
                     }
-                    if (has_mprev) {
-                        // fused ReLU gradient of the layer below: dz = dx * mask
-                        if (ly.out) {
-                            if (lane == 0) bulk_wait_read<0>();
-                            __syncwarp();
-                        }
-#pragma unroll
-                        for (int h = 0; h < SUB; ++h) {
-                            const uint32_t mw = mp[(sc * SW >> 5) + h];
-#pragma unroll
-                            for (int m = 0; m < 4; ++m) {
-                                uint32_t w4[4];
-#pragma unroll
-                                for (int i = 0; i < 4; ++i) {
-                                    const int b = 8 * m + 2 * i;
-                                    const uint32_t keep = ((mw >> b) & 1u ? 0x0000FFFFu : 0u) |
-                                                          ((mw >> (b + 1)) & 1u ? 0xFFFF0000u : 0u);
-                                    w4[i] = gw[h][4 * m + i] & keep;
-                                }
-                                *patch_piece<RB>(buf, lane, 4 * h + m) =
-                                    make_uint4(w4[0], w4[1], w4[2], w4[3]);
-                            }
-                        }
-                        publish();
-                        if (lane == 0 && inside) {
-                            tma_store_4d(mE2, buf, col_half + sc * SW, lo_w, r.beta, hi_w);
-                            bulk_commit();
-                        }
+                    publish();
+                    if (lane == 0 && inside) {
+                        tma_store_4d(mE2, buf, col0, lo_w, r.beta, hi_w);
+                        bulk_commit();
                     }
                 }
                 if (STACKED && alive && l + 1 < L.n_layers) {
@@ -764,7 +835,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const int rows = min(32, p.Mh - qw);
                         const int tok0 = ((qw >> ly.s) << (ly.s + 1)) + (r.beta << ly.s) +
                                          (qw & (ly.k - 1));
-                        atomicAdd(L.counters + (size_t)l * L.n_chunks + (tok0 >> 7), rows * HALF);
+                        atomicAdd(L.counters + (size_t)l * L.n_chunks + (tok0 >> 7), rows * WCOLS);
                     }
                     __syncwarp();
                 }
@@ -778,15 +849,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const CUtensorMap* map = &L.maps[l][S > 1 ? 3 : (w.which ? 5 : 4)];
                 const int row0 = (S > 1 ? (w.which * p.splits_max + w.split) * p.d : 0) +
                                  w.ot * kBlockM + quarter * 32;
-                const int col_half = w.nt * BN + half * HALF;
+                const int col0 = w.nt * BN + cslice * WCOLS;
 #pragma unroll 1
-                for (int c = 0; c < HALF / 32; ++c) {
-                    uint8_t* buf = bufs + (c & 1) * kEpiBufBytes;
+                for (int c = 0; c < WCOLS / 32; ++c) {
                     uint32_t raw[32];
                     load_acc(c * 32, raw);
-                    if (c == HALF / 32 - 1) release_acc();
-                    // the buffer's previous store (two chunks ago) must have been read
-                    if (lane == 0) bulk_wait_read<1>();
+                    if (c == WCOLS / 32 - 1) release_acc();
+                    // the buffer's previous store must have been read
+                    if (lane == 0) bulk_wait_read<0>();
                     __syncwarp();
 #pragma unroll
                     for (int m = 0; m < 8; ++m)
@@ -796,7 +866,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     // d is a multiple of 64, so a warp's 32 rows are all inside or all
                     // past the end (ragged o tile); the latter are not stored
                     if (lane == 0 && w.ot * kBlockM + quarter * 32 < p.d) {
-                        tma_store_2d(map, buf, col_half + c * 32, row0);
+                        tma_store_2d(map, buf, col0 + c * 32, row0);
                         bulk_commit();
                     }
                 }
@@ -835,7 +905,7 @@ static cudaError_t launch_one(const TcLaunch<NL>& L, int grid, cudaStream_t st) 
         if (e != cudaSuccess) return e;
         if (dev < 256) word.fetch_or(bit, std::memory_order_acq_rel);
     }
-    kern<<<grid, kThreads, smem, st>>>(L);
+    kern<<<grid, cta_threads(BN), smem, st>>>(L);
     return cudaGetLastError();
 }
 
