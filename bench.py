@@ -63,11 +63,15 @@ def step_flops(B, n, d, L):
 
 
 class ClockSampler:
-    """nvidia-smi sampled every 200 ms while a timed region runs."""
+    """SM clock and clock-event reasons sampled while a timed region runs:
+    read-only NVML queries polled every ~2 ms from a thread (a timed region can
+    be a few milliseconds long), else nvidia-smi every 200 ms."""
 
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
 
     def __init__(self, local_rank: int):
         vis = os.environ.get("CUDA_VISIBLE_DEVICES")
@@ -75,8 +79,55 @@ class ClockSampler:
         self.gpu = ids[local_rank] if local_rank < len(ids) else str(local_rank)
         self.proc = None
         self.file = None
+        self.nvml = None
+        self.samples = []
+        self.stop = None
+        self.thread = None
+
+    def _open_nvml(self):
+        import ctypes
+        lib = ctypes.CDLL("libnvidia-ml.so.1")
+        if lib.nvmlInit_v2() != 0:
+            raise OSError("nvmlInit failed")
+        handle = ctypes.c_void_p()
+        if self.gpu.isdigit():
+            rc = lib.nvmlDeviceGetHandleByIndex_v2(ctypes.c_uint(int(self.gpu)),
+                                                   ctypes.byref(handle))
+        else:
+            rc = lib.nvmlDeviceGetHandleByUUID(self.gpu.encode(), ctypes.byref(handle))
+        if rc != 0:
+            raise OSError("no NVML handle")
+        reasons = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            lib.nvmlDeviceGetCurrentClocksThrottleReasons
+        mx = ctypes.c_uint()
+        lib.nvmlDeviceGetMaxClockInfo(handle, 1, ctypes.byref(mx))   # 1 = SM clock
+        self.nvml = (lib, handle, reasons, mx.value)
+
+    def _sample(self):
+        import ctypes
+        lib, handle, reasons, mx = self.nvml
+        sm = ctypes.c_uint()
+        r = ctypes.c_ulonglong()
+        if lib.nvmlDeviceGetClockInfo(handle, 1, ctypes.byref(sm)) == 0 and \
+                reasons(handle, ctypes.byref(r)) == 0:
+            self.samples.append((sm.value, mx, r.value))
+
+    def _poll(self):
+        while not self.stop.is_set():
+            self._sample()
+            time.sleep(0.002)
 
     def __enter__(self):
+        import threading
+        try:
+            self._open_nvml()
+            self.stop = threading.Event()
+            self._sample()
+            self.thread = threading.Thread(target=self._poll, daemon=True)
+            self.thread.start()
+            return self
+        except (OSError, AttributeError):
+            self.nvml = None
         try:
             self.file = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
             self.proc = subprocess.Popen(
@@ -88,6 +139,10 @@ class ClockSampler:
         return self
 
     def __exit__(self, *exc):
+        if self.thread is not None:
+            self._sample()
+            self.stop.set()
+            self.thread.join(timeout=5)
         if self.proc is not None:
             self.proc.terminate()
             try:
@@ -96,6 +151,14 @@ class ClockSampler:
                 self.proc.kill()
 
     def summary(self):
+        if self.nvml is not None:
+            if not self.samples:
+                return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+            reasons = sorted({name for _, _, r in self.samples
+                              for bit, name in self.REASONS.items() if r & bit})
+            return {"sm_mhz": statistics.median(sm for sm, _, _ in self.samples),
+                    "sm_max_mhz": max(mx for _, mx, _ in self.samples), "reasons": reasons,
+                    "samples": len(self.samples), "source": "nvml"}
         if self.proc is None or self.file is None:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
         self.file.flush()
@@ -349,33 +412,39 @@ def run_ours(args):
         torch.cuda.synchronize()
         return sum(a.elapsed_time(b) for a, b in evs) / reps
 
-    dz = dy   # a layer's pre-activation gradient has the activations' shape and scale
-    fwd_ms = time_calls(lambda i: H.hcw_stack_fwd(x, Ws[i % L:i % L + 1], Wn[i % L:i % L + 1],
-                                                  bias[i % L:i % L + 1], i % L, -1, flags, y=y,
-                                                  masks=masks[:1], workspace=fws), 2 * L)
-    dx_ms = time_calls(lambda i: H.hcw_layer_bwd_data(dz, dy, Ws[i % L], Wn[i % L], i % L, -1,
-                                                      flags, dx=dx), 2 * L)
-    wws = torch.empty(H.hcw_layer_bwd_weight_workspace_bytes(B, n, d, H.HCW_BF16, flags),
+    # the step's three tensor-core launches, each timed alone on the same inputs:
+    # the stacked forward, the stacked input gradient (with the top layer's
+    # ReLU-gradient pass in front) and the batched weight gradient (bias off)
+    dz_all = torch.empty((L, B, n, d), dtype=torch.bfloat16, device=dev)
+    dws = torch.empty(max(1, H.hcw_stack_bwd_data_workspace_bytes(B, n, d, H.HCW_BF16, flags, L)),
                       dtype=torch.uint8, device=dev)
-    dw_ms = time_calls(lambda i: H.hcw_layer_bwd_weight(x, dz, i % L, -1, flags,
-                                                        dW_self=gWs[0], dW_nbr=gWn[0],
-                                                        want_dbias=False, workspace=wws), 2 * L)
-    # the two halves of the step as the step runs them
-    stack_fwd_ms = time_calls(lambda i: H.hcw_stack_fwd(x, Ws, Wn, bias, 0, -1, flags, y=y,
-                                                        acts=acts, masks=masks, workspace=fws), 3)
-    stack_bwd_ms = time_calls(lambda i: H.hcw_stack_bwd(x, acts, masks, dy, Ws, Wn, 0, -1, flags,
-                                                        dx=dx, dW_self=gWs, dW_nbr=gWn, dbias=gb,
-                                                        workspace=ws), 3)
-    layer_flops = 3.0 * d * d * tokens          # per kernel launch (causal)
-    kernels = {"hcw_tc_kernel<FWD,256>": fwd_ms, "hcw_tc_kernel<DX,256>": dx_ms,
-               "dW (hcw_tc_kernel<DW,256> + split reduce)": dw_ms}
+    wws = torch.empty(max(1, H.hcw_stack_bwd_weight_workspace_bytes(B, n, d, H.HCW_BF16, flags,
+                                                                    L)),
+                      dtype=torch.uint8, device=dev)
+    reps = 5
+    fwd_ms = time_calls(lambda i: H.hcw_stack_fwd(x, Ws, Wn, bias, 0, -1, flags, y=y, acts=acts,
+                                                  masks=masks, workspace=fws), reps)
+    dx_ms = time_calls(lambda i: H.hcw_stack_bwd_data(masks, dy, Ws, Wn, 0, -1, flags, dx=dx,
+                                                      dz=dz_all, workspace=dws), reps)
+    dw_ms = time_calls(lambda i: H.hcw_stack_bwd_weight(x, acts, dz_all, 0, -1, flags,
+                                                        dW_self=gWs, dW_nbr=gWn, want_dbias=False,
+                                                        workspace=wws), reps)
+    dwb_ms = time_calls(lambda i: H.hcw_stack_bwd_weight(x, acts, dz_all, 0, -1, flags,
+                                                         dW_self=gWs, dW_nbr=gWn, dbias=gb,
+                                                         workspace=wws), reps)
+    launch_flops = 3.0 * d * d * tokens * L     # per stacked launch, 16 causal layers
+    kernels = {"hcw_tc_kernel<FWD,256,16> (stacked forward)": fwd_ms,
+               "hcw_tc_kernel<DX,256,16> (stacked input gradient, + top ReLU pass)": dx_ms,
+               "hcw_tc_kernel<DW,256,16> (batched weight gradient)": dw_ms}
     dominant = max(kernels, key=kernels.get)
     dom_ms = kernels[dominant]
     peak = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
-    achieved = layer_flops / (dom_ms * 1e-3) / 1e12
+    achieved = launch_flops / (dom_ms * 1e-3) / 1e12
+    per_kernel = {k: {"ms": v, "tflops": launch_flops / (v * 1e-3) / 1e12,
+                      "frac": launch_flops / (v * 1e-3) / 1e12 / peak} for k, v in kernels.items()}
     step_tflops = step_flops(B, n, d, L) / (ms * 1e-3) / 1e12
     peak_sus = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
-    traffic = recorded_traffic(dominant)
+    traffic = recorded_traffic(dominant.split(" ")[0])
 
     # ---- end to end through the public API with host buffers
     x_h = torch.empty(x.shape, dtype=x.dtype, pin_memory=True)
@@ -437,9 +506,8 @@ def run_ours(args):
             "roofline": {"bound": "tensor", "kernel": dominant, "achieved": achieved,
                          "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                          "traffic": traffic, "peak_source": peak_src + " bf16 burst",
-                         "flops_per_launch": layer_flops, "avg_launch_ms": dom_ms,
-                         "kernel_ms": kernels, "stack_fwd_ms": stack_fwd_ms,
-                         "stack_bwd_ms": stack_bwd_ms},
+                         "flops_per_launch": launch_flops, "avg_launch_ms": dom_ms,
+                         "kernels": per_kernel, "dbias_ms": dwb_ms - dw_ms},
             "step_roofline": {"achieved": step_tflops, "peak": peak_sus, "unit": "TFLOP/s",
                               "frac": step_tflops / peak_sus,
                               "peak_source": peak_src + " bf16 sustained",

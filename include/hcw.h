@@ -204,6 +204,42 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void
 size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags, int L);
 
 /*
+ * The two halves of hcw_stack_bwd, for callers that want them apart (frozen
+ * weights need only the first; the second can run later or elsewhere).
+ *
+ * hcw_stack_bwd_data: input gradients through the stack (the chain rule of
+ * Eq. (1), layers L-1 down to 0).
+ *   masks, dy, W_self, W_nbr as for hcw_stack_bwd.
+ *   dx [B][n][d] gradient of the stack's input (output).
+ *   dz [L][B][n][d] (output): every layer's pre-activation gradient
+ *      dz_l = g_l * act'(z_l), where g_l is the gradient of layer l's
+ *      output -- the input of hcw_stack_bwd_weight.
+ *   workspace: at least hcw_stack_bwd_data_workspace_bytes(...) bytes.
+ */
+int hcw_stack_bwd_data(const void* masks, const void* dy, const void* W_self, const void* W_nbr,
+                       int layer0, int L, int dim_override, int B, int n, int d, int dtype,
+                       unsigned flags, void* dx, void* dz, void* workspace, size_t ws_bytes,
+                       void* stream);
+size_t hcw_stack_bwd_data_workspace_bytes(int B, int n, int d, int dtype, unsigned flags,
+                                          int L);
+
+/*
+ * hcw_stack_bwd_weight: every layer's weight gradients from its input (x for
+ * layer 0, acts[l-1] above) and its dz as written by hcw_stack_bwd_data:
+ *   dW_self[l] = sum_i dz_l,i x_l,i^T,  dW_nbr[l] = sum_i m_i dz_l,i x_l,p(i)^T,
+ *   dbias[l] = sum_i dz_l,i (dbias may be NULL).  fp32 outputs [L][d][d], [L][d].
+ *   workspace: at least hcw_stack_bwd_weight_workspace_bytes(...) bytes.
+ * bf16: up to 16 layers per launch, whole token range per tile (no split
+ * reduction, deterministic), then one batched column sum for the biases.
+ */
+int hcw_stack_bwd_weight(const void* x, const void* acts, const void* dz, int layer0, int L,
+                         int dim_override, int B, int n, int d, int dtype, unsigned flags,
+                         float* dW_self, float* dW_nbr, float* dbias, void* workspace,
+                         size_t ws_bytes, void* stream);
+size_t hcw_stack_bwd_weight_workspace_bytes(int B, int n, int d, int dtype, unsigned flags,
+                                            int L);
+
+/*
  * hcw_layer_bwd_weight for callers that cannot allocate device memory (a
  * host that only lends its own input and output buffers, or code that must
  * not call an allocator): same arguments and results, minus the workspace.

@@ -486,41 +486,39 @@ int layer_bwd_impl(const Shape& sh, int dtype, const void* x, const void* z, con
 }
 
 // ------------------------------------------------------------ stack backward
-// Workspace of hcw_stack_bwd.
-//   bf16: dz of every layer [L] (+ the output gradient g of every layer with
-//   ReLU and residual), completion counters of the stacked input-gradient
-//   launch, the weight-gradient workspace (used only when the layers are run
-//   one by one), column-sum partials of every layer's dbias.
-//   fp32: two output-gradient and two dz buffers, the weight-gradient workspace.
-struct StackBwdLayout {
-    size_t dz_off, g_off, ctr_off, w_off, col_off, total;
-};
-
-StackBwdLayout stack_bwd_layout(const Shape& sh, int dtype, unsigned flags, int L) {
-    StackBwdLayout l;
+// Workspaces of the stack backward.
+//   input gradients, bf16: the output gradient g of every layer when both the
+//   ReLU and the residual are on (the residual term of that layer's input
+//   gradient; otherwise g is dz itself or dy), then the completion counters
+//   of the stacked launch.  fp32: two g buffers used in turn.
+//   weight gradients, bf16: the unit counter of the batched launch, the
+//   single-layer weight-gradient workspace (used when the layers are too few
+//   to fill the GPU and run one by one), the column-sum partials of every
+//   layer's dbias.  fp32: the single-layer workspace.
+//   hcw_stack_bwd: every layer's dz, then both of the above.
+size_t stack_data_ws(const Shape& sh, int dtype, unsigned flags, int L) {
     const size_t a = align256(sh.act_bytes);
-    const WsLayout w = ws_layout(sh.tokens, sh.d, dtype, flags);
     if (dtype == HCW_BF16) {
         const bool keep_g = (flags & HCW_ACT_RELU) && (flags & HCW_RESIDUAL);
-        l.dz_off = 0;
-        l.g_off = (size_t)L * a;
-        l.ctr_off = l.g_off + (keep_g ? (size_t)L * a : 0);
-        l.w_off = l.ctr_off + stack_counter_bytes(sh.tokens, L);
-        l.col_off = l.w_off + w.w_bytes;
-        l.total = l.col_off + (size_t)L * align256(colsum_workspace_bytes(sh.tokens, sh.d));
-    } else {
-        l.dz_off = 0;
-        l.g_off = 2 * a;
-        l.ctr_off = l.w_off = 4 * a;
-        l.col_off = l.w_off;
-        l.total = l.w_off + w.w_bytes;
+        return (keep_g ? (size_t)L * a : 0) + stack_counter_bytes(sh.tokens, L);
     }
-    return l;
+    return 2 * a;
 }
 
-struct StackBwdArgs {
-    const void* x;
-    const void* acts;
+size_t stack_weight_ws(const Shape& sh, int dtype, unsigned flags, int L) {
+    const WsLayout w = ws_layout(sh.tokens, sh.d, dtype, flags);
+    if (dtype == HCW_BF16)
+        return 256 + w.w_bytes + (size_t)L * align256(colsum_workspace_bytes(sh.tokens, sh.d));
+    return w.w_bytes;
+}
+
+size_t stack_dz_bytes(const Shape& sh, int L) { return align256((size_t)L * sh.act_bytes); }
+
+int stack_layer_dim(const Shape& sh, int layer0, int dim_override, int l) {
+    return dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
+}
+
+struct StackData {
     const void* masks;
     const void* dy;
     const uint8_t* Ws;
@@ -528,32 +526,34 @@ struct StackBwdArgs {
     int layer0, L, dim_override;
     unsigned flags;
     void* dx;
+    uint8_t* dz;   // [L][tokens][d], layer stride act_bytes
+    uint8_t* ws;
+};
+
+struct StackWeight {
+    const void* x;
+    const void* acts;
+    const uint8_t* dz;
+    int layer0, L, dim_override;
+    unsigned flags;
     float* dWs;
     float* dWn;
     float* dbias;
     uint8_t* ws;
 };
 
-int layer_dim(const Shape& sh, const StackBwdArgs& a, int l) {
-    return a.dim_override >= 0 ? a.dim_override : (a.layer0 + l) % sh.b;
-}
-
-// bf16: the relu gradient of the top layer, one stacked input-gradient
-// launch per run of <= 16 layers (top down; the ReLU gradient of the layer
-// below fused in), then one weight-gradient launch over all layers and one
-// batched column sum for the biases.
-int stack_bwd_bf16(const Shape& sh, const StackBwdArgs& a, const StackBwdLayout& lay,
-                   cudaStream_t st) {
+// bf16 input gradients: the ReLU gradient of the top layer, then one stacked
+// launch per run of <= 16 layers, top down, whose kernel also applies the
+// ReLU gradient of the layer below.
+int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
     const int d = sh.d, BN = pick_bn(d), L = a.L;
     const bool relu = (a.flags & HCW_ACT_RELU) != 0;
     const bool resid = (a.flags & HCW_RESIDUAL) != 0;
+    const bool keep_g = relu && resid;
     const size_t ab = sh.act_bytes, a256 = align256(ab), wb = (size_t)d * d * 2;
     const size_t mb = mask_bytes(sh);
-    auto dz = [&](int l) -> void* { return a.ws + lay.dz_off + (size_t)l * a256; };
-    auto gbuf = [&](int l) -> void* { return a.ws + lay.g_off + (size_t)l * a256; };
-    auto act = [&](int l) -> const void* {
-        return l == 0 ? a.x : static_cast<const uint8_t*>(a.acts) + (size_t)(l - 1) * ab;
-    };
+    auto dz = [&](int l) -> void* { return a.dz + (size_t)l * ab; };
+    auto gbuf = [&](int l) -> void* { return a.ws + (size_t)l * a256; };
     auto mask = [&](int l) {
         return reinterpret_cast<const uint32_t*>(static_cast<const uint8_t*>(a.masks) +
                                                  (size_t)l * mb);
@@ -561,10 +561,9 @@ int stack_bwd_bf16(const Shape& sh, const StackBwdArgs& a, const StackBwdLayout&
     // output gradient g_l of layer l (the residual term of its input gradient)
     auto g = [&](int l) -> const void* {
         if (l == L - 1) return a.dy;
-        return (relu && resid) ? gbuf(l) : dz(l);
+        return keep_g ? gbuf(l) : dz(l);
     };
     int rc;
-    // dz of the top layer
     if (relu) {
         rc = launched(launch_relu_grad_mask_bf16(static_cast<const __nv_bfloat16*>(a.dy),
                                                  mask(L - 1), static_cast<__nv_bfloat16*>(dz(L - 1)),
@@ -574,17 +573,16 @@ int stack_bwd_bf16(const Shape& sh, const StackBwdArgs& a, const StackBwdLayout&
         rc = cuda_status(cudaMemcpyAsync(dz(L - 1), a.dy, ab, cudaMemcpyDeviceToDevice, st));
     }
     if (rc) return rc;
-    // input gradients, top down
-    int* counters = reinterpret_cast<int*>(a.ws + lay.ctr_off);
+    int* counters = reinterpret_cast<int*>(a.ws + (keep_g ? (size_t)L * a256 : 0));
     const int n_chunks = (int)((sh.tokens + 127) / 128);
+    const int pw = epi_patch_cols(BN);
     static thread_local TcLaunch<kMaxStackLayers> T;
     for (int top = L - 1; top >= 0; top -= kMaxStackLayers) {
         const int cnt = top + 1 < kMaxStackLayers ? top + 1 : kMaxStackLayers;
         memset(&T, 0, sizeof(T));
-        const int pw = epi_patch_cols(BN);
         for (int i = 0; i < cnt; ++i) {
             const int l = top - i;
-            const int s = layer_dim(sh, a, l);
+            const int s = stack_layer_dim(sh, a.layer0, a.dim_override, l);
             const int k = 1 << s;
             // stores: g_{l-1} (map 4) and dz_{l-1} (map 5); at l = 0 the stack's dx
             void* out = l == 0 ? a.dx : (relu ? (resid ? gbuf(l - 1) : nullptr) : dz(l - 1));
@@ -615,19 +613,37 @@ int stack_bwd_bf16(const Shape& sh, const StackBwdArgs& a, const StackBwdLayout&
         rc = launched(launch_tc_stack(MODE_DX, BN, T, total < sms ? total : sms, st), 1);
         if (rc) return rc;
     }
-    // weight gradients: runs of up to 16 independent layers in one launch,
-    // whole token range per tile; too few tiles to fill the GPU -> per layer
+    return HCW_OK;
+}
+
+// bf16 weight gradients: runs of up to 16 independent layers in one launch
+// (whole token range per tile, units handed out longest first), or layer by
+// layer when their tiles cannot fill the GPU; then one batched column sum
+// for every layer's dbias.
+int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
+    const int d = sh.d, BN = pick_bn(d), L = a.L;
+    const size_t ab = sh.act_bytes;
+    const WsLayout wl = ws_layout(sh.tokens, d, HCW_BF16, a.flags);
+    int* sched = reinterpret_cast<int*>(a.ws);
+    uint8_t* wws = a.ws + 256;
+    float* col = reinterpret_cast<float*>(a.ws + 256 + wl.w_bytes);
+    auto dz = [&](int l) -> const void* { return a.dz + (size_t)l * ab; };
+    auto act = [&](int l) -> const void* {
+        return l == 0 ? a.x : static_cast<const uint8_t*>(a.acts) + (size_t)(l - 1) * ab;
+    };
     const WPlan w1 = plan_dw(sh.tokens, d, a.flags);
     const int tiles = w1.n_ot * w1.n_nt;
     const int sms = sm_count();
+    static thread_local TcLaunch<kMaxStackLayers> T;
+    int rc;
     for (int l0 = 0; l0 < L; l0 += kMaxStackLayers) {
         const int cnt = L - l0 < kMaxStackLayers ? L - l0 : kMaxStackLayers;
         if (cnt * tiles * 2 < sms) {
             for (int l = l0; l < l0 + cnt; ++l) {
                 Shape shl = sh;
-                shl.s = layer_dim(sh, a, l);
+                shl.s = stack_layer_dim(sh, a.layer0, a.dim_override, l);
                 rc = dw_bf16(shl, act(l), dz(l), a.flags, a.dWs + (size_t)l * d * d,
-                             a.dWn + (size_t)l * d * d, nullptr, a.ws + lay.w_off, st);
+                             a.dWn + (size_t)l * d * d, nullptr, wws, st);
                 if (rc) return rc;
             }
             continue;
@@ -635,7 +651,7 @@ int stack_bwd_bf16(const Shape& sh, const StackBwdArgs& a, const StackBwdLayout&
         memset(&T, 0, sizeof(T));
         for (int i = 0; i < cnt; ++i) {
             const int l = l0 + i;
-            const int s = layer_dim(sh, a, l);
+            const int s = stack_layer_dim(sh, a.layer0, a.dim_override, l);
             const int k = 1 << s;
             CUtensorMap* m = T.maps[i];
             if (!map_rows(&m[0], dz(l), sh.tokens, d, k, 64) ||
@@ -664,83 +680,139 @@ int stack_bwd_bf16(const Shape& sh, const StackBwdArgs& a, const StackBwdLayout&
         p.n_units = tiles * 2;
         p.timeout_ns = g_timeout_ns;
         T.n_layers = cnt;
-        T.sched = counters;
-        if (cudaMemsetAsync(counters, 0, sizeof(int), st) != cudaSuccess) return HCW_ERR_CUDA;
+        T.sched = sched;
+        if (cudaMemsetAsync(sched, 0, sizeof(int), st) != cudaSuccess) return HCW_ERR_CUDA;
         const int total = p.n_units * cnt;
         rc = launched(launch_tc_stack(MODE_DW, BN, T, total < sms ? total : sms, st), 1);
         if (rc) return rc;
     }
-    // bias gradients of every layer: one batched column sum (the dz buffers
-    // are contiguous when the activation size is a multiple of 256 bytes)
-    if (a.dbias && a256 != ab) {
-        for (int l = 0; l < L; ++l) {
-            rc = launched(launch_colsum_bf16(static_cast<const __nv_bfloat16*>(dz(l)), sh.tokens, d,
-                                             reinterpret_cast<float*>(a.ws + lay.col_off),
-                                             a.dbias + (size_t)l * d, st),
-                          2);
-            if (rc) return rc;
-        }
-        return HCW_OK;
-    }
     if (a.dbias)
         return launched(launch_colsum_bf16_batched(static_cast<const __nv_bfloat16*>(dz(0)), L,
-                                                   sh.tokens, d,
-                                                   reinterpret_cast<float*>(a.ws + lay.col_off),
-                                                   a.dbias, st),
+                                                   sh.tokens, d, col, a.dbias, st),
                         2);
     return HCW_OK;
 }
 
-// fp32: layer by layer (the correctness path).
-int stack_bwd_f32(const Shape& sh, const StackBwdArgs& a, const StackBwdLayout& lay,
-                  cudaStream_t st) {
+// fp32 input gradients, layer by layer (the correctness path).
+int stack_data_f32(const Shape& sh, const StackData& a, cudaStream_t st) {
     const int d = sh.d, L = a.L;
     const bool relu = (a.flags & HCW_ACT_RELU) != 0;
     const size_t ab = sh.act_bytes, a256 = align256(ab), wb = (size_t)d * d * 4;
     const size_t mb = mask_bytes(sh);
-    uint8_t* g[2] = {a.ws + lay.g_off, a.ws + lay.g_off + a256};
-    uint8_t* dzb[2] = {a.ws, a.ws + a256};
+    uint8_t* g[2] = {a.ws, a.ws + a256};
+    auto dz = [&](int l) -> void* { return a.dz + (size_t)l * ab; };
     auto mask = [&](int l) {
         return reinterpret_cast<const uint32_t*>(static_cast<const uint8_t*>(a.masks) +
                                                  (size_t)l * mb);
     };
-    const void* cur_g = a.dy;
-    const void* cur_dz = a.dy;
     int rc;
     if (relu) {
         rc = launched(launch_relu_grad_mask_f32(static_cast<const float*>(a.dy), mask(L - 1),
-                                                reinterpret_cast<float*>(dzb[(L - 1) & 1]),
-                                                sh.tokens, d, st),
+                                                static_cast<float*>(dz(L - 1)), sh.tokens, d, st),
                       1);
-        if (rc) return rc;
-        cur_dz = dzb[(L - 1) & 1];
+    } else {
+        rc = cuda_status(cudaMemcpyAsync(dz(L - 1), a.dy, ab, cudaMemcpyDeviceToDevice, st));
     }
+    if (rc) return rc;
+    const void* cur_g = a.dy;
     for (int l = L - 1; l >= 0; --l) {
         Shape shl = sh;
-        shl.s = layer_dim(sh, a, l);
-        const void* in = l == 0 ? a.x : static_cast<const uint8_t*>(a.acts) + (size_t)(l - 1) * ab;
-        rc = layer_dw_impl(shl, HCW_F32, in, cur_dz, a.flags, a.dWs + (size_t)l * d * d,
-                           a.dWn + (size_t)l * d * d, a.dbias ? a.dbias + (size_t)l * d : nullptr,
-                           a.ws + lay.w_off, st);
-        if (rc) return rc;
-        void* out_g = l == 0 ? a.dx : (void*)g[l & 1];
-        rc = layer_dx_impl(shl, HCW_F32, cur_dz, cur_g, a.Ws + l * wb, a.Wn + l * wb, a.flags,
-                           out_g, st);
+        shl.s = stack_layer_dim(sh, a.layer0, a.dim_override, l);
+        void* out = l == 0 ? a.dx : (relu ? (void*)g[l & 1] : dz(l - 1));
+        rc = layer_dx_impl(shl, HCW_F32, dz(l), cur_g, a.Ws + l * wb, a.Wn + l * wb, a.flags, out,
+                           st);
         if (rc) return rc;
         if (l == 0) break;
-        const void* next_dz = out_g;
         if (relu) {
-            rc = launched(launch_relu_grad_mask_f32(static_cast<const float*>(out_g), mask(l - 1),
-                                                    reinterpret_cast<float*>(dzb[(l - 1) & 1]),
-                                                    sh.tokens, d, st),
+            rc = launched(launch_relu_grad_mask_f32(static_cast<const float*>(out), mask(l - 1),
+                                                    static_cast<float*>(dz(l - 1)), sh.tokens, d,
+                                                    st),
                           1);
             if (rc) return rc;
-            next_dz = dzb[(l - 1) & 1];
         }
-        cur_g = out_g;
-        cur_dz = next_dz;
+        cur_g = out;
     }
     return HCW_OK;
+}
+
+// fp32 weight gradients, layer by layer.
+int stack_weight_f32(const Shape& sh, const StackWeight& a, cudaStream_t st) {
+    const int d = sh.d;
+    const size_t ab = sh.act_bytes;
+    for (int l = 0; l < a.L; ++l) {
+        Shape shl = sh;
+        shl.s = stack_layer_dim(sh, a.layer0, a.dim_override, l);
+        const void* in = l == 0 ? a.x : static_cast<const uint8_t*>(a.acts) + (size_t)(l - 1) * ab;
+        const int rc = layer_dw_impl(shl, HCW_F32, in, a.dz + (size_t)l * ab, a.flags,
+                                     a.dWs + (size_t)l * d * d, a.dWn + (size_t)l * d * d,
+                                     a.dbias ? a.dbias + (size_t)l * d : nullptr, a.ws, st);
+        if (rc) return rc;
+    }
+    return HCW_OK;
+}
+
+// Argument checks of the two halves (sizes, pointers, alignment, overlaps).
+int check_stack_data(const Shape& sh, int dtype, unsigned flags, int L, const void* masks,
+                     const void* dy, const void* Ws, const void* Wn, const void* dx,
+                     const void* dz, const void* ws, size_t ws_bytes) {
+    const bool relu = (flags & HCW_ACT_RELU) != 0;
+    if (!dy || !Ws || !Wn || !dx || !dz || (relu && !masks)) return HCW_ERR_INVALID_ARG;
+    const void* ptrs[] = {masks, dy, Ws, Wn, dx, dz};
+    for (const void* q : ptrs)
+        if (q && !aligned16(q)) return HCW_ERR_ALIGNMENT;
+    const size_t need = stack_data_ws(sh, dtype, flags, L);
+    if (ws_bytes < need || (need && !ws)) return HCW_ERR_WORKSPACE;
+    if (ws && !aligned16(ws)) return HCW_ERR_ALIGNMENT;
+    const size_t ab = sh.act_bytes, zb = (size_t)L * ab;
+    const size_t mbs = relu ? (size_t)L * mask_bytes(sh) : 0;
+    const size_t wb = (size_t)L * sh.d * sh.d * elem_size(dtype);
+    const void* ins[][2] = {{dy, (const void*)ab}, {masks, (const void*)mbs},
+                            {Ws, (const void*)wb}, {Wn, (const void*)wb}};
+    for (auto& q : ins) {
+        const size_t n = reinterpret_cast<size_t>(q[1]);
+        if (overlaps(dx, ab, q[0], n) || overlaps(dz, zb, q[0], n) ||
+            overlaps(ws, ws_bytes, q[0], n))
+            return HCW_ERR_ALIASING;
+    }
+    if (overlaps(dx, ab, dz, zb) || overlaps(ws, ws_bytes, dx, ab) || overlaps(ws, ws_bytes, dz, zb))
+        return HCW_ERR_ALIASING;
+    return HCW_OK;
+}
+
+int check_stack_weight(const Shape& sh, int dtype, unsigned flags, int L, const void* x,
+                       const void* acts, const void* dz, const float* dWs, const float* dWn,
+                       const float* dbias, const void* ws, size_t ws_bytes) {
+    if (!x || !dz || !dWs || !dWn || (L > 1 && !acts)) return HCW_ERR_INVALID_ARG;
+    const void* ptrs[] = {x, acts, dz, dWs, dWn, dbias};
+    for (const void* q : ptrs)
+        if (q && !aligned16(q)) return HCW_ERR_ALIGNMENT;
+    const size_t need = stack_weight_ws(sh, dtype, flags, L);
+    if (ws_bytes < need || (need && !ws)) return HCW_ERR_WORKSPACE;
+    if (ws && !aligned16(ws)) return HCW_ERR_ALIGNMENT;
+    const size_t ab = sh.act_bytes, gb = (size_t)L * sh.d * sh.d * 4, bb = (size_t)L * sh.d * 4;
+    const size_t acts_b = (size_t)(L - 1) * ab;
+    const void* outs[][2] = {{dWs, (const void*)gb}, {dWn, (const void*)gb},
+                             {dbias, (const void*)bb}, {ws, (const void*)ws_bytes}};
+    const void* ins[][2] = {{x, (const void*)ab}, {acts, (const void*)acts_b},
+                            {dz, (const void*)((size_t)L * ab)}};
+    for (int i = 0; i < 4; ++i) {
+        const size_t ni = reinterpret_cast<size_t>(outs[i][1]);
+        for (auto& q : ins)
+            if (overlaps(outs[i][0], ni, q[0], reinterpret_cast<size_t>(q[1])))
+                return HCW_ERR_ALIASING;
+        for (int j = i + 1; j < 4; ++j)
+            if (overlaps(outs[i][0], ni, outs[j][0], reinterpret_cast<size_t>(outs[j][1])))
+                return HCW_ERR_ALIASING;
+    }
+    return HCW_OK;
+}
+
+int zero_weight_grads(int L, int d, float* dWs, float* dWn, float* dbias, cudaStream_t st) {
+    const size_t gbytes = (size_t)L * d * d * sizeof(float);
+    cudaError_t e = cudaMemsetAsync(dWs, 0, gbytes, st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(dWn, 0, gbytes, st);
+    if (e == cudaSuccess && dbias) e = cudaMemsetAsync(dbias, 0, (size_t)L * d * 4, st);
+    return cuda_status(e);
 }
 
 int check_fwd_ptrs(const Shape& sh, int dtype, const void* x, const void* Ws, const void* Wn,
@@ -989,10 +1061,65 @@ int hcw_stack_fwd(const void* x, const void* W_self, const void* W_nbr, const fl
     return HCW_OK;
 }
 
+size_t hcw_stack_bwd_data_workspace_bytes(int B, int n, int d, int dtype, unsigned flags,
+                                          int L) {
+    Shape sh;
+    if (L < 1 || check_shape(0, -1, B, n, d, dtype, flags, &sh)) return 0;
+    return stack_data_ws(sh, dtype, flags, L);
+}
+
+size_t hcw_stack_bwd_weight_workspace_bytes(int B, int n, int d, int dtype, unsigned flags,
+                                            int L) {
+    Shape sh;
+    if (L < 1 || check_shape(0, -1, B, n, d, dtype, flags, &sh)) return 0;
+    return stack_weight_ws(sh, dtype, flags, L);
+}
+
 size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags, int L) {
     Shape sh;
     if (L < 1 || check_shape(0, -1, B, n, d, dtype, flags, &sh)) return 0;
-    return stack_bwd_layout(sh, dtype, flags, L).total;
+    return stack_dz_bytes(sh, L) + align256(stack_data_ws(sh, dtype, flags, L)) +
+           stack_weight_ws(sh, dtype, flags, L);
+}
+
+int hcw_stack_bwd_data(const void* masks, const void* dy, const void* W_self, const void* W_nbr,
+                       int layer0, int L, int dim_override, int B, int n, int d, int dtype,
+                       unsigned flags, void* dx, void* dz, void* workspace, size_t ws_bytes,
+                       void* stream) {
+    Shape sh;
+    if (L < 1) return HCW_ERR_INVALID_ARG;
+    int rc = check_shape(layer0, dim_override, B, n, d, dtype, flags, &sh);
+    if (rc) return rc;
+    if (sh.tokens == 0) return HCW_OK;
+    rc = check_stack_data(sh, dtype, flags, L, masks, dy, W_self, W_nbr, dx, dz, workspace,
+                          ws_bytes);
+    if (rc) return rc;
+    StackData a{masks, dy, static_cast<const uint8_t*>(W_self), static_cast<const uint8_t*>(W_nbr),
+                layer0, L, dim_override, flags, dx, static_cast<uint8_t*>(dz),
+                static_cast<uint8_t*>(workspace)};
+    return dtype == HCW_BF16 ? stack_data_bf16(sh, a, (cudaStream_t)stream)
+                             : stack_data_f32(sh, a, (cudaStream_t)stream);
+}
+
+int hcw_stack_bwd_weight(const void* x, const void* acts, const void* dz, int layer0, int L,
+                         int dim_override, int B, int n, int d, int dtype, unsigned flags,
+                         float* dW_self, float* dW_nbr, float* dbias, void* workspace,
+                         size_t ws_bytes, void* stream) {
+    Shape sh;
+    if (L < 1) return HCW_ERR_INVALID_ARG;
+    int rc = check_shape(layer0, dim_override, B, n, d, dtype, flags, &sh);
+    if (rc) return rc;
+    if (sh.tokens == 0) {
+        if (!dW_self || !dW_nbr) return HCW_ERR_INVALID_ARG;
+        return zero_weight_grads(L, d, dW_self, dW_nbr, dbias, (cudaStream_t)stream);
+    }
+    rc = check_stack_weight(sh, dtype, flags, L, x, acts, dz, dW_self, dW_nbr, dbias, workspace,
+                            ws_bytes);
+    if (rc) return rc;
+    StackWeight a{x, acts, static_cast<const uint8_t*>(dz), layer0, L, dim_override, flags,
+                  dW_self, dW_nbr, dbias, static_cast<uint8_t*>(workspace)};
+    return dtype == HCW_BF16 ? stack_weight_bf16(sh, a, (cudaStream_t)stream)
+                             : stack_weight_f32(sh, a, (cudaStream_t)stream);
 }
 
 int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void* dy,
@@ -1003,50 +1130,39 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void
     if (L < 1) return HCW_ERR_INVALID_ARG;
     int rc = check_shape(layer0, dim_override, B, n, d, dtype, flags, &sh);
     if (rc) return rc;
+    cudaStream_t st = (cudaStream_t)stream;
     if (sh.tokens == 0) {
         if (!dW_self || !dW_nbr) return HCW_ERR_INVALID_ARG;
-        cudaStream_t st0 = (cudaStream_t)stream;
-        const size_t gbytes = (size_t)L * d * d * sizeof(float);
-        cudaError_t e = cudaMemsetAsync(dW_self, 0, gbytes, st0);
-        if (e == cudaSuccess) e = cudaMemsetAsync(dW_nbr, 0, gbytes, st0);
-        if (e == cudaSuccess && dbias) e = cudaMemsetAsync(dbias, 0, (size_t)L * d * 4, st0);
-        return cuda_status(e);
+        return zero_weight_grads(L, d, dW_self, dW_nbr, dbias, st);
     }
-    const bool relu = (flags & HCW_ACT_RELU) != 0;
-    if ((L > 1 && !acts) || (relu && !masks)) return HCW_ERR_INVALID_ARG;
-    rc = check_bwd_ptrs(sh, dtype, flags & ~HCW_ACT_RELU, x, nullptr, dy, W_self, W_nbr, dx,
-                        dW_self, dW_nbr, dbias);
-    if (rc) return rc;
-    if ((acts && !aligned16(acts)) || (masks && !aligned16(masks))) return HCW_ERR_ALIGNMENT;
-    const size_t ab = sh.act_bytes, gb = (size_t)d * d * 4, mb = mask_bytes(sh);
-    const StackBwdLayout lay = stack_bwd_layout(sh, dtype, flags, L);
-    if (ws_bytes < lay.total || !workspace) return HCW_ERR_WORKSPACE;
+    // workspace: [dz of every layer][input-gradient scratch][weight-gradient scratch]
+    const size_t zb = stack_dz_bytes(sh, L);
+    const size_t db = align256(stack_data_ws(sh, dtype, flags, L));
+    const size_t wb = stack_weight_ws(sh, dtype, flags, L);
+    if (ws_bytes < zb + db + wb || !workspace) return HCW_ERR_WORKSPACE;
     if (!aligned16(workspace)) return HCW_ERR_ALIGNMENT;
-    const size_t acts_b = (size_t)(L > 1 ? L - 1 : 0) * ab;
-    if (overlaps(workspace, ws_bytes, dx, ab) || overlaps(workspace, ws_bytes, dy, ab) ||
-        overlaps(workspace, ws_bytes, x, ab) || overlaps(workspace, ws_bytes, acts, acts_b) ||
-        overlaps(workspace, ws_bytes, masks, relu ? (size_t)L * mb : 0) ||
-        overlaps(dW_self, (size_t)L * gb, dW_nbr, (size_t)L * gb) || overlaps(dx, ab, acts, acts_b) ||
-        overlaps(dx, ab, masks, relu ? (size_t)L * mb : 0))
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    rc = check_stack_data(sh, dtype, flags, L, masks, dy, W_self, W_nbr, dx, ws, ws + zb, db);
+    if (rc) return rc;
+    rc = check_stack_weight(sh, dtype, flags, L, x, acts, ws, dW_self, dW_nbr, dbias, ws + zb + db,
+                            wb);
+    if (rc) return rc;
+    // the weight gradients read x and acts; the input gradients write dx
+    const size_t ab = sh.act_bytes;
+    if (overlaps(dx, ab, x, ab) || overlaps(dx, ab, acts, (size_t)(L - 1) * ab) ||
+        overlaps(ws, ws_bytes, x, ab) || overlaps(ws, ws_bytes, acts, (size_t)(L - 1) * ab) ||
+        overlaps(dx, ab, dW_self, (size_t)L * d * d * 4) ||
+        overlaps(dx, ab, dW_nbr, (size_t)L * d * d * 4) ||
+        overlaps(dx, ab, dbias, dbias ? (size_t)L * d * 4 : 0))
         return HCW_ERR_ALIASING;
-    StackBwdArgs a;
-    a.x = x;
-    a.acts = acts;
-    a.masks = masks;
-    a.dy = dy;
-    a.Ws = static_cast<const uint8_t*>(W_self);
-    a.Wn = static_cast<const uint8_t*>(W_nbr);
-    a.layer0 = layer0;
-    a.L = L;
-    a.dim_override = dim_override;
-    a.flags = flags;
-    a.dx = dx;
-    a.dWs = dW_self;
-    a.dWn = dW_nbr;
-    a.dbias = dbias;
-    a.ws = static_cast<uint8_t*>(workspace);
-    return dtype == HCW_BF16 ? stack_bwd_bf16(sh, a, lay, (cudaStream_t)stream)
-                             : stack_bwd_f32(sh, a, lay, (cudaStream_t)stream);
+    StackData da{masks, dy, static_cast<const uint8_t*>(W_self),
+                 static_cast<const uint8_t*>(W_nbr), layer0, L, dim_override, flags, dx, ws,
+                 ws + zb};
+    rc = dtype == HCW_BF16 ? stack_data_bf16(sh, da, st) : stack_data_f32(sh, da, st);
+    if (rc) return rc;
+    StackWeight wa{x, acts, ws, layer0, L, dim_override, flags, dW_self, dW_nbr, dbias,
+                   ws + zb + db};
+    return dtype == HCW_BF16 ? stack_weight_bf16(sh, wa, st) : stack_weight_f32(sh, wa, st);
 }
 
 unsigned long long hcw_launch_count(void) { return g_launches.load(); }

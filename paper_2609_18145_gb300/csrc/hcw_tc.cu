@@ -27,10 +27,11 @@
 // dx row is owned by one CTA, no atomics.
 //
 // DW contracts over tokens: A = dz^T and B = x^T (or the partner rows of x)
-// are loaded as MN-major operands straight from the token-major activations;
-// the token range is split so that the units fill the GPU, and the fp32
-// partials are reduced in a fixed order by a separate kernel
-// (deterministic).
+// are loaded as MN-major operands straight from the token-major activations.
+// A launch over up to 16 layers gives every (layer, part, output tile) one
+// unit over the whole token range; a single layer splits the token range so
+// that its units fill the GPU and a separate kernel reduces the fp32
+// partials in a fixed order.  Both are deterministic.
 //
 // Roles: warp 0 issues TMA loads into a ring of shared-memory stages; warp 1
 // owns TMEM (2 x BN fp32 columns, a double-buffered accumulator) and issues

@@ -63,6 +63,12 @@ _SIGNATURES = {
                        _P], _I),
     "hcw_stack_fwd_workspace_bytes": ([_I, _I, _I, _I, _U, _I], _SZ),
     "hcw_stack_workspace_bytes": ([_I, _I, _I, _I, _U, _I], _SZ),
+    "hcw_stack_bwd_data": ([_P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _SZ,
+                            _P], _I),
+    "hcw_stack_bwd_data_workspace_bytes": ([_I, _I, _I, _I, _U, _I], _SZ),
+    "hcw_stack_bwd_weight": ([_P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P, _SZ,
+                              _P], _I),
+    "hcw_stack_bwd_weight_workspace_bytes": ([_I, _I, _I, _I, _U, _I], _SZ),
     "hcw_stack_bwd": ([_P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P,
                        _P, _P, _SZ, _P], _I),
     "hcw_sync_status": ([_P], _I),
@@ -294,6 +300,56 @@ def hcw_stack_bwd(x, acts, masks, dy, W_self, W_nbr, layer0: int = 0, dim_overri
                                _ptr(dx), _ptr(dW_self), _ptr(dW_nbr), _ptr(dbias), _ptr(ws),
                                ws.numel(), _stream(stream)), "hcw_stack_bwd")
     return dx, dW_self, dW_nbr, dbias
+
+
+def hcw_stack_bwd_data_workspace_bytes(B: int, n: int, d: int, dtype: int, flags: int,
+                                       L: int) -> int:
+    return int(lib().hcw_stack_bwd_data_workspace_bytes(B, n, d, dtype, flags, L))
+
+
+def hcw_stack_bwd_weight_workspace_bytes(B: int, n: int, d: int, dtype: int, flags: int,
+                                         L: int) -> int:
+    return int(lib().hcw_stack_bwd_weight_workspace_bytes(B, n, d, dtype, flags, L))
+
+
+def hcw_stack_bwd_data(masks, dy, W_self, W_nbr, layer0: int = 0, dim_override: int = -1,
+                       flags: int = 0, dx=None, dz=None, workspace=None, stream=None):
+    """Input gradients through the stack; returns (dx, dz[L])."""
+    _dev(masks, dy, W_self, W_nbr, dx, dz, workspace)
+    B, n, d = dy.shape
+    L = W_self.shape[0]
+    dt = _dtype_code(dy)
+    dx = torch.empty_like(dy) if dx is None else dx
+    dz = torch.empty((L, B, n, d), dtype=dy.dtype, device=dy.device) if dz is None else dz
+    need = hcw_stack_bwd_data_workspace_bytes(B, n, d, dt, flags, L)
+    ws = _workspace(need, dy.device, workspace)
+    _check(lib().hcw_stack_bwd_data(_ptr(masks), _ptr(dy), _ptr(W_self), _ptr(W_nbr), layer0, L,
+                                    dim_override, B, n, d, dt, flags, _ptr(dx), _ptr(dz),
+                                    _ptr(ws), ws.numel(), _stream(stream)), "hcw_stack_bwd_data")
+    return dx, dz
+
+
+def hcw_stack_bwd_weight(x, acts, dz, layer0: int = 0, dim_override: int = -1, flags: int = 0,
+                         dW_self=None, dW_nbr=None, dbias=None, want_dbias: bool = True,
+                         workspace=None, stream=None):
+    """Weight gradients of every layer from its input and dz; returns
+    (dW_self[L], dW_nbr[L], dbias[L] or None)."""
+    _dev(x, acts, dz, dW_self, dW_nbr, dbias, workspace)
+    B, n, d = x.shape
+    L = dz.shape[0]
+    dt = _dtype_code(x)
+    f32 = dict(dtype=torch.float32, device=x.device)
+    dW_self = torch.empty(L, d, d, **f32) if dW_self is None else dW_self
+    dW_nbr = torch.empty(L, d, d, **f32) if dW_nbr is None else dW_nbr
+    if dbias is None and want_dbias:
+        dbias = torch.empty(L, d, **f32)
+    need = hcw_stack_bwd_weight_workspace_bytes(B, n, d, dt, flags, L)
+    ws = _workspace(need, x.device, workspace)
+    _check(lib().hcw_stack_bwd_weight(_ptr(x), _ptr(acts), _ptr(dz), layer0, L, dim_override,
+                                      B, n, d, dt, flags, _ptr(dW_self), _ptr(dW_nbr),
+                                      _ptr(dbias), _ptr(ws), ws.numel(), _stream(stream)),
+           "hcw_stack_bwd_weight")
+    return dW_self, dW_nbr, dbias
 
 
 def hcw_sync_status(stream=None) -> int:

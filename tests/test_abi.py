@@ -140,6 +140,59 @@ def test_workspace_sizes_f32(hcw):
     assert hcw.hcw_workspace_bytes(4, 48, 64, hcw.HCW_F32, 0) == 0   # invalid n
 
 
+def test_stack_backward_halves_validation_codes(hcw):
+    P = ctypes.c_void_p
+    L = hcw.lib()
+    B, n, d, Ly = 4, 16, 64, 3
+    act = B * n * d * 2
+    M, DY, WS, WN, DX, DZ, W = (0x10000000 * k for k in range(1, 8))
+    flags = hcw.HCW_CAUSAL | hcw.HCW_RESIDUAL | hcw.HCW_ACT_RELU
+    need = hcw.hcw_stack_bwd_data_workspace_bytes(B, n, d, hcw.HCW_BF16, flags, Ly)
+    assert need > 0
+    args = dict(m=M, dy=DY, ws=WS, wn=WN, dx=DX, dz=DZ, w=W, wsb=need, flags=flags, Ly=Ly)
+
+    def data(**kw):
+        a = dict(args, **kw)
+        return L.hcw_stack_bwd_data(P(a["m"]), P(a["dy"]), P(a["ws"]), P(a["wn"]), 0, a["Ly"],
+                                    -1, B, n, d, hcw.HCW_BF16, a["flags"], P(a["dx"]),
+                                    P(a["dz"]), P(a["w"]), a["wsb"], None)
+
+    assert data(m=0) == hcw.HCW_ERR_INVALID_ARG            # ReLU needs the masks
+    assert data(dz=0) == hcw.HCW_ERR_INVALID_ARG
+    assert data(Ly=0) == hcw.HCW_ERR_INVALID_ARG
+    assert data(wsb=need - 1) == hcw.HCW_ERR_WORKSPACE
+    assert data(dz=DZ + 8) == hcw.HCW_ERR_ALIGNMENT
+    assert data(dx=DZ + (Ly - 1) * act) == hcw.HCW_ERR_ALIASING   # dx inside dz
+    assert data(w=DZ) == hcw.HCW_ERR_ALIASING               # workspace over dz
+    assert data(dz=DY) == hcw.HCW_ERR_ALIASING              # dz over dy
+
+    wneed = hcw.hcw_stack_bwd_weight_workspace_bytes(B, n, d, hcw.HCW_BF16, flags, Ly)
+    assert wneed > 0
+    X, A, GS, GN, GB = (0x20000000 * k for k in range(1, 6))
+
+    def weight(**kw):
+        a = dict(dict(x=X, acts=A, dz=DZ, gs=GS, gn=GN, gb=GB, w=W, wsb=wneed), **kw)
+        return L.hcw_stack_bwd_weight(P(a["x"]), P(a["acts"]), P(a["dz"]), 0, Ly, -1, B, n, d,
+                                      hcw.HCW_BF16, flags, P(a["gs"]), P(a["gn"]), P(a["gb"]),
+                                      P(a["w"]), a["wsb"], None)
+
+    assert weight(acts=0) == hcw.HCW_ERR_INVALID_ARG        # L > 1 needs the layer inputs
+    assert weight(wsb=wneed - 1) == hcw.HCW_ERR_WORKSPACE
+    assert weight(gn=GS) == hcw.HCW_ERR_ALIASING
+    assert weight(gs=DZ) == hcw.HCW_ERR_ALIASING            # gradient written over dz
+    assert weight(gb=GB + 4) == hcw.HCW_ERR_ALIGNMENT
+
+
+def test_stack_workspace_is_the_sum_of_its_parts(hcw):
+    for dt, flags in ((hcw.HCW_BF16, 7), (hcw.HCW_BF16, 1), (hcw.HCW_F32, 7)):
+        B, n, d, Ly = 64, 256, 512, 16
+        total = hcw.hcw_stack_workspace_bytes(B, n, d, dt, flags, Ly)
+        es = 2 if dt == hcw.HCW_BF16 else 4
+        parts = (Ly * B * n * d * es + hcw.hcw_stack_bwd_data_workspace_bytes(B, n, d, dt, flags, Ly)
+                 + hcw.hcw_stack_bwd_weight_workspace_bytes(B, n, d, dt, flags, Ly))
+        assert parts <= total <= parts + 512
+
+
 @pytest.mark.timeout(60)
 def test_workspace_query_terminates_for_wide_layers(hcw):
     # more output tiles than SMs: the split search must stop at one split per part

@@ -348,6 +348,38 @@ def test_split_backward_matches_fused(H):
     assert torch.equal(gb, c)
 
 
+@pytest.mark.parametrize("dtype,flags", [(torch.bfloat16, CAUSAL | RESIDUAL | RELU),
+                                         (torch.bfloat16, CAUSAL), (torch.bfloat16, RELU),
+                                         (torch.float32, CAUSAL | RESIDUAL | RELU),
+                                         (torch.float32, RESIDUAL)])
+def test_stack_backward_halves_match_the_whole(H, dtype, flags):
+    """hcw_stack_bwd_data then hcw_stack_bwd_weight give exactly what
+    hcw_stack_bwd gives, and the dz they pass on is each layer's dy * act'(z)
+    chain (checked on the top layer, where it is dy masked)."""
+    d = 64 if dtype == torch.float32 else 256
+    B, n, L = 4, 64, 5
+    pr = synth.problem(B, n, d, L=L, seed=21, w_std=(1 / (2 * d)) ** 0.5)
+    x, _ = dev(pr.x, dtype)
+    Ws, _ = dev(pr.W_self, dtype)
+    Wn, _ = dev(pr.W_nbr, dtype)
+    dy, _ = dev(pr.dy, dtype)
+    bias = torch.from_numpy(pr.bias).cuda()
+    y, acts, masks = H.hcw_stack_fwd(x, Ws, Wn, bias, 1, -1, flags)
+    dx, gWs, gWn, gb = H.hcw_stack_bwd(x, acts, masks, dy, Ws, Wn, 1, -1, flags)
+    dx2, dz = H.hcw_stack_bwd_data(masks, dy, Ws, Wn, 1, -1, flags)
+    a, b, c = H.hcw_stack_bwd_weight(x, acts, dz, 1, -1, flags)
+    torch.cuda.synchronize()
+    assert H.hcw_sync_status() == H.HCW_OK
+    assert torch.equal(dx, dx2) and torch.equal(gWs, a) and torch.equal(gWn, b)
+    assert torch.equal(gb, c)
+    top = dy.clone()
+    if flags & RELU:
+        bits = masks[L - 1].to(torch.int64) & 0xFFFFFFFF
+        keep = ((bits.unsqueeze(-1) >> torch.arange(32, device=bits.device)) & 1).bool()
+        top = torch.where(keep.reshape(top.shape), top, torch.zeros_like(top))
+    assert torch.equal(dz[L - 1], top)
+
+
 def test_launch_counter_counts_kernels(H):
     pr = synth.problem(2, 16, 64, L=1, seed=1)
     x, _ = dev(pr.x, torch.bfloat16)
