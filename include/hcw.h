@@ -190,9 +190,9 @@ size_t hcw_stack_fwd_workspace_bytes(int B, int n, int d, int dtype, unsigned fl
  * bf16: the input gradients of runs of up to 16 layers go in one persistent
  * launch (top down, a tile starting as soon as the rows it reads are
  * written), whose kernel also applies the ReLU gradient of the layer below;
- * then one launch computes the weight gradients of up to 16 layers (whole
- * token range per tile, no split reduction) and one batched pass the bias
- * gradients.  The workspace keeps every layer's dz.
+ * then one launch computes the weight and bias gradients of up to 16 layers
+ * (whole token range per tile, no split reduction).  The workspace keeps
+ * every layer's dz.
  */
 int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void* dy,
                   const void* W_self, const void* W_nbr, int layer0, int L, int dim_override,
@@ -230,7 +230,7 @@ size_t hcw_stack_bwd_data_workspace_bytes(int B, int n, int d, int dtype, unsign
  *   dbias[l] = sum_i dz_l,i (dbias may be NULL).  fp32 outputs [L][d][d], [L][d].
  *   workspace: at least hcw_stack_bwd_weight_workspace_bytes(...) bytes.
  * bf16: up to 16 layers per launch, whole token range per tile (no split
- * reduction, deterministic), then one batched column sum for the biases.
+ * reduction, deterministic); the same kernel sums dz's columns into dbias.
  */
 int hcw_stack_bwd_weight(const void* x, const void* acts, const void* dz, int layer0, int L,
                          int dim_override, int B, int n, int d, int dtype, unsigned flags,

@@ -491,10 +491,9 @@ int layer_bwd_impl(const Shape& sh, int dtype, const void* x, const void* z, con
 //   ReLU and the residual are on (the residual term of that layer's input
 //   gradient; otherwise g is dz itself or dy), then the completion counters
 //   of the stacked launch.  fp32: two g buffers used in turn.
-//   weight gradients, bf16: the unit counter of the batched launch, the
+//   weight gradients, bf16: the unit counter of the batched launch, then the
 //   single-layer weight-gradient workspace (used when the layers are too few
-//   to fill the GPU and run one by one), the column-sum partials of every
-//   layer's dbias.  fp32: the single-layer workspace.
+//   to fill the GPU and run one by one).  fp32: the single-layer workspace.
 //   hcw_stack_bwd: every layer's dz, then both of the above.
 size_t stack_data_ws(const Shape& sh, int dtype, unsigned flags, int L) {
     const size_t a = align256(sh.act_bytes);
@@ -507,8 +506,7 @@ size_t stack_data_ws(const Shape& sh, int dtype, unsigned flags, int L) {
 
 size_t stack_weight_ws(const Shape& sh, int dtype, unsigned flags, int L) {
     const WsLayout w = ws_layout(sh.tokens, sh.d, dtype, flags);
-    if (dtype == HCW_BF16)
-        return 256 + w.w_bytes + (size_t)L * align256(colsum_workspace_bytes(sh.tokens, sh.d));
+    if (dtype == HCW_BF16) return 256 + w.w_bytes;
     return w.w_bytes;
 }
 
@@ -617,16 +615,15 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
 }
 
 // bf16 weight gradients: runs of up to 16 independent layers in one launch
-// (whole token range per tile, units handed out longest first), or layer by
-// layer when their tiles cannot fill the GPU; then one batched column sum
-// for every layer's dbias.
+// (whole token range per tile, units handed out longest first; the kernel
+// also sums dz's columns into dbias), or layer by layer when their tiles
+// cannot fill the GPU.
 int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
     const int d = sh.d, BN = pick_bn(d), L = a.L;
     const size_t ab = sh.act_bytes;
     const WsLayout wl = ws_layout(sh.tokens, d, HCW_BF16, a.flags);
     int* sched = reinterpret_cast<int*>(a.ws);
     uint8_t* wws = a.ws + 256;
-    float* col = reinterpret_cast<float*>(a.ws + 256 + wl.w_bytes);
     auto dz = [&](int l) -> const void* { return a.dz + (size_t)l * ab; };
     auto act = [&](int l) -> const void* {
         return l == 0 ? a.x : static_cast<const uint8_t*>(a.acts) + (size_t)(l - 1) * ab;
@@ -643,7 +640,8 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
                 Shape shl = sh;
                 shl.s = stack_layer_dim(sh, a.layer0, a.dim_override, l);
                 rc = dw_bf16(shl, act(l), dz(l), a.flags, a.dWs + (size_t)l * d * d,
-                             a.dWn + (size_t)l * d * d, nullptr, wws, st);
+                             a.dWn + (size_t)l * d * d, a.dbias ? a.dbias + (size_t)l * d : nullptr,
+                             wws, st);
                 if (rc) return rc;
             }
             continue;
@@ -661,7 +659,8 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
                 return HCW_ERR_CUDA;
             m[2] = m[1];
             m[3] = m[4];
-            T.layer[i] = {s, k, nullptr, nullptr, nullptr, false, nullptr, false};
+            T.layer[i] = {s, k, nullptr, nullptr, nullptr, false, nullptr, false,
+                          a.dbias ? a.dbias + (size_t)l * d : nullptr};
         }
         TcParams& p = T.p;
         memset(&p, 0, sizeof(p));
@@ -686,10 +685,6 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
         rc = launched(launch_tc_stack(MODE_DW, BN, T, total < sms ? total : sms, st), 1);
         if (rc) return rc;
     }
-    if (a.dbias)
-        return launched(launch_colsum_bf16_batched(static_cast<const __nv_bfloat16*>(dz(0)), L,
-                                                   sh.tokens, d, col, a.dbias, st),
-                        2);
     return HCW_OK;
 }
 

@@ -55,6 +55,7 @@ struct TcLayer {
     bool out;                     // DX: the input gradient dx is stored (map 4)
     const uint32_t* mprev;        // DX: ReLU mask words of the layer below (fused ReLU grad)
     bool dz_out;                  // DX: dz of the layer below = dx * mask is stored (map 5)
+    float* colsum;                // DW, whole token range per unit: dbias = column sums of dz
 };
 
 // Columns of one epilogue patch (the inner extent of the 32-row residual and

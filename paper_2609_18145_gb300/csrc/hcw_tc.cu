@@ -58,6 +58,7 @@ namespace {
 
 constexpr int kMaxEpiWarps = 16;
 constexpr int kUnitQ = 8;                          // claimed units in flight per CTA
+constexpr int kDwHelpers = 4;                      // DW: epilogue warps that also release stages
 constexpr int kBlockM = 128;
 constexpr int kBlockK = 64;                        // bf16 elements per 128-byte row
 constexpr int kABytes = kBlockM * kBlockK * 2;     // 16 KB
@@ -341,7 +342,9 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
             for (int i = 0; i < 6; ++i) tma_prefetch_desc(&L.maps[l][i]);
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&bars->full[s], 1);
-            mbar_init(&bars->empty[s], 1);
+            // DW: the MMA commit and the helper warps (which read the dz tiles for
+            // the bias gradient) both release a stage
+            mbar_init(&bars->empty[s], MODE == MODE_DW ? 1 + kDwHelpers : 1);
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&bars->tfull[a], 1);
@@ -592,6 +595,8 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
         uint8_t* buf = epi_smem + (size_t)e * kEpiBufBytes;
         float* wbias = bias_smem + e * WCOLS;
         uint32_t ld_phase = 0;
+        int hstage = 0;          // DW helper warps: ring position, as the MMA thread's
+        uint32_t hphase = 0;
         int acc = 0;
         uint32_t acc_phase = 0;
         bool alive = true;
@@ -842,6 +847,66 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                 }
             } else {
                 const WUnit& w = wu;
+                if (e < kDwHelpers) {
+                    // Helper warps follow the MMA thread through the unit's stages and
+                    // release each one; when the unit covers every token of its
+                    // output-row tile (self part, first column tile, no split), they
+                    // also add up the dz tile's columns on the way: dbias of 128
+                    // rows.  Thread t sums the 16-byte piece c of box t / 64 (64 dz
+                    // rows each) over the tile rows r = t % 8 (mod 8), then the eight
+                    // row phases are added with shuffles: a fixed order.
+                    const int steps = w.kb1 - w.kb0;
+                    const bool do_cs = ly.colsum != nullptr && w.which == 0 && w.nt == 0 &&
+                                       p.splits_self == 1;
+                    const int t = e * 32 + lane;
+                    const int box = t >> 6, c = (t >> 3) & 7, tp = t & 7;
+                    float cs[8];
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) cs[i] = 0.f;
+                    for (int ks = 0; ks < steps; ++ks) {
+                        if (!wait_bar(&bars->full[hstage], hphase)) {
+                            alive = false;
+                            break;
+                        }
+                        if (do_cs) {
+                            const uint8_t* sA = smem + (size_t)hstage * SB + box * 8192;
+#pragma unroll
+                            for (int i = 0; i < 8; ++i) {
+                                const int r = tp + 8 * i;
+                                const uint4 q = *reinterpret_cast<const uint4*>(
+                                    sA + r * 128 + ((c ^ tp) << 4));
+                                const uint32_t wv[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+                                for (int j = 0; j < 4; ++j) {
+                                    const float2 f = unpack_bf16x2(wv[j]);
+                                    cs[2 * j] += f.x;
+                                    cs[2 * j + 1] += f.y;
+                                }
+                            }
+                        }
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(&bars->empty[hstage]);
+                        if (++hstage == STAGES) {
+                            hstage = 0;
+                            hphase ^= 1;
+                        }
+                    }
+                    if (!alive) break;
+                    if (do_cs) {
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            cs[i] += __shfl_xor_sync(0xffffffffu, cs[i], 1);
+                            cs[i] += __shfl_xor_sync(0xffffffffu, cs[i], 2);
+                            cs[i] += __shfl_xor_sync(0xffffffffu, cs[i], 4);
+                        }
+                        const int o0 = w.ot * kBlockM + box * 64 + c * 8;
+                        if (tp == 0 && o0 < p.d) {
+                            float4* dst = reinterpret_cast<float4*>(ly.colsum + o0);
+                            dst[0] = make_float4(cs[0], cs[1], cs[2], cs[3]);
+                            dst[1] = make_float4(cs[4], cs[5], cs[6], cs[7]);
+                        }
+                    }
+                }
                 if (!wait_acc()) {
                     alive = false;
                     break;

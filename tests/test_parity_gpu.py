@@ -380,6 +380,31 @@ def test_stack_backward_halves_match_the_whole(H, dtype, flags):
     assert torch.equal(dz[L - 1], top)
 
 
+def test_batched_weight_gradient_against_fp64_sums(H):
+    """16 layers whose tiles fill the GPU: one weight-gradient launch for all of
+    them, the bias gradient summed inside it.  dW_self[l] = dz_l^T x_l and
+    dbias[l] = column sums of dz_l, recomputed in fp64 from the same bf16
+    tensors (any summation order agrees to fp32 accumulation error)."""
+    B, n, d, L = 8, 256, 512, 16
+    flags = CAUSAL | RESIDUAL | RELU
+    pr = synth.problem(B, n, d, L=L, seed=33, w_std=(1 / (2 * d)) ** 0.5)
+    x, _ = dev(pr.x, torch.bfloat16)
+    Ws, _ = dev(pr.W_self, torch.bfloat16)
+    Wn, _ = dev(pr.W_nbr, torch.bfloat16)
+    dy, _ = dev(pr.dy, torch.bfloat16)
+    bias = torch.from_numpy(pr.bias).cuda()
+    y, acts, masks = H.hcw_stack_fwd(x, Ws, Wn, bias, 0, -1, flags)
+    dx, dz = H.hcw_stack_bwd_data(masks, dy, Ws, Wn, 0, -1, flags)
+    gWs, gWn, gb = H.hcw_stack_bwd_weight(x, acts, dz, 0, -1, flags)
+    torch.cuda.synchronize()
+    assert H.hcw_sync_status() == H.HCW_OK
+    for l in range(L):
+        inp = (x if l == 0 else acts[l - 1]).reshape(-1, d).double()
+        g = dz[l].reshape(-1, d).double()
+        assert rel(host(gb[l]), host(g.sum(0))) <= 1e-5, l
+        assert rel(host(gWs[l]), host(g.T @ inp)) <= 1e-5, l
+
+
 def test_launch_counter_counts_kernels(H):
     pr = synth.problem(2, 16, 64, L=1, seed=1)
     x, _ = dev(pr.x, torch.bfloat16)
