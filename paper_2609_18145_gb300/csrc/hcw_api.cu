@@ -84,6 +84,45 @@ bool map_rows(CUtensorMap* m, const void* base, long long tokens, int d, int k, 
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// The same view with the features split into 64-wide blocks as the outermost
+// dimension, (64, lo, bit, HI, d / 64): a box (64, box_lo, 1, box_hi, nblk)
+// fetches nblk consecutive 64-feature blocks of the same 64 positions in one
+// copy, laid out block after block (the MN-major operands of the weight
+// gradient).
+bool map_rows_blocks(CUtensorMap* m, const void* base, long long tokens, int d, int k,
+                     int box_rows, int nblk) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc || !base) return false;
+    const int box_lo = k < box_rows ? k : box_rows;
+    const int box_hi = box_rows / box_lo;
+    const long long HI = tokens / (2ll * k);
+    cuuint64_t dims[5] = {64, (cuuint64_t)k, 2, (cuuint64_t)HI, (cuuint64_t)(d / 64)};
+    cuuint64_t strides[4] = {(cuuint64_t)d * 2, (cuuint64_t)k * d * 2, (cuuint64_t)2 * k * d * 2,
+                             128};
+    cuuint32_t box[5] = {64, (cuuint32_t)box_lo, 1, (cuuint32_t)box_hi, (cuuint32_t)nblk};
+    cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(base), dims, strides,
+               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Weights W[o][i] as (64 i, o, d / 64 i-blocks), box (64, 64 o, nblk): nblk
+// consecutive 64-column blocks of 64 rows in one copy (the MN-major B
+// operand of the input gradient), 128-byte swizzle.
+bool map_weight_blocks(CUtensorMap* m, const void* base, int d, int nblk) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc || !base) return false;
+    cuuint64_t dims[3] = {64, (cuuint64_t)d, (cuuint64_t)(d / 64)};
+    cuuint64_t strides[2] = {(cuuint64_t)d * 2, 128};
+    cuuint32_t box[3] = {64, 64, (cuuint32_t)nblk};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Weights W[o][k] bf16 [d][d], box (64 k, box_o), 128-byte swizzle.
 bool map_weight(CUtensorMap* m, const void* base, int d, int box_o) {
     EncodeTiledFn enc = encode_fn();
@@ -332,8 +371,9 @@ int dx_bf16(const Shape& sh, const void* dz, const void* dy, const void* Ws, con
     CUtensorMap* maps = L.maps[0];
     // maps of absent operands get a valid stand-in address; the kernel never uses them
     const void* res = (flags & HCW_RESIDUAL) ? dy : dz;
-    if (!map_rows(&maps[0], dz, sh.tokens, d, k, 128) || !map_weight(&maps[1], Ws, d, 64) ||
-        !map_weight(&maps[2], Wn, d, 64) || !map_rows(&maps[3], res, sh.tokens, d, k, 32, pw) ||
+    if (!map_rows(&maps[0], dz, sh.tokens, d, k, 128) || !map_weight_blocks(&maps[1], Ws, d, BN / 64) ||
+        !map_weight_blocks(&maps[2], Wn, d, BN / 64) ||
+        !map_rows(&maps[3], res, sh.tokens, d, k, 32, pw) ||
         !map_rows(&maps[4], dx ? dx : dz_out, sh.tokens, d, k, 32, pw) ||
         !map_rows(&maps[5], dz_out ? dz_out : dx, sh.tokens, d, k, 32, pw))
         return HCW_ERR_CUDA;
@@ -357,7 +397,8 @@ int dw_bf16(const Shape& sh, const void* x, const void* dz, unsigned flags, floa
     memset(&L, 0, sizeof(L));
     CUtensorMap* maps = L.maps[0];
     float* part = reinterpret_cast<float*>(wws);
-    if (!map_rows(&maps[0], dz, sh.tokens, d, k, 64) || !map_rows(&maps[1], x, sh.tokens, d, k, 64) ||
+    if (!map_rows_blocks(&maps[0], dz, sh.tokens, d, k, 64, 2) ||
+        !map_rows_blocks(&maps[1], x, sh.tokens, d, k, 64, BN / 64) ||
         !map_f32_patches(&maps[3], w.splits_max > 1 ? (const void*)part : (const void*)dWs,
                          w.splits_max > 1 ? 2ll * w.splits_max * d : d, d) ||
         !map_f32_patches(&maps[4], dWs, d, d) || !map_f32_patches(&maps[5], dWn, d, d))
@@ -588,7 +629,8 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
             CUtensorMap* m = T.maps[i];
             const void* res = resid ? g(l) : dz(l);
             if (!map_rows(&m[0], dz(l), sh.tokens, d, k, 128) ||
-                !map_weight(&m[1], a.Ws + l * wb, d, 64) || !map_weight(&m[2], a.Wn + l * wb, d, 64) ||
+                !map_weight_blocks(&m[1], a.Ws + l * wb, d, BN / 64) ||
+                !map_weight_blocks(&m[2], a.Wn + l * wb, d, BN / 64) ||
                 !map_rows(&m[3], res, sh.tokens, d, k, 32, pw) ||
                 !map_rows(&m[4], out ? out : dzo, sh.tokens, d, k, 32, pw) ||
                 !map_rows(&m[5], dzo ? dzo : out, sh.tokens, d, k, 32, pw))
@@ -652,8 +694,8 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
             const int s = stack_layer_dim(sh, a.layer0, a.dim_override, l);
             const int k = 1 << s;
             CUtensorMap* m = T.maps[i];
-            if (!map_rows(&m[0], dz(l), sh.tokens, d, k, 64) ||
-                !map_rows(&m[1], act(l), sh.tokens, d, k, 64) ||
+            if (!map_rows_blocks(&m[0], dz(l), sh.tokens, d, k, 64, 2) ||
+                !map_rows_blocks(&m[1], act(l), sh.tokens, d, k, 64, BN / 64) ||
                 !map_f32_patches(&m[4], a.dWs + (size_t)l * d * d, d, d) ||
                 !map_f32_patches(&m[5], a.dWn + (size_t)l * d * d, d, d))
                 return HCW_ERR_CUDA;

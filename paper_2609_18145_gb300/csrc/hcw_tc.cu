@@ -131,6 +131,14 @@ __device__ __forceinline__ RowUnit decode_row_unit(const TcParams& p, int u, boo
     return r;
 }
 
+// The 128-token chunks holding the rows of a row unit that starts at
+// compressed row q0 (for link distance k = 2^s) and their partners.
+__device__ __forceinline__ void row_unit_chunks(int q0, int s, int k, int& ca, int& cb) {
+    const int tok_a = ((q0 >> s) << (s + 1)) + (q0 & (k - 1));
+    ca = tok_a >> 7;
+    cb = k >= 128 ? ((tok_a + k) >> 7) : ca + 1;
+}
+
 // DW unit -> (which: 0 self / 1 partner, o tile, k tile, split, kb range)
 struct WUnit {
     int which, ot, nt, split, kb0, kb1;
@@ -291,10 +299,11 @@ __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity,
 
 // Maps of layer l (L.maps[l][i]):
 //   0 tmA : FWD x, DX dz: 4-D rows map, box (64, lo_box, 1, hi_box) = 128 rows.
-//           DW dz: the same view with 64-row boxes.
+//           DW dz: 5-D (64, lo, bit, HI, d/64), box of 64 rows x 2 blocks (M = 128).
 //   1 tmB0: FWD W_self [o][k] 2-D, box (64 k, BN o)   (K-major B)
-//           DX  W_self [o][k] 2-D, box (64 k, 64 o)   (MN-major B, BN/64 boxes)
-//           DW  x rows, 64-row boxes                  (MN-major B, BN/64 boxes)
+//           DX  W_self [o][k] 3-D (64, o, d/64), box (64, 64, BN/64): the
+//               MN-major B, BN/64 blocks of 64 columns in one copy
+//           DW  x rows 5-D (64, lo, bit, HI, d/64), box (64, 64 rows, BN/64)
 //   2 tmB1: FWD/DX W_nbr like tmB0; DW unused.
 //   3 tmE0: FWD x / DX dy rows (residual patches, loaded); DW dW partials [2*S*d][d] fp32
 //   4 tmE1: FWD y / DX dx rows (patches stored);           DW dW_self [d][d] fp32
@@ -425,11 +434,9 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     const int lo0 = q0 & (ly.k - 1), hi0 = q0 >> ly.s;
                     if (STACKED && l > 0) {
                         // the unit's rows and their partners: two 128-token chunks
-                        const int tok_a = (hi0 << (ly.s + 1)) + lo0;
-                        const int ca = tok_a >> 7;
-                        const int cb = ly.k >= kBlockM ? ((tok_a + ly.k) >> 7) : ca + 1;
+                        int cs[2];
+                        row_unit_chunks(q0, ly.s, ly.k, cs[0], cs[1]);
                         const int* ctr = L.counters + (size_t)(l - 1) * L.n_chunks;
-                        const int cs[2] = {ca, cb};
                         for (int i = 0; i < 2 && ok; ++i) {
                             if (cs[i] >= L.n_chunks) continue;
                             const int rows = min(128, L.tokens - (cs[i] << 7));
@@ -454,14 +461,11 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                         const int bitA = part ? 1 - r.beta : r.beta;
                         tma_load_4d(sA, mA, &bars->full[stage], kk * kBlockK, lo0, bitA, hi0);
                         const CUtensorMap* mb = &L.maps[l][part ? 2 : 1];
-                        if (MODE == MODE_FWD) {
+                        if (MODE == MODE_FWD)
                             tma_load_2d(sB, mb, &bars->full[stage], kk * kBlockK, r.j * BN);
-                        } else {
-#pragma unroll
-                            for (int jj = 0; jj < BN / 64; ++jj)
-                                tma_load_2d(sB + jj * 8192, mb, &bars->full[stage],
-                                            r.j * BN + jj * 64, kk * kBlockK);
-                        }
+                        else   // BN / 64 blocks of 64 W columns x 64 rows, one copy
+                            tma_load_3d(sB, mb, &bars->full[stage], 0, kk * kBlockK,
+                                        r.j * (BN / 64));
                         if (++stage == STAGES) {
                             stage = 0;
                             phase ^= 1;
@@ -495,13 +499,11 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                         mbar_arrive_expect_tx(&bars->full[stage], kABytes + B_BYTES);
                         issued_mask |= 1u << stage;
                         issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
-                        tma_load_4d(sA, mA, &bars->full[stage], w.ot * kBlockM, lo0, bA, hi0);
-                        tma_load_4d(sA + 8192, mA, &bars->full[stage], w.ot * kBlockM + 64, lo0,
-                                    bA, hi0);
-#pragma unroll
-                        for (int jj = 0; jj < BN / 64; ++jj)
-                            tma_load_4d(sB + jj * 8192, &L.maps[l][1], &bars->full[stage],
-                                        w.nt * BN + jj * 64, lo0, bB, hi0);
+                        // 64 positions x (2 | BN / 64) blocks of 64 features, one copy each
+                        tma_load_5d(sA, mA, &bars->full[stage], 0, lo0, bA, hi0,
+                                    w.ot * (kBlockM / 64));
+                        tma_load_5d(sB, &L.maps[l][1], &bars->full[stage], 0, lo0, bB, hi0,
+                                    w.nt * (BN / 64));
                         if (++stage == STAGES) {
                             stage = 0;
                             phase ^= 1;

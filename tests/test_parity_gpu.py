@@ -306,8 +306,9 @@ def test_charlm_w256_full_launch_sampled(H):
 def test_stack_backward_is_the_chain_of_layer_backwards(H):
     """The stack's forward equals hcw_layer_fwd layer by layer and its ReLU masks
     are exactly (z > 0) of those layers; hcw_stack_bwd on its own saved state
-    equals hcw_layer_bwd applied layer by layer from the top (all bit-exact):
-    the stack plumbing and the fused ReLU gradient add nothing."""
+    equals hcw_layer_bwd applied layer by layer from the top (dx bit-exact,
+    weight and bias gradients up to fp32 summation order): the stack plumbing
+    and the fused ReLU gradient add nothing."""
     for flags in (CAUSAL | RESIDUAL | RELU, CAUSAL | RELU, RESIDUAL):
         B, n, d, L = 4, 256, 512, 5
         pr = synth.problem(B, n, d, L=L, seed=4, w_std=(1 / (2 * d)) ** 0.5)
@@ -330,7 +331,10 @@ def test_stack_backward_is_the_chain_of_layer_backwards(H):
         for l in range(L - 1, -1, -1):
             inp = x if l == 0 else acts[l - 1]
             g, a, b, c = H.hcw_layer_bwd(inp, zs[l], g, Ws[l], Wn[l], 3 + l, -1, flags)
-            assert torch.equal(a, gWs[l]) and torch.equal(b, gWn[l]) and torch.equal(c, gb[l])
+            # the stack accumulates each weight gradient over all tokens in one
+            # pass, the layer call in token splits: same terms, other fp32 order
+            assert rel(host(gWs[l]), host(a)) <= 1e-5 and rel(host(gWn[l]), host(b)) <= 1e-5
+            assert rel(host(gb[l]), host(c)) <= 1e-5
         assert torch.equal(g, dx)
 
 
