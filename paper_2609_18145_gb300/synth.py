@@ -96,10 +96,23 @@ def to_bf16_exact(a: np.ndarray):
     return t, t.to(torch.float64).numpy()
 
 
+def device_normal(shape, seed: int, device):
+    """N(0, 1) float32 drawn on `device` by torch's seeded generator, for inputs
+    too large to draw on the host (the 2^20-token scaling shapes)."""
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    return torch.randn(tuple(shape), generator=g, device=device, dtype=torch.float32)
+
+
 # The workloads, by what they are.  Used by the benchmark and the tests.
 WORKLOADS = {
     "tiny_n16_d32": dict(n=16, d=32, L=4, B=4, causal=False, w_std=(1 / 32) ** 0.5),
     "reach_n64_d128": dict(n=64, d=128, L=6, B=256, causal=False, x_ids="uniform16"),
     "charlm_w64_d512": dict(n=64, d=512, L=16, B=64, causal=True, x_ids="zipf256"),
     "charlm_w256_d512": dict(n=256, d=512, L=16, B=64, causal=True, x_ids="zipf256"),
+    # scaling sweep: 2^20 tokens per batch, L = log2 n rotated layers, d = 1024
+    "scale_n256_d1024": dict(n=256, d=1024, L=8, B=4096, causal=False),
+    "scale_n4096_d1024": dict(n=4096, d=1024, L=12, B=256, causal=False),
+    "scale_n65536_d1024": dict(n=65536, d=1024, L=16, B=16, causal=False),
 }

@@ -262,15 +262,17 @@ def test_reach_workload_full_size(H):
         assert rel(g, r) <= TOL_BF16, what
 
 
-def test_charlm_w256_full_launch_sampled(H):
-    """The timed workload (B = 64, n = 256, d = 512, 16 causal layers, residual,
-    ReLU, bias) in its full launch configuration; the oracle recomputes two
-    sampled sequences.  Forward: the device's rows of those sequences against
-    the oracle.  Backward: the upstream gradient is zero outside them and the
-    device backward sees the oracle's saved activations for them (same ReLU
-    decisions), so its weight gradients over the whole batch must equal the
-    oracle's over the two sequences, and dx must vanish elsewhere."""
-    w = synth.WORKLOADS["charlm_w256_d512"]
+@pytest.mark.parametrize("workload", ["charlm_w256_d512", "charlm_w64_d512"])
+def test_charlm_full_launch_sampled(H, workload):
+    """The char-LM workloads (B = 64, n = 256 or 64, d = 512, 16 causal layers,
+    residual, ReLU, bias) in their full launch configuration; the oracle
+    recomputes two sampled sequences.  Forward: the device's rows of those
+    sequences against the oracle.  Backward: the upstream gradient is zero
+    outside them and the device backward sees the oracle's saved activations
+    for them (same ReLU decisions), so its weight gradients over the whole
+    batch must equal the oracle's over the two sequences, and dx must vanish
+    elsewhere."""
+    w = synth.WORKLOADS[workload]
     B, n, d, L = w["B"], w["n"], w["d"], w["L"]
     flags = CAUSAL | RESIDUAL | RELU
     pr = synth.problem(B, n, d, L=L, seed=0, w_std=(1 / (2 * d)) ** 0.5, x_ids="zipf256")
@@ -301,6 +303,113 @@ def test_charlm_w256_full_launch_sampled(H):
     assert rel(host(gWs), rWs) <= TOL_BF16
     assert rel(host(gWn), rWn) <= TOL_BF16
     assert rel(host(gb), rgb) <= TOL_BF16
+
+
+def test_scaling_n256_d1024_full_launch_sampled(H):
+    """Scaling shape n = 256, d = 1024, 8 rotated non-causal layers, 2^20 tokens
+    (4096 sequences) with random weights, in its full launch configuration;
+    the oracle recomputes one sequence forward, and the backward (upstream
+    gradient zero elsewhere) gives that sequence's weight gradients."""
+    w = synth.WORKLOADS["scale_n256_d1024"]
+    B, n, d, L = w["B"], w["n"], w["d"], w["L"]
+    pick = 1234
+    g = torch.Generator().manual_seed(7)
+    Ws = (torch.randn((L, d, d), generator=g) * (1 / (2 * d)) ** 0.5).to(torch.bfloat16)
+    Wn = (torch.randn((L, d, d), generator=g) * (1 / (2 * d)) ** 0.5).to(torch.bfloat16)
+    bias = torch.randn((L, d), generator=g) * 0.1
+    x = synth.device_normal((B, n, d), 31, "cuda").to(torch.bfloat16)
+    xs = torch.randn((n, d), generator=g).to(torch.bfloat16)     # the sampled sequence
+    x[pick] = xs.cuda()
+    dys = torch.randn((n, d), generator=g).to(torch.bfloat16)
+    dy = torch.zeros((B, n, d), dtype=torch.bfloat16, device="cuda")
+    dy[pick] = dys.cuda()
+    y, acts, _ = H.hcw_stack_fwd(x, Ws.cuda(), Wn.cuda(), bias.cuda(), 0, -1, 0)
+    x64 = xs.double().numpy()[None]
+    W64 = (Ws.double().numpy(), Wn.double().numpy())
+    ry, racts, rzs = O.stack_fwd(x64, W64[0], W64[1], bias.double().numpy(), 0, L, -1, 0,
+                                 round_bf16=True)
+    assert rel(host(y[pick])[None], ry) <= TOL_BF16
+    assert rel(host(acts[:, pick])[:, None], racts[1:]) <= TOL_BF16
+    acts[:, pick] = torch.from_numpy(racts[1:, 0]).to(torch.bfloat16).cuda()
+    dx, gWs, gWn, gb = H.hcw_stack_bwd(x, acts, None, dy, Ws.cuda(), Wn.cuda(), 0, -1, 0)
+    torch.cuda.synchronize()
+    assert H.hcw_sync_status() == H.HCW_OK
+    rdx, rWs, rWn, rgb = O.stack_bwd(racts, rzs, dys.double().numpy()[None], W64[0], W64[1],
+                                     0, L, -1, 0, round_bf16=True)
+    assert rel(host(dx[pick])[None], rdx) <= TOL_BF16
+    others = torch.arange(B, device="cuda") != pick
+    assert float(dx[others].float().abs().max()) == 0.0
+    assert rel(host(gWs), rWs) <= TOL_BF16
+    assert rel(host(gWn), rWn) <= TOL_BF16
+    assert rel(host(gb), rgb) <= TOL_BF16
+
+
+def _block_means(a, l):
+    """Mean of a [n, d] sequence over blocks of 2^l consecutive positions,
+    broadcast back to every position of the block."""
+    n, d = a.shape
+    m = a.reshape(n >> l, 1 << l, d).mean(axis=1)
+    return np.repeat(m, 1 << l, axis=0)
+
+
+def _low_means(a, l):
+    """Mean over the positions that agree with each position on bits 0..l-1
+    (the high bits l..b-1 averaged out), broadcast back."""
+    n, d = a.shape
+    m = a.reshape(n >> l, 1 << l, d).mean(axis=0)
+    return np.tile(m, (n >> l, 1))
+
+
+@pytest.mark.parametrize("workload", ["scale_n4096_d1024", "scale_n65536_d1024"])
+def test_scaling_sweep_identity_weights_any_size(H, workload):
+    """Scaling shapes (2^20 tokens, d = 1024, L = log2 n non-causal layers) with
+    W_self = W_nbr = I/2: layer l averages each position with its partner
+    across bit l, so (the closed form of the pins) layer l's output is the
+    mean over the 2^(l+1)-position block, y is the sequence mean, and the
+    backward is the same averaging: dx = mean of dy over the sequence, and
+    with dz_l the mean of dy over the bits above l, dW_self[l][o][i] =
+    sum_t dz_l[t][o] x_l[t][i] and dW_nbr[l][o][i] = sum_t dz_l[t][o]
+    x_l[t ^ 2^l][i].  Every product is exact, so the device differs from these
+    fp64 values only by its bf16 stores; checked on every position of two
+    sequences (upstream gradient on one of them) and sampled weight-gradient
+    entries."""
+    w = synth.WORKLOADS[workload]
+    B, n, d, L = w["B"], w["n"], w["d"], w["L"]
+    half = torch.eye(d, dtype=torch.bfloat16, device="cuda") * 0.5
+    Ws = half.expand(L, d, d).contiguous()
+    x = synth.device_normal((B, n, d), 41, "cuda").to(torch.bfloat16)
+    dy = torch.zeros((B, n, d), dtype=torch.bfloat16, device="cuda")
+    b0, b1 = 0, B - 1
+    dy[b0] = synth.device_normal((n, d), 42, "cuda").to(torch.bfloat16)
+    y, acts, _ = H.hcw_stack_fwd(x, Ws, Ws, None, 0, -1, 0)
+    dx, dz = H.hcw_stack_bwd_data(None, dy, Ws, Ws, 0, -1, 0)
+    gWs, gWn, gb = H.hcw_stack_bwd_weight(x, acts, dz, 0, -1, 0)
+    torch.cuda.synchronize()
+    assert H.hcw_sync_status() == H.HCW_OK
+    for b in (b0, b1):
+        xb = host(x[b])
+        assert rel(host(y[b]), _block_means(xb, L)) <= TOL_BF16, b
+        for l in (0, L // 2, L - 2):
+            assert rel(host(acts[l, b]), _block_means(xb, l + 1)) <= TOL_BF16, (b, l)
+    dyb = host(dy[b0])
+    assert rel(host(dx[b0]), _block_means(dyb, L)) <= TOL_BF16
+    assert float(dx[b1].float().abs().max()) == 0.0
+    xb = host(x[b0])
+    rng = np.random.default_rng(5)
+    for l in (0, 1, L // 2, L - 1):
+        xl = _block_means(xb, l)                 # layer l's input
+        gl = _low_means(dyb, l + 1)              # gradient at layer l's output (= dz_l)
+        part = np.arange(n) ^ (1 << l)
+        o = rng.integers(0, d, 16)
+        i = rng.integers(0, d, 16)
+        ref_s = np.einsum("tk,tk->k", gl[:, o], xl[:, i])
+        ref_n = np.einsum("tk,tk->k", gl[:, o], xl[part][:, i])
+        got_s = host(gWs[l])[o, i]
+        got_n = host(gWn[l])[o, i]
+        scale = np.abs(ref_s).max() + np.abs(ref_n).max()
+        assert np.abs(got_s - ref_s).max() <= TOL_BF16 * scale, l
+        assert np.abs(got_n - ref_n).max() <= TOL_BF16 * scale, l
+        assert rel(host(gb[l]), gl.sum(axis=0)) <= TOL_BF16, l
 
 
 def test_stack_backward_is_the_chain_of_layer_backwards(H):
