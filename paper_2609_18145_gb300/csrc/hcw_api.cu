@@ -702,8 +702,14 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
             m[2] = m[1];
             m[3] = m[4];
             T.layer[i] = {s, k, nullptr, nullptr, nullptr, false, nullptr, false,
-                          a.dbias ? a.dbias + (size_t)l * d : nullptr};
+                          a.dbias ? a.dbias + (size_t)l * d : nullptr,
+                          a.dWs + (size_t)l * d * d, a.dWn + (size_t)l * d * d};
         }
+        // One unit per (layer, output tile) accumulating the self and the partner
+        // part together reads each dz and input block once (the separate parts
+        // read the receiving rows twice and leave a long tail of short units);
+        // used when those units alone fill most of the GPU.
+        const bool fused = 5 * cnt * tiles >= 3 * sms;
         TcParams& p = T.p;
         memset(&p, 0, sizeof(p));
         p.d = d;
@@ -718,13 +724,15 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
         p.splits_nbr = 1;
         p.splits_max = 1;
         p.causal = (a.flags & HCW_CAUSAL) ? 1 : 0;
-        p.n_units = tiles * 2;
+        p.n_units = fused ? tiles : tiles * 2;
         p.timeout_ns = g_timeout_ns;
         T.n_layers = cnt;
         T.sched = sched;
         if (cudaMemsetAsync(sched, 0, sizeof(int), st) != cudaSuccess) return HCW_ERR_CUDA;
         const int total = p.n_units * cnt;
-        rc = launched(launch_tc_stack(MODE_DW, BN, T, total < sms ? total : sms, st), 1);
+        rc = launched(launch_tc_stack(fused ? MODE_DWF : MODE_DW, BN, T, total < sms ? total : sms,
+                                      st),
+                      1);
         if (rc) return rc;
     }
     return HCW_OK;

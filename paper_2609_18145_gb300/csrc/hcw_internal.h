@@ -10,7 +10,9 @@
 
 namespace hcw {
 
-enum TcMode { MODE_FWD = 0, MODE_DX = 1, MODE_DW = 2 };
+// MODE_DWF: weight gradients of a run of layers, one unit per (layer, output
+// tile) that accumulates the self and the partner part together.
+enum TcMode { MODE_FWD = 0, MODE_DX = 1, MODE_DW = 2, MODE_DWF = 3 };
 
 // Work description of one tensor-core launch (see hcw_tc.cu for the unit
 // decomposition).  Row indices are "compressed": for a fixed value beta of
@@ -56,6 +58,8 @@ struct TcLayer {
     const uint32_t* mprev;        // DX: ReLU mask words of the layer below (fused ReLU grad)
     bool dz_out;                  // DX: dz of the layer below = dx * mask is stored (map 5)
     float* colsum;                // DW, whole token range per unit: dbias = column sums of dz
+    float* dws;                   // MODE_DWF: dW_self, dW_nbr [d][d] fp32 (stored directly)
+    float* dwn;
 };
 
 // Columns of one epilogue patch (the inner extent of the 32-row residual and

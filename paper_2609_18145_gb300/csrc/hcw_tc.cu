@@ -63,6 +63,7 @@ constexpr int kBlockM = 128;
 constexpr int kBlockK = 64;                        // bf16 elements per 128-byte row
 constexpr int kABytes = kBlockM * kBlockK * 2;     // 16 KB
 constexpr int kRingBytes = 144 * 1024;             // TMA stage ring
+constexpr int kRingBytesDwf = 192 * 1024;          // MODE_DWF: no epilogue buffers
 constexpr int kEpiBufBytes = 4096;                 // one epilogue patch: 32 rows x <= 128 B
 
 // epilogue warps (a multiple of 4: one group per TMEM lane quarter), threads,
@@ -72,8 +73,12 @@ __host__ __device__ constexpr int cta_threads(int BN) { return 64 + 32 * epi_war
 __host__ __device__ constexpr int warp_cols(int BN) { return BN / (epi_warps(BN) / 4); }
 
 __host__ __device__ constexpr int stage_bytes(int BN) { return kABytes + BN * kBlockK * 2; }
-__host__ __device__ constexpr int num_stages(int BN) {
-    return (kRingBytes / stage_bytes(BN)) > 8 ? 8 : (kRingBytes / stage_bytes(BN));
+__host__ __device__ constexpr int num_stages(int BN, int MODE = MODE_FWD) {
+    // MODE_DWF takes its stages in pairs (the bit-0 and bit-1 rows of a block):
+    // an even count
+    return MODE == MODE_DWF
+               ? ((kRingBytesDwf / stage_bytes(BN)) > 8 ? 8 : (kRingBytesDwf / stage_bytes(BN))) & ~1
+               : ((kRingBytes / stage_bytes(BN)) > 8 ? 8 : (kRingBytes / stage_bytes(BN)));
 }
 
 struct __align__(8) Barriers {
@@ -91,11 +96,18 @@ struct __align__(8) Barriers {
     int q_read;           // slot reads so far (the MMA thread and every epilogue warp)
 };
 
-template <int BN>
+// epilogue patch buffers and bias slices (MODE_DWF stores from registers)
+template <int MODE, int BN>
+__host__ __device__ constexpr size_t epi_smem_bytes() {
+    return MODE == MODE_DWF ? 0
+                            : (size_t)epi_warps(BN) * kEpiBufBytes +
+                                  (size_t)epi_warps(BN) * warp_cols(BN) * 4;
+}
+
+template <int MODE, int BN>
 __host__ __device__ constexpr size_t smem_total() {
-    return 1024 /* alignment slack */ + (size_t)num_stages(BN) * stage_bytes(BN) +
-           (size_t)epi_warps(BN) * kEpiBufBytes + (size_t)epi_warps(BN) * warp_cols(BN) * 4 +
-           sizeof(Barriers);
+    return 1024 /* alignment slack */ + (size_t)num_stages(BN, MODE) * stage_bytes(BN) +
+           epi_smem_bytes<MODE, BN>() + sizeof(Barriers);
 }
 
 // FWD/DX unit -> (row bit beta, row block t, column tile j, number of K steps)
@@ -322,11 +334,13 @@ __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity,
 template <int MODE, int BN, int NL>
 __global__ void __launch_bounds__(cta_threads(BN), 1)
     hcw_tc_kernel(const __grid_constant__ TcLaunch<NL> L) {
-    constexpr int STAGES = num_stages(BN);
+    constexpr int STAGES = num_stages(BN, MODE);
+    constexpr bool DWF = MODE == MODE_DWF;
+    static_assert(!DWF || STAGES % 2 == 0, "pairs of stages");
     constexpr int SB = stage_bytes(BN);
     constexpr int B_BYTES = BN * kBlockK * 2;
     constexpr uint32_t TMEM_COLS = 2 * BN;
-    constexpr uint32_t IDESC = idesc_bf16_f32(kBlockM, BN, MODE == MODE_DW ? 1 : 0,
+    constexpr uint32_t IDESC = idesc_bf16_f32(kBlockM, BN, (MODE == MODE_DW || DWF) ? 1 : 0,
                                               MODE == MODE_FWD ? 0 : 1);
     constexpr int EW = epi_warps(BN);
     constexpr int WCOLS = warp_cols(BN);               // columns per epilogue warp
@@ -340,8 +354,8 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     uint8_t* epi_smem = smem + (size_t)STAGES * SB;               // 1024-aligned
-    float* bias_smem = reinterpret_cast<float*>(epi_smem + (size_t)EW * kEpiBufBytes);
-    Barriers* bars = reinterpret_cast<Barriers*>(bias_smem + EW * WCOLS);
+    float* bias_smem = reinterpret_cast<float*>(epi_smem + (DWF ? 0 : (size_t)EW * kEpiBufBytes));
+    Barriers* bars = reinterpret_cast<Barriers*>(bias_smem + (DWF ? 0 : EW * WCOLS));
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -353,7 +367,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
             mbar_init(&bars->full[s], 1);
             // DW: the MMA commit and the helper warps (which read the dz tiles for
             // the bias gradient) both release a stage
-            mbar_init(&bars->empty[s], MODE == MODE_DW ? 1 + kDwHelpers : 1);
+            mbar_init(&bars->empty[s], (MODE == MODE_DW || DWF) ? 1 + kDwHelpers : 1);
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&bars->tfull[a], 1);
@@ -428,7 +442,37 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                 if (MODE == MODE_DW) w = decode_w_any(p, u, STACKED, L.n_layers, l);
                 const TcLayer& ly = L.layer[l];
                 const CUtensorMap* mA = &L.maps[l][0];
-                if (MODE != MODE_DW) {
+                if (DWF) {
+                    // unit (layer, output-row tile ot, column tile nt): for every block of
+                    // 64 compressed rows, its bit-0 rows then its bit-1 rows (a pair of
+                    // stages), dz and the layer input each in one copy
+                    const int ot = ul / p.n_nt, nt = ul - ot * p.n_nt;
+                    const CUtensorMap* mX = &L.maps[l][1];
+                    st_release_cta_shared(&bars->dep_unit, ordinal);
+                    for (int pq = 0; pq < p.qb && ok; ++pq) {
+                        const int q0 = pq * 64;
+                        const int lo0 = q0 & (ly.k - 1), hi0 = q0 >> ly.s;
+                        for (int bit = 0; bit < 2; ++bit) {
+                            if (!mbar_wait(&bars->empty[stage], phase ^ 1, abort, tmo)) {
+                                ok = false;
+                                break;
+                            }
+                            uint8_t* sA = smem + (size_t)stage * SB;
+                            uint8_t* sB = sA + kABytes;
+                            mbar_arrive_expect_tx(&bars->full[stage], kABytes + B_BYTES);
+                            issued_mask |= 1u << stage;
+                            issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+                            tma_load_5d(sA, mA, &bars->full[stage], 0, lo0, bit, hi0,
+                                        ot * (kBlockM / 64));
+                            tma_load_5d(sB, mX, &bars->full[stage], 0, lo0, bit, hi0,
+                                        nt * (BN / 64));
+                            if (++stage == STAGES) {
+                                stage = 0;
+                                phase ^= 1;
+                            }
+                        }
+                    }
+                } else if (MODE != MODE_DW) {
                     const RowUnit r = decode_row_unit(p, ul, STACKED);
                     const int q0 = r.t * kBlockM;
                     const int lo0 = q0 & (ly.k - 1), hi0 = q0 >> ly.s;
@@ -534,6 +578,57 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                 }
                 if (u < 0) break;
                 const int ul = STACKED ? u % upl : u;
+                if (DWF) {
+                    // self-part accumulator at TMEM column 0, partner part at BN
+                    if (!mbar_wait(&bars->tempty[0], acc_phase ^ 1, abort, tmo)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t d_self = tmem_base, d_nbr = tmem_base + BN;
+                    for (int pq = 0; pq < p.qb && ok; ++pq) {
+                        // stage (bit-0 rows) and stage + 1 (bit-1 rows): STAGES is even
+                        if (!mbar_wait(&bars->full[stage], phase, abort, tmo) ||
+                            !mbar_wait(&bars->full[stage + 1], phase, abort, tmo)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t a0 = smem_u32(smem + (size_t)stage * SB), x0 = a0 + kABytes;
+                        const uint32_t a1 = a0 + SB, x1 = a1 + kABytes;
+                        auto dsc = [](uint32_t base, int kk) {
+                            return smem_desc_sw128(base + kk * 2048, 8192, 1024);
+                        };
+#pragma unroll
+                        for (int kk = 0; kk < kBlockK / 16; ++kk)
+                            mma_bf16_f32(d_self, dsc(a0, kk), dsc(x0, kk), IDESC, (pq | kk) != 0);
+#pragma unroll
+                        for (int kk = 0; kk < kBlockK / 16; ++kk)
+                            mma_bf16_f32(d_self, dsc(a1, kk), dsc(x1, kk), IDESC, 1);
+                        // bit-1 rows receive from their bit-0 partners (causal); both
+                        // directions without the causal rule
+#pragma unroll
+                        for (int kk = 0; kk < kBlockK / 16; ++kk)
+                            mma_bf16_f32(d_nbr, dsc(a1, kk), dsc(x0, kk), IDESC, (pq | kk) != 0);
+                        if (!p.causal) {
+#pragma unroll
+                            for (int kk = 0; kk < kBlockK / 16; ++kk)
+                                mma_bf16_f32(d_nbr, dsc(a0, kk), dsc(x1, kk), IDESC, 1);
+                        }
+                        any = true;
+                        mma_commit(&bars->empty[stage]);
+                        mma_commit(&bars->empty[stage + 1]);
+                        stage += 2;
+                        if (stage == STAGES) {
+                            stage = 0;
+                            phase ^= 1;
+                        }
+                    }
+                    if (!ok) break;
+                    mma_commit(&bars->tfull[0]);
+                    acc_phase ^= 1;
+                    continue;
+                }
                 int steps;
                 if (MODE != MODE_DW) {
                     steps = decode_row_unit(p, ul, STACKED).steps;
@@ -646,6 +741,59 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
             }
             return __shfl_sync(0xffffffffu, ok, 0) != 0;
         };
+        // Helper warps (e < kDwHelpers) of the weight-gradient modes follow the
+        // MMA thread through a unit's `steps` stages and release each one; with
+        // do_cs (a unit that covers every token of its output-row tile) they
+        // also add up the dz tile's columns on the way: dbias of rows o_base ..
+        // o_base + 127.  Thread t sums the 16-byte piece c of box t / 64 (64 dz
+        // rows each) over the tile rows r = t % 8 (mod 8), then the eight row
+        // phases are added with shuffles: a fixed order.
+        auto helper_pass = [&](int steps, bool do_cs, float* colsum, int o_base) -> bool {
+            const int t = e * 32 + lane;
+            const int box = t >> 6, c = (t >> 3) & 7, tp = t & 7;
+            float cs[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) cs[i] = 0.f;
+            for (int ks = 0; ks < steps; ++ks) {
+                if (!wait_bar(&bars->full[hstage], hphase)) return false;
+                if (do_cs) {
+                    const uint8_t* sA = smem + (size_t)hstage * SB + box * 8192;
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        const int r = tp + 8 * i;
+                        const uint4 q = *reinterpret_cast<const uint4*>(sA + r * 128 + ((c ^ tp) << 4));
+                        const uint32_t wv[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            const float2 f = unpack_bf16x2(wv[j]);
+                            cs[2 * j] += f.x;
+                            cs[2 * j + 1] += f.y;
+                        }
+                    }
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&bars->empty[hstage]);
+                if (++hstage == STAGES) {
+                    hstage = 0;
+                    hphase ^= 1;
+                }
+            }
+            if (do_cs) {
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    cs[i] += __shfl_xor_sync(0xffffffffu, cs[i], 1);
+                    cs[i] += __shfl_xor_sync(0xffffffffu, cs[i], 2);
+                    cs[i] += __shfl_xor_sync(0xffffffffu, cs[i], 4);
+                }
+                const int o0 = o_base + box * 64 + c * 8;
+                if (tp == 0 && o0 < p.d) {
+                    float4* dst = reinterpret_cast<float4*>(colsum + o0);
+                    dst[0] = make_float4(cs[0], cs[1], cs[2], cs[3]);
+                    dst[1] = make_float4(cs[4], cs[5], cs[6], cs[7]);
+                }
+            }
+            return true;
+        };
         for (; alive; ++ordinal) {
             int u = 0;
             if (lane == 0) u = consume_unit(ordinal);
@@ -660,7 +808,43 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
             WUnit wu{};
             if (MODE == MODE_DW) wu = decode_w_any(p, u, STACKED, L.n_layers, l);
             const TcLayer& ly = L.layer[l];
-            if (MODE != MODE_DW) {
+            if (DWF) {
+                const int ot = ul / p.n_nt, nt = ul - ot * p.n_nt;
+                if (e < kDwHelpers &&
+                    !helper_pass(2 * p.qb, ly.colsum != nullptr && nt == 0, ly.colsum,
+                                 ot * kBlockM)) {
+                    alive = false;
+                    break;
+                }
+                if (!wait_acc()) {
+                    alive = false;
+                    break;
+                }
+                // every lane holds one row of the tile: 32 fp32 columns per TMEM load,
+                // stored straight to global memory (no buffers in this mode); the
+                // self part, then the partner part
+                const int row = ot * kBlockM + quarter * 32 + lane;
+#pragma unroll 1
+                for (int which = 0; which < 2; ++which) {
+                    float* base = which ? ly.dwn : ly.dws;
+#pragma unroll 1
+                    for (int c = 0; c < WCOLS / 32; ++c) {
+                        uint32_t raw[32];
+                        load_acc(which * BN + c * 32, raw);
+                        if (which == 1 && c == WCOLS / 32 - 1) release_acc();
+                        if (row < p.d) {
+                            float4* dst = reinterpret_cast<float4*>(
+                                base + (size_t)row * p.d + nt * BN + cslice * WCOLS + c * 32);
+#pragma unroll
+                            for (int m = 0; m < 8; ++m)
+                                dst[m] = make_float4(__uint_as_float(raw[4 * m]),
+                                                     __uint_as_float(raw[4 * m + 1]),
+                                                     __uint_as_float(raw[4 * m + 2]),
+                                                     __uint_as_float(raw[4 * m + 3]));
+                        }
+                    }
+                }
+            } else if (MODE != MODE_DW) {
                 constexpr int RB = WCOLS * 2;                  // patch row bytes (128 or 64)
                 constexpr int SUB = WCOLS / 32;                // 32-column sub-chunks per patch
                 const RowUnit r = decode_row_unit(p, ul, STACKED);
@@ -849,65 +1033,13 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                 }
             } else {
                 const WUnit& w = wu;
-                if (e < kDwHelpers) {
-                    // Helper warps follow the MMA thread through the unit's stages and
-                    // release each one; when the unit covers every token of its
-                    // output-row tile (self part, first column tile, no split), they
-                    // also add up the dz tile's columns on the way: dbias of 128
-                    // rows.  Thread t sums the 16-byte piece c of box t / 64 (64 dz
-                    // rows each) over the tile rows r = t % 8 (mod 8), then the eight
-                    // row phases are added with shuffles: a fixed order.
-                    const int steps = w.kb1 - w.kb0;
-                    const bool do_cs = ly.colsum != nullptr && w.which == 0 && w.nt == 0 &&
-                                       p.splits_self == 1;
-                    const int t = e * 32 + lane;
-                    const int box = t >> 6, c = (t >> 3) & 7, tp = t & 7;
-                    float cs[8];
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) cs[i] = 0.f;
-                    for (int ks = 0; ks < steps; ++ks) {
-                        if (!wait_bar(&bars->full[hstage], hphase)) {
-                            alive = false;
-                            break;
-                        }
-                        if (do_cs) {
-                            const uint8_t* sA = smem + (size_t)hstage * SB + box * 8192;
-#pragma unroll
-                            for (int i = 0; i < 8; ++i) {
-                                const int r = tp + 8 * i;
-                                const uint4 q = *reinterpret_cast<const uint4*>(
-                                    sA + r * 128 + ((c ^ tp) << 4));
-                                const uint32_t wv[4] = {q.x, q.y, q.z, q.w};
-#pragma unroll
-                                for (int j = 0; j < 4; ++j) {
-                                    const float2 f = unpack_bf16x2(wv[j]);
-                                    cs[2 * j] += f.x;
-                                    cs[2 * j + 1] += f.y;
-                                }
-                            }
-                        }
-                        __syncwarp();
-                        if (lane == 0) mbar_arrive(&bars->empty[hstage]);
-                        if (++hstage == STAGES) {
-                            hstage = 0;
-                            hphase ^= 1;
-                        }
-                    }
-                    if (!alive) break;
-                    if (do_cs) {
-#pragma unroll
-                        for (int i = 0; i < 8; ++i) {
-                            cs[i] += __shfl_xor_sync(0xffffffffu, cs[i], 1);
-                            cs[i] += __shfl_xor_sync(0xffffffffu, cs[i], 2);
-                            cs[i] += __shfl_xor_sync(0xffffffffu, cs[i], 4);
-                        }
-                        const int o0 = w.ot * kBlockM + box * 64 + c * 8;
-                        if (tp == 0 && o0 < p.d) {
-                            float4* dst = reinterpret_cast<float4*>(ly.colsum + o0);
-                            dst[0] = make_float4(cs[0], cs[1], cs[2], cs[3]);
-                            dst[1] = make_float4(cs[4], cs[5], cs[6], cs[7]);
-                        }
-                    }
+                if (e < kDwHelpers &&
+                    !helper_pass(w.kb1 - w.kb0,
+                                 ly.colsum != nullptr && w.which == 0 && w.nt == 0 &&
+                                     p.splits_self == 1,
+                                 ly.colsum, w.ot * kBlockM)) {
+                    alive = false;
+                    break;
                 }
                 if (!wait_acc()) {
                     alive = false;
@@ -939,8 +1071,12 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     }
                 }
             }
-            acc ^= 1;
-            if (acc == 0) acc_phase ^= 1;
+            if (DWF) {
+                acc_phase ^= 1;   // one accumulator pair per unit
+            } else {
+                acc ^= 1;
+                if (acc == 0) acc_phase ^= 1;
+            }
         }
         // every store of this warp has landed before the CTA exits
         if (lane == 0) bulk_wait<0>();
@@ -958,7 +1094,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
 
 template <int MODE, int BN, int NL>
 static cudaError_t launch_one(const TcLaunch<NL>& L, int grid, cudaStream_t st) {
-    constexpr size_t smem = smem_total<BN>();
+    constexpr size_t smem = smem_total<MODE, BN>();
     static_assert(smem <= 232448, "shared memory budget");
     auto kern = hcw_tc_kernel<MODE, BN, NL>;
     // the shared-memory opt-in is a per-device function attribute: set it once per device
@@ -1006,12 +1142,16 @@ cudaError_t launch_tc_stack(int mode, int BN, const TcLaunch<kMaxStackLayers>& L
     HCW_TC_STACK_CASE(MODE_DW, 256)
     HCW_TC_STACK_CASE(MODE_DW, 128)
     HCW_TC_STACK_CASE(MODE_DW, 64)
+    HCW_TC_STACK_CASE(MODE_DWF, 256)
+    HCW_TC_STACK_CASE(MODE_DWF, 128)
+    HCW_TC_STACK_CASE(MODE_DWF, 64)
 #undef HCW_TC_STACK_CASE
     return cudaErrorInvalidValue;
 }
 
 size_t tc_smem_bytes(int BN) {
-    return BN == 256 ? smem_total<256>() : BN == 128 ? smem_total<128>() : smem_total<64>();
+    return BN == 256 ? smem_total<MODE_FWD, 256>()
+                     : BN == 128 ? smem_total<MODE_FWD, 128>() : smem_total<MODE_FWD, 64>();
 }
 
 int tc_stages(int BN) {

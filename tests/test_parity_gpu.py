@@ -495,9 +495,11 @@ def test_stack_backward_halves_match_the_whole(H, dtype, flags):
 
 def test_batched_weight_gradient_against_fp64_sums(H):
     """16 layers whose tiles fill the GPU: one weight-gradient launch for all of
-    them, the bias gradient summed inside it.  dW_self[l] = dz_l^T x_l and
-    dbias[l] = column sums of dz_l, recomputed in fp64 from the same bf16
-    tensors (any summation order agrees to fp32 accumulation error)."""
+    them (a unit per layer and output tile, self and partner parts together),
+    the bias gradient summed inside it.  dW_self[l] = dz_l^T x_l, dW_nbr[l] =
+    sum over receiving positions of dz_l,i x_l,i-2^s, dbias[l] = column sums
+    of dz_l, recomputed in fp64 from the same bf16 tensors (any summation
+    order agrees to fp32 accumulation error)."""
     B, n, d, L = 8, 256, 512, 16
     flags = CAUSAL | RESIDUAL | RELU
     pr = synth.problem(B, n, d, L=L, seed=33, w_std=(1 / (2 * d)) ** 0.5)
@@ -512,10 +514,17 @@ def test_batched_weight_gradient_against_fp64_sums(H):
     torch.cuda.synchronize()
     assert H.hcw_sync_status() == H.HCW_OK
     for l in range(L):
-        inp = (x if l == 0 else acts[l - 1]).reshape(-1, d).double()
+        inp3 = (x if l == 0 else acts[l - 1]).double()
+        inp = inp3.reshape(-1, d)
         g = dz[l].reshape(-1, d).double()
         assert rel(host(gb[l]), host(g.sum(0))) <= 1e-5, l
         assert rel(host(gWs[l]), host(g.T @ inp)) <= 1e-5, l
+        # causal partner part: positions with bit s set receive from i - 2^s
+        s = l % int(np.log2(n))
+        recv = torch.tensor([i for i in range(n) if (i >> s) & 1], device="cuda")
+        gr = dz[l][:, recv].reshape(-1, d).double()
+        xp = inp3[:, recv - (1 << s)].reshape(-1, d)
+        assert rel(host(gWn[l]), host(gr.T @ xp)) <= 1e-5, l
 
 
 def test_launch_counter_counts_kernels(H):
