@@ -708,8 +708,17 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
         // One unit per (layer, output tile) accumulating the self and the partner
         // part together reads each dz and input block once (the separate parts
         // read the receiving rows twice and leave a long tail of short units);
-        // used when those units alone fill most of the GPU.
+        // used when those units alone fill most of the GPU.  On pairs of SMs
+        // (256-row tiles, cta_group::2) each SM takes in a third less per stage.
         const bool fused = 5 * cnt * tiles >= 3 * sms;
+        const bool paired = fused && BN >= 128 && w1.n_ot % 2 == 0;
+        if (paired)
+            for (int i = 0; i < cnt; ++i) {
+                const int l = l0 + i;
+                const int k = 1 << stack_layer_dim(sh, a.layer0, a.dim_override, l);
+                if (!map_rows_blocks(&T.maps[i][1], act(l), sh.tokens, d, k, 64, BN / 128))
+                    return HCW_ERR_CUDA;
+            }
         TcParams& p = T.p;
         memset(&p, 0, sizeof(p));
         p.d = d;
@@ -730,9 +739,15 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
         T.sched = sched;
         if (cudaMemsetAsync(sched, 0, sizeof(int), st) != cudaSuccess) return HCW_ERR_CUDA;
         const int total = p.n_units * cnt;
-        rc = launched(launch_tc_stack(fused ? MODE_DWF : MODE_DW, BN, T, total < sms ? total : sms,
-                                      st),
-                      1);
+        if (paired) {
+            // clusters of two CTAs, one 256-row tile per cluster
+            const int pairs = total / 2 < sms / 2 ? total / 2 : sms / 2;
+            rc = launched(launch_tc_stack(MODE_DWP, BN, T, 2 * pairs, st), 1);
+        } else {
+            rc = launched(launch_tc_stack(fused ? MODE_DWF : MODE_DW, BN, T,
+                                          total < sms ? total : sms, st),
+                          1);
+        }
         if (rc) return rc;
     }
     return HCW_OK;

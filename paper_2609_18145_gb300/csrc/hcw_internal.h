@@ -12,7 +12,8 @@ namespace hcw {
 
 // MODE_DWF: weight gradients of a run of layers, one unit per (layer, output
 // tile) that accumulates the self and the partner part together.
-enum TcMode { MODE_FWD = 0, MODE_DX = 1, MODE_DW = 2, MODE_DWF = 3 };
+// MODE_DWP: the same on pairs of SMs (cta_group::2, 256-row tiles, BN >= 128).
+enum TcMode { MODE_FWD = 0, MODE_DX = 1, MODE_DW = 2, MODE_DWF = 3, MODE_DWP = 4 };
 
 // Work description of one tensor-core launch (see hcw_tc.cu for the unit
 // decomposition).  Row indices are "compressed": for a fixed value beta of

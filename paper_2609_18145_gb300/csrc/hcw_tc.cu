@@ -277,6 +277,39 @@ __device__ __forceinline__ bool wait_counter(const int* ctr, int target, volatil
     }
 }
 
+__device__ __forceinline__ int ld_relaxed_gpu(const int* p) {
+    int v;
+    asm volatile("ld.relaxed.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// Adds v to *p with release semantics: every write this thread made visible
+// before it (here: TMA stores that have completed, after a proxy fence) is
+// seen by whoever acquires the new value.
+__device__ __forceinline__ void red_release_gpu_add(int* p, int v) {
+    asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ void fence_acq_rel_gpu() {
+    asm volatile("fence.acq_rel.gpu;" ::: "memory");
+}
+
+// Bounded wait until both counters reach their targets (n of them: 1 or 2),
+// with acquire semantics.  The first look reads both at once (relaxed) and,
+// when both are complete, acquires with one fence; otherwise each is waited
+// for in turn like wait_counter.
+__device__ __forceinline__ bool wait_counters2(const int* c0, int t0, const int* c1, int t1, int n,
+                                               volatile int* abort, uint64_t timeout_ns) {
+    const int v0 = ld_relaxed_gpu(c0);
+    const int v1 = n > 1 ? ld_relaxed_gpu(c1) : t1;
+    if (v0 >= t0 && v1 >= t1) {
+        fence_acq_rel_gpu();
+        return true;
+    }
+    return wait_counter(c0, t0, abort, timeout_ns) &&
+           (n < 2 || wait_counter(c1, t1, abort, timeout_ns));
+}
+
 // Bounded wait until the shared counter *p >= target (acquire); records a
 // timeout like mbar_wait.
 __device__ __forceinline__ bool wait_shared_geq(const int* p, int target, volatile int* abort,
@@ -481,11 +514,13 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                         int cs[2];
                         row_unit_chunks(q0, ly.s, ly.k, cs[0], cs[1]);
                         const int* ctr = L.counters + (size_t)(l - 1) * L.n_chunks;
-                        for (int i = 0; i < 2 && ok; ++i) {
-                            if (cs[i] >= L.n_chunks) continue;
-                            const int rows = min(128, L.tokens - (cs[i] << 7));
-                            ok = wait_counter(ctr + cs[i], rows * p.d, abort, tmo);
-                        }
+                        // chunks past the end (ragged tail) have nothing to wait for
+                        const int nc = (cs[0] < L.n_chunks) + (cs[1] < L.n_chunks);
+                        if (cs[0] >= L.n_chunks) cs[0] = cs[1];
+                        if (nc > 0)
+                            ok = wait_counters2(
+                                ctr + cs[0], min(128, L.tokens - (cs[0] << 7)) * p.d, ctr + cs[1],
+                                min(128, L.tokens - (cs[1] << 7)) * p.d, nc, abort, tmo);
                         if (!ok) break;
                         fence_proxy_async_global();
                     }
@@ -1023,11 +1058,11 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     if (lane == 0 && inside) {
                         bulk_wait<0>();
                         fence_proxy_async_global();
-                        __threadfence();
                         const int rows = min(32, p.Mh - qw);
                         const int tok0 = ((qw >> ly.s) << (ly.s + 1)) + (r.beta << ly.s) +
                                          (qw & (ly.k - 1));
-                        atomicAdd(L.counters + (size_t)l * L.n_chunks + (tok0 >> 7), rows * WCOLS);
+                        red_release_gpu_add(L.counters + (size_t)l * L.n_chunks + (tok0 >> 7),
+                                            rows * WCOLS);
                     }
                     __syncwarp();
                 }
@@ -1092,6 +1127,351 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
     }
 }
 
+// ---------------------------------------------------------------- CTA pairs
+// Weight gradients of a run of layers on pairs of SMs (MODE_DWP): a cluster of
+// two CTAs computes a 256 x BN tile of dW_self and of dW_nbr with
+// tcgen05.mma.cta_group::2.  CTA r of the pair holds the dz rows of output
+// tile 2 * tp + r (its half of A, M = 128 of 256) and input columns r * BN/2
+// .. (r+1) * BN/2 - 1 of the column tile (its half of B); the leader (rank 0)
+// issues the MMAs, and each CTA's TMEM receives its 128 rows of both
+// accumulators.  Per 64-token stage an SM now takes in 32 KB instead of 48 KB
+// for the same MMA work.  Token blocks go in pairs of stages (bit-0 rows, then
+// bit-1 rows) as in MODE_DWF.
+//
+// Synchronisation.  Both CTAs' copies of a stage complete on the leader's
+// full barrier (the leader expects the pair's bytes).  The leader's commits
+// arrive, in both CTAs, on `consumed` (a stage's MMAs are done) and `tfull`
+// (a tile is done).  Four helper warps per CTA wait for `consumed`, add up
+// their dz tile's columns (dbias) and release the stage on their own CTA's
+// `empty`; every epilogue warp of both CTAs releases the accumulators on the
+// leader's `tempty`.  Every wait is bounded; an aborting CTA still reaches the
+// final cluster barrier, which both CTAs need to free the pair's TMEM.
+struct __align__(8) PairBarriers {
+    uint64_t full[8];
+    uint64_t consumed[8];
+    uint64_t empty[8];
+    uint64_t tfull;
+    uint64_t tempty;
+    uint64_t drain;
+    uint32_t tmem_base;
+    int abort;
+};
+
+template <int BN>
+__host__ __device__ constexpr int pair_stage_bytes() { return kABytes + (BN / 2) * kBlockK * 2; }
+template <int BN>
+__host__ __device__ constexpr int pair_stages() {
+    return ((kRingBytesDwf / pair_stage_bytes<BN>()) > 8 ? 8
+                                                         : (kRingBytesDwf / pair_stage_bytes<BN>())) &
+           ~1;
+}
+template <int BN>
+__host__ __device__ constexpr size_t pair_smem_total() {
+    return 1024 + (size_t)pair_stages<BN>() * pair_stage_bytes<BN>() + sizeof(PairBarriers);
+}
+
+template <int BN>
+__global__ void __launch_bounds__(cta_threads(BN), 1)
+    hcw_dwp_kernel(const __grid_constant__ TcLaunch<kMaxStackLayers> L) {
+    constexpr int STAGES = pair_stages<BN>();
+    constexpr int SB = pair_stage_bytes<BN>();
+    constexpr int NH = BN / 2;                          // B columns per CTA
+    constexpr uint32_t TMEM_COLS = 2 * BN;              // self and partner accumulators
+    constexpr uint32_t IDESC = idesc_bf16_f32(2 * kBlockM, BN, 1, 1);
+    constexpr int EW = epi_warps(BN);
+    constexpr int WCOLS = warp_cols(BN);
+    static_assert(STAGES % 2 == 0 && STAGES >= 2, "pairs of stages");
+    const TcParams& p = L.p;
+    const uint32_t rank = cluster_ctarank();
+    const int pair = (int)blockIdx.x >> 1, n_pairs = (int)gridDim.x >> 1;
+    const int tpl = p.n_ot / 2;                         // 256-row tiles per layer
+    const int upl = tpl * p.n_nt;
+    const int n_units = upl * L.n_layers;
+
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>(
+        (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    PairBarriers* bars = reinterpret_cast<PairBarriers*>(smem + (size_t)STAGES * SB);
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int l = 0; l < L.n_layers; ++l) {
+            tma_prefetch_desc(&L.maps[l][0]);
+            tma_prefetch_desc(&L.maps[l][1]);
+        }
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(&bars->full[s], 1);
+            mbar_init(&bars->consumed[s], 1);
+            mbar_init(&bars->empty[s], kDwHelpers);
+        }
+        mbar_init(&bars->tfull, 1);
+        mbar_init(&bars->tempty, 2 * EW);
+        mbar_init(&bars->drain, 1);
+        bars->abort = 0;
+        fence_mbar_init();
+    }
+    if (warp == 1) {
+        tmem_alloc_pair(&bars->tmem_base, TMEM_COLS);
+        tmem_relinquish_pair();
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync_all();   // both CTAs' barriers exist before any cross-CTA arrive
+    tc_fence_after();
+    const uint32_t tmem_base = bars->tmem_base;
+    volatile int* abort = &bars->abort;
+    const uint64_t tmo = p.timeout_ns;
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer (both CTAs)
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            uint32_t issued_mask = 0, issued_phase = 0;
+            bool ok = true;
+            for (int u = pair; u < n_units && ok; u += n_pairs) {
+                const int l = u / upl, ul = u - l * upl;
+                const int tp = ul / p.n_nt, nt = ul - tp * p.n_nt;
+                const TcLayer& ly = L.layer[l];
+                for (int pq = 0; pq < p.qb && ok; ++pq) {
+                    const int q0 = pq * 64;
+                    const int lo0 = q0 & (ly.k - 1), hi0 = q0 >> ly.s;
+                    for (int bit = 0; bit < 2; ++bit) {
+                        if (!mbar_wait(&bars->empty[stage], phase ^ 1, abort, tmo)) {
+                            ok = false;
+                            break;
+                        }
+                        uint8_t* sA = smem + (size_t)stage * SB;
+                        if (rank == 0) mbar_arrive_expect_tx(&bars->full[stage], 2 * SB);
+                        issued_mask |= 1u << stage;
+                        issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+                        const uint32_t fb = mapa_shared(&bars->full[stage], 0);
+                        tma_load_5d_pair(sA, &L.maps[l][0], fb, 0, lo0, bit, hi0,
+                                         (2 * tp + (int)rank) * (kBlockM / 64));
+                        tma_load_5d_pair(sA + kABytes, &L.maps[l][1], fb, 0, lo0, bit, hi0,
+                                         nt * (BN / 64) + (int)rank * (NH / 64));
+                        if (++stage == STAGES) {
+                            stage = 0;
+                            phase ^= 1;
+                        }
+                    }
+                }
+            }
+            if (!ok && rank == 0) {
+                // every copy of the pair completes on the leader's barriers: let them land
+                for (int s = 0; s < STAGES; ++s)
+                    if (issued_mask & (1u << s))
+                        mbar_wait_drain(&bars->full[s], (issued_phase >> s) & 1u, tmo);
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer (leader)
+        if (lane == 0 && rank == 0) {
+            int stage = 0;
+            uint32_t phase = 0, acc_phase = 0;
+            bool ok = true, any = false;
+            for (int u = pair; u < n_units && ok; u += n_pairs) {
+                if (!mbar_wait(&bars->tempty, acc_phase ^ 1, abort, tmo)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d_self = tmem_base, d_nbr = tmem_base + BN;
+                for (int pq = 0; pq < p.qb && ok; ++pq) {
+                    if (!mbar_wait(&bars->full[stage], phase, abort, tmo) ||
+                        !mbar_wait(&bars->full[stage + 1], phase, abort, tmo)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a0 = smem_u32(smem + (size_t)stage * SB), x0 = a0 + kABytes;
+                    const uint32_t a1 = a0 + SB, x1 = a1 + kABytes;
+                    auto dsc = [](uint32_t base, int kk) {
+                        return smem_desc_sw128(base + kk * 2048, 8192, 1024);
+                    };
+#pragma unroll
+                    for (int kk = 0; kk < kBlockK / 16; ++kk)
+                        mma_bf16_f32_pair(d_self, dsc(a0, kk), dsc(x0, kk), IDESC, (pq | kk) != 0);
+#pragma unroll
+                    for (int kk = 0; kk < kBlockK / 16; ++kk)
+                        mma_bf16_f32_pair(d_self, dsc(a1, kk), dsc(x1, kk), IDESC, 1);
+#pragma unroll
+                    for (int kk = 0; kk < kBlockK / 16; ++kk)
+                        mma_bf16_f32_pair(d_nbr, dsc(a1, kk), dsc(x0, kk), IDESC, (pq | kk) != 0);
+                    if (!p.causal) {
+#pragma unroll
+                        for (int kk = 0; kk < kBlockK / 16; ++kk)
+                            mma_bf16_f32_pair(d_nbr, dsc(a0, kk), dsc(x1, kk), IDESC, 1);
+                    }
+                    any = true;
+                    mma_commit_pair(&bars->consumed[stage], 3);
+                    mma_commit_pair(&bars->consumed[stage + 1], 3);
+                    stage += 2;
+                    if (stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1;
+                    }
+                }
+                if (!ok) break;
+                mma_commit_pair(&bars->tfull, 3);
+                acc_phase ^= 1;
+            }
+            if (any) {
+                // the pair's MMAs have completed before TMEM can be freed
+                mma_commit_pair(&bars->drain, 1);
+                mbar_wait_drain(&bars->drain, 0, tmo);
+            }
+        }
+    } else {
+        // ------------------------------------------------------------ epilogue (both CTAs)
+        const int e = warp - 2;
+        const int quarter = warp & 3;
+        const int cslice = e >> 2;
+        const uint32_t tempty_leader = mapa_shared(&bars->tempty, 0);
+        int hstage = 0;
+        uint32_t hphase = 0, acc_phase = 0;
+        bool alive = true;
+        for (int u = pair; u < n_units && alive; u += n_pairs) {
+            const int l = u / upl, ul = u - l * upl;
+            const int tp = ul / p.n_nt, nt = ul - tp * p.n_nt;
+            const int ot = 2 * tp + (int)rank;
+            const TcLayer& ly = L.layer[l];
+            if (e < kDwHelpers) {
+                // release this CTA's stages once the pair's MMAs have read them, and
+                // sum the dz tile's columns on the way (dbias, output rows of tile ot)
+                const bool do_cs = ly.colsum != nullptr && nt == 0;
+                const int t = e * 32 + lane;
+                const int box = t >> 6, c = (t >> 3) & 7, tph = t & 7;
+                float cs[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) cs[i] = 0.f;
+                for (int ks = 0; ks < 2 * p.qb; ++ks) {
+                    const bool okw = mbar_wait(&bars->consumed[hstage], hphase, abort, tmo);
+                    if (!__all_sync(0xffffffffu, okw)) {
+                        alive = false;
+                        break;
+                    }
+                    if (do_cs) {
+                        const uint8_t* sA = smem + (size_t)hstage * SB + box * 8192;
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const int r = tph + 8 * i;
+                            const uint4 q =
+                                *reinterpret_cast<const uint4*>(sA + r * 128 + ((c ^ tph) << 4));
+                            const uint32_t wv[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+                            for (int j = 0; j < 4; ++j) {
+                                const float2 f = unpack_bf16x2(wv[j]);
+                                cs[2 * j] += f.x;
+                                cs[2 * j + 1] += f.y;
+                            }
+                        }
+                    }
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&bars->empty[hstage]);
+                    if (++hstage == STAGES) {
+                        hstage = 0;
+                        hphase ^= 1;
+                    }
+                }
+                if (!alive) break;
+                if (do_cs) {
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) {
+                        cs[i] += __shfl_xor_sync(0xffffffffu, cs[i], 1);
+                        cs[i] += __shfl_xor_sync(0xffffffffu, cs[i], 2);
+                        cs[i] += __shfl_xor_sync(0xffffffffu, cs[i], 4);
+                    }
+                    const int o0 = ot * kBlockM + box * 64 + c * 8;
+                    if (tph == 0 && o0 < p.d) {
+                        float4* dst = reinterpret_cast<float4*>(ly.colsum + o0);
+                        dst[0] = make_float4(cs[0], cs[1], cs[2], cs[3]);
+                        dst[1] = make_float4(cs[4], cs[5], cs[6], cs[7]);
+                    }
+                }
+            }
+            const bool okt = mbar_wait(&bars->tfull, acc_phase, abort, tmo);
+            if (!__all_sync(0xffffffffu, okt)) {
+                alive = false;
+                break;
+            }
+            tc_fence_after();
+            // this CTA's 128 rows of the tile: one row per lane, 32 fp32 columns per load
+            const int row = ot * kBlockM + quarter * 32 + lane;
+#pragma unroll 1
+            for (int which = 0; which < 2; ++which) {
+                float* base = which ? ly.dwn : ly.dws;
+#pragma unroll 1
+                for (int c = 0; c < WCOLS / 32; ++c) {
+                    uint32_t raw[32];
+                    __syncwarp();
+                    tmem_ld_32x32b_x32(tmem_base + ((uint32_t)(quarter * 32) << 16) +
+                                           (uint32_t)(which * BN + cslice * WCOLS + c * 32),
+                                       raw);
+                    tmem_ld_wait_regs(raw);
+                    if (which == 1 && c == WCOLS / 32 - 1) {
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive_remote(tempty_leader);
+                    }
+                    if (row < p.d) {
+                        float4* dst = reinterpret_cast<float4*>(
+                            base + (size_t)row * p.d + nt * BN + cslice * WCOLS + c * 32);
+#pragma unroll
+                        for (int m = 0; m < 8; ++m)
+                            dst[m] = make_float4(__uint_as_float(raw[4 * m]),
+                                                 __uint_as_float(raw[4 * m + 1]),
+                                                 __uint_as_float(raw[4 * m + 2]),
+                                                 __uint_as_float(raw[4 * m + 3]));
+                    }
+                }
+            }
+            acc_phase ^= 1;
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync_all();   // neither CTA frees the pair's TMEM while the other uses it
+    if (warp == 1) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc_pair(tmem_base, TMEM_COLS);
+    }
+}
+
+template <int BN>
+static cudaError_t launch_pair(const TcLaunch<kMaxStackLayers>& L, int grid, cudaStream_t st) {
+    constexpr size_t smem = pair_smem_total<BN>();
+    static_assert(smem <= 232448, "shared memory budget");
+    auto kern = hcw_dwp_kernel<BN>;
+    static std::atomic<uint64_t> configured[4] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const uint64_t bit = 1ull << (dev & 63);
+    std::atomic<uint64_t>& word = configured[(dev >> 6) & 3];
+    if (dev >= 256 || !(word.load(std::memory_order_acquire) & bit)) {
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        if (dev < 256) word.fetch_or(bit, std::memory_order_acq_rel);
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3((unsigned)cta_threads(BN));
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, L);
+}
+
 template <int MODE, int BN, int NL>
 static cudaError_t launch_one(const TcLaunch<NL>& L, int grid, cudaStream_t st) {
     constexpr size_t smem = smem_total<MODE, BN>();
@@ -1131,6 +1511,11 @@ cudaError_t launch_tc(int mode, int BN, const TcLaunch<1>& L, int grid, cudaStre
 
 cudaError_t launch_tc_stack(int mode, int BN, const TcLaunch<kMaxStackLayers>& L, int grid,
                             cudaStream_t st) {
+    if (mode == MODE_DWP) {
+        if (BN == 256) return launch_pair<256>(L, grid, st);
+        if (BN == 128) return launch_pair<128>(L, grid, st);
+        return cudaErrorInvalidValue;
+    }
 #define HCW_TC_STACK_CASE(M, N) \
     if (mode == M && BN == N) return launch_one<M, N, kMaxStackLayers>(L, grid, st);
     HCW_TC_STACK_CASE(MODE_FWD, 256)
