@@ -292,12 +292,15 @@ void row_unit_params(TcParams& p, const Shape& sh, int BN, unsigned flags, bool 
 
 // The five forward maps of one layer: x rows (128-row boxes), W_self, W_nbr,
 // x rows (32-row residual patches), y rows (32-row output patches).
+// pair: the weight boxes hold half a column tile (each CTA of a pair loads
+// its half of B)
 bool fwd_maps(CUtensorMap* m, const Shape& sh, int s, const void* x, const void* Ws,
-              const void* Wn, const void* y) {
+              const void* Wn, const void* y, bool pair = false) {
     const int d = sh.d, BN = pick_bn(d), k = 1 << s;
     const int pw = epi_patch_cols(BN);
-    if (!map_rows(&m[0], x, sh.tokens, d, k, 128) || !map_weight(&m[1], Ws, d, BN) ||
-        !map_weight(&m[2], Wn, d, BN) || !map_rows(&m[3], x, sh.tokens, d, k, 32, pw) ||
+    const int box_o = pair ? BN / 2 : BN;
+    if (!map_rows(&m[0], x, sh.tokens, d, k, 128) || !map_weight(&m[1], Ws, d, box_o) ||
+        !map_weight(&m[2], Wn, d, box_o) || !map_rows(&m[3], x, sh.tokens, d, k, 32, pw) ||
         !map_rows(&m[4], y, sh.tokens, d, k, 32, pw))
         return false;
     m[5] = m[4];   // unused by the forward
@@ -327,6 +330,29 @@ size_t stack_counter_bytes(long long tokens, int L) {
     return align256((size_t)layers * (size_t)((tokens + 127) / 128) * sizeof(int) + 16);
 }
 
+// Whether a stacked forward / input-gradient launch runs on pairs of SMs
+// (tcgen05 cta_group::2, 256-row tiles): 256-column tiles and at least two
+// row blocks.  Each SM of a pair loads its own rows and half of the weight
+// tile per stage.
+bool use_pairs(const Shape& sh) {
+    return pick_bn(sh.d) == 256 && sh.tokens / 2 > 128;
+}
+
+// Row-unit geometry of a pair launch: units count row-block pairs.
+void pair_units(TcParams& p) { p.n_units = ((p.n_rb + 1) / 2) * p.n_nt * 2; }
+
+// Launch a stacked forward / input-gradient run, on pairs of SMs if `pair`.
+int launch_rows(int mode, int BN, TcLaunch<kMaxStackLayers>& T, int n, bool pair,
+                cudaStream_t st) {
+    const int sms = sm_count();
+    const int total = T.p.n_units * n;
+    if (pair) {
+        const int pairs = total < sms / 2 ? total : sms / 2;
+        return launched(launch_tc_stack_pair(mode, BN, T, 2 * pairs, st), 1);
+    }
+    return launched(launch_tc_stack(mode, BN, T, total < sms ? total : sms, st), 1);
+}
+
 // Layers [l0, l0 + n) of a bf16 stack in one persistent launch.  in_ptr(l),
 // out_ptr(l), mask_ptr(l) give each layer's input, output and mask.
 template <class In, class Out, class Mask>
@@ -335,17 +361,19 @@ int stack_fwd_group(const Shape& sh, int l0, int n, int layer0, int dim_override
                     In in_ptr, Out out_ptr, Mask mask_ptr, int* counters, cudaStream_t st) {
     const int d = sh.d, BN = pick_bn(d);
     const size_t wb = (size_t)d * d * 2;
+    const bool pair = use_pairs(sh);
     static thread_local TcLaunch<kMaxStackLayers> L;
     memset(&L, 0, sizeof(L));
     for (int i = 0; i < n; ++i) {
         const int l = l0 + i;
         const int s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
-        if (!fwd_maps(L.maps[i], sh, s, in_ptr(l), Ws + l * wb, Wn + l * wb, out_ptr(l)))
+        if (!fwd_maps(L.maps[i], sh, s, in_ptr(l), Ws + l * wb, Wn + l * wb, out_ptr(l), pair))
             return HCW_ERR_CUDA;
         L.layer[i] = {s, 1 << s, bias ? bias + (size_t)l * d : nullptr, mask_ptr(l), nullptr,
                       true, nullptr, false};
     }
     row_unit_params(L.p, sh, BN, flags, false);
+    if (pair) pair_units(L.p);
     L.p.flags = flags;
     L.n_layers = n;
     L.counters = counters;
@@ -354,10 +382,7 @@ int stack_fwd_group(const Shape& sh, int l0, int n, int layer0, int dim_override
     L.sched = counters + (size_t)n * L.n_chunks;
     cudaError_t e = cudaMemsetAsync(counters, 0, ((size_t)n * L.n_chunks + 1) * sizeof(int), st);
     if (e != cudaSuccess) return HCW_ERR_CUDA;
-    const int sms = sm_count();
-    const int total = L.p.n_units * n;
-    const int grid = total < sms ? total : sms;
-    return launched(launch_tc_stack(MODE_FWD, BN, L, grid, st), 1);
+    return launch_rows(MODE_FWD, BN, L, n, pair, st);
 }
 
 // dx: a row gathers dz from its partner exactly when the partner received from it
@@ -614,6 +639,7 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
     if (rc) return rc;
     int* counters = reinterpret_cast<int*>(a.ws + (keep_g ? (size_t)L * a256 : 0));
     const int n_chunks = (int)((sh.tokens + 127) / 128);
+    const bool pair = use_pairs(sh);
     const int pw = epi_patch_cols(BN);
     static thread_local TcLaunch<kMaxStackLayers> T;
     for (int top = L - 1; top >= 0; top -= kMaxStackLayers) {
@@ -629,8 +655,8 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
             CUtensorMap* m = T.maps[i];
             const void* res = resid ? g(l) : dz(l);
             if (!map_rows(&m[0], dz(l), sh.tokens, d, k, 128) ||
-                !map_weight_blocks(&m[1], a.Ws + l * wb, d, BN / 64) ||
-                !map_weight_blocks(&m[2], a.Wn + l * wb, d, BN / 64) ||
+                !map_weight_blocks(&m[1], a.Ws + l * wb, d, (pair ? BN / 2 : BN) / 64) ||
+                !map_weight_blocks(&m[2], a.Wn + l * wb, d, (pair ? BN / 2 : BN) / 64) ||
                 !map_rows(&m[3], res, sh.tokens, d, k, 32, pw) ||
                 !map_rows(&m[4], out ? out : dzo, sh.tokens, d, k, 32, pw) ||
                 !map_rows(&m[5], dzo ? dzo : out, sh.tokens, d, k, 32, pw))
@@ -639,6 +665,7 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
                           dzo ? mask(l - 1) : nullptr, dzo != nullptr};
         }
         row_unit_params(T.p, sh, BN, a.flags, true);
+        if (pair) pair_units(T.p);
         T.p.flags = a.flags & HCW_RESIDUAL;
         T.n_layers = cnt;
         T.counters = counters;
@@ -648,9 +675,7 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
         if (cudaMemsetAsync(counters, 0, ((size_t)cnt * n_chunks + 1) * sizeof(int), st) !=
             cudaSuccess)
             return HCW_ERR_CUDA;
-        const int sms = sm_count();
-        const int total = T.p.n_units * cnt;
-        rc = launched(launch_tc_stack(MODE_DX, BN, T, total < sms ? total : sms, st), 1);
+        rc = launch_rows(MODE_DX, BN, T, cnt, pair, st);
         if (rc) return rc;
     }
     return HCW_OK;

@@ -92,6 +92,10 @@ cudaError_t launch_tc(int mode, int BN, const TcLaunch<1>& L, int grid, cudaStre
 // layers, the long self-part units of every layer first).
 cudaError_t launch_tc_stack(int mode, int BN, const TcLaunch<kMaxStackLayers>& L, int grid,
                             cudaStream_t stream);
+// The same for MODE_FWD / MODE_DX on clusters of two CTAs (256-row tiles,
+// cta_group::2; BN 256, even grid).  L.p counts pair units: row-block pairs.
+cudaError_t launch_tc_stack_pair(int mode, int BN, const TcLaunch<kMaxStackLayers>& L, int grid,
+                                 cudaStream_t stream);
 
 // Dynamic shared memory the tensor-core kernel uses for this N tile.
 size_t tc_smem_bytes(int BN);

@@ -96,6 +96,12 @@ struct __align__(8) Barriers {
     int q_read;           // slot reads so far (the MMA thread and every epilogue warp)
 };
 
+// Stages of the pair variant of the row kernels: this CTA's A and half of B.
+__host__ __device__ constexpr int pair_row_stage_bytes(int BN) { return kABytes + BN * kBlockK; }
+__host__ __device__ constexpr int tc_pair_stages(int BN) {
+    return (kRingBytes / pair_row_stage_bytes(BN)) > 8 ? 8 : (kRingBytes / pair_row_stage_bytes(BN));
+}
+
 // epilogue patch buffers and bias slices (MODE_DWF stores from registers)
 template <int MODE, int BN>
 __host__ __device__ constexpr size_t epi_smem_bytes() {
@@ -104,9 +110,11 @@ __host__ __device__ constexpr size_t epi_smem_bytes() {
                                   (size_t)epi_warps(BN) * warp_cols(BN) * 4;
 }
 
-template <int MODE, int BN>
+template <int MODE, int BN, bool PAIR = false>
 __host__ __device__ constexpr size_t smem_total() {
-    return 1024 /* alignment slack */ + (size_t)num_stages(BN, MODE) * stage_bytes(BN) +
+    return 1024 /* alignment slack */ +
+           (PAIR ? (size_t)tc_pair_stages(BN) * pair_row_stage_bytes(BN)
+                 : (size_t)num_stages(BN, MODE) * stage_bytes(BN)) +
            epi_smem_bytes<MODE, BN>() + sizeof(Barriers);
 }
 
@@ -312,12 +320,14 @@ __device__ __forceinline__ bool wait_counters2(const int* c0, int t0, const int*
 
 // Bounded wait until the shared counter *p >= target (acquire); records a
 // timeout like mbar_wait.
+template <bool CLUSTER = false>
 __device__ __forceinline__ bool wait_shared_geq(const int* p, int target, volatile int* abort,
                                                 uint64_t timeout_ns) {
-    if (ld_acquire_cta_shared(p) >= target) return true;
+    auto load = [&]() { return CLUSTER ? ld_acquire_cluster_local(p) : ld_acquire_cta_shared(p); };
+    if (load() >= target) return true;
     const uint64_t t0 = globaltimer_ns();
     for (uint32_t it = 1;; ++it) {
-        if (ld_acquire_cta_shared(p) >= target) return true;
+        if (load() >= target) return true;
         if ((it & 63u) == 0) {
             if (*abort) return false;
             if (globaltimer_ns() - t0 > timeout_ns) {
@@ -364,16 +374,22 @@ __device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity,
 // elements of a patch once its TMA stores have landed).  All earlier units
 // of the launch have smaller indices and each CTA takes its units in order,
 // so the lowest unfinished unit can always proceed.
-template <int MODE, int BN, int NL>
+template <int MODE, int BN, int NL, bool PAIR>
 __global__ void __launch_bounds__(cta_threads(BN), 1)
     hcw_tc_kernel(const __grid_constant__ TcLaunch<NL> L) {
-    constexpr int STAGES = num_stages(BN, MODE);
+    // PAIR (stacked forward / input gradient): clusters of two CTAs, 256-row
+    // tiles with tcgen05.mma.cta_group::2; each CTA loads its own 128 rows and
+    // half of the weight tile, the leader issues the MMAs (see hcw_dwp_kernel)
+    static_assert(!PAIR || ((MODE == MODE_FWD || MODE == MODE_DX) && NL > 1), "pair modes");
+    constexpr int STAGES = PAIR ? tc_pair_stages(BN) : num_stages(BN, MODE);
     constexpr bool DWF = MODE == MODE_DWF;
     static_assert(!DWF || STAGES % 2 == 0, "pairs of stages");
-    constexpr int SB = stage_bytes(BN);
     constexpr int B_BYTES = BN * kBlockK * 2;
+    constexpr int B_LOAD = PAIR ? B_BYTES / 2 : B_BYTES;    // B bytes this CTA loads per stage
+    constexpr int SB = kABytes + B_LOAD;
     constexpr uint32_t TMEM_COLS = 2 * BN;
-    constexpr uint32_t IDESC = idesc_bf16_f32(kBlockM, BN, (MODE == MODE_DW || DWF) ? 1 : 0,
+    constexpr uint32_t IDESC = idesc_bf16_f32(PAIR ? 2 * kBlockM : kBlockM, BN,
+                                              (MODE == MODE_DW || DWF) ? 1 : 0,
                                               MODE == MODE_FWD ? 0 : 1);
     constexpr int EW = epi_warps(BN);
     constexpr int WCOLS = warp_cols(BN);               // columns per epilogue warp
@@ -404,7 +420,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(&bars->tfull[a], 1);
-            mbar_init(&bars->tempty[a], EW);
+            mbar_init(&bars->tempty[a], PAIR ? 2 * EW : EW);
         }
         for (int e = 0; e < EW; ++e) mbar_init(&bars->epi_load[e], 1);
         mbar_init(&bars->drain, 1);
@@ -415,12 +431,19 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
         fence_mbar_init();
     }
     if (warp == 1) {
-        tmem_alloc(&bars->tmem_base, TMEM_COLS);
-        tmem_relinquish();
+        if (PAIR) {
+            tmem_alloc_pair(&bars->tmem_base, TMEM_COLS);
+            tmem_relinquish_pair();
+        } else {
+            tmem_alloc(&bars->tmem_base, TMEM_COLS);
+            tmem_relinquish();
+        }
     }
     tc_fence_before();
     __syncthreads();
+    if (PAIR) cluster_sync_all();   // both CTAs' barriers exist before any cross-CTA access
     tc_fence_after();
+    const uint32_t rank = PAIR ? cluster_ctarank() : 0;
     const uint32_t tmem_base = bars->tmem_base;
     volatile int* abort = &bars->abort;
     const uint64_t tmo = p.timeout_ns;
@@ -436,7 +459,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
             const int u = (int)blockIdx.x + ord * (int)gridDim.x;
             return u < n_units ? u : -1;
         }
-        if (!wait_shared_geq(&bars->q_pub, ord, abort, tmo)) return -2;
+        if (!wait_shared_geq<PAIR>(&bars->q_pub, ord, abort, tmo)) return -2;
         const int u = *reinterpret_cast<volatile int*>(&bars->unit_q[ord % kUnitQ]);
         __threadfence_block();
         atomicAdd(&bars->q_read, 1);
@@ -452,7 +475,14 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
             bool ok = true;
             for (int ordinal = 0; ok; ++ordinal) {
                 int u;
-                if (dyn) {
+                if (PAIR && rank == 1) {
+                    // the pair's units come from the leader, through this CTA's slots
+                    u = consume_unit(ordinal);
+                    if (u == -2) {
+                        ok = false;
+                        break;
+                    }
+                } else if (dyn) {
                     u = atomicAdd(L.sched, 1);
                     if (u >= n_units) u = -1;
                     // the slot's previous unit has been read by every consumer
@@ -461,6 +491,29 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                                          tmo)) {
                         ok = false;
                         break;
+                    }
+                    if (PAIR) {
+                        // ... and in the other CTA of the pair
+                        const uint32_t peer_read = mapa_shared(&bars->q_read, 1);
+                        const int need = (ordinal - kUnitQ + 1) * (EW + 1);
+                        bool okp = true;
+                        if (ordinal >= kUnitQ && ld_acquire_cluster_remote(peer_read) < need) {
+                            const uint64_t t0 = globaltimer_ns();
+                            while (ld_acquire_cluster_remote(peer_read) < need) {
+                                if (*abort || globaltimer_ns() - t0 > tmo) {
+                                    if (!*abort) atomicExch(&g_error_word, kErrTimeout);
+                                    *abort = 1;
+                                    okp = false;
+                                    break;
+                                }
+                            }
+                        }
+                        if (!okp) {
+                            ok = false;
+                            break;
+                        }
+                        st_remote(mapa_shared(&bars->unit_q[ordinal % kUnitQ], 1), u);
+                        st_release_cluster_remote(mapa_shared(&bars->q_pub, 1), ordinal);
                     }
                     bars->unit_q[ordinal % kUnitQ] = u;
                     st_release_cta_shared(&bars->q_pub, ordinal);
@@ -506,7 +559,8 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                         }
                     }
                 } else if (MODE != MODE_DW) {
-                    const RowUnit r = decode_row_unit(p, ul, STACKED);
+                    RowUnit r = decode_row_unit(p, ul, STACKED);
+                    if (PAIR) r.t = 2 * r.t + (int)rank;   // this CTA's half of the 256 rows
                     const int q0 = r.t * kBlockM;
                     const int lo0 = q0 & (ly.k - 1), hi0 = q0 >> ly.s;
                     if (STACKED && l > 0) {
@@ -532,19 +586,32 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                         }
                         uint8_t* sA = smem + (size_t)stage * SB;
                         uint8_t* sB = sA + kABytes;
-                        mbar_arrive_expect_tx(&bars->full[stage], kABytes + B_BYTES);
                         issued_mask |= 1u << stage;
                         issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
                         const int part = ks >= p.nK;
                         const int kk = part ? ks - p.nK : ks;
                         const int bitA = part ? 1 - r.beta : r.beta;
-                        tma_load_4d(sA, mA, &bars->full[stage], kk * kBlockK, lo0, bitA, hi0);
                         const CUtensorMap* mb = &L.maps[l][part ? 2 : 1];
-                        if (MODE == MODE_FWD)
-                            tma_load_2d(sB, mb, &bars->full[stage], kk * kBlockK, r.j * BN);
-                        else   // BN / 64 blocks of 64 W columns x 64 rows, one copy
-                            tma_load_3d(sB, mb, &bars->full[stage], 0, kk * kBlockK,
-                                        r.j * (BN / 64));
+                        if (PAIR) {
+                            // both CTAs' copies complete on the leader's barrier
+                            if (rank == 0) mbar_arrive_expect_tx(&bars->full[stage], 2 * SB);
+                            const uint32_t fb = mapa_shared(&bars->full[stage], 0);
+                            tma_load_4d_pair(sA, mA, fb, kk * kBlockK, lo0, bitA, hi0);
+                            if (MODE == MODE_FWD)
+                                tma_load_2d_pair(sB, mb, fb, kk * kBlockK,
+                                                 r.j * BN + (int)rank * (BN / 2));
+                            else
+                                tma_load_3d_pair(sB, mb, fb, 0, kk * kBlockK,
+                                                 r.j * (BN / 64) + (int)rank * (BN / 128));
+                        } else {
+                            mbar_arrive_expect_tx(&bars->full[stage], kABytes + B_BYTES);
+                            tma_load_4d(sA, mA, &bars->full[stage], kk * kBlockK, lo0, bitA, hi0);
+                            if (MODE == MODE_FWD)
+                                tma_load_2d(sB, mb, &bars->full[stage], kk * kBlockK, r.j * BN);
+                            else   // BN / 64 blocks of 64 W columns x 64 rows, one copy
+                                tma_load_3d(sB, mb, &bars->full[stage], 0, kk * kBlockK,
+                                            r.j * (BN / 64));
+                        }
                         if (++stage == STAGES) {
                             stage = 0;
                             phase ^= 1;
@@ -590,8 +657,9 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     }
                 }
             }
-            if (!ok) {
-                // let every copy this thread started land before the CTA exits
+            if (!ok && (!PAIR || rank == 0)) {
+                // let every copy this thread started land before the CTA exits (a
+                // pair's copies all complete on the leader's barriers)
                 for (int s = 0; s < STAGES; ++s)
                     if (issued_mask & (1u << s))
                         mbar_wait_drain(&bars->full[s], (issued_phase >> s) & 1u, tmo);
@@ -599,7 +667,8 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
+        // (a pair's MMAs are issued by its leader alone)
+        if (lane == 0 && (!PAIR || rank == 0)) {
             int stage = 0;
             uint32_t phase = 0;
             int acc = 0;
@@ -697,23 +766,35 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                             bdesc = smem_desc_sw128(b_addr + kk * 32, 16, 1024);
                         else
                             bdesc = smem_desc_sw128(b_addr + kk * 2048, 8192, 1024);
-                        mma_bf16_f32(d_tmem, adesc, bdesc, IDESC, (ks | kk) != 0);
+                        if (PAIR)
+                            mma_bf16_f32_pair(d_tmem, adesc, bdesc, IDESC, (ks | kk) != 0);
+                        else
+                            mma_bf16_f32(d_tmem, adesc, bdesc, IDESC, (ks | kk) != 0);
                     }
                     any = true;
-                    mma_commit(&bars->empty[stage]);
+                    if (PAIR)
+                        mma_commit_pair(&bars->empty[stage], 3);   // both CTAs' stage
+                    else
+                        mma_commit(&bars->empty[stage]);
                     if (++stage == STAGES) {
                         stage = 0;
                         phase ^= 1;
                     }
                 }
                 if (!ok) break;
-                mma_commit(&bars->tfull[acc]);
+                if (PAIR)
+                    mma_commit_pair(&bars->tfull[acc], 3);
+                else
+                    mma_commit(&bars->tfull[acc]);
                 acc ^= 1;
                 if (acc == 0) acc_phase ^= 1;
             }
             if (!ok && any) {
                 // wait for the MMAs already issued before TMEM is released
-                mma_commit(&bars->drain);
+                if (PAIR)
+                    mma_commit_pair(&bars->drain, 1);
+                else
+                    mma_commit(&bars->drain);
                 mbar_wait_drain(&bars->drain, 0, tmo);
             }
         }
@@ -754,7 +835,12 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
         auto release_acc = [&]() {
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&bars->tempty[acc]);
+            if (lane == 0) {
+                if (PAIR)
+                    mbar_arrive_remote(mapa_shared(&bars->tempty[acc], 0));   // the leader's
+                else
+                    mbar_arrive(&bars->tempty[acc]);
+            }
         };
         // make this warp's shared-memory writes visible to TMA, then store
         auto publish = [&]() {
@@ -882,7 +968,8 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
             } else if (MODE != MODE_DW) {
                 constexpr int RB = WCOLS * 2;                  // patch row bytes (128 or 64)
                 constexpr int SUB = WCOLS / 32;                // 32-column sub-chunks per patch
-                const RowUnit r = decode_row_unit(p, ul, STACKED);
+                RowUnit r = decode_row_unit(p, ul, STACKED);
+                if (PAIR) r.t = 2 * r.t + (int)rank;
                 const int qw = r.t * kBlockM + quarter * 32;   // first compressed row of the warp
                 const int lo_w = qw & (ly.k - 1), hi_w = qw >> ly.s;
                 const int q_row = qw + lane;
@@ -1120,10 +1207,14 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
 
     tc_fence_before();
     __syncthreads();
+    if (PAIR) cluster_sync_all();   // neither CTA frees the pair's TMEM while the other uses it
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
-        tmem_dealloc(tmem_base, TMEM_COLS);
+        if (PAIR)
+            tmem_dealloc_pair(tmem_base, TMEM_COLS);
+        else
+            tmem_dealloc(tmem_base, TMEM_COLS);
     }
 }
 
@@ -1472,11 +1563,11 @@ static cudaError_t launch_pair(const TcLaunch<kMaxStackLayers>& L, int grid, cud
     return cudaLaunchKernelEx(&cfg, kern, L);
 }
 
-template <int MODE, int BN, int NL>
+template <int MODE, int BN, int NL, bool PAIR = false>
 static cudaError_t launch_one(const TcLaunch<NL>& L, int grid, cudaStream_t st) {
-    constexpr size_t smem = smem_total<MODE, BN>();
+    constexpr size_t smem = smem_total<MODE, BN, PAIR>();
     static_assert(smem <= 232448, "shared memory budget");
-    auto kern = hcw_tc_kernel<MODE, BN, NL>;
+    auto kern = hcw_tc_kernel<MODE, BN, NL, PAIR>;
     // the shared-memory opt-in is a per-device function attribute: set it once per device
     static std::atomic<uint64_t> configured[4] = {};
     int dev = 0;
@@ -1489,8 +1580,24 @@ static cudaError_t launch_one(const TcLaunch<NL>& L, int grid, cudaStream_t st) 
         if (e != cudaSuccess) return e;
         if (dev < 256) word.fetch_or(bit, std::memory_order_acq_rel);
     }
-    kern<<<grid, cta_threads(BN), smem, st>>>(L);
-    return cudaGetLastError();
+    if (!PAIR) {
+        kern<<<grid, cta_threads(BN), smem, st>>>(L);
+        return cudaGetLastError();
+    }
+    // clusters of two CTAs (the grid is even)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3((unsigned)cta_threads(BN));
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, L);
 }
 
 cudaError_t launch_tc(int mode, int BN, const TcLaunch<1>& L, int grid, cudaStream_t st) {
@@ -1531,6 +1638,14 @@ cudaError_t launch_tc_stack(int mode, int BN, const TcLaunch<kMaxStackLayers>& L
     HCW_TC_STACK_CASE(MODE_DWF, 128)
     HCW_TC_STACK_CASE(MODE_DWF, 64)
 #undef HCW_TC_STACK_CASE
+    return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_tc_stack_pair(int mode, int BN, const TcLaunch<kMaxStackLayers>& L, int grid,
+                                 cudaStream_t st) {
+    if (BN != 256 || grid % 2) return cudaErrorInvalidValue;
+    if (mode == MODE_FWD) return launch_one<MODE_FWD, 256, kMaxStackLayers, true>(L, grid, st);
+    if (mode == MODE_DX) return launch_one<MODE_DX, 256, kMaxStackLayers, true>(L, grid, st);
     return cudaErrorInvalidValue;
 }
 

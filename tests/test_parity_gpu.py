@@ -231,6 +231,12 @@ STACK_CASES = [
      (1 / 256) ** 0.5),
     ("n256_d512_bf16_causal_res_relu", torch.bfloat16, 2, 256, 512, 16,
      CAUSAL | RESIDUAL | RELU, (1 / 1024) ** 0.5),
+    # 256-column tiles on pairs of SMs with an odd number of 128-row blocks (the
+    # last pair's second CTA has no rows)
+    ("n64_d256_bf16_odd_row_blocks", torch.bfloat16, 10, 64, 256, 6,
+     CAUSAL | RESIDUAL | RELU, (1 / 512) ** 0.5),
+    ("n64_d256_bf16_odd_row_blocks_noncausal", torch.bfloat16, 10, 64, 256, 6,
+     RESIDUAL, (1 / 512) ** 0.5),
 ]
 
 
