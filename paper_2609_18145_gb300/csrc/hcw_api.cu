@@ -326,8 +326,10 @@ int fwd_bf16(const Shape& sh, const void* x, const void* Ws, const void* Wn, con
 // group and 128-token chunk.
 size_t stack_counter_bytes(long long tokens, int L) {
     const int layers = L < kMaxStackLayers ? L : kMaxStackLayers;
-    // per (layer, 128-token chunk) completion counters, then the unit counter
-    return align256((size_t)layers * (size_t)((tokens + 127) / 128) * sizeof(int) + 16);
+    // per (layer, 128-token chunk) completion counters, the unit counter, and
+    // the chunk counters of the top layer's dz written by the launch itself
+    const size_t chunks = (size_t)((tokens + 127) / 128);
+    return align256(((size_t)layers * chunks + 1 + chunks) * sizeof(int) + 16);
 }
 
 // Whether a stacked forward / input-gradient launch runs on pairs of SMs
@@ -628,15 +630,7 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
         return keep_g ? gbuf(l) : dz(l);
     };
     int rc;
-    if (relu) {
-        rc = launched(launch_relu_grad_mask_bf16(static_cast<const __nv_bfloat16*>(a.dy),
-                                                 mask(L - 1), static_cast<__nv_bfloat16*>(dz(L - 1)),
-                                                 sh.tokens, d, st),
-                      1);
-    } else {
-        rc = cuda_status(cudaMemcpyAsync(dz(L - 1), a.dy, ab, cudaMemcpyDeviceToDevice, st));
-    }
-    if (rc) return rc;
+    // the top layer's dz = dy * act'(z) is written by the first launch itself
     int* counters = reinterpret_cast<int*>(a.ws + (keep_g ? (size_t)L * a256 : 0));
     const int n_chunks = (int)((sh.tokens + 127) / 128);
     const bool pair = use_pairs(sh);
@@ -672,8 +666,14 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
         T.n_chunks = n_chunks;
         T.tokens = (int)sh.tokens;
         T.sched = counters + (size_t)cnt * n_chunks;
-        if (cudaMemsetAsync(counters, 0, ((size_t)cnt * n_chunks + 1) * sizeof(int), st) !=
-            cudaSuccess)
+        if (top == L - 1) {
+            T.top_dy = static_cast<const __nv_bfloat16*>(a.dy);
+            T.top_mask = relu ? mask(L - 1) : nullptr;
+            T.top_dz = static_cast<__nv_bfloat16*>(dz(L - 1));
+            T.in_counters = T.sched + 1;
+        }
+        if (cudaMemsetAsync(counters, 0, ((size_t)cnt * n_chunks + 1 + n_chunks) * sizeof(int),
+                            st) != cudaSuccess)
             return HCW_ERR_CUDA;
         rc = launch_rows(MODE_DX, BN, T, cnt, pair, st);
         if (rc) return rc;

@@ -83,6 +83,14 @@ struct TcLaunch {
     int n_chunks;
     int tokens;
     int* sched;   // stacked launches: next unit to hand out (zeroed per launch), or null
+    // Stacked input gradient, first run of layers: the launch itself writes the
+    // top layer's dz = dy * act'(z) (mask bits; a plain copy without them)
+    // before its units read it, counting each 128-token chunk in in_counters
+    // (zeroed before the launch).  Null top_dy: that dz is already in memory.
+    const __nv_bfloat16* top_dy;
+    const uint32_t* top_mask;
+    __nv_bfloat16* top_dz;
+    int* in_counters;
 };
 
 // Launch one tensor-core pass (one layer).

@@ -563,11 +563,13 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     if (PAIR) r.t = 2 * r.t + (int)rank;   // this CTA's half of the 256 rows
                     const int q0 = r.t * kBlockM;
                     const int lo0 = q0 & (ly.k - 1), hi0 = q0 >> ly.s;
-                    if (STACKED && l > 0) {
-                        // the unit's rows and their partners: two 128-token chunks
+                    if (STACKED && (l > 0 || (MODE == MODE_DX && L.top_dy != nullptr))) {
+                        // the unit's rows and their partners: two 128-token chunks,
+                        // written by the layer before (or by this launch's prologue)
                         int cs[2];
                         row_unit_chunks(q0, ly.s, ly.k, cs[0], cs[1]);
-                        const int* ctr = L.counters + (size_t)(l - 1) * L.n_chunks;
+                        const int* ctr = l > 0 ? L.counters + (size_t)(l - 1) * L.n_chunks
+                                               : L.in_counters;
                         // chunks past the end (ragged tail) have nothing to wait for
                         const int nc = (cs[0] < L.n_chunks) + (cs[1] < L.n_chunks);
                         if (cs[0] >= L.n_chunks) cs[0] = cs[1];
@@ -915,6 +917,42 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
             }
             return true;
         };
+        if (MODE == MODE_DX && STACKED && L.top_dy != nullptr) {
+            // The top layer's dz = dy * mask (or dy) for this CTA's 128-token
+            // chunks (b, b + grid, ...), 16-byte pieces, then each warp counts the
+            // elements it wrote in the chunk's counter (release after a proxy fence:
+            // the readers are TMA copies).
+            const int gpr = p.d / 8;                        // 16-byte pieces per row
+            for (int c = (int)blockIdx.x; c < L.n_chunks; c += (int)gridDim.x) {
+                const int rows = min(128, L.tokens - (c << 7));
+                int mine = 0;
+                for (int r = e; r < rows; r += EW, ++mine) {
+                    const size_t row = ((size_t)c << 7) + r;
+                    const uint4* src = reinterpret_cast<const uint4*>(L.top_dy + row * p.d);
+                    uint4* dst = reinterpret_cast<uint4*>(L.top_dz + row * p.d);
+                    for (int g = lane; g < gpr; g += 32) {
+                        uint4 v = src[g];
+                        if (L.top_mask) {
+                            const uint32_t bits =
+                                (L.top_mask[row * (p.d >> 5) + (g >> 2)] >> ((g & 3) * 8)) & 0xFFu;
+                            uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                            for (int i = 0; i < 4; ++i)
+                                w[i] &= ((bits >> (2 * i)) & 1u ? 0x0000FFFFu : 0u) |
+                                        ((bits >> (2 * i + 1)) & 1u ? 0xFFFF0000u : 0u);
+                            v = make_uint4(w[0], w[1], w[2], w[3]);
+                        }
+                        dst[g] = v;
+                    }
+                }
+                __syncwarp();
+                if (lane == 0 && mine > 0) {
+                    __threadfence();
+                    fence_proxy_async_global();
+                    red_release_gpu_add(L.in_counters + c, mine * p.d);
+                }
+            }
+        }
         for (; alive; ++ordinal) {
             int u = 0;
             if (lane == 0) u = consume_unit(ordinal);
