@@ -919,37 +919,53 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
         };
         if (MODE == MODE_DX && STACKED && L.top_dy != nullptr) {
             // The top layer's dz = dy * mask (or dy) for this CTA's 128-token
-            // chunks (b, b + grid, ...), 16-byte pieces, then each warp counts the
-            // elements it wrote in the chunk's counter (release after a proxy fence:
-            // the readers are TMA copies).
+            // chunks (b, b + grid, ...).  The chunk's 16-byte pieces are spread
+            // over the epilogue warps, eight loads in flight per lane; each warp
+            // then counts the elements it wrote in the chunk's counter (a release
+            // after a proxy fence: the readers are TMA copies).
             const int gpr = p.d / 8;                        // 16-byte pieces per row
+            constexpr int kU = 8;
             for (int c = (int)blockIdx.x; c < L.n_chunks; c += (int)gridDim.x) {
                 const int rows = min(128, L.tokens - (c << 7));
+                const int n = rows * gpr;                   // pieces in the chunk
+                const size_t base = ((size_t)c << 7) * (size_t)gpr;
+                const uint4* src = reinterpret_cast<const uint4*>(L.top_dy) + base;
+                uint4* dst = reinterpret_cast<uint4*>(L.top_dz) + base;
+                const uint32_t* mrow = L.top_mask ? L.top_mask + ((size_t)c << 7) * (p.d >> 5)
+                                                  : nullptr;
                 int mine = 0;
-                for (int r = e; r < rows; r += EW, ++mine) {
-                    const size_t row = ((size_t)c << 7) + r;
-                    const uint4* src = reinterpret_cast<const uint4*>(L.top_dy + row * p.d);
-                    uint4* dst = reinterpret_cast<uint4*>(L.top_dz + row * p.d);
-                    for (int g = lane; g < gpr; g += 32) {
-                        uint4 v = src[g];
-                        if (L.top_mask) {
-                            const uint32_t bits =
-                                (L.top_mask[row * (p.d >> 5) + (g >> 2)] >> ((g & 3) * 8)) & 0xFFu;
-                            uint32_t w[4] = {v.x, v.y, v.z, v.w};
+                for (int i0 = e * 32 + lane; i0 < n; i0 += kU * EW * 32) {
+                    uint4 v[kU];
+                    uint32_t mw[kU];
 #pragma unroll
-                            for (int i = 0; i < 4; ++i)
-                                w[i] &= ((bits >> (2 * i)) & 1u ? 0x0000FFFFu : 0u) |
-                                        ((bits >> (2 * i + 1)) & 1u ? 0xFFFF0000u : 0u);
-                            v = make_uint4(w[0], w[1], w[2], w[3]);
+                    for (int j = 0; j < kU; ++j) {
+                        const int i = i0 + j * EW * 32;
+                        if (i < n) {
+                            v[j] = src[i];
+                            // piece i covers columns 8 (i % gpr) .. + 7 of row i / gpr
+                            mw[j] = mrow ? mrow[(i / gpr) * (p.d >> 5) + ((i % gpr) >> 2)] : ~0u;
                         }
-                        dst[g] = v;
+                    }
+#pragma unroll
+                    for (int j = 0; j < kU; ++j) {
+                        const int i = i0 + j * EW * 32;
+                        if (i < n) {
+                            const uint32_t bits = (mw[j] >> (((i % gpr) & 3) * 8)) & 0xFFu;
+                            uint32_t w[4] = {v[j].x, v[j].y, v[j].z, v[j].w};
+#pragma unroll
+                            for (int q = 0; q < 4; ++q)
+                                w[q] &= ((bits >> (2 * q)) & 1u ? 0x0000FFFFu : 0u) |
+                                        ((bits >> (2 * q + 1)) & 1u ? 0xFFFF0000u : 0u);
+                            dst[i] = make_uint4(w[0], w[1], w[2], w[3]);
+                            mine += 8;
+                        }
                     }
                 }
-                __syncwarp();
+                mine = __reduce_add_sync(0xffffffffu, mine);
                 if (lane == 0 && mine > 0) {
                     __threadfence();
                     fence_proxy_async_global();
-                    red_release_gpu_add(L.in_counters + c, mine * p.d);
+                    red_release_gpu_add(L.in_counters + c, mine);
                 }
             }
         }
