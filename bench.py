@@ -433,10 +433,11 @@ def run_ours(args):
                                                          dW_self=gWs, dW_nbr=gWn, dbias=gb,
                                                          workspace=wws), reps)
     launch_flops = 3.0 * d * d * tokens * L     # per stacked launch, 16 causal layers
-    kernels = {"hcw_tc_kernel<FWD,256,16> (stacked forward)": fwd_ms,
-               "hcw_tc_kernel<DX,256,16> (stacked input gradient, + top ReLU pass)": dx_ms,
-               "hcw_tc_kernel<DWF,256,16> (weight and bias gradients, a unit per layer and "
-               "output tile)": dw_ms}
+    kernels = {"hcw_tc_kernel<FWD,256,16> (stacked forward on SM pairs)": fwd_ms,
+               "hcw_tc_kernel<DX,256,16> (stacked input gradient on SM pairs, top dz included)":
+                   dx_ms,
+               "hcw_dwp_kernel<256> (weight and bias gradients on SM pairs, a unit per layer "
+               "and 256 x 256 output tile)": dw_ms}
     dominant = max(kernels, key=kernels.get)
     dom_ms = kernels[dominant]
     peak = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
