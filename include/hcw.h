@@ -262,6 +262,31 @@ int hcw_layer_bwd_weight_noalloc(const void* x, const void* dz, int layer, int d
                                  int B, int n, int d, int dtype, unsigned flags,
                                  float* dW_self, float* dW_nbr, float* dbias, void* stream);
 
+/*
+ * Which kernels run the bf16 stacked forward and input gradient
+ * (hcw_stack_fwd, hcw_stack_bwd_data, hcw_stack_bwd).  Process-wide.
+ *   HCW_STACK_AUTO       resident where the shape fits and its pairs of SMs
+ *                        fill most of the GPU (B*n/128 >= 5/8 of the SMs),
+ *                        else streaming.  The default.
+ *   HCW_STACK_RESIDENT   resident wherever the shape fits.
+ *   HCW_STACK_STREAMING  streaming only.
+ * Resident: a cluster of two CTAs keeps 256 consecutive tokens (whole
+ * samples) in shared memory through a run of up to 16 layers.  Only the
+ * weights stream in, and each layer's output is written once.  The shape must
+ * have d in {128, 256, 512}, n <= 256 and B*n a multiple of 256.  The causal
+ * partner product costs 4d^2 flops per token there (every lane computed, half
+ * kept) instead of 3d^2.
+ * Streaming: every layer's tiles pass through global memory (L2); any shape.
+ * The resident input gradient keeps the residual stream g in fp32 between
+ * layers, where the streaming kernels round it to bf16 at every layer, so the
+ * two differ at bf16 rounding level.
+ * Returns the previous mode, or -1 (mode unchanged) for an unknown mode.
+ */
+#define HCW_STACK_AUTO      0
+#define HCW_STACK_RESIDENT  1
+#define HCW_STACK_STREAMING 2
+int hcw_set_stack_kernels(int mode);
+
 /* Number of kernels this library has launched in this process (all devices). */
 unsigned long long hcw_launch_count(void);
 

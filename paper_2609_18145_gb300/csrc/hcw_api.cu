@@ -340,6 +340,19 @@ bool use_pairs(const Shape& sh) {
     return pick_bn(sh.d) == 256 && sh.tokens / 2 > 128;
 }
 
+// Whether a bf16 stacked forward / input gradient runs on the resident
+// kernels (hcw_res.cu): the shape fits them (d in {128, 256, 512}, n <= 256,
+// whole 256-token tiles) and, unless hcw_set_stack_kernels says otherwise,
+// their pairs fill most of the GPU (one pair per 256 tokens, no more).
+std::atomic<int> g_stack_kernels{HCW_STACK_AUTO};
+
+bool use_resident(const Shape& sh) {
+    const int mode = g_stack_kernels.load(std::memory_order_relaxed);
+    if (mode == HCW_STACK_STREAMING || !res_supported(sh.d, sh.n, sh.tokens)) return false;
+    if (mode == HCW_STACK_RESIDENT) return true;
+    return sh.tokens / 128 >= (5 * (long long)sm_count()) / 8;
+}
+
 // Row-unit geometry of a pair launch: units count row-block pairs.
 void pair_units(TcParams& p) { p.n_units = ((p.n_rb + 1) / 2) * p.n_nt * 2; }
 
@@ -385,6 +398,34 @@ int stack_fwd_group(const Shape& sh, int l0, int n, int layer0, int dim_override
     cudaError_t e = cudaMemsetAsync(counters, 0, ((size_t)n * L.n_chunks + 1) * sizeof(int), st);
     if (e != cudaSuccess) return HCW_ERR_CUDA;
     return launch_rows(MODE_FWD, BN, L, n, pair, st);
+}
+
+// Layers [l0, l0 + n) of a bf16 stack in one resident launch (hcw_res.cu).
+template <class In, class Out, class Mask>
+int stack_fwd_resident(const Shape& sh, int l0, int n, int layer0, int dim_override,
+                       const uint8_t* Ws, const uint8_t* Wn, const float* bias, unsigned flags,
+                       In in_ptr, Out out_ptr, Mask mask_ptr, cudaStream_t st) {
+    const int d = sh.d, N = d >= 256 ? d / 2 : d;
+    const size_t wb = (size_t)d * d * 2;
+    static thread_local ResLaunch R;
+    memset(&R, 0, sizeof(R));
+    for (int i = 0; i < n; ++i) {
+        const int l = l0 + i;
+        const int s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
+        if (!map_weight(&R.wmap[i][0], Ws + l * wb, d, N / 2) ||
+            !map_weight(&R.wmap[i][1], Wn + l * wb, d, N / 2))
+            return HCW_ERR_CUDA;
+        R.layer[i] = {s, RES_Y, out_ptr(l), bias ? bias + (size_t)l * d : nullptr, mask_ptr(l),
+                      nullptr};
+    }
+    R.in = in_ptr(l0);
+    R.n_layers = n;
+    R.d = d;
+    R.n = sh.n;
+    R.tokens = (int)sh.tokens;
+    R.flags = flags;
+    R.timeout_ns = g_timeout_ns;
+    return launched(launch_res(MODE_FWD, R, st), 1);
 }
 
 // dx: a row gathers dz from its partner exactly when the partner received from it
@@ -563,12 +604,21 @@ int layer_bwd_impl(const Shape& sh, int dtype, const void* x, const void* z, con
 //   single-layer weight-gradient workspace (used when the layers are too few
 //   to fill the GPU and run one by one).  fp32: the single-layer workspace.
 //   hcw_stack_bwd: every layer's dz, then both of the above.
+// bf16: bytes in front of the counters.  The streaming kernels keep every
+// layer's g there (ReLU with the residual); the resident kernels use the first
+// 2 act_bytes as one fp32 [tokens][d] buffer (g where rows change CTA, and
+// between launches of more than 16 layers).
+size_t stack_g_region(const Shape& sh, unsigned flags, int L) {
+    const size_t a = align256(sh.act_bytes);
+    const bool keep_g = (flags & HCW_ACT_RELU) && (flags & HCW_RESIDUAL);
+    size_t r = keep_g ? (size_t)L * a : 0;
+    if (res_supported(sh.d, sh.n, sh.tokens) && r < 2 * a) r = 2 * a;
+    return r;
+}
+
 size_t stack_data_ws(const Shape& sh, int dtype, unsigned flags, int L) {
     const size_t a = align256(sh.act_bytes);
-    if (dtype == HCW_BF16) {
-        const bool keep_g = (flags & HCW_ACT_RELU) && (flags & HCW_RESIDUAL);
-        return (keep_g ? (size_t)L * a : 0) + stack_counter_bytes(sh.tokens, L);
-    }
+    if (dtype == HCW_BF16) return stack_g_region(sh, flags, L) + stack_counter_bytes(sh.tokens, L);
     return 2 * a;
 }
 
@@ -608,10 +658,66 @@ struct StackWeight {
     uint8_t* ws;
 };
 
+// bf16 input gradients on the resident kernels: one launch per run of <= 16
+// layers, top down.  The first launch starts from dy; a run that stops above
+// layer 0 leaves g (fp32) in the workspace for the next one.
+int stack_data_resident(const Shape& sh, const StackData& a, cudaStream_t st) {
+    const int d = sh.d, L = a.L, N = d >= 256 ? d / 2 : d;
+    const bool relu = (a.flags & HCW_ACT_RELU) != 0;
+    const size_t ab = sh.act_bytes, wb = (size_t)d * d * 2;
+    const size_t mb = mask_bytes(sh);
+    float* gs = reinterpret_cast<float*>(a.ws);
+    auto dz = [&](int l) -> void* { return a.dz + (size_t)l * ab; };
+    auto mask = [&](int l) {
+        return reinterpret_cast<const uint32_t*>(static_cast<const uint8_t*>(a.masks) +
+                                                 (size_t)l * mb);
+    };
+    static thread_local ResLaunch R;
+    for (int top = L - 1; top >= 0; top -= kMaxStackLayers) {
+        const int cnt = top + 1 < kMaxStackLayers ? top + 1 : kMaxStackLayers;
+        memset(&R, 0, sizeof(R));
+        for (int i = 0; i < cnt; ++i) {
+            const int l = top - i;
+            const int s = stack_layer_dim(sh, a.layer0, a.dim_override, l);
+            if (!map_weight_blocks(&R.wmap[i][0], a.Ws + l * wb, d, N / 128) ||
+                !map_weight_blocks(&R.wmap[i][1], a.Wn + l * wb, d, N / 128))
+                return HCW_ERR_CUDA;
+            ResLayer& y = R.layer[i];
+            y.s = s;
+            if (l == 0) {
+                y.out_kind = RES_DX;
+                y.out = a.dx;
+            } else if (i == cnt - 1) {
+                y.out_kind = RES_G;
+                y.out = gs;
+            } else {
+                y.out_kind = RES_DZ;
+                y.out = dz(l - 1);
+                y.mprev = relu ? mask(l - 1) : nullptr;
+            }
+        }
+        R.in = top == L - 1 ? a.dy : static_cast<const void*>(gs);
+        R.in_f32 = top == L - 1 ? 0 : 1;
+        R.in_mask = relu ? mask(top) : nullptr;
+        R.in_dz = static_cast<__nv_bfloat16*>(dz(top));
+        R.gscratch = gs;
+        R.n_layers = cnt;
+        R.d = d;
+        R.n = sh.n;
+        R.tokens = (int)sh.tokens;
+        R.flags = a.flags;
+        R.timeout_ns = g_timeout_ns;
+        const int rc = launched(launch_res(MODE_DX, R, st), 1);
+        if (rc) return rc;
+    }
+    return HCW_OK;
+}
+
 // bf16 input gradients: the ReLU gradient of the top layer, then one stacked
 // launch per run of <= 16 layers, top down, whose kernel also applies the
 // ReLU gradient of the layer below.
 int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
+    if (use_resident(sh)) return stack_data_resident(sh, a, st);
     const int d = sh.d, BN = pick_bn(d), L = a.L;
     const bool relu = (a.flags & HCW_ACT_RELU) != 0;
     const bool resid = (a.flags & HCW_RESIDUAL) != 0;
@@ -631,7 +737,7 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
     };
     int rc;
     // the top layer's dz = dy * act'(z) is written by the first launch itself
-    int* counters = reinterpret_cast<int*>(a.ws + (keep_g ? (size_t)L * a256 : 0));
+    int* counters = reinterpret_cast<int*>(a.ws + stack_g_region(sh, a.flags, L));
     const int n_chunks = (int)((sh.tokens + 127) / 128);
     const bool pair = use_pairs(sh);
     const int pw = epi_patch_cols(BN);
@@ -1126,10 +1232,16 @@ int hcw_stack_fwd(const void* x, const void* W_self, const void* W_nbr, const fl
         // up to kMaxStackLayers layers per persistent launch
         for (int l0 = 0; l0 < L; l0 += kMaxStackLayers) {
             const int cnt = L - l0 < kMaxStackLayers ? L - l0 : kMaxStackLayers;
-            rc = stack_fwd_group(sh, l0, cnt, layer0, dim_override,
-                                 static_cast<const uint8_t*>(W_self),
-                                 static_cast<const uint8_t*>(W_nbr), bias, flags, in_ptr, out_ptr,
-                                 mask_ptr, static_cast<int*>(workspace), st);
+            if (use_resident(sh))
+                rc = stack_fwd_resident(sh, l0, cnt, layer0, dim_override,
+                                        static_cast<const uint8_t*>(W_self),
+                                        static_cast<const uint8_t*>(W_nbr), bias, flags, in_ptr,
+                                        out_ptr, mask_ptr, st);
+            else
+                rc = stack_fwd_group(sh, l0, cnt, layer0, dim_override,
+                                     static_cast<const uint8_t*>(W_self),
+                                     static_cast<const uint8_t*>(W_nbr), bias, flags, in_ptr,
+                                     out_ptr, mask_ptr, static_cast<int*>(workspace), st);
             if (rc) return rc;
         }
         return HCW_OK;
@@ -1250,12 +1362,21 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void
     return dtype == HCW_BF16 ? stack_weight_bf16(sh, wa, st) : stack_weight_f32(sh, wa, st);
 }
 
+int hcw_set_stack_kernels(int mode) {
+    if (mode != HCW_STACK_AUTO && mode != HCW_STACK_RESIDENT && mode != HCW_STACK_STREAMING)
+        return -1;
+    return g_stack_kernels.exchange(mode);
+}
+
 unsigned long long hcw_launch_count(void) { return g_launches.load(); }
 
 int hcw_sync_status(void* stream) {
     if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return HCW_ERR_CUDA;
-    int word = 0;
-    if (error_word_read_clear(&word) != cudaSuccess) return HCW_ERR_CUDA;
+    int word = 0, word_res = 0;
+    if (error_word_read_clear(&word) != cudaSuccess ||
+        res_error_word_read_clear(&word_res) != cudaSuccess)
+        return HCW_ERR_CUDA;
+    if (!word) word = word_res;
     if (word) return word == HCW_ERR_TIMEOUT ? HCW_ERR_TIMEOUT : HCW_ERR_CUDA;
     return HCW_OK;
 }

@@ -105,6 +105,55 @@ cudaError_t launch_tc_stack(int mode, int BN, const TcLaunch<kMaxStackLayers>& L
 cudaError_t launch_tc_stack_pair(int mode, int BN, const TcLaunch<kMaxStackLayers>& L, int grid,
                                  cudaStream_t stream);
 
+// ---- Resident stacked launches (hcw_res.cu) ----
+// A cluster of two CTAs keeps 256 consecutive tokens (whole samples, n <= 256)
+// of the running activations (forward) or gradient (input gradient) in shared
+// memory through every layer of the run; only the weights stream in.
+enum ResOut {
+    RES_Y = 0,    // forward: y_l, bf16 [tokens][d] (+ ReLU mask words in mout)
+    RES_DZ = 1,   // input gradient: dz_{l-1} = bf16(g_{l-1}) * mask_{l-1}, bf16
+    RES_DX = 2,   // input gradient of the stack's first layer: dx = bf16(g_{-1})
+    RES_G = 3     // input gradient continued by a later launch: g_{l-1}, fp32
+};
+
+struct ResLayer {
+    int s;                    // cube dimension
+    int out_kind;             // ResOut
+    void* out;                // where the layer's result goes (see ResOut)
+    const float* bias;        // forward: bias [d] or null
+    uint32_t* mout;           // forward: ReLU mask words [tokens][d/32] or null
+    const uint32_t* mprev;    // RES_DZ: mask words of the layer below, or null (no ReLU)
+};
+
+struct ResLaunch {
+    // per layer (in processing order: the forward bottom up, the input
+    // gradient top down): W_self and W_nbr as the B operand, half a column
+    // chunk per CTA (forward: K-major 2-D boxes; input gradient: MN-major
+    // 3-D block boxes)
+    CUtensorMap wmap[kMaxStackLayers][2];
+    ResLayer layer[kMaxStackLayers];
+    const void* in;           // forward: the first layer's input, bf16 [tokens][d];
+                              // input gradient: the top layer's output gradient,
+                              // bf16 dy, or fp32 g (in_f32) from an earlier launch
+    int in_f32;
+    const uint32_t* in_mask;  // input gradient: the top layer's mask words, or null
+    __nv_bfloat16* in_dz;     // input gradient: the top layer's dz is stored here
+    float* gscratch;          // input gradient, residual: fp32 [tokens][d] used when the
+                              // rows change CTA between layers (n = 256)
+    int n_layers;
+    int d, n, tokens;
+    unsigned flags;           // HCW_CAUSAL | HCW_RESIDUAL | HCW_ACT_RELU
+    unsigned long long timeout_ns;
+};
+
+// Whether the resident kernels take this shape: d in {128, 256, 512},
+// n <= 256, whole 256-token tiles.
+bool res_supported(int d, int n, long long tokens);
+// Launch MODE_FWD or MODE_DX over tokens / 256 clusters of two CTAs.
+cudaError_t launch_res(int mode, const ResLaunch& L, cudaStream_t stream);
+// Read the resident kernels' error word and reset it to 0 (synchronous).
+cudaError_t res_error_word_read_clear(int* word);
+
 // Dynamic shared memory the tensor-core kernel uses for this N tile.
 size_t tc_smem_bytes(int BN);
 int tc_stages(int BN);

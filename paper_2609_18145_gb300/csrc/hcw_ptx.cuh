@@ -4,16 +4,19 @@
 #pragma once
 
 #include <cuda.h>
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
 namespace hcw {
 
-// Error word (one per device): kernels that give up on a bounded wait write a
-// non-zero code here; hcw_sync_status reads and clears it.  Defined here
-// because the tensor-core translation unit (hcw_tc.cu) is the only one that
-// includes this header.
+// Error word (one per device and translation unit): kernels that give up on a
+// bounded wait write a non-zero code here; hcw_sync_status reads and clears
+// the word of every translation unit that includes this header (hcw_tc.cu,
+// hcw_res.cu), each through its own read-and-clear function.
+namespace {
 __device__ int g_error_word = 0;
+}
 
 constexpr int kErrTimeout = 6;
 
@@ -63,6 +66,20 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
     return ok != 0;
 }
 
+// The same with acquire semantics at cluster scope: what the other CTA of the
+// cluster wrote before its release-arrive on this barrier is visible after.
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
 // Bounded wait for the phase with the given parity to complete.  Gives up
 // (returns false) when *abort becomes non-zero or after timeout_ns; on a
 // timeout it records kErrTimeout in the device error word and raises *abort
@@ -82,6 +99,35 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
             }
         }
     }
+}
+
+// mbar_wait with cluster-scope acquire (mbar_try_wait_cluster).
+__device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity,
+                                                  volatile int* abort, uint64_t timeout_ns) {
+    if (mbar_try_wait_cluster(bar, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t it = 1;; ++it) {
+        if (mbar_try_wait_cluster(bar, parity)) return true;
+        if ((it & 63u) == 0) {
+            if (*abort) return false;
+            if (globaltimer_ns() - t0 > timeout_ns) {
+                atomicExch(&g_error_word, kErrTimeout);
+                *abort = 1;
+                return false;
+            }
+        }
+    }
+}
+
+// Wait that only gives up on time (used to drain in-flight work after an
+// abort, when the abort flag is already set).
+__device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity,
+                                                uint64_t timeout_ns) {
+    const uint64_t t0 = globaltimer_ns();
+    while (!mbar_try_wait(bar, parity)) {
+        if (globaltimer_ns() - t0 > timeout_ns) return false;
+    }
+    return true;
 }
 
 // ------------------------------------------------------------------ TMA
@@ -233,6 +279,30 @@ __device__ __forceinline__ void tmem_ld_wait() {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// Wait for this thread's tcgen05.ld and tie the destination registers to the
+// wait so the compiler cannot read them earlier.
+__device__ __forceinline__ void tmem_ld_wait_regs(uint32_t (&r)[32]) {
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
+                   "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]),
+                   "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]),
+                   "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
+                   "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]),
+                   "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
+                 :
+                 : "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<uint32_t*>(&h);
+}
+
+__device__ __forceinline__ float2 unpack_bf16x2(uint32_t w) {
+    __nv_bfloat162 h = *reinterpret_cast<__nv_bfloat162*>(&w);
+    return __bfloat1622float2(h);
+}
+
 // ------------------------------------------------------------------ CTA pairs
 // A cluster of two CTAs on two SMs: the leader (rank 0) issues the pair's
 // tcgen05.mma.cta_group::2 instructions; each CTA holds half of A (its rows)
@@ -356,6 +426,43 @@ __device__ __forceinline__ void mma_bf16_f32_pair(uint32_t d_tmem, uint64_t ades
         : "memory");
 }
 
+// Pair MMA whose D rows are written only in the lanes enabled by `disable`:
+// bit j of word i set = TMEM lane 32 i + j keeps its value (the same four
+// words for both CTAs of the pair).  Always accumulates.
+__device__ __forceinline__ void mma_bf16_f32_pair_masked(uint32_t d_tmem, uint64_t adesc,
+                                                         uint64_t bdesc, uint32_t idesc,
+                                                         const uint32_t (&disable)[4]) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %12, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, "
+        "{%4, %5, %6, %7, %8, %9, %10, %11}, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(disable[0]), "r"(disable[1]), "r"(disable[2]),
+        "r"(disable[3]), "r"(disable[0]), "r"(disable[1]), "r"(disable[2]), "r"(disable[3]),
+        "r"(1u)
+        : "memory");
+}
+
+// 32 lanes x 32 columns of 32-bit TMEM words from registers: thread t of the
+// warp writes lane (base lane + t), columns c..c+31 from r[0..31].
+__device__ __forceinline__ void tmem_st_32x32b_x32(uint32_t taddr, const uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, "
+        "%17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(
+            taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+        "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+        "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
+        "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
+        "r"(r[29]), "r"(r[30]), "r"(r[31])
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_st_wait() {
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
 // Arrive once on `bar` (same offset) in each CTA of `cta_mask` when every
 // pair MMA issued so far by this thread has completed.
 __device__ __forceinline__ void mma_commit_pair(uint64_t* bar, uint16_t cta_mask) {
@@ -380,6 +487,19 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo
     desc |= (uint64_t)1 << 46;
     desc |= (uint64_t)2 << 61;
     return desc;
+}
+
+// Descriptor of a K-major operand without swizzle whose rows are 16 bytes
+// apart: core matrices of 8 rows x 16 bytes, 8-row groups 128 bytes apart
+// (SBO), 16-byte column chunks `chunk_bytes` apart (LBO).  Any 16-byte-aligned
+// start is legal, so a window shifted by any number of rows is one descriptor.
+__device__ __forceinline__ uint64_t smem_desc_rows16(uint32_t saddr, uint32_t chunk_bytes) {
+    uint64_t desc = 0;
+    desc |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    desc |= (uint64_t)((chunk_bytes >> 4) & 0x3FFFu) << 16;
+    desc |= (uint64_t)(128u >> 4) << 32;
+    desc |= (uint64_t)1 << 46;
+    return desc;   // swizzle mode 0
 }
 
 // Instruction descriptor for kind::f16 with bf16 A/B and fp32 D.

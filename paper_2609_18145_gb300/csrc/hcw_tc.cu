@@ -210,16 +210,6 @@ __device__ __forceinline__ WUnit decode_w_any(const TcParams& p, int u, bool sta
     return decode_w_unit(p, local);
 }
 
-__device__ __forceinline__ uint32_t pack_bf16x2(float a, float b) {
-    __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
-    return *reinterpret_cast<uint32_t*>(&h);
-}
-
-__device__ __forceinline__ float2 unpack_bf16x2(uint32_t w) {
-    __nv_bfloat162 h = *reinterpret_cast<__nv_bfloat162*>(&w);
-    return __bfloat1622float2(h);
-}
-
 // 16-byte piece m of patch row r in an epilogue buffer, in the layout of the
 // TMA box that fills / drains it: 128-byte rows with the 128-byte swizzle
 // (piece m ^ (r & 7)), or 64-byte rows with the 64-byte swizzle
@@ -229,20 +219,6 @@ template <int ROW_BYTES>
 __device__ __forceinline__ uint4* patch_piece(uint8_t* buf, int r, int m) {
     if (ROW_BYTES == 128) return reinterpret_cast<uint4*>(buf + r * 128 + ((m ^ (r & 7)) << 4));
     return reinterpret_cast<uint4*>(buf + r * 64 + ((m ^ ((r >> 1) & 3)) << 4));
-}
-
-// Wait for this thread's tcgen05.ld and tie the destination registers to the
-// wait so the compiler cannot read them earlier.
-__device__ __forceinline__ void tmem_ld_wait_regs(uint32_t (&r)[32]) {
-    asm volatile("tcgen05.wait::ld.sync.aligned;"
-                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]),
-                   "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]),
-                   "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]),
-                   "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]),
-                   "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]),
-                   "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]), "+r"(r[31])
-                 :
-                 : "memory");
 }
 
 __device__ __forceinline__ int ld_acquire_gpu(const int* p) {
@@ -337,17 +313,6 @@ __device__ __forceinline__ bool wait_shared_geq(const int* p, int target, volati
             }
         }
     }
-}
-
-// Wait that only gives up on time (used to drain in-flight work after an
-// abort, when the abort flag is already set).
-__device__ __forceinline__ bool mbar_wait_drain(uint64_t* bar, uint32_t parity,
-                                                uint64_t timeout_ns) {
-    const uint64_t t0 = globaltimer_ns();
-    while (!mbar_try_wait(bar, parity)) {
-        if (globaltimer_ns() - t0 > timeout_ns) return false;
-    }
-    return true;
 }
 
 }  // namespace

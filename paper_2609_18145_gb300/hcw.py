@@ -27,6 +27,10 @@ HCW_ERR_CUDA = 5
 HCW_ERR_TIMEOUT = 6
 HCW_ERR_WORKSPACE = 7
 
+HCW_STACK_AUTO = 0
+HCW_STACK_RESIDENT = 1
+HCW_STACK_STREAMING = 2
+
 HCW_BF16 = 0
 HCW_F32 = 1
 
@@ -71,6 +75,7 @@ _SIGNATURES = {
     "hcw_stack_bwd_weight_workspace_bytes": ([_I, _I, _I, _I, _U, _I], _SZ),
     "hcw_stack_bwd": ([_P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P,
                        _P, _P, _SZ, _P], _I),
+    "hcw_set_stack_kernels": ([_I], _I),
     "hcw_sync_status": ([_P], _I),
     "hcw_selftest_wait": ([_LL, _P], _I),
 }
@@ -243,6 +248,15 @@ def hcw_layer_bwd_weight(x, dz, layer: int = 0, dim_override: int = -1, flags: i
                                       _ptr(dW_self), _ptr(dW_nbr), _ptr(dbias), _ptr(ws),
                                       ws.numel(), _stream(stream)), "hcw_layer_bwd_weight")
     return dW_self, dW_nbr, dbias
+
+
+def hcw_set_stack_kernels(mode: int) -> int:
+    """Select the bf16 stacked-launch kernels (HCW_STACK_AUTO, _RESIDENT or
+    _STREAMING) for this process; returns the previous mode."""
+    prev = int(lib().hcw_set_stack_kernels(int(mode)))
+    if prev < 0:
+        raise ValueError("hcw_set_stack_kernels: unknown mode %r" % (mode,))
+    return prev
 
 
 def hcw_launch_count() -> int:

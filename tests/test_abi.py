@@ -200,3 +200,18 @@ def test_workspace_query_terminates_for_wide_layers(hcw):
         a = hcw.hcw_layer_bwd_weight_workspace_bytes(1 << 20, 4, d, hcw.HCW_BF16, 0)
         b = hcw.hcw_workspace_bytes(1 << 20, 4, d, hcw.HCW_BF16, hcw.HCW_CAUSAL)
         assert a > 0 and b > 0
+
+
+def test_stack_kernel_selection_is_a_process_setting(hcw):
+    lib = hcw.lib()
+    prev = lib.hcw_set_stack_kernels(hcw.HCW_STACK_RESIDENT)
+    try:
+        assert prev in (hcw.HCW_STACK_AUTO, hcw.HCW_STACK_RESIDENT, hcw.HCW_STACK_STREAMING)
+        assert lib.hcw_set_stack_kernels(hcw.HCW_STACK_STREAMING) == hcw.HCW_STACK_RESIDENT
+        assert lib.hcw_set_stack_kernels(7) == -1          # unknown: unchanged
+        assert lib.hcw_set_stack_kernels(-1) == -1
+        assert lib.hcw_set_stack_kernels(hcw.HCW_STACK_AUTO) == hcw.HCW_STACK_STREAMING
+        with pytest.raises(ValueError):
+            hcw.hcw_set_stack_kernels(3)
+    finally:
+        lib.hcw_set_stack_kernels(prev)

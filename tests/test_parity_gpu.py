@@ -251,6 +251,82 @@ def test_stack_forward_backward(H, case):
             assert rel(g, r) <= tol, (name, what, rel(g, r))
 
 
+@pytest.fixture
+def resident(H):
+    """Run the bf16 stacks on the resident kernels wherever the shape fits."""
+    prev = H.hcw_set_stack_kernels(H.HCW_STACK_RESIDENT)
+    yield
+    H.hcw_set_stack_kernels(prev)
+
+
+RESIDENT_CASES = [
+    # name, B, n, d, L, flags, w_std, layer0, dim: every shape fits the resident
+    # kernels (d in {128, 256, 512}, n <= 256, B*n a multiple of 256)
+    # n = 256: the layers with s = 7 use the other CTA split (rows change CTA twice
+    # per rotation); two accumulator chunks of 256 columns
+    ("n256_d512_causal_res_relu", 2, 256, 512, 16, CAUSAL | RESIDUAL | RELU, (1 / 1024) ** 0.5,
+     0, -1),
+    # both partner windows, starting mid-rotation
+    ("n256_d512_noncausal_res", 2, 256, 512, 10, RESIDUAL, (1 / 1024) ** 0.5, 3, -1),
+    # chunks of 128 columns; no residual (the input gradient starts each layer from 0)
+    ("n256_d256_causal_relu", 2, 256, 256, 9, CAUSAL | RELU, (1 / 512) ** 0.5, 5, -1),
+    # two samples of 128 per CTA pair, no split change
+    ("n128_d512_causal_res", 2, 128, 512, 7, CAUSAL | RESIDUAL, (1 / 1024) ** 0.5, 0, -1),
+    # one accumulator chunk (d = 128), eight samples of 32 per pair
+    ("n32_d128_noncausal_relu", 8, 32, 128, 5, RELU, (1 / 256) ** 0.5, 0, -1),
+    # the fixed control on dimension 7: every layer on the other split
+    ("n256_d128_dim7", 2, 256, 128, 4, CAUSAL | RESIDUAL | RELU, (1 / 256) ** 0.5, 0, 7),
+    # 20 layers: two launches, the second continuing from the first's output
+    # (forward) and from its fp32 residual stream (input gradient)
+    ("n256_d128_20_layers", 2, 256, 128, 20, CAUSAL | RESIDUAL | RELU, (1 / 256) ** 0.5, 0, -1),
+]
+
+
+@pytest.mark.parametrize("case", RESIDENT_CASES, ids=lambda c: c[0])
+def test_resident_stack_forward_backward(H, resident, case):
+    name, B, n, d, L, flags, w_std, layer0, dim = case
+    pr = synth.problem(B, n, d, L=L, seed=13, w_std=w_std)
+    got, ref = run_stack(H, pr, torch.bfloat16, L, flags, layer0=layer0, dim=dim)
+    assert H.hcw_sync_status() == H.HCW_OK
+    for g, r, what in zip(got, ref, WHAT):
+        if g.size:
+            assert rel(g, r) <= TOL_BF16, (name, what, rel(g, r))
+
+
+@pytest.mark.parametrize("flags", [CAUSAL | RESIDUAL | RELU, RESIDUAL, CAUSAL])
+def test_resident_and_streaming_stacks_agree(H, flags):
+    """The same stack on both kernel families.  Forward: the resident kernel
+    issues the same MMAs in the same K order (self part, then partner part)
+    and the same epilogue arithmetic, so y, the saved activations and the ReLU
+    masks are identical.  Input gradient: the resident kernel keeps the
+    residual stream in fp32 between layers (the streaming one rounds it to
+    bf16 at each), so dx and the weight gradients agree to bf16 rounding."""
+    B, n, d, L = 4, 256, 512, 9
+    pr = synth.problem(B, n, d, L=L, seed=17, w_std=(1 / (2 * d)) ** 0.5)
+    x, _ = dev(pr.x, torch.bfloat16)
+    Ws, _ = dev(pr.W_self, torch.bfloat16)
+    Wn, _ = dev(pr.W_nbr, torch.bfloat16)
+    dy, _ = dev(pr.dy, torch.bfloat16)
+    bias = torch.from_numpy(pr.bias).cuda()
+    out = {}
+    for mode in (H.HCW_STACK_STREAMING, H.HCW_STACK_RESIDENT):
+        prev = H.hcw_set_stack_kernels(mode)
+        try:
+            y, acts, masks = H.hcw_stack_fwd(x, Ws, Wn, bias, 2, -1, flags)
+            res = H.hcw_stack_bwd(x, acts, masks, dy, Ws, Wn, 2, -1, flags)
+            torch.cuda.synchronize()
+            assert H.hcw_sync_status() == H.HCW_OK
+        finally:
+            H.hcw_set_stack_kernels(prev)
+        out[mode] = (y, acts, masks) + tuple(res)
+    a, b = out[H.HCW_STACK_STREAMING], out[H.HCW_STACK_RESIDENT]
+    assert torch.equal(a[0], b[0]) and torch.equal(a[1], b[1])
+    if flags & RELU:
+        assert torch.equal(a[2], b[2])
+    for i, what in ((3, "dx"), (4, "dW_self"), (5, "dW_nbr"), (6, "dbias")):
+        assert rel(host(b[i]), host(a[i])) <= 1e-2, what
+
+
 def test_stack_fixed_dimension_control(H):
     pr = synth.problem(16, 64, 128, L=6, seed=5, w_std=(1 / 256) ** 0.5)
     got, ref = run_stack(H, pr, torch.bfloat16, 6, 0, dim=0)
@@ -467,16 +543,28 @@ def test_split_backward_matches_fused(H):
     assert torch.equal(gb, c)
 
 
+@pytest.mark.parametrize("kernels", ["auto", "resident"])
 @pytest.mark.parametrize("dtype,flags", [(torch.bfloat16, CAUSAL | RESIDUAL | RELU),
                                          (torch.bfloat16, CAUSAL), (torch.bfloat16, RELU),
                                          (torch.float32, CAUSAL | RESIDUAL | RELU),
                                          (torch.float32, RESIDUAL)])
-def test_stack_backward_halves_match_the_whole(H, dtype, flags):
+def test_stack_backward_halves_match_the_whole(H, dtype, flags, kernels):
     """hcw_stack_bwd_data then hcw_stack_bwd_weight give exactly what
     hcw_stack_bwd gives, and the dz they pass on is each layer's dy * act'(z)
     chain (checked on the top layer, where it is dy masked)."""
+    if kernels == "resident" and dtype == torch.float32:
+        pytest.skip("the resident kernels are bf16 only")
     d = 64 if dtype == torch.float32 else 256
     B, n, L = 4, 64, 5
+    prev = H.hcw_set_stack_kernels(H.HCW_STACK_RESIDENT if kernels == "resident"
+                                   else H.HCW_STACK_AUTO)
+    try:
+        _halves_match_the_whole(H, dtype, flags, d, B, n, L)
+    finally:
+        H.hcw_set_stack_kernels(prev)
+
+
+def _halves_match_the_whole(H, dtype, flags, d, B, n, L):
     pr = synth.problem(B, n, d, L=L, seed=21, w_std=(1 / (2 * d)) ** 0.5)
     x, _ = dev(pr.x, dtype)
     Ws, _ = dev(pr.W_self, dtype)
