@@ -36,6 +36,7 @@ METRIC = "HypercubeMix fwd+bwd tokens/s at n=256,d=512 bf16; % of roofline"
 WORKLOAD = "charlm_w256_d512"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 L2_FLUSH_BYTES = 256 << 20
+STACK_KERNELS = {"auto": 0, "resident": 1, "streaming": 2}   # hcw_set_stack_kernels modes
 
 
 def load_peaks():
@@ -189,7 +190,7 @@ class ClockSampler:
 
 def kernel_source_sha():
     h = hashlib.sha256()
-    for f in ("hcw_tc.cu", "hcw_ptx.cuh", "hcw_api.cu"):
+    for f in ("hcw_tc.cu", "hcw_res.cu", "hcw_ptx.cuh", "hcw_api.cu"):
         with open(os.path.join(ROOT, "paper_2609_18145_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
@@ -308,6 +309,7 @@ def run_ours(args):
     replicas.init("nccl")
     dev = torch.device("cuda", local_rank)
     H.lib()
+    H.hcw_set_stack_kernels(STACK_KERNELS[args.stack_kernels])
 
     w = workload()
     B, n, d, L, flags = w["B"], w["n"], w["d"], w["L"], w["flags"]
@@ -433,9 +435,16 @@ def run_ours(args):
                                                          dW_self=gWs, dW_nbr=gWn, dbias=gb,
                                                          workspace=wws), reps)
     launch_flops = 3.0 * d * d * tokens * L     # per stacked launch, 16 causal layers
-    kernels = {"hcw_tc_kernel<FWD,256,16> (stacked forward on SM pairs)": fwd_ms,
-               "hcw_tc_kernel<DX,256,16> (stacked input gradient on SM pairs, top dz included)":
-                   dx_ms,
+    family = H.hcw_stack_kernels_used(B, n, d)
+    if family == H.HCW_STACK_RESIDENT:
+        fwd_name = ("hcw_res_kernel<FWD,%d> (resident stacked forward: 256 tokens per SM pair "
+                    "through all layers)" % d)
+        dx_name = ("hcw_res_kernel<DX,%d> (resident stacked input gradient, top dz included)"
+                   % d)
+    else:
+        fwd_name = "hcw_tc_kernel<FWD,256,16> (stacked forward on SM pairs)"
+        dx_name = "hcw_tc_kernel<DX,256,16> (stacked input gradient on SM pairs, top dz included)"
+    kernels = {fwd_name: fwd_ms, dx_name: dx_ms,
                "hcw_dwp_kernel<256> (weight and bias gradients on SM pairs, a unit per layer "
                "and 256 x 256 output tile)": dw_ms}
     dominant = max(kernels, key=kernels.get)
@@ -504,6 +513,8 @@ def run_ours(args):
                        "act": "relu", "bias": True,
                        "l2": "flushed before every timed step (256 MiB write, untimed)",
                        "parallelism": "replicas" if world > 1 else "single",
+                       "stack_kernels": "resident" if family == H.HCW_STACK_RESIDENT
+                                        else "streaming",
                        "launch": "host calls" if args.no_graph else "CUDA graph of the step's calls"},
             "roofline": {"bound": "tensor", "kernel": dominant, "achieved": achieved,
                          "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
@@ -538,6 +549,7 @@ def run_kernel_only(args):
     B, n, d, flags = args.batch, w["n"], w["d"], w["flags"]
     dev = torch.device("cuda", 0)
     H.lib()
+    H.hcw_set_stack_kernels(STACK_KERNELS[args.stack_kernels])
     pr = synth.problem(B, n, d, L=1, seed=0, w_std=(1 / (2 * d)) ** 0.5, x_ids="zipf256")
     x = torch.from_numpy(pr.x).to(torch.bfloat16).to(dev)
     dz = torch.from_numpy(pr.dy).to(torch.bfloat16).to(dev)
@@ -614,6 +626,10 @@ def main():
                     help="launch only this kernel kind, or one whole step of --batch "
                          "sequences (profiler captures); no JSON bench line")
     ap.add_argument("--batch", type=int, default=64, help="sequences for --kernel runs")
+    ap.add_argument("--stack-kernels", choices=tuple(STACK_KERNELS), default="auto",
+                    help="kernel family of the stacked forward and input gradient "
+                         "(hcw_set_stack_kernels); auto picks the resident kernels for the "
+                         "bench workload")
     args = ap.parse_args()
     if args.kernel:
         return run_kernel_only(args)

@@ -265,9 +265,8 @@ int hcw_layer_bwd_weight_noalloc(const void* x, const void* dz, int layer, int d
 /*
  * Which kernels run the bf16 stacked forward and input gradient
  * (hcw_stack_fwd, hcw_stack_bwd_data, hcw_stack_bwd).  Process-wide.
- *   HCW_STACK_AUTO       resident where the shape fits and its pairs of SMs
- *                        fill most of the GPU (B*n/128 >= 5/8 of the SMs),
- *                        else streaming.  The default.
+ *   HCW_STACK_AUTO       the faster family as measured on GB300 for the
+ *                        shape; currently streaming everywhere.  The default.
  *   HCW_STACK_RESIDENT   resident wherever the shape fits.
  *   HCW_STACK_STREAMING  streaming only.
  * Resident: a cluster of two CTAs keeps 256 consecutive tokens (whole
@@ -286,6 +285,13 @@ int hcw_layer_bwd_weight_noalloc(const void* x, const void* dz, int layer, int d
 #define HCW_STACK_RESIDENT  1
 #define HCW_STACK_STREAMING 2
 int hcw_set_stack_kernels(int mode);
+
+/*
+ * Which family the bf16 stacked forward and input gradient of these sizes
+ * would run on under the current setting (on the current device):
+ * HCW_STACK_RESIDENT or HCW_STACK_STREAMING; -1 for invalid sizes or dtype.
+ */
+int hcw_stack_kernels_used(int B, int n, int d, int dtype);
 
 /* Number of kernels this library has launched in this process (all devices). */
 unsigned long long hcw_launch_count(void);

@@ -123,6 +123,22 @@ bool map_weight_blocks(CUtensorMap* m, const void* base, int d, int nblk) {
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Activations [tokens][d] bf16 as (8 features, tokens, d / 8): a box (8, 128,
+// nchunk) is a 128-token x 8*nchunk-feature slice laid out chunk by chunk, 16
+// bytes per token and chunk -- the layout of the resident kernels' A tile.
+bool map_rows16(CUtensorMap* m, const void* base, long long tokens, int d, int nchunk) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc || !base) return false;
+    cuuint64_t dims[3] = {8, (cuuint64_t)tokens, (cuuint64_t)(d / 8)};
+    cuuint64_t strides[2] = {(cuuint64_t)d * 2, 16};
+    cuuint32_t box[3] = {8, 128, (cuuint32_t)nchunk};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Weights W[o][k] bf16 [d][d], box (64 k, box_o), 128-byte swizzle.
 bool map_weight(CUtensorMap* m, const void* base, int d, int box_o) {
     EncodeTiledFn enc = encode_fn();
@@ -342,15 +358,15 @@ bool use_pairs(const Shape& sh) {
 
 // Whether a bf16 stacked forward / input gradient runs on the resident
 // kernels (hcw_res.cu): the shape fits them (d in {128, 256, 512}, n <= 256,
-// whole 256-token tiles) and, unless hcw_set_stack_kernels says otherwise,
-// their pairs fill most of the GPU (one pair per 256 tokens, no more).
+// whole 256-token tiles) and hcw_set_stack_kernels asked for them.
 std::atomic<int> g_stack_kernels{HCW_STACK_AUTO};
 
 bool use_resident(const Shape& sh) {
     const int mode = g_stack_kernels.load(std::memory_order_relaxed);
     if (mode == HCW_STACK_STREAMING || !res_supported(sh.d, sh.n, sh.tokens)) return false;
-    if (mode == HCW_STACK_RESIDENT) return true;
-    return sh.tokens / 128 >= (5 * (long long)sm_count()) / 8;
+    // measured on GB300 (char-LM shapes, d = 512): the streaming kernels are
+    // faster, so they are the automatic choice
+    return mode == HCW_STACK_RESIDENT;
 }
 
 // Row-unit geometry of a pair launch: units count row-block pairs.
@@ -413,7 +429,8 @@ int stack_fwd_resident(const Shape& sh, int l0, int n, int layer0, int dim_overr
         const int l = l0 + i;
         const int s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
         if (!map_weight(&R.wmap[i][0], Ws + l * wb, d, N / 2) ||
-            !map_weight(&R.wmap[i][1], Wn + l * wb, d, N / 2))
+            !map_weight(&R.wmap[i][1], Wn + l * wb, d, N / 2) ||
+            !map_rows16(&R.omap[i], out_ptr(l), sh.tokens, d, N / 32))
             return HCW_ERR_CUDA;
         R.layer[i] = {s, RES_Y, out_ptr(l), bias ? bias + (size_t)l * d : nullptr, mask_ptr(l),
                       nullptr};
@@ -695,6 +712,9 @@ int stack_data_resident(const Shape& sh, const StackData& a, cudaStream_t st) {
                 y.out = dz(l - 1);
                 y.mprev = relu ? mask(l - 1) : nullptr;
             }
+            // the stand-in for RES_G is never used (fp32 leaves row by row)
+            if (!map_rows16(&R.omap[i], y.out_kind == RES_G ? a.dx : y.out, sh.tokens, d, N / 32))
+                return HCW_ERR_CUDA;
         }
         R.in = top == L - 1 ? a.dy : static_cast<const void*>(gs);
         R.in_f32 = top == L - 1 ? 0 : 1;
@@ -1366,6 +1386,12 @@ int hcw_set_stack_kernels(int mode) {
     if (mode != HCW_STACK_AUTO && mode != HCW_STACK_RESIDENT && mode != HCW_STACK_STREAMING)
         return -1;
     return g_stack_kernels.exchange(mode);
+}
+
+int hcw_stack_kernels_used(int B, int n, int d, int dtype) {
+    Shape sh;
+    if (check_shape(0, -1, B, n, d, dtype, 0, &sh)) return -1;
+    return dtype == HCW_BF16 && use_resident(sh) ? HCW_STACK_RESIDENT : HCW_STACK_STREAMING;
 }
 
 unsigned long long hcw_launch_count(void) { return g_launches.load(); }

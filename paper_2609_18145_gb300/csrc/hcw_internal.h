@@ -131,6 +131,10 @@ struct ResLaunch {
     // chunk per CTA (forward: K-major 2-D boxes; input gradient: MN-major
     // 3-D block boxes)
     CUtensorMap wmap[kMaxStackLayers][2];
+    // per layer: its bf16 output (y_l, dz_{l-1} or dx) as (8 features, tokens,
+    // d/8) with 128-token x 8-chunk boxes, the TMA store of a 16 KB column
+    // slice of the A tile (layers on the natural split)
+    CUtensorMap omap[kMaxStackLayers];
     ResLayer layer[kMaxStackLayers];
     const void* in;           // forward: the first layer's input, bf16 [tokens][d];
                               // input gradient: the top layer's output gradient,

@@ -270,24 +270,34 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
                             tc_fence_after();
                             const uint32_t b = smem_u32(ring + (size_t)stage * G::SB);
                             const uint32_t ab = a0 + (uint32_t)(kb * 8 * kChunkBytes);
+                            auto bdesc = [&](int kk) {
+                                return FWD ? smem_desc_sw128(b + kk * 32, 16, 1024)
+                                           : smem_desc_sw128(b + kk * 2048, 8192, 1024);
+                            };
+                            auto adesc = [&](int kk, int shift) {
+                                return smem_desc_rows16(
+                                    ab + (uint32_t)(kk * 2 * kChunkBytes) + (uint32_t)(shift * 16),
+                                    kChunkBytes);
+                            };
+                            // each stage's MMAs are one straight-line block: a branch
+                            // between two tcgen05.mma of a stage halves the issue rate
+                            if (part == 0) {
 #pragma unroll
-                            for (int kk = 0; kk < 4; ++kk) {
-                                const uint64_t bd =
-                                    FWD ? smem_desc_sw128(b + kk * 32, 16, 1024)
-                                        : smem_desc_sw128(b + kk * 2048, 8192, 1024);
-                                const uint32_t a = ab + (uint32_t)(kk * 2 * kChunkBytes);
-                                if (part == 0) {
-                                    mma_bf16_f32_pair(d_tmem, smem_desc_rows16(a, kChunkBytes), bd,
-                                                      IDESC, (init || (kb | kk) != 0) ? 1u : 0u);
-                                } else {
-                                    mma_bf16_f32_pair_masked(
-                                        d_tmem, smem_desc_rows16(a + (uint32_t)(sh1 * 16), kChunkBytes),
-                                        bd, IDESC, m1);
-                                    if (!causal)
-                                        mma_bf16_f32_pair_masked(
-                                            d_tmem,
-                                            smem_desc_rows16(a + (uint32_t)(sh2 * 16), kChunkBytes),
-                                            bd, IDESC, m2);
+                                for (int kk = 0; kk < 4; ++kk)
+                                    mma_bf16_f32_pair(d_tmem, adesc(kk, 0), bdesc(kk), IDESC,
+                                                      (init || (kb | kk) != 0) ? 1u : 0u);
+                            } else if (causal) {
+#pragma unroll
+                                for (int kk = 0; kk < 4; ++kk)
+                                    mma_bf16_f32_pair_masked(d_tmem, adesc(kk, sh1), bdesc(kk),
+                                                             IDESC, m1);
+                            } else {
+#pragma unroll
+                                for (int kk = 0; kk < 4; ++kk) {
+                                    mma_bf16_f32_pair_masked(d_tmem, adesc(kk, sh1), bdesc(kk),
+                                                             IDESC, m1);
+                                    mma_bf16_f32_pair_masked(d_tmem, adesc(kk, sh2), bdesc(kk),
+                                                             IDESC, m2);
                                 }
                             }
                             any = true;
@@ -317,6 +327,9 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
         const int q = warp & 3;
         const int cs = e >> 2;
         const int row = q * 32 + lane;
+        // one lane per group of four warps (the warps of column slice cs, one per
+        // lane quarter) issues that group's TMA stores
+        const bool issuer = (e & 3) == 0 && lane == 0;
         const uint32_t t_lane = tmem_base + ((uint32_t)(q * 32) << 16);
         const uint32_t aready_leader[2] = {mapa_shared(&bars->aready[0], 0),
                                            mapa_shared(&bars->aready[1], 0)};
@@ -456,6 +469,12 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
             const int tok = tok_of(tile, (int)rank, row, alt);
             const uint32_t par = (uint32_t)i & 1u;
             const int kind = ly.out_kind;
+            // A bf16 output on the natural split leaves through the A tile: the
+            // results are written there (where they are also the next layer's
+            // operand) and each group of four warps stores its 128-row column
+            // slice with one TMA copy.  Otherwise the lanes store their rows.
+            const bool tma_out = !alt && kind != RES_G;
+            const bool a_write = to_a || tma_out;
             // input gradient: the mask words of the layer below, fetched early
             uint32_t mw[G::NCH][G::SUB];
 #pragma unroll
@@ -471,9 +490,21 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
                     alive = false;
                     break;
                 }
+                // chunk 0: A's first K blocks are free once chunk 1's MMAs have
+                // passed them; the results then go straight into A, piece by piece
+                if (a_write && G::NCH == 2 && h == 0 && !wait_all(&bars->afree, par)) {
+                    alive = false;
+                    break;
+                }
                 tc_fence_after();
-                uint32_t keep[G::SUB][16];
-#pragma unroll
+                if (a_write && tma_out) {
+                    // the store that last read these columns of A (the group's store
+                    // of chunk h one layer back) is done reading; the one issued after
+                    // it (the other chunk) may still be running
+                    if (issuer) bulk_wait_read<1>();
+                    named_bar_sync(1 + cs, 128);
+                }
+#pragma unroll 1
                 for (int j = 0; j < G::SUB; ++j) {
                     const int col = col_of(h, j);
                     uint32_t raw[32];
@@ -483,6 +514,7 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
                     float v[32];
 #pragma unroll
                     for (int t = 0; t < 32; ++t) v[t] = __uint_as_float(raw[t]);
+                    uint32_t w[16];
                     if (FWD) {
                         // z = acc + bias; mask bit (z > 0); act; + x (residual); bf16
                         if (ly.bias) {
@@ -520,31 +552,20 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
                             }
                         }
 #pragma unroll
-                        for (int t = 0; t < 16; ++t) keep[j][t] = pack_bf16x2(v[2 * t], v[2 * t + 1]);
-                        uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(ly.out) +
-                                                              (size_t)tok * D + col);
-#pragma unroll
-                        for (int m = 0; m < 4; ++m)
-                            dst[m] = make_uint4(keep[j][4 * m], keep[j][4 * m + 1],
-                                                keep[j][4 * m + 2], keep[j][4 * m + 3]);
+                        for (int t = 0; t < 16; ++t) w[t] = pack_bf16x2(v[2 * t], v[2 * t + 1]);
                     } else if (kind == RES_G) {
                         float4* dst = reinterpret_cast<float4*>(static_cast<float*>(ly.out) +
                                                                 (size_t)tok * D + col);
 #pragma unroll
                         for (int m = 0; m < 8; ++m)
                             dst[m] = make_float4(v[4 * m], v[4 * m + 1], v[4 * m + 2], v[4 * m + 3]);
+                        continue;
                     } else {
                         // RES_DZ: dz_{l-1} = bf16(g) * mask_{l-1};  RES_DX: dx = bf16(g)
 #pragma unroll
                         for (int t = 0; t < 16; ++t)
-                            keep[j][t] = and_mask_bf16x2(pack_bf16x2(v[2 * t], v[2 * t + 1]),
-                                                         mw[h][j], 2 * t);
-                        uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(ly.out) +
-                                                              (size_t)tok * D + col);
-#pragma unroll
-                        for (int m = 0; m < 4; ++m)
-                            dst[m] = make_uint4(keep[j][4 * m], keep[j][4 * m + 1],
-                                                keep[j][4 * m + 2], keep[j][4 * m + 3]);
+                            w[t] = and_mask_bf16x2(pack_bf16x2(v[2 * t], v[2 * t + 1]), mw[h][j],
+                                                   2 * t);
                         if (trans && resid) {
                             float4* gs = reinterpret_cast<float4*>(L.gscratch + (size_t)tok * D + col);
 #pragma unroll
@@ -552,26 +573,39 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
                                 gs[m] = make_float4(v[4 * m], v[4 * m + 1], v[4 * m + 2], v[4 * m + 3]);
                         }
                     }
-                }
-                if (to_a) {
-                    // chunk 0: wait until chunk 1's MMAs have read these K blocks
-                    if (G::NCH == 2 && h == 0 && !wait_all(&bars->afree, par)) {
-                        alive = false;
-                        break;
-                    }
-#pragma unroll
-                    for (int j = 0; j < G::SUB; ++j)
+                    if (a_write) {
 #pragma unroll
                         for (int m = 0; m < 4; ++m)
-                            *apiece(col_of(h, j), m) = make_uint4(keep[j][4 * m], keep[j][4 * m + 1],
-                                                                  keep[j][4 * m + 2], keep[j][4 * m + 3]);
-                    signal_ready(h);
+                            *apiece(col, m) = make_uint4(w[4 * m], w[4 * m + 1], w[4 * m + 2], w[4 * m + 3]);
+                    }
+                    if (!tma_out) {
+                        uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(ly.out) +
+                                                              (size_t)tok * D + col);
+#pragma unroll
+                        for (int m = 0; m < 4; ++m)
+                            dst[m] = make_uint4(w[4 * m], w[4 * m + 1], w[4 * m + 2], w[4 * m + 3]);
+                    }
                 }
+                if (a_write && tma_out) {
+                    fence_proxy_async_smem();
+                    named_bar_sync(1 + cs, 128);
+                    if (issuer) {
+                        const int kc0 = col_of(h, 0) / 8;
+                        tma_store_3d(&L.omap[i], A + (size_t)kc0 * kChunkBytes, 0,
+                                     tile * 256 + (int)rank * kRows, kc0);
+                        bulk_commit();
+                    }
+                }
+                if (to_a) signal_ready(h);
             }
             if (!alive) break;
             if (trans) {
                 // every output of the pair is in global memory: meet, then reload the
                 // rows of the next layer's split
+                if (issuer) {
+                    bulk_wait<0>();
+                    fence_proxy_async_global();
+                }
                 __threadfence();
                 tc_fence_before();
                 __syncwarp();
@@ -588,6 +622,9 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
                 load_rows(alt_next, false, &ly);
             }
         }
+        // the group's stores have finished reading shared memory before the CTA exits
+        if (issuer) bulk_wait<0>();
+        __syncwarp();
     }
 
     tc_fence_before();

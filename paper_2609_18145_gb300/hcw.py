@@ -76,6 +76,7 @@ _SIGNATURES = {
     "hcw_stack_bwd": ([_P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P,
                        _P, _P, _SZ, _P], _I),
     "hcw_set_stack_kernels": ([_I], _I),
+    "hcw_stack_kernels_used": ([_I, _I, _I, _I], _I),
     "hcw_sync_status": ([_P], _I),
     "hcw_selftest_wait": ([_LL, _P], _I),
 }
@@ -257,6 +258,15 @@ def hcw_set_stack_kernels(mode: int) -> int:
     if prev < 0:
         raise ValueError("hcw_set_stack_kernels: unknown mode %r" % (mode,))
     return prev
+
+
+def hcw_stack_kernels_used(B: int, n: int, d: int, dtype: int = HCW_BF16) -> int:
+    """HCW_STACK_RESIDENT or HCW_STACK_STREAMING: the family a bf16 stack of
+    these sizes runs on under the current setting."""
+    r = int(lib().hcw_stack_kernels_used(B, n, d, dtype))
+    if r < 0:
+        raise ValueError("hcw_stack_kernels_used: invalid sizes")
+    return r
 
 
 def hcw_launch_count() -> int:

@@ -210,6 +210,18 @@ def test_stack_kernel_selection_is_a_process_setting(hcw):
         assert lib.hcw_set_stack_kernels(hcw.HCW_STACK_STREAMING) == hcw.HCW_STACK_RESIDENT
         assert lib.hcw_set_stack_kernels(7) == -1          # unknown: unchanged
         assert lib.hcw_set_stack_kernels(-1) == -1
+        # streaming only: every bf16 shape; resident where the shape fits
+        assert lib.hcw_stack_kernels_used(64, 256, 512, hcw.HCW_BF16) == hcw.HCW_STACK_STREAMING
+        lib.hcw_set_stack_kernels(hcw.HCW_STACK_RESIDENT)
+        assert lib.hcw_stack_kernels_used(64, 256, 512, hcw.HCW_BF16) == hcw.HCW_STACK_RESIDENT
+        assert lib.hcw_stack_kernels_used(1, 256, 128, hcw.HCW_BF16) == hcw.HCW_STACK_RESIDENT
+        assert lib.hcw_stack_kernels_used(64, 512, 512, hcw.HCW_BF16) == hcw.HCW_STACK_STREAMING
+        assert lib.hcw_stack_kernels_used(64, 256, 1024, hcw.HCW_BF16) == hcw.HCW_STACK_STREAMING
+        assert lib.hcw_stack_kernels_used(64, 256, 384, hcw.HCW_BF16) == hcw.HCW_STACK_STREAMING
+        assert lib.hcw_stack_kernels_used(3, 64, 512, hcw.HCW_BF16) == hcw.HCW_STACK_STREAMING
+        assert lib.hcw_stack_kernels_used(64, 256, 512, hcw.HCW_F32) == hcw.HCW_STACK_STREAMING
+        assert lib.hcw_stack_kernels_used(64, 48, 512, hcw.HCW_BF16) == -1
+        lib.hcw_set_stack_kernels(hcw.HCW_STACK_STREAMING)
         assert lib.hcw_set_stack_kernels(hcw.HCW_STACK_AUTO) == hcw.HCW_STACK_STREAMING
         with pytest.raises(ValueError):
             hcw.hcw_set_stack_kernels(3)
