@@ -276,9 +276,11 @@ int hcw_layer_bwd_weight_noalloc(const void* x, const void* dz, int layer, int d
  * partner product costs 4d^2 flops per token there (every lane computed, half
  * kept) instead of 3d^2.
  * Streaming: every layer's tiles pass through global memory (L2); any shape.
- * The resident input gradient keeps the residual stream g in fp32 between
- * layers, where the streaming kernels round it to bf16 at every layer, so the
- * two differ at bf16 rounding level.
+ * The two families add the products in different orders (resident: the self
+ * and partner products K block by K block; streaming: the self part first),
+ * and the resident input gradient keeps the residual stream g in fp32 between
+ * layers where the streaming kernels round it to bf16 at every layer: their
+ * results differ at bf16 rounding level.
  * Returns the previous mode, or -1 (mode unchanged) for an unknown mode.
  */
 #define HCW_STACK_AUTO      0

@@ -123,15 +123,17 @@ bool map_weight_blocks(CUtensorMap* m, const void* base, int d, int nblk) {
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// Activations [tokens][d] bf16 as (8 features, tokens, d / 8): a box (8, 128,
-// nchunk) is a 128-token x 8*nchunk-feature slice laid out chunk by chunk, 16
-// bytes per token and chunk -- the layout of the resident kernels' A tile.
-bool map_rows16(CUtensorMap* m, const void* base, long long tokens, int d, int nchunk) {
+// Activations [tokens][d] bf16 as (8 features, tokens, d / 8): a box (8,
+// box_tokens, nchunk) is a box_tokens x 8*nchunk-feature slice laid out chunk
+// by chunk, 16 bytes per token and chunk -- the layout of the resident
+// kernels' A tile.
+bool map_rows16(CUtensorMap* m, const void* base, long long tokens, int d, int nchunk,
+                int box_tokens) {
     EncodeTiledFn enc = encode_fn();
     if (!enc || !base) return false;
     cuuint64_t dims[3] = {8, (cuuint64_t)tokens, (cuuint64_t)(d / 8)};
     cuuint64_t strides[2] = {(cuuint64_t)d * 2, 16};
-    cuuint32_t box[3] = {8, 128, (cuuint32_t)nchunk};
+    cuuint32_t box[3] = {8, (cuuint32_t)box_tokens, (cuuint32_t)nchunk};
     cuuint32_t estr[3] = {1, 1, 1};
     return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
                box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
@@ -430,7 +432,7 @@ int stack_fwd_resident(const Shape& sh, int l0, int n, int layer0, int dim_overr
         const int s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
         if (!map_weight(&R.wmap[i][0], Ws + l * wb, d, N / 2) ||
             !map_weight(&R.wmap[i][1], Wn + l * wb, d, N / 2) ||
-            !map_rows16(&R.omap[i], out_ptr(l), sh.tokens, d, N / 32))
+            !map_rows16(&R.imap[i], out_ptr(l), sh.tokens, d, 1, 64))
             return HCW_ERR_CUDA;
         R.layer[i] = {s, RES_Y, out_ptr(l), bias ? bias + (size_t)l * d : nullptr, mask_ptr(l),
                       nullptr};
@@ -713,7 +715,8 @@ int stack_data_resident(const Shape& sh, const StackData& a, cudaStream_t st) {
                 y.mprev = relu ? mask(l - 1) : nullptr;
             }
             // the stand-in for RES_G is never used (fp32 leaves row by row)
-            if (!map_rows16(&R.omap[i], y.out_kind == RES_G ? a.dx : y.out, sh.tokens, d, N / 32))
+            const void* ob = y.out_kind == RES_G ? a.dx : y.out;
+            if (!map_rows16(&R.imap[i], ob, sh.tokens, d, 1, 64))
                 return HCW_ERR_CUDA;
         }
         R.in = top == L - 1 ? a.dy : static_cast<const void*>(gs);

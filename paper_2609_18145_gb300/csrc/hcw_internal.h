@@ -132,9 +132,9 @@ struct ResLaunch {
     // 3-D block boxes)
     CUtensorMap wmap[kMaxStackLayers][2];
     // per layer: its bf16 output (y_l, dz_{l-1} or dx) as (8 features, tokens,
-    // d/8) with 128-token x 8-chunk boxes, the TMA store of a 16 KB column
-    // slice of the A tile (layers on the natural split)
-    CUtensorMap omap[kMaxStackLayers];
+    // d/8) with 64-token x 1-chunk boxes: where the rows change CTA (n = 256),
+    // the next layer's A tile is reloaded from it chunk by chunk
+    CUtensorMap imap[kMaxStackLayers];
     ResLayer layer[kMaxStackLayers];
     const void* in;           // forward: the first layer's input, bf16 [tokens][d];
                               // input gradient: the top layer's output gradient,

@@ -33,7 +33,7 @@
 // partners again share a CTA, at lane distance 64.  Between layers of
 // different splits the rows go through global memory once, since the layer's
 // output is stored there anyway: both CTAs meet on a barrier, then reload
-// their new rows.
+// their new rows with TMA (64-token boxes, one 16-byte column chunk each).
 //
 // Input gradient.  This is the mirror image: a row gathers dz from its
 // partner when the partner received from it.  The residual stream g (the
@@ -44,12 +44,13 @@
 // layer's MMAs.  (The streaming kernels round g to bf16 at every layer; here
 // it is rounded only where it leaves the chip.)
 //
-// Overlap.  For d >= 256 the N columns form two accumulators ("chunks").  The
-// epilogue of chunk 0 runs during chunk 1's MMAs.  It writes its columns into
-// the A tile as soon as those MMAs have read the matching K blocks: the MMA
-// thread commits once chunk 1's partner part has passed the middle K block.
-// The next layer's chunk-0 self part then starts on those blocks while chunk
-// 1's epilogue runs.
+// Overlap.  For d >= 256 the N columns form two accumulators ("chunks"), each
+// accumulated K block by K block (self product, then partner product of the
+// block).  The epilogue of chunk 0 runs during chunk 1's MMAs and writes its
+// columns into the A tile once those MMAs have passed the matching K blocks
+// (the MMA thread commits when chunk 1 reaches the middle block).  The next
+// layer's chunk 0 then runs its first half of the K blocks while chunk 1's
+// epilogue runs.
 //
 // Roles (576 threads).
 //   - Warp 0, lane 0: issues the TMA weight loads into a ring.  Both CTAs do
@@ -86,7 +87,9 @@ struct Geo {
     static constexpr int NK = D / 64;                   // 64-deep K blocks per part
     static constexpr int A_BYTES = (D / 8) * kChunkBytes;
     static constexpr int SB = (N / 2) * 64 * 2;         // one B stage (this CTA's half)
-    static constexpr int FIXED = 1024 /* alignment */ + A_BYTES + kGuard + 256 /* barriers */;
+    static constexpr int BIAS_BYTES = 2 * D * 4;            // two layers' bias (forward)
+    static constexpr int FIXED = 1024 /* alignment */ + A_BYTES + kGuard + BIAS_BYTES +
+                                 256 /* barriers */;
     static constexpr int ST_RAW = (kSmemMax - FIXED) / SB;
     static constexpr int STAGES = ST_RAW > 8 ? 8 : ST_RAW;
     static constexpr size_t SMEM = (size_t)FIXED + (size_t)STAGES * SB;
@@ -104,6 +107,7 @@ struct __align__(8) ResBars {
     uint64_t afree;        // chunk 1's MMAs have read the first half of the K blocks
     uint64_t aready[2];    // leader: both CTAs' A columns of chunk h written (2 x kEW arrivals)
     uint64_t xsync;        // both CTAs' outputs of a layer are in global memory
+    uint64_t xload;        // the A tile of the next split has landed (TMA)
     uint64_t drain;
     uint32_t tmem_base;
     int abort;
@@ -151,7 +155,8 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     uint8_t* ring = smem;
     uint8_t* A = smem + (size_t)G::STAGES * G::SB;
-    ResBars* bars = reinterpret_cast<ResBars*>(A + G::A_BYTES + kGuard);
+    float* bias_s = reinterpret_cast<float*>(A + G::A_BYTES + kGuard);   // [2][D]
+    ResBars* bars = reinterpret_cast<ResBars*>(A + G::A_BYTES + kGuard + G::BIAS_BYTES);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -176,6 +181,7 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
         mbar_init(&bars->aready[0], 2 * kEW);
         mbar_init(&bars->aready[1], 2 * kEW);
         mbar_init(&bars->xsync, 2 * kEW);
+        mbar_init(&bars->xload, 1);
         mbar_init(&bars->drain, 1);
         bars->abort = 0;
         fence_mbar_init();
@@ -200,10 +206,10 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
             bool ok = true;
             for (int i = 0; i < L.n_layers && ok; ++i)
                 for (int h = 0; h < G::NCH && ok; ++h)
-                    for (int part = 0; part < 2 && ok; ++part) {
-                        const CUtensorMap* m = &L.wmap[i][part];
+                    for (int kb = 0; kb < G::NK && ok; ++kb) {
                         const int col = h * G::N + (int)rank * (G::N / 2);
-                        for (int kb = 0; kb < G::NK; ++kb) {
+                        for (int part = 0; part < 2; ++part) {
+                            const CUtensorMap* m = &L.wmap[i][part];
                             if (!mbar_wait(&bars->empty[stage], phase ^ 1, abort, tmo)) {
                                 ok = false;
                                 break;
@@ -253,8 +259,8 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
                 const uint32_t par = (uint32_t)i & 1u;
                 for (int h = 0; h < G::NCH && ok; ++h) {
                     const uint32_t d_tmem = tmem_base + (uint32_t)(h * G::N);
-                    for (int part = 0; part < 2 && ok; ++part)
-                        for (int kb = 0; kb < G::NK; ++kb) {
+                    for (int kb = 0; kb < G::NK && ok; ++kb)
+                        for (int part = 0; part < 2; ++part) {
                             if (h == 0 && part == 0 && (kb == 0 || (G::NCH == 2 && kb == G::NK / 2))) {
                                 if (!mbar_wait_cluster(&bars->aready[kb == 0 ? 0 : 1], par, abort,
                                                        tmo)) {
@@ -327,15 +333,13 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
         const int q = warp & 3;
         const int cs = e >> 2;
         const int row = q * 32 + lane;
-        // one lane per group of four warps (the warps of column slice cs, one per
-        // lane quarter) issues that group's TMA stores
-        const bool issuer = (e & 3) == 0 && lane == 0;
+        const int gw = e & 3;   // this warp within its group (the 4 warps of column slice cs)
         const uint32_t t_lane = tmem_base + ((uint32_t)(q * 32) << 16);
         const uint32_t aready_leader[2] = {mapa_shared(&bars->aready[0], 0),
                                            mapa_shared(&bars->aready[1], 0)};
         const uint32_t xs_own = mapa_shared(&bars->xsync, rank);
         const uint32_t xs_peer = mapa_shared(&bars->xsync, rank ^ 1u);
-        uint32_t xs_phase = 0;
+        uint32_t xs_phase = 0, xl_phase = 0;
         bool alive = true;
 
         auto col_of = [&](int h, int j) { return h * G::N + cs * G::WC + j * 32; };
@@ -358,9 +362,9 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
             __syncwarp();
             if (lane == 0) mbar_arrive_remote(aready_leader[h]);
         };
-        // rows of the split `alt` into A (and, input gradient with the residual,
-        // g into TMEM) from global memory.  first: the launch's input.
-        auto load_rows = [&](bool alt, bool first, const ResLayer* src_layer) {
+        // The launch's input rows of the split `alt` into A (and, input gradient
+        // with the residual, g into TMEM).
+        auto load_input = [&](bool alt) {
             const int tok = tok_of(tile, (int)rank, row, alt);
 #pragma unroll 1
             for (int h = 0; h < G::NCH; ++h)
@@ -369,14 +373,13 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
                     const int col = col_of(h, j);
                     if (FWD) {
                         const uint4* src = reinterpret_cast<const uint4*>(
-                            static_cast<const __nv_bfloat16*>(first ? L.in : src_layer->out) +
-                            (size_t)tok * D + col);
+                            static_cast<const __nv_bfloat16*>(L.in) + (size_t)tok * D + col);
                         uint4 v[4];
 #pragma unroll
-                        for (int m = 0; m < 4; ++m) v[m] = first ? __ldg(src + m) : __ldcg(src + m);
+                        for (int m = 0; m < 4; ++m) v[m] = __ldg(src + m);
 #pragma unroll
                         for (int m = 0; m < 4; ++m) *apiece(col, m) = v[m];
-                    } else if (first) {
+                    } else {
                         // g = the top layer's output gradient; dz = bf16(g) * mask
                         uint32_t g[32];
                         if (L.in_f32) {
@@ -426,30 +429,6 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
                             dst[m] = v;
                             *apiece(col, m) = v;
                         }
-                    } else {
-                        // after a change of split: dz_{l-1} (stored by the layer) and g
-                        const uint4* src = reinterpret_cast<const uint4*>(
-                            static_cast<const __nv_bfloat16*>(src_layer->out) + (size_t)tok * D + col);
-                        uint4 v[4];
-#pragma unroll
-                        for (int m = 0; m < 4; ++m) v[m] = __ldcg(src + m);
-#pragma unroll
-                        for (int m = 0; m < 4; ++m) *apiece(col, m) = v[m];
-                        if (resid) {
-                            const float4* gs =
-                                reinterpret_cast<const float4*>(L.gscratch + (size_t)tok * D + col);
-                            uint32_t g[32];
-#pragma unroll
-                            for (int m = 0; m < 8; ++m) {
-                                const float4 f = __ldcg(gs + m);
-                                g[4 * m] = __float_as_uint(f.x);
-                                g[4 * m + 1] = __float_as_uint(f.y);
-                                g[4 * m + 2] = __float_as_uint(f.z);
-                                g[4 * m + 3] = __float_as_uint(f.w);
-                            }
-                            __syncwarp();
-                            tmem_st_32x32b_x32(t_lane + (uint32_t)col, g);
-                        }
                     }
                 }
             if (!FWD && resid) tmem_st_wait();
@@ -457,7 +436,7 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
             if (G::NCH == 2) signal_ready(1);
         };
 
-        load_rows(alt_split(L.layer[0].s, L.n), true, nullptr);
+        load_input(alt_split(L.layer[0].s, L.n));
 
         for (int i = 0; i < L.n_layers && alive; ++i) {
             const ResLayer& ly = L.layer[i];
@@ -469,12 +448,6 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
             const int tok = tok_of(tile, (int)rank, row, alt);
             const uint32_t par = (uint32_t)i & 1u;
             const int kind = ly.out_kind;
-            // A bf16 output on the natural split leaves through the A tile: the
-            // results are written there (where they are also the next layer's
-            // operand) and each group of four warps stores its 128-row column
-            // slice with one TMA copy.  Otherwise the lanes store their rows.
-            const bool tma_out = !alt && kind != RES_G;
-            const bool a_write = to_a || tma_out;
             // input gradient: the mask words of the layer below, fetched early
             uint32_t mw[G::NCH][G::SUB];
 #pragma unroll
@@ -484,26 +457,27 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
                     mw[h][j] = (!FWD && kind == RES_DZ && ly.mprev)
                                    ? __ldg(ly.mprev + (size_t)tok * WPR + col_of(h, j) / 32)
                                    : ~0u;
+            // forward: this layer's bias into shared memory (buffer i & 1, last read
+            // two layers back), one value a thread, visible after the barrier below
+            float* bias_l = bias_s + (i & 1) * D;
+            if (FWD) {
+                const int t = e * 32 + lane;
+                if (t < D) bias_l[t] = ly.bias ? __ldg(ly.bias + t) : 0.f;
+                named_bar_sync(5, 32 * kEW);
+            }
 #pragma unroll 1
             for (int h = 0; h < G::NCH; ++h) {
                 if (!wait_all(&bars->tfull[h], par)) {
                     alive = false;
                     break;
                 }
-                // chunk 0: A's first K blocks are free once chunk 1's MMAs have
-                // passed them; the results then go straight into A, piece by piece
-                if (a_write && G::NCH == 2 && h == 0 && !wait_all(&bars->afree, par)) {
+                // chunk 0: A's first K blocks are free once chunk 1's MMAs have passed
+                // them (the results go to A: as the next operand and to be stored)
+                if (kind != RES_G && G::NCH == 2 && h == 0 && !wait_all(&bars->afree, par)) {
                     alive = false;
                     break;
                 }
                 tc_fence_after();
-                if (a_write && tma_out) {
-                    // the store that last read these columns of A (the group's store
-                    // of chunk h one layer back) is done reading; the one issued after
-                    // it (the other chunk) may still be running
-                    if (issuer) bulk_wait_read<1>();
-                    named_bar_sync(1 + cs, 128);
-                }
 #pragma unroll 1
                 for (int j = 0; j < G::SUB; ++j) {
                     const int col = col_of(h, j);
@@ -517,16 +491,14 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
                     uint32_t w[16];
                     if (FWD) {
                         // z = acc + bias; mask bit (z > 0); act; + x (residual); bf16
-                        if (ly.bias) {
-                            const float4* b4 = reinterpret_cast<const float4*>(ly.bias + col);
+                        const float4* b4 = reinterpret_cast<const float4*>(bias_l + col);
 #pragma unroll
-                            for (int m = 0; m < 8; ++m) {
-                                const float4 bb = __ldg(b4 + m);
-                                v[4 * m] += bb.x;
-                                v[4 * m + 1] += bb.y;
-                                v[4 * m + 2] += bb.z;
-                                v[4 * m + 3] += bb.w;
-                            }
+                        for (int m = 0; m < 8; ++m) {
+                            const float4 bb = b4[m];
+                            v[4 * m] += bb.x;
+                            v[4 * m + 1] += bb.y;
+                            v[4 * m + 2] += bb.z;
+                            v[4 * m + 3] += bb.w;
                         }
                         if (ly.mout) {
                             uint32_t bits = 0;
@@ -573,40 +545,39 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
                                 gs[m] = make_float4(v[4 * m], v[4 * m + 1], v[4 * m + 2], v[4 * m + 3]);
                         }
                     }
-                    if (a_write) {
 #pragma unroll
-                        for (int m = 0; m < 4; ++m)
-                            *apiece(col, m) = make_uint4(w[4 * m], w[4 * m + 1], w[4 * m + 2], w[4 * m + 3]);
-                    }
-                    if (!tma_out) {
-                        uint4* dst = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(ly.out) +
-                                                              (size_t)tok * D + col);
-#pragma unroll
-                        for (int m = 0; m < 4; ++m)
-                            dst[m] = make_uint4(w[4 * m], w[4 * m + 1], w[4 * m + 2], w[4 * m + 3]);
-                    }
+                    for (int m = 0; m < 4; ++m)
+                        *apiece(col, m) = make_uint4(w[4 * m], w[4 * m + 1], w[4 * m + 2], w[4 * m + 3]);
                 }
-                if (a_write && tma_out) {
-                    fence_proxy_async_smem();
-                    named_bar_sync(1 + cs, 128);
-                    if (issuer) {
-                        const int kc0 = col_of(h, 0) / 8;
-                        tma_store_3d(&L.omap[i], A + (size_t)kc0 * kChunkBytes, 0,
-                                     tile * 256 + (int)rank * kRows, kc0);
-                        bulk_commit();
-                    }
-                }
+                if (kind == RES_G) continue;
                 if (to_a) signal_ready(h);
+                // The group's 128 rows x WC columns are in A: store them to global
+                // memory with row-contiguous pieces (lane = 8 rows x 4 chunks: per row
+                // 64 contiguous bytes, per chunk 128 contiguous bytes of A).
+                named_bar_sync(1 + cs, 128);
+                {
+                    constexpr int KCW = G::WC / 8;                   // chunks of the slice
+                    constexpr int PIECES = kRows * KCW;              // 16-byte pieces
+                    const int kc_base = col_of(h, 0) / 8;
+                    __nv_bfloat16* ob = static_cast<__nv_bfloat16*>(ly.out);
+#pragma unroll
+                    for (int it = 0; it < PIECES / 128; ++it) {
+                        const int blk = it * 4 + gw;                 // 32 pieces of this warp
+                        const int r = (blk % (kRows / 8)) * 8 + (lane & 7);
+                        const int kc = (blk / (kRows / 8)) * 4 + (lane >> 3);
+                        const uint4 v4 = *reinterpret_cast<const uint4*>(
+                            A + (size_t)(kc_base + kc) * kChunkBytes + r * 16);
+                        const int tr = tok_of(tile, (int)rank, r, alt);
+                        *reinterpret_cast<uint4*>(ob + (size_t)tr * D + (kc_base + kc) * 8) = v4;
+                    }
+                }
             }
             if (!alive) break;
             if (trans) {
                 // every output of the pair is in global memory: meet, then reload the
                 // rows of the next layer's split
-                if (issuer) {
-                    bulk_wait<0>();
-                    fence_proxy_async_global();
-                }
                 __threadfence();
+                fence_proxy_async_global();
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0) {
@@ -619,12 +590,51 @@ __global__ void __launch_bounds__(kThreads, 1) hcw_res_kernel(const __grid_const
                 }
                 xs_phase ^= 1u;
                 tc_fence_after();
-                load_rows(alt_next, false, &ly);
+                // the next split's rows: 64-token boxes of one 16-byte chunk each, all
+                // completing on xload (one lane issues them)
+                if (warp == 2 && lane == 0) {
+                    mbar_arrive_expect_tx(&bars->xload, (uint32_t)G::A_BYTES);
+                    for (int kc = 0; kc < D / 8; ++kc)
+                        for (int half = 0; half < 2; ++half) {
+                            const int t0 = alt_next ? tile * 256 + half * 128 + (int)rank * 64
+                                                    : tile * 256 + (int)rank * kRows + half * 64;
+                            tma_load_3d(A + (size_t)kc * kChunkBytes + half * 1024, &L.imap[i],
+                                        &bars->xload, 0, t0, kc);
+                        }
+                }
+                if (!FWD && resid) {
+                    // g of the rows this lane now holds, into TMEM
+                    const int tok2 = tok_of(tile, (int)rank, row, alt_next);
+#pragma unroll 1
+                    for (int h = 0; h < G::NCH; ++h)
+#pragma unroll 1
+                        for (int j = 0; j < G::SUB; ++j) {
+                            const int col = col_of(h, j);
+                            const float4* gs =
+                                reinterpret_cast<const float4*>(L.gscratch + (size_t)tok2 * D + col);
+                            uint32_t g[32];
+#pragma unroll
+                            for (int m = 0; m < 8; ++m) {
+                                const float4 f = __ldcg(gs + m);
+                                g[4 * m] = __float_as_uint(f.x);
+                                g[4 * m + 1] = __float_as_uint(f.y);
+                                g[4 * m + 2] = __float_as_uint(f.z);
+                                g[4 * m + 3] = __float_as_uint(f.w);
+                            }
+                            __syncwarp();
+                            tmem_st_32x32b_x32(t_lane + (uint32_t)col, g);
+                        }
+                    tmem_st_wait();
+                }
+                if (!wait_all(&bars->xload, xl_phase)) {
+                    alive = false;
+                    break;
+                }
+                xl_phase ^= 1u;
+                signal_ready(0);
+                if (G::NCH == 2) signal_ready(1);
             }
         }
-        // the group's stores have finished reading shared memory before the CTA exits
-        if (issuer) bulk_wait<0>();
-        __syncwarp();
     }
 
     tc_fence_before();

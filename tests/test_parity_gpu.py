@@ -296,11 +296,12 @@ def test_resident_stack_forward_backward(H, resident, case):
 @pytest.mark.parametrize("flags", [CAUSAL | RESIDUAL | RELU, RESIDUAL, CAUSAL])
 def test_resident_and_streaming_stacks_agree(H, flags):
     """The same stack on both kernel families.  Forward: the resident kernel
-    issues the same MMAs in the same K order (self part, then partner part)
-    and the same epilogue arithmetic, so y, the saved activations and the ReLU
-    masks are identical.  Input gradient: the resident kernel keeps the
-    residual stream in fp32 between layers (the streaming one rounds it to
-    bf16 at each), so dx and the weight gradients agree to bf16 rounding."""
+    sums the self and partner products K block by K block (the streaming one
+    sums the self part first), so y and the saved activations agree to bf16
+    rounding and only pre-activations within rounding of 0 may take the other
+    ReLU decision.  Input gradient: the resident kernel keeps the residual
+    stream in fp32 between layers (the streaming one rounds it to bf16 at
+    each), so dx and the weight gradients agree to bf16 rounding."""
     B, n, d, L = 4, 256, 512, 9
     pr = synth.problem(B, n, d, L=L, seed=17, w_std=(1 / (2 * d)) ** 0.5)
     x, _ = dev(pr.x, torch.bfloat16)
@@ -309,20 +310,27 @@ def test_resident_and_streaming_stacks_agree(H, flags):
     dy, _ = dev(pr.dy, torch.bfloat16)
     bias = torch.from_numpy(pr.bias).cuda()
     out = {}
+    saved = None
     for mode in (H.HCW_STACK_STREAMING, H.HCW_STACK_RESIDENT):
         prev = H.hcw_set_stack_kernels(mode)
         try:
             y, acts, masks = H.hcw_stack_fwd(x, Ws, Wn, bias, 2, -1, flags)
-            res = H.hcw_stack_bwd(x, acts, masks, dy, Ws, Wn, 2, -1, flags)
+            # both backwards run on the streaming forward's saved state (same ReLU
+            # decisions)
+            saved = saved or (acts, masks)
+            res = H.hcw_stack_bwd(x, saved[0], saved[1], dy, Ws, Wn, 2, -1, flags)
             torch.cuda.synchronize()
             assert H.hcw_sync_status() == H.HCW_OK
         finally:
             H.hcw_set_stack_kernels(prev)
         out[mode] = (y, acts, masks) + tuple(res)
     a, b = out[H.HCW_STACK_STREAMING], out[H.HCW_STACK_RESIDENT]
-    assert torch.equal(a[0], b[0]) and torch.equal(a[1], b[1])
+    assert rel(host(b[0]), host(a[0])) <= 1e-2 and rel(host(b[1]), host(a[1])) <= 1e-2
     if flags & RELU:
-        assert torch.equal(a[2], b[2])
+        differ = torch.bitwise_xor(a[2], b[2])
+        flipped = int(sum(bin(int(w) & 0xFFFFFFFF).count("1") for w in differ.flatten().cpu()
+                          if int(w) != 0))
+        assert flipped <= 1e-3 * a[2].numel() * 32, flipped
     for i, what in ((3, "dx"), (4, "dW_self"), (5, "dW_nbr"), (6, "dbias")):
         assert rel(host(b[i]), host(a[i])) <= 1e-2, what
 
