@@ -177,6 +177,21 @@ int hcw_stack_fwd(const void* x, const void* W_self, const void* W_nbr, const fl
                   unsigned flags, void* y, void* acts, void* masks, void* workspace,
                   size_t ws_bytes, void* stream);
 
+/*
+ * hcw_stack_fwd with an explicit schedule (Sec. 3.3 "Schedules", and the
+ * variants of Sec. 4, "Order does not matter; coverage does": a random
+ * permutation of the dimensions, a Gray-code order): stack layer l uses cube
+ * dimension dims[l] instead of (layer0 + l) mod log2 n.
+ *   dims   host array of L ints, each in [0, log2 n), read during the call
+ *          (HCW_ERR_INVALID_ARG if NULL or out of range).
+ * Every other argument, the workspace and the outputs as for hcw_stack_fwd;
+ * hcw_stack_bwd_dims with the same dims is its backward.
+ */
+int hcw_stack_fwd_dims(const void* x, const void* W_self, const void* W_nbr, const float* bias,
+                       const int* dims, int L, int B, int n, int d, int dtype, unsigned flags,
+                       void* y, void* acts, void* masks, void* workspace, size_t ws_bytes,
+                       void* stream);
+
 /* Workspace bytes hcw_stack_fwd needs for these sizes and L layers (0 is possible). */
 size_t hcw_stack_fwd_workspace_bytes(int B, int n, int d, int dtype, unsigned flags, int L);
 
@@ -199,6 +214,16 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void
                   int B, int n, int d, int dtype, unsigned flags,
                   void* dx, float* dW_self, float* dW_nbr, float* dbias,
                   void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * Backward of hcw_stack_fwd_dims: hcw_stack_bwd with the schedule dims (host
+ * array of L ints in [0, log2 n), as given to the forward).
+ */
+int hcw_stack_bwd_dims(const void* x, const void* acts, const void* masks, const void* dy,
+                       const void* W_self, const void* W_nbr, const int* dims, int L, int B,
+                       int n, int d, int dtype, unsigned flags, void* dx, float* dW_self,
+                       float* dW_nbr, float* dbias, void* workspace, size_t ws_bytes,
+                       void* stream);
 
 /* Workspace bytes hcw_stack_bwd needs for L layers. */
 size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags, int L);

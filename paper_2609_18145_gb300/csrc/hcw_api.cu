@@ -200,6 +200,19 @@ int check_shape(int layer, int dim_override, int B, int n, int d, int dtype, uns
     return HCW_OK;
 }
 
+// Layer schedule of a stack (Sec. 3.3, Sec. 4): stack layer l uses cube
+// dimension dims[l] when a schedule array is given, else dim_override for
+// every layer (the fixed control), else (layer0 + l) mod log2 n (rot).
+struct Sched {
+    const int* dims;
+    int layer0;
+    int dim_override;
+    int dim(const Shape& sh, int l) const {
+        if (dims) return dims[l];
+        return dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
+    }
+};
+
 // Bytes of one layer's ReLU mask: ceil(d/32) 32-bit words per token.
 size_t mask_bytes(const Shape& sh) { return (size_t)sh.tokens * ((sh.d + 31) / 32) * 4; }
 
@@ -389,7 +402,7 @@ int launch_rows(int mode, int BN, TcLaunch<kMaxStackLayers>& T, int n, bool pair
 // Layers [l0, l0 + n) of a bf16 stack in one persistent launch.  in_ptr(l),
 // out_ptr(l), mask_ptr(l) give each layer's input, output and mask.
 template <class In, class Out, class Mask>
-int stack_fwd_group(const Shape& sh, int l0, int n, int layer0, int dim_override,
+int stack_fwd_group(const Shape& sh, int l0, int n, const Sched& sc,
                     const uint8_t* Ws, const uint8_t* Wn, const float* bias, unsigned flags,
                     In in_ptr, Out out_ptr, Mask mask_ptr, int* counters, cudaStream_t st) {
     const int d = sh.d, BN = pick_bn(d);
@@ -399,7 +412,7 @@ int stack_fwd_group(const Shape& sh, int l0, int n, int layer0, int dim_override
     memset(&L, 0, sizeof(L));
     for (int i = 0; i < n; ++i) {
         const int l = l0 + i;
-        const int s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
+        const int s = sc.dim(sh, l);
         if (!fwd_maps(L.maps[i], sh, s, in_ptr(l), Ws + l * wb, Wn + l * wb, out_ptr(l), pair))
             return HCW_ERR_CUDA;
         L.layer[i] = {s, 1 << s, bias ? bias + (size_t)l * d : nullptr, mask_ptr(l), nullptr,
@@ -420,7 +433,7 @@ int stack_fwd_group(const Shape& sh, int l0, int n, int layer0, int dim_override
 
 // Layers [l0, l0 + n) of a bf16 stack in one resident launch (hcw_res.cu).
 template <class In, class Out, class Mask>
-int stack_fwd_resident(const Shape& sh, int l0, int n, int layer0, int dim_override,
+int stack_fwd_resident(const Shape& sh, int l0, int n, const Sched& sc,
                        const uint8_t* Ws, const uint8_t* Wn, const float* bias, unsigned flags,
                        In in_ptr, Out out_ptr, Mask mask_ptr, cudaStream_t st) {
     const int d = sh.d, N = d >= 256 ? d / 2 : d;
@@ -429,7 +442,7 @@ int stack_fwd_resident(const Shape& sh, int l0, int n, int layer0, int dim_overr
     memset(&R, 0, sizeof(R));
     for (int i = 0; i < n; ++i) {
         const int l = l0 + i;
-        const int s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
+        const int s = sc.dim(sh, l);
         if (!map_weight(&R.wmap[i][0], Ws + l * wb, d, N / 2) ||
             !map_weight(&R.wmap[i][1], Wn + l * wb, d, N / 2) ||
             !map_rows16(&R.imap[i], out_ptr(l), sh.tokens, d, 1, 64))
@@ -649,16 +662,14 @@ size_t stack_weight_ws(const Shape& sh, int dtype, unsigned flags, int L) {
 
 size_t stack_dz_bytes(const Shape& sh, int L) { return align256((size_t)L * sh.act_bytes); }
 
-int stack_layer_dim(const Shape& sh, int layer0, int dim_override, int l) {
-    return dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
-}
 
 struct StackData {
     const void* masks;
     const void* dy;
     const uint8_t* Ws;
     const uint8_t* Wn;
-    int layer0, L, dim_override;
+    Sched sc;
+    int L;
     unsigned flags;
     void* dx;
     uint8_t* dz;   // [L][tokens][d], layer stride act_bytes
@@ -669,7 +680,8 @@ struct StackWeight {
     const void* x;
     const void* acts;
     const uint8_t* dz;
-    int layer0, L, dim_override;
+    Sched sc;
+    int L;
     unsigned flags;
     float* dWs;
     float* dWn;
@@ -697,7 +709,7 @@ int stack_data_resident(const Shape& sh, const StackData& a, cudaStream_t st) {
         memset(&R, 0, sizeof(R));
         for (int i = 0; i < cnt; ++i) {
             const int l = top - i;
-            const int s = stack_layer_dim(sh, a.layer0, a.dim_override, l);
+            const int s = a.sc.dim(sh, l);
             if (!map_weight_blocks(&R.wmap[i][0], a.Ws + l * wb, d, N / 128) ||
                 !map_weight_blocks(&R.wmap[i][1], a.Wn + l * wb, d, N / 128))
                 return HCW_ERR_CUDA;
@@ -770,7 +782,7 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
         memset(&T, 0, sizeof(T));
         for (int i = 0; i < cnt; ++i) {
             const int l = top - i;
-            const int s = stack_layer_dim(sh, a.layer0, a.dim_override, l);
+            const int s = a.sc.dim(sh, l);
             const int k = 1 << s;
             // stores: g_{l-1} (map 4) and dz_{l-1} (map 5); at l = 0 the stack's dx
             void* out = l == 0 ? a.dx : (relu ? (resid ? gbuf(l - 1) : nullptr) : dz(l - 1));
@@ -834,7 +846,7 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
         if (cnt * tiles * 2 < sms) {
             for (int l = l0; l < l0 + cnt; ++l) {
                 Shape shl = sh;
-                shl.s = stack_layer_dim(sh, a.layer0, a.dim_override, l);
+                shl.s = a.sc.dim(sh, l);
                 rc = dw_bf16(shl, act(l), dz(l), a.flags, a.dWs + (size_t)l * d * d,
                              a.dWn + (size_t)l * d * d, a.dbias ? a.dbias + (size_t)l * d : nullptr,
                              wws, st);
@@ -845,7 +857,7 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
         memset(&T, 0, sizeof(T));
         for (int i = 0; i < cnt; ++i) {
             const int l = l0 + i;
-            const int s = stack_layer_dim(sh, a.layer0, a.dim_override, l);
+            const int s = a.sc.dim(sh, l);
             const int k = 1 << s;
             CUtensorMap* m = T.maps[i];
             if (!map_rows_blocks(&m[0], dz(l), sh.tokens, d, k, 64, 2) ||
@@ -869,7 +881,7 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
         if (paired)
             for (int i = 0; i < cnt; ++i) {
                 const int l = l0 + i;
-                const int k = 1 << stack_layer_dim(sh, a.layer0, a.dim_override, l);
+                const int k = 1 << a.sc.dim(sh, l);
                 if (!map_rows_blocks(&T.maps[i][1], act(l), sh.tokens, d, k, 64, BN / 128))
                     return HCW_ERR_CUDA;
             }
@@ -931,7 +943,7 @@ int stack_data_f32(const Shape& sh, const StackData& a, cudaStream_t st) {
     const void* cur_g = a.dy;
     for (int l = L - 1; l >= 0; --l) {
         Shape shl = sh;
-        shl.s = stack_layer_dim(sh, a.layer0, a.dim_override, l);
+        shl.s = a.sc.dim(sh, l);
         void* out = l == 0 ? a.dx : (relu ? (void*)g[l & 1] : dz(l - 1));
         rc = layer_dx_impl(shl, HCW_F32, dz(l), cur_g, a.Ws + l * wb, a.Wn + l * wb, a.flags, out,
                            st);
@@ -955,7 +967,7 @@ int stack_weight_f32(const Shape& sh, const StackWeight& a, cudaStream_t st) {
     const size_t ab = sh.act_bytes;
     for (int l = 0; l < a.L; ++l) {
         Shape shl = sh;
-        shl.s = stack_layer_dim(sh, a.layer0, a.dim_override, l);
+        shl.s = a.sc.dim(sh, l);
         const void* in = l == 0 ? a.x : static_cast<const uint8_t*>(a.acts) + (size_t)(l - 1) * ab;
         const int rc = layer_dw_impl(shl, HCW_F32, in, a.dz + (size_t)l * ab, a.flags,
                                      a.dWs + (size_t)l * d * d, a.dWn + (size_t)l * d * d,
@@ -1059,6 +1071,119 @@ int check_bwd_ptrs(const Shape& sh, int dtype, unsigned flags, const void* x, co
         overlaps(dbias, sh.d * 4, dWs, gb) || overlaps(dbias, sh.d * 4, dWn, gb))
         return HCW_ERR_ALIASING;
     return HCW_OK;
+}
+
+// A schedule array of L cube dimensions, each in [0, log2 n).
+int check_dims(const Shape& sh, const int* dims, int L) {
+    if (!dims) return HCW_ERR_INVALID_ARG;
+    for (int l = 0; l < L; ++l)
+        if (dims[l] < 0 || dims[l] >= sh.b) return HCW_ERR_INVALID_ARG;
+    return HCW_OK;
+}
+
+int stack_fwd_impl(const Shape& sh, const void* x, const void* W_self, const void* W_nbr,
+                   const float* bias, const Sched& sc, int L, int dtype, unsigned flags, void* y,
+                   void* acts, void* masks, void* workspace, size_t ws_bytes, void* stream) {
+    const int B = sh.B, n = sh.n, d = sh.d;
+    int rc;
+    if (sh.tokens == 0) return HCW_OK;
+    if (L > 1 && !acts) return HCW_ERR_INVALID_ARG;
+    if ((acts && !aligned16(acts)) || (masks && !aligned16(masks)) ||
+        (workspace && !aligned16(workspace)))
+        return HCW_ERR_ALIGNMENT;
+    const size_t ab = sh.act_bytes, wb = (size_t)d * d * elem_size(dtype);
+    const size_t mb = mask_bytes(sh);
+    const size_t need = hcw_stack_fwd_workspace_bytes(B, n, d, dtype, flags, L);
+    if (ws_bytes < need || (need && !workspace)) return HCW_ERR_WORKSPACE;
+    rc = check_fwd_ptrs(sh, dtype, x, W_self, W_nbr, bias, y, nullptr);
+    if (rc) return rc;
+    const size_t acts_b = (size_t)(L - 1) * ab, m_b = (size_t)L * mb;
+    if (overlaps(acts, acts_b, x, ab) || overlaps(acts, acts_b, y, ab) ||
+        overlaps(masks, m_b, x, ab) || overlaps(masks, m_b, y, ab) ||
+        overlaps(masks, m_b, acts, acts_b) || overlaps(acts, acts_b, W_self, L * wb) ||
+        overlaps(acts, acts_b, W_nbr, L * wb) || overlaps(workspace, need, x, ab) ||
+        overlaps(workspace, need, y, ab) || overlaps(workspace, need, acts, acts_b) ||
+        overlaps(workspace, need, masks, m_b))
+        return HCW_ERR_ALIASING;
+    cudaStream_t st = (cudaStream_t)stream;
+    const bool want_mask = masks && (flags & HCW_ACT_RELU);
+    auto in_ptr = [&](int l) -> const void* {
+        return l == 0 ? x : static_cast<const uint8_t*>(acts) + (size_t)(l - 1) * ab;
+    };
+    auto out_ptr = [&](int l) -> void* {
+        return l == L - 1 ? y : static_cast<uint8_t*>(acts) + (size_t)l * ab;
+    };
+    auto mask_ptr = [&](int l) -> uint32_t* {
+        return want_mask ? reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(masks) + (size_t)l * mb)
+                         : nullptr;
+    };
+    if (dtype == HCW_BF16) {
+        // up to kMaxStackLayers layers per persistent launch
+        for (int l0 = 0; l0 < L; l0 += kMaxStackLayers) {
+            const int cnt = L - l0 < kMaxStackLayers ? L - l0 : kMaxStackLayers;
+            if (use_resident(sh))
+                rc = stack_fwd_resident(sh, l0, cnt, sc,
+                                        static_cast<const uint8_t*>(W_self),
+                                        static_cast<const uint8_t*>(W_nbr), bias, flags, in_ptr,
+                                        out_ptr, mask_ptr, st);
+            else
+                rc = stack_fwd_group(sh, l0, cnt, sc,
+                                     static_cast<const uint8_t*>(W_self),
+                                     static_cast<const uint8_t*>(W_nbr), bias, flags, in_ptr,
+                                     out_ptr, mask_ptr, static_cast<int*>(workspace), st);
+            if (rc) return rc;
+        }
+        return HCW_OK;
+    }
+    for (int l = 0; l < L; ++l) {
+        Shape shl = sh;
+        shl.s = sc.dim(sh, l);
+        rc = layer_fwd_impl(shl, dtype, in_ptr(l), static_cast<const uint8_t*>(W_self) + l * wb,
+                            static_cast<const uint8_t*>(W_nbr) + l * wb,
+                            bias ? bias + (size_t)l * d : nullptr, flags, out_ptr(l), nullptr, st,
+                            mask_ptr(l));
+        if (rc) return rc;
+    }
+    return HCW_OK;
+}
+
+int stack_bwd_impl(const Shape& sh, const void* x, const void* acts, const void* masks,
+                   const void* dy, const void* W_self, const void* W_nbr, const Sched& sc, int L,
+                   int dtype, unsigned flags, void* dx, float* dW_self, float* dW_nbr,
+                   float* dbias, void* workspace, size_t ws_bytes, void* stream) {
+    const int d = sh.d;
+    int rc;
+    cudaStream_t st = (cudaStream_t)stream;
+    if (sh.tokens == 0) {
+        if (!dW_self || !dW_nbr) return HCW_ERR_INVALID_ARG;
+        return zero_weight_grads(L, d, dW_self, dW_nbr, dbias, st);
+    }
+    // workspace: [dz of every layer][input-gradient scratch][weight-gradient scratch]
+    const size_t zb = stack_dz_bytes(sh, L);
+    const size_t db = align256(stack_data_ws(sh, dtype, flags, L));
+    const size_t wb = stack_weight_ws(sh, dtype, flags, L);
+    if (ws_bytes < zb + db + wb || !workspace) return HCW_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return HCW_ERR_ALIGNMENT;
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    rc = check_stack_data(sh, dtype, flags, L, masks, dy, W_self, W_nbr, dx, ws, ws + zb, db);
+    if (rc) return rc;
+    rc = check_stack_weight(sh, dtype, flags, L, x, acts, ws, dW_self, dW_nbr, dbias, ws + zb + db,
+                            wb);
+    if (rc) return rc;
+    // the weight gradients read x and acts; the input gradients write dx
+    const size_t ab = sh.act_bytes;
+    if (overlaps(dx, ab, x, ab) || overlaps(dx, ab, acts, (size_t)(L - 1) * ab) ||
+        overlaps(ws, ws_bytes, x, ab) || overlaps(ws, ws_bytes, acts, (size_t)(L - 1) * ab) ||
+        overlaps(dx, ab, dW_self, (size_t)L * d * d * 4) ||
+        overlaps(dx, ab, dW_nbr, (size_t)L * d * d * 4) ||
+        overlaps(dx, ab, dbias, dbias ? (size_t)L * d * 4 : 0))
+        return HCW_ERR_ALIASING;
+    StackData da{masks, dy, static_cast<const uint8_t*>(W_self),
+                 static_cast<const uint8_t*>(W_nbr), sc, L, flags, dx, ws, ws + zb};
+    rc = dtype == HCW_BF16 ? stack_data_bf16(sh, da, st) : stack_data_f32(sh, da, st);
+    if (rc) return rc;
+    StackWeight wa{x, acts, ws, sc, L, flags, dW_self, dW_nbr, dbias, ws + zb + db};
+    return dtype == HCW_BF16 ? stack_weight_bf16(sh, wa, st) : stack_weight_f32(sh, wa, st);
 }
 
 }  // namespace
@@ -1220,65 +1345,22 @@ int hcw_stack_fwd(const void* x, const void* W_self, const void* W_nbr, const fl
     if (L < 1) return HCW_ERR_INVALID_ARG;
     int rc = check_shape(layer0, dim_override, B, n, d, dtype, flags, &sh);
     if (rc) return rc;
-    if (sh.tokens == 0) return HCW_OK;
-    if (L > 1 && !acts) return HCW_ERR_INVALID_ARG;
-    if ((acts && !aligned16(acts)) || (masks && !aligned16(masks)) ||
-        (workspace && !aligned16(workspace)))
-        return HCW_ERR_ALIGNMENT;
-    const size_t ab = sh.act_bytes, wb = (size_t)d * d * elem_size(dtype);
-    const size_t mb = mask_bytes(sh);
-    const size_t need = hcw_stack_fwd_workspace_bytes(B, n, d, dtype, flags, L);
-    if (ws_bytes < need || (need && !workspace)) return HCW_ERR_WORKSPACE;
-    rc = check_fwd_ptrs(sh, dtype, x, W_self, W_nbr, bias, y, nullptr);
+    return stack_fwd_impl(sh, x, W_self, W_nbr, bias, Sched{nullptr, layer0, dim_override}, L,
+                          dtype, flags, y, acts, masks, workspace, ws_bytes, stream);
+}
+
+int hcw_stack_fwd_dims(const void* x, const void* W_self, const void* W_nbr, const float* bias,
+                       const int* dims, int L, int B, int n, int d, int dtype, unsigned flags,
+                       void* y, void* acts, void* masks, void* workspace, size_t ws_bytes,
+                       void* stream) {
+    Shape sh;
+    if (L < 1) return HCW_ERR_INVALID_ARG;
+    int rc = check_shape(0, -1, B, n, d, dtype, flags, &sh);
     if (rc) return rc;
-    const size_t acts_b = (size_t)(L - 1) * ab, m_b = (size_t)L * mb;
-    if (overlaps(acts, acts_b, x, ab) || overlaps(acts, acts_b, y, ab) ||
-        overlaps(masks, m_b, x, ab) || overlaps(masks, m_b, y, ab) ||
-        overlaps(masks, m_b, acts, acts_b) || overlaps(acts, acts_b, W_self, L * wb) ||
-        overlaps(acts, acts_b, W_nbr, L * wb) || overlaps(workspace, need, x, ab) ||
-        overlaps(workspace, need, y, ab) || overlaps(workspace, need, acts, acts_b) ||
-        overlaps(workspace, need, masks, m_b))
-        return HCW_ERR_ALIASING;
-    cudaStream_t st = (cudaStream_t)stream;
-    const bool want_mask = masks && (flags & HCW_ACT_RELU);
-    auto in_ptr = [&](int l) -> const void* {
-        return l == 0 ? x : static_cast<const uint8_t*>(acts) + (size_t)(l - 1) * ab;
-    };
-    auto out_ptr = [&](int l) -> void* {
-        return l == L - 1 ? y : static_cast<uint8_t*>(acts) + (size_t)l * ab;
-    };
-    auto mask_ptr = [&](int l) -> uint32_t* {
-        return want_mask ? reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(masks) + (size_t)l * mb)
-                         : nullptr;
-    };
-    if (dtype == HCW_BF16) {
-        // up to kMaxStackLayers layers per persistent launch
-        for (int l0 = 0; l0 < L; l0 += kMaxStackLayers) {
-            const int cnt = L - l0 < kMaxStackLayers ? L - l0 : kMaxStackLayers;
-            if (use_resident(sh))
-                rc = stack_fwd_resident(sh, l0, cnt, layer0, dim_override,
-                                        static_cast<const uint8_t*>(W_self),
-                                        static_cast<const uint8_t*>(W_nbr), bias, flags, in_ptr,
-                                        out_ptr, mask_ptr, st);
-            else
-                rc = stack_fwd_group(sh, l0, cnt, layer0, dim_override,
-                                     static_cast<const uint8_t*>(W_self),
-                                     static_cast<const uint8_t*>(W_nbr), bias, flags, in_ptr,
-                                     out_ptr, mask_ptr, static_cast<int*>(workspace), st);
-            if (rc) return rc;
-        }
-        return HCW_OK;
-    }
-    for (int l = 0; l < L; ++l) {
-        Shape shl = sh;
-        shl.s = dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
-        rc = layer_fwd_impl(shl, dtype, in_ptr(l), static_cast<const uint8_t*>(W_self) + l * wb,
-                            static_cast<const uint8_t*>(W_nbr) + l * wb,
-                            bias ? bias + (size_t)l * d : nullptr, flags, out_ptr(l), nullptr, st,
-                            mask_ptr(l));
-        if (rc) return rc;
-    }
-    return HCW_OK;
+    rc = check_dims(sh, dims, L);
+    if (rc) return rc;
+    return stack_fwd_impl(sh, x, W_self, W_nbr, bias, Sched{dims, 0, -1}, L, dtype, flags, y,
+                          acts, masks, workspace, ws_bytes, stream);
 }
 
 size_t hcw_stack_bwd_data_workspace_bytes(int B, int n, int d, int dtype, unsigned flags,
@@ -1315,7 +1397,7 @@ int hcw_stack_bwd_data(const void* masks, const void* dy, const void* W_self, co
                           ws_bytes);
     if (rc) return rc;
     StackData a{masks, dy, static_cast<const uint8_t*>(W_self), static_cast<const uint8_t*>(W_nbr),
-                layer0, L, dim_override, flags, dx, static_cast<uint8_t*>(dz),
+                Sched{nullptr, layer0, dim_override}, L, flags, dx, static_cast<uint8_t*>(dz),
                 static_cast<uint8_t*>(workspace)};
     return dtype == HCW_BF16 ? stack_data_bf16(sh, a, (cudaStream_t)stream)
                              : stack_data_f32(sh, a, (cudaStream_t)stream);
@@ -1336,8 +1418,8 @@ int hcw_stack_bwd_weight(const void* x, const void* acts, const void* dz, int la
     rc = check_stack_weight(sh, dtype, flags, L, x, acts, dz, dW_self, dW_nbr, dbias, workspace,
                             ws_bytes);
     if (rc) return rc;
-    StackWeight a{x, acts, static_cast<const uint8_t*>(dz), layer0, L, dim_override, flags,
-                  dW_self, dW_nbr, dbias, static_cast<uint8_t*>(workspace)};
+    StackWeight a{x, acts, static_cast<const uint8_t*>(dz), Sched{nullptr, layer0, dim_override}, L,
+                  flags, dW_self, dW_nbr, dbias, static_cast<uint8_t*>(workspace)};
     return dtype == HCW_BF16 ? stack_weight_bf16(sh, a, (cudaStream_t)stream)
                              : stack_weight_f32(sh, a, (cudaStream_t)stream);
 }
@@ -1350,39 +1432,24 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void
     if (L < 1) return HCW_ERR_INVALID_ARG;
     int rc = check_shape(layer0, dim_override, B, n, d, dtype, flags, &sh);
     if (rc) return rc;
-    cudaStream_t st = (cudaStream_t)stream;
-    if (sh.tokens == 0) {
-        if (!dW_self || !dW_nbr) return HCW_ERR_INVALID_ARG;
-        return zero_weight_grads(L, d, dW_self, dW_nbr, dbias, st);
-    }
-    // workspace: [dz of every layer][input-gradient scratch][weight-gradient scratch]
-    const size_t zb = stack_dz_bytes(sh, L);
-    const size_t db = align256(stack_data_ws(sh, dtype, flags, L));
-    const size_t wb = stack_weight_ws(sh, dtype, flags, L);
-    if (ws_bytes < zb + db + wb || !workspace) return HCW_ERR_WORKSPACE;
-    if (!aligned16(workspace)) return HCW_ERR_ALIGNMENT;
-    uint8_t* ws = static_cast<uint8_t*>(workspace);
-    rc = check_stack_data(sh, dtype, flags, L, masks, dy, W_self, W_nbr, dx, ws, ws + zb, db);
+    return stack_bwd_impl(sh, x, acts, masks, dy, W_self, W_nbr,
+                          Sched{nullptr, layer0, dim_override}, L, dtype, flags, dx, dW_self,
+                          dW_nbr, dbias, workspace, ws_bytes, stream);
+}
+
+int hcw_stack_bwd_dims(const void* x, const void* acts, const void* masks, const void* dy,
+                       const void* W_self, const void* W_nbr, const int* dims, int L, int B,
+                       int n, int d, int dtype, unsigned flags, void* dx, float* dW_self,
+                       float* dW_nbr, float* dbias, void* workspace, size_t ws_bytes,
+                       void* stream) {
+    Shape sh;
+    if (L < 1) return HCW_ERR_INVALID_ARG;
+    int rc = check_shape(0, -1, B, n, d, dtype, flags, &sh);
     if (rc) return rc;
-    rc = check_stack_weight(sh, dtype, flags, L, x, acts, ws, dW_self, dW_nbr, dbias, ws + zb + db,
-                            wb);
+    rc = check_dims(sh, dims, L);
     if (rc) return rc;
-    // the weight gradients read x and acts; the input gradients write dx
-    const size_t ab = sh.act_bytes;
-    if (overlaps(dx, ab, x, ab) || overlaps(dx, ab, acts, (size_t)(L - 1) * ab) ||
-        overlaps(ws, ws_bytes, x, ab) || overlaps(ws, ws_bytes, acts, (size_t)(L - 1) * ab) ||
-        overlaps(dx, ab, dW_self, (size_t)L * d * d * 4) ||
-        overlaps(dx, ab, dW_nbr, (size_t)L * d * d * 4) ||
-        overlaps(dx, ab, dbias, dbias ? (size_t)L * d * 4 : 0))
-        return HCW_ERR_ALIASING;
-    StackData da{masks, dy, static_cast<const uint8_t*>(W_self),
-                 static_cast<const uint8_t*>(W_nbr), layer0, L, dim_override, flags, dx, ws,
-                 ws + zb};
-    rc = dtype == HCW_BF16 ? stack_data_bf16(sh, da, st) : stack_data_f32(sh, da, st);
-    if (rc) return rc;
-    StackWeight wa{x, acts, ws, layer0, L, dim_override, flags, dW_self, dW_nbr, dbias,
-                   ws + zb + db};
-    return dtype == HCW_BF16 ? stack_weight_bf16(sh, wa, st) : stack_weight_f32(sh, wa, st);
+    return stack_bwd_impl(sh, x, acts, masks, dy, W_self, W_nbr, Sched{dims, 0, -1}, L, dtype,
+                          flags, dx, dW_self, dW_nbr, dbias, workspace, ws_bytes, stream);
 }
 
 int hcw_set_stack_kernels(int mode) {

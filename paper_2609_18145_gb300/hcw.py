@@ -65,6 +65,10 @@ _SIGNATURES = {
     "hcw_launch_count": ([], ctypes.c_ulonglong),
     "hcw_stack_fwd": ([_P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P, _SZ,
                        _P], _I),
+    "hcw_stack_fwd_dims": ([_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P, _SZ,
+                            _P], _I),
+    "hcw_stack_bwd_dims": ([_P, _P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P,
+                            _P, _SZ, _P], _I),
     "hcw_stack_fwd_workspace_bytes": ([_I, _I, _I, _I, _U, _I], _SZ),
     "hcw_stack_workspace_bytes": ([_I, _I, _I, _I, _U, _I], _SZ),
     "hcw_stack_bwd_data": ([_P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _SZ,
@@ -278,12 +282,22 @@ def hcw_stack_fwd_workspace_bytes(B: int, n: int, d: int, dtype: int, flags: int
     return int(lib().hcw_stack_fwd_workspace_bytes(B, n, d, dtype, flags, L))
 
 
+def _dims_array(dims, L):
+    """A layer schedule as a C int array of L dimensions (kept alive by the caller)."""
+    vals = [int(v) for v in dims]
+    if len(vals) != L:
+        raise ValueError("dims needs one cube dimension per layer (%d), got %d" % (L, len(vals)))
+    return (ctypes.c_int * L)(*vals)
+
+
 def hcw_stack_fwd(x, W_self, W_nbr, bias=None, layer0: int = 0, dim_override: int = -1,
                   flags: int = 0, y=None, acts=None, masks=None, want_masks: bool = None,
-                  workspace=None, stream=None):
+                  workspace=None, stream=None, dims=None):
     """Stack forward over L = W_self.shape[0] layers; returns (y, acts, masks).
     masks (ReLU only) are int32 words [L, B, n, ceil(d/32)], bit o%32 of word
-    o/32 = (z > 0); allocated when the stack uses ReLU unless want_masks=False."""
+    o/32 = (z > 0); allocated when the stack uses ReLU unless want_masks=False.
+    dims (a sequence of L cube dimensions) calls hcw_stack_fwd_dims instead;
+    layer0 and dim_override are then unused."""
     _dev(x, W_self, W_nbr, bias, y, acts, masks, workspace)
     B, n, d = x.shape
     L = W_self.shape[0]
@@ -296,6 +310,13 @@ def hcw_stack_fwd(x, W_self, W_nbr, bias=None, layer0: int = 0, dim_override: in
     if masks is None and want_masks:
         masks = torch.empty((L, B, n, (d + 31) // 32), dtype=torch.int32, device=x.device)
     ws = _workspace(hcw_stack_fwd_workspace_bytes(B, n, d, dt, flags, L), x.device, workspace)
+    if dims is not None:
+        arr = _dims_array(dims, L)
+        _check(lib().hcw_stack_fwd_dims(_ptr(x), _ptr(W_self), _ptr(W_nbr), _ptr(bias),
+                                        ctypes.cast(arr, _P), L, B, n, d, dt, flags, _ptr(y),
+                                        _ptr(acts), _ptr(masks), _ptr(ws), ws.numel(),
+                                        _stream(stream)), "hcw_stack_fwd_dims")
+        return y, acts, masks
     _check(lib().hcw_stack_fwd(_ptr(x), _ptr(W_self), _ptr(W_nbr), _ptr(bias), layer0, L,
                                dim_override, B, n, d, dt, flags, _ptr(y), _ptr(acts),
                                _ptr(masks), _ptr(ws), ws.numel(), _stream(stream)),
@@ -303,10 +324,16 @@ def hcw_stack_fwd(x, W_self, W_nbr, bias=None, layer0: int = 0, dim_override: in
     return y, acts, masks
 
 
+def hcw_stack_fwd_dims(x, W_self, W_nbr, bias, dims, flags: int = 0, **kw):
+    """hcw_stack_fwd with layer l on cube dimension dims[l]."""
+    return hcw_stack_fwd(x, W_self, W_nbr, bias, flags=flags, dims=dims, **kw)
+
+
 def hcw_stack_bwd(x, acts, masks, dy, W_self, W_nbr, layer0: int = 0, dim_override: int = -1,
                   flags: int = 0, dx=None, dW_self=None, dW_nbr=None, dbias=None,
-                  want_dbias: bool = True, workspace=None, stream=None):
-    """Stack backward; returns (dx, dW_self[L], dW_nbr[L], dbias[L])."""
+                  want_dbias: bool = True, workspace=None, stream=None, dims=None):
+    """Stack backward; returns (dx, dW_self[L], dW_nbr[L], dbias[L]).  dims as
+    for hcw_stack_fwd (calls hcw_stack_bwd_dims)."""
     _dev(x, acts, masks, dy, W_self, W_nbr, dx, dW_self, dW_nbr, dbias, workspace)
     B, n, d = x.shape
     L = W_self.shape[0]
@@ -319,11 +346,24 @@ def hcw_stack_bwd(x, acts, masks, dy, W_self, W_nbr, layer0: int = 0, dim_overri
         dbias = torch.empty(L, d, **f32)
     need = hcw_stack_workspace_bytes(B, n, d, dt, flags, L)
     ws = _workspace(need, x.device, workspace)
+    if dims is not None:
+        arr = _dims_array(dims, L)
+        _check(lib().hcw_stack_bwd_dims(_ptr(x), _ptr(acts), _ptr(masks), _ptr(dy),
+                                        _ptr(W_self), _ptr(W_nbr), ctypes.cast(arr, _P), L, B,
+                                        n, d, dt, flags, _ptr(dx), _ptr(dW_self), _ptr(dW_nbr),
+                                        _ptr(dbias), _ptr(ws), ws.numel(), _stream(stream)),
+               "hcw_stack_bwd_dims")
+        return dx, dW_self, dW_nbr, dbias
     _check(lib().hcw_stack_bwd(_ptr(x), _ptr(acts), _ptr(masks), _ptr(dy), _ptr(W_self),
                                _ptr(W_nbr), layer0, L, dim_override, B, n, d, dt, flags,
                                _ptr(dx), _ptr(dW_self), _ptr(dW_nbr), _ptr(dbias), _ptr(ws),
                                ws.numel(), _stream(stream)), "hcw_stack_bwd")
     return dx, dW_self, dW_nbr, dbias
+
+
+def hcw_stack_bwd_dims(x, acts, masks, dy, W_self, W_nbr, dims, flags: int = 0, **kw):
+    """hcw_stack_bwd of a stack run with hcw_stack_fwd_dims(dims)."""
+    return hcw_stack_bwd(x, acts, masks, dy, W_self, W_nbr, flags=flags, dims=dims, **kw)
 
 
 def hcw_stack_bwd_data_workspace_bytes(B: int, n: int, d: int, dtype: int, flags: int,

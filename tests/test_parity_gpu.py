@@ -335,6 +335,84 @@ def test_resident_and_streaming_stacks_agree(H, flags):
         assert rel(host(b[i]), host(a[i])) <= 1e-2, what
 
 
+def gray_dims(L):
+    """Dimension flipped at each step of the binary reflected Gray code (Sec. 4: it
+    visits dimension 0 every other layer and dimension b-1 only late)."""
+    return [(g & -g).bit_length() - 1 for g in range(1, L + 1)]
+
+
+SCHEDULE_CASES = [
+    # name, kernels, B, n, d, flags, dims
+    ("gray16_n64", "auto", 8, 64, 128, CAUSAL | RESIDUAL | RELU, gray_dims(16)),
+    ("perm_twice_n64", "auto", 8, 64, 128, RESIDUAL, [3, 0, 5, 1, 4, 2, 2, 4, 1, 5, 0, 3]),
+    ("gray16_n64_resident", "resident", 8, 64, 128, CAUSAL | RESIDUAL | RELU, gray_dims(16)),
+    # n = 256: dimension 7 at irregular places (twice in a row, first, last):
+    # the resident kernels change CTA split there
+    ("n256_dim7_resident", "resident", 2, 256, 128, CAUSAL | RESIDUAL | RELU,
+     [7, 7, 0, 3, 7, 6, 5, 7]),
+    ("n256_dim7_streaming", "streaming", 2, 256, 128, CAUSAL | RESIDUAL | RELU,
+     [7, 7, 0, 3, 7, 6, 5, 7]),
+]
+
+
+@pytest.mark.parametrize("case", SCHEDULE_CASES, ids=lambda c: c[0])
+def test_stack_with_a_schedule_array(H, case):
+    """hcw_stack_fwd_dims / hcw_stack_bwd_dims against the oracle's stacks on
+    the same schedule (Sec. 3.3 schedules; Sec. 4 permutation and Gray order)."""
+    name, kernels, B, n, d, flags, dims = case
+    L = len(dims)
+    pr = synth.problem(B, n, d, L=L, seed=19, w_std=(1 / (2 * d)) ** 0.5)
+    mode = {"auto": H.HCW_STACK_AUTO, "resident": H.HCW_STACK_RESIDENT,
+            "streaming": H.HCW_STACK_STREAMING}[kernels]
+    prev = H.hcw_set_stack_kernels(mode)
+    try:
+        x, x64 = dev(pr.x, torch.bfloat16)
+        Ws, Ws64 = dev(pr.W_self, torch.bfloat16)
+        Wn, Wn64 = dev(pr.W_nbr, torch.bfloat16)
+        dy, dy64 = dev(pr.dy, torch.bfloat16)
+        bias = torch.from_numpy(pr.bias).cuda()
+        y, acts, masks = H.hcw_stack_fwd_dims(x, Ws, Wn, bias, dims, flags)
+        ry, racts, rzs = O.stack_fwd(x64, Ws64, Wn64, pr.bias.astype(np.float64), 0, L, -1,
+                                     flags, round_bf16=True, dims=dims)
+        assert rel(host(y), ry) <= TOL_BF16, name
+        assert rel(host(acts), racts[1:]) <= TOL_BF16, name
+        o_acts = torch.from_numpy(racts[1:]).to(torch.bfloat16).cuda()
+        o_masks = masks_from_z(rzs).cuda() if flags & RELU else None
+        dx, gWs, gWn, gb = H.hcw_stack_bwd_dims(x, o_acts, o_masks, dy, Ws, Wn, dims, flags)
+        torch.cuda.synchronize()
+        assert H.hcw_sync_status() == H.HCW_OK
+        rdx, rWs, rWn, rgb = O.stack_bwd(racts, rzs, dy64, Ws64, Wn64, 0, L, -1, flags,
+                                         round_bf16=True, dims=dims)
+        for got, ref, what in ((dx, rdx, "dx"), (gWs, rWs, "dW_self"), (gWn, rWn, "dW_nbr"),
+                               (gb, rgb, "dbias")):
+            assert rel(host(got), ref) <= TOL_BF16, (name, what)
+    finally:
+        H.hcw_set_stack_kernels(prev)
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_schedule_array_of_the_rotation_equals_the_rotated_stack(H, dtype):
+    """dims = (layer0 + l) mod log2 n reproduces hcw_stack_fwd / hcw_stack_bwd
+    with that layer0 exactly (the same kernels run on the same dimensions)."""
+    B, n, d, L, layer0 = 4, 64, 64 if dtype == torch.float32 else 128, 9, 2
+    flags = CAUSAL | RESIDUAL | RELU
+    pr = synth.problem(B, n, d, L=L, seed=23, w_std=(1 / (2 * d)) ** 0.5)
+    x, _ = dev(pr.x, dtype)
+    Ws, _ = dev(pr.W_self, dtype)
+    Wn, _ = dev(pr.W_nbr, dtype)
+    dy, _ = dev(pr.dy, dtype)
+    bias = torch.from_numpy(pr.bias).cuda()
+    dims = [(layer0 + l) % 6 for l in range(L)]
+    a = H.hcw_stack_fwd(x, Ws, Wn, bias, layer0, -1, flags)
+    b = H.hcw_stack_fwd_dims(x, Ws, Wn, bias, dims, flags)
+    for u, v in zip(a, b):
+        assert torch.equal(u, v)
+    ga = H.hcw_stack_bwd(x, a[1], a[2], dy, Ws, Wn, layer0, -1, flags)
+    gb = H.hcw_stack_bwd_dims(x, a[1], a[2], dy, Ws, Wn, dims, flags)
+    for u, v in zip(ga, gb):
+        assert torch.equal(u, v)
+
+
 def test_stack_fixed_dimension_control(H):
     pr = synth.problem(16, 64, 128, L=6, seed=5, w_std=(1 / 256) ** 0.5)
     got, ref = run_stack(H, pr, torch.bfloat16, 6, 0, dim=0)
