@@ -40,8 +40,14 @@
  *
  *   Stack (Sec. 3.3, "rot"): layer l of a stack starting at layer index
  *   layer0 uses dimension (layer0 + l) mod b, or a fixed dimension (the
- *   "fixed" control of Sec. 3.3), or an explicit list of dimensions (the
- *   order variants of Sec. 4).
+ *   "fixed" control of Sec. 3.3), or an explicit list of layers (the order
+ *   variants of Sec. 4, and the schedules of Sec. 3.3 / App. A).  In a list,
+ *   an entry s >= 0 is the hypercube link along dimension s ("jump 2^s" of
+ *   App. A), and an entry s < 0 is the shift of Eq. (1) itself with distance
+ *   k = -s: position i receives x_{i-k} when i >= k, within its sample
+ *   ("near" of App. A is k = 1, the "local" schedule of Sec. 3.3).  A shift
+ *   always links the earlier position to the later one, so the causal rule
+ *   does not change it.
  *
  * Precision: every sum is an fp64 loop in index order.  With round_bf16 set,
  * every stored activation (y, z, dx) is rounded to bfloat16 (round to
@@ -99,6 +105,24 @@ int oracle_receives(int i, int s, unsigned flags) {
     return oracle_partner(i, s) < i;
 }
 
+/* The link of a layer, s >= 0 (hypercube dimension) or s < 0 (shift by -s).
+ * link_partner: the position whose input position i takes at this layer.
+ * link_receives: whether position i takes it (n = positions per sample).
+ * link_reader: the position that takes x_i as its partner input, or -1. */
+static int link_partner(int i, int s) { return s >= 0 ? oracle_partner(i, s) : i + s; }
+
+static int link_receives(int i, int s, int n, unsigned flags) {
+    (void)n;
+    if (s < 0) return i + s >= 0;
+    return oracle_receives(i, s, flags);
+}
+
+static int link_reader(int i, int s, int n, unsigned flags) {
+    if (s < 0) return (i - s < n) ? i - s : -1;
+    int p = oracle_partner(i, s);
+    return oracle_receives(p, s, flags) ? p : -1;
+}
+
 /* partner[i] = p(i) if position i receives at this layer, else -1. */
 int oracle_partner_table(int layer, int dim_override, int n, unsigned flags, int* partner) {
     int s = oracle_dim(layer, dim_override, n);
@@ -137,7 +161,7 @@ static double act_grad(double z, unsigned flags) {
     return 1.0;
 }
 
-/* One layer forward along cube dimension s.  z_out may be NULL. */
+/* One layer forward with link s (see link_partner).  z_out may be NULL. */
 static void layer_fwd_dim(const double* x, const double* Ws, const double* Wn,
                           const double* bias, int s, int B, int n, int d,
                           unsigned flags, int round_bf16, double* y, double* z_out) {
@@ -148,8 +172,8 @@ static void layer_fwd_dim(const double* x, const double* Ws, const double* Wn,
     for (long long r = 0; r < rows; r++) {
         int b = (int)(r / n), i = (int)(r % n);
         const double* xi = x + ((size_t)b * n + i) * d;
-        int recv = oracle_receives(i, s, flags);
-        const double* xp = x + ((size_t)b * n + oracle_partner(i, s)) * d;
+        int recv = link_receives(i, s, n, flags);
+        const double* xp = recv ? x + ((size_t)b * n + link_partner(i, s)) * d : NULL;
         for (int o = 0; o < d; o++) {
             double z = bias ? bias[o] : 0.0;
             for (int k = 0; k < d; k++) z += Ws[(size_t)o * d + k] * xi[k];
@@ -167,8 +191,8 @@ static void layer_fwd_dim(const double* x, const double* Ws, const double* Wn,
     }
 }
 
-/* One layer backward along cube dimension s.  z may be NULL when no
- * activation is used.  dW_self, dW_nbr, dbias may each be NULL. */
+/* One layer backward with link s.  z may be NULL when no activation is
+ * used.  dW_self, dW_nbr, dbias may each be NULL. */
 static void layer_bwd_dim(const double* x, const double* z, const double* dy,
                           const double* Ws, const double* Wn, int s, int B, int n, int d,
                           unsigned flags, int round_bf16, double* dx,
@@ -185,15 +209,14 @@ static void layer_bwd_dim(const double* x, const double* z, const double* dy,
 #endif
         for (long long r = 0; r < rows; r++) {
             int b = (int)(r / n), i = (int)(r % n);
-            int p = oracle_partner(i, s);
-            int p_recv = oracle_receives(p, s, flags);   /* does p(i) read x_i? */
+            int j = link_reader(i, s, n, flags);          /* who reads x_i, if anyone */
             const double* dzi = dz + ((size_t)b * n + i) * d;
-            const double* dzp = dz + ((size_t)b * n + p) * d;
+            const double* dzj = j >= 0 ? dz + ((size_t)b * n + j) * d : NULL;
             for (int k = 0; k < d; k++) {
                 double g = 0.0;
                 for (int o = 0; o < d; o++) g += dzi[o] * Ws[(size_t)o * d + k];
-                if (p_recv)
-                    for (int o = 0; o < d; o++) g += dzp[o] * Wn[(size_t)o * d + k];
+                if (dzj)
+                    for (int o = 0; o < d; o++) g += dzj[o] * Wn[(size_t)o * d + k];
                 if (flags & ORACLE_RESIDUAL) g += dy[((size_t)b * n + i) * d + k];
                 if (round_bf16) g = oracle_round_bf16(g);
                 dx[((size_t)b * n + i) * d + k] = g;
@@ -211,8 +234,8 @@ static void layer_bwd_dim(const double* x, const double* z, const double* dy,
                     int b = (int)(r / n), i = (int)(r % n);
                     double dzo = dz[((size_t)b * n + i) * d + o];
                     gs += dzo * x[((size_t)b * n + i) * d + k];
-                    if (oracle_receives(i, s, flags))
-                        gn += dzo * x[((size_t)b * n + oracle_partner(i, s)) * d + k];
+                    if (link_receives(i, s, n, flags))
+                        gn += dzo * x[((size_t)b * n + link_partner(i, s)) * d + k];
                 }
                 if (dWs) dWs[(size_t)o * d + k] = gs;
                 if (dWn) dWn[(size_t)o * d + k] = gn;
@@ -249,12 +272,21 @@ int oracle_layer_bwd(const double* x, const double* z, const double* dy,
     return 0;
 }
 
-/* Dimension of stack layer l: dims[l] if a schedule is given, else the
- * rotated (or fixed) rule applied to layer index layer0 + l. */
+/* Marker of an invalid layer (a shift is a negative link). */
+#define NO_LINK (-(1 << 30))
+
+/* Link of stack layer l: dims[l] if a schedule is given (a dimension in
+ * [0, b) or a shift -k with 1 <= k < n), else the rotated (or fixed) rule
+ * applied to layer index layer0 + l; NO_LINK if invalid. */
 static int stack_dim(const int* dims, int layer0, int l, int dim_override, int n) {
     int b = log2_exact(n);
-    if (dims) return (dims[l] >= 0 && dims[l] < b) ? dims[l] : -1;
-    return oracle_dim(layer0 + l, dim_override, n);
+    if (b < 1) return NO_LINK;
+    if (dims) {
+        if (dims[l] >= 0) return dims[l] < b ? dims[l] : NO_LINK;
+        return -dims[l] < n ? dims[l] : NO_LINK;
+    }
+    int s = oracle_dim(layer0 + l, dim_override, n);
+    return s >= 0 ? s : NO_LINK;
 }
 
 /* Stack forward.  acts [L][B][n][d] receives each layer's input (acts[0] is
@@ -267,7 +299,7 @@ int oracle_stack_fwd(const double* x, const double* Ws, const double* Wn, const 
     size_t act = (size_t)B * n * d;
     if (L < 1) return -1;
     for (int l = 0; l < L; l++)
-        if (stack_dim(dims, layer0, l, dim_override, n) < 0) return -1;
+        if (stack_dim(dims, layer0, l, dim_override, n) == NO_LINK) return -1;
     memcpy(acts, x, act * sizeof(double));
     for (int l = 0; l < L; l++) {
         int s = stack_dim(dims, layer0, l, dim_override, n);
@@ -295,7 +327,7 @@ int oracle_stack_bwd(const double* acts, const double* zs, const double* dy,
     memcpy(g, dy, act * sizeof(double));
     for (int l = L - 1; l >= 0; l--) {
         int s = stack_dim(dims, layer0, l, dim_override, n);
-        if (s < 0) { free(g); free(g_next); return -1; }
+        if (s == NO_LINK) { free(g); free(g_next); return -1; }
         layer_bwd_dim(acts + (size_t)l * act, zs ? zs + (size_t)l * act : NULL, g,
                       Ws + (size_t)l * d * d, Wn + (size_t)l * d * d, s, B, n, d, flags,
                       round_bf16, g_next, dWs + (size_t)l * d * d, dWn + (size_t)l * d * d,
