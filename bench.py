@@ -37,6 +37,11 @@ WORKLOAD = "charlm_w256_d512"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 L2_FLUSH_BYTES = 256 << 20
 STACK_KERNELS = {"auto": 0, "resident": 1, "streaming": 2}   # hcw_set_stack_kernels modes
+# Layer schedules (hcw_stack_fwd_dims): None = the rotated stack of the workload.
+# hy256 = the near and jump layers of the paper's window-256 hybrid (App. A:
+# near jump128 near [attn] near jump32 near jump16 near [attn] near jump4 near
+# jump2 near jump1, the two attention layers left out); -1 = near (shift by 1).
+SCHEDULES = {"rot": None, "hy256": [-1, 7, -1, -1, 5, -1, 4, -1, -1, 2, -1, 1, -1, 0]}
 
 
 def load_peaks():
@@ -56,11 +61,18 @@ def workload():
     return w
 
 
-def step_flops(B, n, d, L):
+def step_flops(B, n, d, L, dims=None):
     """Algorithmic flops of one fwd+bwd step (causal): per token and layer
     3d^2 forward (half the positions use both maps), 3d^2 input gradient,
-    3d^2 weight gradients (flop = 2 MAC)."""
-    return 9.0 * d * d * B * n * L
+    3d^2 weight gradients (flop = 2 MAC).  With a schedule, a shift layer by
+    k uses both maps on the n - k positions that have a predecessor k back."""
+    if dims is None:
+        return 9.0 * d * d * B * n * L
+    per_token = 0.0
+    for s in dims:
+        frac = 0.5 if s >= 0 else (n + s) / n
+        per_token += 3.0 * (2.0 * d * d + 2.0 * d * d * frac)
+    return per_token * B * n
 
 
 class ClockSampler:
@@ -213,12 +225,13 @@ def recorded_traffic(kernel: str):
 
 # ---------------------------------------------------------------- oracle timing
 
-def time_oracle(w, seconds_target: float, seed: int = 0, max_seqs: int = 64):
+def time_oracle(w, seconds_target: float, seed: int = 0, max_seqs: int = 64, dims=None):
     """Time the fp64 oracle's stack forward + backward on a bounded sample of
-    the workload (whole sequences); returns (tokens/s, seconds, sequences, threads)."""
+    the workload (whole sequences), on the layer schedule dims if given;
+    returns (tokens/s, seconds, sequences, threads)."""
     from oracle import oracle as O
     from paper_2609_18145_gb300 import synth
-    n, d, L = w["n"], w["d"], w["L"]
+    n, d, L = w["n"], w["d"], w["L"] if dims is None else len(dims)
 
     def run(seqs):
         pr = synth.problem(seqs, n, d, L=L, seed=seed, w_std=(1 / (2 * d)) ** 0.5,
@@ -229,8 +242,8 @@ def time_oracle(w, seconds_target: float, seed: int = 0, max_seqs: int = 64):
         _, dy = synth.to_bf16_exact(pr.dy)
         t0 = time.perf_counter()
         _, acts, zs = O.stack_fwd(x, Ws, Wn, pr.bias.astype(np.float64), 0, L, -1, w["flags"],
-                                  round_bf16=True)
-        O.stack_bwd(acts, zs, dy, Ws, Wn, 0, L, -1, w["flags"], round_bf16=True)
+                                  round_bf16=True, dims=dims)
+        O.stack_bwd(acts, zs, dy, Ws, Wn, 0, L, -1, w["flags"], round_bf16=True, dims=dims)
         return time.perf_counter() - t0
 
     t1 = run(1)
@@ -313,6 +326,9 @@ def run_ours(args):
 
     w = workload()
     B, n, d, L, flags = w["B"], w["n"], w["d"], w["L"], w["flags"]
+    dims = SCHEDULES[args.schedule]
+    if dims is not None:
+        L = len(dims)
     tokens = B * n
     peaks, peak_src = load_peaks()
 
@@ -342,9 +358,9 @@ def run_ours(args):
 
     def step_calls(xin, dyin):
         H.hcw_stack_fwd(xin, Ws, Wn, bias, 0, -1, flags, y=y, acts=acts, masks=masks,
-                        workspace=fws)
+                        workspace=fws, dims=dims)
         H.hcw_stack_bwd(xin, acts, masks, dyin, Ws, Wn, 0, -1, flags, dx=dx, dW_self=gWs,
-                        dW_nbr=gWn, dbias=gb, workspace=ws)
+                        dW_nbr=gWn, dbias=gb, workspace=ws, dims=dims)
 
     def capture(xin, dyin):
         # the step's launches, recorded once and replayed: no host work per step
@@ -424,36 +440,59 @@ def run_ours(args):
                                                                     L)),
                       dtype=torch.uint8, device=dev)
     reps = 5
-    fwd_ms = time_calls(lambda i: H.hcw_stack_fwd(x, Ws, Wn, bias, 0, -1, flags, y=y, acts=acts,
-                                                  masks=masks, workspace=fws), reps)
-    dx_ms = time_calls(lambda i: H.hcw_stack_bwd_data(masks, dy, Ws, Wn, 0, -1, flags, dx=dx,
-                                                      dz=dz_all, workspace=dws), reps)
-    dw_ms = time_calls(lambda i: H.hcw_stack_bwd_weight(x, acts, dz_all, 0, -1, flags,
-                                                        dW_self=gWs, dW_nbr=gWn, want_dbias=False,
-                                                        workspace=wws), reps)
-    dwb_ms = time_calls(lambda i: H.hcw_stack_bwd_weight(x, acts, dz_all, 0, -1, flags,
-                                                         dW_self=gWs, dW_nbr=gWn, dbias=gb,
-                                                         workspace=wws), reps)
-    launch_flops = 3.0 * d * d * tokens * L     # per stacked launch, 16 causal layers
-    family = H.hcw_stack_kernels_used(B, n, d)
-    if family == H.HCW_STACK_RESIDENT:
-        fwd_name = ("hcw_res_kernel<FWD,%d> (resident stacked forward: 256 tokens per SM pair "
-                    "through all layers)" % d)
-        dx_name = ("hcw_res_kernel<DX,%d> (resident stacked input gradient, top dz included)"
-                   % d)
+    if dims is not None:
+        # a schedule with shift layers runs layer by layer: time its forward and
+        # its backward (input and weight gradients) as two launch sequences
+        f_ms = time_calls(lambda i: H.hcw_stack_fwd(x, Ws, Wn, bias, 0, -1, flags, y=y,
+                                                    acts=acts, masks=masks, workspace=fws,
+                                                    dims=dims), reps)
+        b_ms = time_calls(lambda i: H.hcw_stack_bwd(x, acts, masks, dy, Ws, Wn, 0, -1, flags,
+                                                    dx=dx, dW_self=gWs, dW_nbr=gWn, dbias=gb,
+                                                    workspace=ws, dims=dims), reps)
+        f_flops = step_flops(B, n, d, L, dims) / 3.0
+        kflops = {"forward of the %s schedule, layer by layer" % args.schedule: f_flops,
+                  "backward of the %s schedule (input and weight gradients), layer by layer"
+                  % args.schedule: 2.0 * f_flops}
+        kernels = dict(zip(kflops, (f_ms, b_ms)))
+        dwb_ms = dw_ms = 0.0
     else:
-        fwd_name = "hcw_tc_kernel<FWD,256,16> (stacked forward on SM pairs)"
-        dx_name = "hcw_tc_kernel<DX,256,16> (stacked input gradient on SM pairs, top dz included)"
-    kernels = {fwd_name: fwd_ms, dx_name: dx_ms,
-               "hcw_dwp_kernel<256> (weight and bias gradients on SM pairs, a unit per layer "
-               "and 256 x 256 output tile)": dw_ms}
+        kflops = None
+        fwd_ms = time_calls(lambda i: H.hcw_stack_fwd(x, Ws, Wn, bias, 0, -1, flags, y=y,
+                                                      acts=acts, masks=masks, workspace=fws),
+                            reps)
+    family = H.hcw_stack_kernels_used(B, n, d)
+    if dims is None:
+        dx_ms = time_calls(lambda i: H.hcw_stack_bwd_data(masks, dy, Ws, Wn, 0, -1, flags,
+                                                          dx=dx, dz=dz_all, workspace=dws), reps)
+        dw_ms = time_calls(lambda i: H.hcw_stack_bwd_weight(x, acts, dz_all, 0, -1, flags,
+                                                            dW_self=gWs, dW_nbr=gWn,
+                                                            want_dbias=False, workspace=wws),
+                           reps)
+        dwb_ms = time_calls(lambda i: H.hcw_stack_bwd_weight(x, acts, dz_all, 0, -1, flags,
+                                                             dW_self=gWs, dW_nbr=gWn, dbias=gb,
+                                                             workspace=wws), reps)
+        if family == H.HCW_STACK_RESIDENT:
+            fwd_name = ("hcw_res_kernel<FWD,%d> (resident stacked forward: 256 tokens per SM "
+                        "pair through all layers)" % d)
+            dx_name = ("hcw_res_kernel<DX,%d> (resident stacked input gradient, top dz "
+                       "included)" % d)
+        else:
+            fwd_name = "hcw_tc_kernel<FWD,256,16> (stacked forward on SM pairs)"
+            dx_name = ("hcw_tc_kernel<DX,256,16> (stacked input gradient on SM pairs, top dz "
+                       "included)")
+        kernels = {fwd_name: fwd_ms, dx_name: dx_ms,
+                   "hcw_dwp_kernel<256> (weight and bias gradients on SM pairs, a unit per "
+                   "layer and 256 x 256 output tile)": dw_ms}
+        # per stacked launch, 16 causal layers
+        kflops = {k: 3.0 * d * d * tokens * L for k in kernels}
     dominant = max(kernels, key=kernels.get)
     dom_ms = kernels[dominant]
+    launch_flops = kflops[dominant]
     peak = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
     achieved = launch_flops / (dom_ms * 1e-3) / 1e12
-    per_kernel = {k: {"ms": v, "tflops": launch_flops / (v * 1e-3) / 1e12,
-                      "frac": launch_flops / (v * 1e-3) / 1e12 / peak} for k, v in kernels.items()}
-    step_tflops = step_flops(B, n, d, L) / (ms * 1e-3) / 1e12
+    per_kernel = {k: {"ms": v, "tflops": kflops[k] / (v * 1e-3) / 1e12,
+                      "frac": kflops[k] / (v * 1e-3) / 1e12 / peak} for k, v in kernels.items()}
+    step_tflops = step_flops(B, n, d, L, dims) / (ms * 1e-3) / 1e12
     peak_sus = peaks.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
     traffic = recorded_traffic(dominant.split(" ")[0])
 
@@ -496,10 +535,10 @@ def run_ours(args):
     # ---- the oracle on the host cores, bounded sample (rank 0, N = 1 only)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        v, secs, seqs, threads = time_oracle(w, 10.0)
+        v, secs, seqs, threads = time_oracle(w, 10.0, dims=dims)
         cpu = {"value": v, "unit": "tokens/s", "cores": threads, "kind": "oracle",
-               "sample": "%d of the 64 sequences (n=256), 16 layers fwd+bwd, fp64, %.1f s"
-                         % (seqs, secs)}
+               "sample": "%d of the 64 sequences (n=256), %d layers (%s) fwd+bwd, fp64, %.1f s"
+                         % (seqs, L, args.schedule, secs)}
 
     replicas.barrier()
     if rank == 0:
@@ -513,8 +552,10 @@ def run_ours(args):
                        "act": "relu", "bias": True,
                        "l2": "flushed before every timed step (256 MiB write, untimed)",
                        "parallelism": "replicas" if world > 1 else "single",
-                       "stack_kernels": "resident" if family == H.HCW_STACK_RESIDENT
-                                        else "streaming",
+                       "stack_kernels": ("layer by layer" if dims is not None else
+                                         "resident" if family == H.HCW_STACK_RESIDENT
+                                         else "streaming"),
+                       "schedule": args.schedule,
                        "launch": "host calls" if args.no_graph else "CUDA graph of the step's calls"},
             "roofline": {"bound": "tensor", "kernel": dominant, "achieved": achieved,
                          "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
@@ -524,7 +565,7 @@ def run_ours(args):
             "step_roofline": {"achieved": step_tflops, "peak": peak_sus, "unit": "TFLOP/s",
                               "frac": step_tflops / peak_sus,
                               "peak_source": peak_src + " bf16 sustained",
-                              "flops_per_step": step_flops(B, n, d, L)},
+                              "flops_per_step": step_flops(B, n, d, L, dims)},
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms},
@@ -626,6 +667,9 @@ def main():
                     help="launch only this kernel kind, or one whole step of --batch "
                          "sequences (profiler captures); no JSON bench line")
     ap.add_argument("--batch", type=int, default=64, help="sequences for --kernel runs")
+    ap.add_argument("--schedule", choices=tuple(SCHEDULES), default="rot",
+                    help="layer schedule of the stack: rot (the workload's rotated stack) or "
+                         "hy256 (the near and jump layers of the paper's window-256 hybrid)")
     ap.add_argument("--stack-kernels", choices=tuple(STACK_KERNELS), default="auto",
                     help="kernel family of the stacked forward and input gradient "
                          "(hcw_set_stack_kernels); auto picks the resident kernels for the "

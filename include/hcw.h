@@ -182,8 +182,16 @@ int hcw_stack_fwd(const void* x, const void* W_self, const void* W_nbr, const fl
  * variants of Sec. 4, "Order does not matter; coverage does": a random
  * permutation of the dimensions, a Gray-code order): stack layer l uses cube
  * dimension dims[l] instead of (layer0 + l) mod log2 n.
- *   dims   host array of L ints, each in [0, log2 n), read during the call
- *          (HCW_ERR_INVALID_ARG if NULL or out of range).
+ *   dims   host array of L ints, read during the call (HCW_ERR_INVALID_ARG if
+ *          NULL or out of range).  An entry s in [0, log2 n) is the hypercube
+ *          link along dimension s ("jump 2^s" of App. A); an entry -k with
+ *          1 <= k < n is Eq. (1)'s shift itself: position i takes x_{i-k}
+ *          when i >= k within its sample ("near" of App. A is -1, the
+ *          "local" schedule of Sec. 3.3).  A shift links the earlier position
+ *          to the later one whether or not HCW_CAUSAL is set.
+ * Schedules with a shift layer run layer by layer (bf16: the single-layer
+ * tensor-core launches, the shifted partner rows materialised row-aligned in
+ * the workspace); others run on the stacked launches.
  * Every other argument, the workspace and the outputs as for hcw_stack_fwd;
  * hcw_stack_bwd_dims with the same dims is its backward.
  */
@@ -217,7 +225,7 @@ int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void
 
 /*
  * Backward of hcw_stack_fwd_dims: hcw_stack_bwd with the schedule dims (host
- * array of L ints in [0, log2 n), as given to the forward).
+ * array of L layers, as given to the forward).
  */
 int hcw_stack_bwd_dims(const void* x, const void* acts, const void* masks, const void* dy,
                        const void* W_self, const void* W_nbr, const int* dims, int L, int B,

@@ -207,11 +207,22 @@ struct Sched {
     const int* dims;
     int layer0;
     int dim_override;
+    // s >= 0: hypercube dimension; s < 0: shift of Eq. (1) by -s (schedules only)
     int dim(const Shape& sh, int l) const {
         if (dims) return dims[l];
         return dim_override >= 0 ? dim_override : (layer0 + l) % sh.b;
     }
+    bool has_shift(int L) const {
+        if (!dims) return false;
+        for (int l = 0; l < L; ++l)
+            if (dims[l] < 0) return true;
+        return false;
+    }
 };
+
+// Row grouping of a shift layer's launches: any cube dimension serves (the
+// partner rows come row-aligned from a second tensor); 2^6 = 64-row runs.
+int shift_group_dim(const Shape& sh) { return sh.b - 1 < 6 ? sh.b - 1 : 6; }
 
 // Bytes of one layer's ReLU mask: ceil(d/32) 32-bit words per token.
 size_t mask_bytes(const Shape& sh) { return (size_t)sh.tokens * ((sh.d + 31) / 32) * 4; }
@@ -338,14 +349,20 @@ bool fwd_maps(CUtensorMap* m, const Shape& sh, int s, const void* x, const void*
     return true;
 }
 
+// xpair (a shift layer): the partner part reads the same rows of xpair, and
+// every row takes both parts.
 int fwd_bf16(const Shape& sh, const void* x, const void* Ws, const void* Wn, const float* bias,
-             unsigned flags, void* y, void* z, uint32_t* mask, cudaStream_t st) {
+             unsigned flags, void* y, void* z, uint32_t* mask, cudaStream_t st,
+             const void* xpair = nullptr) {
     const int BN = pick_bn(sh.d);
     TcLaunch<1> L;
     memset(&L, 0, sizeof(L));
     if (!fwd_maps(L.maps[0], sh, sh.s, x, Ws, Wn, y)) return HCW_ERR_CUDA;
+    if (xpair && !map_rows(&L.maps[0][5], xpair, sh.tokens, sh.d, 1 << sh.s, 128))
+        return HCW_ERR_CUDA;
     L.layer[0] = {sh.s, 1 << sh.s, bias, mask, static_cast<__nv_bfloat16*>(z), true, nullptr, false};
-    row_unit_params(L.p, sh, BN, flags, false);
+    L.layer[0].pair_rows = xpair != nullptr;
+    row_unit_params(L.p, sh, BN, xpair ? flags & ~HCW_CAUSAL : flags, false);
     L.p.flags = flags;
     L.n_layers = 1;
     const int sms = sm_count();
@@ -461,9 +478,11 @@ int stack_fwd_resident(const Shape& sh, int l0, int n, const Sched& sc,
 }
 
 // dx: a row gathers dz from its partner exactly when the partner received from it
+// dzpair (a shift layer): the partner part reads the same rows of dzpair
+// (the dz of each row's reader), and every row takes both parts.
 int dx_bf16(const Shape& sh, const void* dz, const void* dy, const void* Ws, const void* Wn,
             unsigned flags, void* dx, cudaStream_t st, const uint32_t* mprev = nullptr,
-            void* dz_out = nullptr) {
+            void* dz_out = nullptr, const void* dzpair = nullptr) {
     const int d = sh.d, BN = pick_bn(d), k = 1 << sh.s;
     const int pw = epi_patch_cols(BN);
     TcLaunch<1> L;
@@ -477,8 +496,10 @@ int dx_bf16(const Shape& sh, const void* dz, const void* dy, const void* Ws, con
         !map_rows(&maps[4], dx ? dx : dz_out, sh.tokens, d, k, 32, pw) ||
         !map_rows(&maps[5], dz_out ? dz_out : dx, sh.tokens, d, k, 32, pw))
         return HCW_ERR_CUDA;
+    if (dzpair && !map_rows(&maps[5], dzpair, sh.tokens, d, k, 128)) return HCW_ERR_CUDA;
     L.layer[0] = {sh.s, k, nullptr, nullptr, nullptr, dx != nullptr, mprev, dz_out != nullptr};
-    row_unit_params(L.p, sh, BN, flags, true);
+    L.layer[0].pair_rows = dzpair != nullptr;
+    row_unit_params(L.p, sh, BN, dzpair ? flags & ~HCW_CAUSAL : flags, true);
     L.p.flags = flags & HCW_RESIDUAL;
     L.n_layers = 1;
     const int sms = sm_count();
@@ -537,6 +558,50 @@ int dw_bf16(const Shape& sh, const void* x, const void* dz, unsigned flags, floa
                                            st),
                         2);
     return HCW_OK;
+}
+
+// dW[o][k] = sum_t a[t][o] x[t][k]: the self part of the weight gradient alone
+// (dW_self with a = dz; for a shift layer also dW_nbr, with a = the readers' dz).
+int dw_self_bf16(const Shape& sh, const void* x, const void* a, unsigned flags, float* dW,
+                 uint8_t* wws, cudaStream_t st) {
+    const int d = sh.d, BN = pick_bn(d), k = 1 << sh.s;
+    const WPlan w = plan_dw(sh.tokens, d, flags);
+    TcLaunch<1> L;
+    memset(&L, 0, sizeof(L));
+    CUtensorMap* maps = L.maps[0];
+    float* part = reinterpret_cast<float*>(wws);
+    if (!map_rows_blocks(&maps[0], a, sh.tokens, d, k, 64, 2) ||
+        !map_rows_blocks(&maps[1], x, sh.tokens, d, k, 64, BN / 64) ||
+        !map_f32_patches(&maps[3], w.splits_max > 1 ? (const void*)part : (const void*)dW,
+                         w.splits_max > 1 ? 2ll * w.splits_max * d : d, d) ||
+        !map_f32_patches(&maps[4], dW, d, d))
+        return HCW_ERR_CUDA;
+    maps[2] = maps[1];   // unused
+    maps[5] = maps[4];   // unused: no partner part
+    L.layer[0] = {sh.s, k, nullptr, nullptr, nullptr, false, nullptr, false};
+    TcParams& p = L.p;
+    p.d = d;
+    p.Mh = (int)(sh.tokens / 2);
+    p.n_nt = w.n_nt;
+    p.n_ot = w.n_ot;
+    p.qb = w.qb;
+    p.nkb_self = w.nkb_self;
+    p.nkb_nbr = w.nkb_nbr;
+    p.kb_per_unit = w.kb_per_unit;
+    p.splits_self = w.splits_self;   // the plan's split of the self part: fits the partials
+    p.splits_nbr = 0;
+    p.splits_max = w.splits_max;
+    p.causal = 0;
+    p.n_units = w.n_ot * w.n_nt * w.splits_self;
+    p.timeout_ns = g_timeout_ns;
+    L.n_layers = 1;
+    const int sms = sm_count();
+    const int grid = p.n_units < sms ? p.n_units : sms;
+    int rc = launched(launch_tc(MODE_DW, BN, L, grid, st), 1);
+    if (rc) return rc;
+    if (w.splits_self > 1)
+        rc = launched(launch_splitk_reduce(part, w.splits_max, w.splits_self, 0, d, dW, dW, st), 1);
+    return rc;
 }
 
 int fwd_f32(const Shape& sh, const void* x, const void* Ws, const void* Wn, const float* bias,
@@ -644,7 +709,9 @@ size_t stack_g_region(const Shape& sh, unsigned flags, int L) {
     const size_t a = align256(sh.act_bytes);
     const bool keep_g = (flags & HCW_ACT_RELU) && (flags & HCW_RESIDUAL);
     size_t r = keep_g ? (size_t)L * a : 0;
-    if (res_supported(sh.d, sh.n, sh.tokens) && r < 2 * a) r = 2 * a;
+    // schedules with shift layers run layer by layer: two g buffers in turn and
+    // the readers' dz of a shift layer
+    if (r < 3 * a) r = 3 * a;
     return r;
 }
 
@@ -654,9 +721,11 @@ size_t stack_data_ws(const Shape& sh, int dtype, unsigned flags, int L) {
     return 2 * a;
 }
 
+// bf16: [unit counter (256 B)][weight-gradient workspace][the readers' dz of a
+// shift layer (one activation buffer)]
 size_t stack_weight_ws(const Shape& sh, int dtype, unsigned flags, int L) {
     const WsLayout w = ws_layout(sh.tokens, sh.d, dtype, flags);
-    if (dtype == HCW_BF16) return 256 + w.w_bytes;
+    if (dtype == HCW_BF16) return 256 + align256(w.w_bytes) + align256(sh.act_bytes);
     return w.w_bytes;
 }
 
@@ -751,7 +820,54 @@ int stack_data_resident(const Shape& sh, const StackData& a, cudaStream_t st) {
 // bf16 input gradients: the ReLU gradient of the top layer, then one stacked
 // launch per run of <= 16 layers, top down, whose kernel also applies the
 // ReLU gradient of the layer below.
+// bf16 input gradients of a schedule with shift layers, layer by layer: dz_l
+// from the ReLU gradient (or a copy of g), then the layer's input gradient --
+// a shift layer with the readers' dz, S_{-k} dz, as its row-aligned partner.
+int stack_data_layers_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
+    const int d = sh.d, L = a.L;
+    const bool relu = (a.flags & HCW_ACT_RELU) != 0;
+    const size_t ab = sh.act_bytes, a256 = align256(ab), wb = (size_t)d * d * 2;
+    const size_t mb = mask_bytes(sh);
+    void* gbuf[2] = {a.ws, a.ws + a256};
+    void* v = a.ws + 2 * a256;
+    const void* g = a.dy;
+    int rc;
+    for (int l = L - 1; l >= 0; --l) {
+        void* dzl = a.dz + (size_t)l * ab;
+        if (relu)
+            rc = launched(launch_relu_grad_mask_bf16(
+                              static_cast<const __nv_bfloat16*>(g),
+                              reinterpret_cast<const uint32_t*>(static_cast<const uint8_t*>(a.masks) +
+                                                                (size_t)l * mb),
+                              static_cast<__nv_bfloat16*>(dzl), sh.tokens, d, st),
+                          1);
+        else
+            rc = cuda_status(cudaMemcpyAsync(dzl, g, ab, cudaMemcpyDeviceToDevice, st));
+        if (rc) return rc;
+        void* out = l == 0 ? a.dx : gbuf[l & 1];
+        const int s = a.sc.dim(sh, l);
+        Shape shl = sh;
+        if (s >= 0) {
+            shl.s = s;
+            rc = dx_bf16(shl, dzl, g, a.Ws + l * wb, a.Wn + l * wb, a.flags, out, st);
+        } else {
+            rc = launched(launch_shift_rows_bf16(static_cast<const __nv_bfloat16*>(dzl),
+                                                 static_cast<__nv_bfloat16*>(v), sh.tokens, sh.n,
+                                                 d, s, st),
+                          1);
+            if (rc) return rc;
+            shl.s = shift_group_dim(sh);
+            rc = dx_bf16(shl, dzl, g, a.Ws + l * wb, a.Wn + l * wb, a.flags, out, st, nullptr,
+                         nullptr, v);
+        }
+        if (rc) return rc;
+        g = out;
+    }
+    return HCW_OK;
+}
+
 int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
+    if (a.sc.has_shift(a.L)) return stack_data_layers_bf16(sh, a, st);
     if (use_resident(sh)) return stack_data_resident(sh, a, st);
     const int d = sh.d, BN = pick_bn(d), L = a.L;
     const bool relu = (a.flags & HCW_ACT_RELU) != 0;
@@ -831,6 +947,44 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
     const size_t ab = sh.act_bytes;
     const WsLayout wl = ws_layout(sh.tokens, d, HCW_BF16, a.flags);
     int* sched = reinterpret_cast<int*>(a.ws);
+    if (a.sc.has_shift(L)) {
+        // layer by layer; a shift layer's dW_nbr = sum_t (S_{-k} dz)_t^T x_t, the
+        // self-part GEMM of the readers' dz against the layer input
+        uint8_t* wws = a.ws + 256;
+        void* v = a.ws + 256 + align256(wl.w_bytes);
+        for (int l = 0; l < L; ++l) {
+            const void* xl =
+                l == 0 ? a.x : static_cast<const uint8_t*>(a.acts) + (size_t)(l - 1) * ab;
+            const void* dzl = a.dz + (size_t)l * ab;
+            float* gs = a.dWs + (size_t)l * d * d;
+            float* gn = a.dWn + (size_t)l * d * d;
+            float* gb = a.dbias ? a.dbias + (size_t)l * d : nullptr;
+            const int s = a.sc.dim(sh, l);
+            Shape shl = sh;
+            int rc;
+            if (s >= 0) {
+                shl.s = s;
+                rc = dw_bf16(shl, xl, dzl, a.flags, gs, gn, gb, wws, st);
+            } else {
+                shl.s = shift_group_dim(sh);
+                rc = dw_self_bf16(shl, xl, dzl, a.flags, gs, wws, st);
+                if (!rc)
+                    rc = launched(launch_shift_rows_bf16(static_cast<const __nv_bfloat16*>(dzl),
+                                                         static_cast<__nv_bfloat16*>(v),
+                                                         sh.tokens, sh.n, d, s, st),
+                                  1);
+                if (!rc) rc = dw_self_bf16(shl, xl, v, a.flags, gn, wws, st);
+                if (!rc && gb)
+                    rc = launched(launch_colsum_bf16(static_cast<const __nv_bfloat16*>(dzl),
+                                                     sh.tokens, d,
+                                                     reinterpret_cast<float*>(wws + wl.col_off),
+                                                     gb, st),
+                                  2);
+            }
+            if (rc) return rc;
+        }
+        return HCW_OK;
+    }
     uint8_t* wws = a.ws + 256;
     auto dz = [&](int l) -> const void* { return a.dz + (size_t)l * ab; };
     auto act = [&](int l) -> const void* {
@@ -1073,11 +1227,13 @@ int check_bwd_ptrs(const Shape& sh, int dtype, unsigned flags, const void* x, co
     return HCW_OK;
 }
 
-// A schedule array of L cube dimensions, each in [0, log2 n).
+// A schedule array of L layers: a cube dimension in [0, log2 n), or a shift
+// -k with 1 <= k < n.
 int check_dims(const Shape& sh, const int* dims, int L) {
     if (!dims) return HCW_ERR_INVALID_ARG;
     for (int l = 0; l < L; ++l)
-        if (dims[l] < 0 || dims[l] >= sh.b) return HCW_ERR_INVALID_ARG;
+        if (dims[l] >= sh.b || (dims[l] < 0 && -(long long)dims[l] >= sh.n))
+            return HCW_ERR_INVALID_ARG;
     return HCW_OK;
 }
 
@@ -1117,6 +1273,34 @@ int stack_fwd_impl(const Shape& sh, const void* x, const void* W_self, const voi
         return want_mask ? reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(masks) + (size_t)l * mb)
                          : nullptr;
     };
+    if (dtype == HCW_BF16 && sc.has_shift(L)) {
+        // layer by layer; a shift layer reads its partner rows S_k x, materialised
+        // row-aligned behind the counters of the workspace
+        void* u = static_cast<uint8_t*>(workspace) + stack_counter_bytes(sh.tokens, L);
+        for (int l = 0; l < L; ++l) {
+            const int s = sc.dim(sh, l);
+            Shape shl = sh;
+            const uint8_t* ws_l = static_cast<const uint8_t*>(W_self) + l * wb;
+            const uint8_t* wn_l = static_cast<const uint8_t*>(W_nbr) + l * wb;
+            const float* b_l = bias ? bias + (size_t)l * d : nullptr;
+            if (s >= 0) {
+                shl.s = s;
+                rc = fwd_bf16(shl, in_ptr(l), ws_l, wn_l, b_l, flags, out_ptr(l), nullptr,
+                              mask_ptr(l), st);
+            } else {
+                rc = launched(launch_shift_rows_bf16(static_cast<const __nv_bfloat16*>(in_ptr(l)),
+                                                     static_cast<__nv_bfloat16*>(u), sh.tokens,
+                                                     n, d, -s, st),
+                              1);
+                if (rc) return rc;
+                shl.s = shift_group_dim(sh);
+                rc = fwd_bf16(shl, in_ptr(l), ws_l, wn_l, b_l, flags, out_ptr(l), nullptr,
+                              mask_ptr(l), st, u);
+            }
+            if (rc) return rc;
+        }
+        return HCW_OK;
+    }
     if (dtype == HCW_BF16) {
         // up to kMaxStackLayers layers per persistent launch
         for (int l0 = 0; l0 < L; l0 += kMaxStackLayers) {
@@ -1334,7 +1518,10 @@ int hcw_layer_bwd_weight(const void* x, const void* dz, int layer, int dim_overr
 size_t hcw_stack_fwd_workspace_bytes(int B, int n, int d, int dtype, unsigned flags, int L) {
     Shape sh;
     if (L < 1 || check_shape(0, -1, B, n, d, dtype, flags, &sh)) return 0;
-    return dtype == HCW_BF16 && sh.tokens > 0 ? stack_counter_bytes(sh.tokens, L) : 0;
+    // bf16: the stacked launches' counters, then the shifted input of a shift layer
+    return dtype == HCW_BF16 && sh.tokens > 0
+               ? stack_counter_bytes(sh.tokens, L) + align256(sh.act_bytes)
+               : 0;
 }
 
 int hcw_stack_fwd(const void* x, const void* W_self, const void* W_nbr, const float* bias,

@@ -61,6 +61,10 @@ struct TcLayer {
     float* colsum;                // DW, whole token range per unit: dbias = column sums of dz
     float* dws;                   // MODE_DWF: dW_self, dW_nbr [d][d] fp32 (stored directly)
     float* dwn;
+    // FWD / DX of one layer: the partner part reads the same rows of a second
+    // tensor (map 5) instead of the partner rows of map 0 -- a shift layer of
+    // Eq. (1), whose partner rows are materialised row-aligned beforehand
+    bool pair_rows;
 };
 
 // Columns of one epilogue patch (the inner extent of the 32-row residual and
@@ -197,6 +201,10 @@ cudaError_t launch_splitk_reduce(const float* partial, int splits_max, int split
                                  int splits_nbr, int d, float* dWs, float* dWn,
                                  cudaStream_t st);
 cudaError_t launch_partner_table(int s, int n, unsigned flags, int* out, cudaStream_t st);
+// out[b][i] = in[b][i - k] where 0 <= i - k < n, else 0 (bf16 [rows][d], k of
+// either sign): the row-aligned partner operand of a shift layer.
+cudaError_t launch_shift_rows_bf16(const __nv_bfloat16* in, __nv_bfloat16* out, long long rows,
+                                   int n, int d, int k, cudaStream_t st);
 cudaError_t launch_wait_selftest(unsigned long long timeout_ns, cudaStream_t st);
 // Read the current device's error word and reset it to 0 (synchronous).
 cudaError_t error_word_read_clear(int* word);

@@ -5,18 +5,29 @@
 //     mask, deterministic column sums (dbias), split-K reduction of dW;
 //   * the device partner table (same index code as the kernels).
 //
-// Index rules (Sec. 3.1): partner p(i) = i XOR 2^s inside each sample;
-// causal: i receives from p(i) iff bit s of i is set.
+// Index rules, per layer link s inside each sample of n positions:
+//   s >= 0 (Sec. 3.1): partner p(i) = i XOR 2^s; causal: i receives from p(i)
+//          iff bit s of i is set;
+//   s < 0  (Eq. (1) with k = -s, "near" of App. A is k = 1): p(i) = i - k, and
+//          i receives iff i >= k (a shift always links earlier to later).
 #include "hcw_internal.h"
 
 namespace hcw {
 
 namespace {
 
-__device__ __forceinline__ int partner_of(int i, int s) { return i ^ (1 << s); }
+__device__ __forceinline__ int partner_of(int i, int s) { return s >= 0 ? i ^ (1 << s) : i + s; }
 
 __device__ __forceinline__ bool receives(int i, int s, unsigned flags) {
+    if (s < 0) return i + s >= 0;
     return !(flags & 1u) || ((i >> s) & 1);
+}
+
+// the position that takes x_i as its partner input at link s, or -1
+__device__ __forceinline__ int reader_of(int i, int s, int n, unsigned flags) {
+    if (s < 0) return i - s < n ? i - s : -1;
+    const int p = i ^ (1 << s);
+    return receives(p, s, flags) ? p : -1;
 }
 
 constexpr int T = 32;   // tile edge of the fp32 kernels
@@ -41,9 +52,8 @@ __global__ void f32_fwd_kernel(const float* __restrict__ x, const float* __restr
             float a = 0.f, b = 0.f;
             if (r < rows && k < d) {
                 const int i = (int)(r % n);
-                const long long rp = r - i + partner_of(i, s);
                 a = x[r * d + k];
-                b = receives(i, s, flags) ? x[rp * d + k] : 0.f;
+                b = receives(i, s, flags) ? x[(r - i + partner_of(i, s)) * d + k] : 0.f;
             }
             xs[rr][tx] = a;
             xp[rr][tx] = b;
@@ -100,10 +110,9 @@ __global__ void f32_dx_kernel(const float* __restrict__ dz, const float* __restr
             float a = 0.f, b = 0.f;
             if (r < rows && o < d) {
                 const int i = (int)(r % n);
-                const int pi = partner_of(i, s);
-                const long long rp = r - i + pi;
+                const int j = reader_of(i, s, n, flags);
                 a = dz[r * d + o];
-                b = receives(pi, s, flags) ? dz[rp * d + o] : 0.f;
+                b = j >= 0 ? dz[(r - i + j) * d + o] : 0.f;
             }
             gs[rr][tx] = a;
             gp[rr][tx] = b;
@@ -150,11 +159,10 @@ __global__ void f32_dw_kernel(const float* __restrict__ x, const float* __restri
             float g = 0.f, a = 0.f, b = 0.f;
             if (r < rows) {
                 const int i = (int)(r % n);
-                const long long rp = r - i + partner_of(i, s);
                 if (o0 + tx < d) g = dz[r * d + o0 + tx];
                 if (k0 + tx < d) {
                     a = x[r * d + k0 + tx];
-                    b = receives(i, s, flags) ? x[rp * d + k0 + tx] : 0.f;
+                    b = receives(i, s, flags) ? x[(r - i + partner_of(i, s)) * d + k0 + tx] : 0.f;
                 }
             }
             gz[rr][tx] = g;
@@ -343,6 +351,22 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ partial, int spli
     }
 }
 
+// out[b][i] = in[b][i - k] for 0 <= i - k < n, else 0 (k of either sign):
+// the partner rows of a shift layer (k > 0) or their readers (k < 0), as a
+// row-aligned second operand.  One thread per 16-byte piece.
+__global__ void shift_rows_kernel(const uint4* __restrict__ in, uint4* __restrict__ out,
+                                  long long rows, int n, int pieces, int k) {
+    const long long total = rows * pieces;
+    for (long long t = (long long)blockIdx.x * blockDim.x + threadIdx.x; t < total;
+         t += (long long)gridDim.x * blockDim.x) {
+        const long long r = t / pieces;
+        const int c = (int)(t - r * pieces);
+        const int i = (int)(r % n);
+        const int j = i - k;
+        out[t] = (j >= 0 && j < n) ? in[(r - i + j) * pieces + c] : make_uint4(0, 0, 0, 0);
+    }
+}
+
 __global__ void partner_table_kernel(int s, int n, unsigned flags, int* out) {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i < n) out[i] = receives(i, s, flags) ? partner_of(i, s) : -1;
@@ -455,6 +479,14 @@ cudaError_t launch_splitk_reduce(const float* partial, int splits_max, int split
     const size_t total4 = (size_t)d * d / 4;
     splitk_reduce_kernel<<<blocks_for(2 * total4, 256), 256, 0, st>>>(
         partial, splits_max, splits_self, splits_nbr, d, dWs, dWn);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_shift_rows_bf16(const __nv_bfloat16* in, __nv_bfloat16* out, long long rows,
+                                   int n, int d, int k, cudaStream_t st) {
+    const int pieces = d / 8;   // d % 64 == 0 on the bf16 path
+    shift_rows_kernel<<<blocks_for((size_t)rows * pieces, 256), 256, 0, st>>>(
+        reinterpret_cast<const uint4*>(in), reinterpret_cast<uint4*>(out), rows, n, pieces, k);
     return cudaGetLastError();
 }
 

@@ -553,13 +553,17 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                         issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
                         const int part = ks >= p.nK;
                         const int kk = part ? ks - p.nK : ks;
-                        const int bitA = part ? 1 - r.beta : r.beta;
+                        // partner part: the rows of the other bit value, or (pair_rows)
+                        // the same rows of the row-aligned partner tensor (map 5)
+                        const bool same = part && ly.pair_rows;
+                        const int bitA = part && !same ? 1 - r.beta : r.beta;
+                        const CUtensorMap* mAk = same ? &L.maps[l][5] : mA;
                         const CUtensorMap* mb = &L.maps[l][part ? 2 : 1];
                         if (PAIR) {
                             // both CTAs' copies complete on the leader's barrier
                             if (rank == 0) mbar_arrive_expect_tx(&bars->full[stage], 2 * SB);
                             const uint32_t fb = mapa_shared(&bars->full[stage], 0);
-                            tma_load_4d_pair(sA, mA, fb, kk * kBlockK, lo0, bitA, hi0);
+                            tma_load_4d_pair(sA, mAk, fb, kk * kBlockK, lo0, bitA, hi0);
                             if (MODE == MODE_FWD)
                                 tma_load_2d_pair(sB, mb, fb, kk * kBlockK,
                                                  r.j * BN + (int)rank * (BN / 2));
@@ -568,7 +572,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                                                  r.j * (BN / 64) + (int)rank * (BN / 128));
                         } else {
                             mbar_arrive_expect_tx(&bars->full[stage], kABytes + B_BYTES);
-                            tma_load_4d(sA, mA, &bars->full[stage], kk * kBlockK, lo0, bitA, hi0);
+                            tma_load_4d(sA, mAk, &bars->full[stage], kk * kBlockK, lo0, bitA, hi0);
                             if (MODE == MODE_FWD)
                                 tma_load_2d(sB, mb, &bars->full[stage], kk * kBlockK, r.j * BN);
                             else   // BN / 64 blocks of 64 W columns x 64 rows, one copy

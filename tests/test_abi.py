@@ -230,13 +230,20 @@ def test_stack_kernel_selection_is_a_process_setting(hcw):
 
 
 def test_schedule_entry_points_reject_bad_dims_before_any_launch(hcw):
-    """hcw_stack_fwd_dims / hcw_stack_bwd_dims check the schedule (one cube
-    dimension in [0, log2 n) per layer) before touching a buffer."""
+    """hcw_stack_fwd_dims / hcw_stack_bwd_dims check the schedule (per layer a
+    cube dimension in [0, log2 n), or a shift -k with 1 <= k < n) before
+    touching a buffer."""
     lib = hcw.lib()
     fake = ctypes.c_void_p(256)   # never dereferenced: the schedule check comes first
     B, n, d, L = 2, 64, 128, 4
     before = hcw.hcw_launch_count()
-    for dims in (None, [0, 1, 6, 2], [0, -1, 2, 3], [5, 4, 3, 64]):
+    # a valid schedule with near (-1) and a shift of 63 gets past the check and
+    # stops at the missing workspace
+    ok = (ctypes.c_int * L)(0, -1, 5, -63)
+    rc = lib.hcw_stack_fwd_dims(fake, fake, fake, None, ctypes.cast(ok, ctypes.c_void_p), L, B, n,
+                                d, hcw.HCW_BF16, 0, fake, fake, None, None, 0, None)
+    assert rc == hcw.HCW_ERR_WORKSPACE
+    for dims in (None, [0, 1, 6, 2], [0, -64, 2, 3], [5, 4, 3, 64]):
         arr = None if dims is None else (ctypes.c_int * L)(*dims)
         ptr = None if arr is None else ctypes.cast(arr, ctypes.c_void_p)
         rc = lib.hcw_stack_fwd_dims(fake, fake, fake, None, ptr, L, B, n, d, hcw.HCW_BF16, 0,

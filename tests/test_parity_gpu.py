@@ -352,6 +352,15 @@ SCHEDULE_CASES = [
      [7, 7, 0, 3, 7, 6, 5, 7]),
     ("n256_dim7_streaming", "streaming", 2, 256, 128, CAUSAL | RESIDUAL | RELU,
      [7, 7, 0, 3, 7, 6, 5, 7]),
+    # shift layers of Eq. (1) (-k; near = -1): the mixa schedule at window 64
+    # (Sec. 3.3: local and long-range layers alternate, jumps 32 .. 1)
+    ("mixa_n64", "auto", 8, 64, 128, CAUSAL | RESIDUAL | RELU,
+     [-1, 5, -1, 4, -1, 3, -1, 2, -1, 1, -1, 0]),
+    # the near and jump layers of the hybrid256 schedule (App. A, attention left out)
+    ("hybrid256_sparse_n256", "auto", 2, 256, 128, CAUSAL | RESIDUAL | RELU,
+     [-1, 7, -1, -1, 5, -1, 4, -1, -1, 2, -1, 1, -1, 0]),
+    # long shifts, no activation, d = 256 tiles
+    ("long_shifts_n128_d256", "auto", 4, 128, 256, RESIDUAL, [-3, -64, 2, -127, -1]),
 ]
 
 
@@ -388,6 +397,33 @@ def test_stack_with_a_schedule_array(H, case):
             assert rel(host(got), ref) <= TOL_BF16, (name, what)
     finally:
         H.hcw_set_stack_kernels(prev)
+
+
+@pytest.mark.parametrize("flags", [CAUSAL | RESIDUAL | RELU, 0])
+def test_shift_schedule_fp32(H, flags):
+    """The fp32 path (CUDA-core kernels) on a schedule of near, jump and shift
+    layers against the oracle at the fp32 tolerance."""
+    B, n, d = 3, 32, 48
+    dims = [-1, 4, -1, 3, -5, 0, -1]
+    L = len(dims)
+    pr = synth.problem(B, n, d, L=L, seed=29, w_std=(1 / (2 * d)) ** 0.5)
+    x, x64 = dev(pr.x, torch.float32)
+    Ws, Ws64 = dev(pr.W_self, torch.float32)
+    Wn, Wn64 = dev(pr.W_nbr, torch.float32)
+    dy, dy64 = dev(pr.dy, torch.float32)
+    bias = torch.from_numpy(pr.bias).cuda()
+    y, acts, masks = H.hcw_stack_fwd_dims(x, Ws, Wn, bias, dims, flags)
+    ry, racts, rzs = O.stack_fwd(x64, Ws64, Wn64, pr.bias.astype(np.float64), 0, L, -1, flags,
+                                 dims=dims)
+    assert rel(host(y), ry) <= TOL_F32 and rel(host(acts), racts[1:]) <= TOL_F32
+    o_acts = torch.from_numpy(racts[1:]).float().cuda()
+    o_masks = masks_from_z(rzs).cuda() if flags & RELU else None
+    dx, gWs, gWn, gb = H.hcw_stack_bwd_dims(x, o_acts, o_masks, dy, Ws, Wn, dims, flags)
+    torch.cuda.synchronize()
+    rdx, rWs, rWn, rgb = O.stack_bwd(racts, rzs, dy64, Ws64, Wn64, 0, L, -1, flags, dims=dims)
+    for got, ref, what in ((dx, rdx, "dx"), (gWs, rWs, "dW_self"), (gWn, rWn, "dW_nbr"),
+                           (gb, rgb, "dbias")):
+        assert rel(host(got), ref) <= TOL_F32, what
 
 
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
