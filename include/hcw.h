@@ -328,6 +328,37 @@ int hcw_set_stack_kernels(int mode);
  */
 int hcw_stack_kernels_used(int B, int n, int d, int dtype);
 
+/*
+ * One decode step of a causal stack, bf16 (Sec. 6, "Deployability": the
+ * decode path runs one token at a time, and a sparse layer needs only the
+ * last k inputs it links to, so its cache does not grow).
+ * B sequences advance together to position t (0 <= t < n of their windows).
+ * Layer l links t to t - k_l (k_l = 2^s for the hypercube link along
+ * dimension s, which t takes when bit s of t is set; k_l = k for a shift,
+ * taken when t >= k); the layers are dims[l] as for hcw_stack_fwd_dims, or
+ * (dims NULL) dimension (layer0 + l) mod log2 n.
+ *   x_t     [B][d]: the layer-0 input at position t.
+ *   y_t     [B][d]: the stack's output at position t (written).
+ *   cache   hcw_decode_cache_bytes(...) bytes: per layer a ring of its last k_l
+ *           inputs, [k_l][B][d] one after another in layer order; slot
+ *           (p mod k_l) holds position p.  The step reads slot t mod k_l (the
+ *           input of position t - k_l) and then overwrites it with the input
+ *           at t.  Slots are read only for partners p >= 0, so the ring needs
+ *           no initialisation; steps must come in order t = 0, 1, ....
+ *   workspace  hcw_decode_workspace_bytes(B, d, L) bytes (the layer inputs).
+ * Needs HCW_CAUSAL (without it a hypercube link reads a later position) and
+ * L <= 64.  y_t equals row t of hcw_stack_fwd over the window to bf16
+ * rounding.  Calls are asynchronous on `stream`.
+ */
+int hcw_decode_step(const void* x_t, const void* W_self, const void* W_nbr, const float* bias,
+                    const int* dims, int layer0, int L, int t, int B, int n, int d,
+                    unsigned flags, void* cache, void* y_t, void* workspace, size_t ws_bytes,
+                    void* stream);
+/* Bytes of the decode rings for this schedule (0 for invalid sizes). */
+size_t hcw_decode_cache_bytes(const int* dims, int layer0, int L, int B, int n, int d);
+/* Workspace bytes of hcw_decode_step. */
+size_t hcw_decode_workspace_bytes(int B, int d, int L);
+
 /* Number of kernels this library has launched in this process (all devices). */
 unsigned long long hcw_launch_count(void);
 

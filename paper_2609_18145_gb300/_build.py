@@ -20,7 +20,7 @@ INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libhcw.so")
 BUILD_DIR = os.path.join(PKG, "_build")
 
-SOURCES = ["hcw_api.cu", "hcw_tc.cu", "hcw_res.cu", "hcw_simt.cu"]
+SOURCES = ["hcw_api.cu", "hcw_tc.cu", "hcw_res.cu", "hcw_simt.cu", "hcw_decode.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
               "--expt-relaxed-constexpr", "-I", INCLUDE, "-I", CSRC]

@@ -1370,6 +1370,21 @@ int stack_bwd_impl(const Shape& sh, const void* x, const void* acts, const void*
     return dtype == HCW_BF16 ? stack_weight_bf16(sh, wa, st) : stack_weight_f32(sh, wa, st);
 }
 
+// Link distance of decode layer l: 2^s for the hypercube link along
+// dimension s, k for a shift by k.
+int decode_link(const int* dims, int layer0, int b, int l) {
+    const int s = dims ? dims[l] : (layer0 + l) % b;
+    return s >= 0 ? 1 << s : -s;
+}
+
+int decode_check(const int* dims, int layer0, int L, int B, int n, int d, Shape* sh) {
+    if (L < 1 || L > kMaxDecodeLayers || B < 1 || layer0 < 0) return HCW_ERR_INVALID_ARG;
+    int rc = check_shape(0, -1, B, n, d, HCW_BF16, 0, sh);
+    if (rc) return rc;
+    if (dims) return check_dims(*sh, dims, L);
+    return HCW_OK;
+}
+
 }  // namespace
 }  // namespace hcw
 
@@ -1637,6 +1652,74 @@ int hcw_stack_bwd_dims(const void* x, const void* acts, const void* masks, const
     if (rc) return rc;
     return stack_bwd_impl(sh, x, acts, masks, dy, W_self, W_nbr, Sched{dims, 0, -1}, L, dtype,
                           flags, dx, dW_self, dW_nbr, dbias, workspace, ws_bytes, stream);
+}
+
+size_t hcw_decode_cache_bytes(const int* dims, int layer0, int L, int B, int n, int d) {
+    Shape sh;
+    if (decode_check(dims, layer0, L, B, n, d, &sh)) return 0;
+    size_t slots = 0;
+    for (int l = 0; l < L; ++l) slots += (size_t)decode_link(dims, layer0, sh.b, l);
+    return slots * (size_t)B * d * 2;
+}
+
+size_t hcw_decode_workspace_bytes(int B, int d, int L) {
+    if (B < 1 || d < 1 || L < 1 || L > kMaxDecodeLayers) return 0;
+    return (size_t)(L > 1 ? L - 1 : 1) * B * d * 2;
+}
+
+int hcw_decode_step(const void* x_t, const void* W_self, const void* W_nbr, const float* bias,
+                    const int* dims, int layer0, int L, int t, int B, int n, int d,
+                    unsigned flags, void* cache, void* y_t, void* workspace, size_t ws_bytes,
+                    void* stream) {
+    Shape sh;
+    int rc = decode_check(dims, layer0, L, B, n, d, &sh);
+    if (rc) return rc;
+    // decoding is causal: a hypercube link without the causal rule would read a
+    // later position
+    if (!(flags & HCW_CAUSAL) || (flags & ~kAllFlags) || t < 0 || t >= n) return HCW_ERR_INVALID_ARG;
+    if (!x_t || !W_self || !W_nbr || !cache || !y_t) return HCW_ERR_INVALID_ARG;
+    const void* ptrs[] = {x_t, W_self, W_nbr, bias, cache, y_t, workspace};
+    for (const void* q : ptrs)
+        if (q && !aligned16(q)) return HCW_ERR_ALIGNMENT;
+    const size_t row_bytes = (size_t)B * d * 2;
+    const size_t need = hcw_decode_workspace_bytes(B, d, L);
+    if (ws_bytes < need || !workspace) return HCW_ERR_WORKSPACE;
+    const size_t cache_b = hcw_decode_cache_bytes(dims, layer0, L, B, n, d);
+    const size_t wb = (size_t)L * d * d * 2;
+    if (overlaps(y_t, row_bytes, x_t, row_bytes) || overlaps(y_t, row_bytes, cache, cache_b) ||
+        overlaps(y_t, row_bytes, workspace, need) || overlaps(workspace, need, cache, cache_b) ||
+        overlaps(workspace, need, x_t, row_bytes) || overlaps(cache, cache_b, x_t, row_bytes) ||
+        overlaps(cache, cache_b, W_self, wb) || overlaps(cache, cache_b, W_nbr, wb))
+        return HCW_ERR_ALIASING;
+    cudaStream_t st = (cudaStream_t)stream;
+    auto* ring = static_cast<__nv_bfloat16*>(cache);
+    auto* inputs = static_cast<__nv_bfloat16*>(workspace);
+    const size_t per = (size_t)B * d;
+    __nv_bfloat16* slots[kMaxDecodeLayers];
+    size_t off = 0;
+    for (int l = 0; l < L; ++l) {
+        const int s = dims ? dims[l] : (layer0 + l) % sh.b;
+        const int k = decode_link(dims, layer0, sh.b, l);
+        const bool recv = s >= 0 ? ((t >> s) & 1) != 0 : t >= k;
+        __nv_bfloat16* slot = ring + off + (size_t)(t % k) * per;
+        slots[l] = slot;
+        const __nv_bfloat16* in = l == 0 ? static_cast<const __nv_bfloat16*>(x_t)
+                                         : inputs + (size_t)(l - 1) * per;
+        __nv_bfloat16* out = l == L - 1 ? static_cast<__nv_bfloat16*>(y_t)
+                                        : inputs + (size_t)l * per;
+        rc = launched(launch_decode_layer(
+                          in, recv ? slot : nullptr,
+                          static_cast<const __nv_bfloat16*>(W_self) + (size_t)l * d * d,
+                          static_cast<const __nv_bfloat16*>(W_nbr) + (size_t)l * d * d,
+                          bias ? bias + (size_t)l * d : nullptr, B, d, flags, out, st),
+                      1);
+        if (rc) return rc;
+        off += (size_t)k * per;
+    }
+    // every layer's input at t into its ring slot (read above as t's partner)
+    return launched(launch_decode_commit(static_cast<const __nv_bfloat16*>(x_t), inputs, slots, L,
+                                         B, d, st),
+                    1);
 }
 
 int hcw_set_stack_kernels(int mode) {

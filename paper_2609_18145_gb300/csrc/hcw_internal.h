@@ -162,6 +162,19 @@ cudaError_t launch_res(int mode, const ResLaunch& L, cudaStream_t stream);
 // Read the resident kernels' error word and reset it to 0 (synchronous).
 cudaError_t res_error_word_read_clear(int* word);
 
+// ---- One-token decode (hcw_decode.cu) ----
+constexpr int kMaxDecodeLayers = 64;   // layers of one decode step
+// out = act(x Ws^T + partner Wn^T + bias) (+ x) for B rows of width d, bf16 in
+// and out, fp32 accumulation; partner null: no partner part.
+cudaError_t launch_decode_layer(const __nv_bfloat16* x, const __nv_bfloat16* partner,
+                                const __nv_bfloat16* Ws, const __nv_bfloat16* Wn,
+                                const float* bias, int B, int d, unsigned flags,
+                                __nv_bfloat16* out, cudaStream_t st);
+// slots[l] <- the input of layer l ([B][d]: x0 for l = 0, inputs[l - 1] after)
+cudaError_t launch_decode_commit(const __nv_bfloat16* x0, const __nv_bfloat16* inputs,
+                                 __nv_bfloat16* const* slots, int L, int B, int d,
+                                 cudaStream_t st);
+
 // Dynamic shared memory the tensor-core kernel uses for this N tile.
 size_t tc_smem_bytes(int BN);
 int tc_stages(int BN);

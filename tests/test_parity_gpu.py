@@ -449,6 +449,48 @@ def test_schedule_array_of_the_rotation_equals_the_rotated_stack(H, dtype):
         assert torch.equal(u, v)
 
 
+DECODE_CASES = [
+    # name, B, n, d, flags, dims (None = rot), layer0, L
+    ("rot_n64", 4, 64, 128, CAUSAL | RESIDUAL | RELU, None, 0, 12),
+    ("rot_n64_from_layer3_no_relu", 3, 64, 64, CAUSAL | RESIDUAL, None, 3, 7),
+    ("mixa_n64", 4, 64, 128, CAUSAL | RESIDUAL | RELU, [-1, 5, -1, 4, -1, 3, -1, 2, -1, 1, -1, 0],
+     0, 12),
+    ("hybrid256_sparse_n256", 2, 256, 128, CAUSAL | RESIDUAL | RELU,
+     [-1, 7, -1, -1, 5, -1, 4, -1, -1, 2, -1, 1, -1, 0], 0, 14),
+]
+
+
+@pytest.mark.parametrize("case", DECODE_CASES, ids=lambda c: c[0])
+def test_decode_steps_reproduce_the_window_forward(H, case):
+    """Sec. 6: decoding one token at a time with bounded rings gives, at every
+    position t, the output row t of the stack run over the whole window: the
+    oracle's forward (bf16 storage) at the bf16 tolerance, and the device's
+    stacked forward likewise."""
+    name, B, n, d, flags, dims, layer0, L = case
+    pr = synth.problem(B, n, d, L=L, seed=31, w_std=(1 / (2 * d)) ** 0.5)
+    x, x64 = dev(pr.x, torch.bfloat16)
+    Ws, Ws64 = dev(pr.W_self, torch.bfloat16)
+    Wn, Wn64 = dev(pr.W_nbr, torch.bfloat16)
+    bias = torch.from_numpy(pr.bias).cuda()
+    cache = torch.empty(H.hcw_decode_cache_bytes(L, B, n, d, dims=dims, layer0=layer0),
+                        dtype=torch.uint8, device="cuda")
+    ys = torch.empty_like(x)
+    for t in range(n):
+        xt = x[:, t].contiguous()
+        ys[:, t] = H.hcw_decode_step(xt, Ws, Wn, bias, t, n, cache, flags, dims=dims,
+                                     layer0=layer0)
+    torch.cuda.synchronize()
+    assert H.hcw_sync_status() == H.HCW_OK
+    ry, _, _ = O.stack_fwd(x64, Ws64, Wn64, pr.bias.astype(np.float64), layer0, L, -1, flags,
+                           round_bf16=True, dims=dims)
+    assert rel(host(ys), ry) <= TOL_BF16, name
+    if dims is None:
+        y, _, _ = H.hcw_stack_fwd(x, Ws, Wn, bias, layer0, -1, flags)
+    else:
+        y, _, _ = H.hcw_stack_fwd_dims(x, Ws, Wn, bias, dims, flags)
+    assert rel(host(ys), host(y)) <= TOL_BF16, name
+
+
 def test_stack_fixed_dimension_control(H):
     pr = synth.problem(16, 64, 128, L=6, seed=5, w_std=(1 / 256) ** 0.5)
     got, ref = run_stack(H, pr, torch.bfloat16, 6, 0, dim=0)
