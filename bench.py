@@ -604,6 +604,8 @@ def run_kernel_only(args):
     wws = torch.empty(max(1, H.hcw_layer_bwd_weight_workspace_bytes(B, n, d, H.HCW_BF16, flags)),
                       dtype=torch.uint8, device=dev)
     layer = 3
+    if args.kernel == "decode":
+        return run_decode(args, w, dev)
     if args.kernel == "step":
         # one whole step (stack forward + stack backward) of --batch sequences
         L = w["L"]
@@ -652,6 +654,74 @@ def run_kernel_only(args):
     return 0
 
 
+def run_decode(args, w, dev):
+    """Decode one whole window of --batch sequences position by position
+    (hcw_decode_step, Sec. 6) with the workload's layers, issued from the host
+    and as one CUDA graph of the window, and print the time per position."""
+    import torch
+
+    from paper_2609_18145_gb300 import hcw as H
+    from paper_2609_18145_gb300 import synth
+
+    B, n, d, L, flags = args.batch, w["n"], w["d"], w["L"], w["flags"]
+    dims = SCHEDULES[args.schedule]
+    if dims is not None:
+        L = len(dims)
+    ps = synth.problem(B, n, d, L=L, seed=0, w_std=(1 / (2 * d)) ** 0.5, x_ids="zipf256")
+    xs = torch.from_numpy(ps.x).to(torch.bfloat16).transpose(0, 1).contiguous().to(dev)  # [n,B,d]
+    Ws = torch.from_numpy(ps.W_self).to(torch.bfloat16).to(dev)
+    Wn = torch.from_numpy(ps.W_nbr).to(torch.bfloat16).to(dev)
+    bias = torch.from_numpy(ps.bias).to(dev)
+    cache = torch.zeros(max(1, H.hcw_decode_cache_bytes(L, B, n, d, dims=dims)), dtype=torch.uint8,
+                        device=dev)
+    ys = torch.empty_like(xs)
+
+    def window():
+        for t in range(n):
+            H.hcw_decode_step(xs[t], Ws, Wn, bias, t, n, cache, flags, dims=dims, y=ys[t])
+
+    def timed(fn, reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        a.record()
+        for _ in range(reps):
+            fn()
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / reps
+
+    for _ in range(max(1, args.warmup)):
+        window()
+    c0 = H.hcw_launch_count()
+    host_ms = timed(window, max(1, args.steps))
+    launches = (H.hcw_launch_count() - c0) / max(1, args.steps) / n
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        window()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            window()
+    torch.cuda.synchronize()
+    g.replay()
+    graph_ms = timed(g.replay, max(1, args.steps))
+    if H.hcw_sync_status() != H.HCW_OK:
+        raise SystemExit("device error")
+    wbytes = 2.0 * L * d * d * 2
+    peaks, _ = load_peaks()
+    us = graph_ms * 1e3 / n
+    print(json.dumps({
+        "kernel": "decode", "batch": B, "n": n, "d": d, "L": L, "schedule": args.schedule,
+        "cache_bytes": cache.numel(), "launches_per_position": launches,
+        "us_per_position_host_issued": round(host_ms * 1e3 / n, 2),
+        "us_per_position_graph": round(us, 2),
+        "tokens_per_s_graph": round(B / (us * 1e-6)),
+        "weight_bytes_per_position": wbytes,
+        "weight_gbs_graph": round(wbytes / (us * 1e-6) / 1e9, 1),
+        "hbm_peak_gbs": peaks.get("hbm_gbs")}), flush=True)
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -663,17 +733,17 @@ def main():
                          "CUDA graph of them")
     ap.add_argument("--no-cpu-baseline", action="store_true",
                     help="skip timing the CPU oracle (it is only timed at N = 1 anyway)")
-    ap.add_argument("--kernel", choices=("fwd", "dx", "dw", "step"),
-                    help="launch only this kernel kind, or one whole step of --batch "
-                         "sequences (profiler captures); no JSON bench line")
+    ap.add_argument("--kernel", choices=("fwd", "dx", "dw", "step", "decode"),
+                    help="launch only this kernel kind, one whole step of --batch sequences "
+                         "(profiler captures), or decode one window of --batch sequences "
+                         "token by token; no bench line")
     ap.add_argument("--batch", type=int, default=64, help="sequences for --kernel runs")
     ap.add_argument("--schedule", choices=tuple(SCHEDULES), default="rot",
                     help="layer schedule of the stack: rot (the workload's rotated stack) or "
                          "hy256 (the near and jump layers of the paper's window-256 hybrid)")
     ap.add_argument("--stack-kernels", choices=tuple(STACK_KERNELS), default="auto",
                     help="kernel family of the stacked forward and input gradient "
-                         "(hcw_set_stack_kernels); auto picks the resident kernels for the "
-                         "bench workload")
+                         "(hcw_set_stack_kernels); auto is the streaming family")
     args = ap.parse_args()
     if args.kernel:
         return run_kernel_only(args)

@@ -339,25 +339,26 @@ int hcw_stack_kernels_used(int B, int n, int d, int dtype);
  * (dims NULL) dimension (layer0 + l) mod log2 n.
  *   x_t     [B][d]: the layer-0 input at position t.
  *   y_t     [B][d]: the stack's output at position t (written).
- *   cache   hcw_decode_cache_bytes(...) bytes: per layer a ring of its last k_l
- *           inputs, [k_l][B][d] one after another in layer order; slot
- *           (p mod k_l) holds position p.  The step reads slot t mod k_l (the
- *           input of position t - k_l) and then overwrites it with the input
- *           at t.  Slots are read only for partners p >= 0, so the ring needs
- *           no initialisation; steps must come in order t = 0, 1, ....
- *   workspace  hcw_decode_workspace_bytes(B, d, L) bytes (the layer inputs).
- * Needs HCW_CAUSAL (without it a hypercube link reads a later position) and
- * L <= 64.  y_t equals row t of hcw_stack_fwd over the window to bf16
- * rounding.  Calls are asynchronous on `stream`.
+ *   cache   hcw_decode_cache_bytes(...) bytes: per layer a ring of k_l + 1
+ *           slots, [k_l + 1][B][d] one after another in layer order; slot
+ *           (p mod (k_l + 1)) holds the layer's input at position p.  The
+ *           step reads the slot of t - k_l, (t + 1) mod (k_l + 1), and writes
+ *           the input at t into slot t mod (k_l + 1), a different one, so every
+ *           layer's output goes straight into the next layer's ring.  Slots are
+ *           read only for partners p >= 0, so the ring needs no
+ *           initialisation; steps must come in order t = 0, 1, ....
+ * The whole step (every layer) is one kernel launch: a cluster of up to 16
+ * CTAs per 16 sequences, exchanging each layer's output in distributed
+ * shared memory.  Needs HCW_CAUSAL (without it a hypercube link reads a later
+ * position), L <= 64 and d <= 1024 (HCW_ERR_UNSUPPORTED above).  y_t equals
+ * row t of hcw_stack_fwd over the window to bf16 rounding.  Calls are
+ * asynchronous on `stream`.
  */
 int hcw_decode_step(const void* x_t, const void* W_self, const void* W_nbr, const float* bias,
                     const int* dims, int layer0, int L, int t, int B, int n, int d,
-                    unsigned flags, void* cache, void* y_t, void* workspace, size_t ws_bytes,
-                    void* stream);
+                    unsigned flags, void* cache, void* y_t, void* stream);
 /* Bytes of the decode rings for this schedule (0 for invalid sizes). */
 size_t hcw_decode_cache_bytes(const int* dims, int layer0, int L, int B, int n, int d);
-/* Workspace bytes of hcw_decode_step. */
-size_t hcw_decode_workspace_bytes(int B, int d, int L);
 
 /* Number of kernels this library has launched in this process (all devices). */
 unsigned long long hcw_launch_count(void);

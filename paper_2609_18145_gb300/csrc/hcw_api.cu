@@ -155,6 +155,24 @@ bool map_weight(CUtensorMap* m, const void* base, int d, int box_o) {
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// bf16 matrix [rows][d] viewed as (64 features, rows, d / 64 tiles), box
+// (64, box_rows, box_tiles), 128-byte swizzle: one copy lands box_tiles
+// consecutive 64-feature tiles of box_rows rows each (the decode's weight
+// chunks, ring rows and inputs).
+bool map_tiles_sw128(CUtensorMap* m, const void* base, long long rows, int d, int box_rows,
+                     int box_tiles) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc || !base || rows < 1) return false;
+    cuuint64_t dims[3] = {64, (cuuint64_t)rows, (cuuint64_t)(d / 64)};
+    cuuint64_t strides[2] = {(cuuint64_t)d * 2, 128};
+    cuuint32_t box[3] = {64, (cuuint32_t)box_rows, (cuuint32_t)box_tiles};
+    cuuint32_t estr[3] = {1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides,
+               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // fp32 matrix [rows][d], box (32 columns, 32 rows), 128-byte swizzle: the
 // patches the weight-gradient epilogue stores.
 bool map_f32_patches(CUtensorMap* m, const void* base, long long rows, int d) {
@@ -1658,19 +1676,13 @@ size_t hcw_decode_cache_bytes(const int* dims, int layer0, int L, int B, int n, 
     Shape sh;
     if (decode_check(dims, layer0, L, B, n, d, &sh)) return 0;
     size_t slots = 0;
-    for (int l = 0; l < L; ++l) slots += (size_t)decode_link(dims, layer0, sh.b, l);
+    for (int l = 0; l < L; ++l) slots += (size_t)decode_link(dims, layer0, sh.b, l) + 1;
     return slots * (size_t)B * d * 2;
-}
-
-size_t hcw_decode_workspace_bytes(int B, int d, int L) {
-    if (B < 1 || d < 1 || L < 1 || L > kMaxDecodeLayers) return 0;
-    return (size_t)(L > 1 ? L - 1 : 1) * B * d * 2;
 }
 
 int hcw_decode_step(const void* x_t, const void* W_self, const void* W_nbr, const float* bias,
                     const int* dims, int layer0, int L, int t, int B, int n, int d,
-                    unsigned flags, void* cache, void* y_t, void* workspace, size_t ws_bytes,
-                    void* stream) {
+                    unsigned flags, void* cache, void* y_t, void* stream) {
     Shape sh;
     int rc = decode_check(dims, layer0, L, B, n, d, &sh);
     if (rc) return rc;
@@ -1678,48 +1690,51 @@ int hcw_decode_step(const void* x_t, const void* W_self, const void* W_nbr, cons
     // later position
     if (!(flags & HCW_CAUSAL) || (flags & ~kAllFlags) || t < 0 || t >= n) return HCW_ERR_INVALID_ARG;
     if (!x_t || !W_self || !W_nbr || !cache || !y_t) return HCW_ERR_INVALID_ARG;
-    const void* ptrs[] = {x_t, W_self, W_nbr, bias, cache, y_t, workspace};
+    DecodeGeo geo;
+    if (!decode_geometry(d, &geo)) return HCW_ERR_UNSUPPORTED;
+    const void* ptrs[] = {x_t, W_self, W_nbr, bias, cache, y_t};
     for (const void* q : ptrs)
         if (q && !aligned16(q)) return HCW_ERR_ALIGNMENT;
     const size_t row_bytes = (size_t)B * d * 2;
-    const size_t need = hcw_decode_workspace_bytes(B, d, L);
-    if (ws_bytes < need || !workspace) return HCW_ERR_WORKSPACE;
     const size_t cache_b = hcw_decode_cache_bytes(dims, layer0, L, B, n, d);
     const size_t wb = (size_t)L * d * d * 2;
     if (overlaps(y_t, row_bytes, x_t, row_bytes) || overlaps(y_t, row_bytes, cache, cache_b) ||
-        overlaps(y_t, row_bytes, workspace, need) || overlaps(workspace, need, cache, cache_b) ||
-        overlaps(workspace, need, x_t, row_bytes) || overlaps(cache, cache_b, x_t, row_bytes) ||
-        overlaps(cache, cache_b, W_self, wb) || overlaps(cache, cache_b, W_nbr, wb))
+        overlaps(cache, cache_b, x_t, row_bytes) || overlaps(cache, cache_b, W_self, wb) ||
+        overlaps(cache, cache_b, W_nbr, wb))
         return HCW_ERR_ALIASING;
     cudaStream_t st = (cudaStream_t)stream;
     auto* ring = static_cast<__nv_bfloat16*>(cache);
-    auto* inputs = static_cast<__nv_bfloat16*>(workspace);
     const size_t per = (size_t)B * d;
-    __nv_bfloat16* slots[kMaxDecodeLayers];
-    size_t off = 0;
+    DecodeLaunch p;
+    // ring of layer l: k_l + 1 slots of [B][d] from off[l]; position q in slot q mod (k_l + 1)
+    size_t off[kMaxDecodeLayers + 1];
+    int kl[kMaxDecodeLayers];
+    off[0] = 0;
+    for (int l = 0; l < L; ++l) {
+        kl[l] = decode_link(dims, layer0, sh.b, l);
+        off[l + 1] = off[l] + (size_t)(kl[l] + 1) * per;
+    }
+    // element offset of the slot of position q in layer l's ring
+    auto slot = [&](int l, int q) { return off[l] + (size_t)(q % (kl[l] + 1)) * per; };
     for (int l = 0; l < L; ++l) {
         const int s = dims ? dims[l] : (layer0 + l) % sh.b;
-        const int k = decode_link(dims, layer0, sh.b, l);
-        const bool recv = s >= 0 ? ((t >> s) & 1) != 0 : t >= k;
-        __nv_bfloat16* slot = ring + off + (size_t)(t % k) * per;
-        slots[l] = slot;
-        const __nv_bfloat16* in = l == 0 ? static_cast<const __nv_bfloat16*>(x_t)
-                                         : inputs + (size_t)(l - 1) * per;
-        __nv_bfloat16* out = l == L - 1 ? static_cast<__nv_bfloat16*>(y_t)
-                                        : inputs + (size_t)l * per;
-        rc = launched(launch_decode_layer(
-                          in, recv ? slot : nullptr,
-                          static_cast<const __nv_bfloat16*>(W_self) + (size_t)l * d * d,
-                          static_cast<const __nv_bfloat16*>(W_nbr) + (size_t)l * d * d,
-                          bias ? bias + (size_t)l * d : nullptr, B, d, flags, out, st),
-                      1);
-        if (rc) return rc;
-        off += (size_t)k * per;
+        const bool recv = s >= 0 ? ((t >> s) & 1) != 0 : t >= kl[l];
+        p.prow[l] = recv ? (int)(slot(l, t + 1) / d) : -1;   // the slot of t - k_l
+        p.out[l] = l == L - 1 ? static_cast<__nv_bfloat16*>(y_t) : ring + slot(l + 1, t);
     }
-    // every layer's input at t into its ring slot (read above as t's partner)
-    return launched(launch_decode_commit(static_cast<const __nv_bfloat16*>(x_t), inputs, slots, L,
-                                         B, d, st),
-                    1);
+    if (!map_tiles_sw128(&p.mWs, W_self, (long long)L * d, d, geo.oc, geo.kc / 64) ||
+        !map_tiles_sw128(&p.mWn, W_nbr, (long long)L * d, d, geo.oc, geo.kc / 64) ||
+        !map_tiles_sw128(&p.mCache, cache, (long long)(off[L] / d), d, 16, d / 64) ||
+        !map_tiles_sw128(&p.mX, x_t, B, d, 16, d / 64))
+        return HCW_ERR_CUDA;
+    p.bias = bias;
+    p.ring0 = ring + slot(0, t);
+    p.g = geo;
+    p.L = L;
+    p.B = B;
+    p.flags = flags;
+    p.timeout_ns = g_timeout_ns;
+    return launched(launch_decode(p, st), 1);
 }
 
 int hcw_set_stack_kernels(int mode) {
@@ -1738,11 +1753,13 @@ unsigned long long hcw_launch_count(void) { return g_launches.load(); }
 
 int hcw_sync_status(void* stream) {
     if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return HCW_ERR_CUDA;
-    int word = 0, word_res = 0;
+    int word = 0, word_res = 0, word_dec = 0;
     if (error_word_read_clear(&word) != cudaSuccess ||
-        res_error_word_read_clear(&word_res) != cudaSuccess)
+        res_error_word_read_clear(&word_res) != cudaSuccess ||
+        decode_error_word_read_clear(&word_dec) != cudaSuccess)
         return HCW_ERR_CUDA;
     if (!word) word = word_res;
+    if (!word) word = word_dec;
     if (word) return word == HCW_ERR_TIMEOUT ? HCW_ERR_TIMEOUT : HCW_ERR_CUDA;
     return HCW_OK;
 }

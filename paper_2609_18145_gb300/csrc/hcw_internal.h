@@ -164,16 +164,37 @@ cudaError_t res_error_word_read_clear(int* word);
 
 // ---- One-token decode (hcw_decode.cu) ----
 constexpr int kMaxDecodeLayers = 64;   // layers of one decode step
-// out = act(x Ws^T + partner Wn^T + bias) (+ x) for B rows of width d, bf16 in
-// and out, fp32 accumulation; partner null: no partner part.
-cudaError_t launch_decode_layer(const __nv_bfloat16* x, const __nv_bfloat16* partner,
-                                const __nv_bfloat16* Ws, const __nv_bfloat16* Wn,
-                                const float* bias, int B, int d, unsigned flags,
-                                __nv_bfloat16* out, cudaStream_t st);
-// slots[l] <- the input of layer l ([B][d]: x0 for l = 0, inputs[l - 1] after)
-cudaError_t launch_decode_commit(const __nv_bfloat16* x0, const __nv_bfloat16* inputs,
-                                 __nv_bfloat16* const* slots, int L, int B, int d,
-                                 cudaStream_t st);
+// Split of one decode layer over a cluster: CTA q of csize owns output columns
+// [q oc, (q + 1) oc); weights stream in K chunks of kc through `stages` stages.
+struct DecodeGeo {
+    int d, oc, csize, kc, nchunks, stages;
+};
+// false: no cluster split for this d (the decode supports d <= 1024)
+bool decode_geometry(int d, DecodeGeo* g);
+size_t decode_smem_bytes(const DecodeGeo& g);
+// One position of a decode: per layer l, out[l] = act(in_l Ws_l^T +
+// partner_l Wn_l^T + bias_l) (+ in_l) over B rows of width d (bf16 in and
+// out, fp32 accumulation), in_0 = x_t and in_l = out[l - 1]; partner_l is the
+// B rows from row prow[l] of the cache map (prow[l] < 0: no partner part).
+// x_t is also copied to ring0.  Maps (128-byte swizzle, matrices viewed as
+// (64 features, rows, 64-feature tiles)): mWs / mWn over [L d][d] with box
+// (64, oc, kc / 64), mCache over the rings as [rows][d] and mX over x_t [B][d]
+// with box (64, 16, d / 64).
+struct DecodeLaunch {
+    CUtensorMap mWs, mWn, mCache, mX;
+    int prow[kMaxDecodeLayers];
+    __nv_bfloat16* out[kMaxDecodeLayers];
+    const float* bias;
+    __nv_bfloat16* ring0;
+    DecodeGeo g;
+    int L, B;
+    unsigned flags;
+    unsigned long long timeout_ns;
+};
+// One launch of every layer of the step: a cluster per 16 rows.
+cudaError_t launch_decode(const DecodeLaunch& p, cudaStream_t st);
+// Read the decode kernel's error word and reset it to 0 (synchronous).
+cudaError_t decode_error_word_read_clear(int* word);
 
 // Dynamic shared memory the tensor-core kernel uses for this N tile.
 size_t tc_smem_bytes(int BN);

@@ -79,10 +79,9 @@ _SIGNATURES = {
     "hcw_stack_bwd_weight_workspace_bytes": ([_I, _I, _I, _I, _U, _I], _SZ),
     "hcw_stack_bwd": ([_P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P,
                        _P, _P, _SZ, _P], _I),
-    "hcw_decode_step": ([_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P, _SZ, _P],
+    "hcw_decode_step": ([_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P],
                         _I),
     "hcw_decode_cache_bytes": ([_P, _I, _I, _I, _I, _I], _SZ),
-    "hcw_decode_workspace_bytes": ([_I, _I, _I], _SZ),
     "hcw_set_stack_kernels": ([_I], _I),
     "hcw_stack_kernels_used": ([_I, _I, _I, _I], _I),
     "hcw_sync_status": ([_P], _I),
@@ -265,24 +264,19 @@ def hcw_decode_cache_bytes(L: int, B: int, n: int, d: int, dims=None, layer0: in
                                             L, B, n, d))
 
 
-def hcw_decode_workspace_bytes(B: int, d: int, L: int) -> int:
-    return int(lib().hcw_decode_workspace_bytes(B, d, L))
-
-
 def hcw_decode_step(x_t, W_self, W_nbr, bias, t: int, n: int, cache, flags: int,
-                    dims=None, layer0: int = 0, y=None, workspace=None, stream=None):
+                    dims=None, layer0: int = 0, y=None, stream=None):
     """One decode step at position t (Sec. 6): x_t [B, d] bf16 in, returns y_t
     [B, d]; cache is the rings tensor of hcw_decode_cache_bytes (updated)."""
-    _dev(x_t, W_self, W_nbr, bias, cache, y, workspace)
+    _dev(x_t, W_self, W_nbr, bias, cache, y)
     B, d = x_t.shape
     L = W_self.shape[0]
     y = torch.empty_like(x_t) if y is None else y
-    ws = _workspace(hcw_decode_workspace_bytes(B, d, L), x_t.device, workspace)
     arr = None if dims is None else _dims_array(dims, L)
     _check(lib().hcw_decode_step(_ptr(x_t), _ptr(W_self), _ptr(W_nbr), _ptr(bias),
                                  None if arr is None else ctypes.cast(arr, _P), layer0, L, t, B,
-                                 n, d, flags, _ptr(cache), _ptr(y), _ptr(ws), ws.numel(),
-                                 _stream(stream)), "hcw_decode_step")
+                                 n, d, flags, _ptr(cache), _ptr(y), _stream(stream)),
+           "hcw_decode_step")
     return y
 
 

@@ -259,30 +259,31 @@ def test_schedule_entry_points_reject_bad_dims_before_any_launch(hcw):
 
 def test_decode_cache_is_bounded_by_the_link_distances(hcw):
     """Sec. 6: a layer keeps only the last k inputs it links to.  The rings
-    hold sum_l k_l slots of B x d bf16, not the window: the rotated stack at
-    n = 256 keeps 2 x (1 + 2 + ... + 128) = 510 slots instead of 16 x 256."""
+    hold sum_l (k_l + 1) slots of B x d bf16 (the input at t goes to a slot
+    apart from the one of t - k), not the window: the rotated stack at n = 256
+    keeps 2 x (1 + 2 + ... + 128) + 16 = 526 slots instead of 16 x 256."""
     B, d = 3, 64
-    assert hcw.hcw_decode_cache_bytes(16, B, 256, d) == 510 * B * d * 2
+    assert hcw.hcw_decode_cache_bytes(16, B, 256, d) == 526 * B * d * 2
     hy = [-1, 7, -1, -1, 5, -1, 4, -1, -1, 2, -1, 1, -1, 0]   # 8 near + jumps 128 .. 1
-    assert hcw.hcw_decode_cache_bytes(len(hy), B, 256, d, dims=hy) == (8 + 183) * B * d * 2
-    assert hcw.hcw_decode_cache_bytes(3, B, 256, d, dims=[0, -255, 2]) == (1 + 255 + 4) * B * d * 2
+    assert hcw.hcw_decode_cache_bytes(len(hy), B, 256, d, dims=hy) == (8 + 183 + 14) * B * d * 2
+    assert hcw.hcw_decode_cache_bytes(3, B, 256, d, dims=[0, -255, 2]) == (2 + 256 + 5) * B * d * 2
     assert hcw.hcw_decode_cache_bytes(2, B, 48, d) == 0              # n not a power of two
-    assert hcw.hcw_decode_workspace_bytes(B, d, 16) == 15 * B * d * 2
 
 
 def test_decode_step_rejects_bad_arguments_before_any_launch(hcw):
     lib = hcw.lib()
     fake = ctypes.c_void_p(256)
     B, n, d, L = 2, 64, 128, 4
-    ws_b = hcw.hcw_decode_workspace_bytes(B, d, L)
     before = hcw.hcw_launch_count()
 
-    def step(t, flags, ws=ws_b):
-        return lib.hcw_decode_step(fake, fake, fake, None, None, 0, L, t, B, n, d, flags, fake,
-                                   ctypes.c_void_p(1 << 20), fake, ws, None)
+    def step(t, flags, d=d, y=ctypes.c_void_p(1 << 20)):
+        return lib.hcw_decode_step(fake, fake, fake, None, None, 0, L, t, B, n, d, flags, fake, y,
+                                   None)
 
     assert step(0, 0) == hcw.HCW_ERR_INVALID_ARG             # decoding needs the causal rule
     assert step(n, hcw.HCW_CAUSAL) == hcw.HCW_ERR_INVALID_ARG
     assert step(-1, hcw.HCW_CAUSAL) == hcw.HCW_ERR_INVALID_ARG
-    assert step(0, hcw.HCW_CAUSAL, ws=ws_b - 16) == hcw.HCW_ERR_WORKSPACE
+    assert step(0, hcw.HCW_CAUSAL, d=2048) == hcw.HCW_ERR_UNSUPPORTED   # one cluster: d <= 1024
+    assert step(0, hcw.HCW_CAUSAL, y=ctypes.c_void_p(264)) == hcw.HCW_ERR_ALIGNMENT
+    assert step(0, hcw.HCW_CAUSAL, y=fake) == hcw.HCW_ERR_ALIASING       # y_t on the cache
     assert hcw.hcw_launch_count() == before

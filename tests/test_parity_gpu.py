@@ -457,6 +457,12 @@ DECODE_CASES = [
      0, 12),
     ("hybrid256_sparse_n256", 2, 256, 128, CAUSAL | RESIDUAL | RELU,
      [-1, 7, -1, -1, 5, -1, 4, -1, -1, 2, -1, 1, -1, 0], 0, 14),
+    # two row blocks (the second ragged), a cluster of 10 CTAs of 64 columns,
+    # weight chunks 128 wide
+    ("rot_n32_B20_d640", 20, 32, 640, CAUSAL | RESIDUAL | RELU, None, 1, 5),
+    # d = 1024: 16 CTAs of 64 columns, 8 chunks a part; d = 192: 12 CTAs of 16
+    ("rot_n16_B3_d1024", 3, 16, 1024, CAUSAL | RESIDUAL | RELU, None, 0, 4),
+    ("mixa_n32_B33_d192", 33, 32, 192, CAUSAL | RESIDUAL | RELU, [-1, 4, -3, 2, 1, -1, 0], 0, 7),
 ]
 
 
@@ -489,6 +495,34 @@ def test_decode_steps_reproduce_the_window_forward(H, case):
     else:
         y, _, _ = H.hcw_stack_fwd_dims(x, Ws, Wn, bias, dims, flags)
     assert rel(host(ys), host(y)) <= TOL_BF16, name
+
+
+def test_decode_windows_back_to_back_share_the_cache(H):
+    """A new window restarts at t = 0 on the same rings; its outputs are those
+    of a fresh decode on a cache full of garbage, bit for bit (no slot is read
+    before it is written)."""
+    B, n, d, L, flags = 5, 16, 128, 6, CAUSAL | RESIDUAL | RELU
+    pr = synth.problem(B, n, d, L=L, seed=32, w_std=(1 / (2 * d)) ** 0.5)
+    Ws = torch.from_numpy(pr.W_self).to(torch.bfloat16).cuda()
+    Wn = torch.from_numpy(pr.W_nbr).to(torch.bfloat16).cuda()
+    bias = torch.from_numpy(pr.bias).cuda()
+    xa = torch.from_numpy(pr.x).to(torch.bfloat16).cuda()
+    xb = torch.from_numpy(synth.problem(B, n, d, L=1, seed=33).x).to(torch.bfloat16).cuda()
+
+    def window(x, cache):
+        ys = torch.empty_like(x)
+        for t in range(n):
+            ys[:, t] = H.hcw_decode_step(x[:, t].contiguous(), Ws, Wn, bias, t, n, cache, flags)
+        return ys
+
+    nb = H.hcw_decode_cache_bytes(L, B, n, d)
+    cache = torch.empty(nb, dtype=torch.uint8, device="cuda")
+    window(xa, cache)
+    yb = window(xb, cache)
+    fresh = window(xb, torch.full((nb,), 0x7F, dtype=torch.uint8, device="cuda"))
+    torch.cuda.synchronize()
+    assert H.hcw_sync_status() == H.HCW_OK
+    assert torch.equal(yb, fresh)
 
 
 def test_stack_fixed_dimension_control(H):
