@@ -83,16 +83,21 @@ __device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t pa
 // Bounded wait for the phase with the given parity to complete.  Gives up
 // (returns false) when *abort becomes non-zero or after timeout_ns; on a
 // timeout it records kErrTimeout in the device error word and raises *abort
-// so that the CTA's other roles stop too.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
-                                          uint64_t timeout_ns) {
-    if (mbar_try_wait(bar, parity)) return true;
-    const uint64_t t0 = globaltimer_ns();
-    for (uint32_t it = 1;; ++it) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if ((it & 63u) == 0) {
+// so that the CTA's other roles stop too.  The clock starts only after 256
+// unsuccessful polls, so a wait that ends soon never reads the global timer.
+template <bool kCluster>
+__device__ __forceinline__ bool mbar_wait_impl(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                               uint64_t timeout_ns) {
+    uint64_t t0 = 0;
+    for (uint32_t it = 0;; ++it) {
+        if (kCluster ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity))
+            return true;
+        if ((it & 255u) == 255u) {
             if (*abort) return false;
-            if (globaltimer_ns() - t0 > timeout_ns) {
+            const uint64_t now = globaltimer_ns();
+            if (t0 == 0) {
+                t0 = now;
+            } else if (now - t0 > timeout_ns) {
                 atomicExch(&g_error_word, kErrTimeout);
                 *abort = 1;
                 return false;
@@ -101,22 +106,15 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
     }
 }
 
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                          uint64_t timeout_ns) {
+    return mbar_wait_impl<false>(bar, parity, abort, timeout_ns);
+}
+
 // mbar_wait with cluster-scope acquire (mbar_try_wait_cluster).
 __device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity,
                                                   volatile int* abort, uint64_t timeout_ns) {
-    if (mbar_try_wait_cluster(bar, parity)) return true;
-    const uint64_t t0 = globaltimer_ns();
-    for (uint32_t it = 1;; ++it) {
-        if (mbar_try_wait_cluster(bar, parity)) return true;
-        if ((it & 63u) == 0) {
-            if (*abort) return false;
-            if (globaltimer_ns() - t0 > timeout_ns) {
-                atomicExch(&g_error_word, kErrTimeout);
-                *abort = 1;
-                return false;
-            }
-        }
-    }
+    return mbar_wait_impl<true>(bar, parity, abort, timeout_ns);
 }
 
 // Wait that only gives up on time (used to drain in-flight work after an
