@@ -116,3 +116,60 @@ WORKLOADS = {
     "scale_n4096_d1024": dict(n=4096, d=1024, L=12, B=256, causal=False),
     "scale_n65536_d1024": dict(n=65536, d=1024, L=16, B=16, causal=False),
 }
+
+
+@dataclass
+class BlockProblem:
+    """Seeded inputs of the character-LM block around a stack (float32, not yet
+    rounded): ids of a window of n + 1 symbols (inputs ids[:, :n], next-symbol
+    targets ids[:, 1:]), the token and position tables, per layer the two
+    LayerNorms, the mixing maps and the FFN (hidden h), the final LayerNorm
+    and the output head."""
+    ids: np.ndarray      # [B, n + 1] int64 in [0, V)
+    E: np.ndarray        # [V, d]
+    P: np.ndarray        # [n, d]
+    ln1_g: np.ndarray    # [L, d]
+    ln1_b: np.ndarray    # [L, d]
+    W_self: np.ndarray   # [L, d, d]
+    W_nbr: np.ndarray    # [L, d, d]
+    ln2_g: np.ndarray    # [L, d]
+    ln2_b: np.ndarray    # [L, d]
+    W1: np.ndarray       # [L, h, d]
+    b1: np.ndarray       # [L, h]
+    W2: np.ndarray       # [L, d, h]
+    b2: np.ndarray       # [L, d]
+    lnf_g: np.ndarray    # [d]
+    lnf_b: np.ndarray    # [d]
+    Wh: np.ndarray       # [V, d]
+    bh: np.ndarray       # [V]
+
+
+def block_problem(B: int, n: int, d: int, h: int, V: int, L: int, seed: int = 0) -> BlockProblem:
+    """Draw one seeded block problem: Zipf(1.1) ids over V symbols; E ~ N(0, 1);
+    P ~ N(0, 0.1^2); LayerNorm scales 1 + N(0, 0.1^2) and shifts N(0, 0.1^2);
+    W_self, W_nbr ~ N(0, 1/(2d)); W1 ~ N(0, 1/d), W2 ~ N(0, 1/h), Wh ~ N(0, 1/d);
+    biases N(0, 0.1^2)."""
+    s = seed * 100
+
+    def nrm(shape, k, std):
+        return normal(shape, s + k, std)
+
+    return BlockProblem(
+        ids=zipf_ids(B, n + 1, s + 1, vocab=V),
+        E=nrm((V, d), 2, 1.0),
+        P=nrm((n, d), 3, 0.1),
+        ln1_g=(1.0 + nrm((L, d), 4, 0.1)).astype(np.float32),
+        ln1_b=nrm((L, d), 5, 0.1),
+        W_self=nrm((L, d, d), 6, (1.0 / (2 * d)) ** 0.5),
+        W_nbr=nrm((L, d, d), 7, (1.0 / (2 * d)) ** 0.5),
+        ln2_g=(1.0 + nrm((L, d), 8, 0.1)).astype(np.float32),
+        ln2_b=nrm((L, d), 9, 0.1),
+        W1=nrm((L, h, d), 10, (1.0 / d) ** 0.5),
+        b1=nrm((L, h), 11, 0.1),
+        W2=nrm((L, d, h), 12, (1.0 / h) ** 0.5),
+        b2=nrm((L, d), 13, 0.1),
+        lnf_g=(1.0 + nrm((d,), 14, 0.1)).astype(np.float32),
+        lnf_b=nrm((d,), 15, 0.1),
+        Wh=nrm((V, d), 16, (1.0 / d) ** 0.5),
+        bh=nrm((V,), 17, 0.1),
+    )
