@@ -360,6 +360,77 @@ int hcw_decode_step(const void* x_t, const void* W_self, const void* W_nbr, cons
 /* Bytes of the decode rings for this schedule (0 for invalid sizes). */
 size_t hcw_decode_cache_bytes(const int* dims, int layer0, int L, int B, int n, int d);
 
+/*
+ * One training step (forward, loss, backward) of the character-LM block
+ * around the mixing stack, bf16 (App. A: width d, hidden h = 1024 = 2d at
+ * d = 512; the weight counts of Table B2ecost / B1cost fit token and position
+ * embeddings, two LayerNorms and an FFN with biases per layer, a final
+ * LayerNorm and an output head with bias):
+ *   x = E[ids[:, :n]] + P
+ *   per layer l:  x += M_l(LN1_l(x))     M_l: Eq. (1) without bias or activation,
+ *                                        causal, cube dimension l mod log2 n
+ *                 x += W2_l relu(W1_l LN2_l(x) + b1_l) + b2_l
+ *   logits = LNf(x) Wh^T + bh
+ *   loss = mean over the B n positions of logsumexp(logits) - logits[next symbol]
+ * LayerNorm: biased variance, eps = 1e-5, per-feature scale and shift.
+ * Shapes (all device memory, row-major; ids and loss 4-byte aligned, the
+ * rest 16-byte aligned):
+ *   ids [B][n + 1] int32 in [0, V): inputs ids[:, :n], targets ids[:, 1:]
+ *   E [V][d], P [n][d], W_self / W_nbr [L][d][d], W1 [L][h][d], W2 [L][d][h],
+ *   Wh [V][d]: bf16;  LayerNorm scales / shifts ln1_*, ln2_* [L][d], lnf_* [d],
+ *   b1 [L][h], b2 [L][d], bh [V]: fp32.
+ * Gradients (hcw_block_grads, same shapes, fp32) are overwritten, not
+ * accumulated; *loss (one fp32 on the device) is overwritten.  The mixing
+ * products run on this library's tcgen05 layer kernels, the FFN and head
+ * products on cuBLAS (bf16 operands, fp32 accumulation and output).
+ * Needs n a power of two, d a multiple of 64 and <= 1024, h a multiple of 8,
+ * V >= 2.  An id outside [0, V) is read as 0 and reported by hcw_sync_status
+ * as HCW_ERR_INVALID_ARG.  Asynchronous on `stream`.
+ */
+typedef struct {
+    const void* E;
+    const void* P;
+    const float* ln1_g;
+    const float* ln1_b;
+    const void* W_self;
+    const void* W_nbr;
+    const float* ln2_g;
+    const float* ln2_b;
+    const void* W1;
+    const float* b1;
+    const void* W2;
+    const float* b2;
+    const float* lnf_g;
+    const float* lnf_b;
+    const void* Wh;
+    const float* bh;
+} hcw_block_params;
+
+typedef struct {
+    float* E;
+    float* P;
+    float* ln1_g;
+    float* ln1_b;
+    float* W_self;
+    float* W_nbr;
+    float* ln2_g;
+    float* ln2_b;
+    float* W1;
+    float* b1;
+    float* W2;
+    float* b2;
+    float* lnf_g;
+    float* lnf_b;
+    float* Wh;
+    float* bh;
+} hcw_block_grads;
+
+/* Workspace bytes of hcw_block_step (0 for invalid sizes). */
+size_t hcw_block_workspace_bytes(int B, int n, int d, int h, int V, int L);
+int hcw_block_step(const int* ids, const hcw_block_params* params, const hcw_block_grads* grads,
+                   int B, int n, int d, int h, int V, int L, float* loss, void* workspace,
+                   size_t ws_bytes, void* stream);
+
 /* Number of kernels this library has launched in this process (all devices). */
 unsigned long long hcw_launch_count(void);
 

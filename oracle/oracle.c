@@ -151,6 +151,11 @@ double oracle_round_bf16(double v) {
     return v < 0 ? -r : r;
 }
 
+/* oracle_round_bf16 applied to each of a[0 .. count) in place. */
+void oracle_round_bf16_array(double* a, long long count) {
+    for (long long i = 0; i < count; ++i) a[i] = oracle_round_bf16(a[i]);
+}
+
 static double act_fwd(double z, unsigned flags) {
     if (flags & ORACLE_ACT_RELU) return z > 0.0 ? z : 0.0;
     return z;

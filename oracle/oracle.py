@@ -55,6 +55,7 @@ def _load():
             lib.oracle_partner_table.argtypes = [I, I, I, U, P]
             lib.oracle_round_bf16.argtypes = [ctypes.c_double]
             lib.oracle_round_bf16.restype = ctypes.c_double
+            lib.oracle_round_bf16_array.argtypes = [P, ctypes.c_longlong]
             lib.oracle_layer_fwd.argtypes = [P, P, P, P, I, I, I, I, I, U, I, P, P]
             lib.oracle_layer_bwd.argtypes = [P, P, P, P, P, I, I, I, I, I, U, I, P, P, P, P]
             lib.oracle_stack_fwd.argtypes = [P, P, P, P, P, I, I, I, I, I, I, U, I, P, P, P]
@@ -100,9 +101,9 @@ def partner_table(layer: int, dim_override: int, n: int, flags: int) -> np.ndarr
 
 def round_bf16(v):
     """Round each value to the nearest bfloat16 (ties to even)."""
-    f = _load().oracle_round_bf16
-    arr = np.asarray(v, dtype=np.float64)
-    return np.vectorize(lambda t: f(float(t)), otypes=[np.float64])(arr)
+    arr = np.array(v, dtype=np.float64, order="C", copy=True)
+    _load().oracle_round_bf16_array(_p(arr), arr.size)
+    return arr if arr.ndim else float(arr)
 
 
 def layer_fwd(x, W_self, W_nbr, bias, layer, dim_override, flags, round_bf16=False,

@@ -1,0 +1,518 @@
+// hcw_block.cu -- one training step (forward, loss, backward) of the
+// character-LM block around the mixing stack (App. A: width d, hidden 1024 =
+// 2d at d = 512; the weight counts of Table B2ecost / B1cost fit token and
+// position embeddings, two LayerNorms and an FFN with biases per layer, a
+// final LayerNorm and an output head with bias):
+//
+//   x = E[ids] + P
+//   per layer l:  x += M_l(LN1_l(x))                M_l: Eq. (1), causal, rotated
+//                 x += W2_l relu(W1_l LN2_l(x) + b1_l) + b2_l
+//   logits = LNf(x) Wh^T + bh,   loss = mean next-symbol cross-entropy
+//
+// The mixing sublayer runs on this library's layer kernels (hcw_layer_fwd /
+// hcw_layer_bwd: tcgen05, bf16); the FFN and head products are plain GEMMs and
+// go to cuBLAS; the row kernels here (embedding, residual add + LayerNorm,
+// bias + ReLU, cross-entropy, their gradients, column sums) are memory-bound
+// and each makes one pass over its rows.  The residual stream x and its
+// gradient are fp32; the GEMM operands are bf16 (h, M(h), g, relu(u), hf,
+// dlogits, bf16(dx), the FFN pre-activation gradient); GEMM outputs are fp32.
+#include <cublas_v2.h>
+
+#include <mutex>
+
+#include "hcw.h"
+#include "hcw_internal.h"
+#include "hcw_ptx.cuh"
+
+namespace hcw {
+
+namespace {
+
+constexpr float kLnEps = 1e-5f;
+constexpr int kRowWarps = 8;   // rows (one warp each) per CTA of the row kernels
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+
+// symbol of input position t of sequence b (ids: [B][n + 1]); an id outside
+// [0, V) reads symbol 0 and records HCW_ERR_INVALID_ARG in the error word
+__device__ __forceinline__ int symbol(const int* ids, int b, int t, int n, int V) {
+    const int v = ids[(size_t)b * (n + 1) + t];
+    if (v < 0 || v >= V) {
+        atomicExch(&g_error_word, HCW_ERR_INVALID_ARG);
+        return 0;
+    }
+    return v;
+}
+
+// x[b n + t][c] = E[ids[b][t]][c] + P[t][c]   (fp32 out)
+__global__ void embed_fwd_kernel(const int* ids, const __nv_bfloat16* E, const __nv_bfloat16* P,
+                                 float* x, int B, int n, int d, int V) {
+    const size_t total = (size_t)B * n * d;
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (size_t)gridDim.x * blockDim.x) {
+        const int c = (int)(i % d);
+        const size_t r = i / d;
+        const int t = (int)(r % n), b = (int)(r / n);
+        const int v = symbol(ids, b, t, n, V);
+        x[i] = __bfloat162float(E[(size_t)v * d + c]) + __bfloat162float(P[(size_t)t * d + c]);
+    }
+}
+
+// One warp per row: x = x_in (+ add1 bf16) (+ add2 fp32) (+ badd[c]); x_out = x
+// when given; y = bf16((x - mean) rstd g + b); stats = (mean, rstd).  d <= 1024.
+__global__ void __launch_bounds__(kRowWarps * 32)
+    ln_fwd_kernel(const float* x_in, const __nv_bfloat16* add1, const float* add2,
+                  const float* badd, float* x_out, const float* g, const float* b,
+                  __nv_bfloat16* y, float2* stats, int T, int d) {
+    const int lane = threadIdx.x & 31;
+    const int row = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
+    if (row >= T) return;
+    const int nv = d >> 5;
+    const size_t base = (size_t)row * d;
+    float v[32];
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+        if (i < nv) {
+            const int c = i * 32 + lane;
+            float t = x_in[base + c];
+            if (add1) t += __bfloat162float(add1[base + c]);
+            if (add2) t += add2[base + c];
+            if (badd) t += badd[c];
+            v[i] = t;
+            s += t;
+        }
+    }
+    const float mean = warp_sum(s) / d;
+    float q = 0.f;
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+        if (i < nv) q += (v[i] - mean) * (v[i] - mean);
+    const float rstd = rsqrtf(warp_sum(q) / d + kLnEps);
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+        if (i < nv) {
+            const int c = i * 32 + lane;
+            if (x_out) x_out[base + c] = v[i];
+            y[base + c] = __float2bfloat16_rn((v[i] - mean) * rstd * g[c] + b[c]);
+        }
+    }
+    if (lane == 0) stats[row] = make_float2(mean, rstd);
+}
+
+// a = bf16(relu(U + b1[col]))   U: [T][h] fp32 (the GEMM output)
+__global__ void bias_relu_kernel(const float* U, const float* b1, __nv_bfloat16* a, size_t total,
+                                 int h) {
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (size_t)gridDim.x * blockDim.x) {
+        const float u = U[i] + b1[i % h];
+        a[i] = __float2bfloat16_rn(u > 0.f ? u : 0.f);
+    }
+}
+
+// One warp per position r = b n + t: z = logits[r] + bh, target v* =
+// ids[b][t + 1]; loss += (logsumexp(z) - z[v*]) / N; dlog[r][v] =
+// bf16((softmax(z)[v] - [v == v*]) / N).
+__global__ void __launch_bounds__(kRowWarps * 32)
+    ce_kernel(const float* logits, const float* bh, const int* ids, __nv_bfloat16* dlog,
+              float* loss, int B, int n, int V, float inv_N) {
+    const int lane = threadIdx.x & 31;
+    const int r = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
+    if (r >= B * n) return;
+    const int b = r / n, t = r % n;
+    const int tgt = symbol(ids, b, t + 1, n, V);
+    const float* z = logits + (size_t)r * V;
+    float m = -INFINITY;
+    for (int v = lane; v < V; v += 32) m = fmaxf(m, z[v] + bh[v]);
+    m = warp_max(m);
+    float s = 0.f;
+    for (int v = lane; v < V; v += 32) s += expf(z[v] + bh[v] - m);
+    const float lse = m + logf(warp_sum(s));
+    for (int v = lane; v < V; v += 32) {
+        const float p = expf(z[v] + bh[v] - lse) - (v == tgt ? 1.f : 0.f);
+        dlog[(size_t)r * V + v] = __float2bfloat16_rn(p * inv_N);
+    }
+    if (lane == 0) atomicAdd(loss, (lse - (z[tgt] + bh[tgt])) * inv_N);
+}
+
+// dpre = bf16(da where relu(u) > 0, else 0)   (a = relu(u) holds the mask)
+__global__ void relu_bwd_kernel(const float* da, const __nv_bfloat16* a, __nv_bfloat16* dpre,
+                                size_t total) {
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (size_t)gridDim.x * blockDim.x)
+        dpre[i] = __float2bfloat16_rn(__bfloat162float(a[i]) > 0.f ? da[i] : 0.f);
+}
+
+// out[c] += sum over rows [r0, r0 + kColRows) of M[r][c]   (bf16 M [T][C];
+// out zeroed before the launch; one CTA per block of rows)
+constexpr int kColRows = 128;
+__global__ void colsum_kernel(const __nv_bfloat16* M, float* out, int T, int C) {
+    const int r0 = blockIdx.x * kColRows;
+    const int r1 = min(T, r0 + kColRows);
+    for (int c = threadIdx.x; c < C; c += blockDim.x) {
+        float s = 0.f;
+        for (int r = r0; r < r1; ++r) s += __bfloat162float(M[(size_t)r * C + c]);
+        atomicAdd(out + c, s);
+    }
+}
+
+// LayerNorm backward, one warp per row (rows r = blockIdx.x * 8 + warp, then
+// strided by the grid): with xhat = (x - mean) rstd and dxhat = dy g,
+//   dx = rstd (dxhat - mean(dxhat) - xhat mean(dxhat xhat))  (+ dres)
+// written to dx_out (fp32) and, when dxb is given, as bf16; the scale and
+// shift gradients sum dy xhat and dy over the CTA's rows in shared memory,
+// then one atomic add per column and CTA.  dy is fp32 (dyf) or bf16 (dyb).
+// The CTA's rows go through shared-memory atomics (at most 8 rows at a time
+// on one column).
+__global__ void __launch_bounds__(kRowWarps * 32)
+    ln_bwd_kernel(const float* dyf, const __nv_bfloat16* dyb, const float* x, const float2* stats,
+                  const float* g, const float* dres, float* dx_out, __nv_bfloat16* dxb,
+                  float* dgam, float* dbet, int T, int d) {
+    extern __shared__ float part[];   // [2][d]: dgam, dbet partials of this CTA
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int c = threadIdx.x; c < 2 * d; c += blockDim.x) part[c] = 0.f;
+    __syncthreads();
+    const int nv = d >> 5;
+    for (int row = blockIdx.x * kRowWarps + warp; row < T; row += gridDim.x * kRowWarps) {
+        const size_t base = (size_t)row * d;
+        const float2 st = stats[row];
+        float xh[32], dh[32];
+        float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+            if (i < nv) {
+                const int c = i * 32 + lane;
+                const float dy = dyf ? dyf[base + c] : __bfloat162float(dyb[base + c]);
+                xh[i] = (x[base + c] - st.x) * st.y;
+                dh[i] = dy * g[c];
+                s1 += dh[i];
+                s2 += dh[i] * xh[i];
+                atomicAdd(&part[c], dy * xh[i]);
+                atomicAdd(&part[d + c], dy);
+            }
+        }
+        const float m1 = warp_sum(s1) / d, m2 = warp_sum(s2) / d;
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+            if (i < nv) {
+                const int c = i * 32 + lane;
+                float v = st.y * (dh[i] - m1 - xh[i] * m2);
+                if (dres) v += dres[base + c];
+                dx_out[base + c] = v;
+                if (dxb) dxb[base + c] = __float2bfloat16_rn(v);
+            }
+        }
+    }
+    __syncthreads();
+    for (int c = threadIdx.x; c < d; c += blockDim.x) {
+        atomicAdd(dgam + c, part[c]);
+        atomicAdd(dbet + c, part[d + c]);
+    }
+}
+
+// dE[ids[b][t]] += dx[b n + t]   (dE zeroed before the launch)
+__global__ void embed_bwd_kernel(const int* ids, const float* dx, float* dE, int B, int n, int d,
+                                 int V) {
+    const size_t total = (size_t)B * n * d;
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (size_t)gridDim.x * blockDim.x) {
+        const int c = (int)(i % d);
+        const size_t r = i / d;
+        const int v = symbol(ids, (int)(r / n), (int)(r % n), n, V);
+        atomicAdd(dE + (size_t)v * d + c, dx[i]);
+    }
+}
+
+// dP[t][c] = sum over b of dx[b n + t][c]
+__global__ void pos_bwd_kernel(const float* dx, float* dP, int B, int n, int d) {
+    const size_t total = (size_t)n * d;
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+         i += (size_t)gridDim.x * blockDim.x) {
+        float s = 0.f;
+        for (int b = 0; b < B; ++b) s += dx[(size_t)b * n * d + i];
+        dP[i] = s;
+    }
+}
+
+}  // namespace
+
+namespace {
+
+// cuBLAS handle of each device, created on first use and kept for the process
+cublasHandle_t blas_handle() {
+    static std::mutex mu;
+    static cublasHandle_t handles[64] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> lock(mu);
+    if (!handles[dev] && cublasCreate(&handles[dev]) != CUBLAS_STATUS_SUCCESS)
+        handles[dev] = nullptr;
+    return handles[dev];
+}
+
+// Row-major C[M][N] (fp32) = op(A) op(B) with bf16 operands and fp32
+// accumulation; A is [M][K] ([K][M] when ta), B is [K][N] ([N][K] when tb).
+// cuBLAS is column-major, where the row-major C is C^T = op(B)^T op(A)^T.
+bool gemm(cublasHandle_t h, int M, int N, int K, const void* A, bool ta, const void* B, bool tb,
+          float* C) {
+    const float one = 1.f, zero = 0.f;
+    return cublasGemmEx(h, tb ? CUBLAS_OP_T : CUBLAS_OP_N, ta ? CUBLAS_OP_T : CUBLAS_OP_N, N, M,
+                        K, &one, B, CUDA_R_16BF, tb ? K : N, A, CUDA_R_16BF, ta ? M : K, &zero, C,
+                        CUDA_R_32F, N, CUBLAS_COMPUTE_32F,
+                        CUBLAS_GEMM_DEFAULT) == CUBLAS_STATUS_SUCCESS;
+}
+
+size_t round256(size_t v) { return (v + 255) & ~(size_t)255; }
+
+// Workspace of one step (byte offsets; T = B n tokens):
+//   xs   [2L + 1][T][d] fp32   x_0 .. x_L (layer inputs, x_L the head's), then
+//                              the L mid-layer streams (after the mixing)
+//   h1, g [L][T][d] bf16       LN1 / LN2 outputs (mixing and FFN inputs)
+//   a    [L][T][h] bf16        relu(u), the FFN's hidden activations
+//   st1, st2 [L][T], stf [T]   LayerNorm (mean, rstd)
+//   m, hf [T][d] bf16          mixing output (per layer), head input
+//   U    [T][max(h, V, d)] fp32  every GEMM output with T rows, in turn
+//   dlog [T][V] bf16; dx [T][d] fp32; dxb [T][d] bf16; dpre [T][h] bf16;
+//   dh [T][d] bf16; then the mixing backward's own workspace
+struct BlockWs {
+    size_t xs, h1, g, a, st1, st2, stf, m, hf, U, dlog, dx, dxb, dpre, dh, lws, lws_bytes, total;
+};
+
+BlockWs block_ws(int B, int n, int d, int h, int V, int L) {
+    const size_t T = (size_t)B * n;
+    const size_t wide = (size_t)(h > V ? (h > d ? h : d) : (V > d ? V : d));
+    BlockWs w;
+    size_t o = 0;
+    auto take = [&](size_t bytes) {
+        const size_t at = o;
+        o += round256(bytes);
+        return at;
+    };
+    w.xs = take((2 * (size_t)L + 1) * T * d * 4);
+    w.h1 = take((size_t)L * T * d * 2);
+    w.g = take((size_t)L * T * d * 2);
+    w.a = take((size_t)L * T * h * 2);
+    w.st1 = take((size_t)L * T * 8);
+    w.st2 = take((size_t)L * T * 8);
+    w.stf = take(T * 8);
+    w.m = take(T * d * 2);
+    w.hf = take(T * d * 2);
+    w.U = take(T * wide * 4);
+    w.dlog = take(T * V * 2);
+    w.dx = take(T * d * 4);
+    w.dxb = take(T * d * 2);
+    w.dpre = take(T * h * 2);
+    w.dh = take(T * d * 2);
+    w.lws_bytes = hcw_workspace_bytes(B, n, d, HCW_BF16, HCW_CAUSAL);
+    w.lws = take(w.lws_bytes);
+    w.total = o;
+    return w;
+}
+
+}  // namespace
+
+namespace {
+
+int sms_now() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
+        return 148;
+    return n;
+}
+
+bool block_sizes_ok(int B, int n, int d, int h, int V, int L) {
+    return B >= 1 && n >= 2 && (n & (n - 1)) == 0 && d >= 64 && d % 64 == 0 && d <= 1024 &&
+           h >= 8 && h % 8 == 0 && V >= 2 && L >= 1 && (long long)B * n * (n + 1) < (1ll << 40);
+}
+
+bool a16(const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
+
+// launch status of the kernel just launched (counted when it succeeded)
+int ok_launch() { return count_launch(cudaGetLastError(), 1); }
+
+unsigned elem_grid(size_t total) {
+    const size_t want = (total + 255) / 256, cap = (size_t)sms_now() * 16;
+    return (unsigned)(want < cap ? (want ? want : 1) : cap);
+}
+
+int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads& gr, int B, int n,
+               int d, int h, int V, int L, float* loss, uint8_t* ws, cudaStream_t st) {
+    const int T = B * n;
+    const BlockWs w = block_ws(B, n, d, h, V, L);
+    const size_t Td = (size_t)T * d, Th = (size_t)T * h;
+    float* xs = reinterpret_cast<float*>(ws + w.xs);
+    auto X = [&](int l) { return xs + (size_t)l * Td; };              // x_l, l = 0..L
+    auto XM = [&](int l) { return xs + (size_t)(L + 1 + l) * Td; };   // mid-layer stream
+    auto H1 = [&](int l) { return reinterpret_cast<__nv_bfloat16*>(ws + w.h1) + (size_t)l * Td; };
+    auto G = [&](int l) { return reinterpret_cast<__nv_bfloat16*>(ws + w.g) + (size_t)l * Td; };
+    auto A = [&](int l) { return reinterpret_cast<__nv_bfloat16*>(ws + w.a) + (size_t)l * Th; };
+    auto S1 = [&](int l) { return reinterpret_cast<float2*>(ws + w.st1) + (size_t)l * T; };
+    auto S2 = [&](int l) { return reinterpret_cast<float2*>(ws + w.st2) + (size_t)l * T; };
+    float2* sf = reinterpret_cast<float2*>(ws + w.stf);
+    auto* m = reinterpret_cast<__nv_bfloat16*>(ws + w.m);
+    auto* hf = reinterpret_cast<__nv_bfloat16*>(ws + w.hf);
+    float* U = reinterpret_cast<float*>(ws + w.U);
+    auto* dlog = reinterpret_cast<__nv_bfloat16*>(ws + w.dlog);
+    float* dx = reinterpret_cast<float*>(ws + w.dx);
+    auto* dxb = reinterpret_cast<__nv_bfloat16*>(ws + w.dxb);
+    auto* dpre = reinterpret_cast<__nv_bfloat16*>(ws + w.dpre);
+    auto* dh = reinterpret_cast<__nv_bfloat16*>(ws + w.dh);
+    auto bf = [](const void* q, size_t off) {
+        return static_cast<const __nv_bfloat16*>(q) + off;
+    };
+    cublasHandle_t hb = blas_handle();
+    if (!hb || cublasSetStream(hb, st) != CUBLAS_STATUS_SUCCESS) return HCW_ERR_CUDA;
+    const unsigned rows_grid = (unsigned)((T + kRowWarps - 1) / kRowWarps);
+    const unsigned ln_bwd_grid = rows_grid < (unsigned)sms_now() * 4 ? rows_grid : sms_now() * 4;
+    const size_t ln_smem = (size_t)2 * d * sizeof(float);
+    int rc;
+#define HCW_TRY(expr)          \
+    do {                       \
+        rc = (expr);           \
+        if (rc) return rc;     \
+    } while (0)
+#define HCW_CU(expr) HCW_TRY((expr) == cudaSuccess ? HCW_OK : HCW_ERR_CUDA)
+#define HCW_BLAS(expr) HCW_TRY((expr) ? HCW_OK : HCW_ERR_CUDA)
+    // gradients that are sums (atomics) start at zero; so does the loss
+    HCW_CU(cudaMemsetAsync(loss, 0, sizeof(float), st));
+    HCW_CU(cudaMemsetAsync(gr.E, 0, (size_t)V * d * 4, st));
+    float* zero_d[] = {gr.ln1_g, gr.ln1_b, gr.ln2_g, gr.ln2_b, gr.b2};
+    for (float* q : zero_d) HCW_CU(cudaMemsetAsync(q, 0, (size_t)L * d * 4, st));
+    HCW_CU(cudaMemsetAsync(gr.b1, 0, (size_t)L * h * 4, st));
+    HCW_CU(cudaMemsetAsync(gr.lnf_g, 0, (size_t)d * 4, st));
+    HCW_CU(cudaMemsetAsync(gr.lnf_b, 0, (size_t)d * 4, st));
+    HCW_CU(cudaMemsetAsync(gr.bh, 0, (size_t)V * 4, st));
+
+    // ------------------------------------------------------------ forward
+    embed_fwd_kernel<<<elem_grid(Td), 256, 0, st>>>(ids, bf(p.E, 0), bf(p.P, 0), X(0), B, n, d, V);
+    HCW_TRY(ok_launch());
+    ln_fwd_kernel<<<rows_grid, kRowWarps * 32, 0, st>>>(X(0), nullptr, nullptr, nullptr, nullptr,
+                                                        p.ln1_g, p.ln1_b, H1(0), S1(0), T, d);
+    HCW_TRY(ok_launch());
+    for (int l = 0; l < L; ++l) {
+        HCW_TRY(hcw_layer_fwd(H1(l), bf(p.W_self, (size_t)l * d * d), bf(p.W_nbr, (size_t)l * d * d),
+                              nullptr, l, -1, B, n, d, HCW_BF16, HCW_CAUSAL, m, nullptr, st));
+        ln_fwd_kernel<<<rows_grid, kRowWarps * 32, 0, st>>>(
+            X(l), m, nullptr, nullptr, XM(l), p.ln2_g + (size_t)l * d, p.ln2_b + (size_t)l * d, G(l),
+            S2(l), T, d);
+        HCW_TRY(ok_launch());
+        HCW_BLAS(gemm(hb, T, h, d, G(l), false, bf(p.W1, (size_t)l * h * d), true, U));
+        bias_relu_kernel<<<elem_grid(Th), 256, 0, st>>>(U, p.b1 + (size_t)l * h, A(l), Th, h);
+        HCW_TRY(ok_launch());
+        HCW_BLAS(gemm(hb, T, d, h, A(l), false, bf(p.W2, (size_t)l * d * h), true, U));
+        const bool top = l + 1 == L;
+        ln_fwd_kernel<<<rows_grid, kRowWarps * 32, 0, st>>>(
+            XM(l), nullptr, U, p.b2 + (size_t)l * d, X(l + 1),
+            top ? p.lnf_g : p.ln1_g + (size_t)(l + 1) * d,
+            top ? p.lnf_b : p.ln1_b + (size_t)(l + 1) * d, top ? hf : H1(l + 1), top ? sf : S1(l + 1),
+            T, d);
+        HCW_TRY(ok_launch());
+    }
+    HCW_BLAS(gemm(hb, T, V, d, hf, false, p.Wh, true, U));
+    ce_kernel<<<rows_grid, kRowWarps * 32, 0, st>>>(U, p.bh, ids, dlog, loss, B, n, V, 1.f / T);
+    HCW_TRY(ok_launch());
+
+    // ----------------------------------------------------------- backward
+    const unsigned gridT = (unsigned)((T + kColRows - 1) / kColRows);
+    HCW_BLAS(gemm(hb, V, d, T, dlog, true, hf, false, gr.Wh));   // dWh = dlog^T hf
+    colsum_kernel<<<gridT, 256, 0, st>>>(dlog, gr.bh, T, V);
+    HCW_TRY(ok_launch());
+    HCW_BLAS(gemm(hb, T, d, V, dlog, false, p.Wh, false, U));    // dhf = dlog Wh
+    ln_bwd_kernel<<<ln_bwd_grid, kRowWarps * 32, ln_smem, st>>>(
+        U, nullptr, X(L), sf, p.lnf_g, nullptr, dx, dxb, gr.lnf_g, gr.lnf_b, T, d);
+    HCW_TRY(ok_launch());
+    for (int l = L - 1; l >= 0; --l) {
+        // FFN sublayer: dxb = bf16(dx) is the gradient of its output
+        HCW_BLAS(gemm(hb, d, h, T, dxb, true, A(l), false, gr.W2 + (size_t)l * d * h));
+        colsum_kernel<<<gridT, 256, 0, st>>>(dxb, gr.b2 + (size_t)l * d, T, d);
+        HCW_TRY(ok_launch());
+        HCW_BLAS(gemm(hb, T, h, d, dxb, false, bf(p.W2, (size_t)l * d * h), false, U));   // da
+        relu_bwd_kernel<<<elem_grid(Th), 256, 0, st>>>(U, A(l), dpre, Th);
+        HCW_TRY(ok_launch());
+        colsum_kernel<<<gridT, 256, 0, st>>>(dpre, gr.b1 + (size_t)l * h, T, h);
+        HCW_TRY(ok_launch());
+        HCW_BLAS(gemm(hb, h, d, T, dpre, true, G(l), false, gr.W1 + (size_t)l * h * d));
+        HCW_BLAS(gemm(hb, T, d, h, dpre, false, bf(p.W1, (size_t)l * h * d), false, U));  // dg
+        ln_bwd_kernel<<<ln_bwd_grid, kRowWarps * 32, ln_smem, st>>>(
+            U, nullptr, XM(l), S2(l), p.ln2_g + (size_t)l * d, dx, dx, dxb,
+            gr.ln2_g + (size_t)l * d, gr.ln2_b + (size_t)l * d, T, d);
+        HCW_TRY(ok_launch());
+        // mixing sublayer: dxb = bf16(dx) is the gradient of M_l(h)
+        HCW_TRY(hcw_layer_bwd(H1(l), nullptr, dxb, bf(p.W_self, (size_t)l * d * d),
+                              bf(p.W_nbr, (size_t)l * d * d), l, -1, B, n, d, HCW_BF16, HCW_CAUSAL,
+                              dh, gr.W_self + (size_t)l * d * d, gr.W_nbr + (size_t)l * d * d,
+                              nullptr, w.lws_bytes ? ws + w.lws : nullptr, w.lws_bytes, st));
+        ln_bwd_kernel<<<ln_bwd_grid, kRowWarps * 32, ln_smem, st>>>(
+            nullptr, dh, X(l), S1(l), p.ln1_g + (size_t)l * d, dx, dx, dxb,
+            gr.ln1_g + (size_t)l * d, gr.ln1_b + (size_t)l * d, T, d);
+        HCW_TRY(ok_launch());
+    }
+    embed_bwd_kernel<<<elem_grid(Td), 256, 0, st>>>(ids, dx, gr.E, B, n, d, V);
+    HCW_TRY(ok_launch());
+    pos_bwd_kernel<<<elem_grid((size_t)n * d), 256, 0, st>>>(dx, gr.P, B, n, d);
+    return ok_launch();
+#undef HCW_TRY
+#undef HCW_CU
+#undef HCW_BLAS
+}
+
+}  // namespace
+
+cudaError_t block_error_word_read_clear(int* word) {
+    const int zero = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(word, g_error_word, sizeof(int));
+    if (e == cudaSuccess && *word) e = cudaMemcpyToSymbol(g_error_word, &zero, sizeof(int));
+    return e;
+}
+
+}  // namespace hcw
+
+using namespace hcw;
+
+extern "C" {
+
+size_t hcw_block_workspace_bytes(int B, int n, int d, int h, int V, int L) {
+    if (!block_sizes_ok(B, n, d, h, V, L)) return 0;
+    return block_ws(B, n, d, h, V, L).total;
+}
+
+int hcw_block_step(const int* ids, const hcw_block_params* params, const hcw_block_grads* grads,
+                   int B, int n, int d, int h, int V, int L, float* loss, void* workspace,
+                   size_t ws_bytes, void* stream) {
+    if (!params || !grads || !ids || !loss) return HCW_ERR_INVALID_ARG;
+    if (!block_sizes_ok(B, n, d, h, V, L))
+        return (d > 1024 && d % 64 == 0) ? HCW_ERR_UNSUPPORTED : HCW_ERR_INVALID_ARG;
+    const hcw_block_params& p = *params;
+    const hcw_block_grads& g = *grads;
+    const void* in[] = {p.E, p.P, p.ln1_g, p.ln1_b, p.W_self, p.W_nbr, p.ln2_g, p.ln2_b, p.W1,
+                        p.b1, p.W2, p.b2, p.lnf_g, p.lnf_b, p.Wh, p.bh};
+    const void* out[] = {g.E, g.P, g.ln1_g, g.ln1_b, g.W_self, g.W_nbr, g.ln2_g, g.ln2_b, g.W1,
+                         g.b1, g.W2, g.b2, g.lnf_g, g.lnf_b, g.Wh, g.bh, loss};
+    for (const void* q : in)
+        if (!q) return HCW_ERR_INVALID_ARG;
+    for (const void* q : out)
+        if (!q) return HCW_ERR_INVALID_ARG;
+    for (const void* q : in)
+        if (!a16(q)) return HCW_ERR_ALIGNMENT;
+    for (const void* q : out)
+        if (q != loss && !a16(q)) return HCW_ERR_ALIGNMENT;
+    // ids and the loss are read and written as 4-byte scalars
+    if ((reinterpret_cast<uintptr_t>(loss) & 3) || (reinterpret_cast<uintptr_t>(ids) & 3))
+        return HCW_ERR_ALIGNMENT;
+    const size_t need = block_ws(B, n, d, h, V, L).total;
+    if (!workspace || ws_bytes < need || !a16(workspace)) return HCW_ERR_WORKSPACE;
+    return block_step(ids, p, g, B, n, d, h, V, L, loss, static_cast<uint8_t*>(workspace),
+                      (cudaStream_t)stream);
+}
+
+}  // extern "C"

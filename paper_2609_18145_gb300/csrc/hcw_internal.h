@@ -196,6 +196,13 @@ cudaError_t launch_decode(const DecodeLaunch& p, cudaStream_t st);
 // Read the decode kernel's error word and reset it to 0 (synchronous).
 cudaError_t decode_error_word_read_clear(int* word);
 
+// ---- Character-LM block (hcw_block.cu) ----
+// Read the block kernels' error word and reset it to 0 (synchronous).
+cudaError_t block_error_word_read_clear(int* word);
+// HCW_OK after counting `kernels` launches if e is cudaSuccess, else HCW_ERR_CUDA
+// (the launch counter lives with the C API in hcw_api.cu).
+int count_launch(cudaError_t e, int kernels);
+
 // Dynamic shared memory the tensor-core kernel uses for this N tile.
 size_t tc_smem_bytes(int BN);
 int tc_stages(int BN);

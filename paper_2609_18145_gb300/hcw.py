@@ -82,6 +82,8 @@ _SIGNATURES = {
     "hcw_decode_step": ([_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P],
                         _I),
     "hcw_decode_cache_bytes": ([_P, _I, _I, _I, _I, _I], _SZ),
+    "hcw_block_workspace_bytes": ([_I, _I, _I, _I, _I, _I], _SZ),
+    "hcw_block_step": ([_P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _SZ, _P], _I),
     "hcw_set_stack_kernels": ([_I], _I),
     "hcw_stack_kernels_used": ([_I, _I, _I, _I], _I),
     "hcw_sync_status": ([_P], _I),
@@ -278,6 +280,44 @@ def hcw_decode_step(x_t, W_self, W_nbr, bias, t: int, n: int, cache, flags: int,
                                  n, d, flags, _ptr(cache), _ptr(y), _stream(stream)),
            "hcw_decode_step")
     return y
+
+
+BLOCK_FIELDS = ("E", "P", "ln1_g", "ln1_b", "W_self", "W_nbr", "ln2_g", "ln2_b", "W1", "b1",
+                "W2", "b2", "lnf_g", "lnf_b", "Wh", "bh")
+
+
+class _BlockPtrs(ctypes.Structure):
+    """hcw_block_params / hcw_block_grads: sixteen device pointers in BLOCK_FIELDS order."""
+    _fields_ = [(f, ctypes.c_void_p) for f in BLOCK_FIELDS]
+
+
+def hcw_block_workspace_bytes(B: int, n: int, d: int, h: int, V: int, L: int) -> int:
+    return int(lib().hcw_block_workspace_bytes(B, n, d, h, V, L))
+
+
+def hcw_block_step(ids, params: dict, grads: dict | None = None, loss=None, workspace=None,
+                   stream=None):
+    """One training step of the character-LM block (forward, loss, backward).
+    ids [B, n + 1] int32; params: BLOCK_FIELDS -> device tensors (bf16 tables
+    and maps, fp32 LayerNorm parameters and biases).  Returns (loss [1] fp32,
+    grads: BLOCK_FIELDS -> fp32 tensors of the parameters' shapes)."""
+    _dev(ids, loss, workspace, *params.values())
+    B, n1 = ids.shape
+    n = n1 - 1
+    V, d = params["E"].shape
+    L, h = params["W1"].shape[0], params["W1"].shape[1]
+    dev = ids.device
+    if grads is None:
+        grads = {f: torch.empty(tuple(params[f].shape), dtype=torch.float32, device=dev)
+                 for f in BLOCK_FIELDS}
+    loss = torch.empty(1, dtype=torch.float32, device=dev) if loss is None else loss
+    ws = _workspace(hcw_block_workspace_bytes(B, n, d, h, V, L), dev, workspace)
+    P = _BlockPtrs(*[params[f].data_ptr() for f in BLOCK_FIELDS])
+    G = _BlockPtrs(*[grads[f].data_ptr() for f in BLOCK_FIELDS])
+    _check(lib().hcw_block_step(_ptr(ids), ctypes.byref(P), ctypes.byref(G), B, n, d, h, V, L,
+                                _ptr(loss), _ptr(ws), ws.numel(), _stream(stream)),
+           "hcw_block_step")
+    return loss, grads
 
 
 def hcw_set_stack_kernels(mode: int) -> int:

@@ -287,3 +287,33 @@ def test_decode_step_rejects_bad_arguments_before_any_launch(hcw):
     assert step(0, hcw.HCW_CAUSAL, y=ctypes.c_void_p(264)) == hcw.HCW_ERR_ALIGNMENT
     assert step(0, hcw.HCW_CAUSAL, y=fake) == hcw.HCW_ERR_ALIASING       # y_t on the cache
     assert hcw.hcw_launch_count() == before
+
+
+def test_block_workspace_size_and_validation(hcw):
+    """The block step validates sizes, pointers, alignment and the workspace
+    before any launch."""
+    assert hcw.hcw_block_workspace_bytes(2, 16, 64, 128, 11, 2) > 0
+    assert hcw.hcw_block_workspace_bytes(2, 12, 64, 128, 11, 2) == 0    # n not a power of two
+    assert hcw.hcw_block_workspace_bytes(2, 16, 96, 128, 11, 2) == 0    # d not a multiple of 64
+    assert hcw.hcw_block_workspace_bytes(2, 16, 64, 12, 11, 2) == 0     # h not a multiple of 8
+    assert hcw.hcw_block_workspace_bytes(2, 16, 64, 128, 1, 2) == 0     # V < 2
+    lib = hcw.lib()
+    fake = 1 << 20
+    P = hcw._BlockPtrs(*([fake] * len(hcw.BLOCK_FIELDS)))
+    G = hcw._BlockPtrs(*([fake + (1 << 16)] * len(hcw.BLOCK_FIELDS)))
+    ws_b = hcw.hcw_block_workspace_bytes(2, 16, 64, 128, 11, 2)
+    before = hcw.hcw_launch_count()
+
+    def step(P=P, G=G, d=64, ids=ctypes.c_void_p(fake), loss=ctypes.c_void_p(fake), ws=ws_b):
+        return lib.hcw_block_step(ids, ctypes.byref(P), ctypes.byref(G), 2, 16, d, 128, 11, 2,
+                                  loss, ctypes.c_void_p(1 << 30), ws, None)
+
+    assert lib.hcw_block_step(ctypes.c_void_p(fake), None, ctypes.byref(G), 2, 16, 64, 128, 11, 2,
+                              ctypes.c_void_p(fake), ctypes.c_void_p(1 << 30), ws_b,
+                              None) == hcw.HCW_ERR_INVALID_ARG
+    assert step(d=2048) == hcw.HCW_ERR_UNSUPPORTED           # LayerNorm rows: d <= 1024
+    assert step(ids=None) == hcw.HCW_ERR_INVALID_ARG
+    Pbad = hcw._BlockPtrs(*([fake] * 15 + [fake + 4]))
+    assert step(P=Pbad) == hcw.HCW_ERR_ALIGNMENT
+    assert step(ws=ws_b - 256) == hcw.HCW_ERR_WORKSPACE
+    assert hcw.hcw_launch_count() == before

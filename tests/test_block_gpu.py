@@ -1,0 +1,145 @@
+"""GPU parity of the character-LM block step (hcw_block_step) against the fp64
+oracle (oracle/block.py) in its bf16-storage mode, and batch properties at the
+full size of the window-256 configuration."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import block as OB
+from paper_2609_18145_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+BF16 = {"E", "P", "W_self", "W_nbr", "W1", "W2", "Wh"}
+# Tolerance.  Both sides round the same tensors to bf16, but they compute in
+# fp32 (device) and fp64 (oracle): once their values differ by more than the
+# distance to a rounding boundary they round differently, and each of the 2L
+# sublayers adds up to half an ulp (2^-9 relative) of independent difference to
+# the gradient flowing down from the head, like a random walk: about
+# 2^-9 sqrt(2L) with a safety factor of 4 gives 1.1e-2 sqrt(L).  Measured at
+# n = 256, d = 512, h = 1024: relative Frobenius errors 1e-4 (head) to 3.2e-2
+# (E, P) at L = 16 and up to 1.3e-2 at L = 4.  ReLU decisions on fp32 and
+# fp64 pre-activations within rounding of 0 can differ too and move one row.
+# So each gradient tensor is held to a relative Frobenius error of
+# max(2e-2, 1.25e-2 sqrt(L)).  A single differing ReLU decision moves one
+# token's whole contribution to one row of dW1 (7.6 % of max |dW1| measured
+# with 64 tokens), so the relative max error only guards against gross
+# errors (0.25).
+TOL_LOSS = 5e-3      # relative, on the mean loss
+
+
+def tol_grad(L):
+    return max(2e-2, 1.25e-2 * L ** 0.5)
+
+
+@pytest.fixture(scope="module")
+def H():
+    if not torch.cuda.is_available():
+        pytest.skip("no GPU")
+    from paper_2609_18145_gb300 import hcw
+    hcw.lib()
+    return hcw
+
+
+def device_problem(pr):
+    """Device tensors of a BlockProblem and the exact float64 values they hold."""
+    params, exact = {}, {}
+    for f in OB_FIELDS:
+        a = np.asarray(getattr(pr, f), dtype=np.float32)
+        t = torch.from_numpy(a).to(torch.bfloat16 if f in BF16 else torch.float32)
+        exact[f] = t.to(torch.float64).numpy()
+        params[f] = t.cuda().contiguous()
+    ids = torch.from_numpy(np.asarray(pr.ids, dtype=np.int32)).cuda()
+    return ids, params, exact
+
+
+OB_FIELDS = ("E", "P", "ln1_g", "ln1_b", "W_self", "W_nbr", "ln2_g", "ln2_b", "W1", "b1", "W2",
+             "b2", "lnf_g", "lnf_b", "Wh", "bh")
+
+
+def as_problem(pr, exact):
+    q = synth.BlockProblem(**{f: exact[f] for f in OB_FIELDS}, ids=np.asarray(pr.ids))
+    return q
+
+
+def rel(a, b):
+    return float(np.abs(a - b).max() / max(np.abs(b).max(), 1e-30))
+
+
+def relf(a, b):
+    return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-30))
+
+
+def check_grads(got, ref, L):
+    t = tol_grad(L)
+    for f in OB_FIELDS:
+        a = got[f]
+        assert relf(a, ref[f]) <= t, (f, relf(a, ref[f]), rel(a, ref[f]))
+        assert rel(a, ref[f]) <= 0.25, (f, relf(a, ref[f]), rel(a, ref[f]))
+
+
+CASES = [
+    # B, n, d, h, V, L
+    (2, 16, 64, 128, 11, 3),
+    (3, 32, 128, 256, 256, 4),
+    (1, 64, 192, 136, 37, 2),
+]
+
+
+@pytest.mark.parametrize("case", CASES, ids=lambda c: "B%d_n%d_d%d_h%d_V%d_L%d" % c)
+def test_block_step_matches_the_oracle(H, case):
+    B, n, d, h, V, L = case
+    pr = synth.block_problem(B, n, d, h, V, L, seed=7)
+    ids, params, exact = device_problem(pr)
+    loss, grads = H.hcw_block_step(ids, params)
+    torch.cuda.synchronize()
+    assert H.hcw_sync_status() == H.HCW_OK
+    ref_loss, ref = OB.step(as_problem(pr, exact), round_bf16=True)
+    assert abs(float(loss.item()) - ref_loss) <= TOL_LOSS * abs(ref_loss)
+    check_grads({f: g.cpu().numpy().astype(np.float64) for f, g in grads.items()}, ref, L)
+
+
+def test_an_id_outside_the_vocabulary_is_reported(H):
+    B, n, d, h, V, L = 2, 16, 64, 128, 11, 1
+    pr = synth.block_problem(B, n, d, h, V, L, seed=8)
+    ids, params, _ = device_problem(pr)
+    ids[1, 3] = V
+    H.hcw_block_step(ids, params)
+    assert H.hcw_sync_status() == H.HCW_ERR_INVALID_ARG
+    assert H.hcw_sync_status() == H.HCW_OK      # the report is read once
+
+
+def test_full_size_batch_is_the_weighted_sum_of_its_parts(H):
+    """Window 256, d = 512, h = 1024, V = 256, 16 layers, B = 64 (the metric's
+    shape): sequences are independent, so the batch's loss and gradients are
+    the size-weighted sums of those of 32 two-sequence steps; and the first
+    two sequences match the oracle."""
+    B, n, d, h, V, L = 64, 256, 512, 1024, 256, 16
+    pr = synth.block_problem(B, n, d, h, V, L, seed=9)
+    ids, params, exact = device_problem(pr)
+    loss, grads = H.hcw_block_step(ids, params)
+    grads = {f: g.clone() for f, g in grads.items()}
+    part_loss = 0.0
+    part = {f: torch.zeros_like(g) for f, g in grads.items()}
+    ws = torch.empty(H.hcw_block_workspace_bytes(2, n, d, h, V, L), dtype=torch.uint8,
+                     device="cuda")
+    first = None
+    for c in range(B // 2):
+        lc, gc = H.hcw_block_step(ids[2 * c:2 * c + 2].contiguous(), params, workspace=ws)
+        part_loss += float(lc.item()) * 2 / B
+        for f in OB_FIELDS:
+            part[f] += gc[f] * (2 / B)
+        if c == 0:
+            first = (float(lc.item()), {f: g.cpu().numpy().astype(np.float64) for f, g in gc.items()})
+    torch.cuda.synchronize()
+    assert H.hcw_sync_status() == H.HCW_OK
+    assert np.isfinite(float(loss.item()))
+    assert abs(float(loss.item()) - part_loss) <= 1e-4 * abs(part_loss)
+    for f in OB_FIELDS:
+        a, b = grads[f].cpu().numpy(), part[f].cpu().numpy()
+        assert rel(a, b) <= 1e-2, f
+    sub = synth.block_problem(B, n, d, h, V, L, seed=9)
+    sub.ids = np.asarray(pr.ids)[:2]
+    ref_loss, ref = OB.step(as_problem(sub, exact), round_bf16=True)
+    assert abs(first[0] - ref_loss) <= TOL_LOSS * abs(ref_loss)
+    check_grads(first[1], ref, L)
