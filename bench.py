@@ -606,6 +606,8 @@ def run_kernel_only(args):
     layer = 3
     if args.kernel == "decode":
         return run_decode(args, w, dev)
+    if args.kernel == "block":
+        return run_block(args, w, dev)
     if args.kernel == "step":
         # one whole step (stack forward + stack backward) of --batch sequences
         L = w["L"]
@@ -722,6 +724,72 @@ def run_decode(args, w, dev):
     return 0
 
 
+BLOCK_BF16 = {"E", "P", "W_self", "W_nbr", "W1", "W2", "Wh"}
+
+
+def run_block(args, w, dev):
+    """Time one training step (forward, loss, backward) of the character-LM
+    block around the workload's stack (hcw_block_step: hidden 2d, 256 symbols)
+    for --batch sequences, issued from the host and as a CUDA graph."""
+    import torch
+
+    from paper_2609_18145_gb300 import hcw as H
+    from paper_2609_18145_gb300 import synth
+
+    B, n, d, L = args.batch, w["n"], w["d"], w["L"]
+    h, V = 2 * d, 256
+    pr = synth.block_problem(B, n, d, h, V, L, seed=0)
+    params = {f: torch.from_numpy(getattr(pr, f)).to(
+        torch.bfloat16 if f in BLOCK_BF16 else torch.float32).to(dev).contiguous()
+        for f in H.BLOCK_FIELDS}
+    ids = torch.from_numpy(pr.ids.astype("int32")).to(dev)
+    grads = {f: torch.empty(tuple(params[f].shape), dtype=torch.float32, device=dev)
+             for f in H.BLOCK_FIELDS}
+    loss = torch.empty(1, dtype=torch.float32, device=dev)
+    ws = torch.empty(H.hcw_block_workspace_bytes(B, n, d, h, V, L), dtype=torch.uint8, device=dev)
+
+    def step():
+        H.hcw_block_step(ids, params, grads, loss=loss, workspace=ws)
+
+    def timed(fn, reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        a.record()
+        for _ in range(reps):
+            fn()
+        b.record()
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / reps
+
+    for _ in range(max(1, args.warmup)):
+        step()
+    c0 = H.hcw_launch_count()
+    host_ms = timed(step, max(1, args.steps))
+    launches = (H.hcw_launch_count() - c0) / max(1, args.steps)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        step()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=s):
+            step()
+    torch.cuda.synchronize()
+    g.replay()
+    graph_ms = timed(g.replay, max(1, args.steps))
+    if H.hcw_sync_status() != H.HCW_OK:
+        raise SystemExit("device error")
+    T = B * n
+    flops = T * (L * (9.0 * d * d + 12.0 * d * h) + 6.0 * d * V)
+    print(json.dumps({
+        "kernel": "block", "batch": B, "n": n, "d": d, "hidden": h, "vocab": V, "L": L,
+        "loss": float(loss.item()), "launches_per_step": launches,
+        "ms_per_step_host_issued": round(host_ms, 4), "ms_per_step_graph": round(graph_ms, 4),
+        "tokens_per_s_graph": round(T / (graph_ms * 1e-3)),
+        "flops_per_step": flops, "tflops_graph": round(flops / (graph_ms * 1e-3) / 1e12, 1)}),
+        flush=True)
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
     ap.add_argument("--gpus", type=int, default=1)
@@ -733,10 +801,11 @@ def main():
                          "CUDA graph of them")
     ap.add_argument("--no-cpu-baseline", action="store_true",
                     help="skip timing the CPU oracle (it is only timed at N = 1 anyway)")
-    ap.add_argument("--kernel", choices=("fwd", "dx", "dw", "step", "decode"),
+    ap.add_argument("--kernel", choices=("fwd", "dx", "dw", "step", "decode", "block"),
                     help="launch only this kernel kind, one whole step of --batch sequences "
-                         "(profiler captures), or decode one window of --batch sequences "
-                         "token by token; no bench line")
+                         "(profiler captures), decode one window of --batch sequences "
+                         "token by token, or one training step of the character-LM block "
+                         "around the stack; no bench line")
     ap.add_argument("--batch", type=int, default=64, help="sequences for --kernel runs")
     ap.add_argument("--schedule", choices=tuple(SCHEDULES), default="rot",
                     help="layer schedule of the stack: rot (the workload's rotated stack) or "

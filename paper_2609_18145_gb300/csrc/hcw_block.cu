@@ -109,13 +109,26 @@ __global__ void __launch_bounds__(kRowWarps * 32)
     if (lane == 0) stats[row] = make_float2(mean, rstd);
 }
 
-// a = bf16(relu(U + b1[col]))   U: [T][h] fp32 (the GEMM output)
-__global__ void bias_relu_kernel(const float* U, const float* b1, __nv_bfloat16* a, size_t total,
-                                 int h) {
-    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+// a = bf16(relu(U + b1[col]))   U: [T][h] fp32 (the GEMM output); eight
+// consecutive elements a thread (h % 8 == 0): two 16-byte loads, one store
+__global__ void bias_relu_kernel(const float* U, const float* b1, __nv_bfloat16* a, size_t total8,
+                                 int h8) {
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total8;
          i += (size_t)gridDim.x * blockDim.x) {
-        const float u = U[i] + b1[i % h];
-        a[i] = __float2bfloat16_rn(u > 0.f ? u : 0.f);
+        const int c = (int)(i % h8) * 8;
+        const float4 u0 = reinterpret_cast<const float4*>(U)[2 * i];
+        const float4 u1 = reinterpret_cast<const float4*>(U)[2 * i + 1];
+        const float4 b0 = *reinterpret_cast<const float4*>(b1 + c);
+        const float4 bb = *reinterpret_cast<const float4*>(b1 + c + 4);
+        const float v[8] = {u0.x + b0.x, u0.y + b0.y, u0.z + b0.z, u0.w + b0.w,
+                            u1.x + bb.x, u1.y + bb.y, u1.z + bb.z, u1.w + bb.w};
+        uint4 o;
+        uint32_t* w = &o.x;
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+            w[e] = pack_bf16x2(v[2 * e] > 0.f ? v[2 * e] : 0.f,
+                               v[2 * e + 1] > 0.f ? v[2 * e + 1] : 0.f);
+        reinterpret_cast<uint4*>(a)[i] = o;
     }
 }
 
@@ -144,79 +157,108 @@ __global__ void __launch_bounds__(kRowWarps * 32)
     if (lane == 0) atomicAdd(loss, (lse - (z[tgt] + bh[tgt])) * inv_N);
 }
 
-// dpre = bf16(da where relu(u) > 0, else 0)   (a = relu(u) holds the mask)
+// dpre = bf16(da where relu(u) > 0, else 0)   (a = relu(u) holds the mask);
+// eight consecutive elements a thread
 __global__ void relu_bwd_kernel(const float* da, const __nv_bfloat16* a, __nv_bfloat16* dpre,
-                                size_t total) {
-    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
-         i += (size_t)gridDim.x * blockDim.x)
-        dpre[i] = __float2bfloat16_rn(__bfloat162float(a[i]) > 0.f ? da[i] : 0.f);
-}
-
-// out[c] += sum over rows [r0, r0 + kColRows) of M[r][c]   (bf16 M [T][C];
-// out zeroed before the launch; one CTA per block of rows)
-constexpr int kColRows = 128;
-__global__ void colsum_kernel(const __nv_bfloat16* M, float* out, int T, int C) {
-    const int r0 = blockIdx.x * kColRows;
-    const int r1 = min(T, r0 + kColRows);
-    for (int c = threadIdx.x; c < C; c += blockDim.x) {
-        float s = 0.f;
-        for (int r = r0; r < r1; ++r) s += __bfloat162float(M[(size_t)r * C + c]);
-        atomicAdd(out + c, s);
+                                size_t total8) {
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total8;
+         i += (size_t)gridDim.x * blockDim.x) {
+        const float4 d0 = reinterpret_cast<const float4*>(da)[2 * i];
+        const float4 d1 = reinterpret_cast<const float4*>(da)[2 * i + 1];
+        const uint4 m = reinterpret_cast<const uint4*>(a)[i];
+        const float dv[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
+        const uint32_t mw[4] = {m.x, m.y, m.z, m.w};
+        uint4 o;
+        uint32_t* w = &o.x;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float2 am = unpack_bf16x2(mw[e]);
+            w[e] = pack_bf16x2(am.x > 0.f ? dv[2 * e] : 0.f, am.y > 0.f ? dv[2 * e + 1] : 0.f);
+        }
+        reinterpret_cast<uint4*>(dpre)[i] = o;
     }
 }
 
-// LayerNorm backward, one warp per row (rows r = blockIdx.x * 8 + warp, then
-// strided by the grid): with xhat = (x - mean) rstd and dxhat = dy g,
+// out[c] += sum over a tile of kColRows rows of M[r][c] (bf16 M [T][C]; out
+// zeroed before the launch): grid (ceil(C / 256), ceil(T / kColRows)), a
+// thread per column of its tile, the rows' loads independent of each other
+constexpr int kColRows = 64;
+__global__ void colsum_kernel(const __nv_bfloat16* M, float* out, int T, int C) {
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    if (c >= C) return;
+    const int r0 = blockIdx.y * kColRows;
+    const int r1 = min(T, r0 + kColRows);
+    float s = 0.f;
+#pragma unroll 8
+    for (int r = r0; r < r1; ++r) s += __bfloat162float(M[(size_t)r * C + c]);
+    atomicAdd(out + c, s);
+}
+
+// LayerNorm backward, one warp per row: with xhat = (x - mean) rstd and
+// dxhat = dy g,
 //   dx = rstd (dxhat - mean(dxhat) - xhat mean(dxhat xhat))  (+ dres)
-// written to dx_out (fp32) and, when dxb is given, as bf16; the scale and
-// shift gradients sum dy xhat and dy over the CTA's rows in shared memory,
-// then one atomic add per column and CTA.  dy is fp32 (dyf) or bf16 (dyb).
-// The CTA's rows go through shared-memory atomics (at most 8 rows at a time
-// on one column).
+// written to dx_out (fp32) and, when dxb is given, as bf16.  dy is fp32 (dyf)
+// or bf16 (dyb).  Every load of the row comes before any store: dres and
+// dx_out may be the same buffer (the gradient updated in place), and a load
+// placed after a store could not be moved ahead of it.  NV >= d / 32.
+template <int NV>
 __global__ void __launch_bounds__(kRowWarps * 32)
     ln_bwd_kernel(const float* dyf, const __nv_bfloat16* dyb, const float* x, const float2* stats,
-                  const float* g, const float* dres, float* dx_out, __nv_bfloat16* dxb,
-                  float* dgam, float* dbet, int T, int d) {
-    extern __shared__ float part[];   // [2][d]: dgam, dbet partials of this CTA
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int c = threadIdx.x; c < 2 * d; c += blockDim.x) part[c] = 0.f;
-    __syncthreads();
+                  const float* g, const float* dres, float* dx_out, __nv_bfloat16* dxb, int T,
+                  int d) {
+    const int lane = threadIdx.x & 31;
+    const int row = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
+    if (row >= T) return;
     const int nv = d >> 5;
-    for (int row = blockIdx.x * kRowWarps + warp; row < T; row += gridDim.x * kRowWarps) {
-        const size_t base = (size_t)row * d;
-        const float2 st = stats[row];
-        float xh[32], dh[32];
-        float s1 = 0.f, s2 = 0.f;
+    const size_t base = (size_t)row * d;
+    const float2 st = stats[row];
+    float xh[NV], dh[NV], rv[NV];
+    float s1 = 0.f, s2 = 0.f;
 #pragma unroll
-        for (int i = 0; i < 32; ++i) {
-            if (i < nv) {
-                const int c = i * 32 + lane;
-                const float dy = dyf ? dyf[base + c] : __bfloat162float(dyb[base + c]);
-                xh[i] = (x[base + c] - st.x) * st.y;
-                dh[i] = dy * g[c];
-                s1 += dh[i];
-                s2 += dh[i] * xh[i];
-                atomicAdd(&part[c], dy * xh[i]);
-                atomicAdd(&part[d + c], dy);
-            }
-        }
-        const float m1 = warp_sum(s1) / d, m2 = warp_sum(s2) / d;
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-            if (i < nv) {
-                const int c = i * 32 + lane;
-                float v = st.y * (dh[i] - m1 - xh[i] * m2);
-                if (dres) v += dres[base + c];
-                dx_out[base + c] = v;
-                if (dxb) dxb[base + c] = __float2bfloat16_rn(v);
-            }
+    for (int i = 0; i < NV; ++i) {
+        if (i < nv) {
+            const int c = i * 32 + lane;
+            rv[i] = dres ? dres[base + c] : 0.f;
+            const float dy = dyf ? dyf[base + c] : __bfloat162float(dyb[base + c]);
+            xh[i] = (x[base + c] - st.x) * st.y;
+            dh[i] = dy * g[c];
+            s1 += dh[i];
+            s2 += dh[i] * xh[i];
         }
     }
-    __syncthreads();
-    for (int c = threadIdx.x; c < d; c += blockDim.x) {
-        atomicAdd(dgam + c, part[c]);
-        atomicAdd(dbet + c, part[d + c]);
+    const float m1 = warp_sum(s1) / d, m2 = warp_sum(s2) / d;
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+        if (i < nv) {
+            const int c = i * 32 + lane;
+            const float v = st.y * (dh[i] - m1 - xh[i] * m2) + rv[i];
+            dx_out[base + c] = v;
+            if (dxb) dxb[base + c] = __float2bfloat16_rn(v);
+        }
     }
+}
+
+// LayerNorm scale and shift gradients: dgam[c] += sum of dy xhat, dbet[c] +=
+// sum of dy over a tile of kColRows rows (xhat recomputed from x and the row
+// statistics); grid (ceil(d / 256), ceil(T / kColRows)), a thread per column,
+// dgam and dbet zeroed before the launch
+__global__ void ln_param_kernel(const float* dyf, const __nv_bfloat16* dyb, const float* x,
+                                const float2* stats, int T, int d, float* dgam, float* dbet) {
+    const int c = blockIdx.x * blockDim.x + threadIdx.x;
+    if (c >= d) return;
+    const int r0 = blockIdx.y * kColRows;
+    const int r1 = min(T, r0 + kColRows);
+    float sg = 0.f, sb = 0.f;
+#pragma unroll 8
+    for (int r = r0; r < r1; ++r) {
+        const size_t e = (size_t)r * d + c;
+        const float dy = dyf ? dyf[e] : __bfloat162float(dyb[e]);
+        const float2 st = stats[r];
+        sg += dy * (x[e] - st.x) * st.y;
+        sb += dy;
+    }
+    atomicAdd(dgam + c, sg);
+    atomicAdd(dbet + c, sb);
 }
 
 // dE[ids[b][t]] += dx[b n + t]   (dE zeroed before the launch)
@@ -271,6 +313,14 @@ bool gemm(cublasHandle_t h, int M, int N, int K, const void* A, bool ta, const v
                         CUBLAS_GEMM_DEFAULT) == CUBLAS_STATUS_SUCCESS;
 }
 
+int sms_now() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
+        return 148;
+    return n;
+}
+
 size_t round256(size_t v) { return (v + 255) & ~(size_t)255; }
 
 // Workspace of one step (byte offsets; T = B n tokens):
@@ -282,9 +332,13 @@ size_t round256(size_t v) { return (v + 255) & ~(size_t)255; }
 //   m, hf [T][d] bf16          mixing output (per layer), head input
 //   U    [T][max(h, V, d)] fp32  every GEMM output with T rows, in turn
 //   dlog [T][V] bf16; dx [T][d] fp32; dxb [T][d] bf16; dpre [T][h] bf16;
-//   dh [T][d] bf16; then the mixing backward's own workspace
+//   dh [T][d] bf16; the mixing backward's own workspace; cuBLAS's workspace
+//   (handed to it every step, so that no call allocates and a CUDA graph can
+//   capture the step)
+constexpr size_t kBlasWs = (size_t)32 << 20;
 struct BlockWs {
-    size_t xs, h1, g, a, st1, st2, stf, m, hf, U, dlog, dx, dxb, dpre, dh, lws, lws_bytes, total;
+    size_t xs, h1, g, a, st1, st2, stf, m, hf, U, dlog, dx, dxb, dpre, dh, lws, lws_bytes,
+        blas, total;
 };
 
 BlockWs block_ws(int B, int n, int d, int h, int V, int L) {
@@ -314,6 +368,7 @@ BlockWs block_ws(int B, int n, int d, int h, int V, int L) {
     w.dh = take(T * d * 2);
     w.lws_bytes = hcw_workspace_bytes(B, n, d, HCW_BF16, HCW_CAUSAL);
     w.lws = take(w.lws_bytes);
+    w.blas = take(kBlasWs);
     w.total = o;
     return w;
 }
@@ -321,14 +376,6 @@ BlockWs block_ws(int B, int n, int d, int h, int V, int L) {
 }  // namespace
 
 namespace {
-
-int sms_now() {
-    int dev = 0, n = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
-        return 148;
-    return n;
-}
 
 bool block_sizes_ok(int B, int n, int d, int h, int V, int L) {
     return B >= 1 && n >= 2 && (n & (n - 1)) == 0 && d >= 64 && d % 64 == 0 && d <= 1024 &&
@@ -343,6 +390,24 @@ int ok_launch() { return count_launch(cudaGetLastError(), 1); }
 unsigned elem_grid(size_t total) {
     const size_t want = (total + 255) / 256, cap = (size_t)sms_now() * 16;
     return (unsigned)(want < cap ? (want ? want : 1) : cap);
+}
+
+// the LayerNorm backward (rows with room for d / 32 values a lane, d <= 1024)
+// and its scale / shift gradients (dgam, dbet zeroed before)
+void launch_ln_bwd(cudaStream_t st, const float* dyf, const __nv_bfloat16* dyb, const float* x,
+                   const float2* stats, const float* g, const float* dres, float* dx_out,
+                   __nv_bfloat16* dxb, float* dgam, float* dbet, int T, int d) {
+    const dim3 grid((T + kRowWarps - 1) / kRowWarps), blk(kRowWarps * 32);
+    if (d <= 128)
+        ln_bwd_kernel<4><<<grid, blk, 0, st>>>(dyf, dyb, x, stats, g, dres, dx_out, dxb, T, d);
+    else if (d <= 256)
+        ln_bwd_kernel<8><<<grid, blk, 0, st>>>(dyf, dyb, x, stats, g, dres, dx_out, dxb, T, d);
+    else if (d <= 512)
+        ln_bwd_kernel<16><<<grid, blk, 0, st>>>(dyf, dyb, x, stats, g, dres, dx_out, dxb, T, d);
+    else
+        ln_bwd_kernel<32><<<grid, blk, 0, st>>>(dyf, dyb, x, stats, g, dres, dx_out, dxb, T, d);
+    ln_param_kernel<<<dim3((d + 255) / 256, (T + kColRows - 1) / kColRows), 256, 0, st>>>(
+        dyf, dyb, x, stats, T, d, dgam, dbet);
 }
 
 int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads& gr, int B, int n,
@@ -371,10 +436,10 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
         return static_cast<const __nv_bfloat16*>(q) + off;
     };
     cublasHandle_t hb = blas_handle();
-    if (!hb || cublasSetStream(hb, st) != CUBLAS_STATUS_SUCCESS) return HCW_ERR_CUDA;
+    if (!hb || cublasSetStream(hb, st) != CUBLAS_STATUS_SUCCESS ||
+        cublasSetWorkspace(hb, ws + w.blas, kBlasWs) != CUBLAS_STATUS_SUCCESS)
+        return HCW_ERR_CUDA;
     const unsigned rows_grid = (unsigned)((T + kRowWarps - 1) / kRowWarps);
-    const unsigned ln_bwd_grid = rows_grid < (unsigned)sms_now() * 4 ? rows_grid : sms_now() * 4;
-    const size_t ln_smem = (size_t)2 * d * sizeof(float);
     int rc;
 #define HCW_TRY(expr)          \
     do {                       \
@@ -388,9 +453,9 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
     HCW_CU(cudaMemsetAsync(gr.E, 0, (size_t)V * d * 4, st));
     float* zero_d[] = {gr.ln1_g, gr.ln1_b, gr.ln2_g, gr.ln2_b, gr.b2};
     for (float* q : zero_d) HCW_CU(cudaMemsetAsync(q, 0, (size_t)L * d * 4, st));
-    HCW_CU(cudaMemsetAsync(gr.b1, 0, (size_t)L * h * 4, st));
     HCW_CU(cudaMemsetAsync(gr.lnf_g, 0, (size_t)d * 4, st));
     HCW_CU(cudaMemsetAsync(gr.lnf_b, 0, (size_t)d * 4, st));
+    HCW_CU(cudaMemsetAsync(gr.b1, 0, (size_t)L * h * 4, st));
     HCW_CU(cudaMemsetAsync(gr.bh, 0, (size_t)V * 4, st));
 
     // ------------------------------------------------------------ forward
@@ -407,7 +472,8 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
             S2(l), T, d);
         HCW_TRY(ok_launch());
         HCW_BLAS(gemm(hb, T, h, d, G(l), false, bf(p.W1, (size_t)l * h * d), true, U));
-        bias_relu_kernel<<<elem_grid(Th), 256, 0, st>>>(U, p.b1 + (size_t)l * h, A(l), Th, h);
+        bias_relu_kernel<<<elem_grid(Th / 8), 256, 0, st>>>(U, p.b1 + (size_t)l * h, A(l), Th / 8,
+                                                            h / 8);
         HCW_TRY(ok_launch());
         HCW_BLAS(gemm(hb, T, d, h, A(l), false, bf(p.W2, (size_t)l * d * h), true, U));
         const bool top = l + 1 == L;
@@ -425,37 +491,36 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
     // ----------------------------------------------------------- backward
     const unsigned gridT = (unsigned)((T + kColRows - 1) / kColRows);
     HCW_BLAS(gemm(hb, V, d, T, dlog, true, hf, false, gr.Wh));   // dWh = dlog^T hf
-    colsum_kernel<<<gridT, 256, 0, st>>>(dlog, gr.bh, T, V);
+    colsum_kernel<<<dim3((V + 255) / 256, gridT), 256, 0, st>>>(dlog, gr.bh, T, V);
     HCW_TRY(ok_launch());
     HCW_BLAS(gemm(hb, T, d, V, dlog, false, p.Wh, false, U));    // dhf = dlog Wh
-    ln_bwd_kernel<<<ln_bwd_grid, kRowWarps * 32, ln_smem, st>>>(
-        U, nullptr, X(L), sf, p.lnf_g, nullptr, dx, dxb, gr.lnf_g, gr.lnf_b, T, d);
-    HCW_TRY(ok_launch());
+    launch_ln_bwd(st, U, nullptr, X(L), sf, p.lnf_g, nullptr, dx, dxb, gr.lnf_g, gr.lnf_b, T, d);
+    HCW_TRY(count_launch(cudaGetLastError(), 2));
     for (int l = L - 1; l >= 0; --l) {
         // FFN sublayer: dxb = bf16(dx) is the gradient of its output
         HCW_BLAS(gemm(hb, d, h, T, dxb, true, A(l), false, gr.W2 + (size_t)l * d * h));
-        colsum_kernel<<<gridT, 256, 0, st>>>(dxb, gr.b2 + (size_t)l * d, T, d);
+        colsum_kernel<<<dim3((d + 255) / 256, gridT), 256, 0, st>>>(dxb, gr.b2 + (size_t)l * d, T,
+                                                                     d);
         HCW_TRY(ok_launch());
         HCW_BLAS(gemm(hb, T, h, d, dxb, false, bf(p.W2, (size_t)l * d * h), false, U));   // da
-        relu_bwd_kernel<<<elem_grid(Th), 256, 0, st>>>(U, A(l), dpre, Th);
+        relu_bwd_kernel<<<elem_grid(Th / 8), 256, 0, st>>>(U, A(l), dpre, Th / 8);
         HCW_TRY(ok_launch());
-        colsum_kernel<<<gridT, 256, 0, st>>>(dpre, gr.b1 + (size_t)l * h, T, h);
+        colsum_kernel<<<dim3((h + 255) / 256, gridT), 256, 0, st>>>(dpre, gr.b1 + (size_t)l * h, T,
+                                                                     h);
         HCW_TRY(ok_launch());
         HCW_BLAS(gemm(hb, h, d, T, dpre, true, G(l), false, gr.W1 + (size_t)l * h * d));
         HCW_BLAS(gemm(hb, T, d, h, dpre, false, bf(p.W1, (size_t)l * h * d), false, U));  // dg
-        ln_bwd_kernel<<<ln_bwd_grid, kRowWarps * 32, ln_smem, st>>>(
-            U, nullptr, XM(l), S2(l), p.ln2_g + (size_t)l * d, dx, dx, dxb,
+        launch_ln_bwd(st, U, nullptr, XM(l), S2(l), p.ln2_g + (size_t)l * d, dx, dx, dxb,
             gr.ln2_g + (size_t)l * d, gr.ln2_b + (size_t)l * d, T, d);
-        HCW_TRY(ok_launch());
+        HCW_TRY(count_launch(cudaGetLastError(), 2));
         // mixing sublayer: dxb = bf16(dx) is the gradient of M_l(h)
         HCW_TRY(hcw_layer_bwd(H1(l), nullptr, dxb, bf(p.W_self, (size_t)l * d * d),
                               bf(p.W_nbr, (size_t)l * d * d), l, -1, B, n, d, HCW_BF16, HCW_CAUSAL,
                               dh, gr.W_self + (size_t)l * d * d, gr.W_nbr + (size_t)l * d * d,
                               nullptr, w.lws_bytes ? ws + w.lws : nullptr, w.lws_bytes, st));
-        ln_bwd_kernel<<<ln_bwd_grid, kRowWarps * 32, ln_smem, st>>>(
-            nullptr, dh, X(l), S1(l), p.ln1_g + (size_t)l * d, dx, dx, dxb,
+        launch_ln_bwd(st, nullptr, dh, X(l), S1(l), p.ln1_g + (size_t)l * d, dx, dx, dxb,
             gr.ln1_g + (size_t)l * d, gr.ln1_b + (size_t)l * d, T, d);
-        HCW_TRY(ok_launch());
+        HCW_TRY(count_launch(cudaGetLastError(), 2));
     }
     embed_bwd_kernel<<<elem_grid(Td), 256, 0, st>>>(ids, dx, gr.E, B, n, d, V);
     HCW_TRY(ok_launch());
