@@ -109,6 +109,78 @@ __global__ void __launch_bounds__(kRowWarps * 32)
     if (lane == 0) stats[row] = make_float2(mean, rstd);
 }
 
+// Four consecutive features at element e (a multiple of 4): fp32 as one
+// 16-byte access, bf16 as one 8-byte access.
+__device__ __forceinline__ float4 ld4(const float* p, size_t e) {
+    return *reinterpret_cast<const float4*>(p + e);
+}
+__device__ __forceinline__ float4 ld4(const __nv_bfloat16* p, size_t e) {
+    const uint2 u = *reinterpret_cast<const uint2*>(p + e);
+    const float2 a = unpack_bf16x2(u.x), b = unpack_bf16x2(u.y);
+    return make_float4(a.x, a.y, b.x, b.y);
+}
+__device__ __forceinline__ void st4(float* p, size_t e, float4 v) {
+    *reinterpret_cast<float4*>(p + e) = v;
+}
+__device__ __forceinline__ void st4(__nv_bfloat16* p, size_t e, float4 v) {
+    *reinterpret_cast<uint2*>(p + e) = make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
+}
+__device__ __forceinline__ float4 add4(float4 a, float4 b) {
+    return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w);
+}
+__device__ __forceinline__ float sum4(float4 a) { return a.x + a.y + a.z + a.w; }
+
+// ln_fwd_kernel for d a multiple of 128: lane holds features 4 (i 32 + lane) ..
+// + 3 for i < d / 128 <= NV4.
+template <int NV4>
+__global__ void __launch_bounds__(kRowWarps * 32)
+    ln_fwd4_kernel(const float* x_in, const __nv_bfloat16* add1, const float* add2,
+                   const float* badd, float* x_out, const float* g, const float* b,
+                   __nv_bfloat16* y, float2* stats, int T, int d) {
+    const int lane = threadIdx.x & 31;
+    const int row = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
+    if (row >= T) return;
+    const int nv = d >> 7;
+    const size_t base = (size_t)row * d;
+    float4 v[NV4];
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < NV4; ++i) {
+        if (i < nv) {
+            const int c = (i * 32 + lane) * 4;
+            float4 t = ld4(x_in, base + c);
+            if (add1) t = add4(t, ld4(add1, base + c));
+            if (add2) t = add4(t, ld4(add2, base + c));
+            if (badd) t = add4(t, ld4(badd, (size_t)c));
+            v[i] = t;
+            s += sum4(t);
+        }
+    }
+    const float mean = warp_sum(s) / d;
+    float q = 0.f;
+#pragma unroll
+    for (int i = 0; i < NV4; ++i) {
+        if (i < nv) {
+            const float4 t = v[i];
+            q += (t.x - mean) * (t.x - mean) + (t.y - mean) * (t.y - mean) +
+                 (t.z - mean) * (t.z - mean) + (t.w - mean) * (t.w - mean);
+        }
+    }
+    const float rstd = rsqrtf(warp_sum(q) / d + kLnEps);
+#pragma unroll
+    for (int i = 0; i < NV4; ++i) {
+        if (i < nv) {
+            const int c = (i * 32 + lane) * 4;
+            const float4 t = v[i], gg = ld4(g, (size_t)c), bb = ld4(b, (size_t)c);
+            if (x_out) st4(x_out, base + c, t);
+            st4(y, base + c,
+                make_float4((t.x - mean) * rstd * gg.x + bb.x, (t.y - mean) * rstd * gg.y + bb.y,
+                            (t.z - mean) * rstd * gg.z + bb.z, (t.w - mean) * rstd * gg.w + bb.w));
+        }
+    }
+    if (lane == 0) stats[row] = make_float2(mean, rstd);
+}
+
 // a = bf16(relu(U + b1[col]))   U: [T][h] fp32 (the GEMM output); eight
 // consecutive elements a thread (h % 8 == 0): two 16-byte loads, one store
 __global__ void bias_relu_kernel(const float* U, const float* b1, __nv_bfloat16* a, size_t total8,
@@ -261,6 +333,102 @@ __global__ void ln_param_kernel(const float* dyf, const __nv_bfloat16* dyb, cons
     atomicAdd(dbet + c, sb);
 }
 
+// ln_bwd_kernel for d a multiple of 128 (four features a lane and access).
+template <int NV4, typename DY>
+__global__ void __launch_bounds__(kRowWarps * 32)
+    ln_bwd4_kernel(const DY* dy, const float* x, const float2* stats, const float* g,
+                   const float* dres, float* dx_out, __nv_bfloat16* dxb, int T, int d) {
+    const int lane = threadIdx.x & 31;
+    const int row = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
+    if (row >= T) return;
+    const int nv = d >> 7;
+    const size_t base = (size_t)row * d;
+    const float2 st = stats[row];
+    float4 xh[NV4], dh[NV4], rv[NV4];
+    float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+    for (int i = 0; i < NV4; ++i) {
+        if (i < nv) {
+            const int c = (i * 32 + lane) * 4;
+            rv[i] = dres ? ld4(dres, base + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+            const float4 y = ld4(dy, base + c), xx = ld4(x, base + c), gg = ld4(g, (size_t)c);
+            xh[i] = make_float4((xx.x - st.x) * st.y, (xx.y - st.x) * st.y,
+                                (xx.z - st.x) * st.y, (xx.w - st.x) * st.y);
+            dh[i] = make_float4(y.x * gg.x, y.y * gg.y, y.z * gg.z, y.w * gg.w);
+            s1 += sum4(dh[i]);
+            s2 += dh[i].x * xh[i].x + dh[i].y * xh[i].y + dh[i].z * xh[i].z + dh[i].w * xh[i].w;
+        }
+    }
+    const float m1 = warp_sum(s1) / d, m2 = warp_sum(s2) / d;
+#pragma unroll
+    for (int i = 0; i < NV4; ++i) {
+        if (i < nv) {
+            const int c = (i * 32 + lane) * 4;
+            const float4 v = make_float4(st.y * (dh[i].x - m1 - xh[i].x * m2) + rv[i].x,
+                                         st.y * (dh[i].y - m1 - xh[i].y * m2) + rv[i].y,
+                                         st.y * (dh[i].z - m1 - xh[i].z * m2) + rv[i].z,
+                                         st.y * (dh[i].w - m1 - xh[i].w * m2) + rv[i].w);
+            st4(dx_out, base + c, v);
+            if (dxb) st4(dxb, base + c, v);
+        }
+    }
+}
+
+// ln_param_kernel with four columns a thread (d a multiple of 4) over tiles
+// of kParamRows rows: grid (ceil(d / 512), ceil(T / kParamRows)), 128
+// threads.  Each tile writes its sums as one row of part [tiles][2 d] (dy xhat,
+// then dy); ln_param_reduce_kernel adds the rows up.  No atomics: with every
+// tile adding into the same 2 d addresses they would queue in L2.
+constexpr int kParamRows = 32;
+template <typename DY>
+__global__ void ln_param4_kernel(const DY* dy, const float* x, const float2* stats, int T, int d,
+                                 float* part) {
+    const int c = (blockIdx.x * blockDim.x + threadIdx.x) * 4;
+    if (c >= d) return;
+    const int r0 = blockIdx.y * kParamRows;
+    const int r1 = min(T, r0 + kParamRows);
+    float4 sg = make_float4(0.f, 0.f, 0.f, 0.f), sb = sg;
+#pragma unroll 4
+    for (int r = r0; r < r1; ++r) {
+        const size_t e = (size_t)r * d + c;
+        const float4 y = ld4(dy, e), xx = ld4(x, e);
+        const float2 st = stats[r];
+        sg.x += y.x * (xx.x - st.x) * st.y;
+        sg.y += y.y * (xx.y - st.x) * st.y;
+        sg.z += y.z * (xx.z - st.x) * st.y;
+        sg.w += y.w * (xx.w - st.x) * st.y;
+        sb = add4(sb, y);
+    }
+    float* row = part + (size_t)blockIdx.y * 2 * d;
+    st4(row, (size_t)c, sg);
+    st4(row, (size_t)d + c, sb);
+}
+
+// dgam[c] = sum over the nblk rows of part [nblk][2 d] of column c, dbet[c] of
+// column d + c.  A CTA per 32 columns: warp w adds rows w, w + 8, ... (each
+// warp load one 128-byte row piece), then the eight warp sums meet in shared
+// memory in a fixed order.
+__global__ void __launch_bounds__(256) ln_param_reduce_kernel(const float* part, int nblk, int d,
+                                                              float* dgam, float* dbet) {
+    __shared__ float acc[8][32];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int c = blockIdx.x * 32 + lane;
+    float s = 0.f;
+    if (c < 2 * d)
+        for (int b = warp; b < nblk; b += 8) s += part[(size_t)b * 2 * d + c];
+    acc[warp][lane] = s;
+    __syncthreads();
+    if (warp == 0 && c < 2 * d) {
+        float t = 0.f;
+#pragma unroll
+        for (int w = 0; w < 8; ++w) t += acc[w][lane];
+        if (c < d)
+            dgam[c] = t;
+        else
+            dbet[c - d] = t;
+    }
+}
+
 // dE[ids[b][t]] += dx[b n + t]   (dE zeroed before the launch)
 __global__ void embed_bwd_kernel(const int* ids, const float* dx, float* dE, int B, int n, int d,
                                  int V) {
@@ -337,7 +505,7 @@ size_t round256(size_t v) { return (v + 255) & ~(size_t)255; }
 //   capture the step)
 constexpr size_t kBlasWs = (size_t)32 << 20;
 struct BlockWs {
-    size_t xs, h1, g, a, st1, st2, stf, m, hf, U, dlog, dx, dxb, dpre, dh, lws, lws_bytes,
+    size_t xs, h1, g, a, st1, st2, stf, m, hf, U, dlog, dx, dxb, dpre, dh, lnp, lws, lws_bytes,
         blas, total;
 };
 
@@ -366,6 +534,7 @@ BlockWs block_ws(int B, int n, int d, int h, int V, int L) {
     w.dxb = take(T * d * 2);
     w.dpre = take(T * h * 2);
     w.dh = take(T * d * 2);
+    w.lnp = take((T + kParamRows - 1) / kParamRows * 2 * (size_t)d * 4);   // LayerNorm partials
     w.lws_bytes = hcw_workspace_bytes(B, n, d, HCW_BF16, HCW_CAUSAL);
     w.lws = take(w.lws_bytes);
     w.blas = take(kBlasWs);
@@ -392,11 +561,59 @@ unsigned elem_grid(size_t total) {
     return (unsigned)(want < cap ? (want ? want : 1) : cap);
 }
 
-// the LayerNorm backward (rows with room for d / 32 values a lane, d <= 1024)
-// and its scale / shift gradients (dgam, dbet zeroed before)
-void launch_ln_bwd(cudaStream_t st, const float* dyf, const __nv_bfloat16* dyb, const float* x,
-                   const float2* stats, const float* g, const float* dres, float* dx_out,
-                   __nv_bfloat16* dxb, float* dgam, float* dbet, int T, int d) {
+// LayerNorm forward rows: four features a lane and access when d is a
+// multiple of 128, else one (ln_fwd_kernel)
+void launch_ln_fwd(cudaStream_t st, const float* x_in, const __nv_bfloat16* add1, const float* add2,
+                   const float* badd, float* x_out, const float* g, const float* b,
+                   __nv_bfloat16* y, float2* stats, int T, int d) {
+    const dim3 grid((T + kRowWarps - 1) / kRowWarps), blk(kRowWarps * 32);
+    const int v4 = d / 128;
+    if (d % 128 != 0)
+        ln_fwd_kernel<<<grid, blk, 0, st>>>(x_in, add1, add2, badd, x_out, g, b, y, stats, T, d);
+    else if (v4 <= 1)
+        ln_fwd4_kernel<1><<<grid, blk, 0, st>>>(x_in, add1, add2, badd, x_out, g, b, y, stats, T, d);
+    else if (v4 <= 2)
+        ln_fwd4_kernel<2><<<grid, blk, 0, st>>>(x_in, add1, add2, badd, x_out, g, b, y, stats, T, d);
+    else if (v4 <= 4)
+        ln_fwd4_kernel<4><<<grid, blk, 0, st>>>(x_in, add1, add2, badd, x_out, g, b, y, stats, T, d);
+    else
+        ln_fwd4_kernel<8><<<grid, blk, 0, st>>>(x_in, add1, add2, badd, x_out, g, b, y, stats, T, d);
+}
+
+template <typename DY>
+void launch_ln_bwd4(cudaStream_t st, const DY* dy, const float* x, const float2* stats,
+                    const float* g, const float* dres, float* dx_out, __nv_bfloat16* dxb,
+                    float* part, float* dgam, float* dbet, int T, int d) {
+    const dim3 grid((T + kRowWarps - 1) / kRowWarps), blk(kRowWarps * 32);
+    const int v4 = d / 128;
+    if (v4 <= 1)
+        ln_bwd4_kernel<1, DY><<<grid, blk, 0, st>>>(dy, x, stats, g, dres, dx_out, dxb, T, d);
+    else if (v4 <= 2)
+        ln_bwd4_kernel<2, DY><<<grid, blk, 0, st>>>(dy, x, stats, g, dres, dx_out, dxb, T, d);
+    else if (v4 <= 4)
+        ln_bwd4_kernel<4, DY><<<grid, blk, 0, st>>>(dy, x, stats, g, dres, dx_out, dxb, T, d);
+    else
+        ln_bwd4_kernel<8, DY><<<grid, blk, 0, st>>>(dy, x, stats, g, dres, dx_out, dxb, T, d);
+    const int tiles = (T + kParamRows - 1) / kParamRows;
+    ln_param4_kernel<DY><<<dim3((d / 4 + 127) / 128, tiles), 128, 0, st>>>(dy, x, stats, T, d, part);
+    ln_param_reduce_kernel<<<(2 * d + 31) / 32, 256, 0, st>>>(part, tiles, d, dgam, dbet);
+}
+
+// the LayerNorm backward (rows, then the scale / shift gradients; dgam, dbet
+// zeroed before): four features a lane and access when d is a multiple of
+// 128, else one (ln_bwd_kernel with room for d / 32 values a lane)
+// Returns the number of kernels launched.
+int launch_ln_bwd(cudaStream_t st, const float* dyf, const __nv_bfloat16* dyb, const float* x,
+                  const float2* stats, const float* g, const float* dres, float* dx_out,
+                  __nv_bfloat16* dxb, float* part, float* dgam, float* dbet, int T, int d) {
+    if (d % 128 == 0) {
+        if (dyf)
+            launch_ln_bwd4<float>(st, dyf, x, stats, g, dres, dx_out, dxb, part, dgam, dbet, T, d);
+        else
+            launch_ln_bwd4<__nv_bfloat16>(st, dyb, x, stats, g, dres, dx_out, dxb, part, dgam,
+                                          dbet, T, d);
+        return 3;
+    }
     const dim3 grid((T + kRowWarps - 1) / kRowWarps), blk(kRowWarps * 32);
     if (d <= 128)
         ln_bwd_kernel<4><<<grid, blk, 0, st>>>(dyf, dyb, x, stats, g, dres, dx_out, dxb, T, d);
@@ -408,6 +625,7 @@ void launch_ln_bwd(cudaStream_t st, const float* dyf, const __nv_bfloat16* dyb, 
         ln_bwd_kernel<32><<<grid, blk, 0, st>>>(dyf, dyb, x, stats, g, dres, dx_out, dxb, T, d);
     ln_param_kernel<<<dim3((d + 255) / 256, (T + kColRows - 1) / kColRows), 256, 0, st>>>(
         dyf, dyb, x, stats, T, d, dgam, dbet);
+    return 2;
 }
 
 int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads& gr, int B, int n,
@@ -429,6 +647,7 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
     float* U = reinterpret_cast<float*>(ws + w.U);
     auto* dlog = reinterpret_cast<__nv_bfloat16*>(ws + w.dlog);
     float* dx = reinterpret_cast<float*>(ws + w.dx);
+    float* lnp = reinterpret_cast<float*>(ws + w.lnp);
     auto* dxb = reinterpret_cast<__nv_bfloat16*>(ws + w.dxb);
     auto* dpre = reinterpret_cast<__nv_bfloat16*>(ws + w.dpre);
     auto* dh = reinterpret_cast<__nv_bfloat16*>(ws + w.dh);
@@ -461,14 +680,13 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
     // ------------------------------------------------------------ forward
     embed_fwd_kernel<<<elem_grid(Td), 256, 0, st>>>(ids, bf(p.E, 0), bf(p.P, 0), X(0), B, n, d, V);
     HCW_TRY(ok_launch());
-    ln_fwd_kernel<<<rows_grid, kRowWarps * 32, 0, st>>>(X(0), nullptr, nullptr, nullptr, nullptr,
-                                                        p.ln1_g, p.ln1_b, H1(0), S1(0), T, d);
+    launch_ln_fwd(st, X(0), nullptr, nullptr, nullptr, nullptr, p.ln1_g, p.ln1_b, H1(0), S1(0), T,
+                  d);
     HCW_TRY(ok_launch());
     for (int l = 0; l < L; ++l) {
         HCW_TRY(hcw_layer_fwd(H1(l), bf(p.W_self, (size_t)l * d * d), bf(p.W_nbr, (size_t)l * d * d),
                               nullptr, l, -1, B, n, d, HCW_BF16, HCW_CAUSAL, m, nullptr, st));
-        ln_fwd_kernel<<<rows_grid, kRowWarps * 32, 0, st>>>(
-            X(l), m, nullptr, nullptr, XM(l), p.ln2_g + (size_t)l * d, p.ln2_b + (size_t)l * d, G(l),
+        launch_ln_fwd(st, X(l), m, nullptr, nullptr, XM(l), p.ln2_g + (size_t)l * d, p.ln2_b + (size_t)l * d, G(l),
             S2(l), T, d);
         HCW_TRY(ok_launch());
         HCW_BLAS(gemm(hb, T, h, d, G(l), false, bf(p.W1, (size_t)l * h * d), true, U));
@@ -477,8 +695,7 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
         HCW_TRY(ok_launch());
         HCW_BLAS(gemm(hb, T, d, h, A(l), false, bf(p.W2, (size_t)l * d * h), true, U));
         const bool top = l + 1 == L;
-        ln_fwd_kernel<<<rows_grid, kRowWarps * 32, 0, st>>>(
-            XM(l), nullptr, U, p.b2 + (size_t)l * d, X(l + 1),
+        launch_ln_fwd(st, XM(l), nullptr, U, p.b2 + (size_t)l * d, X(l + 1),
             top ? p.lnf_g : p.ln1_g + (size_t)(l + 1) * d,
             top ? p.lnf_b : p.ln1_b + (size_t)(l + 1) * d, top ? hf : H1(l + 1), top ? sf : S1(l + 1),
             T, d);
@@ -494,8 +711,9 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
     colsum_kernel<<<dim3((V + 255) / 256, gridT), 256, 0, st>>>(dlog, gr.bh, T, V);
     HCW_TRY(ok_launch());
     HCW_BLAS(gemm(hb, T, d, V, dlog, false, p.Wh, false, U));    // dhf = dlog Wh
-    launch_ln_bwd(st, U, nullptr, X(L), sf, p.lnf_g, nullptr, dx, dxb, gr.lnf_g, gr.lnf_b, T, d);
-    HCW_TRY(count_launch(cudaGetLastError(), 2));
+    int nk = launch_ln_bwd(st, U, nullptr, X(L), sf, p.lnf_g, nullptr, dx, dxb, lnp, gr.lnf_g,
+                           gr.lnf_b, T, d);
+    HCW_TRY(count_launch(cudaGetLastError(), nk));
     for (int l = L - 1; l >= 0; --l) {
         // FFN sublayer: dxb = bf16(dx) is the gradient of its output
         HCW_BLAS(gemm(hb, d, h, T, dxb, true, A(l), false, gr.W2 + (size_t)l * d * h));
@@ -510,17 +728,17 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
         HCW_TRY(ok_launch());
         HCW_BLAS(gemm(hb, h, d, T, dpre, true, G(l), false, gr.W1 + (size_t)l * h * d));
         HCW_BLAS(gemm(hb, T, d, h, dpre, false, bf(p.W1, (size_t)l * h * d), false, U));  // dg
-        launch_ln_bwd(st, U, nullptr, XM(l), S2(l), p.ln2_g + (size_t)l * d, dx, dx, dxb,
-            gr.ln2_g + (size_t)l * d, gr.ln2_b + (size_t)l * d, T, d);
-        HCW_TRY(count_launch(cudaGetLastError(), 2));
+        nk = launch_ln_bwd(st, U, nullptr, XM(l), S2(l), p.ln2_g + (size_t)l * d, dx, dx, dxb, lnp,
+                           gr.ln2_g + (size_t)l * d, gr.ln2_b + (size_t)l * d, T, d);
+        HCW_TRY(count_launch(cudaGetLastError(), nk));
         // mixing sublayer: dxb = bf16(dx) is the gradient of M_l(h)
         HCW_TRY(hcw_layer_bwd(H1(l), nullptr, dxb, bf(p.W_self, (size_t)l * d * d),
                               bf(p.W_nbr, (size_t)l * d * d), l, -1, B, n, d, HCW_BF16, HCW_CAUSAL,
                               dh, gr.W_self + (size_t)l * d * d, gr.W_nbr + (size_t)l * d * d,
                               nullptr, w.lws_bytes ? ws + w.lws : nullptr, w.lws_bytes, st));
-        launch_ln_bwd(st, nullptr, dh, X(l), S1(l), p.ln1_g + (size_t)l * d, dx, dx, dxb,
-            gr.ln1_g + (size_t)l * d, gr.ln1_b + (size_t)l * d, T, d);
-        HCW_TRY(count_launch(cudaGetLastError(), 2));
+        nk = launch_ln_bwd(st, nullptr, dh, X(l), S1(l), p.ln1_g + (size_t)l * d, dx, dx, dxb, lnp,
+                           gr.ln1_g + (size_t)l * d, gr.ln1_b + (size_t)l * d, T, d);
+        HCW_TRY(count_launch(cudaGetLastError(), nk));
     }
     embed_bwd_kernel<<<elem_grid(Td), 256, 0, st>>>(ids, dx, gr.E, B, n, d, V);
     HCW_TRY(ok_launch());
