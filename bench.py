@@ -512,7 +512,7 @@ def run_ours(args):
     outs_h = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
     h2d = x_h.numel() * x_h.element_size() + dy_h.numel() * dy_h.element_size()
     d2h = sum(t.numel() * t.element_size() for t in outs_h)
-    e2e_steps = max(4, args.steps // 2)
+    e2e_steps = max(4, args.steps)
     ins = [(x.clone(), dy.clone()) for _ in range(2)]
     stage = [[torch.empty_like(t) for t in outs] for _ in range(2)]
     graphs = [capture(*ins[b]) if not args.no_graph else None for b in range(2)]

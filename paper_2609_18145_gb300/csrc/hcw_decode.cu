@@ -34,8 +34,9 @@
 //     bytes have landed, with no fence or barrier between the CTAs.
 // No layer boundary goes through global memory or a grid-wide barrier.  A tile
 // holds 16 rows, below the 64-row minimum of a tcgen05 MMA, so the contraction
-// uses the warp-level bf16 MMA (m16n8k16); at decode sizes the step is bound by
-// the weight stream and the per-layer handoff, not by the MMAs.
+// uses the warp-level bf16 MMA (m16n8k16).  That path runs at about 1/15 of
+// tcgen05's rate on this GPU, and with the in-kernel weight stream it is one
+// of the two bounds of a layer, about equal in size.
 #include "hcw_internal.h"
 #include "hcw_ptx.cuh"
 
