@@ -385,7 +385,8 @@ size_t hcw_decode_cache_bytes(const int* dims, int layer0, int L, int B, int n, 
  * products on cuBLAS (bf16 operands, fp32 accumulation and output).
  * Needs n a power of two, d a multiple of 64 and <= 1024, h a multiple of 8,
  * V >= 2.  An id outside [0, V) is read as 0 and reported by hcw_sync_status
- * as HCW_ERR_INVALID_ARG.  Asynchronous on `stream`.
+ * as HCW_ERR_INVALID_ARG.  Asynchronous on `stream`; calls from several host
+ * threads on one device enqueue one at a time (they share its cuBLAS handle).
  */
 typedef struct {
     const void* E;

@@ -457,6 +457,15 @@ __global__ void pos_bwd_kernel(const float* dx, float* dP, int B, int n, int d) 
 
 namespace {
 
+// Serialises the steps enqueued on one device: they share its cuBLAS handle,
+// whose stream and workspace each step sets.
+std::mutex& device_step_mutex() {
+    static std::mutex mus[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
+    return mus[dev];
+}
+
 // cuBLAS handle of each device, created on first use and kept for the process
 cublasHandle_t blas_handle() {
     static std::mutex mu;
@@ -794,6 +803,7 @@ int hcw_block_step(const int* ids, const hcw_block_params* params, const hcw_blo
         return HCW_ERR_ALIGNMENT;
     const size_t need = block_ws(B, n, d, h, V, L).total;
     if (!workspace || ws_bytes < need || !a16(workspace)) return HCW_ERR_WORKSPACE;
+    std::lock_guard<std::mutex> lock(device_step_mutex());
     return block_step(ids, p, g, B, n, d, h, V, L, loss, static_cast<uint8_t*>(workspace),
                       (cudaStream_t)stream);
 }
