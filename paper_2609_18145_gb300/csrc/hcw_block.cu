@@ -379,7 +379,7 @@ __global__ void __launch_bounds__(kRowWarps * 32)
 // threads.  Each tile writes its sums as one row of part [tiles][2 d] (dy xhat,
 // then dy); ln_param_reduce_kernel adds the rows up.  No atomics: with every
 // tile adding into the same 2 d addresses they would queue in L2.
-constexpr int kParamRows = 32;
+constexpr int kParamRows = 16;
 template <typename DY>
 __global__ void ln_param4_kernel(const DY* dy, const float* x, const float2* stats, int T, int d,
                                  float* part) {
@@ -388,7 +388,7 @@ __global__ void ln_param4_kernel(const DY* dy, const float* x, const float2* sta
     const int r0 = blockIdx.y * kParamRows;
     const int r1 = min(T, r0 + kParamRows);
     float4 sg = make_float4(0.f, 0.f, 0.f, 0.f), sb = sg;
-#pragma unroll 4
+#pragma unroll 8
     for (int r = r0; r < r1; ++r) {
         const size_t e = (size_t)r * d + c;
         const float4 y = ld4(dy, e), xx = ld4(x, e);
