@@ -463,6 +463,10 @@ DECODE_CASES = [
     # d = 1024: 16 CTAs of 64 columns, 8 chunks a part; d = 192: 12 CTAs of 16
     ("rot_n16_B3_d1024", 3, 16, 1024, CAUSAL | RESIDUAL | RELU, None, 0, 4),
     ("mixa_n32_B33_d192", 33, 32, 192, CAUSAL | RESIDUAL | RELU, [-1, 4, -3, 2, 1, -1, 0], 0, 7),
+    # one sequence, one layer, d = 64 (a cluster of 4); 17 sequences at d = 256
+    # (16 CTAs of 16 columns, a ragged second row block), no residual
+    ("rot_n8_B1_d64_L1", 1, 8, 64, CAUSAL | RESIDUAL | RELU, None, 2, 1),
+    ("rot_n16_B17_d256_plain", 17, 16, 256, CAUSAL | RELU, None, 0, 3),
 ]
 
 
