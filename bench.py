@@ -356,21 +356,22 @@ def run_ours(args):
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
 
-    def step_calls(xin, dyin):
+    def step_calls(xin, dyin, outs=None):
+        oWs, oWn, ob = outs if outs is not None else (gWs, gWn, gb)
         H.hcw_stack_fwd(xin, Ws, Wn, bias, 0, -1, flags, y=y, acts=acts, masks=masks,
                         workspace=fws, dims=dims)
-        H.hcw_stack_bwd(xin, acts, masks, dyin, Ws, Wn, 0, -1, flags, dx=dx, dW_self=gWs,
-                        dW_nbr=gWn, dbias=gb, workspace=ws, dims=dims)
+        H.hcw_stack_bwd(xin, acts, masks, dyin, Ws, Wn, 0, -1, flags, dx=dx, dW_self=oWs,
+                        dW_nbr=oWn, dbias=ob, workspace=ws, dims=dims)
 
-    def capture(xin, dyin):
+    def capture(xin, dyin, outs=None):
         # the step's launches, recorded once and replayed: no host work per step
         g = torch.cuda.CUDAGraph()
         side = torch.cuda.Stream()
         side.wait_stream(torch.cuda.current_stream())
         with torch.cuda.stream(side):
-            step_calls(xin, dyin)          # first call on this stream: one-time set-up
+            step_calls(xin, dyin, outs)    # first call on this stream: one-time set-up
             with torch.cuda.graph(g, stream=side):
-                step_calls(xin, dyin)
+                step_calls(xin, dyin, outs)
         torch.cuda.current_stream().wait_stream(side)
         return g
 
@@ -501,9 +502,9 @@ def run_ours(args):
     # weight and bias gradients) out to pinned host memory.  Steps are
     # pipelined as a training loop would run them: step i + 1's inputs come in
     # on one copy stream and step i's gradients go out on another while step i
-    # (or i + 1) computes, with double-buffered inputs and a device staging
-    # copy of the gradients; the timed span runs from the first input copy to
-    # the last gradient copy, and each step still flushes L2 (inside the span).
+    # (or i + 1) computes, with double-buffered inputs and gradient outputs
+    # (two graphs); the timed span runs from the first input copy to the last
+    # gradient copy, and each step still flushes L2 (inside the span).
     x_h = torch.empty(x.shape, dtype=x.dtype, pin_memory=True)
     dy_h = torch.empty(dy.shape, dtype=dy.dtype, pin_memory=True)
     x_h.copy_(x)
@@ -514,8 +515,8 @@ def run_ours(args):
     d2h = sum(t.numel() * t.element_size() for t in outs_h)
     e2e_steps = max(4, args.steps)
     ins = [(x.clone(), dy.clone()) for _ in range(2)]
-    stage = [[torch.empty_like(t) for t in outs] for _ in range(2)]
-    graphs = [capture(*ins[b]) if not args.no_graph else None for b in range(2)]
+    res = [tuple(torch.empty_like(t) for t in outs) for _ in range(2)]
+    graphs = [capture(*ins[b], res[b]) if not args.no_graph else None for b in range(2)]
     s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
     ev = {k: [torch.cuda.Event() for _ in range(2)] for k in ("in", "used", "out", "sent")}
     replicas.barrier()
@@ -538,21 +539,19 @@ def run_ours(args):
         if i + 1 < e2e_steps:
             load(i + 1)
         stream.wait_event(ev["in"][b])
+        if i >= 2:
+            stream.wait_event(ev["sent"][b])        # step i - 2's gradients have left
         flush.fill_(i & 0xFF)
         if graphs[b] is not None:
             graphs[b].replay()
         else:
-            step_calls(*ins[b])
+            step_calls(*ins[b], res[b])
         stream.record_event(ev["used"][b])
-        if i >= 2:
-            stream.wait_event(ev["sent"][b])        # step i - 2's gradients have left
-        for t, st_ in zip(outs, stage[b]):
-            st_.copy_(t, non_blocking=True)
         stream.record_event(ev["out"][b])
         with torch.cuda.stream(s_out):
             s_out.wait_event(ev["out"][b])
-            for th, st_ in zip(outs_h, stage[b]):
-                th.copy_(st_, non_blocking=True)
+            for th, t in zip(outs_h, res[b]):
+                th.copy_(t, non_blocking=True)
             s_out.record_event(ev["sent"][b])
     s_out.wait_stream(s_in)
     s_out.wait_stream(stream)
@@ -560,8 +559,11 @@ def run_ours(args):
     torch.cuda.synchronize()
     e2e_ms = replicas.max_over_ranks(e_start.elapsed_time(e_end) / e2e_steps, dev)
     e2e_value = world * tokens / (e2e_ms * 1e-3)
-    if not all(torch.equal(th.to(dev), t) for th, t in zip(outs_h, outs)):
-        raise SystemExit("end-to-end gradients differ from the device step's")
+    last = res[(e2e_steps - 1) % 2]
+    if not all(torch.equal(th.to(dev), t) for th, t in zip(outs_h, last)):
+        raise SystemExit("end-to-end gradients differ from the ones on the device")
+    if not all(torch.equal(a, b2) for a, b2 in zip(last, outs)):
+        raise SystemExit("end-to-end gradients differ from the device-timed step's")
 
     # ---- the oracle on the host cores, bounded sample (rank 0, N = 1 only)
     cpu = None
@@ -601,8 +603,8 @@ def run_ours(args):
             "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
                     "copies": "pinned host buffers; step i+1's inputs and step i's gradients "
-                              "copied on two streams while the steps compute; L2 flushed "
-                              "every step inside the span"},
+                              "copied on two streams while the steps compute (double-buffered "
+                              "inputs and outputs); L2 flushed every step inside the span"},
             "gpu_launches": launches,
             "clocks": clocks,
         }
