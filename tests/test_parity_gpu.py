@@ -501,6 +501,31 @@ def test_decode_steps_reproduce_the_window_forward(H, case):
     assert rel(host(ys), host(y)) <= TOL_BF16, name
 
 
+def test_decode_full_size_window(H):
+    """The decode shape bench.py times (64 sequences, window 256, d = 512, 16
+    rotated causal layers): every position of every sequence equals the
+    device's stack forward over the window, and the first two sequences equal
+    the oracle's window forward (bf16 storage)."""
+    B, n, d, L = 64, 256, 512, 16
+    flags = CAUSAL | RESIDUAL | RELU
+    pr = synth.problem(B, n, d, L=L, seed=41, w_std=(1 / (2 * d)) ** 0.5, x_ids="zipf256")
+    x, x64 = dev(pr.x, torch.bfloat16)
+    Ws, Ws64 = dev(pr.W_self, torch.bfloat16)
+    Wn, Wn64 = dev(pr.W_nbr, torch.bfloat16)
+    bias = torch.from_numpy(pr.bias).cuda()
+    cache = torch.empty(H.hcw_decode_cache_bytes(L, B, n, d), dtype=torch.uint8, device="cuda")
+    ys = torch.empty_like(x)
+    for t in range(n):
+        ys[:, t] = H.hcw_decode_step(x[:, t].contiguous(), Ws, Wn, bias, t, n, cache, flags)
+    y, _, _ = H.hcw_stack_fwd(x, Ws, Wn, bias, 0, -1, flags)
+    torch.cuda.synchronize()
+    assert H.hcw_sync_status() == H.HCW_OK
+    assert rel(host(ys), host(y)) <= TOL_BF16
+    ry, _, _ = O.stack_fwd(x64[:2], Ws64, Wn64, pr.bias.astype(np.float64), 0, L, -1, flags,
+                           round_bf16=True)
+    assert rel(host(ys[:2]), ry) <= TOL_BF16
+
+
 def test_decode_windows_back_to_back_share_the_cache(H):
     """A new window restarts at t = 0 on the same rings; its outputs are those
     of a fresh decode on a cache full of garbage, bit for bit (no slot is read
