@@ -282,9 +282,13 @@ size_t hcw_stack_bwd_weight_workspace_bytes(int B, int n, int d, int dtype, unsi
  *   gradient needs more scratch than that (hcw_layer_bwd_weight_workspace_bytes
  *   > 32 MiB) are rejected with HCW_ERR_WORKSPACE before anything runs.
  *   Allocates nothing: no cudaMalloc, cudaFree or allocating library call.
- *   The first call on each device looks up the array's device address
- *   (a one-time set-up per device, with that device current); make that
- *   first call before any stream capture.
+ *   Every call asks the runtime for the array's device address on the
+ *   current device; the first call on a device also loads the library's
+ *   device code there (a one-time set-up per device, with that device
+ *   current): make that first call before any stream capture.  Because the
+ *   address is looked up on every call, a device reset (cudaDeviceReset)
+ *   does not leave a stale address behind.
+ *   dbias, when given, must not overlap x or dz (HCW_ERR_ALIASING).
  *   All calls share the one array: calls whose kernels may overlap on the
  *   GPU (different streams without ordering, or several host threads) race
  *   on it and must be serialised by the caller.  No part of the array needs

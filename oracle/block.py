@@ -152,6 +152,52 @@ def backward(pr, cache, round_bf16=False):
     return gr
 
 
+def relu_margins(pr, round_bf16=True):
+    """Smallest |u| / std(u) over every FFN pre-activation u of the forward:
+    how far the ReLU decisions sit from the kink."""
+    _, cache = forward(pr, round_bf16=round_bf16)
+    worst = np.inf
+    for c in cache["layers"]:
+        u = c["u"]
+        worst = min(worst, float(np.abs(u).min() / max(u.std(), 1e-300)))
+    return worst
+
+
+def with_separated_relu_decisions(pr, round_bf16=True):
+    """A copy of the block problem `pr` whose FFN biases b1 keep every ReLU
+    decision of the forward clear of the kink (test-input construction, not
+    part of the block).
+
+    Two computations of the same forward (here fp64, on the device fp32)
+    differ at rounding level, so a pre-activation within rounding of 0 can be
+    switched on by one and off by the other; both answers are right, but an
+    element-wise comparison of the gradients then fails on one token's row.
+    Layer by layer, in forward order (b1 of layer l moves only what comes after
+    it), this takes the pre-activations v = g W1^T of every hidden unit j over
+    the B n tokens, finds the widest gap between neighbouring sorted values in
+    their middle half, and sets b1[l, j] to minus the gap's midpoint (as an
+    fp32 number): about half the tokens are active, the decisions still depend
+    on the data, and each one sits half a gap (a few per cent of std(u) at
+    these sizes) from 0."""
+    import copy
+    q = copy.copy(pr)
+    b1 = np.array(pr.b1, dtype=np.float64).copy()
+    L, h = b1.shape
+    for l in range(L):
+        q.b1 = b1.copy()
+        _, cache = forward(q, round_bf16=round_bf16)
+        v = (cache["layers"][l]["g"] @ np.asarray(pr.W1[l], dtype=np.float64).T).reshape(-1, h)
+        N = v.shape[0]
+        lo, hi = N // 4, max(N // 4 + 1, (3 * N) // 4)
+        for j in range(h):
+            s = np.sort(v[:, j])
+            gaps = s[lo + 1:hi + 1] - s[lo:hi]
+            k = lo + int(np.argmax(gaps))
+            b1[l, j] = float(np.float32(-(s[k] + s[k + 1]) / 2))
+    q.b1 = b1
+    return q
+
+
 def step(pr, round_bf16=False):
     """(loss, gradients) of one block step."""
     loss, cache = forward(pr, round_bf16=round_bf16)

@@ -1540,12 +1540,14 @@ int hcw_layer_bwd_weight(const void* x, const void* dz, int layer, int dim_overr
     const size_t need = ws_layout(sh.tokens, d, dtype, flags).w_bytes;
     if (sh.tokens > 0 && (ws_bytes < need || (need && !workspace))) return HCW_ERR_WORKSPACE;
     const size_t ab = sh.act_bytes, gb = (size_t)d * d * 4;
+    // the column sums read dz while they write dbias: dbias must not overlap an input
     if (overlaps(dW_self, gb, dW_nbr, gb) || overlaps(dbias, (size_t)d * 4, dW_self, gb) ||
         overlaps(dbias, (size_t)d * 4, dW_nbr, gb) || overlaps(workspace, ws_bytes, x, ab) ||
         overlaps(workspace, ws_bytes, dz, ab) || overlaps(workspace, ws_bytes, dW_self, gb) ||
-        overlaps(workspace, ws_bytes, dW_nbr, gb) || overlaps(dW_self, gb, x, ab) ||
-        overlaps(dW_nbr, gb, x, ab) || overlaps(dW_self, gb, dz, ab) ||
-        overlaps(dW_nbr, gb, dz, ab))
+        overlaps(workspace, ws_bytes, dW_nbr, gb) || overlaps(workspace, ws_bytes, dbias, (size_t)d * 4) ||
+        overlaps(dW_self, gb, x, ab) || overlaps(dW_nbr, gb, x, ab) ||
+        overlaps(dW_self, gb, dz, ab) || overlaps(dW_nbr, gb, dz, ab) ||
+        overlaps(dbias, (size_t)d * 4, x, ab) || overlaps(dbias, (size_t)d * 4, dz, ab))
         return HCW_ERR_ALIASING;
     return layer_dw_impl(sh, dtype, x, dz, flags, dW_self, dW_nbr, dbias,
                          static_cast<uint8_t*>(workspace), (cudaStream_t)stream);
@@ -1792,23 +1794,15 @@ static constexpr size_t kNoAllocScratchBytes = (size_t)32 << 20;   // 32 MiB
 static __device__ __align__(256) unsigned char hcw_noalloc_scratch[kNoAllocScratchBytes];
 
 namespace {
-std::mutex g_noalloc_mu;
-void* g_noalloc_ptr[1024];   // device address of the array, per device ordinal
-
 // The host-side name of the array is a stand-in, not a device address: ask
-// the runtime for the address on the current device (once per device).
+// the runtime for the address on the current device.  The first call on a
+// device loads the module there (its set-up); later calls are a lookup.  The
+// address is asked for on every call rather than kept, so that a context
+// torn down and made again (cudaDeviceReset) never leaves a stale address.
 int noalloc_scratch(void** out) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return HCW_ERR_CUDA;
-    if (dev < 0 || dev >= 1024) return HCW_ERR_UNSUPPORTED;
-    std::lock_guard<std::mutex> lock(g_noalloc_mu);
-    if (!g_noalloc_ptr[dev]) {
-        void* p = nullptr;
-        if (cudaGetSymbolAddress(&p, hcw_noalloc_scratch) != cudaSuccess || !p)
-            return HCW_ERR_CUDA;
-        g_noalloc_ptr[dev] = p;
-    }
-    *out = g_noalloc_ptr[dev];
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, hcw_noalloc_scratch) != cudaSuccess || !p) return HCW_ERR_CUDA;
+    *out = p;
     return HCW_OK;
 }
 }  // namespace
@@ -1821,19 +1815,21 @@ int hcw_layer_bwd_weight_noalloc(const void* x, const void* dz, int layer, int d
     Shape sh;
     int rc = check_shape(layer, dim_override, B, n, d, dtype, flags, &sh);
     if (rc) return rc;
+    // the fixed scratch must hold what the workspace would: larger sizes are
+    // rejected first, before any pointer is looked at
+    if (ws_layout(sh.tokens, d, dtype, flags).w_bytes > kNoAllocScratchBytes)
+        return HCW_ERR_WORKSPACE;
     if (!dW_self || !dW_nbr) return HCW_ERR_INVALID_ARG;
     const void* ptrs[] = {x, dz, dW_self, dW_nbr, dbias};
     for (const void* q : ptrs)
         if (q && !aligned16(q)) return HCW_ERR_ALIGNMENT;
     if (sh.tokens > 0 && (!x || !dz)) return HCW_ERR_INVALID_ARG;
-    // the fixed scratch must hold what the workspace would: reject larger sizes
-    if (ws_layout(sh.tokens, d, dtype, flags).w_bytes > kNoAllocScratchBytes)
-        return HCW_ERR_WORKSPACE;
     const size_t ab = sh.act_bytes, gb = (size_t)d * d * 4;
     if (overlaps(dW_self, gb, dW_nbr, gb) || overlaps(dbias, (size_t)d * 4, dW_self, gb) ||
         overlaps(dbias, (size_t)d * 4, dW_nbr, gb) || overlaps(dW_self, gb, x, ab) ||
         overlaps(dW_nbr, gb, x, ab) || overlaps(dW_self, gb, dz, ab) ||
-        overlaps(dW_nbr, gb, dz, ab))
+        overlaps(dW_nbr, gb, dz, ab) || overlaps(dbias, (size_t)d * 4, x, ab) ||
+        overlaps(dbias, (size_t)d * 4, dz, ab))
         return HCW_ERR_ALIASING;
     void* scratch = nullptr;
     rc = noalloc_scratch(&scratch);

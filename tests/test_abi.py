@@ -131,6 +131,32 @@ def test_backward_validation_codes(hcw):
     assert call(d=0) == hcw.HCW_ERR_INVALID_ARG
 
 
+def test_weight_gradient_rejects_dbias_over_its_inputs(hcw):
+    """The column sums read dz while they write dbias: both weight-gradient
+    entry points (with a workspace, and the one without) refuse a dbias that
+    overlaps x or dz, before anything launches."""
+    P = ctypes.c_void_p
+    L = hcw.lib()
+    B, n, d = 4, 16, 64
+    act = B * n * d * 2
+    X, DZ, GS, GN, GB, W = (0x10000000 * k for k in range(1, 7))
+    need = hcw.hcw_layer_bwd_weight_workspace_bytes(B, n, d, hcw.HCW_BF16, 0)
+
+    def ws(gb):
+        return L.hcw_layer_bwd_weight(P(X), P(DZ), 0, -1, B, n, d, hcw.HCW_BF16, 0, P(GS), P(GN),
+                                      P(gb), P(W), need, None)
+
+    def noalloc(gb):
+        return L.hcw_layer_bwd_weight_noalloc(P(X), P(DZ), 0, -1, B, n, d, hcw.HCW_BF16, 0,
+                                              P(GS), P(GN), P(gb), None)
+
+    for f in (ws, noalloc):
+        assert f(X + act - 256) == hcw.HCW_ERR_ALIASING      # inside x
+        assert f(DZ) == hcw.HCW_ERR_ALIASING                 # on dz
+        assert f(GS + 64) == hcw.HCW_ERR_ALIASING            # inside dW_self
+    assert ws(W + 16) == hcw.HCW_ERR_ALIASING                # inside the workspace
+
+
 def test_workspace_sizes_f32(hcw):
     a = hcw.hcw_workspace_bytes(64, 256, 512, hcw.HCW_F32, 0)
     b = hcw.hcw_workspace_bytes(64, 256, 512, hcw.HCW_F32, hcw.HCW_ACT_RELU)

@@ -11,23 +11,29 @@ from paper_2609_18145_gb300 import synth
 pytestmark = pytest.mark.gpu
 
 BF16 = {"E", "P", "W_self", "W_nbr", "W1", "W2", "Wh"}
-# Tolerance.  Both sides round the same tensors to bf16, but they compute in
-# fp32 (device) and fp64 (oracle): once their values differ by more than the
-# distance to a rounding boundary they round differently, and each of the 2L
-# sublayers adds up to half an ulp (2^-9 relative) of independent difference to
-# the gradient flowing down from the head, like a random walk: about
-# 2^-9 sqrt(2L) with a safety factor of 4 gives 1.1e-2 sqrt(L).  Measured at
-# n = 256, d = 512, h = 1024: relative Frobenius errors 1e-4 (head) to 3.2e-2
-# (E, P) at L = 16 and up to 1.3e-2 at L = 4.  ReLU decisions on fp32 and
-# fp64 pre-activations within rounding of 0 can differ too and move one row.
-# So each gradient tensor is held to a relative Frobenius error of
-# max(2e-2, 1.25e-2 sqrt(L)).  A single differing ReLU decision moves one
-# token's whole contribution to one row of dW1 (7.6 % of max |dW1| measured
-# with 64 tokens), so the relative max error only guards against gross
-# errors (0.25).
 TOL_LOSS = 5e-3      # relative, on the mean loss
+# Element-wise tolerance of the small cases: per gradient tensor,
+# max |device - oracle| / max |oracle| <= 2e-2, the bf16 tolerance of the
+# mixing path.  Both sides round the same tensors to bf16 but compute in fp32
+# (device) and fp64 (oracle); the small cases take problems whose ReLU
+# decisions sit a few per cent of std(u) away from the kink
+# (oracle.block.with_separated_relu_decisions), so both sides take the same
+# decisions and what is left is rounding.
+TOL_ELEM = 2e-2
+MIN_MARGIN = 1e-2    # |u| / std(u) the small cases keep from the kink
 
 
+# The full-size case (L = 16, 16,384 tokens) cannot keep its 2.6e8 ReLU
+# decisions clear of the kink, so it is held to norms.  Both sides round the
+# same tensors to bf16, but once their values differ by more than the distance
+# to a rounding boundary they round differently, and each of the 2L sublayers
+# adds up to half an ulp (2^-9 relative) of independent difference to the
+# gradient flowing down from the head, like a random walk: about
+# 2^-9 sqrt(2L) with a safety factor of 4 gives 1.1e-2 sqrt(L).  A ReLU
+# decision on fp32 and fp64 pre-activations within rounding of 0 can differ
+# too and move one token's row.  So each gradient tensor is held to a relative
+# Frobenius error of max(2e-2, 1.25e-2 sqrt(L)), and the relative max error
+# only guards against gross errors (0.25).
 def tol_grad(L):
     return max(2e-2, 1.25e-2 * L ** 0.5)
 
@@ -71,11 +77,17 @@ def relf(a, b):
 
 
 def check_grads(got, ref, L):
+    """Norm-wise check of the full-size case (see tol_grad)."""
     t = tol_grad(L)
     for f in OB_FIELDS:
         a = got[f]
         assert relf(a, ref[f]) <= t, (f, relf(a, ref[f]), rel(a, ref[f]))
         assert rel(a, ref[f]) <= 0.25, (f, relf(a, ref[f]), rel(a, ref[f]))
+
+
+def check_grads_elementwise(got, ref):
+    for f in OB_FIELDS:
+        assert rel(got[f], ref[f]) <= TOL_ELEM, (f, rel(got[f], ref[f]), relf(got[f], ref[f]))
 
 
 CASES = [
@@ -88,15 +100,22 @@ CASES = [
 
 @pytest.mark.parametrize("case", CASES, ids=lambda c: "B%d_n%d_d%d_h%d_V%d_L%d" % c)
 def test_block_step_matches_the_oracle(H, case):
+    """Loss and every gradient tensor element by element against the oracle's
+    bf16-storage mode, on problems whose ReLU decisions are clear of the
+    kink."""
     B, n, d, h, V, L = case
     pr = synth.block_problem(B, n, d, h, V, L, seed=7)
     ids, params, exact = device_problem(pr)
+    q = OB.with_separated_relu_decisions(as_problem(pr, exact), round_bf16=True)
+    assert OB.relu_margins(q) >= MIN_MARGIN
+    params["b1"] = torch.from_numpy(np.asarray(q.b1, dtype=np.float32)).cuda().contiguous()
     loss, grads = H.hcw_block_step(ids, params)
     torch.cuda.synchronize()
     assert H.hcw_sync_status() == H.HCW_OK
-    ref_loss, ref = OB.step(as_problem(pr, exact), round_bf16=True)
+    ref_loss, ref = OB.step(q, round_bf16=True)
     assert abs(float(loss.item()) - ref_loss) <= TOL_LOSS * abs(ref_loss)
-    check_grads({f: g.cpu().numpy().astype(np.float64) for f, g in grads.items()}, ref, L)
+    check_grads_elementwise({f: g.cpu().numpy().astype(np.float64) for f, g in grads.items()},
+                            ref)
 
 
 def test_an_id_outside_the_vocabulary_is_reported(H):

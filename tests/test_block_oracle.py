@@ -100,3 +100,23 @@ def test_bf16_storage_mode_stays_close_to_fp64():
     for f in FIELDS:
         scale = np.abs(g64[f]).max()
         assert np.abs(g16[f] - g64[f]).max() <= 5e-2 * scale + 1e-12, f
+
+
+def test_separated_relu_decisions_change_only_b1_and_keep_a_margin():
+    """The test-input construction behind the element-wise GPU parity: only
+    the FFN biases move, every pre-activation ends up at least 1 % of its
+    spread from the kink (it starts far closer), and the decisions still
+    depend on the data (each hidden unit is on for some tokens and off for
+    others)."""
+    pr = synth.block_problem(2, 16, 64, 128, 11, 3, seed=7)
+    q = OB.with_separated_relu_decisions(pr, round_bf16=True)
+    for f in ("E", "P", "ln1_g", "ln1_b", "W_self", "W_nbr", "ln2_g", "ln2_b", "W1", "W2", "b2",
+              "lnf_g", "lnf_b", "Wh", "bh"):
+        assert np.array_equal(np.asarray(getattr(q, f)), np.asarray(getattr(pr, f))), f
+    assert OB.relu_margins(pr) < 1e-3
+    assert OB.relu_margins(q) >= 1e-2
+    assert np.array_equal(np.asarray(q.b1, dtype=np.float32).astype(np.float64), q.b1)
+    _, cache = OB.forward(q, round_bf16=True)
+    for c in cache["layers"]:
+        on = (c["u"] > 0).reshape(-1, c["u"].shape[-1]).mean(axis=0)
+        assert on.min() > 0.1 and on.max() < 0.9
