@@ -392,10 +392,11 @@ int fwd_bf16(const Shape& sh, const void* x, const void* Ws, const void* Wn, con
 // group and 128-token chunk.
 size_t stack_counter_bytes(long long tokens, int L) {
     const int layers = L < kMaxStackLayers ? L : kMaxStackLayers;
-    // per (layer, 128-token chunk) completion counters, the unit counter, and
-    // the chunk counters of the top layer's dz written by the launch itself
+    // per (layer, 128-token chunk) completion counters, the unit counter, the
+    // chunk counters of the top layer's dz written by the launch itself, and
+    // (input gradient) per (layer, chunk) counters of the output gradient g
     const size_t chunks = (size_t)((tokens + 127) / 128);
-    return align256(((size_t)layers * chunks + 1 + chunks) * sizeof(int) + 16);
+    return align256((2 * (size_t)layers * chunks + 1 + chunks) * sizeof(int) + 16);
 }
 
 // Whether a stacked forward / input-gradient launch runs on pairs of SMs
@@ -947,7 +948,12 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
             T.top_dz = static_cast<__nv_bfloat16*>(dz(L - 1));
             T.in_counters = T.sched + 1;
         }
-        if (cudaMemsetAsync(counters, 0, ((size_t)cnt * n_chunks + 1 + n_chunks) * sizeof(int),
+        // g apart from dz: with the ReLU and the residual, the kernel publishes
+        // each patch's dz before it stores g
+        if (keep_g) T.g_counters = T.sched + 1 + n_chunks;
+        if (cudaMemsetAsync(counters, 0,
+                            ((size_t)(keep_g ? 2 : 1) * cnt * n_chunks + 1 + n_chunks) *
+                                sizeof(int),
                             st) != cudaSuccess)
             return HCW_ERR_CUDA;
         rc = launch_rows(MODE_DX, BN, T, cnt, pair, st);

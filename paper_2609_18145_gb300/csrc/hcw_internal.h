@@ -75,9 +75,10 @@ constexpr int kMaxStackLayers = 16;   // layers per stacked-forward launch
 
 // maps[l][0..5] = tmA, tmB0, tmB1, tmE0, tmE1, tmE2 of layer l, as documented
 // at hcw_tc_kernel in hcw_tc.cu.
+constexpr int kTcMaps = 6;
 template <int NL>
 struct TcLaunch {
-    CUtensorMap maps[NL][6];
+    CUtensorMap maps[NL][kTcMaps];
     TcLayer layer[NL];
     TcParams p;
     int n_layers;
@@ -95,6 +96,12 @@ struct TcLaunch {
     const uint32_t* top_mask;
     __nv_bfloat16* top_dz;
     int* in_counters;
+    // Stacked input gradient with ReLU and residual: completion counters
+    // [n_layers][n_chunks] of each layer's output gradient g (the residual term
+    // of the layer below), counted apart from dz so that dz -- the operand the
+    // next layer's MMAs wait for -- is published before g is stored.  Null:
+    // g is dz (or absent) and the counters above cover it.
+    int* g_counters;
 };
 
 // Launch one tensor-core pass (one layer).

@@ -349,6 +349,15 @@ __device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
                  : "memory");
 }
 
+// Arrive on a peer CTA's mbarrier to hand back tensor memory whose reads have
+// completed (tcgen05.wait::ld, then tcgen05.fence::before_thread_sync):
+// nothing written to memory is published, so the release is at CTA scope,
+// which does not wait for this thread's outstanding global stores the way a
+// cluster-scope release does.
+__device__ __forceinline__ void mbar_arrive_remote_tmem(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
 // 5-D tile load into this CTA's shared memory that completes its bytes on an
 // mbarrier of either CTA of the pair (its shared::cluster address).
 __device__ __forceinline__ void tma_load_5d_pair(void* dst, const CUtensorMap* m,

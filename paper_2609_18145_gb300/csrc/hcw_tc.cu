@@ -94,6 +94,10 @@ struct __align__(8) Barriers {
     int unit_q[kUnitQ];   // dynamic scheduling: unit claimed for ordinal o, in slot o % kUnitQ
     int q_pub;            // highest ordinal published in unit_q
     int q_read;           // slot reads so far (the MMA thread and every epilogue warp)
+    // stacked row launches: epilogue warps whose stores of the unit in slot o %
+    // kUnitQ have completed, per published output (0: the counters' output,
+    // 1: the input gradient's g); the last one publishes the CTA's rows
+    int pub_done[2][kUnitQ];
 };
 
 // Stages of the pair variant of the row kernels: this CTA's A and half of B.
@@ -274,6 +278,60 @@ __device__ __forceinline__ void fence_acq_rel_gpu() {
     asm volatile("fence.acq_rel.gpu;" ::: "memory");
 }
 
+__device__ __forceinline__ void red_relaxed_gpu_add(int* p, int v) {
+    asm volatile("red.relaxed.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Two fp32 values in one 64-bit register pair, and the packed fp32 arithmetic
+// of the FP32 pipe (each instruction rounds both lanes like its scalar form).
+__device__ __forceinline__ uint64_t f32x2_pack(float a, float b) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+    return r;
+}
+__device__ __forceinline__ float2 f32x2_unpack(uint64_t r) {
+    float a, b;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(r));
+    return make_float2(a, b);
+}
+__device__ __forceinline__ uint64_t f32x2_add(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ uint64_t f32x2_mul(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ uint64_t f32x2_fma(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+__device__ __forceinline__ float mul_sat_f32(float a, float b) {
+    float r;
+    asm("mul.rn.sat.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
+    return r;
+}
+// (2^100, 2^100) as a packed pair
+constexpr uint64_t kF32x2Pow100 = 0x7180000071800000ull;
+// bf16 pair -> fp32 pair (exact: the bf16 bits are the high half of each float)
+__device__ __forceinline__ uint64_t bf16x2_to_f32x2(uint32_t w) {
+    return f32x2_pack(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
+}
+
+// Adds v to the shared int *p with acquire-release semantics at CTA scope and
+// returns the previous value.
+__device__ __forceinline__ int atom_add_acq_rel_cta_shared(int* p, int v) {
+    int old;
+    asm volatile("atom.acq_rel.cta.shared::cta.add.s32 %0, [%1], %2;"
+                 : "=r"(old)
+                 : "r"(smem_u32(p)), "r"(v)
+                 : "memory");
+    return old;
+}
+
 // Bounded wait until both counters reach their targets (n of them: 1 or 2),
 // with acquire semantics.  The first look reads both at once (relaxed) and,
 // when both are complete, acquires with one fence; otherwise each is waited
@@ -372,7 +430,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
 
     if (threadIdx.x == 0) {
         for (int l = 0; l < L.n_layers && l < NL; ++l)
-            for (int i = 0; i < 6; ++i) tma_prefetch_desc(&L.maps[l][i]);
+            for (int i = 0; i < kTcMaps; ++i) tma_prefetch_desc(&L.maps[l][i]);
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&bars->full[s], 1);
             // DW: the MMA commit and the helper warps (which read the dz tiles for
@@ -389,6 +447,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
         bars->dep_unit = -1;
         bars->q_pub = -1;
         bars->q_read = 0;
+        for (int i = 0; i < 2 * kUnitQ; ++i) (&bars->pub_done[0][0])[i] = 0;
         fence_mbar_init();
     }
     if (warp == 1) {
@@ -804,7 +863,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
             __syncwarp();
             if (lane == 0) {
                 if (PAIR)
-                    mbar_arrive_remote(mapa_shared(&bars->tempty[acc], 0));   // the leader's
+                    mbar_arrive_remote_tmem(mapa_shared(&bars->tempty[acc], 0));   // the leader's
                 else
                     mbar_arrive(&bars->tempty[acc]);
             }
@@ -1005,6 +1064,10 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                 const CUtensorMap* mE1 = &L.maps[l][4];
                 const CUtensorMap* mE2 = &L.maps[l][5];
                 const int wpr = p.d >> 5;
+                // the 128-token chunk that holds the patch's rows (32 compressed rows
+                // lie in one chunk for every link distance)
+                const int tok0 = ((qw >> ly.s) << (ly.s + 1)) + (r.beta << ly.s) + (qw & (ly.k - 1));
+                const int chunk = tok0 >> 7;
                 // every earlier store has finished reading the buffer: refill it
                 if (lane == 0) bulk_wait_read<0>();
                 __syncwarp();
@@ -1012,9 +1075,26 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     alive = false;
                     break;
                 }
-                if (has_res && lane == 0) {
-                    mbar_arrive_expect_tx(&bars->epi_load[e], 32 * RB);
-                    tma_load_4d(buf, mE0, &bars->epi_load[e], col0, lo_w, r.beta, hi_w);
+                if (has_res) {
+                    int okg = 1;
+                    if (lane == 0) {
+                        // stacked input gradient: the residual term g of these rows is
+                        // stored by the layer above after its dz; wait until the chunk's g
+                        // is complete (the dz the MMAs read was checked by the producer)
+                        if (MODE == MODE_DX && STACKED && L.g_counters != nullptr && l > 0) {
+                            okg = wait_counter(L.g_counters + (size_t)(l - 1) * L.n_chunks + chunk,
+                                               min(128, L.tokens - (chunk << 7)) * p.d, abort, tmo);
+                            if (okg) fence_proxy_async_global();
+                        }
+                        if (okg) {
+                            mbar_arrive_expect_tx(&bars->epi_load[e], 32 * RB);
+                            tma_load_4d(buf, mE0, &bars->epi_load[e], col0, lo_w, r.beta, hi_w);
+                        }
+                    }
+                    if (__shfl_sync(0xffffffffu, okg, 0) == 0) {
+                        alive = false;
+                        break;
+                    }
                 }
                 uint32_t mp[SUB];
 #pragma unroll
@@ -1067,76 +1147,80 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                 }
                 const bool write_out = fwd || ly.out;
                 uint32_t gw[SUB][16];
+                uint32_t mbits[SUB];
 #pragma unroll
                 for (int h = 0; h < SUB; ++h) {
                     uint32_t raw[32];
                     load_acc(h * 32, raw);
                     if (h == SUB - 1) release_acc();
-                    float v[32];
+                    // The arithmetic runs on the FP32 pipe, two columns per instruction
+                    // where it can (f32x2): the epilogue of a chained unit sits on the
+                    // layer chain, and half-rate integer work (compares, selects, bit
+                    // ors) made it issue-bound.  Eight columns at a time: column pairs
+                    // q = 4m .. 4m + 3.
+                    const bool relu = fwd && (p.flags & 4u);
+                    uint64_t lo = f32x2_pack(0x1p23f, 0.f), hi = lo;   // mask-word halves
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(raw[i]);
-                    if (fwd) {
-                        const float4* b4 = reinterpret_cast<const float4*>(wbias + h * 32);
-#pragma unroll
-                        for (int i = 0; i < 8; ++i) {
-                            const float4 bb = b4[i];
-                            v[4 * i] += bb.x;
-                            v[4 * i + 1] += bb.y;
-                            v[4 * i + 2] += bb.z;
-                            v[4 * i + 3] += bb.w;
-                        }
-                        if (ly.mout) {
-                            uint32_t bits = 0;
-#pragma unroll
-                            for (int i = 0; i < 32; ++i) bits |= (v[i] > 0.f ? 1u : 0u) << i;
-                            if (tok_row >= 0)
-                                ly.mout[(size_t)tok_row * wpr + (col0 >> 5) + h] = bits;
-                        }
-                        if (p.flags & 4u) {
-#pragma unroll
-                            for (int i = 0; i < 32; ++i) v[i] = v[i] > 0.f ? v[i] : 0.f;
-                        }
-                    }
-                    if (has_res) {
-#pragma unroll
-                        for (int m = 0; m < 4; ++m) {
+                    for (int m = 0; m < 4; ++m) {
+                        uint32_t rw[4] = {0u, 0u, 0u, 0u};   // residual (bf16 pairs), or +0
+                        if (has_res) {
                             const uint4 q4 = *patch_piece<RB>(buf, lane, 4 * h + m);
-                            const uint32_t rw[4] = {q4.x, q4.y, q4.z, q4.w};
+                            rw[0] = q4.x;
+                            rw[1] = q4.y;
+                            rw[2] = q4.z;
+                            rw[3] = q4.w;
+                        }
+                        float4 bb[2] = {make_float4(0.f, 0.f, 0.f, 0.f), make_float4(0.f, 0.f, 0.f, 0.f)};
+                        if (fwd) {
+                            const float4* b4 = reinterpret_cast<const float4*>(wbias + h * 32 + 8 * m);
+                            bb[0] = b4[0];
+                            bb[1] = b4[1];
+                        }
 #pragma unroll
-                            for (int i = 0; i < 4; ++i) {
-                                const float2 f = unpack_bf16x2(rw[i]);
-                                v[8 * m + 2 * i] += f.x;
-                                v[8 * m + 2 * i + 1] += f.y;
+                        for (int i = 0; i < 4; ++i) {
+                            const int q = 4 * m + i;
+                            uint64_t v2 = f32x2_pack(__uint_as_float(raw[2 * q]),
+                                                     __uint_as_float(raw[2 * q + 1]));
+                            if (fwd)
+                                v2 = f32x2_add(v2, i & 1 ? f32x2_pack(bb[i >> 1].z, bb[i >> 1].w)
+                                                         : f32x2_pack(bb[i >> 1].x, bb[i >> 1].y));
+                            const uint64_t r2 = bf16x2_to_f32x2(rw[i]);
+                            if (relu) {
+                                // b = [z > 0] exactly as 1.0 / 0.0: z * 2^100 * 2^100 saturated
+                                // to [0, 1] (every positive float, denormals included,
+                                // reaches at least 2^51 before the clamp; zero, negative and
+                                // NaN go to 0).  y = fma(z, b, x) is relu(z) + x with one
+                                // rounding; with x = +0 a negative z gives (-0) + (+0) = +0.
+                                const float2 t = f32x2_unpack(f32x2_mul(v2, kF32x2Pow100));
+                                const uint64_t b2 =
+                                    f32x2_pack(mul_sat_f32(t.x, 0x1p100f), mul_sat_f32(t.y, 0x1p100f));
+                                // the mask word: sum of b_c 2^c, exact in fp32, as two 16-bit
+                                // halves offset by 2^23 (the integer is the low mantissa)
+                                const uint64_t w2 = f32x2_pack((float)(1u << ((2 * q) & 15)),
+                                                               (float)(1u << ((2 * q + 1) & 15)));
+                                if (q < 8)
+                                    lo = f32x2_fma(b2, w2, lo);
+                                else
+                                    hi = f32x2_fma(b2, w2, hi);
+                                v2 = f32x2_fma(v2, b2, r2);
+                            } else if (has_res) {
+                                v2 = f32x2_add(v2, r2);
                             }
+                            const float2 t = f32x2_unpack(v2);
+                            gw[h][q] = pack_bf16x2(t.x, t.y);
                         }
                     }
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) gw[h][i] = pack_bf16x2(v[2 * i], v[2 * i + 1]);
-                    // the lane's own row, the pieces just read: safe to overwrite now
-                    if (write_out) {
-#pragma unroll
-                        for (int m = 0; m < 4; ++m)
-                            *patch_piece<RB>(buf, lane, 4 * h + m) =
-                                make_uint4(gw[h][4 * m], gw[h][4 * m + 1], gw[h][4 * m + 2],
-                                           gw[h][4 * m + 3]);
+                    if (relu) {
+                        const float2 l2 = f32x2_unpack(lo), h2 = f32x2_unpack(hi);
+                        mbits[h] = __byte_perm(__float_as_uint(l2.x + l2.y),
+                                               __float_as_uint(h2.x + h2.y), 0x5410);
+                    } else {
+                        mbits[h] = 0u;
                     }
-                }
-                // the patch: y (FWD) or dx (DX), written over the residual rows
-                if (write_out) {
-                    publish();
-                    if (lane == 0 && inside) {
-                        tma_store_4d(mE1, buf, col0, lo_w, r.beta, hi_w);
-                        bulk_commit();
-                    }
-                }
-                if (has_mprev) {
-                    // fused ReLU gradient of the layer below: dz = dx * mask
-                    if (write_out) {
-                        if (lane == 0) bulk_wait_read<0>();
-                        __syncwarp();
-                    }
-#pragma unroll
-                    for (int h = 0; h < SUB; ++h) {
+                    // the lane's own row, the pieces just read: safe to overwrite now.
+                    // With the ReLU gradient of the layer below, dz = dx * mask goes
+                    // first; otherwise y (FWD) or dx (DX).
+                    if (has_mprev) {
                         const uint32_t mw = mp[h];
 #pragma unroll
                         for (int m = 0; m < 4; ++m) {
@@ -1151,26 +1235,98 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                             *patch_piece<RB>(buf, lane, 4 * h + m) =
                                 make_uint4(w4[0], w4[1], w4[2], w4[3]);
                         }
+                    } else if (write_out) {
+#pragma unroll
+                        for (int m = 0; m < 4; ++m)
+                            *patch_piece<RB>(buf, lane, 4 * h + m) =
+                                make_uint4(gw[h][4 * m], gw[h][4 * m + 1], gw[h][4 * m + 2],
+                                           gw[h][4 * m + 3]);
                     }
+                }
+                // Publish the CTA's rows of the unit to the next layer's units once
+                // every patch's stores have landed.  Each warp waits for its own
+                // stores and counts itself in a shared counter (release at CTA
+                // scope); the last of the unit's warps issues one release at GPU
+                // scope and adds the elements of the CTA's rows to the counters of
+                // the (at most two) 128-token chunks they lie in.  One release per
+                // CTA and unit instead of one per warp: each costs about a
+                // microsecond on the layer chain.
+                const bool signal = STACKED && l + 1 < L.n_layers;
+                auto count = [&](int* ctr, int kind) {
+                    if (lane == 0) {
+                        if (inside) bulk_wait<0>();
+                        fence_proxy_async_global();
+                        int* done = &bars->pub_done[kind][ordinal % kUnitQ];
+                        if (atom_add_acq_rel_cta_shared(done, 1) == EW - 1) {
+                            *done = 0;   // next used by ordinal + kUnitQ, after this unit
+                            const int cols = BN;
+                            int c0 = -1, n0 = 0, c1 = -1, n1 = 0;
+                            for (int qd = 0; qd < 4; ++qd) {
+                                const int q = r.t * kBlockM + 32 * qd;
+                                if (q >= p.Mh) break;
+                                const int c = (((q >> ly.s) << (ly.s + 1)) + (r.beta << ly.s) +
+                                               (q & (ly.k - 1))) >> 7;
+                                const int n = min(32, p.Mh - q) * cols;
+                                if (c0 < 0 || c == c0) {
+                                    c0 = c;
+                                    n0 += n;
+                                } else {
+                                    c1 = c;
+                                    n1 += n;
+                                }
+                            }
+                            fence_acq_rel_gpu();
+                            int* base = ctr + (size_t)l * L.n_chunks;
+                            if (n0) red_relaxed_gpu_add(base + c0, n0);
+                            if (n1) red_relaxed_gpu_add(base + c1, n1);
+                        }
+                    }
+                    __syncwarp();
+                };
+                if (has_mprev) {
+                    // the dz patch (the next layer's MMA operand) first
                     publish();
                     if (lane == 0 && inside) {
                         tma_store_4d(mE2, buf, col0, lo_w, r.beta, hi_w);
                         bulk_commit();
                     }
-                }
-                if (STACKED && alive && l + 1 < L.n_layers) {
-                    // publish the finished patch to the next layer's units: its stores
-                    // have landed, then count its elements in the chunk it lies in
-                    if (lane == 0 && inside) {
-                        bulk_wait<0>();
-                        fence_proxy_async_global();
-                        const int rows = min(32, p.Mh - qw);
-                        const int tok0 = ((qw >> ly.s) << (ly.s + 1)) + (r.beta << ly.s) +
-                                         (qw & (ly.k - 1));
-                        red_release_gpu_add(L.counters + (size_t)l * L.n_chunks + (tok0 >> 7),
-                                            rows * WCOLS);
+                    const bool split_g = write_out && L.g_counters != nullptr;
+                    if (signal && (!write_out || split_g)) count(L.counters, 0);
+                    if (write_out) {
+                        // then the output gradient g (the next layer's residual term)
+                        if (lane == 0) bulk_wait_read<0>();
+                        __syncwarp();
+#pragma unroll
+                        for (int h = 0; h < SUB; ++h)
+#pragma unroll
+                            for (int m = 0; m < 4; ++m)
+                                *patch_piece<RB>(buf, lane, 4 * h + m) =
+                                    make_uint4(gw[h][4 * m], gw[h][4 * m + 1], gw[h][4 * m + 2],
+                                               gw[h][4 * m + 3]);
+                        publish();
+                        if (lane == 0 && inside) {
+                            tma_store_4d(mE1, buf, col0, lo_w, r.beta, hi_w);
+                            bulk_commit();
+                        }
+                        if (signal) count(split_g ? L.g_counters : L.counters, split_g ? 1 : 0);
                     }
-                    __syncwarp();
+                } else {
+                    // the patch: y (FWD) or dx (DX), written over the residual rows
+                    if (write_out) {
+                        publish();
+                        if (lane == 0 && inside) {
+                            tma_store_4d(mE1, buf, col0, lo_w, r.beta, hi_w);
+                            bulk_commit();
+                        }
+                    }
+                    if (signal) count(L.counters, 0);
+                }
+                // FWD: the ReLU mask words, read only by the input gradient (a later
+                // launch), after the signal so that they stay off the layer chain
+                if (fwd && ly.mout && tok_row >= 0) {
+#pragma unroll
+                    for (int h = 0; h < SUB; ++h)
+                        ly.mout[(size_t)tok_row * wpr + (col0 >> 5) + h] = mbits[h];
                 }
             } else {
                 const WUnit& w = wu;
@@ -1523,7 +1679,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     if (which == 1 && c == WCOLS / 32 - 1) {
                         tc_fence_before();
                         __syncwarp();
-                        if (lane == 0) mbar_arrive_remote(tempty_leader);
+                        if (lane == 0) mbar_arrive_remote_tmem(tempty_leader);
                     }
                     if (row < p.d) {
                         float4* dst = reinterpret_cast<float4*>(
