@@ -353,11 +353,21 @@ def run_ours(args):
                      device=dev)
     fws = torch.empty(max(1, H.hcw_stack_fwd_workspace_bytes(B, n, d, H.HCW_BF16, flags, L)),
                       dtype=torch.uint8, device=dev)
+    tws = torch.empty(max(1, H.hcw_stack_train_step_workspace_bytes(B, n, d, H.HCW_BF16, flags,
+                                                                    L)),
+                      dtype=torch.uint8, device=dev)
     flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     stream = torch.cuda.current_stream()
 
     def step_calls(xin, dyin, outs=None):
         oWs, oWn, ob = outs if outs is not None else (gWs, gWn, gb)
+        if dims is None:
+            # one training-step call: the forward and the input gradient in one
+            # launch where the shape allows it, then the weight gradients
+            H.hcw_stack_train_step(xin, Ws, Wn, bias, dyin, 0, -1, flags, y=y, acts=acts,
+                                   masks=masks, dx=dx, dW_self=oWs, dW_nbr=oWn, dbias=ob,
+                                   workspace=tws)
+            return
         H.hcw_stack_fwd(xin, Ws, Wn, bias, 0, -1, flags, y=y, acts=acts, masks=masks,
                         workspace=fws, dims=dims)
         H.hcw_stack_bwd(xin, acts, masks, dyin, Ws, Wn, 0, -1, flags, dx=dx, dW_self=oWs,
@@ -462,7 +472,30 @@ def run_ours(args):
                                                       acts=acts, masks=masks, workspace=fws),
                             reps)
     family = H.hcw_stack_kernels_used(B, n, d)
-    if dims is None:
+    fused = dims is None and family == H.HCW_STACK_STREAMING and d % 256 == 0 and L <= 16
+    if fused:
+        # the step's two launches: the forward and the input gradient in one
+        # launch (the training step without weight gradients), and the batched
+        # weight gradient (bias off), each timed alone on the same inputs
+        fdx_ms = time_calls(lambda i: H.hcw_stack_train_step(x, Ws, Wn, bias, dy, 0, -1, flags,
+                                                             y=y, acts=acts, masks=masks, dx=dx,
+                                                             want_dw=False, workspace=tws),
+                            reps)
+        dz_step = tws[:L * x.numel() * 2].view(torch.bfloat16).view(L, B, n, d)
+        dw_ms = time_calls(lambda i: H.hcw_stack_bwd_weight(x, acts, dz_step, 0, -1, flags,
+                                                            dW_self=gWs, dW_nbr=gWn,
+                                                            want_dbias=False, workspace=wws),
+                           reps)
+        dwb_ms = time_calls(lambda i: H.hcw_stack_bwd_weight(x, acts, dz_step, 0, -1, flags,
+                                                             dW_self=gWs, dW_nbr=gWn, dbias=gb,
+                                                             workspace=wws), reps)
+        fdx_name = ("hcw_tc_kernel<FDX,256,32> (stacked forward and input gradient in one "
+                    "launch on SM pairs, top dz written by the last forward layer)")
+        dw_name = ("hcw_dwp_kernel<256> (weight and bias gradients on SM pairs, a unit per "
+                   "layer and 256 x 256 output tile)")
+        kernels = {fdx_name: fdx_ms, dw_name: dw_ms}
+        kflops = {fdx_name: 2 * 3.0 * d * d * tokens * L, dw_name: 3.0 * d * d * tokens * L}
+    elif dims is None:
         dx_ms = time_calls(lambda i: H.hcw_stack_bwd_data(masks, dy, Ws, Wn, 0, -1, flags,
                                                           dx=dx, dz=dz_all, workspace=dws), reps)
         dw_ms = time_calls(lambda i: H.hcw_stack_bwd_weight(x, acts, dz_all, 0, -1, flags,

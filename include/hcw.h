@@ -237,6 +237,34 @@ int hcw_stack_bwd_dims(const void* x, const void* acts, const void* masks, const
 size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags, int L);
 
 /*
+ * One training step of a stack: hcw_stack_fwd followed by hcw_stack_bwd
+ * (Sec. 3.1 wiring and Eq. (1) maps forward, the chain rule backward), same
+ * layer schedule (layer0, dim_override) and flags.
+ *   Inputs x [B][n][d], W_self, W_nbr [L][d][d], bias [L][d] (or NULL), dy
+ *   [B][n][d] (the gradient of y).  Outputs y, acts, masks exactly as
+ *   hcw_stack_fwd writes them, dx, dW_self, dW_nbr, dbias (or NULL) exactly as
+ *   hcw_stack_bwd writes them.  All buffers are the caller's; dy must not
+ *   overlap y, acts or masks.
+ *   workspace: at least hcw_stack_train_step_workspace_bytes(...) bytes.
+ *   dW_self = dW_nbr = dbias = NULL: the forward and the input gradient only
+ *   (no weight gradients); dW_self and dW_nbr are given together or not at all.
+ * The results equal those of the two separate calls bit for bit.  bf16 on
+ * pairs of SMs with up to 16 layers and no shift layers: the forward and the
+ * input gradient run as one persistent launch (the input gradient of a
+ * 512-token window starts as soon as its forward is done, and the last
+ * forward layer writes the top layer's dz = dy * act'(z) itself), then one
+ * launch computes the weight and bias gradients.  Other shapes run the two
+ * calls.  Errors as for hcw_stack_fwd and hcw_stack_bwd.
+ */
+int hcw_stack_train_step(const void* x, const void* W_self, const void* W_nbr, const float* bias,
+                         const void* dy, int layer0, int L, int dim_override, int B, int n, int d,
+                         int dtype, unsigned flags, void* y, void* acts, void* masks, void* dx,
+                         float* dW_self, float* dW_nbr, float* dbias, void* workspace,
+                         size_t ws_bytes, void* stream);
+size_t hcw_stack_train_step_workspace_bytes(int B, int n, int d, int dtype, unsigned flags,
+                                            int L);
+
+/*
  * The two halves of hcw_stack_bwd, for callers that want them apart (frozen
  * weights need only the first; the second can run later or elsewhere).
  *

@@ -1394,6 +1394,181 @@ int stack_bwd_impl(const Shape& sh, const void* x, const void* acts, const void*
     return dtype == HCW_BF16 ? stack_weight_bf16(sh, wa, st) : stack_weight_f32(sh, wa, st);
 }
 
+// ------------------------------------------------------------ training step
+// Counters of the fused forward + input-gradient launch: per (layer, chunk)
+// completion counters of its 2L layers, the unit counter, the (unused) top-dz
+// chunk counters, and per (layer, chunk) counters of g.
+size_t step_counter_bytes(long long tokens, int L) {
+    const size_t chunks = (size_t)((tokens + 127) / 128);
+    return align256((4 * (size_t)L * chunks + 1 + chunks) * sizeof(int) + 16);
+}
+
+// Whether a training step runs its forward and input gradient as one launch:
+// bf16, the rotated or fixed schedule (no shift layers), the streaming kernels
+// on SM pairs, and up to kMaxStackLayers layers.
+bool step_fused(const Shape& sh, int dtype, const Sched& sc, int L) {
+    return dtype == HCW_BF16 && !sc.has_shift(L) && !use_resident(sh) && use_pairs(sh) &&
+           L <= kMaxStackLayers && sh.tokens > 0;
+}
+
+size_t step_fwd_region(const Shape& sh, int dtype, unsigned flags, int L) {
+    const size_t f = hcw_stack_fwd_workspace_bytes(sh.B, sh.n, sh.d, dtype, flags, L);
+    const size_t c = step_counter_bytes(sh.tokens, L);
+    return align256(f > c ? f : c);
+}
+
+// The forward (layers 0 .. L-1) and the input gradient (layers L-1 .. 0) in one
+// launch on pairs of SMs; the last forward layer writes the top layer's dz.
+int step_fused_launch(const Shape& sh, const void* x, const uint8_t* Ws, const uint8_t* Wn,
+                      const float* bias, const void* dy, const Sched& sc, int L, unsigned flags,
+                      void* y, void* acts, void* masks, void* dx, uint8_t* dz, uint8_t* gws,
+                      int* counters, cudaStream_t st) {
+    const int d = sh.d, BN = pick_bn(d), pw = epi_patch_cols(BN);
+    const size_t ab = sh.act_bytes, a256 = align256(ab), wb = (size_t)d * d * 2;
+    const size_t mb = mask_bytes(sh);
+    const bool relu = (flags & HCW_ACT_RELU) != 0;
+    const bool resid = (flags & HCW_RESIDUAL) != 0;
+    const bool keep_g = relu && resid;
+    auto in_ptr = [&](int l) -> const void* {
+        return l == 0 ? x : static_cast<const uint8_t*>(acts) + (size_t)(l - 1) * ab;
+    };
+    auto out_ptr = [&](int l) -> void* {
+        return l == L - 1 ? y : static_cast<uint8_t*>(acts) + (size_t)l * ab;
+    };
+    auto mask = [&](int l) -> uint32_t* {
+        return relu ? reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(masks) + (size_t)l * mb)
+                    : nullptr;
+    };
+    auto dzp = [&](int l) -> void* { return dz + (size_t)l * ab; };
+    auto gbuf = [&](int l) -> void* { return gws + (size_t)l * a256; };
+    auto g = [&](int l) -> const void* {
+        if (l == L - 1) return dy;
+        return keep_g ? gbuf(l) : dzp(l);
+    };
+    static thread_local TcLaunch<kMaxStepLayers> T;
+    memset(&T, 0, sizeof(T));
+    for (int l = 0; l < L; ++l) {
+        const int s = sc.dim(sh, l);
+        CUtensorMap* m = T.maps[l];
+        if (!fwd_maps(m, sh, s, in_ptr(l), Ws + l * wb, Wn + l * wb, out_ptr(l), true))
+            return HCW_ERR_CUDA;
+        // the last forward layer also stores the top layer's dz (map 5)
+        if (l == L - 1 && !map_rows(&m[5], dzp(L - 1), sh.tokens, d, 1 << s, 32, pw))
+            return HCW_ERR_CUDA;
+        T.layer[l] = {s, 1 << s, bias ? bias + (size_t)l * d : nullptr, mask(l), nullptr, true,
+                      nullptr, false};
+    }
+    for (int i = 0; i < L; ++i) {
+        const int l = L - 1 - i;   // input-gradient layers from the top down
+        const int s = sc.dim(sh, l);
+        const int k = 1 << s;
+        // stores: g_{l-1} (map 4) and dz_{l-1} (map 5); at l = 0 the stack's dx
+        void* out = l == 0 ? dx : (relu ? (resid ? gbuf(l - 1) : nullptr) : dzp(l - 1));
+        void* dzo = (l > 0 && relu) ? dzp(l - 1) : nullptr;
+        CUtensorMap* m = T.maps[L + i];
+        const void* res = resid ? g(l) : dzp(l);
+        if (!map_rows(&m[0], dzp(l), sh.tokens, d, k, 128) ||
+            !map_weight_blocks(&m[1], Ws + l * wb, d, BN / 2 / 64) ||
+            !map_weight_blocks(&m[2], Wn + l * wb, d, BN / 2 / 64) ||
+            !map_rows(&m[3], res, sh.tokens, d, k, 32, pw) ||
+            !map_rows(&m[4], out ? out : dzo, sh.tokens, d, k, 32, pw) ||
+            !map_rows(&m[5], dzo ? dzo : out, sh.tokens, d, k, 32, pw))
+            return HCW_ERR_CUDA;
+        T.layer[L + i] = {s, k, nullptr, nullptr, nullptr, out != nullptr,
+                          dzo ? mask(l - 1) : nullptr, dzo != nullptr};
+    }
+    row_unit_params(T.p, sh, BN, flags, false);
+    pair_units(T.p);
+    T.p.flags = flags;
+    T.n_layers = 2 * L;
+    T.n_fwd = L;
+    const int n_chunks = (int)((sh.tokens + 127) / 128);
+    T.counters = counters;
+    T.n_chunks = n_chunks;
+    T.tokens = (int)sh.tokens;
+    T.sched = counters + (size_t)2 * L * n_chunks;
+    T.in_counters = T.sched + 1;
+    T.g_counters = keep_g ? T.sched + 1 + n_chunks : nullptr;
+    T.top_dy = static_cast<const __nv_bfloat16*>(dy);
+    T.top_dz = static_cast<__nv_bfloat16*>(dzp(L - 1));
+    if (cudaMemsetAsync(counters, 0, step_counter_bytes(sh.tokens, L), st) != cudaSuccess)
+        return HCW_ERR_CUDA;
+    const int sms = sm_count();
+    const int total = T.p.n_units * 2 * L;
+    const int pairs = total < sms / 2 ? total : sms / 2;
+    return launched(launch_tc_step_pair(BN, T, 2 * pairs, st), 1);
+}
+
+int train_step_impl(const Shape& sh, const void* x, const void* W_self, const void* W_nbr,
+                    const float* bias, const void* dy, const Sched& sc, int L, int dtype,
+                    unsigned flags, void* y, void* acts, void* masks, void* dx, float* dW_self,
+                    float* dW_nbr, float* dbias, void* workspace, size_t ws_bytes, void* stream) {
+    const int d = sh.d;
+    cudaStream_t st = (cudaStream_t)stream;
+    // workspace: [backward (dz | input-gradient scratch | weight-gradient
+    // scratch)][forward scratch, or the fused launch's counters]
+    const size_t zb = stack_dz_bytes(sh, L);
+    const size_t db = align256(stack_data_ws(sh, dtype, flags, L));
+    const size_t wbb = stack_weight_ws(sh, dtype, flags, L);
+    const size_t bwd = align256(zb + db + wbb);
+    const size_t fwd = step_fwd_region(sh, dtype, flags, L);
+    // no weight-gradient outputs: the forward and the input gradient only
+    const bool want_dw = dW_self != nullptr || dW_nbr != nullptr;
+    if (want_dw && (!dW_self || !dW_nbr)) return HCW_ERR_INVALID_ARG;
+    if (!want_dw && dbias) return HCW_ERR_INVALID_ARG;
+    if (sh.tokens == 0) return want_dw ? zero_weight_grads(L, d, dW_self, dW_nbr, dbias, st) : HCW_OK;
+    if (ws_bytes < bwd + fwd || !workspace) return HCW_ERR_WORKSPACE;
+    if (!aligned16(workspace)) return HCW_ERR_ALIGNMENT;
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    if (!step_fused(sh, dtype, sc, L)) {
+        int rc = stack_fwd_impl(sh, x, W_self, W_nbr, bias, sc, L, dtype, flags, y, acts, masks,
+                                ws + bwd, fwd, stream);
+        if (rc) return rc;
+        if (want_dw)
+            return stack_bwd_impl(sh, x, acts, masks, dy, W_self, W_nbr, sc, L, dtype, flags, dx,
+                                  dW_self, dW_nbr, dbias, ws, bwd, stream);
+        rc = check_stack_data(sh, dtype, flags, L, masks, dy, W_self, W_nbr, dx, ws, ws + zb, db);
+        if (rc) return rc;
+        StackData da{masks, dy, static_cast<const uint8_t*>(W_self),
+                     static_cast<const uint8_t*>(W_nbr), sc, L, flags, dx, ws, ws + zb};
+        return dtype == HCW_BF16 ? stack_data_bf16(sh, da, st) : stack_data_f32(sh, da, st);
+    }
+    // the checks of the forward and the backward calls, on the same buffers
+    if (L > 1 && !acts) return HCW_ERR_INVALID_ARG;
+    if ((acts && !aligned16(acts)) || (masks && !aligned16(masks))) return HCW_ERR_ALIGNMENT;
+    int rc = check_fwd_ptrs(sh, dtype, x, W_self, W_nbr, bias, y, nullptr);
+    if (rc) return rc;
+    const size_t ab = sh.act_bytes, wb = (size_t)d * d * 2;
+    const size_t acts_b = (size_t)(L - 1) * ab, m_b = (size_t)L * mask_bytes(sh);
+    if (overlaps(acts, acts_b, x, ab) || overlaps(acts, acts_b, y, ab) ||
+        overlaps(masks, m_b, x, ab) || overlaps(masks, m_b, y, ab) ||
+        overlaps(masks, m_b, acts, acts_b) || overlaps(acts, acts_b, W_self, L * wb) ||
+        overlaps(acts, acts_b, W_nbr, L * wb) || overlaps(ws, ws_bytes, x, ab) ||
+        overlaps(ws, ws_bytes, y, ab) || overlaps(ws, ws_bytes, acts, acts_b) ||
+        overlaps(ws, ws_bytes, masks, m_b) || overlaps(dx, ab, y, ab) ||
+        overlaps(dx, ab, acts, acts_b) || overlaps(dx, ab, x, ab) ||
+        overlaps(dx, ab, masks, m_b))
+        return HCW_ERR_ALIASING;
+    rc = check_stack_data(sh, dtype, flags, L, masks, dy, W_self, W_nbr, dx, ws, ws + zb, db);
+    if (rc) return rc;
+    if (want_dw) {
+        rc = check_stack_weight(sh, dtype, flags, L, x, acts, ws, dW_self, dW_nbr, dbias,
+                                ws + zb + db, wbb);
+        if (rc) return rc;
+    }
+    if (overlaps(dx, ab, dW_self, (size_t)L * d * d * 4) ||
+        overlaps(dx, ab, dW_nbr, (size_t)L * d * d * 4) ||
+        overlaps(dx, ab, dbias, dbias ? (size_t)L * d * 4 : 0) ||
+        overlaps(dy, ab, y, ab) || overlaps(dy, ab, acts, acts_b) || overlaps(dy, ab, masks, m_b))
+        return HCW_ERR_ALIASING;
+    rc = step_fused_launch(sh, x, static_cast<const uint8_t*>(W_self),
+                           static_cast<const uint8_t*>(W_nbr), bias, dy, sc, L, flags, y, acts,
+                           masks, dx, ws, ws + zb, reinterpret_cast<int*>(ws + bwd), st);
+    if (rc || !want_dw) return rc;
+    StackWeight wa{x, acts, ws, sc, L, flags, dW_self, dW_nbr, dbias, ws + zb + db};
+    return stack_weight_bf16(sh, wa, st);
+}
+
 // Link distance of decode layer l: 2^s for the hypercube link along
 // dimension s, k for a shift by k.
 int decode_link(const int* dims, int layer0, int b, int l) {
@@ -1653,6 +1828,29 @@ int hcw_stack_bwd_weight(const void* x, const void* acts, const void* dz, int la
                   flags, dW_self, dW_nbr, dbias, static_cast<uint8_t*>(workspace)};
     return dtype == HCW_BF16 ? stack_weight_bf16(sh, a, (cudaStream_t)stream)
                              : stack_weight_f32(sh, a, (cudaStream_t)stream);
+}
+
+size_t hcw_stack_train_step_workspace_bytes(int B, int n, int d, int dtype, unsigned flags,
+                                            int L) {
+    Shape sh;
+    if (L < 1 || check_shape(0, -1, B, n, d, dtype, flags, &sh)) return 0;
+    return align256(stack_dz_bytes(sh, L) + align256(stack_data_ws(sh, dtype, flags, L)) +
+                    stack_weight_ws(sh, dtype, flags, L)) +
+           step_fwd_region(sh, dtype, flags, L);
+}
+
+int hcw_stack_train_step(const void* x, const void* W_self, const void* W_nbr, const float* bias,
+                         const void* dy, int layer0, int L, int dim_override, int B, int n, int d,
+                         int dtype, unsigned flags, void* y, void* acts, void* masks, void* dx,
+                         float* dW_self, float* dW_nbr, float* dbias, void* workspace,
+                         size_t ws_bytes, void* stream) {
+    Shape sh;
+    if (L < 1) return HCW_ERR_INVALID_ARG;
+    int rc = check_shape(layer0, dim_override, B, n, d, dtype, flags, &sh);
+    if (rc) return rc;
+    return train_step_impl(sh, x, W_self, W_nbr, bias, dy, Sched{nullptr, layer0, dim_override}, L,
+                           dtype, flags, y, acts, masks, dx, dW_self, dW_nbr, dbias, workspace,
+                           ws_bytes, stream);
 }
 
 int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void* dy,

@@ -13,7 +13,10 @@ namespace hcw {
 // MODE_DWF: weight gradients of a run of layers, one unit per (layer, output
 // tile) that accumulates the self and the partner part together.
 // MODE_DWP: the same on pairs of SMs (cta_group::2, 256-row tiles, BN >= 128).
-enum TcMode { MODE_FWD = 0, MODE_DX = 1, MODE_DW = 2, MODE_DWF = 3, MODE_DWP = 4 };
+// MODE_FDX: a stacked forward and the stack's input gradient in one launch on
+// pairs of SMs: layers [0, n_fwd) are forward layers, the rest input-gradient
+// layers from the top down.
+enum TcMode { MODE_FWD = 0, MODE_DX = 1, MODE_DW = 2, MODE_DWF = 3, MODE_DWP = 4, MODE_FDX = 5 };
 
 // Work description of one tensor-core launch (see hcw_tc.cu for the unit
 // decomposition).  Row indices are "compressed": for a fixed value beta of
@@ -72,6 +75,7 @@ struct TcLayer {
 constexpr int epi_patch_cols(int BN) { return BN >= 256 ? 64 : 32; }
 
 constexpr int kMaxStackLayers = 16;   // layers per stacked-forward launch
+constexpr int kMaxStepLayers = 2 * kMaxStackLayers;   // forward + input-gradient launch
 
 // maps[l][0..5] = tmA, tmB0, tmB1, tmE0, tmE1, tmE2 of layer l, as documented
 // at hcw_tc_kernel in hcw_tc.cu.
@@ -102,6 +106,9 @@ struct TcLaunch {
     // next layer's MMAs wait for -- is published before g is stored.  Null:
     // g is dz (or absent) and the counters above cover it.
     int* g_counters;
+    // MODE_FDX: the number of forward layers; the last of them also writes the
+    // top layer's dz = dy * act'(z) (top_dy, top_dz) for the layers after it
+    int n_fwd;
 };
 
 // Launch one tensor-core pass (one layer).
@@ -115,6 +122,10 @@ cudaError_t launch_tc_stack(int mode, int BN, const TcLaunch<kMaxStackLayers>& L
 // cta_group::2; BN 256, even grid).  L.p counts pair units: row-block pairs.
 cudaError_t launch_tc_stack_pair(int mode, int BN, const TcLaunch<kMaxStackLayers>& L, int grid,
                                  cudaStream_t stream);
+// MODE_FDX on clusters of two CTAs (BN 256, even grid): L.n_fwd forward layers
+// followed by the input gradient of those layers, top down.
+cudaError_t launch_tc_step_pair(int BN, const TcLaunch<kMaxStepLayers>& L, int grid,
+                                cudaStream_t stream);
 
 // ---- Resident stacked launches (hcw_res.cu) ----
 // A cluster of two CTAs keeps 256 consecutive tokens (whole samples, n <= 256)

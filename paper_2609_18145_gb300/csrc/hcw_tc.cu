@@ -48,6 +48,7 @@
 // HCW_ERR_TIMEOUT, drains its in-flight copies and MMAs, frees TMEM and
 // returns.
 #include <atomic>
+#include <type_traits>
 
 #include "hcw_internal.h"
 #include "hcw_ptx.cuh"
@@ -127,7 +128,8 @@ struct RowUnit {
     int beta, t, j, steps;
 };
 
-__device__ __forceinline__ RowUnit decode_row_unit(const TcParams& p, int u, bool stacked) {
+__device__ __forceinline__ RowUnit decode_row_unit(const TcParams& p, int u, bool stacked,
+                                                   bool mirror = false) {
     RowUnit r;
     const int per_bit = p.n_rb * p.n_nt;
     int g, rem;
@@ -152,6 +154,9 @@ __device__ __forceinline__ RowUnit decode_row_unit(const TcParams& p, int u, boo
         r.beta = p.half_bit;
         r.steps = p.nK;
     }
+    // input-gradient units of a fused launch (parameters set for the forward):
+    // under the causal rule the rows that take both parts are the other bit value
+    if (mirror && p.n_full == 1) r.beta ^= 1;
     return r;
 }
 
@@ -399,7 +404,9 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
     // PAIR (stacked forward / input gradient): clusters of two CTAs, 256-row
     // tiles with tcgen05.mma.cta_group::2; each CTA loads its own 128 rows and
     // half of the weight tile, the leader issues the MMAs (see hcw_dwp_kernel)
-    static_assert(!PAIR || ((MODE == MODE_FWD || MODE == MODE_DX) && NL > 1), "pair modes");
+    static_assert(!PAIR || ((MODE == MODE_FWD || MODE == MODE_DX || MODE == MODE_FDX) && NL > 1),
+                  "pair modes");
+    static_assert(MODE != MODE_FDX || PAIR, "the fused launch runs on pairs");
     constexpr int STAGES = PAIR ? tc_pair_stages(BN) : num_stages(BN, MODE);
     constexpr bool DWF = MODE == MODE_DWF;
     static_assert(!DWF || STAGES % 2 == 0, "pairs of stages");
@@ -410,6 +417,14 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
     constexpr uint32_t IDESC = idesc_bf16_f32(PAIR ? 2 * kBlockM : kBlockM, BN,
                                               (MODE == MODE_DW || DWF) ? 1 : 0,
                                               MODE == MODE_FWD ? 0 : 1);
+    // the fused launch's forward units: B (the weights) K-major
+    constexpr uint32_t IDESC_FWD = idesc_bf16_f32(PAIR ? 2 * kBlockM : kBlockM, BN, 0, 0);
+    // whether layer l of the launch is a forward layer, and (fused launch) the
+    // first input-gradient layer
+    auto is_fwd = [&](int l) {
+        return MODE == MODE_FWD || (MODE == MODE_FDX && l < L.n_fwd);
+    };
+    const int first_dx = MODE == MODE_FDX ? L.n_fwd : 0;
     constexpr int EW = epi_warps(BN);
     constexpr int WCOLS = warp_cols(BN);               // columns per epilogue warp
     static_assert(EW <= kMaxEpiWarps && WCOLS % 32 == 0 && WCOLS <= 64, "epilogue split");
@@ -579,7 +594,8 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                         }
                     }
                 } else if (MODE != MODE_DW) {
-                    RowUnit r = decode_row_unit(p, ul, STACKED);
+                    const bool ufwd = is_fwd(l);
+                    RowUnit r = decode_row_unit(p, ul, STACKED, !ufwd && MODE == MODE_FDX);
                     if (PAIR) r.t = 2 * r.t + (int)rank;   // this CTA's half of the 256 rows
                     const int q0 = r.t * kBlockM;
                     const int lo0 = q0 & (ly.k - 1), hi0 = q0 >> ly.s;
@@ -623,7 +639,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                             if (rank == 0) mbar_arrive_expect_tx(&bars->full[stage], 2 * SB);
                             const uint32_t fb = mapa_shared(&bars->full[stage], 0);
                             tma_load_4d_pair(sA, mAk, fb, kk * kBlockK, lo0, bitA, hi0);
-                            if (MODE == MODE_FWD)
+                            if (ufwd)
                                 tma_load_2d_pair(sB, mb, fb, kk * kBlockK,
                                                  r.j * BN + (int)rank * (BN / 2));
                             else
@@ -632,7 +648,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                         } else {
                             mbar_arrive_expect_tx(&bars->full[stage], kABytes + B_BYTES);
                             tma_load_4d(sA, mAk, &bars->full[stage], kk * kBlockK, lo0, bitA, hi0);
-                            if (MODE == MODE_FWD)
+                            if (ufwd)
                                 tma_load_2d(sB, mb, &bars->full[stage], kk * kBlockK, r.j * BN);
                             else   // BN / 64 blocks of 64 W columns x 64 rows, one copy
                                 tma_load_3d(sB, mb, &bars->full[stage], 0, kk * kBlockK,
@@ -760,6 +776,15 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     continue;
                 }
                 int steps;
+                // the B operand: K-major (forward: W rows) or MN-major (input
+                // gradient: W columns); a fused launch picks it per unit
+                uint32_t idesc = IDESC, b_step = MODE == MODE_FWD ? 32 : 2048,
+                         b_lbo = MODE == MODE_FWD ? 16 : 8192;
+                if (MODE == MODE_FDX && is_fwd(u / upl)) {
+                    idesc = IDESC_FWD;
+                    b_step = 32;
+                    b_lbo = 16;
+                }
                 if (MODE != MODE_DW) {
                     steps = decode_row_unit(p, ul, STACKED).steps;
                 } else {
@@ -788,14 +813,14 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                             adesc = smem_desc_sw128(a_addr + kk * 2048, 8192, 1024);
                         else
                             adesc = smem_desc_sw128(a_addr + kk * 32, 16, 1024);
-                        if (MODE == MODE_FWD)
-                            bdesc = smem_desc_sw128(b_addr + kk * 32, 16, 1024);
-                        else
+                        if (MODE == MODE_DW)
                             bdesc = smem_desc_sw128(b_addr + kk * 2048, 8192, 1024);
-                        if (PAIR)
-                            mma_bf16_f32_pair(d_tmem, adesc, bdesc, IDESC, (ks | kk) != 0);
                         else
-                            mma_bf16_f32(d_tmem, adesc, bdesc, IDESC, (ks | kk) != 0);
+                            bdesc = smem_desc_sw128(b_addr + kk * b_step, b_lbo, 1024);
+                        if (PAIR)
+                            mma_bf16_f32_pair(d_tmem, adesc, bdesc, idesc, (ks | kk) != 0);
+                        else
+                            mma_bf16_f32(d_tmem, adesc, bdesc, idesc, (ks | kk) != 0);
                     }
                     any = true;
                     if (PAIR)
@@ -1044,9 +1069,14 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     }
                 }
             } else if (MODE != MODE_DW) {
+                // One body per direction, each compiled with the direction fixed (a
+                // fused launch picks one per unit): the epilogue sits on the layer
+                // chain, and a run-time direction costs registers and instructions.
+                auto row_epilogue = [&](auto fwd_tag) -> bool {
+                constexpr bool fwd = decltype(fwd_tag)::value;
                 constexpr int RB = WCOLS * 2;                  // patch row bytes (128 or 64)
                 constexpr int SUB = WCOLS / 32;                // 32-column sub-chunks per patch
-                RowUnit r = decode_row_unit(p, ul, STACKED);
+                RowUnit r = decode_row_unit(p, ul, STACKED, !fwd && MODE == MODE_FDX);
                 if (PAIR) r.t = 2 * r.t + (int)rank;
                 const int qw = r.t * kBlockM + quarter * 32;   // first compressed row of the warp
                 const int lo_w = qw & (ly.k - 1), hi_w = qw >> ly.s;
@@ -1058,8 +1088,10 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                 // a patch entirely past the end (ragged tail) loads and stores nothing
                 const bool inside = qw < p.Mh;
                 const bool has_res = (p.flags & 2u) != 0 && inside;
-                const bool fwd = MODE == MODE_FWD;
-                const bool has_mprev = MODE == MODE_DX && ly.mprev != nullptr && ly.dz_out;
+                const bool has_mprev = !fwd && ly.mprev != nullptr && ly.dz_out;
+                // fused launch: the last forward layer also writes the top layer's
+                // dz = dy * act'(z), the first input-gradient layer's operand
+                const bool top_dz = MODE == MODE_FDX && l == L.n_fwd - 1 && L.top_dy != nullptr;
                 const CUtensorMap* mE0 = &L.maps[l][3];
                 const CUtensorMap* mE1 = &L.maps[l][4];
                 const CUtensorMap* mE2 = &L.maps[l][5];
@@ -1072,8 +1104,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                 if (lane == 0) bulk_wait_read<0>();
                 __syncwarp();
                 if (!wait_inputs(ordinal)) {
-                    alive = false;
-                    break;
+                    return false;
                 }
                 if (has_res) {
                     int okg = 1;
@@ -1081,7 +1112,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                         // stacked input gradient: the residual term g of these rows is
                         // stored by the layer above after its dz; wait until the chunk's g
                         // is complete (the dz the MMAs read was checked by the producer)
-                        if (MODE == MODE_DX && STACKED && L.g_counters != nullptr && l > 0) {
+                        if (!fwd && STACKED && L.g_counters != nullptr && l > first_dx) {
                             okg = wait_counter(L.g_counters + (size_t)(l - 1) * L.n_chunks + chunk,
                                                min(128, L.tokens - (chunk << 7)) * p.d, abort, tmo);
                             if (okg) fence_proxy_async_global();
@@ -1092,8 +1123,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                         }
                     }
                     if (__shfl_sync(0xffffffffu, okg, 0) == 0) {
-                        alive = false;
-                        break;
+                        return false;
                     }
                 }
                 uint32_t mp[SUB];
@@ -1109,8 +1139,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     __syncwarp();
                 }
                 if (!wait_acc()) {
-                    alive = false;
-                    break;
+                    return false;
                 }
                 // FWD z (layer API only): the pre-activation, row-wise stores; every
                 // lane joins the warp-wide TMEM loads, rows past the end skip the store
@@ -1141,8 +1170,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     const bool okl = wait_bar(&bars->epi_load[e], ld_phase);
                     ld_phase ^= 1;
                     if (!okl) {
-                        alive = false;
-                        break;
+                        return false;
                     }
                 }
                 const bool write_out = fwd || ly.out;
@@ -1319,6 +1347,42 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                             bulk_commit();
                         }
                     }
+                    if (top_dz) {
+                        // the top layer's dz = dy * [z > 0] (a copy of dy without the
+                        // ReLU) for the same rows and columns, dy read straight from
+                        // global memory, written over the buffer once the y store has
+                        // read it; counted with y below
+                        if (lane == 0) bulk_wait_read<0>();
+                        __syncwarp();
+#pragma unroll
+                        for (int h = 0; h < SUB; ++h) {
+                            uint4 q4[4] = {};
+                            if (tok_row >= 0) {
+                                const uint4* src = reinterpret_cast<const uint4*>(
+                                    L.top_dy + (size_t)tok_row * p.d + col0 + h * 32);
+#pragma unroll
+                                for (int m = 0; m < 4; ++m) q4[m] = __ldg(src + m);
+                            }
+                            const uint32_t mw = (p.flags & 4u) ? mbits[h] : ~0u;
+#pragma unroll
+                            for (int m = 0; m < 4; ++m) {
+                                uint32_t w4[4] = {q4[m].x, q4[m].y, q4[m].z, q4[m].w};
+#pragma unroll
+                                for (int i = 0; i < 4; ++i) {
+                                    const int b = 8 * m + 2 * i;
+                                    w4[i] &= ((mw >> b) & 1u ? 0x0000FFFFu : 0u) |
+                                             ((mw >> (b + 1)) & 1u ? 0xFFFF0000u : 0u);
+                                }
+                                *patch_piece<RB>(buf, lane, 4 * h + m) =
+                                    make_uint4(w4[0], w4[1], w4[2], w4[3]);
+                            }
+                        }
+                        publish();
+                        if (lane == 0 && inside) {
+                            tma_store_4d(mE2, buf, col0, lo_w, r.beta, hi_w);
+                            bulk_commit();
+                        }
+                    }
                     if (signal) count(L.counters, 0);
                 }
                 // FWD: the ReLU mask words, read only by the input gradient (a later
@@ -1327,6 +1391,18 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
 #pragma unroll
                     for (int h = 0; h < SUB; ++h)
                         ly.mout[(size_t)tok_row * wpr + (col0 >> 5) + h] = mbits[h];
+                }
+                return true;
+                };
+                bool ok_unit;
+                if (MODE == MODE_FDX)
+                    ok_unit = is_fwd(l) ? row_epilogue(std::true_type{})
+                                        : row_epilogue(std::false_type{});
+                else
+                    ok_unit = row_epilogue(std::integral_constant<bool, MODE == MODE_FWD>{});
+                if (!ok_unit) {
+                    alive = false;
+                    break;
                 }
             } else {
                 const WUnit& w = wu;
@@ -1822,6 +1898,12 @@ cudaError_t launch_tc_stack_pair(int mode, int BN, const TcLaunch<kMaxStackLayer
     if (mode == MODE_FWD) return launch_one<MODE_FWD, 256, kMaxStackLayers, true>(L, grid, st);
     if (mode == MODE_DX) return launch_one<MODE_DX, 256, kMaxStackLayers, true>(L, grid, st);
     return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_tc_step_pair(int BN, const TcLaunch<kMaxStepLayers>& L, int grid,
+                                cudaStream_t st) {
+    if (BN != 256 || grid % 2) return cudaErrorInvalidValue;
+    return launch_one<MODE_FDX, 256, kMaxStepLayers, true>(L, grid, st);
 }
 
 size_t tc_smem_bytes(int BN) {

@@ -79,6 +79,9 @@ _SIGNATURES = {
     "hcw_stack_bwd_weight_workspace_bytes": ([_I, _I, _I, _I, _U, _I], _SZ),
     "hcw_stack_bwd": ([_P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P,
                        _P, _P, _SZ, _P], _I),
+    "hcw_stack_train_step": ([_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P,
+                              _P, _P, _P, _P, _P, _SZ, _P], _I),
+    "hcw_stack_train_step_workspace_bytes": ([_I, _I, _I, _I, _U, _I], _SZ),
     "hcw_decode_step": ([_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P],
                         _I),
     "hcw_decode_cache_bytes": ([_P, _I, _I, _I, _I, _I], _SZ),
@@ -424,6 +427,44 @@ def hcw_stack_bwd(x, acts, masks, dy, W_self, W_nbr, layer0: int = 0, dim_overri
                                _ptr(dx), _ptr(dW_self), _ptr(dW_nbr), _ptr(dbias), _ptr(ws),
                                ws.numel(), _stream(stream)), "hcw_stack_bwd")
     return dx, dW_self, dW_nbr, dbias
+
+
+def hcw_stack_train_step_workspace_bytes(B: int, n: int, d: int, dtype: int, flags: int,
+                                         L: int) -> int:
+    return int(lib().hcw_stack_train_step_workspace_bytes(B, n, d, dtype, flags, L))
+
+
+def hcw_stack_train_step(x, W_self, W_nbr, bias, dy, layer0: int = 0, dim_override: int = -1,
+                         flags: int = 0, y=None, acts=None, masks=None, dx=None, dW_self=None,
+                         dW_nbr=None, dbias=None, want_dbias: bool = True,
+                         want_dw: bool = True, workspace=None, stream=None):
+    """Forward and backward of a stack in one call; returns (y, acts, masks,
+    dx, dW_self[L], dW_nbr[L], dbias[L]).  want_dw=False: the forward and the
+    input gradient only (the weight-gradient outputs are None)."""
+    _dev(x, W_self, W_nbr, bias, dy, y, acts, masks, dx, dW_self, dW_nbr, dbias, workspace)
+    B, n, d = x.shape
+    L = W_self.shape[0]
+    dt = _dtype_code(x)
+    f32 = dict(dtype=torch.float32, device=x.device)
+    y = torch.empty_like(x) if y is None else y
+    if acts is None and L > 1:
+        acts = torch.empty((L - 1, B, n, d), dtype=x.dtype, device=x.device)
+    if masks is None and flags & HCW_ACT_RELU:
+        masks = torch.empty((L, B, n, (d + 31) // 32), dtype=torch.int32, device=x.device)
+    dx = torch.empty_like(x) if dx is None else dx
+    if want_dw:
+        dW_self = torch.empty(L, d, d, **f32) if dW_self is None else dW_self
+        dW_nbr = torch.empty(L, d, d, **f32) if dW_nbr is None else dW_nbr
+        if dbias is None and want_dbias:
+            dbias = torch.empty(L, d, **f32)
+    ws = _workspace(hcw_stack_train_step_workspace_bytes(B, n, d, dt, flags, L), x.device,
+                    workspace)
+    _check(lib().hcw_stack_train_step(_ptr(x), _ptr(W_self), _ptr(W_nbr), _ptr(bias), _ptr(dy),
+                                      layer0, L, dim_override, B, n, d, dt, flags, _ptr(y),
+                                      _ptr(acts), _ptr(masks), _ptr(dx),
+                                      _ptr(dW_self), _ptr(dW_nbr), _ptr(dbias), _ptr(ws),
+                                      ws.numel(), _stream(stream)), "hcw_stack_train_step")
+    return y, acts, masks, dx, dW_self, dW_nbr, dbias
 
 
 def hcw_stack_bwd_dims(x, acts, masks, dy, W_self, W_nbr, dims, flags: int = 0, **kw):
