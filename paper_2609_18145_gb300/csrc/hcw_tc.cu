@@ -326,6 +326,29 @@ __device__ __forceinline__ uint64_t bf16x2_to_f32x2(uint32_t w) {
     return f32x2_pack(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
 }
 
+// 32 ReLU mask bits (bit c = column c) -> the AND-masks of 16 bf16 column
+// pairs: pair q keeps its low half iff bit 2q is set, its high half iff bit
+// 2q + 1 is.  t[k] = mw << (7 - k) puts bits k, k + 8, k + 16, k + 24 at the
+// sign positions of its four bytes; prmt in sign-replicate mode (selector
+// nibble 8 | byte) turns a selected byte into 0xFF or 0x00 by its sign bit, so
+// each pair's mask is one prmt of t[2i] and t[2i + 1] (the pair's two bits sit
+// in the same byte b = q / 4 of both).
+struct PairMasks {
+    uint32_t t[8];
+    __device__ __forceinline__ explicit PairMasks(uint32_t mw) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) t[k] = mw << (7 - k);
+    }
+    __device__ __forceinline__ uint32_t operator()(int q) const {
+        const int i = q & 3, b = q >> 2;
+        const uint32_t sel = (uint32_t)(8 | b) | (uint32_t)(8 | b) << 4 |
+                             (uint32_t)(12 | b) << 8 | (uint32_t)(12 | b) << 12;
+        uint32_t r;
+        asm("prmt.b32 %0, %1, %2, %3;" : "=r"(r) : "r"(t[2 * i]), "r"(t[2 * i + 1]), "r"(sel));
+        return r;
+    }
+};
+
 // Adds v to the shared int *p with acquire-release semantics at CTA scope and
 // returns the previous value.
 __device__ __forceinline__ int atom_add_acq_rel_cta_shared(int* p, int v) {
@@ -1249,17 +1272,12 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     // With the ReLU gradient of the layer below, dz = dx * mask goes
                     // first; otherwise y (FWD) or dx (DX).
                     if (has_mprev) {
-                        const uint32_t mw = mp[h];
+                        const PairMasks keep(mp[h]);
 #pragma unroll
                         for (int m = 0; m < 4; ++m) {
                             uint32_t w4[4];
 #pragma unroll
-                            for (int i = 0; i < 4; ++i) {
-                                const int b = 8 * m + 2 * i;
-                                const uint32_t keep = ((mw >> b) & 1u ? 0x0000FFFFu : 0u) |
-                                                      ((mw >> (b + 1)) & 1u ? 0xFFFF0000u : 0u);
-                                w4[i] = gw[h][4 * m + i] & keep;
-                            }
+                            for (int i = 0; i < 4; ++i) w4[i] = gw[h][4 * m + i] & keep(4 * m + i);
                             *patch_piece<RB>(buf, lane, 4 * h + m) =
                                 make_uint4(w4[0], w4[1], w4[2], w4[3]);
                         }
@@ -1363,16 +1381,12 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
 #pragma unroll
                                 for (int m = 0; m < 4; ++m) q4[m] = __ldg(src + m);
                             }
-                            const uint32_t mw = (p.flags & 4u) ? mbits[h] : ~0u;
+                            const PairMasks keep((p.flags & 4u) ? mbits[h] : ~0u);
 #pragma unroll
                             for (int m = 0; m < 4; ++m) {
                                 uint32_t w4[4] = {q4[m].x, q4[m].y, q4[m].z, q4[m].w};
 #pragma unroll
-                                for (int i = 0; i < 4; ++i) {
-                                    const int b = 8 * m + 2 * i;
-                                    w4[i] &= ((mw >> b) & 1u ? 0x0000FFFFu : 0u) |
-                                             ((mw >> (b + 1)) & 1u ? 0xFFFF0000u : 0u);
-                                }
+                                for (int i = 0; i < 4; ++i) w4[i] &= keep(4 * m + i);
                                 *patch_piece<RB>(buf, lane, 4 * h + m) =
                                     make_uint4(w4[0], w4[1], w4[2], w4[3]);
                             }
