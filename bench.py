@@ -1,8 +1,9 @@
 #!/usr/bin/env python
 """Throughput of the rotated-hypercube mixing stack on GB300, forward + backward.
 
-One step = hcw_stack_fwd + hcw_stack_bwd over one batch of the char-LM
-window-256 workload: B = 64 sequences of n = 256 positions, d = 512,
+One step = one hcw_stack_train_step call (the work of hcw_stack_fwd +
+hcw_stack_bwd) over one batch of the char-LM window-256 workload: B = 64
+sequences of n = 256 positions, d = 512,
 16 rotated causal layers (dimensions 0..7 twice), residual, ReLU, bias, with
 per-layer weight gradients (Sec. 3.1 wiring, Eq. (1) maps).  Inputs are
 synthetic (Zipf(1.1) byte ids embedded to d; see paper_2609_18145_gb300.synth)
@@ -466,13 +467,13 @@ def run_ours(args):
                   % args.schedule: 2.0 * f_flops}
         kernels = dict(zip(kflops, (f_ms, b_ms)))
         dwb_ms = dw_ms = 0.0
-    else:
+    family = H.hcw_stack_kernels_used(B, n, d)
+    fused = dims is None and family == H.HCW_STACK_STREAMING and d % 256 == 0 and L <= 16
+    if dims is None and not fused:
         kflops = None
         fwd_ms = time_calls(lambda i: H.hcw_stack_fwd(x, Ws, Wn, bias, 0, -1, flags, y=y,
                                                       acts=acts, masks=masks, workspace=fws),
                             reps)
-    family = H.hcw_stack_kernels_used(B, n, d)
-    fused = dims is None and family == H.HCW_STACK_STREAMING and d % 256 == 0 and L <= 16
     if fused:
         # the step's two launches: the forward and the input gradient in one
         # launch (the training step without weight gradients), and the batched
@@ -646,6 +647,226 @@ def run_ours(args):
     return 0
 
 
+# ---------------------------------------------------------------- other workloads
+# The other configurations of the mixing stack, one JSON line each (--workload):
+# the synthetic reachability shape (rotated, and its fixed-dimension control),
+# the character-LM window-64 shape, and the 2^20-token scaling sweep at
+# d = 1024 (L = log2 n), fwd+bwd and forward only.  Same timing rules as the
+# headline line: warm-up, L2 flushed before every timed step, CUDA events.
+WORKLOADS_EXTRA = {
+    # name: (synth.WORKLOADS entry, dim_override, forward only)
+    "reach_n64_d128": ("reach_n64_d128", -1, False),
+    "reach_n64_d128_fixed": ("reach_n64_d128", 0, False),
+    "charlm_w64_d512": ("charlm_w64_d512", -1, False),
+    "scale_n256_d1024": ("scale_n256_d1024", -1, False),
+    "scale_n4096_d1024": ("scale_n4096_d1024", -1, False),
+    "scale_n65536_d1024": ("scale_n65536_d1024", -1, False),
+    "scale_n256_d1024_fwd": ("scale_n256_d1024", -1, True),
+    "scale_n4096_d1024_fwd": ("scale_n4096_d1024", -1, True),
+    "scale_n65536_d1024_fwd": ("scale_n65536_d1024", -1, True),
+}
+
+
+def workload_bytes(d, L, causal, relu, fwd_only):
+    """Algorithmic HBM bytes per token of one step (bf16 activations, each
+    tensor moved once): per layer the forward reads x and writes y (4d), the
+    backward reads the layer input and the output gradient and writes the
+    input gradient (6d); with ReLU one mask bit per feature is written and read
+    back.  Weights (4 d^2 bytes per layer) are amortised over the batch."""
+    m = d / 8.0 if relu else 0.0
+    if fwd_only:
+        return (4.0 * d + m) * L
+    return (10.0 * d + 2.0 * m) * L
+
+
+def workload_flops(d, L, causal, fwd_only):
+    per = (3.0 if causal else 4.0) * d * d      # flop = 2 MAC; causal: half the rows
+    return per * L * (1 if fwd_only else 3)
+
+
+def run_workload(args):
+    import torch
+
+    from oracle import oracle as O
+    from paper_2609_18145_gb300 import hcw as H
+    from paper_2609_18145_gb300 import replicas, synth
+
+    rank, local_rank, world = replicas.env_world()
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA GPU (the compute path has no CPU fallback)")
+    torch.cuda.set_device(local_rank)
+    replicas.init("nccl")
+    dev = torch.device("cuda", local_rank)
+    H.lib()
+    key, dim_over, fwd_only = WORKLOADS_EXTRA[args.workload]
+    w = synth.WORKLOADS[key]
+    B, n, d, L, causal = w["B"], w["n"], w["d"], w["L"], w["causal"]
+    flags = (H.HCW_CAUSAL if causal else 0) | H.HCW_RESIDUAL | H.HCW_ACT_RELU
+    tokens = B * n
+    peaks, peak_src = load_peaks()
+    wstd = (1 / (2 * d)) ** 0.5
+    seed = replicas.batch_seed(0, rank)
+    # inputs: weights from the host generator, activations of the 2^20-token
+    # shapes drawn on the device (4 GiB each in fp32)
+    Ws = torch.from_numpy(synth.normal((L, d, d), 2, wstd)).to(torch.bfloat16).to(dev)
+    Wn = torch.from_numpy(synth.normal((L, d, d), 3, wstd)).to(torch.bfloat16).to(dev)
+    bias = torch.from_numpy(synth.normal((L, d), 4, 0.1)).to(dev)
+    if tokens * d <= (1 << 24):
+        px = synth.problem(B, n, d, L=1, seed=seed, x_ids=w.get("x_ids"))
+        x = torch.from_numpy(px.x).to(torch.bfloat16).to(dev)
+        dy = torch.from_numpy(px.dy).to(torch.bfloat16).to(dev)
+    else:
+        x = synth.device_normal((B, n, d), seed + 1, dev).to(torch.bfloat16)
+        dy = synth.device_normal((B, n, d), seed + 5, dev).to(torch.bfloat16)
+    y = torch.empty_like(x)
+    acts = torch.empty((L - 1, B, n, d), dtype=torch.bfloat16, device=dev)
+    masks = torch.empty((L, B, n, (d + 31) // 32), dtype=torch.int32, device=dev)
+    dx = torch.empty_like(x)
+    gWs = torch.empty((L, d, d), dtype=torch.float32, device=dev)
+    gWn = torch.empty((L, d, d), dtype=torch.float32, device=dev)
+    gb = torch.empty((L, d), dtype=torch.float32, device=dev)
+    if fwd_only:
+        ws = torch.empty(max(1, H.hcw_stack_fwd_workspace_bytes(B, n, d, H.HCW_BF16, flags, L)),
+                         dtype=torch.uint8, device=dev)
+    else:
+        ws = torch.empty(max(1, H.hcw_stack_train_step_workspace_bytes(B, n, d, H.HCW_BF16,
+                                                                       flags, L)),
+                         dtype=torch.uint8, device=dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def step(xin, dyin):
+        if fwd_only:
+            H.hcw_stack_fwd(xin, Ws, Wn, bias, 0, dim_over, flags, y=y, acts=acts, masks=masks,
+                            workspace=ws)
+        else:
+            H.hcw_stack_train_step(xin, Ws, Wn, bias, dyin, 0, dim_over, flags, y=y, acts=acts,
+                                   masks=masks, dx=dx, dW_self=gWs, dW_nbr=gWn, dbias=gb,
+                                   workspace=ws)
+
+    for _ in range(args.warmup):
+        step(x, dy)
+    torch.cuda.synchronize()
+    if H.hcw_sync_status() != H.HCW_OK:
+        raise SystemExit("device error during warm-up")
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    replicas.barrier()
+    torch.cuda.synchronize()
+    launches0 = H.hcw_launch_count()
+    with ClockSampler(local_rank) as clk:
+        for i in range(args.steps):
+            flush.fill_(i & 0xFF)
+            starts[i].record(stream)
+            step(x, dy)
+            ends[i].record(stream)
+        torch.cuda.synchronize()
+    launches = H.hcw_launch_count() - launches0
+    if H.hcw_sync_status() != H.HCW_OK:
+        raise SystemExit("device error during the timed region")
+    ms_local = sum(s.elapsed_time(e) for s, e in zip(starts, ends)) / args.steps
+    ms = replicas.max_over_ranks(ms_local, dev)
+    value = world * tokens / (ms * 1e-3)
+    clocks = clk.summary()
+
+    # roofline of the whole step: the slower of the flops at the bf16 peak and
+    # the algorithmic bytes at the copy bandwidth
+    flops = workload_flops(d, L, causal, fwd_only) * tokens
+    nbytes = workload_bytes(d, L, causal, True, fwd_only) * tokens
+    peak_t = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
+    peak_b = peaks.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+    t_flop, t_byte = flops / (peak_t * 1e12), nbytes / (peak_b * 1e9)
+    sec = ms * 1e-3
+    if t_flop >= t_byte:
+        roof = {"bound": "tensor", "achieved": flops / sec / 1e12, "peak": peak_t,
+                "unit": "TFLOP/s", "frac": t_flop / sec,
+                "peak_source": peak_src + " bf16 burst"}
+    else:
+        roof = {"bound": "hbm", "achieved": nbytes / sec / 1e9, "peak": peak_b, "unit": "GB/s",
+                "frac": t_byte / sec, "peak_source": peak_src + " copy bandwidth"}
+    roof.update({"kernel": "the whole step (%s launches)" % (launches // args.steps),
+                 "traffic": None, "flops_per_step": flops, "algorithmic_bytes_per_step": nbytes})
+
+    # end to end through the public API with host buffers: every step copies
+    # x and dy in from pinned memory and its result out (the weight and bias
+    # gradients, or y for the forward), serially
+    x_h = torch.empty(x.shape, dtype=x.dtype, pin_memory=True)
+    dy_h = torch.empty(dy.shape, dtype=dy.dtype, pin_memory=True)
+    x_h.copy_(x)
+    dy_h.copy_(dy)
+    outs = (y,) if fwd_only else (gWs, gWn, gb)
+    outs_h = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
+    x_d, dy_d = torch.empty_like(x), torch.empty_like(dy)
+    h2d = x_h.numel() * 2 + (0 if fwd_only else dy_h.numel() * 2)
+    d2h = sum(t.numel() * t.element_size() for t in outs_h)
+    e_steps = max(2, min(args.steps, 10))
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for i in range(e_steps):
+        flush.fill_(i & 0xFF)
+        x_d.copy_(x_h, non_blocking=True)
+        if not fwd_only:
+            dy_d.copy_(dy_h, non_blocking=True)
+        step(x_d, dy_d)
+        for th, t in zip(outs_h, outs):
+            th.copy_(t, non_blocking=True)
+    b.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = a.elapsed_time(b) / e_steps
+
+    # the oracle on the host cores, a bounded sample: whole sequences of the
+    # workload for n <= 256, else one layer of one n = 256 sequence (the cost
+    # per token and layer does not depend on n) scaled to the L layers
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        n_s, L_s = (n, L) if n <= 256 else (256, 1)
+        seqs = 1
+        pr = synth.problem(seqs, n_s, d, L=L_s, seed=0, w_std=wstd, x_ids=w.get("x_ids"))
+        _, xo = synth.to_bf16_exact(pr.x)
+        _, wso = synth.to_bf16_exact(pr.W_self)
+        _, wno = synth.to_bf16_exact(pr.W_nbr)
+        _, dyo = synth.to_bf16_exact(pr.dy)
+        t0 = time.perf_counter()
+        _, oa, oz = O.stack_fwd(xo, wso, wno, pr.bias.astype(np.float64), 0, L_s, dim_over,
+                                flags, round_bf16=True)
+        if not fwd_only:
+            O.stack_bwd(oa, oz, dyo, wso, wno, 0, L_s, dim_over, flags, round_bf16=True)
+        secs = time.perf_counter() - t0
+        v = seqs * n_s / secs * L_s / L
+        cpu = {"value": v, "unit": "tokens/s", "cores": O.num_threads(), "kind": "oracle",
+               "sample": "%d sequence(s) of n=%d through %d layer(s), %s, fp64, %.1f s%s"
+                         % (seqs, n_s, L_s, "forward" if fwd_only else "fwd+bwd", secs,
+                            "" if L_s == L else "; scaled to %d layers" % L)}
+
+    replicas.barrier()
+    if rank == 0:
+        print(json.dumps({
+            "metric": "HypercubeMix %s tokens/s at %s bf16; %% of roofline"
+                      % ("forward" if fwd_only else "fwd+bwd", args.workload),
+            "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": args.workload, "n": n, "d": d, "layers": L, "batch": B,
+                       "tokens_per_step_per_gpu": tokens, "causal": causal, "residual": True,
+                       "act": "relu", "bias": True,
+                       "schedule": "fixed dimension 0" if dim_over == 0 else "rotated",
+                       "l2": "flushed before every timed step (256 MiB write, untimed)",
+                       "parallelism": "replicas" if world > 1 else "single",
+                       "launch": "host calls"},
+            "roofline": roof,
+            "cpu_baseline": cpu,
+            "e2e": {"value": world * tokens / (e2e_ms * 1e-3), "unit": "tokens/s",
+                    "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "ms_per_step": e2e_ms,
+                    "copies": "pinned host buffers, serial: inputs in, step, result out"},
+            "gpu_launches": launches,
+            "clocks": clocks,
+        }), flush=True)
+    replicas.finish()
+    return 0
+
+
 def run_kernel_only(args):
     """Launch one kernel kind alone (for profiler captures): the layer
     forward, input-gradient or weight-gradient pass of the workload's shape
@@ -690,16 +911,15 @@ def run_kernel_only(args):
         sWn = torch.empty_like(sWs)
         sb = torch.empty((L, d), dtype=torch.float32, device=dev)
         dxs = torch.empty_like(x)
-        ws = torch.empty(H.hcw_stack_workspace_bytes(B, n, d, H.HCW_BF16, flags, L),
-                         dtype=torch.uint8, device=dev)
-        fws = torch.empty(max(1, H.hcw_stack_fwd_workspace_bytes(B, n, d, H.HCW_BF16, flags, L)),
+        tws = torch.empty(H.hcw_stack_train_step_workspace_bytes(B, n, d, H.HCW_BF16, flags, L),
                           dtype=torch.uint8, device=dev)
 
         def fn():
-            H.hcw_stack_fwd(x, SWs, SWn, Sb, 0, -1, flags, y=y, acts=acts, masks=masks,
-                            workspace=fws)
-            H.hcw_stack_bwd(x, acts, masks, dz, SWs, SWn, 0, -1, flags, dx=dxs, dW_self=sWs,
-                            dW_nbr=sWn, dbias=sb, workspace=ws)
+            # the bench step: one training-step call (forward + input gradient in one
+            # launch, then the weight gradients)
+            H.hcw_stack_train_step(x, SWs, SWn, Sb, dz, 0, -1, flags, y=y, acts=acts,
+                                   masks=masks, dx=dxs, dW_self=sWs, dW_nbr=sWn, dbias=sb,
+                                   workspace=tws)
     elif args.kernel == "fwd":
         fn = lambda: H.hcw_layer_fwd(x, Ws, Wn, bias, layer, -1, flags, y=y, z_save=z)
     elif args.kernel == "dx":
@@ -879,6 +1099,10 @@ def main():
     ap.add_argument("--schedule", choices=tuple(SCHEDULES), default="rot",
                     help="layer schedule of the stack: rot (the workload's rotated stack) or "
                          "hy256 (the near and jump layers of the paper's window-256 hybrid)")
+    ap.add_argument("--workload", choices=("charlm_w256_d512",) + tuple(WORKLOADS_EXTRA),
+                    default="charlm_w256_d512",
+                    help="configuration of the bench line: the metric's char-LM window-256 "
+                         "shape (default), or one of the other configurations")
     ap.add_argument("--stack-kernels", choices=tuple(STACK_KERNELS), default="auto",
                     help="kernel family of the stacked forward and input gradient "
                          "(hcw_set_stack_kernels); auto is the streaming family")
@@ -891,6 +1115,8 @@ def main():
         ap.error("--steps must be at least 1")
     if args.impl == "reference":
         return run_reference(args)
+    if args.workload != WORKLOAD:
+        return run_workload(args)
     return run_ours(args)
 
 

@@ -727,7 +727,8 @@ int layer_bwd_impl(const Shape& sh, int dtype, const void* x, const void* z, con
 size_t stack_g_region(const Shape& sh, unsigned flags, int L) {
     const size_t a = align256(sh.act_bytes);
     const bool keep_g = (flags & HCW_ACT_RELU) && (flags & HCW_RESIDUAL);
-    size_t r = keep_g ? (size_t)L * a : 0;
+    // two g buffers used in turn (see stack_data_bf16)
+    size_t r = keep_g ? 2 * a : 0;
     // schedules with shift layers run layer by layer: two g buffers in turn and
     // the readers' dz of a shift layer
     if (r < 3 * a) r = 3 * a;
@@ -895,7 +896,11 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
     const size_t ab = sh.act_bytes, a256 = align256(ab), wb = (size_t)d * d * 2;
     const size_t mb = mask_bytes(sh);
     auto dz = [&](int l) -> void* { return a.dz + (size_t)l * ab; };
-    auto gbuf = [&](int l) -> void* { return a.ws + (size_t)l * a256; };
+    // Output gradients g in two buffers used in turn: layer l's units write
+    // g_{l-1} over g_{l+1} only for rows whose dz_l chunks are complete, and the
+    // layer-(l+1) units that wrote those chunks had read their g_{l+1} rows (the
+    // residual term) before storing their outputs.
+    auto gbuf = [&](int l) -> void* { return a.ws + (size_t)(l & 1) * a256; };
     auto mask = [&](int l) {
         return reinterpret_cast<const uint32_t*>(static_cast<const uint8_t*>(a.masks) +
                                                  (size_t)l * mb);
@@ -933,6 +938,9 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
                 return HCW_ERR_CUDA;
             T.layer[i] = {s, k, nullptr, nullptr, nullptr, out != nullptr,
                           dzo ? mask(l - 1) : nullptr, dzo != nullptr};
+            // the g buffers written by this launch (not dy, not a previous launch's)
+            if (keep_g && i > 0)
+                T.layer[i].g_discard = static_cast<const __nv_bfloat16*>(res);
         }
         row_unit_params(T.p, sh, BN, a.flags, true);
         if (pair) pair_units(T.p);
@@ -1440,7 +1448,7 @@ int step_fused_launch(const Shape& sh, const void* x, const uint8_t* Ws, const u
                     : nullptr;
     };
     auto dzp = [&](int l) -> void* { return dz + (size_t)l * ab; };
-    auto gbuf = [&](int l) -> void* { return gws + (size_t)l * a256; };
+    auto gbuf = [&](int l) -> void* { return gws + (size_t)(l & 1) * a256; };   // as stack_data_bf16
     auto g = [&](int l) -> const void* {
         if (l == L - 1) return dy;
         return keep_g ? gbuf(l) : dzp(l);
@@ -1476,6 +1484,8 @@ int step_fused_launch(const Shape& sh, const void* x, const uint8_t* Ws, const u
             return HCW_ERR_CUDA;
         T.layer[L + i] = {s, k, nullptr, nullptr, nullptr, out != nullptr,
                           dzo ? mask(l - 1) : nullptr, dzo != nullptr};
+        // the g buffers written by this launch (not dy)
+        if (keep_g && i > 0) T.layer[L + i].g_discard = static_cast<const __nv_bfloat16*>(res);
     }
     row_unit_params(T.p, sh, BN, flags, false);
     pair_units(T.p);

@@ -68,6 +68,11 @@ struct TcLayer {
     // tensor (map 5) instead of the partner rows of map 0 -- a shift layer of
     // Eq. (1), whose partner rows are materialised row-aligned beforehand
     bool pair_rows;
+    // DX of a stacked launch: the residual term (map 3) when it is one of the
+    // launch's own g buffers, [tokens][d] bf16; each epilogue warp discards its
+    // patch's L2 lines once it has read them (nothing reads them again, and
+    // the buffer is written anew two layers later), or null
+    const __nv_bfloat16* g_discard;
 };
 
 // Columns of one epilogue patch (the inner extent of the 32-row residual and

@@ -1195,6 +1195,12 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     if (!okl) {
                         return false;
                     }
+                    // a g row read for the last time: drop its line from L2 without
+                    // writing it back (one 128-byte line per row of the patch)
+                    if (!fwd && ly.g_discard != nullptr && tok_row >= 0 && RB == 128)
+                        asm volatile("discard.global.L2 [%0], 128;" ::"l"(
+                                         ly.g_discard + (size_t)tok_row * p.d + col0)
+                                     : "memory");
                 }
                 const bool write_out = fwd || ly.out;
                 uint32_t gw[SUB][16];
