@@ -414,11 +414,13 @@ size_t hcw_decode_cache_bytes(const int* dims, int layer0, int L, int B, int n, 
  * Gradients (hcw_block_grads, same shapes, fp32) are overwritten, not
  * accumulated; *loss (one fp32 on the device) is overwritten.  The mixing
  * products run on this library's tcgen05 layer kernels, the FFN and head
- * products on cuBLAS (bf16 operands, fp32 accumulation and output).
+ * products on its tcgen05 GEMM (bf16 operands, fp32 accumulation and output;
+ * a weight gradient that splits the tokens adds its partial sums in a fixed
+ * order).
  * Needs n a power of two, d a multiple of 64 and <= 1024, h a multiple of 8,
  * V >= 2.  An id outside [0, V) is read as 0 and reported by hcw_sync_status
- * as HCW_ERR_INVALID_ARG.  Asynchronous on `stream`; calls from several host
- * threads on one device enqueue one at a time (they share its cuBLAS handle).
+ * as HCW_ERR_INVALID_ARG.  Asynchronous on `stream`; no state is shared
+ * between calls other than the workspace each one is given.
  */
 typedef struct {
     const void* E;
@@ -463,6 +465,25 @@ size_t hcw_block_workspace_bytes(int B, int n, int d, int h, int V, int L);
 int hcw_block_step(const int* ids, const hcw_block_params* params, const hcw_block_grads* grads,
                    int B, int n, int d, int h, int V, int L, float* loss, void* workspace,
                    size_t ws_bytes, void* stream);
+
+/*
+ * The block step's plain GEMM on its own (App. A's FFN and head products and
+ * their gradients): row-major C[M][N] = op(A) op(B) in fp32 from bf16
+ * operands with fp32 accumulation, where A is [M][K] (ta = 0) or [K][M]
+ * (ta = 1) and B is [K][N] (tb = 0) or [N][K] (tb = 1), all row-major device
+ * memory.  C is overwritten and must not overlap A, B or the workspace
+ * (HCW_ERR_ALIASING).  M, N, K >= 1 (HCW_ERR_INVALID_ARG).  The workspace (may
+ * be NULL; 16-byte aligned otherwise) holds fp32 partial sums when the K range
+ * is split across CTAs: hcw_gemm_workspace_bytes gives the size that allows
+ * the best split; a smaller one allows fewer splits, NULL none.  Partial sums
+ * are added in split order.  Operands whose rows TMA cannot read (a K-major
+ * row not a multiple of 16 bytes, an MN-major one not a multiple of 64
+ * elements, a pointer not 16-byte aligned) take a plain tiled kernel.
+ * Asynchronous on `stream`.
+ */
+size_t hcw_gemm_workspace_bytes(int M, int N, int K);
+int hcw_gemm_bf16(int M, int N, int K, const void* A, int ta, const void* B, int tb, float* C,
+                  void* workspace, size_t ws_bytes, void* stream);
 
 /* Number of kernels this library has launched in this process (all devices). */
 unsigned long long hcw_launch_count(void);

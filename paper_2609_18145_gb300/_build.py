@@ -21,7 +21,7 @@ LIB = os.path.join(PKG, "libhcw.so")
 BUILD_DIR = os.path.join(PKG, "_build")
 
 SOURCES = ["hcw_api.cu", "hcw_tc.cu", "hcw_res.cu", "hcw_simt.cu", "hcw_decode.cu",
-           "hcw_block.cu"]
+           "hcw_block.cu", "hcw_gemm.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
               "--expt-relaxed-constexpr", "-I", INCLUDE, "-I", CSRC]
@@ -67,7 +67,7 @@ def build(force: bool = False, verbose: bool = False) -> str:
     with cf.ThreadPoolExecutor(len(SOURCES)) as ex:
         objs = list(ex.map(compile_one, SOURCES))
     tmp = LIB + ".%d.tmp" % os.getpid()
-    cmd = [cc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs, "-lcublas", "-lpthread", "-ldl",
+    cmd = [cc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs, "-lpthread", "-ldl",
            "-lrt"]
     if verbose:
         print(" ".join(cmd), flush=True)

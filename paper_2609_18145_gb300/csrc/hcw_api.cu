@@ -1972,15 +1972,17 @@ unsigned long long hcw_launch_count(void) { return g_launches.load(); }
 
 int hcw_sync_status(void* stream) {
     if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return HCW_ERR_CUDA;
-    int word = 0, word_res = 0, word_dec = 0, word_blk = 0;
+    int word = 0, word_res = 0, word_dec = 0, word_blk = 0, word_gemm = 0;
     if (error_word_read_clear(&word) != cudaSuccess ||
         res_error_word_read_clear(&word_res) != cudaSuccess ||
         decode_error_word_read_clear(&word_dec) != cudaSuccess ||
-        block_error_word_read_clear(&word_blk) != cudaSuccess)
+        block_error_word_read_clear(&word_blk) != cudaSuccess ||
+        gemm_error_word_read_clear(&word_gemm) != cudaSuccess)
         return HCW_ERR_CUDA;
     if (!word) word = word_res;
     if (!word) word = word_dec;
     if (!word) word = word_blk;
+    if (!word) word = word_gemm;
     if (word == HCW_ERR_INVALID_ARG) return HCW_ERR_INVALID_ARG;
     if (word) return word == HCW_ERR_TIMEOUT ? HCW_ERR_TIMEOUT : HCW_ERR_CUDA;
     return HCW_OK;

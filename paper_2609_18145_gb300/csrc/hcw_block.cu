@@ -10,16 +10,14 @@
 //   logits = LNf(x) Wh^T + bh,   loss = mean next-symbol cross-entropy
 //
 // The mixing sublayer runs on this library's layer kernels (hcw_layer_fwd /
-// hcw_layer_bwd: tcgen05, bf16); the FFN and head products are plain GEMMs and
-// go to cuBLAS; the row kernels here (embedding, residual add + LayerNorm,
-// bias + ReLU, cross-entropy, their gradients, column sums) are memory-bound
-// and each makes one pass over its rows.  The residual stream x and its
-// gradient are fp32; the GEMM operands are bf16 (h, M(h), g, relu(u), hf,
-// dlogits, bf16(dx), the FFN pre-activation gradient); GEMM outputs are fp32.
-#include <cublas_v2.h>
-
-#include <mutex>
-
+// hcw_layer_bwd: tcgen05, bf16); the FFN and head products run on this
+// library's tcgen05 GEMM (hcw_gemm.cu), whose epilogue also applies the FFN's
+// bias + ReLU and its gradient; the row kernels here (embedding, residual
+// add + LayerNorm, cross-entropy, their gradients, column sums) are
+// memory-bound and each makes one pass over its rows.  The residual stream x
+// and its gradient are fp32; the GEMM operands are bf16 (h, M(h), g, relu(u),
+// hf, dlogits, bf16(dx), the FFN pre-activation gradient); the other GEMM
+// outputs are fp32.
 #include "hcw.h"
 #include "hcw_internal.h"
 #include "hcw_ptx.cuh"
@@ -181,29 +179,6 @@ __global__ void __launch_bounds__(kRowWarps * 32)
     if (lane == 0) stats[row] = make_float2(mean, rstd);
 }
 
-// a = bf16(relu(U + b1[col]))   U: [T][h] fp32 (the GEMM output); eight
-// consecutive elements a thread (h % 8 == 0): two 16-byte loads, one store
-__global__ void bias_relu_kernel(const float* U, const float* b1, __nv_bfloat16* a, size_t total8,
-                                 int h8) {
-    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total8;
-         i += (size_t)gridDim.x * blockDim.x) {
-        const int c = (int)(i % h8) * 8;
-        const float4 u0 = reinterpret_cast<const float4*>(U)[2 * i];
-        const float4 u1 = reinterpret_cast<const float4*>(U)[2 * i + 1];
-        const float4 b0 = *reinterpret_cast<const float4*>(b1 + c);
-        const float4 bb = *reinterpret_cast<const float4*>(b1 + c + 4);
-        const float v[8] = {u0.x + b0.x, u0.y + b0.y, u0.z + b0.z, u0.w + b0.w,
-                            u1.x + bb.x, u1.y + bb.y, u1.z + bb.z, u1.w + bb.w};
-        uint4 o;
-        uint32_t* w = &o.x;
-#pragma unroll
-        for (int e = 0; e < 4; ++e)
-            w[e] = pack_bf16x2(v[2 * e] > 0.f ? v[2 * e] : 0.f,
-                               v[2 * e + 1] > 0.f ? v[2 * e + 1] : 0.f);
-        reinterpret_cast<uint4*>(a)[i] = o;
-    }
-}
-
 // One warp per position r = b n + t: z = logits[r] + bh, target v* =
 // ids[b][t + 1]; loss += (logsumexp(z) - z[v*]) / N; dlog[r][v] =
 // bf16((softmax(z)[v] - [v == v*]) / N).
@@ -227,28 +202,6 @@ __global__ void __launch_bounds__(kRowWarps * 32)
         dlog[(size_t)r * V + v] = __float2bfloat16_rn(p * inv_N);
     }
     if (lane == 0) atomicAdd(loss, (lse - (z[tgt] + bh[tgt])) * inv_N);
-}
-
-// dpre = bf16(da where relu(u) > 0, else 0)   (a = relu(u) holds the mask);
-// eight consecutive elements a thread
-__global__ void relu_bwd_kernel(const float* da, const __nv_bfloat16* a, __nv_bfloat16* dpre,
-                                size_t total8) {
-    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total8;
-         i += (size_t)gridDim.x * blockDim.x) {
-        const float4 d0 = reinterpret_cast<const float4*>(da)[2 * i];
-        const float4 d1 = reinterpret_cast<const float4*>(da)[2 * i + 1];
-        const uint4 m = reinterpret_cast<const uint4*>(a)[i];
-        const float dv[8] = {d0.x, d0.y, d0.z, d0.w, d1.x, d1.y, d1.z, d1.w};
-        const uint32_t mw[4] = {m.x, m.y, m.z, m.w};
-        uint4 o;
-        uint32_t* w = &o.x;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const float2 am = unpack_bf16x2(mw[e]);
-            w[e] = pack_bf16x2(am.x > 0.f ? dv[2 * e] : 0.f, am.y > 0.f ? dv[2 * e + 1] : 0.f);
-        }
-        reinterpret_cast<uint4*>(dpre)[i] = o;
-    }
 }
 
 // out[c] += sum over a tile of kColRows rows of M[r][c] (bf16 M [T][C]; out
@@ -457,37 +410,31 @@ __global__ void pos_bwd_kernel(const float* dx, float* dP, int B, int n, int d) 
 
 namespace {
 
-// Serialises the steps enqueued on one device: they share its cuBLAS handle,
-// whose stream and workspace each step sets.
-std::mutex& device_step_mutex() {
-    static std::mutex mus[64];
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) dev = 0;
-    return mus[dev];
-}
-
-// cuBLAS handle of each device, created on first use and kept for the process
-cublasHandle_t blas_handle() {
-    static std::mutex mu;
-    static cublasHandle_t handles[64] = {};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-    std::lock_guard<std::mutex> lock(mu);
-    if (!handles[dev] && cublasCreate(&handles[dev]) != CUBLAS_STATUS_SUCCESS)
-        handles[dev] = nullptr;
-    return handles[dev];
-}
-
 // Row-major C[M][N] (fp32) = op(A) op(B) with bf16 operands and fp32
 // accumulation; A is [M][K] ([K][M] when ta), B is [K][N] ([N][K] when tb).
-// cuBLAS is column-major, where the row-major C is C^T = op(B)^T op(A)^T.
-bool gemm(cublasHandle_t h, int M, int N, int K, const void* A, bool ta, const void* B, bool tb,
-          float* C) {
-    const float one = 1.f, zero = 0.f;
-    return cublasGemmEx(h, tb ? CUBLAS_OP_T : CUBLAS_OP_N, ta ? CUBLAS_OP_T : CUBLAS_OP_N, N, M,
-                        K, &one, B, CUDA_R_16BF, tb ? K : N, A, CUDA_R_16BF, ta ? M : K, &zero, C,
-                        CUDA_R_32F, N, CUBLAS_COMPUTE_32F,
-                        CUBLAS_GEMM_DEFAULT) == CUBLAS_STATUS_SUCCESS;
+// split_ws holds the partial sums when the GEMM splits K.  HCW_OK after
+// counting its launches, else HCW_ERR_CUDA.
+int gemm(float* split_ws, size_t split_bytes, cudaStream_t st, int M, int N, int K, const void* A,
+         bool ta, const void* B, bool tb, float* C) {
+    int launches = 0;
+    const cudaError_t e =
+        gemm_bf16_f32(M, N, K, A, ta, B, tb, C, split_ws, split_bytes, st, &launches);
+    return count_launch(e, launches);
+}
+
+// The FFN's products with their elementwise step in the epilogue, bf16 out:
+// a = relu(G W1^T + b1) (aux NULL), or dpre = (a > 0) * (dy W2) (bias NULL).
+int gemm_ffn(cudaStream_t st, int M, int N, int K, const void* A, const void* B, bool tb,
+             const float* bias, const __nv_bfloat16* aux, __nv_bfloat16* out) {
+    GemmEpi epi;
+    epi.kind = bias ? EPI_BIAS_RELU : EPI_RELU_GRAD;
+    epi.bias = bias;
+    epi.aux = aux;
+    epi.out = out;
+    int launches = 0;
+    const cudaError_t e =
+        gemm_bf16(M, N, K, A, false, B, tb, nullptr, epi, nullptr, 0, st, &launches);
+    return count_launch(e, launches);
 }
 
 int sms_now() {
@@ -509,13 +456,12 @@ size_t round256(size_t v) { return (v + 255) & ~(size_t)255; }
 //   m, hf [T][d] bf16          mixing output (per layer), head input
 //   U    [T][max(h, V, d)] fp32  every GEMM output with T rows, in turn
 //   dlog [T][V] bf16; dx [T][d] fp32; dxb [T][d] bf16; dpre [T][h] bf16;
-//   dh [T][d] bf16; the mixing backward's own workspace; cuBLAS's workspace
-//   (handed to it every step, so that no call allocates and a CUDA graph can
-//   capture the step)
-constexpr size_t kBlasWs = (size_t)32 << 20;
+//   dh [T][d] bf16; the mixing backward's own workspace; the fp32 partial
+//   sums of the GEMMs that split K (the weight gradients)
+constexpr size_t kSplitWs = (size_t)32 << 20;
 struct BlockWs {
     size_t xs, h1, g, a, st1, st2, stf, m, hf, U, dlog, dx, dxb, dpre, dh, lnp, lws, lws_bytes,
-        blas, total;
+        split, total;
 };
 
 BlockWs block_ws(int B, int n, int d, int h, int V, int L) {
@@ -546,7 +492,7 @@ BlockWs block_ws(int B, int n, int d, int h, int V, int L) {
     w.lnp = take((T + kParamRows - 1) / kParamRows * 2 * (size_t)d * 4);   // LayerNorm partials
     w.lws_bytes = hcw_workspace_bytes(B, n, d, HCW_BF16, HCW_CAUSAL);
     w.lws = take(w.lws_bytes);
-    w.blas = take(kBlasWs);
+    w.split = take(kSplitWs);
     w.total = o;
     return w;
 }
@@ -663,10 +609,7 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
     auto bf = [](const void* q, size_t off) {
         return static_cast<const __nv_bfloat16*>(q) + off;
     };
-    cublasHandle_t hb = blas_handle();
-    if (!hb || cublasSetStream(hb, st) != CUBLAS_STATUS_SUCCESS ||
-        cublasSetWorkspace(hb, ws + w.blas, kBlasWs) != CUBLAS_STATUS_SUCCESS)
-        return HCW_ERR_CUDA;
+    float* split = reinterpret_cast<float*>(ws + w.split);
     const unsigned rows_grid = (unsigned)((T + kRowWarps - 1) / kRowWarps);
     int rc;
 #define HCW_TRY(expr)          \
@@ -675,7 +618,7 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
         if (rc) return rc;     \
     } while (0)
 #define HCW_CU(expr) HCW_TRY((expr) == cudaSuccess ? HCW_OK : HCW_ERR_CUDA)
-#define HCW_BLAS(expr) HCW_TRY((expr) ? HCW_OK : HCW_ERR_CUDA)
+#define HCW_GEMM(...) HCW_TRY(gemm(split, kSplitWs, st, __VA_ARGS__))
     // gradients that are sums (atomics) start at zero; so does the loss
     HCW_CU(cudaMemsetAsync(loss, 0, sizeof(float), st));
     HCW_CU(cudaMemsetAsync(gr.E, 0, (size_t)V * d * 4, st));
@@ -698,11 +641,9 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
         launch_ln_fwd(st, X(l), m, nullptr, nullptr, XM(l), p.ln2_g + (size_t)l * d, p.ln2_b + (size_t)l * d, G(l),
             S2(l), T, d);
         HCW_TRY(ok_launch());
-        HCW_BLAS(gemm(hb, T, h, d, G(l), false, bf(p.W1, (size_t)l * h * d), true, U));
-        bias_relu_kernel<<<elem_grid(Th / 8), 256, 0, st>>>(U, p.b1 + (size_t)l * h, A(l), Th / 8,
-                                                            h / 8);
-        HCW_TRY(ok_launch());
-        HCW_BLAS(gemm(hb, T, d, h, A(l), false, bf(p.W2, (size_t)l * d * h), true, U));
+        HCW_TRY(gemm_ffn(st, T, h, d, G(l), bf(p.W1, (size_t)l * h * d), true,
+                         p.b1 + (size_t)l * h, nullptr, A(l)));   // a = relu(g W1^T + b1)
+        HCW_GEMM(T, d, h, A(l), false, bf(p.W2, (size_t)l * d * h), true, U);
         const bool top = l + 1 == L;
         launch_ln_fwd(st, XM(l), nullptr, U, p.b2 + (size_t)l * d, X(l + 1),
             top ? p.lnf_g : p.ln1_g + (size_t)(l + 1) * d,
@@ -710,33 +651,32 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
             T, d);
         HCW_TRY(ok_launch());
     }
-    HCW_BLAS(gemm(hb, T, V, d, hf, false, p.Wh, true, U));
+    HCW_GEMM(T, V, d, hf, false, p.Wh, true, U);
     ce_kernel<<<rows_grid, kRowWarps * 32, 0, st>>>(U, p.bh, ids, dlog, loss, B, n, V, 1.f / T);
     HCW_TRY(ok_launch());
 
     // ----------------------------------------------------------- backward
     const unsigned gridT = (unsigned)((T + kColRows - 1) / kColRows);
-    HCW_BLAS(gemm(hb, V, d, T, dlog, true, hf, false, gr.Wh));   // dWh = dlog^T hf
+    HCW_GEMM(V, d, T, dlog, true, hf, false, gr.Wh);   // dWh = dlog^T hf
     colsum_kernel<<<dim3((V + 255) / 256, gridT), 256, 0, st>>>(dlog, gr.bh, T, V);
     HCW_TRY(ok_launch());
-    HCW_BLAS(gemm(hb, T, d, V, dlog, false, p.Wh, false, U));    // dhf = dlog Wh
+    HCW_GEMM(T, d, V, dlog, false, p.Wh, false, U);    // dhf = dlog Wh
     int nk = launch_ln_bwd(st, U, nullptr, X(L), sf, p.lnf_g, nullptr, dx, dxb, lnp, gr.lnf_g,
                            gr.lnf_b, T, d);
     HCW_TRY(count_launch(cudaGetLastError(), nk));
     for (int l = L - 1; l >= 0; --l) {
         // FFN sublayer: dxb = bf16(dx) is the gradient of its output
-        HCW_BLAS(gemm(hb, d, h, T, dxb, true, A(l), false, gr.W2 + (size_t)l * d * h));
+        HCW_GEMM(d, h, T, dxb, true, A(l), false, gr.W2 + (size_t)l * d * h);
         colsum_kernel<<<dim3((d + 255) / 256, gridT), 256, 0, st>>>(dxb, gr.b2 + (size_t)l * d, T,
                                                                      d);
         HCW_TRY(ok_launch());
-        HCW_BLAS(gemm(hb, T, h, d, dxb, false, bf(p.W2, (size_t)l * d * h), false, U));   // da
-        relu_bwd_kernel<<<elem_grid(Th / 8), 256, 0, st>>>(U, A(l), dpre, Th / 8);
-        HCW_TRY(ok_launch());
+        HCW_TRY(gemm_ffn(st, T, h, d, dxb, bf(p.W2, (size_t)l * d * h), false, nullptr, A(l),
+                         dpre));   // dpre = (a > 0) * (dxb W2)
         colsum_kernel<<<dim3((h + 255) / 256, gridT), 256, 0, st>>>(dpre, gr.b1 + (size_t)l * h, T,
                                                                      h);
         HCW_TRY(ok_launch());
-        HCW_BLAS(gemm(hb, h, d, T, dpre, true, G(l), false, gr.W1 + (size_t)l * h * d));
-        HCW_BLAS(gemm(hb, T, d, h, dpre, false, bf(p.W1, (size_t)l * h * d), false, U));  // dg
+        HCW_GEMM(h, d, T, dpre, true, G(l), false, gr.W1 + (size_t)l * h * d);
+        HCW_GEMM(T, d, h, dpre, false, bf(p.W1, (size_t)l * h * d), false, U);  // dg
         nk = launch_ln_bwd(st, U, nullptr, XM(l), S2(l), p.ln2_g + (size_t)l * d, dx, dx, dxb, lnp,
                            gr.ln2_g + (size_t)l * d, gr.ln2_b + (size_t)l * d, T, d);
         HCW_TRY(count_launch(cudaGetLastError(), nk));
@@ -755,7 +695,7 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
     return ok_launch();
 #undef HCW_TRY
 #undef HCW_CU
-#undef HCW_BLAS
+#undef HCW_GEMM
 }
 
 }  // namespace
@@ -803,7 +743,6 @@ int hcw_block_step(const int* ids, const hcw_block_params* params, const hcw_blo
         return HCW_ERR_ALIGNMENT;
     const size_t need = block_ws(B, n, d, h, V, L).total;
     if (!workspace || ws_bytes < need || !a16(workspace)) return HCW_ERR_WORKSPACE;
-    std::lock_guard<std::mutex> lock(device_step_mutex());
     return block_step(ids, p, g, B, n, d, h, V, L, loss, static_cast<uint8_t*>(workspace),
                       (cudaStream_t)stream);
 }

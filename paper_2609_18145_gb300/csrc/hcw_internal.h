@@ -219,6 +219,31 @@ cudaError_t launch_decode(const DecodeLaunch& p, cudaStream_t st);
 // Read the decode kernel's error word and reset it to 0 (synchronous).
 cudaError_t decode_error_word_read_clear(int* word);
 
+// ---- Plain GEMMs of the character-LM block (hcw_gemm.cu) ----
+// Row-major C[M][N] (fp32) = op(A) op(B), bf16 operands, fp32 accumulation;
+// A is [M][K] ([K][M] when ta), B is [K][N] ([N][K] when tb).  split_ws
+// (split_ws_bytes, 16-byte aligned, may be NULL) holds the fp32 partial sums
+// of a K split; *launches receives the kernels enqueued (1 or 2).
+cudaError_t gemm_bf16_f32(int M, int N, int K, const void* A, bool ta, const void* B, bool tb,
+                          float* C, float* split_ws, size_t split_ws_bytes, cudaStream_t st,
+                          int* launches);
+// Epilogues of the GEMM: fp32 C; out = bf16(relu(C + bias[col])); or
+// out = bf16(aux[row][col] > 0 ? C : 0).  out and aux are [M][N] bf16.
+enum GemmEpiKind { EPI_F32 = 0, EPI_BIAS_RELU = 1, EPI_RELU_GRAD = 2 };
+struct GemmEpi {
+    int kind;
+    const float* bias;
+    const __nv_bfloat16* aux;
+    __nv_bfloat16* out;
+};
+// gemm_bf16_f32 with an epilogue (C unused unless epi.kind is EPI_F32; only
+// fp32 output splits K).
+cudaError_t gemm_bf16(int M, int N, int K, const void* A, bool ta, const void* B, bool tb,
+                      float* C, const GemmEpi& epi, float* split_ws, size_t split_ws_bytes,
+                      cudaStream_t st, int* launches);
+// Read the GEMM kernel's error word and reset it to 0 (synchronous).
+cudaError_t gemm_error_word_read_clear(int* word);
+
 // ---- Character-LM block (hcw_block.cu) ----
 // Read the block kernels' error word and reset it to 0 (synchronous).
 cudaError_t block_error_word_read_clear(int* word);

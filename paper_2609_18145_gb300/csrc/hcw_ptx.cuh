@@ -13,7 +13,8 @@ namespace hcw {
 // Error word (one per device and translation unit): kernels that give up on a
 // bounded wait write a non-zero code here; hcw_sync_status reads and clears
 // the word of every translation unit that includes this header (hcw_tc.cu,
-// hcw_res.cu, hcw_decode.cu), each through its own read-and-clear function.
+// hcw_res.cu, hcw_decode.cu, hcw_block.cu, hcw_gemm.cu), each through its own
+// read-and-clear function.
 namespace {
 __device__ int g_error_word = 0;
 }

@@ -87,6 +87,8 @@ _SIGNATURES = {
     "hcw_decode_cache_bytes": ([_P, _I, _I, _I, _I, _I], _SZ),
     "hcw_block_workspace_bytes": ([_I, _I, _I, _I, _I, _I], _SZ),
     "hcw_block_step": ([_P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _SZ, _P], _I),
+    "hcw_gemm_workspace_bytes": ([_I, _I, _I], _SZ),
+    "hcw_gemm_bf16": ([_I, _I, _I, _P, _I, _P, _I, _P, _P, _SZ, _P], _I),
     "hcw_set_stack_kernels": ([_I], _I),
     "hcw_stack_kernels_used": ([_I, _I, _I, _I], _I),
     "hcw_sync_status": ([_P], _I),
@@ -321,6 +323,33 @@ def hcw_block_step(ids, params: dict, grads: dict | None = None, loss=None, work
                                 _ptr(loss), _ptr(ws), ws.numel(), _stream(stream)),
            "hcw_block_step")
     return loss, grads
+
+
+def hcw_gemm_workspace_bytes(M: int, N: int, K: int) -> int:
+    return int(lib().hcw_gemm_workspace_bytes(M, N, K))
+
+
+def hcw_gemm_bf16(A, B, ta: bool = False, tb: bool = False, C=None, workspace=None,
+                  split: bool = True, stream=None):
+    """fp32 C = op(A) op(B) from bf16 A ([M, K], or [K, M] with ta) and B
+    ([K, N], or [N, K] with tb).  split=False passes no workspace (no K
+    split).  Returns C [M, N]."""
+    _dev(A, B, C, workspace)
+    if A.dtype != torch.bfloat16 or B.dtype != torch.bfloat16 or A.dim() != 2 or B.dim() != 2:
+        raise ValueError("hcw_gemm_bf16: A and B must be 2-D bf16 tensors")
+    M, K = (A.shape[1], A.shape[0]) if ta else (A.shape[0], A.shape[1])
+    Kb, N = (B.shape[1], B.shape[0]) if tb else (B.shape[0], B.shape[1])
+    if Kb != K:
+        raise ValueError("hcw_gemm_bf16: inner sizes differ (%d, %d)" % (K, Kb))
+    C = torch.empty(M, N, dtype=torch.float32, device=A.device) if C is None else C
+    if split:
+        ws = _workspace(hcw_gemm_workspace_bytes(M, N, K), A.device, workspace)
+        wp, wn = _ptr(ws), ws.numel()
+    else:
+        wp, wn = None, 0
+    _check(lib().hcw_gemm_bf16(M, N, K, _ptr(A), int(bool(ta)), _ptr(B), int(bool(tb)), _ptr(C),
+                               wp, wn, _stream(stream)), "hcw_gemm_bf16")
+    return C
 
 
 def hcw_set_stack_kernels(mode: int) -> int:

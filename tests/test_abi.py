@@ -343,3 +343,36 @@ def test_block_workspace_size_and_validation(hcw):
     assert step(P=Pbad) == hcw.HCW_ERR_ALIGNMENT
     assert step(ws=ws_b - 256) == hcw.HCW_ERR_WORKSPACE
     assert hcw.hcw_launch_count() == before
+
+
+def test_gemm_validation_codes(hcw):
+    """hcw_gemm_bf16 rejects bad sizes, flags, a misaligned workspace and a C
+    that overlaps an operand or the workspace before anything launches."""
+    P = ctypes.c_void_p
+    L = hcw.lib()
+    M, N, K = 256, 512, 128
+    A, B, C, W = (0x1000000 * k for k in range(1, 5))
+
+    def call(M=M, N=N, K=K, a=A, ta=0, b=B, tb=1, c=C, w=None, wsb=0):
+        return L.hcw_gemm_bf16(M, N, K, P(a), ta, P(b), tb, P(c), P(w) if w else None, wsb,
+                               None)
+
+    assert call(M=0) == hcw.HCW_ERR_INVALID_ARG
+    assert call(K=-1) == hcw.HCW_ERR_INVALID_ARG
+    assert call(a=0) == hcw.HCW_ERR_INVALID_ARG
+    assert call(c=0) == hcw.HCW_ERR_INVALID_ARG
+    assert call(ta=2) == hcw.HCW_ERR_INVALID_ARG
+    assert call(w=W + 8, wsb=1 << 20) == hcw.HCW_ERR_ALIGNMENT
+    assert call(c=A + M * K * 2 - 4) == hcw.HCW_ERR_ALIASING      # C's start inside A
+    assert call(c=B - 64) == hcw.HCW_ERR_ALIASING                 # C's end inside B
+    assert call(w=C + 256, wsb=1 << 20) == hcw.HCW_ERR_ALIASING   # workspace inside C
+
+
+def test_gemm_workspace_sizes(hcw):
+    """A weight-gradient shape (few output tiles, long K) asks for a K split;
+    a short K or a wide output asks for none."""
+    s = hcw.hcw_gemm_workspace_bytes(512, 1024, 16384)
+    assert s > 0 and s % (512 * 1024 * 4) == 0
+    assert hcw.hcw_gemm_workspace_bytes(16384, 1024, 512) == 0
+    assert hcw.hcw_gemm_workspace_bytes(256, 256, 128) == 0
+    assert hcw.hcw_gemm_workspace_bytes(0, 256, 128) == 0

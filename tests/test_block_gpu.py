@@ -131,8 +131,8 @@ def test_an_id_outside_the_vocabulary_is_reported(H):
 def test_full_size_batch_is_the_weighted_sum_of_its_parts(H):
     """Window 256, d = 512, h = 1024, V = 256, 16 layers, B = 64 (the metric's
     shape): sequences are independent, so the batch's loss and gradients are
-    the size-weighted sums of those of 32 two-sequence steps; and the first
-    two sequences match the oracle."""
+    the size-weighted sums of those of 32 two-sequence steps (to rounding);
+    and the first two sequences match the oracle."""
     B, n, d, h, V, L = 64, 256, 512, 1024, 256, 16
     pr = synth.block_problem(B, n, d, h, V, L, seed=9)
     ids, params, exact = device_problem(pr)
@@ -154,9 +154,11 @@ def test_full_size_batch_is_the_weighted_sum_of_its_parts(H):
     assert H.hcw_sync_status() == H.HCW_OK
     assert np.isfinite(float(loss.item()))
     assert abs(float(loss.item()) - part_loss) <= 1e-4 * abs(part_loss)
-    for f in OB_FIELDS:
-        a, b = grads[f].cpu().numpy(), part[f].cpu().numpy()
-        assert rel(a, b) <= 1e-2, f
+    # the batch and its parts are both device results, but the GEMMs split K
+    # differently at 16,384 and at 512 tokens, so their sums round apart and
+    # the rounding-flip walk of tol_grad applies between them too
+    check_grads({f: grads[f].cpu().numpy().astype(np.float64) for f in OB_FIELDS},
+                {f: part[f].cpu().numpy().astype(np.float64) for f in OB_FIELDS}, L)
     sub = synth.block_problem(B, n, d, h, V, L, seed=9)
     sub.ids = np.asarray(pr.ids)[:2]
     ref_loss, ref = OB.step(as_problem(sub, exact), round_bf16=True)
