@@ -18,6 +18,8 @@
 // and its gradient are fp32; the GEMM operands are bf16 (h, M(h), g, relu(u),
 // hf, dlogits, bf16(dx), the FFN pre-activation gradient); the other GEMM
 // outputs are fp32.
+#include <mutex>
+
 #include "hcw.h"
 #include "hcw_internal.h"
 #include "hcw_ptx.cuh"
@@ -28,6 +30,10 @@ namespace {
 
 constexpr float kLnEps = 1e-5f;
 constexpr int kRowWarps = 8;   // rows (one warp each) per CTA of the row kernels
+// CTAs of the fused LayerNorm backward at most (rows of its partial sums), and
+// its shared memory at the largest d (1024) with three sums
+constexpr int kLnBwdMaxGrid = 1024;
+constexpr size_t kLnBwdMaxSmem = (size_t)kRowWarps * 3 * 1024 * sizeof(float);
 
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
@@ -219,166 +225,168 @@ __global__ void colsum_kernel(const __nv_bfloat16* M, float* out, int T, int C) 
     atomicAdd(out + c, s);
 }
 
-// LayerNorm backward, one warp per row: with xhat = (x - mean) rstd and
-// dxhat = dy g,
+// W consecutive features at element e (W = 2 or 4; e a multiple of W).
+template <int W>
+__device__ __forceinline__ void ldv(const float* p, size_t e, float (&v)[W]) {
+    if constexpr (W == 4) {
+        const float4 t = *reinterpret_cast<const float4*>(p + e);
+        v[0] = t.x, v[1] = t.y, v[2] = t.z, v[3] = t.w;
+    } else {
+        const float2 t = *reinterpret_cast<const float2*>(p + e);
+        v[0] = t.x, v[1] = t.y;
+    }
+}
+template <int W>
+__device__ __forceinline__ void ldv(const __nv_bfloat16* p, size_t e, float (&v)[W]) {
+    if constexpr (W == 4) {
+        const uint2 u = *reinterpret_cast<const uint2*>(p + e);
+        const float2 a = unpack_bf16x2(u.x), b = unpack_bf16x2(u.y);
+        v[0] = a.x, v[1] = a.y, v[2] = b.x, v[3] = b.y;
+    } else {
+        const float2 a = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(p + e));
+        v[0] = a.x, v[1] = a.y;
+    }
+}
+template <int W>
+__device__ __forceinline__ void stv(float* p, size_t e, const float (&v)[W]) {
+    if constexpr (W == 4)
+        *reinterpret_cast<float4*>(p + e) = make_float4(v[0], v[1], v[2], v[3]);
+    else
+        *reinterpret_cast<float2*>(p + e) = make_float2(v[0], v[1]);
+}
+template <int W>
+__device__ __forceinline__ void stv(__nv_bfloat16* p, size_t e, const float (&v)[W]) {
+    if constexpr (W == 4)
+        *reinterpret_cast<uint2*>(p + e) =
+            make_uint2(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]));
+    else
+        *reinterpret_cast<uint32_t*>(p + e) = pack_bf16x2(v[0], v[1]);
+}
+
+// LayerNorm backward and its parameter sums in one pass over the rows.  Per
+// row (one warp), with xhat = (x - mean) rstd and dxhat = dy g,
 //   dx = rstd (dxhat - mean(dxhat) - xhat mean(dxhat xhat))  (+ dres)
-// written to dx_out (fp32) and, when dxb is given, as bf16.  dy is fp32 (dyf)
-// or bf16 (dyb).  Every load of the row comes before any store: dres and
-// dx_out may be the same buffer (the gradient updated in place), and a load
-// placed after a store could not be moved ahead of it.  NV >= d / 32.
-template <int NV>
+// written to dx_out (fp32) and, when dxb is given, as bf16; dy is fp32 or
+// bf16.  Every load of a row comes before its stores: dres and dx_out may be
+// the same buffer (the gradient updated in place).  Lane l holds features
+// W (32 i + l) .. + W - 1, i < d / (32 W) <= NV.  Warps take rows
+// blockIdx.x * kRowWarps + warp, then every gridDim.x * kRowWarps further on,
+// summing per feature dy xhat (the scale gradient), dy (the shift gradient)
+// and, with ncol = 3, bf16(dx) (the column sums of dxb); the CTA adds its
+// warps' sums in warp order into row blockIdx.x of part [gridDim.x][ncol d],
+// which ln_part_reduce_kernel adds up in row order.
+template <int NV, int W, typename DY>
 __global__ void __launch_bounds__(kRowWarps * 32)
-    ln_bwd_kernel(const float* dyf, const __nv_bfloat16* dyb, const float* x, const float2* stats,
-                  const float* g, const float* dres, float* dx_out, __nv_bfloat16* dxb, int T,
-                  int d) {
-    const int lane = threadIdx.x & 31;
-    const int row = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
-    if (row >= T) return;
-    const int nv = d >> 5;
-    const size_t base = (size_t)row * d;
-    const float2 st = stats[row];
-    float xh[NV], dh[NV], rv[NV];
-    float s1 = 0.f, s2 = 0.f;
-#pragma unroll
-    for (int i = 0; i < NV; ++i) {
-        if (i < nv) {
-            const int c = i * 32 + lane;
-            rv[i] = dres ? dres[base + c] : 0.f;
-            const float dy = dyf ? dyf[base + c] : __bfloat162float(dyb[base + c]);
-            xh[i] = (x[base + c] - st.x) * st.y;
-            dh[i] = dy * g[c];
-            s1 += dh[i];
-            s2 += dh[i] * xh[i];
-        }
-    }
-    const float m1 = warp_sum(s1) / d, m2 = warp_sum(s2) / d;
-#pragma unroll
-    for (int i = 0; i < NV; ++i) {
-        if (i < nv) {
-            const int c = i * 32 + lane;
-            const float v = st.y * (dh[i] - m1 - xh[i] * m2) + rv[i];
-            dx_out[base + c] = v;
-            if (dxb) dxb[base + c] = __float2bfloat16_rn(v);
-        }
-    }
-}
-
-// LayerNorm scale and shift gradients: dgam[c] += sum of dy xhat, dbet[c] +=
-// sum of dy over a tile of kColRows rows (xhat recomputed from x and the row
-// statistics); grid (ceil(d / 256), ceil(T / kColRows)), a thread per column,
-// dgam and dbet zeroed before the launch
-__global__ void ln_param_kernel(const float* dyf, const __nv_bfloat16* dyb, const float* x,
-                                const float2* stats, int T, int d, float* dgam, float* dbet) {
-    const int c = blockIdx.x * blockDim.x + threadIdx.x;
-    if (c >= d) return;
-    const int r0 = blockIdx.y * kColRows;
-    const int r1 = min(T, r0 + kColRows);
-    float sg = 0.f, sb = 0.f;
-#pragma unroll 8
-    for (int r = r0; r < r1; ++r) {
-        const size_t e = (size_t)r * d + c;
-        const float dy = dyf ? dyf[e] : __bfloat162float(dyb[e]);
-        const float2 st = stats[r];
-        sg += dy * (x[e] - st.x) * st.y;
-        sb += dy;
-    }
-    atomicAdd(dgam + c, sg);
-    atomicAdd(dbet + c, sb);
-}
-
-// ln_bwd_kernel for d a multiple of 128 (four features a lane and access).
-template <int NV4, typename DY>
-__global__ void __launch_bounds__(kRowWarps * 32)
-    ln_bwd4_kernel(const DY* dy, const float* x, const float2* stats, const float* g,
-                   const float* dres, float* dx_out, __nv_bfloat16* dxb, int T, int d) {
-    const int lane = threadIdx.x & 31;
-    const int row = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
-    if (row >= T) return;
-    const int nv = d >> 7;
-    const size_t base = (size_t)row * d;
-    const float2 st = stats[row];
-    float4 xh[NV4], dh[NV4], rv[NV4];
-    float s1 = 0.f, s2 = 0.f;
-#pragma unroll
-    for (int i = 0; i < NV4; ++i) {
-        if (i < nv) {
-            const int c = (i * 32 + lane) * 4;
-            rv[i] = dres ? ld4(dres, base + c) : make_float4(0.f, 0.f, 0.f, 0.f);
-            const float4 y = ld4(dy, base + c), xx = ld4(x, base + c), gg = ld4(g, (size_t)c);
-            xh[i] = make_float4((xx.x - st.x) * st.y, (xx.y - st.x) * st.y,
-                                (xx.z - st.x) * st.y, (xx.w - st.x) * st.y);
-            dh[i] = make_float4(y.x * gg.x, y.y * gg.y, y.z * gg.z, y.w * gg.w);
-            s1 += sum4(dh[i]);
-            s2 += dh[i].x * xh[i].x + dh[i].y * xh[i].y + dh[i].z * xh[i].z + dh[i].w * xh[i].w;
-        }
-    }
-    const float m1 = warp_sum(s1) / d, m2 = warp_sum(s2) / d;
-#pragma unroll
-    for (int i = 0; i < NV4; ++i) {
-        if (i < nv) {
-            const int c = (i * 32 + lane) * 4;
-            const float4 v = make_float4(st.y * (dh[i].x - m1 - xh[i].x * m2) + rv[i].x,
-                                         st.y * (dh[i].y - m1 - xh[i].y * m2) + rv[i].y,
-                                         st.y * (dh[i].z - m1 - xh[i].z * m2) + rv[i].z,
-                                         st.y * (dh[i].w - m1 - xh[i].w * m2) + rv[i].w);
-            st4(dx_out, base + c, v);
-            if (dxb) st4(dxb, base + c, v);
-        }
-    }
-}
-
-// ln_param_kernel with four columns a thread (d a multiple of 4) over tiles
-// of kParamRows rows: grid (ceil(d / 512), ceil(T / kParamRows)), 128
-// threads.  Each tile writes its sums as one row of part [tiles][2 d] (dy xhat,
-// then dy); ln_param_reduce_kernel adds the rows up.  No atomics: with every
-// tile adding into the same 2 d addresses they would queue in L2.
-constexpr int kParamRows = 16;
-template <typename DY>
-__global__ void ln_param4_kernel(const DY* dy, const float* x, const float2* stats, int T, int d,
-                                 float* part) {
-    const int c = (blockIdx.x * blockDim.x + threadIdx.x) * 4;
-    if (c >= d) return;
-    const int r0 = blockIdx.y * kParamRows;
-    const int r1 = min(T, r0 + kParamRows);
-    float4 sg = make_float4(0.f, 0.f, 0.f, 0.f), sb = sg;
-#pragma unroll 8
-    for (int r = r0; r < r1; ++r) {
-        const size_t e = (size_t)r * d + c;
-        const float4 y = ld4(dy, e), xx = ld4(x, e);
-        const float2 st = stats[r];
-        sg.x += y.x * (xx.x - st.x) * st.y;
-        sg.y += y.y * (xx.y - st.x) * st.y;
-        sg.z += y.z * (xx.z - st.x) * st.y;
-        sg.w += y.w * (xx.w - st.x) * st.y;
-        sb = add4(sb, y);
-    }
-    float* row = part + (size_t)blockIdx.y * 2 * d;
-    st4(row, (size_t)c, sg);
-    st4(row, (size_t)d + c, sb);
-}
-
-// dgam[c] = sum over the nblk rows of part [nblk][2 d] of column c, dbet[c] of
-// column d + c.  A CTA per 32 columns: warp w adds rows w, w + 8, ... (each
-// warp load one 128-byte row piece), then the eight warp sums meet in shared
-// memory in a fixed order.
-__global__ void __launch_bounds__(256) ln_param_reduce_kernel(const float* part, int nblk, int d,
-                                                              float* dgam, float* dbet) {
-    __shared__ float acc[8][32];
+    ln_bwd_fused_kernel(const DY* dy, const float* x, const float2* stats, const float* g,
+                        const float* dres, float* dx_out, __nv_bfloat16* dxb, int T, int d,
+                        int ncol, float* part) {
+    extern __shared__ float red[];   // [kRowWarps][ncol d]: each warp's sums, then the CTA's
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int c = blockIdx.x * 32 + lane;
-    float s = 0.f;
-    if (c < 2 * d)
-        for (int b = warp; b < nblk; b += 8) s += part[(size_t)b * 2 * d + c];
-    acc[warp][lane] = s;
+    const int nv = d / (32 * W);
+    const int width = ncol * d;
+    float* mine = red + (size_t)warp * width;   // this warp's sums, kept in shared memory
+    for (int c = lane; c < width; c += 32) mine[c] = 0.f;
+    __syncwarp();
+    for (int row = blockIdx.x * kRowWarps + warp; row < T; row += gridDim.x * kRowWarps) {
+        const size_t base = (size_t)row * d;
+        const float2 st = stats[row];
+        float xh[NV][W], dh[NV][W], rv[NV][W];
+        float s1 = 0.f, s2 = 0.f;
+#pragma unroll
+        for (int i = 0; i < NV; ++i) {
+            if (i < nv) {
+                const int c = (i * 32 + lane) * W;
+                float xx[W], gg[W], yv[W], sg[W], sb[W];
+                if (dres) {
+                    ldv<W>(dres, base + c, rv[i]);
+                } else {
+#pragma unroll
+                    for (int j = 0; j < W; ++j) rv[i][j] = 0.f;
+                }
+                ldv<W>(dy, base + c, yv);
+                ldv<W>(x, base + c, xx);
+                ldv<W>(g, (size_t)c, gg);
+                ldv<W>(mine, (size_t)c, sg);
+                ldv<W>(mine, (size_t)d + c, sb);
+#pragma unroll
+                for (int j = 0; j < W; ++j) {
+                    xh[i][j] = (xx[j] - st.x) * st.y;
+                    dh[i][j] = yv[j] * gg[j];
+                    s1 += dh[i][j];
+                    s2 += dh[i][j] * xh[i][j];
+                    sg[j] += yv[j] * xh[i][j];
+                    sb[j] += yv[j];
+                }
+                stv<W>(mine, (size_t)c, sg);
+                stv<W>(mine, (size_t)d + c, sb);
+            }
+        }
+        const float m1 = warp_sum(s1) / d, m2 = warp_sum(s2) / d;
+#pragma unroll
+        for (int i = 0; i < NV; ++i) {
+            if (i < nv) {
+                const int c = (i * 32 + lane) * W;
+                float v[W];
+#pragma unroll
+                for (int j = 0; j < W; ++j) v[j] = st.y * (dh[i][j] - m1 - xh[i][j] * m2) + rv[i][j];
+                stv<W>(dx_out, base + c, v);
+                if (dxb) {
+                    stv<W>(dxb, base + c, v);
+                    if (ncol == 3) {
+                        float sc[W];
+                        ldv<W>(mine, (size_t)2 * d + c, sc);
+#pragma unroll
+                        for (int j = 0; j < W; ++j)
+                            sc[j] += __bfloat162float(__float2bfloat16_rn(v[j]));
+                        stv<W>(mine, (size_t)2 * d + c, sc);
+                    }
+                }
+            }
+        }
+    }
     __syncthreads();
-    if (warp == 0 && c < 2 * d) {
+    for (int c = threadIdx.x; c < width; c += blockDim.x) {
         float t = 0.f;
 #pragma unroll
-        for (int w = 0; w < 8; ++w) t += acc[w][lane];
-        if (c < d)
-            dgam[c] = t;
-        else
-            dbet[c - d] = t;
+        for (int w = 0; w < kRowWarps; ++w) t += red[(size_t)w * width + c];
+        part[(size_t)blockIdx.x * width + c] = t;
+    }
+}
+
+// Sum of the nblk rows of part [nblk][ncol d] per column, in row order:
+// columns [0, d) -> dgam, [d, 2d) -> dbet, [2d, 3d) -> dcol.  A CTA of 32
+// warps per 32 columns, a column a lane: warp w adds rows w, w + 32, ...
+// (sixteen loads in flight), then the 32 warp sums meet in shared memory in
+// warp order.
+constexpr int kReduceWarps = 32;
+__global__ void __launch_bounds__(kReduceWarps * 32)
+    ln_part_reduce_kernel(const float* part, int nblk, int d, int ncol, float* dgam, float* dbet,
+                          float* dcol) {
+    __shared__ float acc[kReduceWarps][33];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int width = ncol * d;
+    const int c = blockIdx.x * 32 + lane;
+    float s = 0.f;
+    if (c < width) {
+        for (int b0 = warp; b0 < nblk; b0 += 16 * kReduceWarps) {
+            float v[16];
+#pragma unroll
+            for (int k = 0; k < 16; ++k) {
+                const int b = b0 + k * kReduceWarps;
+                v[k] = b < nblk ? part[(size_t)b * width + c] : 0.f;
+            }
+#pragma unroll
+            for (int k = 0; k < 16; ++k) s += v[k];
+        }
+    }
+    acc[warp][lane] = s;
+    __syncthreads();
+    if (warp == 0 && c < width) {
+        float t = 0.f;
+#pragma unroll
+        for (int w = 0; w < kReduceWarps; ++w) t += acc[w][lane];
+        const int seg = c / d, cc = c - seg * d;
+        (seg == 0 ? dgam : (seg == 1 ? dbet : dcol))[cc] = t;
     }
 }
 
@@ -489,7 +497,7 @@ BlockWs block_ws(int B, int n, int d, int h, int V, int L) {
     w.dxb = take(T * d * 2);
     w.dpre = take(T * h * 2);
     w.dh = take(T * d * 2);
-    w.lnp = take((T + kParamRows - 1) / kParamRows * 2 * (size_t)d * 4);   // LayerNorm partials
+    w.lnp = take((size_t)kLnBwdMaxGrid * 3 * d * 4);   // LayerNorm backward partial sums
     w.lws_bytes = hcw_workspace_bytes(B, n, d, HCW_BF16, HCW_CAUSAL);
     w.lws = take(w.lws_bytes);
     w.split = take(kSplitWs);
@@ -535,52 +543,109 @@ void launch_ln_fwd(cudaStream_t st, const float* x_in, const __nv_bfloat16* add1
         ln_fwd4_kernel<8><<<grid, blk, 0, st>>>(x_in, add1, add2, badd, x_out, g, b, y, stats, T, d);
 }
 
-template <typename DY>
-void launch_ln_bwd4(cudaStream_t st, const DY* dy, const float* x, const float2* stats,
-                    const float* g, const float* dres, float* dx_out, __nv_bfloat16* dxb,
-                    float* part, float* dgam, float* dbet, int T, int d) {
-    const dim3 grid((T + kRowWarps - 1) / kRowWarps), blk(kRowWarps * 32);
-    const int v4 = d / 128;
-    if (v4 <= 1)
-        ln_bwd4_kernel<1, DY><<<grid, blk, 0, st>>>(dy, x, stats, g, dres, dx_out, dxb, T, d);
-    else if (v4 <= 2)
-        ln_bwd4_kernel<2, DY><<<grid, blk, 0, st>>>(dy, x, stats, g, dres, dx_out, dxb, T, d);
-    else if (v4 <= 4)
-        ln_bwd4_kernel<4, DY><<<grid, blk, 0, st>>>(dy, x, stats, g, dres, dx_out, dxb, T, d);
-    else
-        ln_bwd4_kernel<8, DY><<<grid, blk, 0, st>>>(dy, x, stats, g, dres, dx_out, dxb, T, d);
-    const int tiles = (T + kParamRows - 1) / kParamRows;
-    ln_param4_kernel<DY><<<dim3((d / 4 + 127) / 128, tiles), 128, 0, st>>>(dy, x, stats, T, d, part);
-    ln_param_reduce_kernel<<<(2 * d + 31) / 32, 256, 0, st>>>(part, tiles, d, dgam, dbet);
+template <int NV, int W, typename DY>
+cudaError_t launch_ln_bwd_fused(cudaStream_t st, int grid, const DY* dy, const float* x,
+                                const float2* stats, const float* g, const float* dres,
+                                float* dx_out, __nv_bfloat16* dxb, int T, int d, int ncol,
+                                float* part) {
+    auto kern = ln_bwd_fused_kernel<NV, W, DY>;
+    static std::once_flag once[64];
+    static cudaError_t set_err[64];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    std::call_once(once[dev], [&] {
+        set_err[dev] = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                            (int)kLnBwdMaxSmem);
+    });
+    if (set_err[dev] != cudaSuccess) return set_err[dev];
+    const size_t smem = (size_t)kRowWarps * ncol * d * sizeof(float);
+    kern<<<grid, kRowWarps * 32, smem, st>>>(dy, x, stats, g, dres, dx_out, dxb, T, d, ncol,
+                                              part);
+    return cudaGetLastError();
 }
 
-// the LayerNorm backward (rows, then the scale / shift gradients; dgam, dbet
-// zeroed before): four features a lane and access when d is a multiple of
-// 128, else one (ln_bwd_kernel with room for d / 32 values a lane)
-// Returns the number of kernels launched.
-int launch_ln_bwd(cudaStream_t st, const float* dyf, const __nv_bfloat16* dyb, const float* x,
-                  const float2* stats, const float* g, const float* dres, float* dx_out,
-                  __nv_bfloat16* dxb, float* part, float* dgam, float* dbet, int T, int d) {
+// Resident CTAs per SM of the fused LayerNorm backward for this d (its
+// register use and shared memory), at least 1.
+template <int NV, int W, typename DY>
+int ln_bwd_occupancy(int d, int ncol) {
+    int n = 0;
+    const size_t smem = (size_t)kRowWarps * ncol * d * sizeof(float);
+    if (cudaFuncSetAttribute(ln_bwd_fused_kernel<NV, W, DY>,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kLnBwdMaxSmem) != cudaSuccess ||
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, ln_bwd_fused_kernel<NV, W, DY>,
+                                                      kRowWarps * 32, smem) != cudaSuccess)
+        return 1;
+    return n > 0 ? n : 1;
+}
+
+int ln_bwd_ctas_per_sm(bool f32, int d, int ncol) {
+#define HCW_OCC(NV, W) \
+    return f32 ? ln_bwd_occupancy<NV, W, float>(d, ncol) : ln_bwd_occupancy<NV, W, __nv_bfloat16>(d, ncol)
     if (d % 128 == 0) {
-        if (dyf)
-            launch_ln_bwd4<float>(st, dyf, x, stats, g, dres, dx_out, dxb, part, dgam, dbet, T, d);
-        else
-            launch_ln_bwd4<__nv_bfloat16>(st, dyb, x, stats, g, dres, dx_out, dxb, part, dgam,
-                                          dbet, T, d);
-        return 3;
+        const int nv = d / 128;
+        if (nv <= 1) HCW_OCC(1, 4);
+        if (nv <= 2) HCW_OCC(2, 4);
+        if (nv <= 4) HCW_OCC(4, 4);
+        HCW_OCC(8, 4);
     }
-    const dim3 grid((T + kRowWarps - 1) / kRowWarps), blk(kRowWarps * 32);
-    if (d <= 128)
-        ln_bwd_kernel<4><<<grid, blk, 0, st>>>(dyf, dyb, x, stats, g, dres, dx_out, dxb, T, d);
-    else if (d <= 256)
-        ln_bwd_kernel<8><<<grid, blk, 0, st>>>(dyf, dyb, x, stats, g, dres, dx_out, dxb, T, d);
-    else if (d <= 512)
-        ln_bwd_kernel<16><<<grid, blk, 0, st>>>(dyf, dyb, x, stats, g, dres, dx_out, dxb, T, d);
-    else
-        ln_bwd_kernel<32><<<grid, blk, 0, st>>>(dyf, dyb, x, stats, g, dres, dx_out, dxb, T, d);
-    ln_param_kernel<<<dim3((d + 255) / 256, (T + kColRows - 1) / kColRows), 256, 0, st>>>(
-        dyf, dyb, x, stats, T, d, dgam, dbet);
-    return 2;
+    const int nv = d / 64;
+    if (nv <= 4) HCW_OCC(4, 2);
+    if (nv <= 8) HCW_OCC(8, 2);
+    HCW_OCC(16, 2);
+#undef HCW_OCC
+}
+
+template <typename DY>
+cudaError_t launch_ln_bwd_rows(cudaStream_t st, int grid, const DY* dy, const float* x,
+                               const float2* stats, const float* g, const float* dres,
+                               float* dx_out, __nv_bfloat16* dxb, int T, int d, int ncol,
+                               float* part) {
+#define HCW_LNB(NV, W) \
+    return launch_ln_bwd_fused<NV, W, DY>(st, grid, dy, x, stats, g, dres, dx_out, dxb, T, d, ncol, part)
+    if (d % 128 == 0) {   // four features a lane and access
+        const int nv = d / 128;
+        if (nv <= 1) HCW_LNB(1, 4);
+        if (nv <= 2) HCW_LNB(2, 4);
+        if (nv <= 4) HCW_LNB(4, 4);
+        HCW_LNB(8, 4);
+    }
+    const int nv = d / 64;   // d % 64 == 0: two
+    if (nv <= 4) HCW_LNB(4, 2);
+    if (nv <= 8) HCW_LNB(8, 2);
+    HCW_LNB(16, 2);
+#undef HCW_LNB
+}
+
+// The LayerNorm backward: rows and per-CTA parameter sums in one pass
+// (ln_bwd_fused_kernel), then their fixed-order sum (ln_part_reduce_kernel)
+// into dgam, dbet and, when dcol is given, the column sums of dxb.  Two
+// launches (*nk).
+cudaError_t launch_ln_bwd(cudaStream_t st, const float* dyf, const __nv_bfloat16* dyb,
+                          const float* x, const float2* stats, const float* g, const float* dres,
+                          float* dx_out, __nv_bfloat16* dxb, float* part, float* dgam, float* dbet,
+                          float* dcol, int T, int d, int* nk) {
+    *nk = 0;
+    if (dcol && !dxb) return cudaErrorInvalidValue;
+    const int ncol = dcol ? 3 : 2;
+    // one wave: as many CTAs as fit on the SMs at once, at most one a row group
+    int grid = (T + kRowWarps - 1) / kRowWarps;
+    const int wave = ln_bwd_ctas_per_sm(dyf != nullptr, d, ncol) * sms_now();
+    grid = grid < wave ? grid : wave;
+    grid = grid < kLnBwdMaxGrid ? grid : kLnBwdMaxGrid;
+    cudaError_t e = dyf ? launch_ln_bwd_rows<float>(st, grid, dyf, x, stats, g, dres, dx_out, dxb,
+                                                    T, d, ncol, part)
+                        : launch_ln_bwd_rows<__nv_bfloat16>(st, grid, dyb, x, stats, g, dres,
+                                                            dx_out, dxb, T, d, ncol, part);
+    if (e != cudaSuccess) return e;
+    *nk = 1;
+    ln_part_reduce_kernel<<<(ncol * d + 31) / 32, kReduceWarps * 32, 0, st>>>(part, grid, d, ncol,
+                                                                             dgam, dbet, dcol);
+    e = cudaGetLastError();
+    if (e == cudaSuccess) *nk = 2;
+    return e;
 }
 
 int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads& gr, int B, int n,
@@ -661,15 +726,15 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
     colsum_kernel<<<dim3((V + 255) / 256, gridT), 256, 0, st>>>(dlog, gr.bh, T, V);
     HCW_TRY(ok_launch());
     HCW_GEMM(T, d, V, dlog, false, p.Wh, false, U);    // dhf = dlog Wh
-    int nk = launch_ln_bwd(st, U, nullptr, X(L), sf, p.lnf_g, nullptr, dx, dxb, lnp, gr.lnf_g,
-                           gr.lnf_b, T, d);
-    HCW_TRY(count_launch(cudaGetLastError(), nk));
+    // each LayerNorm backward that writes the gradient of x_{l+1} (LNf, then
+    // LN1 of layer l + 1) also sums its bf16 copy's columns: db2 of layer l
+    int nk = 0;
+    cudaError_t le = launch_ln_bwd(st, U, nullptr, X(L), sf, p.lnf_g, nullptr, dx, dxb, lnp,
+                                   gr.lnf_g, gr.lnf_b, gr.b2 + (size_t)(L - 1) * d, T, d, &nk);
+    HCW_TRY(count_launch(le, nk));
     for (int l = L - 1; l >= 0; --l) {
         // FFN sublayer: dxb = bf16(dx) is the gradient of its output
         HCW_GEMM(d, h, T, dxb, true, A(l), false, gr.W2 + (size_t)l * d * h);
-        colsum_kernel<<<dim3((d + 255) / 256, gridT), 256, 0, st>>>(dxb, gr.b2 + (size_t)l * d, T,
-                                                                     d);
-        HCW_TRY(ok_launch());
         HCW_TRY(gemm_ffn(st, T, h, d, dxb, bf(p.W2, (size_t)l * d * h), false, nullptr, A(l),
                          dpre));   // dpre = (a > 0) * (dxb W2)
         colsum_kernel<<<dim3((h + 255) / 256, gridT), 256, 0, st>>>(dpre, gr.b1 + (size_t)l * h, T,
@@ -677,17 +742,19 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
         HCW_TRY(ok_launch());
         HCW_GEMM(h, d, T, dpre, true, G(l), false, gr.W1 + (size_t)l * h * d);
         HCW_GEMM(T, d, h, dpre, false, bf(p.W1, (size_t)l * h * d), false, U);  // dg
-        nk = launch_ln_bwd(st, U, nullptr, XM(l), S2(l), p.ln2_g + (size_t)l * d, dx, dx, dxb, lnp,
-                           gr.ln2_g + (size_t)l * d, gr.ln2_b + (size_t)l * d, T, d);
-        HCW_TRY(count_launch(cudaGetLastError(), nk));
+        le = launch_ln_bwd(st, U, nullptr, XM(l), S2(l), p.ln2_g + (size_t)l * d, dx, dx, dxb,
+                           lnp, gr.ln2_g + (size_t)l * d, gr.ln2_b + (size_t)l * d, nullptr, T, d,
+                           &nk);
+        HCW_TRY(count_launch(le, nk));
         // mixing sublayer: dxb = bf16(dx) is the gradient of M_l(h)
         HCW_TRY(hcw_layer_bwd(H1(l), nullptr, dxb, bf(p.W_self, (size_t)l * d * d),
                               bf(p.W_nbr, (size_t)l * d * d), l, -1, B, n, d, HCW_BF16, HCW_CAUSAL,
                               dh, gr.W_self + (size_t)l * d * d, gr.W_nbr + (size_t)l * d * d,
                               nullptr, w.lws_bytes ? ws + w.lws : nullptr, w.lws_bytes, st));
-        nk = launch_ln_bwd(st, nullptr, dh, X(l), S1(l), p.ln1_g + (size_t)l * d, dx, dx, dxb, lnp,
-                           gr.ln1_g + (size_t)l * d, gr.ln1_b + (size_t)l * d, T, d);
-        HCW_TRY(count_launch(cudaGetLastError(), nk));
+        le = launch_ln_bwd(st, nullptr, dh, X(l), S1(l), p.ln1_g + (size_t)l * d, dx, dx, dxb,
+                           lnp, gr.ln1_g + (size_t)l * d, gr.ln1_b + (size_t)l * d,
+                           l > 0 ? gr.b2 + (size_t)(l - 1) * d : nullptr, T, d, &nk);
+        HCW_TRY(count_launch(le, nk));
     }
     embed_bwd_kernel<<<elem_grid(Td), 256, 0, st>>>(ids, dx, gr.E, B, n, d, V);
     HCW_TRY(ok_launch());
