@@ -431,14 +431,17 @@ int gemm(float* split_ws, size_t split_bytes, cudaStream_t st, int M, int N, int
 }
 
 // The FFN's products with their elementwise step in the epilogue, bf16 out:
-// a = relu(G W1^T + b1) (aux NULL), or dpre = (a > 0) * (dy W2) (bias NULL).
+// a = relu(G W1^T + b1) (aux NULL), or dpre = (a > 0) * (dy W2) (bias NULL),
+// whose column sums (the gradient of b1) go into colsum (zeroed before).
 int gemm_ffn(cudaStream_t st, int M, int N, int K, const void* A, const void* B, bool tb,
-             const float* bias, const __nv_bfloat16* aux, __nv_bfloat16* out) {
+             const float* bias, const __nv_bfloat16* aux, __nv_bfloat16* out,
+             float* colsum = nullptr) {
     GemmEpi epi;
     epi.kind = bias ? EPI_BIAS_RELU : EPI_RELU_GRAD;
     epi.bias = bias;
     epi.aux = aux;
     epi.out = out;
+    epi.colsum = colsum;
     int launches = 0;
     const cudaError_t e =
         gemm_bf16(M, N, K, A, false, B, tb, nullptr, epi, nullptr, 0, st, &launches);
@@ -735,11 +738,9 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
     for (int l = L - 1; l >= 0; --l) {
         // FFN sublayer: dxb = bf16(dx) is the gradient of its output
         HCW_GEMM(d, h, T, dxb, true, A(l), false, gr.W2 + (size_t)l * d * h);
+        // dpre = (a > 0) * (dxb W2), and db1 = its column sums
         HCW_TRY(gemm_ffn(st, T, h, d, dxb, bf(p.W2, (size_t)l * d * h), false, nullptr, A(l),
-                         dpre));   // dpre = (a > 0) * (dxb W2)
-        colsum_kernel<<<dim3((h + 255) / 256, gridT), 256, 0, st>>>(dpre, gr.b1 + (size_t)l * h, T,
-                                                                     h);
-        HCW_TRY(ok_launch());
+                         dpre, gr.b1 + (size_t)l * h));
         HCW_GEMM(h, d, T, dpre, true, G(l), false, gr.W1 + (size_t)l * h * d);
         HCW_GEMM(T, d, h, dpre, false, bf(p.W1, (size_t)l * h * d), false, U);  // dg
         le = launch_ln_bwd(st, U, nullptr, XM(l), S2(l), p.ln2_g + (size_t)l * d, dx, dx, dxb,

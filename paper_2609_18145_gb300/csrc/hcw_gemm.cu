@@ -81,6 +81,7 @@ struct GemmArgs {
     __nv_bfloat16* out;         // EPI_BIAS_RELU / EPI_RELU_GRAD: [M][N] bf16
     const float* bias;          // EPI_BIAS_RELU: [N]
     const __nv_bfloat16* aux;   // EPI_RELU_GRAD: [M][N]
+    float* colsum;              // EPI_RELU_GRAD: [N] += column sums of the bf16 output, or null
     int M, N, K;
     int mt, nt;                 // tile counts (256-row tiles, 256-column tiles)
     int splits, kps;            // K splits and K steps per split
@@ -378,6 +379,24 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_pair_kernel(const __grid_co
                             tma_store_2d(&a.mOut, buf, c0, row0);
                             bulk_commit();
                         }
+                        if (EPI == EPI_RELU_GRAD && a.colsum) {
+                            // lane l adds up columns c0 + 2l, c0 + 2l + 1 of the patch's
+                            // 32 rows (the stored bf16 values; rows past M hold 0)
+                            const int m = lane >> 2, wd = lane & 3;
+                            float s0 = 0.f, s1 = 0.f;
+#pragma unroll 8
+                            for (int r = 0; r < 32; ++r) {
+                                const float2 f = unpack_bf16x2(*reinterpret_cast<const uint32_t*>(
+                                    buf + r * 128 + ((m ^ (r & 7)) << 4) + 4 * wd));
+                                s0 += f.x;
+                                s1 += f.y;
+                            }
+                            const int col = c0 + 2 * lane;
+                            if (col < a.N) {
+                                atomicAdd(a.colsum + col, s0);
+                                atomicAdd(a.colsum + col + 1, s1);
+                            }
+                        }
                     }
                 }
                 if (!okp) break;
@@ -453,6 +472,12 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_pair_kernel(const __grid_co
                                 pack_bf16x2(v[8 * m + 2], v[8 * m + 3]),
                                 pack_bf16x2(v[8 * m + 4], v[8 * m + 5]),
                                 pack_bf16x2(v[8 * m + 6], v[8 * m + 7]));
+                        if (EPI == EPI_RELU_GRAD && a.colsum) {
+#pragma unroll
+                            for (int i = 0; i < 32; ++i)
+                                atomicAdd(a.colsum + col0 + i,
+                                          __bfloat162float(__float2bfloat16_rn(v[i])));
+                        }
                     } else {
 #pragma unroll
                         for (int i = 0; i < 32; ++i) {
@@ -467,6 +492,8 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_pair_kernel(const __grid_co
                                 x = am > 0.f ? x : 0.f;
                             }
                             dst[i] = __float2bfloat16_rn(x);
+                            if (EPI == EPI_RELU_GRAD && a.colsum)
+                                atomicAdd(a.colsum + col0 + i, __bfloat162float(dst[i]));
                         }
                     }
                 }
@@ -562,6 +589,7 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(int M, int N, int K,
                 e.out[o] = __float2bfloat16_rn(x > 0.f ? x : 0.f);
             } else {
                 e.out[o] = __float2bfloat16_rn(__bfloat162float(e.aux[o]) > 0.f ? acc[i][j] : 0.f);
+                if (e.colsum) atomicAdd(e.colsum + gn, __bfloat162float(e.out[o]));
             }
         }
 }
@@ -738,11 +766,14 @@ cudaError_t gemm_bf16(int M, int N, int K, const void* A, bool ta, const void* B
                       cudaStream_t st, int* launches) {
     *launches = 0;
     if (M <= 0 || N <= 0 || K <= 0 || !A || !B) return cudaErrorInvalidValue;
-    if (epi.kind == EPI_F32 ? !C
-                            : (!epi.out || (epi.kind == EPI_BIAS_RELU && !epi.bias) ||
-                               (epi.kind == EPI_RELU_GRAD && !epi.aux) ||
-                               (epi.kind != EPI_BIAS_RELU && epi.kind != EPI_RELU_GRAD)))
-        return cudaErrorInvalidValue;
+    bool bad;
+    switch (epi.kind) {
+        case EPI_F32: bad = !C; break;
+        case EPI_BIAS_RELU: bad = !epi.out || !epi.bias; break;
+        case EPI_RELU_GRAD: bad = !epi.out || !epi.aux; break;
+        default: bad = true;
+    }
+    if (bad) return cudaErrorInvalidValue;
     const bool a_mn = ta, b_mn = !tb;
     const auto aligned = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
     // what TMA can read: 16-byte row strides, MN-major operands in whole
@@ -787,6 +818,7 @@ cudaError_t gemm_bf16(int M, int N, int K, const void* A, bool ta, const void* B
         a.out = epi.out;
         a.bias = epi.bias;
         a.aux = epi.aux;
+        a.colsum = epi.kind == EPI_RELU_GRAD ? epi.colsum : nullptr;
         a.vec = (N % 8 == 0) && aligned(epi.out) &&
                 (epi.kind == EPI_BIAS_RELU ? aligned(epi.bias) : aligned(epi.aux));
         a.tma_out = a.vec && map_patch_bf16(&a.mOut, epi.out, M, N) &&
@@ -818,6 +850,7 @@ cudaError_t gemm_bf16_f32(int M, int N, int K, const void* A, bool ta, const voi
     epi.bias = nullptr;
     epi.aux = nullptr;
     epi.out = nullptr;
+    epi.colsum = nullptr;
     return gemm_bf16(M, N, K, A, ta, B, tb, C, epi, split_ws, split_ws_bytes, st, launches);
 }
 

@@ -228,13 +228,15 @@ cudaError_t gemm_bf16_f32(int M, int N, int K, const void* A, bool ta, const voi
                           float* C, float* split_ws, size_t split_ws_bytes, cudaStream_t st,
                           int* launches);
 // Epilogues of the GEMM: fp32 C; out = bf16(relu(C + bias[col])); or
-// out = bf16(aux[row][col] > 0 ? C : 0).  out and aux are [M][N] bf16.
+// out = bf16(aux[row][col] > 0 ? C : 0), with colsum[col] (if given) += the
+// column sums of out.  out and aux are [M][N] bf16.
 enum GemmEpiKind { EPI_F32 = 0, EPI_BIAS_RELU = 1, EPI_RELU_GRAD = 2 };
 struct GemmEpi {
     int kind;
     const float* bias;
     const __nv_bfloat16* aux;
     __nv_bfloat16* out;
+    float* colsum;
 };
 // gemm_bf16_f32 with an epilogue (C unused unless epi.kind is EPI_F32; only
 // fp32 output splits K).
