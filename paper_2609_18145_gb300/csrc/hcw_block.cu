@@ -60,6 +60,8 @@ __device__ __forceinline__ int symbol(const int* ids, int b, int t, int n, int V
 // x[b n + t][c] = E[ids[b][t]][c] + P[t][c]   (fp32 out)
 __global__ void embed_fwd_kernel(const int* ids, const __nv_bfloat16* E, const __nv_bfloat16* P,
                                  float* x, int B, int n, int d, int V) {
+    pdl_wait();   // until the kernel before it in the stream has finished
+    pdl_trigger();
     const size_t total = (size_t)B * n * d;
     for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
          i += (size_t)gridDim.x * blockDim.x) {
@@ -77,6 +79,8 @@ __global__ void __launch_bounds__(kRowWarps * 32)
     ln_fwd_kernel(const float* x_in, const __nv_bfloat16* add1, const float* add2,
                   const float* badd, float* x_out, const float* g, const float* b,
                   __nv_bfloat16* y, float2* stats, int T, int d) {
+    pdl_wait();   // until the kernel before it in the stream has finished
+    pdl_trigger();
     const int lane = threadIdx.x & 31;
     const int row = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
     if (row >= T) return;
@@ -141,6 +145,8 @@ __global__ void __launch_bounds__(kRowWarps * 32)
     ln_fwd4_kernel(const float* x_in, const __nv_bfloat16* add1, const float* add2,
                    const float* badd, float* x_out, const float* g, const float* b,
                    __nv_bfloat16* y, float2* stats, int T, int d) {
+    pdl_wait();   // until the kernel before it in the stream has finished
+    pdl_trigger();
     const int lane = threadIdx.x & 31;
     const int row = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
     if (row >= T) return;
@@ -191,6 +197,8 @@ __global__ void __launch_bounds__(kRowWarps * 32)
 __global__ void __launch_bounds__(kRowWarps * 32)
     ce_kernel(const float* logits, const float* bh, const int* ids, __nv_bfloat16* dlog,
               float* loss, int B, int n, int V, float inv_N) {
+    pdl_wait();   // until the kernel before it in the stream has finished
+    pdl_trigger();
     const int lane = threadIdx.x & 31;
     const int r = blockIdx.x * kRowWarps + (threadIdx.x >> 5);
     if (r >= B * n) return;
@@ -215,6 +223,8 @@ __global__ void __launch_bounds__(kRowWarps * 32)
 // thread per column of its tile, the rows' loads independent of each other
 constexpr int kColRows = 64;
 __global__ void colsum_kernel(const __nv_bfloat16* M, float* out, int T, int C) {
+    pdl_wait();   // until the kernel before it in the stream has finished
+    pdl_trigger();
     const int c = blockIdx.x * blockDim.x + threadIdx.x;
     if (c >= C) return;
     const int r0 = blockIdx.y * kColRows;
@@ -280,6 +290,8 @@ __global__ void __launch_bounds__(kRowWarps * 32)
     ln_bwd_fused_kernel(const DY* dy, const float* x, const float2* stats, const float* g,
                         const float* dres, float* dx_out, __nv_bfloat16* dxb, int T, int d,
                         int ncol, float* part) {
+    pdl_wait();   // until the kernel before it in the stream has finished
+    pdl_trigger();
     extern __shared__ float red[];   // [kRowWarps][ncol d]: each warp's sums, then the CTA's
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int nv = d / (32 * W);
@@ -362,6 +374,8 @@ constexpr int kReduceWarps = 32;
 __global__ void __launch_bounds__(kReduceWarps * 32)
     ln_part_reduce_kernel(const float* part, int nblk, int d, int ncol, float* dgam, float* dbet,
                           float* dcol) {
+    pdl_wait();   // until the kernel before it in the stream has finished
+    pdl_trigger();
     __shared__ float acc[kReduceWarps][33];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int width = ncol * d;
@@ -393,6 +407,8 @@ __global__ void __launch_bounds__(kReduceWarps * 32)
 // dE[ids[b][t]] += dx[b n + t]   (dE zeroed before the launch)
 __global__ void embed_bwd_kernel(const int* ids, const float* dx, float* dE, int B, int n, int d,
                                  int V) {
+    pdl_wait();   // until the kernel before it in the stream has finished
+    pdl_trigger();
     const size_t total = (size_t)B * n * d;
     for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
          i += (size_t)gridDim.x * blockDim.x) {
@@ -405,6 +421,8 @@ __global__ void embed_bwd_kernel(const int* ids, const float* dx, float* dE, int
 
 // dP[t][c] = sum over b of dx[b n + t][c]
 __global__ void pos_bwd_kernel(const float* dx, float* dP, int B, int n, int d) {
+    pdl_wait();   // until the kernel before it in the stream has finished
+    pdl_trigger();
     const size_t total = (size_t)n * d;
     for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < total;
          i += (size_t)gridDim.x * blockDim.x) {
@@ -519,8 +537,6 @@ bool block_sizes_ok(int B, int n, int d, int h, int V, int L) {
 
 bool a16(const void* p) { return p && (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 
-// launch status of the kernel just launched (counted when it succeeded)
-int ok_launch() { return count_launch(cudaGetLastError(), 1); }
 
 unsigned elem_grid(size_t total) {
     const size_t want = (total + 255) / 256, cap = (size_t)sms_now() * 16;
@@ -529,21 +545,19 @@ unsigned elem_grid(size_t total) {
 
 // LayerNorm forward rows: four features a lane and access when d is a
 // multiple of 128, else one (ln_fwd_kernel)
-void launch_ln_fwd(cudaStream_t st, const float* x_in, const __nv_bfloat16* add1, const float* add2,
-                   const float* badd, float* x_out, const float* g, const float* b,
-                   __nv_bfloat16* y, float2* stats, int T, int d) {
+cudaError_t launch_ln_fwd(cudaStream_t st, const float* x_in, const __nv_bfloat16* add1,
+                          const float* add2, const float* badd, float* x_out, const float* g,
+                          const float* b, __nv_bfloat16* y, float2* stats, int T, int d) {
     const dim3 grid((T + kRowWarps - 1) / kRowWarps), blk(kRowWarps * 32);
     const int v4 = d / 128;
-    if (d % 128 != 0)
-        ln_fwd_kernel<<<grid, blk, 0, st>>>(x_in, add1, add2, badd, x_out, g, b, y, stats, T, d);
-    else if (v4 <= 1)
-        ln_fwd4_kernel<1><<<grid, blk, 0, st>>>(x_in, add1, add2, badd, x_out, g, b, y, stats, T, d);
-    else if (v4 <= 2)
-        ln_fwd4_kernel<2><<<grid, blk, 0, st>>>(x_in, add1, add2, badd, x_out, g, b, y, stats, T, d);
-    else if (v4 <= 4)
-        ln_fwd4_kernel<4><<<grid, blk, 0, st>>>(x_in, add1, add2, badd, x_out, g, b, y, stats, T, d);
-    else
-        ln_fwd4_kernel<8><<<grid, blk, 0, st>>>(x_in, add1, add2, badd, x_out, g, b, y, stats, T, d);
+#define HCW_LNF(K) \
+    return launch_pdl(K, grid, blk, 0, st, x_in, add1, add2, badd, x_out, g, b, y, stats, T, d)
+    if (d % 128 != 0) HCW_LNF(ln_fwd_kernel);
+    if (v4 <= 1) HCW_LNF(ln_fwd4_kernel<1>);
+    if (v4 <= 2) HCW_LNF(ln_fwd4_kernel<2>);
+    if (v4 <= 4) HCW_LNF(ln_fwd4_kernel<4>);
+    HCW_LNF(ln_fwd4_kernel<8>);
+#undef HCW_LNF
 }
 
 template <int NV, int W, typename DY>
@@ -564,9 +578,8 @@ cudaError_t launch_ln_bwd_fused(cudaStream_t st, int grid, const DY* dy, const f
     });
     if (set_err[dev] != cudaSuccess) return set_err[dev];
     const size_t smem = (size_t)kRowWarps * ncol * d * sizeof(float);
-    kern<<<grid, kRowWarps * 32, smem, st>>>(dy, x, stats, g, dres, dx_out, dxb, T, d, ncol,
-                                              part);
-    return cudaGetLastError();
+    return launch_pdl(kern, dim3(grid), dim3(kRowWarps * 32), smem, st, dy, x, stats, g, dres,
+                      dx_out, dxb, T, d, ncol, part);
 }
 
 // Resident CTAs per SM of the fused LayerNorm backward for this d (its
@@ -644,9 +657,8 @@ cudaError_t launch_ln_bwd(cudaStream_t st, const float* dyf, const __nv_bfloat16
                                                             dx_out, dxb, T, d, ncol, part);
     if (e != cudaSuccess) return e;
     *nk = 1;
-    ln_part_reduce_kernel<<<(ncol * d + 31) / 32, kReduceWarps * 32, 0, st>>>(part, grid, d, ncol,
-                                                                             dgam, dbet, dcol);
-    e = cudaGetLastError();
+    e = launch_pdl(ln_part_reduce_kernel, dim3((ncol * d + 31) / 32), dim3(kReduceWarps * 32), 0,
+                   st, static_cast<const float*>(part), grid, d, ncol, dgam, dbet, dcol);
     if (e == cudaSuccess) *nk = 2;
     return e;
 }
@@ -698,36 +710,42 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
     HCW_CU(cudaMemsetAsync(gr.bh, 0, (size_t)V * 4, st));
 
     // ------------------------------------------------------------ forward
-    embed_fwd_kernel<<<elem_grid(Td), 256, 0, st>>>(ids, bf(p.E, 0), bf(p.P, 0), X(0), B, n, d, V);
-    HCW_TRY(ok_launch());
-    launch_ln_fwd(st, X(0), nullptr, nullptr, nullptr, nullptr, p.ln1_g, p.ln1_b, H1(0), S1(0), T,
-                  d);
-    HCW_TRY(ok_launch());
+    HCW_TRY(count_launch(launch_pdl(embed_fwd_kernel, dim3(elem_grid(Td)), dim3(256), 0, st, ids,
+                                    bf(p.E, 0), bf(p.P, 0), X(0), B, n, d, V),
+                         1));
+    HCW_TRY(count_launch(launch_ln_fwd(st, X(0), nullptr, nullptr, nullptr, nullptr, p.ln1_g,
+                                       p.ln1_b, H1(0), S1(0), T, d),
+                         1));
     for (int l = 0; l < L; ++l) {
         HCW_TRY(hcw_layer_fwd(H1(l), bf(p.W_self, (size_t)l * d * d), bf(p.W_nbr, (size_t)l * d * d),
                               nullptr, l, -1, B, n, d, HCW_BF16, HCW_CAUSAL, m, nullptr, st));
-        launch_ln_fwd(st, X(l), m, nullptr, nullptr, XM(l), p.ln2_g + (size_t)l * d, p.ln2_b + (size_t)l * d, G(l),
-            S2(l), T, d);
-        HCW_TRY(ok_launch());
+        HCW_TRY(count_launch(launch_ln_fwd(st, X(l), m, nullptr, nullptr, XM(l),
+                                           p.ln2_g + (size_t)l * d, p.ln2_b + (size_t)l * d, G(l),
+                                           S2(l), T, d),
+                             1));
         HCW_TRY(gemm_ffn(st, T, h, d, G(l), bf(p.W1, (size_t)l * h * d), true,
                          p.b1 + (size_t)l * h, nullptr, A(l)));   // a = relu(g W1^T + b1)
         HCW_GEMM(T, d, h, A(l), false, bf(p.W2, (size_t)l * d * h), true, U);
         const bool top = l + 1 == L;
-        launch_ln_fwd(st, XM(l), nullptr, U, p.b2 + (size_t)l * d, X(l + 1),
-            top ? p.lnf_g : p.ln1_g + (size_t)(l + 1) * d,
-            top ? p.lnf_b : p.ln1_b + (size_t)(l + 1) * d, top ? hf : H1(l + 1), top ? sf : S1(l + 1),
-            T, d);
-        HCW_TRY(ok_launch());
+        HCW_TRY(count_launch(
+            launch_ln_fwd(st, XM(l), nullptr, U, p.b2 + (size_t)l * d, X(l + 1),
+                          top ? p.lnf_g : p.ln1_g + (size_t)(l + 1) * d,
+                          top ? p.lnf_b : p.ln1_b + (size_t)(l + 1) * d, top ? hf : H1(l + 1),
+                          top ? sf : S1(l + 1), T, d),
+            1));
     }
     HCW_GEMM(T, V, d, hf, false, p.Wh, true, U);
-    ce_kernel<<<rows_grid, kRowWarps * 32, 0, st>>>(U, p.bh, ids, dlog, loss, B, n, V, 1.f / T);
-    HCW_TRY(ok_launch());
+    HCW_TRY(count_launch(launch_pdl(ce_kernel, dim3(rows_grid), dim3(kRowWarps * 32), 0, st,
+                                    static_cast<const float*>(U), p.bh, ids, dlog, loss, B, n, V,
+                                    1.f / T),
+                         1));
 
     // ----------------------------------------------------------- backward
     const unsigned gridT = (unsigned)((T + kColRows - 1) / kColRows);
     HCW_GEMM(V, d, T, dlog, true, hf, false, gr.Wh);   // dWh = dlog^T hf
-    colsum_kernel<<<dim3((V + 255) / 256, gridT), 256, 0, st>>>(dlog, gr.bh, T, V);
-    HCW_TRY(ok_launch());
+    HCW_TRY(count_launch(launch_pdl(colsum_kernel, dim3((V + 255) / 256, gridT), dim3(256), 0, st,
+                                    static_cast<const __nv_bfloat16*>(dlog), gr.bh, T, V),
+                         1));
     HCW_GEMM(T, d, V, dlog, false, p.Wh, false, U);    // dhf = dlog Wh
     // each LayerNorm backward that writes the gradient of x_{l+1} (LNf, then
     // LN1 of layer l + 1) also sums its bf16 copy's columns: db2 of layer l
@@ -757,10 +775,12 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
                            l > 0 ? gr.b2 + (size_t)(l - 1) * d : nullptr, T, d, &nk);
         HCW_TRY(count_launch(le, nk));
     }
-    embed_bwd_kernel<<<elem_grid(Td), 256, 0, st>>>(ids, dx, gr.E, B, n, d, V);
-    HCW_TRY(ok_launch());
-    pos_bwd_kernel<<<elem_grid((size_t)n * d), 256, 0, st>>>(dx, gr.P, B, n, d);
-    return ok_launch();
+    HCW_TRY(count_launch(launch_pdl(embed_bwd_kernel, dim3(elem_grid(Td)), dim3(256), 0, st, ids,
+                                    static_cast<const float*>(dx), gr.E, B, n, d, V),
+                         1));
+    return count_launch(launch_pdl(pos_bwd_kernel, dim3(elem_grid((size_t)n * d)), dim3(256), 0,
+                                   st, static_cast<const float*>(dx), gr.P, B, n, d),
+                        1);
 #undef HCW_TRY
 #undef HCW_CU
 #undef HCW_GEMM

@@ -130,6 +130,10 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_pair_kernel(const __grid_co
     __syncthreads();
     cluster_sync_all();   // both CTAs' barriers exist before any cross-CTA arrive
     tc_fence_after();
+    // the prologue above touched no global memory: it overlaps the end of the
+    // kernel before this one when launched as a programmatic dependent
+    pdl_wait();
+    pdl_trigger();
     const uint32_t tmem_base = bars->tmem_base;
     volatile int* abort = &bars->abort;
     // unit u -> (split, tile row, tile column), tile columns fastest: the pairs
@@ -521,6 +525,8 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_pair_kernel(const __grid_co
 // C[i] = sum over the splits s, in order, of part[s][i]; four at a time
 __global__ void gemm_split_reduce_kernel(const float* part, int splits, size_t count, float* C,
                                          bool vec) {
+    pdl_wait();   // until the kernel before it in the stream has finished
+    pdl_trigger();
     const size_t n4 = vec ? count / 4 : 0;
     for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4;
          i += (size_t)gridDim.x * blockDim.x) {
@@ -549,6 +555,8 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(int M, int N, int K,
                                                          const __nv_bfloat16* A, bool ta,
                                                          const __nv_bfloat16* B, bool tb,
                                                          float* C, GemmEpi e) {
+    pdl_wait();   // until the kernel before it in the stream has finished
+    pdl_trigger();
     __shared__ float As[16][65];
     __shared__ float Bs[16][65];
     const int tm = blockIdx.y * 64, tn = blockIdx.x * 64;
@@ -697,13 +705,15 @@ cudaError_t launch_gemm_pair(const GemmArgs& a, int grid, cudaStream_t st) {
     cfg.blockDim = dim3((unsigned)kGThreads);
     cfg.dynamicSmemBytes = kGSmem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
@@ -783,10 +793,11 @@ cudaError_t gemm_bf16(int M, int N, int K, const void* A, bool ta, const void* B
                     gemm_encode_fn() != nullptr;
     if (!tc) {
         dim3 grid((unsigned)((N + 63) / 64), (unsigned)((M + 63) / 64));
-        gemm_simt_kernel<<<grid, 256, 0, st>>>(M, N, K, static_cast<const __nv_bfloat16*>(A), ta,
-                                               static_cast<const __nv_bfloat16*>(B), tb, C, epi);
-        *launches = 1;
-        return cudaGetLastError();
+        const cudaError_t e = launch_pdl(gemm_simt_kernel, grid, dim3(256), 0, st, M, N, K,
+                                         static_cast<const __nv_bfloat16*>(A), ta,
+                                         static_cast<const __nv_bfloat16*>(B), tb, C, epi);
+        if (e == cudaSuccess) *launches = 1;
+        return e;
     }
     // boxes no larger than the operand (the rows / blocks a smaller box leaves
     // in shared memory only reach output rows and columns that are not stored)
@@ -834,9 +845,9 @@ cudaError_t gemm_bf16(int M, int N, int K, const void* A, bool ta, const void* B
         const size_t count = (size_t)M * N;
         const size_t want = (count / 4 + 255) / 256;
         const unsigned g = (unsigned)(want < (size_t)sms * 8 ? (want ? want : 1) : (size_t)sms * 8);
-        gemm_split_reduce_kernel<<<g, 256, 0, st>>>(split_ws, a.splits, count, C,
-                                                     aligned(C) && aligned(split_ws));
-        e = cudaGetLastError();
+        e = launch_pdl(gemm_split_reduce_kernel, dim3(g), dim3(256), 0, st,
+                       static_cast<const float*>(split_ws), a.splits, count, C,
+                       aligned(C) && aligned(split_ws));
         if (e == cudaSuccess) *launches = 2;
     }
     return e;

@@ -219,6 +219,25 @@ cudaError_t launch_decode(const DecodeLaunch& p, cudaStream_t st);
 // Read the decode kernel's error word and reset it to 0 (synchronous).
 cudaError_t decode_error_word_read_clear(int* word);
 
+// Launch `kern` with programmatic stream serialization: it may start while the
+// kernel before it in the stream finishes, and must call pdl_wait()
+// (hcw_ptx.cuh) before it touches memory that kernel reads or writes.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t st, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 // ---- Plain GEMMs of the character-LM block (hcw_gemm.cu) ----
 // Row-major C[M][N] (fp32) = op(A) op(B), bf16 operands, fp32 accumulation;
 // A is [M][K] ([K][M] when ta), B is [K][N] ([N][K] when tb).  split_ws
