@@ -981,21 +981,31 @@ def run_decode(args, w, dev):
         torch.cuda.synchronize()
         return a.elapsed_time(b) / reps
 
+    def graph_time():
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            window()
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=s):
+                window()
+        torch.cuda.synchronize()
+        g.replay()
+        return timed(g.replay, max(1, args.steps))
+
     for _ in range(max(1, args.warmup)):
         window()
     c0 = H.hcw_launch_count()
     host_ms = timed(window, max(1, args.steps))
     launches = (H.hcw_launch_count() - c0) / max(1, args.steps) / n
-    s = torch.cuda.Stream()
-    s.wait_stream(torch.cuda.current_stream())
-    with torch.cuda.stream(s):
+    graph_ms = graph_time()
+    # the same window with the tcgen05 contraction (hcw_set_decode_kernel)
+    prev = H.hcw_set_decode_kernel(H.HCW_DECODE_TCGEN05)
+    try:
         window()
-        g = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(g, stream=s):
-            window()
-    torch.cuda.synchronize()
-    g.replay()
-    graph_ms = timed(g.replay, max(1, args.steps))
+        tc_ms = graph_time()
+    finally:
+        H.hcw_set_decode_kernel(prev)
     if H.hcw_sync_status() != H.HCW_OK:
         raise SystemExit("device error")
     wbytes = 2.0 * L * d * d * 2
@@ -1006,6 +1016,7 @@ def run_decode(args, w, dev):
         "cache_bytes": cache.numel(), "launches_per_position": launches,
         "us_per_position_host_issued": round(host_ms * 1e3 / n, 2),
         "us_per_position_graph": round(us, 2),
+        "us_per_position_graph_tcgen05": round(tc_ms * 1e3 / n, 2),
         "tokens_per_s_graph": round(B / (us * 1e-6)),
         "weight_bytes_per_position": wbytes,
         "weight_gbs_graph": round(wbytes / (us * 1e-6) / 1e9, 1),

@@ -393,6 +393,20 @@ int hcw_decode_step(const void* x_t, const void* W_self, const void* W_nbr, cons
 size_t hcw_decode_cache_bytes(const int* dims, int layer0, int L, int B, int n, int d);
 
 /*
+ * The contraction hcw_decode_step runs, for this process:
+ *   HCW_DECODE_WARP_MMA (default): eight warps per CTA share the K range with
+ *     the warp-level bf16 MMA and add their partial blocks;
+ *   HCW_DECODE_TCGEN05: one thread issues tcgen05.mma (M = 64 over the 16
+ *     rows of a row block, N = the CTA's output columns) into TMEM.
+ * Both accumulate in fp32 and round the same tensors to bf16; they add the
+ * products in different orders, so their results differ at bf16 rounding
+ * level.  Returns the previous mode, or -1 (mode unchanged) for an unknown mode.
+ */
+#define HCW_DECODE_WARP_MMA 0
+#define HCW_DECODE_TCGEN05  1
+int hcw_set_decode_kernel(int mode);
+
+/*
  * One training step (forward, loss, backward) of the character-LM block
  * around the mixing stack, bf16 (App. A: width d, hidden h = 1024 = 2d at
  * d = 512; the weight counts of Table B2ecost / B1cost fit token and position

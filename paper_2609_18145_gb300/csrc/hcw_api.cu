@@ -411,6 +411,7 @@ bool use_pairs(const Shape& sh) {
 // kernels (hcw_res.cu): the shape fits them (d in {128, 256, 512}, n <= 256,
 // whole 256-token tiles) and hcw_set_stack_kernels asked for them.
 std::atomic<int> g_stack_kernels{HCW_STACK_AUTO};
+std::atomic<int> g_decode_kernel{HCW_DECODE_WARP_MMA};
 
 bool use_resident(const Shape& sh) {
     const int mode = g_stack_kernels.load(std::memory_order_relaxed);
@@ -1953,7 +1954,13 @@ int hcw_decode_step(const void* x_t, const void* W_self, const void* W_nbr, cons
     p.B = B;
     p.flags = flags;
     p.timeout_ns = g_timeout_ns;
+    p.tc = g_decode_kernel.load(std::memory_order_relaxed) == HCW_DECODE_TCGEN05;
     return launched(launch_decode(p, st), 1);
+}
+
+int hcw_set_decode_kernel(int mode) {
+    if (mode != HCW_DECODE_WARP_MMA && mode != HCW_DECODE_TCGEN05) return -1;
+    return g_decode_kernel.exchange(mode);
 }
 
 int hcw_set_stack_kernels(int mode) {

@@ -32,11 +32,26 @@
 //     stores (distributed shared memory) that count their bytes on that CTA's
 //     "input ready" mbarrier: the layer input is complete when all 16 x d x 2
 //     bytes have landed, with no fence or barrier between the CTAs.
-// No layer boundary goes through global memory or a grid-wide barrier.  A tile
-// holds 16 rows, below the 64-row minimum of a tcgen05 MMA, so the contraction
-// uses the warp-level bf16 MMA (m16n8k16).  That path runs at about 1/15 of
-// tcgen05's rate on this GPU, and with the in-kernel weight stream it is one
-// of the two bounds of a layer, about equal in size.
+// No layer boundary goes through global memory or a grid-wide barrier.
+//
+// Two contractions (decode_kernel<TC>, chosen with hcw_set_decode_kernel):
+//   - TC = false (the default): eight warps share the K range with the
+//     warp-level bf16 MMA (m16n8k16) and add their 16 x 8 blocks into the
+//     CTA's row sums;
+//   - TC = true: one thread issues tcgen05.mma.  A tile holds 16 rows, below
+//     the 64-row minimum, so the MMA runs with M = 64 on the 16 rows (its
+//     other 48 rows read whatever follows in shared memory; only D's rows
+//     0..15, TMEM lanes 0..15, are used) and N = OC.  The operands are already
+//     in the MMA's K-major 128-byte-swizzled layout.  Warp 7 issues, warp 0
+//     drains D into the row sums, and a layer's partner part is contracted
+//     into the other of two accumulators while the layer before is drained.
+// A layer is a chain (input in, contraction, epilogue, pushes out).  Issuing
+// a layer's 32 partner-part MMAs (N = OC = 32 at d = 512, K = 16) only after
+// its input arrived costs 0.75 us a layer, so one thread's tcgen05.mma run
+// about 45 cycles each in sequence, where the eight warps' MMAs run side by
+// side; the commit, the TMEM drain and a proxy fence (the remote stores are
+// generic writes that the MMA reads through the async proxy) add to the chain.
+// So the tensor-core version is the slower of the two here.
 #include "hcw_internal.h"
 #include "hcw_ptx.cuh"
 
@@ -45,8 +60,13 @@ namespace hcw {
 namespace {
 
 constexpr int kRows = 16;          // rows of a row block
-constexpr int kMmaWarps = 8;       // warps 0..7: MMA + epilogue; warp 8: producer
+constexpr int kMmaWarps = 8;       // warps 0..7: MMA + epilogue (TC: warp 7 issues, warps
+                                   // 0..6 run the epilogue); warp 8: producer
 constexpr int kThreads = (kMmaWarps + 1) * 32;
+// TC: accumulators a layer's K tiles alternate over, for each layer parity (64
+// columns each); four in turn measured no faster than one
+constexpr int kNAcc = 1;
+constexpr uint32_t kTmemCols = 2 * kNAcc * 64 < 32 ? 32 : 2 * kNAcc * 64;
 constexpr int kMaxStages = 8;
 
 struct DecodeArgs {
@@ -66,12 +86,15 @@ struct DecodeArgs {
 // barrier slots
 enum : int {
     B_FULL = 0,                       // [kMaxStages] stage filled (tx bytes)
-    B_EMPTY = kMaxStages,             // [kMaxStages] stage consumed by the 8 MMA warps
+    B_EMPTY = kMaxStages,             // [kMaxStages] stage consumed (8 MMA warps, or a commit)
     B_XS_READY = 2 * kMaxStages,      // [2] layer input complete (tx bytes from every cluster CTA)
     B_X0 = 2 * kMaxStages + 2,        // x_t rows loaded
     B_XP_FULL = 2 * kMaxStages + 3,   // [2] partner rows loaded
-    B_XP_FREE = 2 * kMaxStages + 5,   // [2] partner buffer consumed by the 8 MMA warps
-    B_COUNT = 2 * kMaxStages + 7
+    B_XP_FREE = 2 * kMaxStages + 5,   // [2] partner buffer consumed (8 MMA warps, or a commit)
+    B_DFULL = 2 * kMaxStages + 7,     // TC: [2] a layer's accumulator complete (commit)
+    B_TFREE = 2 * kMaxStages + 9,     // TC: [2] a layer's accumulator drained by warp 0
+    B_DRAIN = 2 * kMaxStages + 11,    // TC: the issuer's last MMAs completed
+    B_COUNT = 2 * kMaxStages + 12
 };
 
 // Shared memory (1024-byte aligned): Xs[2] (layer inputs) and Xp[2] (partner
@@ -95,6 +118,9 @@ struct Smem {
         return reinterpret_cast<uint64_t*>(red(2));
     }
     __device__ int* abort_word() const { return reinterpret_cast<int*>(bars() + B_COUNT); }
+    __device__ uint32_t* tmem_slot() const {
+        return reinterpret_cast<uint32_t*>(abort_word() + 1);
+    }
 };
 
 // byte offset of the 16-byte chunk holding features [8 c, 8 c + 8) of row r
@@ -141,6 +167,201 @@ __device__ __forceinline__ int chunk_len(const DecodeGeo& g, int c) {
     return g.d - k0 < g.kc ? g.d - k0 : g.kc;
 }
 
+// The end of a layer for one epilogue thread (8 columns of one row, v =
+// the row sums plus bias): ReLU, residual, bf16; the result goes into every
+// cluster CTA's next-layer input (remote stores counted on its input barrier)
+// and, for a valid row, to the layer's output in global memory.
+__device__ __forceinline__ void decode_epilogue(const DecodeArgs& a, const Smem& sm, float (&v)[8],
+                                                uint4 xin, int l, int xb, int q, int row0,
+                                                int vr, int pr, int pc8, uint32_t poff) {
+    const DecodeGeo& g = a.g;
+    const int d = g.d, col0 = q * g.oc;
+    if (a.flags & 4u) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) v[e] = v[e] > 0.f ? v[e] : 0.f;
+    }
+    if (a.flags & 2u) {
+        const uint32_t w[4] = {xin.x, xin.y, xin.z, xin.w};
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const float2 f = unpack_bf16x2(w[e]);
+            v[2 * e] += f.x;
+            v[2 * e + 1] += f.y;
+        }
+    }
+    uint4 pk;
+    pk.x = pack_bf16x2(v[0], v[1]);
+    pk.y = pack_bf16x2(v[2], v[3]);
+    pk.z = pack_bf16x2(v[4], v[5]);
+    pk.w = pack_bf16x2(v[6], v[7]);
+    if (l + 1 < a.L) {
+        const uint8_t* dst = sm.xs(xb ^ 1) + poff;
+        const uint64_t* rb = &sm.bars()[B_XS_READY + (xb ^ 1)];
+        for (int cr = 0; cr < g.csize; ++cr)
+            st_async_v4(mapa_shared(dst, cr), pk, mapa_shared(rb, cr));
+    }
+    if (pr < vr) {
+        if (l == 0)   // position t's layer-0 input into layer 0's ring
+            *reinterpret_cast<uint4*>(a.ring0 + (size_t)(row0 + pr) * d + col0 + pc8) = xin;
+        *reinterpret_cast<uint4*>(a.out[l] + (size_t)(row0 + pr) * d + col0 + pc8) = pk;
+    }
+}
+
+// The MMA and epilogue warps of decode_kernel<true>: warp 7 issues the
+// tcgen05 MMAs, warp 0 drains each layer's accumulator into the row sums, and
+// warps 0..6 run the epilogue (bias, ReLU, residual, bf16, pushes).
+__device__ __forceinline__ void decode_tc_body(const DecodeArgs& a, const Smem& sm, int warp,
+                                            int lane, int q, int row0, int vr) {
+    const DecodeGeo& g = a.g;
+    uint64_t* bars = sm.bars();
+    const int d = g.d, oc = g.oc, col0 = q * oc, nch = g.nchunks;
+    const uint32_t xtile = kRows * 128, wtile = (uint32_t)oc * 128;
+    volatile int* abort = sm.abort_word();
+    const uint32_t IDESC = idesc_bf16_f32(64, oc, 0, 0);
+    const uint32_t tmem_base = *reinterpret_cast<volatile uint32_t*>(sm.tmem_slot());
+    const int packs = kRows * oc / 8;   // epilogue: a thread per 8 columns of a row
+    const int pr = threadIdx.x / (oc / 8), pc8 = (threadIdx.x % (oc / 8)) * 8;
+    const uint32_t poff = sw_off(pr, col0 + pc8, xtile);
+    bool ok = true;
+    if (warp == kMmaWarps - 1) {
+        if (lane == 0) {
+            // ---------------------------------------------- MMA issuer
+            uint32_t it = 0;
+            int xp_uses[2] = {0, 0};
+            for (int l = 0; l < a.L && ok; ++l) {
+                const int xb = l & 1, ab = l & 1;
+                const bool recv = a.prow[l] >= 0;
+                // the accumulator of this parity has been drained (layer l - 2)
+                if (l >= 2)
+                    ok = mbar_wait(&bars[B_TFREE + ab], ((l - 2) >> 1) & 1, abort, a.timeout_ns);
+                if (!ok) break;
+                tc_fence_after();
+                // K tile j of the layer goes to accumulator j mod kNAcc: consecutive
+                // MMAs do not wait on each other's result
+                int tix = 0;
+                for (int part = recv ? 1 : 0; part >= 0 && ok; --part) {
+                    uint32_t X;
+                    if (part) {
+                        ok = mbar_wait(&bars[B_XP_FULL + xb], xp_uses[xb]++ & 1, abort,
+                                       a.timeout_ns);
+                        X = smem_u32(sm.xpart(xb));
+                    } else {
+                        ok = l == 0 ? mbar_wait(&bars[B_X0], 0, abort, a.timeout_ns)
+                                    : mbar_wait_cluster(&bars[B_XS_READY + xb], ((l - 1) >> 1) & 1,
+                                                        abort, a.timeout_ns);
+                        X = smem_u32(sm.xs(xb));
+                        // the input came by remote stores (generic proxy); the MMAs
+                        // read it through the async proxy
+                        if (ok) fence_proxy_async_smem();
+                    }
+                    if (!ok) break;
+                    tc_fence_after();
+                    for (int c = 0; c < nch && ok; ++c, ++it) {
+                        const int s = (int)(it % (uint32_t)g.stages);
+                        ok = mbar_wait(&bars[B_FULL + s], (it / g.stages) & 1, abort, a.timeout_ns);
+                        if (!ok) break;
+                        tc_fence_after();
+                        const uint32_t W = smem_u32(sm.stage(s));
+                        const int tiles = chunk_len(g, c) / 64, t0 = c * g.kc / 64;
+                        for (int t = 0; t < tiles; ++t, ++tix) {
+                            const uint32_t d_tmem =
+                                tmem_base + (uint32_t)((ab * kNAcc + tix % kNAcc) * 64);
+#pragma unroll
+                            for (int kk = 0; kk < 4; ++kk) {
+                                const uint64_t ad = smem_desc_sw128(
+                                    X + (uint32_t)(t0 + t) * xtile + kk * 32, 16, 1024);
+                                const uint64_t bd =
+                                    smem_desc_sw128(W + (uint32_t)t * wtile + kk * 32, 16, 1024);
+                                mma_bf16_f32(d_tmem, ad, bd, IDESC,
+                                             (tix < kNAcc && kk == 0) ? 0u : 1u);
+                            }
+                        }
+                        mma_commit(&bars[B_EMPTY + s]);
+                    }
+                    if (ok && part) mma_commit(&bars[B_XP_FREE + xb]);
+                }
+                if (ok) mma_commit(&bars[B_DFULL + ab]);
+            }
+            if (!ok) *abort = 1;
+            // the MMAs have completed before the CTA frees TMEM at the end
+            if (it > 0) {
+                mma_commit(&bars[B_DRAIN]);
+                mbar_wait_drain(&bars[B_DRAIN], 0, a.timeout_ns);
+            }
+        }
+        __syncwarp();
+        return;
+    }
+    for (int l = 0; l < a.L; ++l) {
+        const int xb = l & 1, ab = l & 1;
+        // the next layer's input arrives as 16 x d x 2 bytes from the cluster
+        if (threadIdx.x == 0 && l + 1 < a.L)
+            mbar_arrive_expect_tx(&bars[B_XS_READY + (xb ^ 1)], (uint32_t)kRows * d * 2);
+        // this thread's bias values, loaded while the layer runs
+        float4 bv0 = make_float4(0.f, 0.f, 0.f, 0.f), bv1 = bv0;
+        if (a.bias && (int)threadIdx.x < packs) {
+            const float4* bl = reinterpret_cast<const float4*>(a.bias + (size_t)l * d + col0 + pc8);
+            bv0 = __ldg(bl);
+            bv1 = __ldg(bl + 1);
+        }
+        float* red = sm.red(xb);
+        if (warp == 0) {
+            // D rows 0..15 (TMEM lanes 0..15) into this layer's row sums
+            bool r = ok && mbar_wait(&bars[B_DFULL + ab], (l >> 1) & 1, abort, a.timeout_ns);
+            ok = __all_sync(0xffffffffu, r);
+            if (ok) {
+                tc_fence_after();
+                // the accumulators the layer's K tiles went to, added in order
+                const int ntiles = (a.prow[l] >= 0 ? 2 : 1) * (d / 64);
+                const int nacc = ntiles < kNAcc ? ntiles : kNAcc;
+                for (int c0 = 0; c0 < oc; c0 += 32) {
+                    float sum[32];
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) sum[e] = 0.f;
+                    for (int ac = 0; ac < nacc; ++ac) {
+                        uint32_t raw[32];
+                        tmem_ld_32x32b_x32(
+                            tmem_base + (uint32_t)((ab * kNAcc + ac) * 64 + c0), raw);
+                        tmem_ld_wait_regs(raw);
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) sum[e] += __uint_as_float(raw[e]);
+                    }
+                    const int nc = oc - c0 < 32 ? oc - c0 : 32;
+                    if (lane < kRows) {
+#pragma unroll
+                        for (int e = 0; e < 32; ++e)
+                            if (e < nc) red[lane * oc + c0 + e] = sum[e];
+                    }
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&bars[B_TFREE + ab]);
+            }
+        }
+        // the layer input (the residual) is complete here: every thread takes
+        // the barrier's acquire before it reads it
+        {
+            bool r = ok && (l == 0 ? mbar_wait(&bars[B_X0], 0, abort, a.timeout_ns)
+                                   : mbar_wait_cluster(&bars[B_XS_READY + xb], ((l - 1) >> 1) & 1,
+                                                       abort, a.timeout_ns));
+            ok = __all_sync(0xffffffffu, r);
+        }
+        // every thread past this point has finished the previous layer's
+        // epilogue, so the other row-sum buffer is free again
+        named_bar_sync(1, (kMmaWarps - 1) * 32);
+        if (ok && (int)threadIdx.x < packs) {
+            const uint4 xin = *reinterpret_cast<const uint4*>(sm.xs(xb) + poff);
+            const float* rr = red + pr * oc + pc8;
+            const float bvals[8] = {bv0.x, bv0.y, bv0.z, bv0.w, bv1.x, bv1.y, bv1.z, bv1.w};
+            float v[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) v[e] = rr[e] + bvals[e];
+            decode_epilogue(a, sm, v, xin, l, xb, q, row0, vr, pr, pc8, poff);
+        }
+    }
+}
+
+template <bool TC>
 __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_constant__ DecodeArgs a) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* base = reinterpret_cast<uint8_t*>(
@@ -162,19 +383,28 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
         *abort = 0;
         for (int s = 0; s < g.stages; ++s) {
             mbar_init(&bars[B_FULL + s], 1);
-            mbar_init(&bars[B_EMPTY + s], kMmaWarps);
+            mbar_init(&bars[B_EMPTY + s], TC ? 1 : kMmaWarps);
         }
         mbar_init(&bars[B_XS_READY + 0], 1);
         mbar_init(&bars[B_XS_READY + 1], 1);
         mbar_init(&bars[B_X0], 1);
         for (int b = 0; b < 2; ++b) {
             mbar_init(&bars[B_XP_FULL + b], 1);
-            mbar_init(&bars[B_XP_FREE + b], kMmaWarps);
+            mbar_init(&bars[B_XP_FREE + b], TC ? 1 : kMmaWarps);
+            mbar_init(&bars[B_DFULL + b], 1);
+            mbar_init(&bars[B_TFREE + b], 1);
         }
+        mbar_init(&bars[B_DRAIN], 1);
         fence_mbar_init();
     }
+    if (TC && warp == 0) {
+        tmem_alloc(sm.tmem_slot(), kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
     __syncthreads();
     cluster_sync_all();   // barriers initialised in every CTA of the cluster
+    tc_fence_after();
 
     if (warp == kMmaWarps) {
         // ---------------------------------------------------------- producer
@@ -236,6 +466,8 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
             }
         }
         __syncwarp();
+    } else if (TC) {
+        decode_tc_body(a, sm, warp, lane, q, row0, vr);
     } else {
         // ---------------------------------------------------- MMA + epilogue
         const int nb_count = oc / 8;               // n8 blocks: 2, 4 or 8
@@ -346,42 +578,18 @@ __global__ void __launch_bounds__(kThreads, 1) decode_kernel(const __grid_consta
                     v[e] = rr[e] + bvals[e];
                     rr[e] = 0.f;
                 }
-                if (a.flags & 4u) {
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) v[e] = v[e] > 0.f ? v[e] : 0.f;
-                }
-                if (a.flags & 2u) {
-                    const uint32_t w[4] = {xin.x, xin.y, xin.z, xin.w};
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const float2 f = unpack_bf16x2(w[e]);
-                        v[2 * e] += f.x;
-                        v[2 * e + 1] += f.y;
-                    }
-                }
-                uint4 pk;
-                pk.x = pack_bf16x2(v[0], v[1]);
-                pk.y = pack_bf16x2(v[2], v[3]);
-                pk.z = pack_bf16x2(v[4], v[5]);
-                pk.w = pack_bf16x2(v[6], v[7]);
-                if (l + 1 < a.L) {
-                    const uint8_t* dst = sm.xs(xb ^ 1) + poff;
-                    const uint64_t* rb = &bars[B_XS_READY + (xb ^ 1)];
-                    for (int cr = 0; cr < g.csize; ++cr)
-                        st_async_v4(mapa_shared(dst, cr), pk, mapa_shared(rb, cr));
-                }
-                if (pr < vr) {
-                    if (l == 0)   // position t's layer-0 input into layer 0's ring
-                        *reinterpret_cast<uint4*>(a.ring0 + (size_t)(row0 + pr) * d + col0 + pc8) =
-                            xin;
-                    *reinterpret_cast<uint4*>(a.out[l] + (size_t)(row0 + pr) * d + col0 + pc8) =
-                        pk;
-                }
+                decode_epilogue(a, sm, v, xin, l, xb, q, row0, vr, pr, pc8, poff);
             }
         }
     }
+    tc_fence_before();
     __syncthreads();
     cluster_sync_all();   // no CTA leaves while a peer may still write its shared memory
+    if (TC && warp == 0) {
+        __syncwarp();
+        tc_fence_after();
+        tmem_dealloc(*sm.tmem_slot(), kTmemCols);
+    }
 }
 
 }  // namespace
@@ -429,10 +637,11 @@ cudaError_t launch_decode(const DecodeLaunch& p, cudaStream_t st) {
     a.flags = p.flags;
     a.timeout_ns = p.timeout_ns;
     const size_t smem = decode_smem_bytes(p.g);
-    cudaError_t e = cudaFuncSetAttribute(decode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    auto kern = p.tc ? decode_kernel<true> : decode_kernel<false>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)smem);
     if (e == cudaSuccess && p.g.csize > 8)
-        e = cudaFuncSetAttribute(decode_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
     const int blocks = (p.B + kRows - 1) / kRows;
     cudaLaunchConfig_t cfg = {};
@@ -448,10 +657,10 @@ cudaError_t launch_decode(const DecodeLaunch& p, cudaStream_t st) {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int clusters = 0;
-    e = cudaOccupancyMaxActiveClusters(&clusters, decode_kernel, &cfg);
+    e = cudaOccupancyMaxActiveClusters(&clusters, kern, &cfg);
     if (e != cudaSuccess) return e;
     if (clusters < 1) return cudaErrorInvalidConfiguration;
-    return cudaLaunchKernelEx(&cfg, decode_kernel, a);
+    return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
 cudaError_t decode_error_word_read_clear(int* word) {

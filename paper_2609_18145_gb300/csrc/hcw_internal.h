@@ -213,6 +213,7 @@ struct DecodeLaunch {
     int L, B;
     unsigned flags;
     unsigned long long timeout_ns;
+    bool tc;   // contraction on tcgen05 (else the warp-level MMA)
 };
 // One launch of every layer of the step: a cluster per 16 rows.
 cudaError_t launch_decode(const DecodeLaunch& p, cudaStream_t st);

@@ -30,6 +30,8 @@ HCW_ERR_WORKSPACE = 7
 HCW_STACK_AUTO = 0
 HCW_STACK_RESIDENT = 1
 HCW_STACK_STREAMING = 2
+HCW_DECODE_WARP_MMA = 0
+HCW_DECODE_TCGEN05 = 1
 
 HCW_BF16 = 0
 HCW_F32 = 1
@@ -90,6 +92,7 @@ _SIGNATURES = {
     "hcw_gemm_workspace_bytes": ([_I, _I, _I], _SZ),
     "hcw_gemm_bf16": ([_I, _I, _I, _P, _I, _P, _I, _P, _P, _SZ, _P], _I),
     "hcw_set_stack_kernels": ([_I], _I),
+    "hcw_set_decode_kernel": ([_I], _I),
     "hcw_stack_kernels_used": ([_I, _I, _I, _I], _I),
     "hcw_sync_status": ([_P], _I),
     "hcw_selftest_wait": ([_LL, _P], _I),
@@ -350,6 +353,15 @@ def hcw_gemm_bf16(A, B, ta: bool = False, tb: bool = False, C=None, workspace=No
     _check(lib().hcw_gemm_bf16(M, N, K, _ptr(A), int(bool(ta)), _ptr(B), int(bool(tb)), _ptr(C),
                                wp, wn, _stream(stream)), "hcw_gemm_bf16")
     return C
+
+
+def hcw_set_decode_kernel(mode: int) -> int:
+    """Select the contraction of hcw_decode_step (HCW_DECODE_WARP_MMA or
+    HCW_DECODE_TCGEN05) for this process; returns the previous mode."""
+    prev = int(lib().hcw_set_decode_kernel(int(mode)))
+    if prev < 0:
+        raise ValueError("hcw_set_decode_kernel: unknown mode %r" % (mode,))
+    return prev
 
 
 def hcw_set_stack_kernels(mode: int) -> int:

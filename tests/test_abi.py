@@ -376,3 +376,16 @@ def test_gemm_workspace_sizes(hcw):
     assert hcw.hcw_gemm_workspace_bytes(16384, 1024, 512) == 0
     assert hcw.hcw_gemm_workspace_bytes(256, 256, 128) == 0
     assert hcw.hcw_gemm_workspace_bytes(0, 256, 128) == 0
+
+
+def test_decode_kernel_switch(hcw):
+    """hcw_set_decode_kernel returns the previous contraction and refuses an
+    unknown one without changing it."""
+    L = hcw.lib()
+    prev = L.hcw_set_decode_kernel(hcw.HCW_DECODE_TCGEN05)
+    try:
+        assert prev in (hcw.HCW_DECODE_WARP_MMA, hcw.HCW_DECODE_TCGEN05)
+        assert L.hcw_set_decode_kernel(7) == -1
+        assert L.hcw_set_decode_kernel(hcw.HCW_DECODE_WARP_MMA) == hcw.HCW_DECODE_TCGEN05
+    finally:
+        L.hcw_set_decode_kernel(prev)

@@ -470,8 +470,17 @@ DECODE_CASES = [
 ]
 
 
+@pytest.fixture(params=["warp_mma", "tcgen05"])
+def decode_kernel(H, request):
+    """Run the test under each contraction of hcw_decode_step."""
+    mode = H.HCW_DECODE_WARP_MMA if request.param == "warp_mma" else H.HCW_DECODE_TCGEN05
+    prev = H.hcw_set_decode_kernel(mode)
+    yield request.param
+    H.hcw_set_decode_kernel(prev)
+
+
 @pytest.mark.parametrize("case", DECODE_CASES, ids=lambda c: c[0])
-def test_decode_steps_reproduce_the_window_forward(H, case):
+def test_decode_steps_reproduce_the_window_forward(H, case, decode_kernel):
     """Sec. 6: decoding one token at a time with bounded rings gives, at every
     position t, the output row t of the stack run over the whole window: the
     oracle's forward (bf16 storage) at the bf16 tolerance, and the device's
@@ -501,7 +510,7 @@ def test_decode_steps_reproduce_the_window_forward(H, case):
     assert rel(host(ys), host(y)) <= TOL_BF16, name
 
 
-def test_decode_full_size_window(H):
+def test_decode_full_size_window(H, decode_kernel):
     """The decode shape bench.py times (64 sequences, window 256, d = 512, 16
     rotated causal layers): every position of every sequence equals the
     device's stack forward over the window, and the first two sequences equal
@@ -526,7 +535,7 @@ def test_decode_full_size_window(H):
     assert rel(host(ys[:2]), ry) <= TOL_BF16
 
 
-def test_decode_windows_back_to_back_share_the_cache(H):
+def test_decode_windows_back_to_back_share_the_cache(H, decode_kernel):
     """A new window restarts at t = 0 on the same rings; its outputs are those
     of a fresh decode on a cache full of garbage, bit for bit (no slot is read
     before it is written)."""
