@@ -254,16 +254,18 @@ __global__ void relu_grad_mask_kernel(const V* __restrict__ dy, const uint32_t* 
     }
 }
 
-constexpr int kColRows = 256;   // rows per partial of the column sum
+// rows per partial of the column sum: 64 up to 65,536 rows (enough CTAs to
+// fill the GPU), 256 above (the partials stay small)
+inline long long col_rows(long long rows) { return rows <= 65536 ? 64 : 256; }
 
 // partial[c][o] = sum_{r in chunk c} dz[r][o] for any d (block: 32 columns x
 // 8 row lanes).
 __global__ void colsum_partial_f32_kernel(const float* __restrict__ dz, long long rows, int d,
-                                          float* __restrict__ partial) {
+                                          int crows, float* __restrict__ partial) {
     __shared__ float red[8][33];
     const int o = blockIdx.x * 32 + threadIdx.x;
-    const long long r0 = (long long)blockIdx.y * kColRows;
-    const long long r1 = min(rows, r0 + kColRows);
+    const long long r0 = (long long)blockIdx.y * crows;
+    const long long r1 = min(rows, r0 + crows);
     float acc = 0.f;
     if (o < d)
         for (long long r = r0 + threadIdx.y; r < r1; r += 8) acc += dz[r * d + o];
@@ -280,7 +282,7 @@ __global__ void colsum_partial_f32_kernel(const float* __restrict__ dz, long lon
 // column groups of 16 bytes x 4 row lanes; each thread sums its group over every 4th row of
 // the chunk, then the 4 row lanes are added in a fixed order.
 template <typename V>
-__global__ void colsum_partial_kernel(const V* __restrict__ dz, long long rows, int d,
+__global__ void colsum_partial_kernel(const V* __restrict__ dz, long long rows, int d, int crows,
                                       float* __restrict__ partial) {
     constexpr int VEC = 16 / sizeof(V);
     __shared__ float red[4][64][VEC + 1];
@@ -289,8 +291,8 @@ __global__ void colsum_partial_kernel(const V* __restrict__ dz, long long rows, 
     partial += (size_t)blockIdx.z * gridDim.y * d;
     const int gpr = d / VEC;
     const int g = blockIdx.x * 64 + threadIdx.x;
-    const long long r0 = (long long)blockIdx.y * kColRows;
-    const long long r1 = min(rows, r0 + kColRows);
+    const long long r0 = (long long)blockIdx.y * crows;
+    const long long r1 = min(rows, r0 + crows);
     float acc[VEC];
 #pragma unroll
     for (int i = 0; i < VEC; ++i) acc[i] = 0.f;
@@ -316,15 +318,29 @@ __global__ void colsum_partial_kernel(const V* __restrict__ dz, long long rows, 
     }
 }
 
-__global__ void colsum_final_kernel(const float* __restrict__ partial, int chunks, int d,
-                                    float* __restrict__ out) {
-    const int o = blockIdx.x * blockDim.x + threadIdx.x;
+// out[o] = sum over the chunks c of partial[c][o], in chunk order: a CTA of 32
+// warps per 32 columns, a column a lane; warp w adds chunks w, w + 32, ...,
+// then the warp sums meet in shared memory in warp order.
+__global__ void __launch_bounds__(1024) colsum_final_kernel(const float* __restrict__ partial,
+                                                            int chunks, int d,
+                                                            float* __restrict__ out) {
+    __shared__ float red[32][33];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int o = blockIdx.x * 32 + lane;
     partial += (size_t)blockIdx.y * chunks * d;
     out += (size_t)blockIdx.y * d;
-    if (o >= d) return;
     float s = 0.f;
-    for (int c = 0; c < chunks; ++c) s += partial[(long long)c * d + o];
-    out[o] = s;
+    if (o < d) {
+#pragma unroll 4
+        for (int c = warp; c < chunks; c += 32) s += partial[(long long)c * d + o];
+    }
+    red[warp][lane] = s;
+    __syncthreads();
+    if (warp == 0 && o < d) {
+        float t = 0.f;
+        for (int w = 0; w < 32; ++w) t += red[w][lane];
+        out[o] = t;
+    }
 }
 
 __global__ void splitk_reduce_kernel(const float* __restrict__ partial, int splits_max,
@@ -434,27 +450,28 @@ cudaError_t launch_relu_grad_bf16(const __nv_bfloat16* dy, const __nv_bfloat16* 
 }
 
 size_t colsum_workspace_bytes(long long rows, int d) {
-    const long long chunks = (rows + kColRows - 1) / kColRows;
+    const long long chunks = (rows + col_rows(rows) - 1) / col_rows(rows);
     return (size_t)(chunks < 1 ? 1 : chunks) * (size_t)d * sizeof(float);
 }
 
 template <typename V>
 static cudaError_t colsum(const V* dz, long long rows, int d, float* partial, float* out,
                           cudaStream_t st, int batch = 1) {
-    const long long chunks = (rows + kColRows - 1) / kColRows;
+    const int crows = (int)col_rows(rows);
+    const long long chunks = (rows + crows - 1) / crows;
     if (chunks == 0) {
         cudaError_t e = cudaMemsetAsync(out, 0, (size_t)batch * d * sizeof(float), st);
         return e;
     }
     if (sizeof(V) == 4) {
         colsum_partial_f32_kernel<<<dim3((d + 31) / 32, (unsigned)chunks, 1), dim3(32, 8), 0, st>>>(
-            reinterpret_cast<const float*>(dz), rows, d, partial);
+            reinterpret_cast<const float*>(dz), rows, d, crows, partial);
     } else {
         constexpr int VEC = 16 / sizeof(V);
         dim3 grid((d / VEC + 63) / 64, (unsigned)chunks, (unsigned)batch);
-        colsum_partial_kernel<V><<<grid, dim3(64, 4), 0, st>>>(dz, rows, d, partial);
+        colsum_partial_kernel<V><<<grid, dim3(64, 4), 0, st>>>(dz, rows, d, crows, partial);
     }
-    colsum_final_kernel<<<dim3((d + 127) / 128, batch), 128, 0, st>>>(partial, (int)chunks, d, out);
+    colsum_final_kernel<<<dim3((d + 31) / 32, batch), 1024, 0, st>>>(partial, (int)chunks, d, out);
     return cudaGetLastError();
 }
 
