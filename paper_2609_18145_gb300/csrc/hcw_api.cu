@@ -107,6 +107,24 @@ bool map_rows_blocks(CUtensorMap* m, const void* base, long long tokens, int d, 
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Activations [samples][n][d] bf16 as (64 features, position, sample, d / 64
+// blocks), box (64, 64 positions, 1, nblk): 64 consecutive positions of one
+// sample; positions outside [0, n) load as zeros (a shift layer's partner rows,
+// read at p - k).
+bool map_positions_blocks(CUtensorMap* m, const void* base, long long tokens, int n, int d,
+                          int nblk) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc || !base || n < 64) return false;
+    cuuint64_t dims[4] = {64, (cuuint64_t)n, (cuuint64_t)(tokens / n), (cuuint64_t)(d / 64)};
+    cuuint64_t strides[3] = {(cuuint64_t)d * 2, (cuuint64_t)n * d * 2, 128};
+    cuuint32_t box[4] = {64, 64, 1, (cuuint32_t)nblk};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides,
+               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Weights W[o][i] as (64 i, o, d / 64 i-blocks), box (64, 64 o, nblk): nblk
 // consecutive 64-column blocks of 64 rows in one copy (the MN-major B
 // operand of the input gradient), 128-byte swizzle.
@@ -980,7 +998,18 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
     const size_t ab = sh.act_bytes;
     const WsLayout wl = ws_layout(sh.tokens, d, HCW_BF16, a.flags);
     int* sched = reinterpret_cast<int*>(a.ws);
-    if (a.sc.has_shift(L)) {
+    // Shift layers join the batched launch on SM pairs (their partner rows come
+    // from a (position, sample) view, 64 positions of one sample per stage,
+    // hence n >= 128); otherwise every layer runs on its own.
+    const WPlan wp = plan_dw(sh.tokens, d, a.flags);
+    const bool shift_batched = sh.n >= 128 && BN >= 128 && wp.n_ot % 2 == 0 && [&] {
+        for (int l0 = 0; l0 < L; l0 += kMaxStackLayers) {
+            const int cnt = L - l0 < kMaxStackLayers ? L - l0 : kMaxStackLayers;
+            if (5 * cnt * wp.n_ot * wp.n_nt < 3 * sm_count()) return false;
+        }
+        return true;
+    }();
+    if (a.sc.has_shift(L) && !shift_batched) {
         // layer by layer; a shift layer's dW_nbr = sum_t (S_{-k} dz)_t^T x_t, the
         // self-part GEMM of the readers' dz against the layer input
         uint8_t* wws = a.ws + 256;
@@ -1044,7 +1073,9 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
         memset(&T, 0, sizeof(T));
         for (int i = 0; i < cnt; ++i) {
             const int l = l0 + i;
-            const int s = a.sc.dim(sh, l);
+            const int sl = a.sc.dim(sh, l);
+            // a shift layer's rows are grouped as a hypercube view with k = 64
+            const int s = sl >= 0 ? sl : 6;
             const int k = 1 << s;
             CUtensorMap* m = T.maps[i];
             if (!map_rows_blocks(&m[0], dz(l), sh.tokens, d, k, 64, 2) ||
@@ -1054,9 +1085,12 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
                 return HCW_ERR_CUDA;
             m[2] = m[1];
             m[3] = m[4];
+            if (sl < 0 && !map_positions_blocks(&m[2], act(l), sh.tokens, sh.n, d, BN / 128))
+                return HCW_ERR_CUDA;
             T.layer[i] = {s, k, nullptr, nullptr, nullptr, false, nullptr, false,
                           a.dbias ? a.dbias + (size_t)l * d : nullptr,
                           a.dWs + (size_t)l * d * d, a.dWn + (size_t)l * d * d};
+            T.layer[i].shift = sl < 0 ? -sl : 0;
         }
         // One unit per (layer, output tile) accumulating the self and the partner
         // part together reads each dz and input block once (the separate parts
@@ -1068,7 +1102,7 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
         if (paired)
             for (int i = 0; i < cnt; ++i) {
                 const int l = l0 + i;
-                const int k = 1 << a.sc.dim(sh, l);
+                const int k = 1 << T.layer[i].s;
                 if (!map_rows_blocks(&T.maps[i][1], act(l), sh.tokens, d, k, 64, BN / 128))
                     return HCW_ERR_CUDA;
             }
@@ -1087,6 +1121,7 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
         p.splits_max = 1;
         p.causal = (a.flags & HCW_CAUSAL) ? 1 : 0;
         p.n_units = fused ? tiles : tiles * 2;
+        p.seq_n = sh.n;
         p.timeout_ns = g_timeout_ns;
         T.n_layers = cnt;
         T.sched = sched;

@@ -1519,24 +1519,31 @@ struct __align__(8) PairBarriers {
     int abort;
 };
 
-template <int BN>
-__host__ __device__ constexpr int pair_stage_bytes() { return kABytes + (BN / 2) * kBlockK * 2; }
-template <int BN>
+// A stage: this CTA's dz rows (A), its input columns (B) and, in a launch
+// with shift layers, the same columns of the rows `shift` positions earlier (B2).
+template <int BN, bool SHIFT>
+__host__ __device__ constexpr int pair_stage_bytes() {
+    return kABytes + (SHIFT ? 2 : 1) * (BN / 2) * kBlockK * 2;
+}
+template <int BN, bool SHIFT>
 __host__ __device__ constexpr int pair_stages() {
-    return ((kRingBytesDwf / pair_stage_bytes<BN>()) > 8 ? 8
-                                                         : (kRingBytesDwf / pair_stage_bytes<BN>())) &
+    return ((kRingBytesDwf / pair_stage_bytes<BN, SHIFT>()) > 8
+                ? 8
+                : (kRingBytesDwf / pair_stage_bytes<BN, SHIFT>())) &
            ~1;
 }
-template <int BN>
+template <int BN, bool SHIFT>
 __host__ __device__ constexpr size_t pair_smem_total() {
-    return 1024 + (size_t)pair_stages<BN>() * pair_stage_bytes<BN>() + sizeof(PairBarriers);
+    return 1024 + (size_t)pair_stages<BN, SHIFT>() * pair_stage_bytes<BN, SHIFT>() +
+           sizeof(PairBarriers);
 }
 
-template <int BN>
+template <int BN, bool SHIFT>
 __global__ void __launch_bounds__(cta_threads(BN), 1)
     hcw_dwp_kernel(const __grid_constant__ TcLaunch<kMaxStackLayers> L) {
-    constexpr int STAGES = pair_stages<BN>();
-    constexpr int SB = pair_stage_bytes<BN>();
+    constexpr int STAGES = pair_stages<BN, SHIFT>();
+    constexpr int SB = pair_stage_bytes<BN, SHIFT>();
+    constexpr int B2_OFF = kABytes + (BN / 2) * kBlockK * 2;   // SHIFT: the B2 tile
     constexpr int NH = BN / 2;                          // B columns per CTA
     constexpr uint32_t TMEM_COLS = 2 * BN;              // self and partner accumulators
     constexpr uint32_t IDESC = idesc_bf16_f32(2 * kBlockM, BN, 1, 1);
@@ -1605,7 +1612,10 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                             break;
                         }
                         uint8_t* sA = smem + (size_t)stage * SB;
-                        if (rank == 0) mbar_arrive_expect_tx(&bars->full[stage], 2 * SB);
+                        const bool shl = SHIFT && ly.shift > 0;
+                        if (rank == 0)
+                            mbar_arrive_expect_tx(&bars->full[stage],
+                                                  2 * (shl ? SB : B2_OFF));
                         issued_mask |= 1u << stage;
                         issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
                         const uint32_t fb = mapa_shared(&bars->full[stage], 0);
@@ -1613,6 +1623,14 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                                          (2 * tp + (int)rank) * (kBlockM / 64));
                         tma_load_5d_pair(sA + kABytes, &L.maps[l][1], fb, 0, lo0, bit, hi0,
                                          nt * (BN / 64) + (int)rank * (NH / 64));
+                        if (shl) {
+                            // the stage's 64 positions p of one sample, and the same
+                            // columns at p - shift (zeros before the sample's start)
+                            const long long tok = (long long)hi0 * 2 * ly.k + bit * ly.k + lo0;
+                            const int smp = (int)(tok / p.seq_n), pos = (int)(tok % p.seq_n);
+                            tma_load_4d_pair(sA + B2_OFF, &L.maps[l][2], fb, 0, pos - ly.shift,
+                                             smp, nt * (BN / 64) + (int)rank * (NH / 64));
+                        }
                         if (++stage == STAGES) {
                             stage = 0;
                             phase ^= 1;
@@ -1658,13 +1676,24 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
 #pragma unroll
                     for (int kk = 0; kk < kBlockK / 16; ++kk)
                         mma_bf16_f32_pair(d_self, dsc(a1, kk), dsc(x1, kk), IDESC, 1);
-#pragma unroll
-                    for (int kk = 0; kk < kBlockK / 16; ++kk)
-                        mma_bf16_f32_pair(d_nbr, dsc(a1, kk), dsc(x0, kk), IDESC, (pq | kk) != 0);
-                    if (!p.causal) {
+                    if (SHIFT && L.layer[u / upl].shift > 0) {
+                        // a shift layer: every row's partner is the row shift earlier
+                        const uint32_t y0 = a0 + B2_OFF, y1 = a1 + B2_OFF;
 #pragma unroll
                         for (int kk = 0; kk < kBlockK / 16; ++kk)
-                            mma_bf16_f32_pair(d_nbr, dsc(a0, kk), dsc(x1, kk), IDESC, 1);
+                            mma_bf16_f32_pair(d_nbr, dsc(a0, kk), dsc(y0, kk), IDESC, (pq | kk) != 0);
+#pragma unroll
+                        for (int kk = 0; kk < kBlockK / 16; ++kk)
+                            mma_bf16_f32_pair(d_nbr, dsc(a1, kk), dsc(y1, kk), IDESC, 1);
+                    } else {
+#pragma unroll
+                        for (int kk = 0; kk < kBlockK / 16; ++kk)
+                            mma_bf16_f32_pair(d_nbr, dsc(a1, kk), dsc(x0, kk), IDESC, (pq | kk) != 0);
+                        if (!p.causal) {
+#pragma unroll
+                            for (int kk = 0; kk < kBlockK / 16; ++kk)
+                                mma_bf16_f32_pair(d_nbr, dsc(a0, kk), dsc(x1, kk), IDESC, 1);
+                        }
                     }
                     any = true;
                     mma_commit_pair(&bars->consumed[stage], 3);
@@ -1803,11 +1832,11 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
     }
 }
 
-template <int BN>
+template <int BN, bool SHIFT>
 static cudaError_t launch_pair(const TcLaunch<kMaxStackLayers>& L, int grid, cudaStream_t st) {
-    constexpr size_t smem = pair_smem_total<BN>();
+    constexpr size_t smem = pair_smem_total<BN, SHIFT>();
     static_assert(smem <= 232448, "shared memory budget");
-    auto kern = hcw_dwp_kernel<BN>;
+    auto kern = hcw_dwp_kernel<BN, SHIFT>;
     static std::atomic<uint64_t> configured[4] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -1890,8 +1919,12 @@ cudaError_t launch_tc(int mode, int BN, const TcLaunch<1>& L, int grid, cudaStre
 cudaError_t launch_tc_stack(int mode, int BN, const TcLaunch<kMaxStackLayers>& L, int grid,
                             cudaStream_t st) {
     if (mode == MODE_DWP) {
-        if (BN == 256) return launch_pair<256>(L, grid, st);
-        if (BN == 128) return launch_pair<128>(L, grid, st);
+        bool shift = false;
+        for (int i = 0; i < L.n_layers; ++i) shift = shift || L.layer[i].shift > 0;
+        if (BN == 256) return shift ? launch_pair<256, true>(L, grid, st)
+                                    : launch_pair<256, false>(L, grid, st);
+        if (BN == 128) return shift ? launch_pair<128, true>(L, grid, st)
+                                    : launch_pair<128, false>(L, grid, st);
         return cudaErrorInvalidValue;
     }
 #define HCW_TC_STACK_CASE(M, N) \

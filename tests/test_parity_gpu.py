@@ -361,6 +361,12 @@ SCHEDULE_CASES = [
      [-1, 7, -1, -1, 5, -1, 4, -1, -1, 2, -1, 1, -1, 0]),
     # long shifts, no activation, d = 256 tiles
     ("long_shifts_n128_d256", "auto", 4, 128, 256, RESIDUAL, [-3, -64, 2, -127, -1]),
+    # enough layers and tiles at d = 512 for the batched weight-gradient launch
+    # on SM pairs, shift layers included (their partner rows read at p - k)
+    ("hybrid256_n256_d512_batched_dw", "auto", 2, 256, 512, CAUSAL | RESIDUAL | RELU,
+     [-1, 7, -1, -1, 5, -1, 4, -1, -1, 2, -1, 1, -1, 0]),
+    ("long_shifts_n256_d512_batched_dw", "auto", 2, 256, 512, RESIDUAL,
+     [-3, -64, 2, -127, -1, 5, -200, 0, -1, 7, -2, 3, -130, -255]),
 ]
 
 
