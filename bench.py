@@ -453,8 +453,8 @@ def run_ours(args):
                       dtype=torch.uint8, device=dev)
     reps = 5
     if dims is not None:
-        # a schedule with shift layers runs layer by layer: time its forward and
-        # its backward (input and weight gradients) as two launch sequences
+        # a schedule with shift layers: time its forward and its backward (input
+        # and weight gradients) as two launch sequences
         f_ms = time_calls(lambda i: H.hcw_stack_fwd(x, Ws, Wn, bias, 0, -1, flags, y=y,
                                                     acts=acts, masks=masks, workspace=fws,
                                                     dims=dims), reps)
@@ -462,8 +462,8 @@ def run_ours(args):
                                                     dx=dx, dW_self=gWs, dW_nbr=gWn, dbias=gb,
                                                     workspace=ws, dims=dims), reps)
         f_flops = step_flops(B, n, d, L, dims) / 3.0
-        kflops = {"forward of the %s schedule, layer by layer" % args.schedule: f_flops,
-                  "backward of the %s schedule (input and weight gradients), layer by layer"
+        kflops = {"forward of the %s schedule" % args.schedule: f_flops,
+                  "backward of the %s schedule (input and weight gradients)"
                   % args.schedule: 2.0 * f_flops}
         kernels = dict(zip(kflops, (f_ms, b_ms)))
         dwb_ms = dw_ms = 0.0
@@ -619,7 +619,7 @@ def run_ours(args):
                        "act": "relu", "bias": True,
                        "l2": "flushed before every timed step (256 MiB write, untimed)",
                        "parallelism": "replicas" if world > 1 else "single",
-                       "stack_kernels": ("layer by layer" if dims is not None else
+                       "stack_kernels": ("shift schedule" if dims is not None else
                                          "resident" if family == H.HCW_STACK_RESIDENT
                                          else "streaming"),
                        "schedule": args.schedule,

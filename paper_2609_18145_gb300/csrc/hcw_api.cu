@@ -125,6 +125,25 @@ bool map_positions_blocks(CUtensorMap* m, const void* base, long long tokens, in
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Activations [samples][n][d] bf16 as (d, position, sample, 1), box (64
+// features, box_rows positions, 1, 1), 128-byte swizzle: box_rows consecutive
+// positions of one sample; positions outside [0, n) load as zeros (the
+// partner rows of a shift layer in a stacked launch).
+bool map_positions(CUtensorMap* m, const void* base, long long tokens, int n, int d,
+                   int box_rows) {
+    EncodeTiledFn enc = encode_fn();
+    if (!enc || !base || n < box_rows) return false;
+    cuuint64_t dims[4] = {(cuuint64_t)d, (cuuint64_t)n, (cuuint64_t)(tokens / n), 1};
+    cuuint64_t strides[3] = {(cuuint64_t)d * 2, (cuuint64_t)n * d * 2,
+                             (cuuint64_t)tokens * d * 2};
+    cuuint32_t box[4] = {64, (cuuint32_t)box_rows, 1, 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides,
+               box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // Weights W[o][i] as (64 i, o, d / 64 i-blocks), box (64, 64 o, nblk): nblk
 // consecutive 64-column blocks of 64 rows in one copy (the MN-major B
 // operand of the input gradient), 128-byte swizzle.
@@ -259,6 +278,12 @@ struct Sched {
 // Row grouping of a shift layer's launches: any cube dimension serves (the
 // partner rows come row-aligned from a second tensor); 2^6 = 64-row runs.
 int shift_group_dim(const Shape& sh) { return sh.b - 1 < 6 ? sh.b - 1 : 6; }
+
+// Stacked forward / input-gradient launches take shift layers when a 128-row
+// unit lies inside one sample and the tokens form whole 256-token row-block
+// pairs (the k = 128 grouping): n >= 128, tokens a multiple of 256.
+constexpr int kShiftStackDim = 7;
+bool shift_stackable(const Shape& sh) { return sh.n >= 128 && sh.tokens % 256 == 0; }
 
 // Bytes of one layer's ReLU mask: ceil(d/32) 32-bit words per token.
 size_t mask_bytes(const Shape& sh) { return (size_t)sh.tokens * ((sh.d + 31) / 32) * 4; }
@@ -467,13 +492,18 @@ int stack_fwd_group(const Shape& sh, int l0, int n, const Sched& sc,
     memset(&L, 0, sizeof(L));
     for (int i = 0; i < n; ++i) {
         const int l = l0 + i;
-        const int s = sc.dim(sh, l);
-        if (!fwd_maps(L.maps[i], sh, s, in_ptr(l), Ws + l * wb, Wn + l * wb, out_ptr(l), pair))
+        const int sl = sc.dim(sh, l);
+        // a shift layer: rows in runs of 128 positions, its input as positions
+        const int s = sl >= 0 ? sl : kShiftStackDim;
+        if (!fwd_maps(L.maps[i], sh, s, in_ptr(l), Ws + l * wb, Wn + l * wb, out_ptr(l), pair) ||
+            (sl < 0 && !map_positions(&L.maps[i][0], in_ptr(l), sh.tokens, sh.n, d, 128)))
             return HCW_ERR_CUDA;
         L.layer[i] = {s, 1 << s, bias ? bias + (size_t)l * d : nullptr, mask_ptr(l), nullptr,
                       true, nullptr, false};
+        L.layer[i].shift = sl < 0 ? -sl : 0;
     }
     row_unit_params(L.p, sh, BN, flags, false);
+    L.p.seq_n = sh.n;
     if (pair) pair_units(L.p);
     L.p.flags = flags;
     L.n_layers = n;
@@ -906,7 +936,8 @@ int stack_data_layers_bf16(const Shape& sh, const StackData& a, cudaStream_t st)
 }
 
 int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
-    if (a.sc.has_shift(a.L)) return stack_data_layers_bf16(sh, a, st);
+    if (a.sc.has_shift(a.L) && (!shift_stackable(sh) || use_resident(sh)))
+        return stack_data_layers_bf16(sh, a, st);
     if (use_resident(sh)) return stack_data_resident(sh, a, st);
     const int d = sh.d, BN = pick_bn(d), L = a.L;
     const bool relu = (a.flags & HCW_ACT_RELU) != 0;
@@ -941,7 +972,9 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
         memset(&T, 0, sizeof(T));
         for (int i = 0; i < cnt; ++i) {
             const int l = top - i;
-            const int s = a.sc.dim(sh, l);
+            const int sl = a.sc.dim(sh, l);
+            // a shift layer: rows in runs of 128 positions, dz as positions
+            const int s = sl >= 0 ? sl : kShiftStackDim;
             const int k = 1 << s;
             // stores: g_{l-1} (map 4) and dz_{l-1} (map 5); at l = 0 the stack's dx
             void* out = l == 0 ? a.dx : (relu ? (resid ? gbuf(l - 1) : nullptr) : dz(l - 1));
@@ -955,14 +988,18 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
                 !map_rows(&m[4], out ? out : dzo, sh.tokens, d, k, 32, pw) ||
                 !map_rows(&m[5], dzo ? dzo : out, sh.tokens, d, k, 32, pw))
                 return HCW_ERR_CUDA;
+            if (sl < 0 && !map_positions(&m[0], dz(l), sh.tokens, sh.n, d, 128))
+                return HCW_ERR_CUDA;
             T.layer[i] = {s, k, nullptr, nullptr, nullptr, out != nullptr,
                           dzo ? mask(l - 1) : nullptr, dzo != nullptr};
+            T.layer[i].shift = sl < 0 ? -sl : 0;
             // the g buffers written by this launch (not dy, not a previous launch's)
             if (keep_g && i > 0)
                 T.layer[i].g_discard = static_cast<const __nv_bfloat16*>(res);
         }
         row_unit_params(T.p, sh, BN, a.flags, true);
         if (pair) pair_units(T.p);
+        T.p.seq_n = sh.n;
         T.p.flags = a.flags & HCW_RESIDUAL;
         T.n_layers = cnt;
         T.counters = counters;
@@ -1341,7 +1378,7 @@ int stack_fwd_impl(const Shape& sh, const void* x, const void* W_self, const voi
         return want_mask ? reinterpret_cast<uint32_t*>(static_cast<uint8_t*>(masks) + (size_t)l * mb)
                          : nullptr;
     };
-    if (dtype == HCW_BF16 && sc.has_shift(L)) {
+    if (dtype == HCW_BF16 && sc.has_shift(L) && (!shift_stackable(sh) || use_resident(sh))) {
         // layer by layer; a shift layer reads its partner rows S_k x, materialised
         // row-aligned behind the counters of the workspace
         void* u = static_cast<uint8_t*>(workspace) + stack_counter_bytes(sh.tokens, L);
@@ -1373,7 +1410,7 @@ int stack_fwd_impl(const Shape& sh, const void* x, const void* W_self, const voi
         // up to kMaxStackLayers layers per persistent launch
         for (int l0 = 0; l0 < L; l0 += kMaxStackLayers) {
             const int cnt = L - l0 < kMaxStackLayers ? L - l0 : kMaxStackLayers;
-            if (use_resident(sh))
+            if (use_resident(sh) && !sc.has_shift(L))
                 rc = stack_fwd_resident(sh, l0, cnt, sc,
                                         static_cast<const uint8_t*>(W_self),
                                         static_cast<const uint8_t*>(W_nbr), bias, flags, in_ptr,

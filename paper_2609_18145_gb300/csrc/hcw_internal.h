@@ -44,7 +44,7 @@ struct TcParams {
     int splits_nbr;
     int causal;
     int n_units;    // units of one layer
-    int seq_n;      // MODE_DWP with shift layers: positions per sample
+    int seq_n;      // launches with shift layers: positions per sample
     // epilogue
     unsigned flags;
     int splits_max;
@@ -74,12 +74,15 @@ struct TcLayer {
     // patch's L2 lines once it has read them (nothing reads them again, and
     // the buffer is written anew two layers later), or null
     const __nv_bfloat16* g_discard;
-    // MODE_DWP: a shift layer of Eq. (1) by `shift` positions (0: a hypercube
-    // layer).  Its rows are grouped as a hypercube view with k = 64 (64
+    // A shift layer of Eq. (1) by `shift` positions (0: a hypercube layer).
+    // MODE_DWP: its rows are grouped as a hypercube view with k = 64 (64
     // consecutive positions per stage); map 2 views the layer input as (64
     // features, position, sample, d / 64 blocks), so the rows p - shift of a
     // stage's positions p load as one box, the ones before the sample's start
-    // as zeros
+    // as zeros.  Stacked FWD / DX: the rows are grouped with k = 128 (runs of
+    // 128 positions), and map 0 views the input as (features, position,
+    // sample, 1), so the partner rows p - shift (forward) or p + shift (input
+    // gradient) load as one box, zeros outside the sample
     int shift;
 };
 

@@ -129,7 +129,7 @@ struct RowUnit {
 };
 
 __device__ __forceinline__ RowUnit decode_row_unit(const TcParams& p, int u, bool stacked,
-                                                   bool mirror = false) {
+                                                   bool mirror = false, bool shift = false) {
     RowUnit r;
     const int per_bit = p.n_rb * p.n_nt;
     int g, rem;
@@ -146,6 +146,14 @@ __device__ __forceinline__ RowUnit decode_row_unit(const TcParams& p, int u, boo
         rem = u - r.t * 2 * p.n_nt;
         g = rem / p.n_nt;
         r.j = rem - g * p.n_nt;
+    }
+    if (shift) {
+        // a shift layer of Eq. (1) in a stacked launch: every row takes both
+        // parts (the rows before k read zeros); g picks one of the row block's
+        // two 128-token runs
+        r.beta = g;
+        r.steps = 2 * p.nK;
+        return r;
     }
     if (g < p.n_full) {
         r.beta = g == 0 ? p.full_bit0 : p.full_bit1;
@@ -167,6 +175,15 @@ __device__ __forceinline__ void row_unit_chunks(int q0, int s, int k, int& ca, i
     ca = tok_a >> 7;
     cb = k >= 128 ? ((tok_a + k) >> 7) : ca + 1;
 }
+
+// Bounded waits for the inputs of a shift-layer unit of a stacked launch: its
+// own 128 tokens [tok0, tok0 + 128) (positions pos0 .. pos0 + 127 of one
+// sample of n) and its partner rows at offset `off` (-k forward, +k input
+// gradient), clipped to the sample -- rows outside it load as zeros and are
+// nobody's output.  At most three 128-token chunks.
+__device__ bool wait_shift_chunks(const int* ctr, int n_chunks, int tokens, int d, int tok0,
+                                  int pos0, int n, int off, volatile int* abort,
+                                  uint64_t timeout_ns);
 
 // DW unit -> (which: 0 self / 1 partner, o tile, k tile, split, kb range)
 struct WUnit {
@@ -374,6 +391,27 @@ __device__ __forceinline__ bool wait_counters2(const int* c0, int t0, const int*
     }
     return wait_counter(c0, t0, abort, timeout_ns) &&
            (n < 2 || wait_counter(c1, t1, abort, timeout_ns));
+}
+
+__device__ bool wait_shift_chunks(const int* ctr, int n_chunks, int tokens, int d, int tok0,
+                                  int pos0, int n, int off, volatile int* abort,
+                                  uint64_t timeout_ns) {
+    int c[3];
+    int nc = 0;
+    c[nc++] = tok0 >> 7;
+    const int a = max(pos0 + off, 0), b = min(pos0 + off + 127, n - 1);
+    if (a <= b) {
+        const int base = tok0 - pos0;   // the sample's first token
+        const int ca = (base + a) >> 7, cb = (base + b) >> 7;
+        if (ca != c[0]) c[nc++] = ca;
+        if (cb != ca && cb != c[0]) c[nc++] = cb;
+    }
+    for (int i = 0; i < nc; ++i) {
+        if (c[i] >= n_chunks) continue;   // rows past the end: nothing to wait for
+        if (!wait_counter(ctr + c[i], min(128, tokens - (c[i] << 7)) * d, abort, timeout_ns))
+            return false;
+    }
+    return true;
 }
 
 // Bounded wait until the shared counter *p >= target (acquire); records a
@@ -618,24 +656,40 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     }
                 } else if (MODE != MODE_DW) {
                     const bool ufwd = is_fwd(l);
-                    RowUnit r = decode_row_unit(p, ul, STACKED, !ufwd && MODE == MODE_FDX);
+                    // a shift layer (stacked launches): map 0 views the input as
+                    // (features, position, sample, 1); the unit's 128 tokens are
+                    // positions pos0 .. pos0 + 127 of sample smp, their partners
+                    // pos0 + soff .. (zeros outside the sample)
+                    const bool shl = STACKED && ly.shift > 0;
+                    RowUnit r = decode_row_unit(p, ul, STACKED, !ufwd && MODE == MODE_FDX, shl);
                     if (PAIR) r.t = 2 * r.t + (int)rank;   // this CTA's half of the 256 rows
                     const int q0 = r.t * kBlockM;
                     const int lo0 = q0 & (ly.k - 1), hi0 = q0 >> ly.s;
+                    const int tok0 = (hi0 << (ly.s + 1)) + (r.beta << ly.s) + lo0;
+                    const int smp = shl ? tok0 / p.seq_n : 0;
+                    const int pos0 = shl ? tok0 - smp * p.seq_n : 0;
+                    const int soff = ufwd ? -ly.shift : ly.shift;
                     if (STACKED && (l > 0 || (MODE == MODE_DX && L.top_dy != nullptr))) {
                         // the unit's rows and their partners: two 128-token chunks,
                         // written by the layer before (or by this launch's prologue)
-                        int cs[2];
-                        row_unit_chunks(q0, ly.s, ly.k, cs[0], cs[1]);
                         const int* ctr = l > 0 ? L.counters + (size_t)(l - 1) * L.n_chunks
                                                : L.in_counters;
-                        // chunks past the end (ragged tail) have nothing to wait for
-                        const int nc = (cs[0] < L.n_chunks) + (cs[1] < L.n_chunks);
-                        if (cs[0] >= L.n_chunks) cs[0] = cs[1];
-                        if (nc > 0)
-                            ok = wait_counters2(
-                                ctr + cs[0], min(128, L.tokens - (cs[0] << 7)) * p.d, ctr + cs[1],
-                                min(128, L.tokens - (cs[1] << 7)) * p.d, nc, abort, tmo);
+                        if (shl) {
+                            ok = wait_shift_chunks(ctr, L.n_chunks, L.tokens, p.d, tok0, pos0,
+                                                   p.seq_n, soff, abort, tmo);
+                        } else {
+                            int cs[2];
+                            row_unit_chunks(q0, ly.s, ly.k, cs[0], cs[1]);
+                            // chunks past the end (ragged tail) have nothing to wait for
+                            const int nc = (cs[0] < L.n_chunks) + (cs[1] < L.n_chunks);
+                            if (cs[0] >= L.n_chunks) cs[0] = cs[1];
+                            if (nc > 0)
+                                ok = wait_counters2(ctr + cs[0],
+                                                    min(128, L.tokens - (cs[0] << 7)) * p.d,
+                                                    ctr + cs[1],
+                                                    min(128, L.tokens - (cs[1] << 7)) * p.d, nc,
+                                                    abort, tmo);
+                        }
                         if (!ok) break;
                         fence_proxy_async_global();
                     }
@@ -654,14 +708,21 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                         // partner part: the rows of the other bit value, or (pair_rows)
                         // the same rows of the row-aligned partner tensor (map 5)
                         const bool same = part && ly.pair_rows;
-                        const int bitA = part && !same ? 1 - r.beta : r.beta;
                         const CUtensorMap* mAk = same ? &L.maps[l][5] : mA;
                         const CUtensorMap* mb = &L.maps[l][part ? 2 : 1];
+                        // A box coordinates after the feature block: (lo, bit, HI) of
+                        // the hypercube view, or (position, sample, 0) of a shift layer
+                        int c1 = lo0, c2 = part && !same ? 1 - r.beta : r.beta, c3 = hi0;
+                        if (shl) {
+                            c1 = part ? pos0 + soff : pos0;
+                            c2 = smp;
+                            c3 = 0;
+                        }
                         if (PAIR) {
                             // both CTAs' copies complete on the leader's barrier
                             if (rank == 0) mbar_arrive_expect_tx(&bars->full[stage], 2 * SB);
                             const uint32_t fb = mapa_shared(&bars->full[stage], 0);
-                            tma_load_4d_pair(sA, mAk, fb, kk * kBlockK, lo0, bitA, hi0);
+                            tma_load_4d_pair(sA, mAk, fb, kk * kBlockK, c1, c2, c3);
                             if (ufwd)
                                 tma_load_2d_pair(sB, mb, fb, kk * kBlockK,
                                                  r.j * BN + (int)rank * (BN / 2));
@@ -670,7 +731,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                                                  r.j * (BN / 64) + (int)rank * (BN / 128));
                         } else {
                             mbar_arrive_expect_tx(&bars->full[stage], kABytes + B_BYTES);
-                            tma_load_4d(sA, mAk, &bars->full[stage], kk * kBlockK, lo0, bitA, hi0);
+                            tma_load_4d(sA, mAk, &bars->full[stage], kk * kBlockK, c1, c2, c3);
                             if (ufwd)
                                 tma_load_2d(sB, mb, &bars->full[stage], kk * kBlockK, r.j * BN);
                             else   // BN / 64 blocks of 64 W columns x 64 rows, one copy
@@ -809,7 +870,9 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     b_lbo = 16;
                 }
                 if (MODE != MODE_DW) {
-                    steps = decode_row_unit(p, ul, STACKED).steps;
+                    steps = decode_row_unit(p, ul, STACKED, false,
+                                            STACKED && L.layer[u / upl].shift > 0)
+                                .steps;
                 } else {
                     int lw;
                     const WUnit w = decode_w_any(p, u, STACKED, L.n_layers, lw);
@@ -1099,7 +1162,8 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                 constexpr bool fwd = decltype(fwd_tag)::value;
                 constexpr int RB = WCOLS * 2;                  // patch row bytes (128 or 64)
                 constexpr int SUB = WCOLS / 32;                // 32-column sub-chunks per patch
-                RowUnit r = decode_row_unit(p, ul, STACKED, !fwd && MODE == MODE_FDX);
+                RowUnit r = decode_row_unit(p, ul, STACKED, !fwd && MODE == MODE_FDX,
+                                            STACKED && ly.shift > 0);
                 if (PAIR) r.t = 2 * r.t + (int)rank;
                 const int qw = r.t * kBlockM + quarter * 32;   // first compressed row of the warp
                 const int lo_w = qw & (ly.k - 1), hi_w = qw >> ly.s;

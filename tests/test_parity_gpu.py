@@ -367,6 +367,13 @@ SCHEDULE_CASES = [
      [-1, 7, -1, -1, 5, -1, 4, -1, -1, 2, -1, 1, -1, 0]),
     ("long_shifts_n256_d512_batched_dw", "auto", 2, 256, 512, RESIDUAL,
      [-3, -64, 2, -127, -1, 5, -200, 0, -1, 7, -2, 3, -130, -255]),
+    # n = 128 with an odd batch: the tokens are not whole 256-token row-block
+    # pairs, so shift schedules run layer by layer
+    ("shifts_n128_b3_layer_by_layer", "auto", 3, 128, 128, CAUSAL | RESIDUAL | RELU,
+     [-1, 6, -2, 3, -127, 0]),
+    # 20 layers: two stacked launches, shifts on both sides of the boundary
+    ("mixed20_n256_d256", "auto", 2, 256, 256, CAUSAL | RESIDUAL | RELU,
+     [-1, 7, -3, 6, -1, 5, -100, 4, -1, 3, -255, 2, -1, 1, -17, 0, -1, 7, -2, 6]),
 ]
 
 
