@@ -326,6 +326,19 @@ WPlan plan_dw(long long tokens, int d, unsigned flags) {
     return w;
 }
 
+// SM pairs of the batched weight-gradient launch of a training step when it
+// runs on pairs behind the fused forward / input-gradient launch (the
+// conditions of stack_weight_bf16 for one launch of <= kMaxStackLayers
+// layers), else 0.
+int dw_early_pairs(const Shape& sh, unsigned flags, int L) {
+    if (L > kMaxStackLayers || pick_bn(sh.d) < 128) return 0;
+    const WPlan w = plan_dw(sh.tokens, sh.d, flags);
+    const int tiles = w.n_ot * w.n_nt, sms = sm_count();
+    if (L * tiles * 2 < sms || 5 * L * tiles < 3 * sms || w.n_ot % 2 != 0) return 0;
+    const int total = tiles * L;
+    return total / 2 < sms / 2 ? total / 2 : sms / 2;
+}
+
 // Workspace of the weight gradient (bf16: dW split partials, both dtypes:
 // column-sum partials of dbias) and of the full layer backward, which adds
 // the masked gradient dz = dy * act'(z) in front when an activation is used:
@@ -825,6 +838,11 @@ struct StackWeight {
     float* dWn;
     float* dbias;
     uint8_t* ws;
+    // the fused forward / input-gradient launch just issued on the stream, or
+    // null: its completion counters, where row 2 L - 2 - l counts dz_l.  A
+    // batched launch on SM pairs then starts as its programmatic dependent
+    // and waits on those counters instead of the launch's end.
+    const int* fdx_counters = nullptr;
 };
 
 // bf16 input gradients on the resident kernels: one launch per run of <= 16
@@ -1162,7 +1180,17 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
         p.timeout_ns = g_timeout_ns;
         T.n_layers = cnt;
         T.sched = sched;
-        if (cudaMemsetAsync(sched, 0, sizeof(int), st) != cudaSuccess) return HCW_ERR_CUDA;
+        // the pair launch hands out its units statically (no unit counter); right
+        // behind the fused launch it starts early, on the SMs that launch leaves
+        const bool early = paired && a.fdx_counters != nullptr && L <= kMaxStackLayers;
+        if (early) {
+            T.dep_counters = a.fdx_counters;
+            T.n_chunks = (int)((sh.tokens + 127) / 128);
+            T.tokens = (int)sh.tokens;
+            for (int i = 0; i < cnt; ++i) T.layer[i].dep_row = 2 * L - 2 - (l0 + i);
+        } else if (cudaMemsetAsync(sched, 0, sizeof(int), st) != cudaSuccess) {
+            return HCW_ERR_CUDA;
+        }
         const int total = p.n_units * cnt;
         if (paired) {
             // clusters of two CTAs, one 256-row tile per cluster
@@ -1503,7 +1531,7 @@ size_t step_fwd_region(const Shape& sh, int dtype, unsigned flags, int L) {
 int step_fused_launch(const Shape& sh, const void* x, const uint8_t* Ws, const uint8_t* Wn,
                       const float* bias, const void* dy, const Sched& sc, int L, unsigned flags,
                       void* y, void* acts, void* masks, void* dx, uint8_t* dz, uint8_t* gws,
-                      int* counters, cudaStream_t st) {
+                      int* counters, cudaStream_t st, int dw_pairs = 0) {
     const int d = sh.d, BN = pick_bn(d), pw = epi_patch_cols(BN);
     const size_t ab = sh.act_bytes, a256 = align256(ab), wb = (size_t)d * d * 2;
     const size_t mb = mask_bytes(sh);
@@ -1579,6 +1607,20 @@ int step_fused_launch(const Shape& sh, const void* x, const uint8_t* Ws, const u
     const int sms = sm_count();
     const int total = T.p.n_units * 2 * L;
     const int pairs = total < sms / 2 ? total : sms / 2;
+    // With a weight-gradient launch of dw_pairs pairs right behind: the last
+    // layer runs on the pairs that launch leaves idle, when they get through it
+    // in well under the weight gradient's time (its units take K = 2d or d
+    // steps of 64; a weight-gradient unit takes three or four per 64 compressed
+    // rows of each bit value); the rest of the SMs go to the weight gradient
+    // as soon as they are done with the earlier layers.
+    if (dw_pairs > 0 && pairs == sms / 2 && pairs > dw_pairs) {
+        const int tail = pairs - dw_pairs;
+        const long long tail_steps =
+            (long long)T.p.n_units * (T.p.n_full == 2 ? 4 : 3) * T.p.nK / 2 / tail;
+        const long long dw_steps =
+            (long long)((T.p.Mh + 63) / 64) * ((flags & HCW_CAUSAL) ? 3 : 4);
+        if (4 * tail_steps <= 3 * dw_steps) T.tail_pairs = tail;
+    }
     return launched(launch_tc_step_pair(BN, T, 2 * pairs, st), 1);
 }
 
@@ -1646,9 +1688,11 @@ int train_step_impl(const Shape& sh, const void* x, const void* W_self, const vo
         return HCW_ERR_ALIASING;
     rc = step_fused_launch(sh, x, static_cast<const uint8_t*>(W_self),
                            static_cast<const uint8_t*>(W_nbr), bias, dy, sc, L, flags, y, acts,
-                           masks, dx, ws, ws + zb, reinterpret_cast<int*>(ws + bwd), st);
+                           masks, dx, ws, ws + zb, reinterpret_cast<int*>(ws + bwd), st,
+                           want_dw ? dw_early_pairs(sh, flags, L) : 0);
     if (rc || !want_dw) return rc;
-    StackWeight wa{x, acts, ws, sc, L, flags, dW_self, dW_nbr, dbias, ws + zb + db};
+    StackWeight wa{x, acts, ws, sc, L, flags, dW_self, dW_nbr, dbias, ws + zb + db,
+                   reinterpret_cast<const int*>(ws + bwd)};
     return stack_weight_bf16(sh, wa, st);
 }
 

@@ -84,6 +84,9 @@ struct TcLayer {
     // sample, 1), so the partner rows p - shift (forward) or p + shift (input
     // gradient) load as one box, zeros outside the sample
     int shift;
+    // MODE_DWP started early (TcLaunch::dep_counters): the row of the
+    // completion counters that counts this layer's dz
+    int dep_row;
 };
 
 // Columns of one epilogue patch (the inner extent of the 32-row residual and
@@ -125,6 +128,19 @@ struct TcLaunch {
     // MODE_FDX: the number of forward layers; the last of them also writes the
     // top layer's dz = dy * act'(z) (top_dy, top_dz) for the layers after it
     int n_fwd;
+    // MODE_DWP launched as a programmatic dependent of the MODE_FDX launch that
+    // writes its dz: that launch's completion counters [rows][n_chunks]
+    // (layer.dep_row picks a layer's row).  A unit first waits until every
+    // chunk of its layer's dz is complete; the layers go from the top down (the
+    // order in which the input gradient finishes them).  Null: the operands
+    // are complete when the launch starts.
+    const int* dep_counters;
+    // MODE_FDX followed by such a weight-gradient launch: only pairs
+    // [0, tail_pairs) take units of the last layer (the input gradient of
+    // layer 0, which nothing in the step reads); the others leave once every
+    // earlier unit is claimed, and the weight gradient starts on their SMs.
+    // 0: every pair takes units to the end.
+    int tail_pairs;
 };
 
 // Launch one tensor-core pass (one layer).
@@ -132,6 +148,8 @@ cudaError_t launch_tc(int mode, int BN, const TcLaunch<1>& L, int grid, cudaStre
 // Launch a run of layers: MODE_FWD (layers in order) or MODE_DX (layers from
 // the top down) with chunk-level dependencies, or MODE_DW (independent
 // layers, the long self-part units of every layer first).
+// MODE_DWP with L.dep_counters set is launched as a programmatic dependent of
+// the preceding kernel in the stream.
 cudaError_t launch_tc_stack(int mode, int BN, const TcLaunch<kMaxStackLayers>& L, int grid,
                             cudaStream_t stream);
 // The same for MODE_FWD / MODE_DX on clusters of two CTAs (256-row tiles,

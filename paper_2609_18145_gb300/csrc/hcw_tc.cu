@@ -414,6 +414,48 @@ __device__ bool wait_shift_chunks(const int* ctr, int n_chunks, int tokens, int 
     return true;
 }
 
+// Warp-wide bounded wait until every one of the n_chunks completion counters
+// ctr[c] shows its 128-token chunk complete (min(128, tokens - 128 c) * d
+// elements).  Each lane polls every 32nd counter; the lanes acquire what they
+// observed (a fence after the relaxed loads) and meet in a warp barrier before
+// any of them goes on.  Records a timeout like mbar_wait.
+__device__ bool wait_chunks_warp(const int* ctr, int n_chunks, int tokens, int d,
+                                 volatile int* abort, uint64_t timeout_ns) {
+    const int lane = threadIdx.x & 31;
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t it = 0;; ++it) {
+        bool mine = true;
+        for (int c0 = 0; c0 < n_chunks; c0 += 128) {
+            int v[4], need[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int c = c0 + lane + 32 * j;
+                need[j] = c < n_chunks ? min(128, tokens - (c << 7)) * d : 0;
+                v[j] = c < n_chunks ? ld_relaxed_gpu(ctr + c) : 0;
+            }
+#pragma unroll
+            for (int j = 0; j < 4; ++j) mine = mine && v[j] >= need[j];
+        }
+        if (__all_sync(0xffffffffu, mine)) {
+            fence_acq_rel_gpu();
+            __syncwarp();
+            return true;
+        }
+        __nanosleep(200);
+        int give_up = 0;
+        if (lane == 0 && (it & 15u) == 15u) {
+            if (*abort) {
+                give_up = 1;
+            } else if (globaltimer_ns() - t0 > timeout_ns) {
+                atomicExch(&g_error_word, kErrTimeout);
+                *abort = 1;
+                give_up = 1;
+            }
+        }
+        if (__shfl_sync(0xffffffffu, give_up, 0)) return false;
+    }
+}
+
 // Bounded wait until the shared counter *p >= target (acquire); records a
 // timeout like mbar_wait.
 template <bool CLUSTER = false>
@@ -505,8 +547,11 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
     const int lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
-        for (int l = 0; l < L.n_layers && l < NL; ++l)
-            for (int i = 0; i < kTcMaps; ++i) tma_prefetch_desc(&L.maps[l][i]);
+        // the first layer's tensor maps; the last epilogue warp prefetches the
+        // others while the first units load (a 32-layer launch's 192 maps in
+        // this thread took ~3.5 us of the prologue, and one layer's at a time
+        // in the producer lengthened every layer step)
+        for (int i = 0; i < kTcMaps; ++i) tma_prefetch_desc(&L.maps[0][i]);
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&bars->full[s], 1);
             // DW: the MMA commit and the helper warps (which read the dz tiles for
@@ -543,6 +588,10 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
     const uint32_t tmem_base = bars->tmem_base;
     volatile int* abort = &bars->abort;
     const uint64_t tmo = p.timeout_ns;
+    // the weight-gradient launch behind the fused one may take the SMs this
+    // launch's CTAs leave at its end; it waits for its operands on the
+    // completion counters (every CTA of this launch is resident by then)
+    if (MODE == MODE_FDX) pdl_trigger();
     // Stacked launches hand out units dynamically, in increasing order, from a
     // global counter: CTAs that draw short units take more of them, so no CTA
     // runs far behind the others and stalls the next layer's units.  The
@@ -579,7 +628,14 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                         break;
                     }
                 } else if (dyn) {
-                    u = atomicAdd(L.sched, 1);
+                    // a pair outside the tail pairs leaves once the last layer's
+                    // units are being handed out (a unit it still draws by a race
+                    // it runs: any CTA may run any unit)
+                    if (L.tail_pairs > 0 && ((int)blockIdx.x >> (PAIR ? 1 : 0)) >= L.tail_pairs &&
+                        ld_relaxed_gpu(L.sched) >= (L.n_layers - 1) * upl)
+                        u = n_units;
+                    else
+                        u = atomicAdd(L.sched, 1);
                     if (u >= n_units) u = -1;
                     // the slot's previous unit has been read by every consumer
                     if (ordinal >= kUnitQ &&
@@ -944,6 +1000,9 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
         const int cslice = e >> 2;
         uint8_t* buf = epi_smem + (size_t)e * kEpiBufBytes;
         float* wbias = bias_smem + e * WCOLS;
+        if (STACKED && e == EW - 1)
+            for (int i = kTcMaps + lane; i < L.n_layers * kTcMaps; i += 32)
+                tma_prefetch_desc(&L.maps[i / kTcMaps][i % kTcMaps]);
         uint32_t ld_phase = 0;
         int hstage = 0;          // DW helper warps: ring position, as the MMA thread's
         uint32_t hphase = 0;
@@ -1579,6 +1638,7 @@ struct __align__(8) PairBarriers {
     uint64_t tfull;
     uint64_t tempty;
     uint64_t drain;
+    uint64_t ring_idle;   // the helper warps are done with the CTA's last unit's stages
     uint32_t tmem_base;
     int abort;
 };
@@ -1614,6 +1674,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
     constexpr int EW = epi_warps(BN);
     constexpr int WCOLS = warp_cols(BN);
     static_assert(STAGES % 2 == 0 && STAGES >= 2, "pairs of stages");
+    static_assert(EW * 2 * kEpiBufBytes <= STAGES * SB, "patch buffers inside the ring");
     const TcParams& p = L.p;
     const uint32_t rank = cluster_ctarank();
     const int pair = (int)blockIdx.x >> 1, n_pairs = (int)gridDim.x >> 1;
@@ -1641,6 +1702,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
         mbar_init(&bars->tfull, 1);
         mbar_init(&bars->tempty, 2 * EW);
         mbar_init(&bars->drain, 1);
+        mbar_init(&bars->ring_idle, kDwHelpers);
         bars->abort = 0;
         fence_mbar_init();
     }
@@ -1656,17 +1718,35 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
     volatile int* abort = &bars->abort;
     const uint64_t tmo = p.timeout_ns;
 
+    // unit u -> (layer, tile); a launch behind the fused input gradient takes
+    // the layers from the top down, the order in which their dz complete
+    const bool dep = L.dep_counters != nullptr;
+    auto unit_layer = [&](int u, int& ul) {
+        const int lu = u / upl;
+        ul = u - lu * upl;
+        return dep ? L.n_layers - 1 - lu : lu;
+    };
+
     if (warp == 0) {
         // ------------------------------------------------------------ producer (both CTAs)
-        if (lane == 0) {
-            int stage = 0;
-            uint32_t phase = 0;
-            uint32_t issued_mask = 0, issued_phase = 0;
-            bool ok = true;
-            for (int u = pair; u < n_units && ok; u += n_pairs) {
-                const int l = u / upl, ul = u - l * upl;
-                const int tp = ul / p.n_nt, nt = ul - tp * p.n_nt;
-                const TcLayer& ly = L.layer[l];
+        // lane 0 issues the copies; the whole warp waits for a unit's operands
+        // when the launch started before they were complete
+        int stage = 0;
+        uint32_t phase = 0;
+        uint32_t issued_mask = 0, issued_phase = 0;
+        bool ok = true;
+        for (int u = pair; u < n_units && ok; u += n_pairs) {
+            int ul;
+            const int l = unit_layer(u, ul);
+            const int tp = ul / p.n_nt, nt = ul - tp * p.n_nt;
+            const TcLayer& ly = L.layer[l];
+            if (dep) {
+                ok = wait_chunks_warp(L.dep_counters + (size_t)ly.dep_row * L.n_chunks,
+                                      L.n_chunks, L.tokens, p.d, abort, tmo);
+                if (!ok) break;
+            }
+            if (lane == 0) {
+                if (dep) fence_proxy_async_global();   // the copies read what was acquired
                 for (int pq = 0; pq < p.qb && ok; ++pq) {
                     const int q0 = pq * 64;
                     const int lo0 = q0 & (ly.k - 1), hi0 = q0 >> ly.s;
@@ -1702,12 +1782,13 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     }
                 }
             }
-            if (!ok && rank == 0) {
-                // every copy of the pair completes on the leader's barriers: let them land
-                for (int s = 0; s < STAGES; ++s)
-                    if (issued_mask & (1u << s))
-                        mbar_wait_drain(&bars->full[s], (issued_phase >> s) & 1u, tmo);
-            }
+            ok = __shfl_sync(0xffffffffu, ok, 0) != 0;
+        }
+        if (!ok && rank == 0 && lane == 0) {
+            // every copy of the pair completes on the leader's barriers: let them land
+            for (int s = 0; s < STAGES; ++s)
+                if (issued_mask & (1u << s))
+                    mbar_wait_drain(&bars->full[s], (issued_phase >> s) & 1u, tmo);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer (leader)
@@ -1740,7 +1821,8 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
 #pragma unroll
                     for (int kk = 0; kk < kBlockK / 16; ++kk)
                         mma_bf16_f32_pair(d_self, dsc(a1, kk), dsc(x1, kk), IDESC, 1);
-                    if (SHIFT && L.layer[u / upl].shift > 0) {
+                    int ul_unused;
+                    if (SHIFT && L.layer[unit_layer(u, ul_unused)].shift > 0) {
                         // a shift layer: every row's partner is the row shift earlier
                         const uint32_t y0 = a0 + B2_OFF, y1 = a1 + B2_OFF;
 #pragma unroll
@@ -1788,10 +1870,12 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
         uint32_t hphase = 0, acc_phase = 0;
         bool alive = true;
         for (int u = pair; u < n_units && alive; u += n_pairs) {
-            const int l = u / upl, ul = u - l * upl;
+            int ul;
+            const int l = unit_layer(u, ul);
             const int tp = ul / p.n_nt, nt = ul - tp * p.n_nt;
             const int ot = 2 * tp + (int)rank;
             const TcLayer& ly = L.layer[l];
+            const bool last = u + n_pairs >= n_units;   // no further unit: the ring goes idle
             if (e < kDwHelpers) {
                 // release this CTA's stages once the pair's MMAs have read them, and
                 // sum the dz tile's columns on the way (dbias, output rows of tile ot)
@@ -1845,6 +1929,8 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                         dst[1] = make_float4(cs[4], cs[5], cs[6], cs[7]);
                     }
                 }
+                __syncwarp();
+                if (last && lane == 0) mbar_arrive(&bars->ring_idle);
             }
             const bool okt = mbar_wait(&bars->tfull, acc_phase, abort, tmo);
             if (!__all_sync(0xffffffffu, okt)) {
@@ -1852,6 +1938,16 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                 break;
             }
             tc_fence_after();
+            // The CTA's last unit: the ring is idle once the helper warps are done
+            // with it, so the tiles go out through shared memory by TMA (two 4 KB
+            // patch buffers per warp, whole 128-byte rows): per-lane row stores at
+            // the end of the launch, all SMs at once, took ~13 us to drain.
+            // Earlier units store from registers while the next unit's operands
+            // stream into the ring.
+            const bool staged =
+                last && __all_sync(0xffffffffu, mbar_wait(&bars->ring_idle, 0, abort, tmo));
+            uint8_t* sbuf = smem + (size_t)e * 2 * kEpiBufBytes;
+            int nbuf = 0;
             // this CTA's 128 rows of the tile: one row per lane, 32 fp32 columns per load
             const int row = ot * kBlockM + quarter * 32 + lane;
 #pragma unroll 1
@@ -1870,6 +1966,27 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                         __syncwarp();
                         if (lane == 0) mbar_arrive_remote_tmem(tempty_leader);
                     }
+                    if (staged) {
+                        uint8_t* buf = sbuf + (nbuf & 1) * kEpiBufBytes;
+                        // the buffer's store before last has been read
+                        if (lane == 0 && nbuf >= 2) bulk_wait_read<1>();
+                        __syncwarp();
+#pragma unroll
+                        for (int m = 0; m < 8; ++m)
+                            *patch_piece<128>(buf, lane, m) = make_uint4(
+                                raw[4 * m], raw[4 * m + 1], raw[4 * m + 2], raw[4 * m + 3]);
+                        fence_proxy_async_smem();
+                        __syncwarp();
+                        // d is a multiple of 64: a warp's 32 rows are all inside or all
+                        // past the end of a ragged tile
+                        if (lane == 0 && ot * kBlockM + quarter * 32 < p.d) {
+                            tma_store_2d(&L.maps[l][4 + which], buf, nt * BN + cslice * WCOLS + c * 32,
+                                         ot * kBlockM + quarter * 32);
+                            bulk_commit();
+                        }
+                        ++nbuf;
+                        continue;
+                    }
                     if (row < p.d) {
                         float4* dst = reinterpret_cast<float4*>(
                             base + (size_t)row * p.d + nt * BN + cslice * WCOLS + c * 32);
@@ -1884,6 +2001,9 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
             }
             acc_phase ^= 1;
         }
+        // every TMA store of this warp has landed before the CTA exits
+        if (lane == 0) bulk_wait<0>();
+        __syncwarp();
     }
 
     tc_fence_before();
@@ -1896,6 +2016,8 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
     }
 }
 
+// A launch with dep_counters is a programmatic dependent of the preceding
+// kernel (the fused forward / input-gradient launch that triggers it).
 template <int BN, bool SHIFT>
 static cudaError_t launch_pair(const TcLaunch<kMaxStackLayers>& L, int grid, cudaStream_t st) {
     constexpr size_t smem = pair_smem_total<BN, SHIFT>();
@@ -1917,13 +2039,15 @@ static cudaError_t launch_pair(const TcLaunch<kMaxStackLayers>& L, int grid, cud
     cfg.blockDim = dim3((unsigned)cta_threads(BN));
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = L.dep_counters ? 2 : 1;
     return cudaLaunchKernelEx(&cfg, kern, L);
 }
 

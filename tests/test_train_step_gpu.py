@@ -45,6 +45,10 @@ CASES = [
     (6, 64, 512, 7, 2, RESIDUAL | RELU),               # non-causal
     (3, 64, 512, 2, 0, CAUSAL | RESIDUAL | RELU),
     (8, 64, 128, 6, 0, RESIDUAL | RELU),               # not on pairs: the two calls
+    # enough layers for the batched weight gradient on SM pairs, which then
+    # starts behind the fused launch and waits on its completion counters
+    (4, 256, 512, 12, 5, CAUSAL | RESIDUAL | RELU),
+    (2, 512, 512, 12, 0, RESIDUAL | RELU),
 ]
 
 
