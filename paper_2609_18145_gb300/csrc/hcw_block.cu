@@ -485,12 +485,15 @@ size_t round256(size_t v) { return (v + 255) & ~(size_t)255; }
 //   m, hf [T][d] bf16          mixing output (per layer), head input
 //   U    [T][max(h, V, d)] fp32  every GEMM output with T rows, in turn
 //   dlog [T][V] bf16; dx [T][d] fp32; dxb [T][d] bf16; dpre [T][h] bf16;
-//   dh [T][d] bf16; the mixing backward's own workspace; the fp32 partial
+//   dh [T][d] bf16; the LayerNorm backward's partial sums
+//   dzm  [L][T][d] bf16        each mixing layer's output gradient (its dz),
+//                              read by the batched weight-gradient launch,
+//                              and that launch's scratch; the fp32 partial
 //   sums of the GEMMs that split K (the weight gradients)
 constexpr size_t kSplitWs = (size_t)32 << 20;
 struct BlockWs {
-    size_t xs, h1, g, a, st1, st2, stf, m, hf, U, dlog, dx, dxb, dpre, dh, lnp, lws, lws_bytes,
-        split, total;
+    size_t xs, h1, g, a, st1, st2, stf, m, hf, U, dlog, dx, dxb, dpre, dh, lnp, dzm, sws,
+        sws_bytes, split, total;
 };
 
 BlockWs block_ws(int B, int n, int d, int h, int V, int L) {
@@ -519,8 +522,11 @@ BlockWs block_ws(int B, int n, int d, int h, int V, int L) {
     w.dpre = take(T * h * 2);
     w.dh = take(T * d * 2);
     w.lnp = take((size_t)kLnBwdMaxGrid * 3 * d * 4);   // LayerNorm backward partial sums
-    w.lws_bytes = hcw_workspace_bytes(B, n, d, HCW_BF16, HCW_CAUSAL);
-    w.lws = take(w.lws_bytes);
+    // every mixing layer's output gradient, kept for one batched weight-gradient
+    // launch at the end of the backward, and that launch's scratch
+    w.dzm = take((size_t)L * T * d * 2);
+    w.sws_bytes = hcw_stack_bwd_weight_workspace_bytes(B, n, d, HCW_BF16, HCW_CAUSAL, L);
+    w.sws = take(w.sws_bytes);
     w.split = take(kSplitWs);
     w.total = o;
     return w;
@@ -674,6 +680,7 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
     auto H1 = [&](int l) { return reinterpret_cast<__nv_bfloat16*>(ws + w.h1) + (size_t)l * Td; };
     auto G = [&](int l) { return reinterpret_cast<__nv_bfloat16*>(ws + w.g) + (size_t)l * Td; };
     auto A = [&](int l) { return reinterpret_cast<__nv_bfloat16*>(ws + w.a) + (size_t)l * Th; };
+    auto DZM = [&](int l) { return reinterpret_cast<__nv_bfloat16*>(ws + w.dzm) + (size_t)l * Td; };
     auto S1 = [&](int l) { return reinterpret_cast<float2*>(ws + w.st1) + (size_t)l * T; };
     auto S2 = [&](int l) { return reinterpret_cast<float2*>(ws + w.st2) + (size_t)l * T; };
     float2* sf = reinterpret_cast<float2*>(ws + w.stf);
@@ -761,20 +768,26 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
                          dpre, gr.b1 + (size_t)l * h));
         HCW_GEMM(h, d, T, dpre, true, G(l), false, gr.W1 + (size_t)l * h * d);
         HCW_GEMM(T, d, h, dpre, false, bf(p.W1, (size_t)l * h * d), false, U);  // dg
-        le = launch_ln_bwd(st, U, nullptr, XM(l), S2(l), p.ln2_g + (size_t)l * d, dx, dx, dxb,
-                           lnp, gr.ln2_g + (size_t)l * d, gr.ln2_b + (size_t)l * d, nullptr, T, d,
-                           &nk);
+        le = launch_ln_bwd(st, U, nullptr, XM(l), S2(l), p.ln2_g + (size_t)l * d, dx, dx,
+                           DZM(l), lnp, gr.ln2_g + (size_t)l * d, gr.ln2_b + (size_t)l * d,
+                           nullptr, T, d, &nk);
         HCW_TRY(count_launch(le, nk));
-        // mixing sublayer: dxb = bf16(dx) is the gradient of M_l(h)
-        HCW_TRY(hcw_layer_bwd(H1(l), nullptr, dxb, bf(p.W_self, (size_t)l * d * d),
-                              bf(p.W_nbr, (size_t)l * d * d), l, -1, B, n, d, HCW_BF16, HCW_CAUSAL,
-                              dh, gr.W_self + (size_t)l * d * d, gr.W_nbr + (size_t)l * d * d,
-                              nullptr, w.lws_bytes ? ws + w.lws : nullptr, w.lws_bytes, st));
+        // mixing sublayer: DZM(l) = bf16(dx) is the gradient of M_l(h) (its dz: no
+        // activation); its input gradient now, its weight gradient with the other
+        // layers' after the loop
+        HCW_TRY(hcw_layer_bwd_data(DZM(l), nullptr, bf(p.W_self, (size_t)l * d * d),
+                                   bf(p.W_nbr, (size_t)l * d * d), l, -1, B, n, d, HCW_BF16,
+                                   HCW_CAUSAL, dh, st));
         le = launch_ln_bwd(st, nullptr, dh, X(l), S1(l), p.ln1_g + (size_t)l * d, dx, dx, dxb,
                            lnp, gr.ln1_g + (size_t)l * d, gr.ln1_b + (size_t)l * d,
                            l > 0 ? gr.b2 + (size_t)(l - 1) * d : nullptr, T, d, &nk);
         HCW_TRY(count_launch(le, nk));
     }
+    // the mixing layers' weight gradients, all layers in one batched launch: x_l =
+    // H1(l) (contiguous over l), dz_l = DZM(l)
+    HCW_TRY(hcw_stack_bwd_weight(H1(0), L > 1 ? H1(1) : nullptr, DZM(0), 0, L, -1, B, n, d,
+                                 HCW_BF16, HCW_CAUSAL, gr.W_self, gr.W_nbr, nullptr,
+                                 w.sws_bytes ? ws + w.sws : nullptr, w.sws_bytes, st));
     HCW_TRY(count_launch(launch_pdl(embed_bwd_kernel, dim3(elem_grid(Td)), dim3(256), 0, st, ids,
                                     static_cast<const float*>(dx), gr.E, B, n, d, V),
                          1));
