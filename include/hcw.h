@@ -499,6 +499,23 @@ size_t hcw_gemm_workspace_bytes(int M, int N, int K);
 int hcw_gemm_bf16(int M, int N, int K, const void* A, int ta, const void* B, int tb, float* C,
                   void* workspace, size_t ws_bytes, void* stream);
 
+/*
+ * `batch` products contracted over their rows, in one launch (the weight
+ * gradients of App. A's FFN for every layer of the block at once):
+ *   C[b] = A_b^T B_b,   b = 0 .. batch - 1
+ * A_b is the row-major [K][M] bf16 matrix at A + b * a_stride elements, B_b
+ * the row-major [K][N] bf16 matrix at B + b * b_stride elements, C[b] the
+ * row-major [M][N] fp32 matrix at C + b * M * N (overwritten).  Every output
+ * tile takes the whole K range in one fp32 accumulator (no partial sums, no
+ * workspace).  M, N, K, batch >= 1 and strides >= 0 (HCW_ERR_INVALID_ARG);
+ * C must not overlap the operands' spans (HCW_ERR_ALIASING).  Shapes TMA
+ * cannot read (M or N not a multiple of 64, a pointer or a stride not
+ * 16-byte aligned) run one product at a time on hcw_gemm_bf16's path.
+ * Asynchronous on `stream`.
+ */
+int hcw_gemm_bf16_batched(int M, int N, int K, const void* A, long long a_stride, const void* B,
+                          long long b_stride, float* C, int batch, void* stream);
+
 /* Number of kernels this library has launched in this process (all devices). */
 unsigned long long hcw_launch_count(void);
 

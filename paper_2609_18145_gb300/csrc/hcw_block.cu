@@ -484,7 +484,9 @@ size_t round256(size_t v) { return (v + 255) & ~(size_t)255; }
 //   st1, st2 [L][T], stf [T]   LayerNorm (mean, rstd)
 //   m, hf [T][d] bf16          mixing output (per layer), head input
 //   U    [T][max(h, V, d)] fp32  every GEMM output with T rows, in turn
-//   dlog [T][V] bf16; dx [T][d] fp32; dxb [T][d] bf16; dpre [T][h] bf16;
+//   dlog [T][V] bf16; dx [T][d] fp32
+//   dxf  [L][T][d] bf16        each FFN output's gradient (bf16 of dx)
+//   dpre [L][T][h] bf16        each FFN pre-activation gradient
 //   dh [T][d] bf16; the LayerNorm backward's partial sums
 //   dzm  [L][T][d] bf16        each mixing layer's output gradient (its dz),
 //                              read by the batched weight-gradient launch,
@@ -492,7 +494,7 @@ size_t round256(size_t v) { return (v + 255) & ~(size_t)255; }
 //   sums of the GEMMs that split K (the weight gradients)
 constexpr size_t kSplitWs = (size_t)32 << 20;
 struct BlockWs {
-    size_t xs, h1, g, a, st1, st2, stf, m, hf, U, dlog, dx, dxb, dpre, dh, lnp, dzm, sws,
+    size_t xs, h1, g, a, st1, st2, stf, m, hf, U, dlog, dx, dxf, dpre, dh, lnp, dzm, sws,
         sws_bytes, split, total;
 };
 
@@ -518,8 +520,10 @@ BlockWs block_ws(int B, int n, int d, int h, int V, int L) {
     w.U = take(T * wide * 4);
     w.dlog = take(T * V * 2);
     w.dx = take(T * d * 4);
-    w.dxb = take(T * d * 2);
-    w.dpre = take(T * h * 2);
+    // per layer: the FFN output's gradient (bf16) and the pre-activation
+    // gradient, the operands of the batched FFN weight gradients after the loop
+    w.dxf = take((size_t)L * T * d * 2);
+    w.dpre = take((size_t)L * T * h * 2);
     w.dh = take(T * d * 2);
     w.lnp = take((size_t)kLnBwdMaxGrid * 3 * d * 4);   // LayerNorm backward partial sums
     // every mixing layer's output gradient, kept for one batched weight-gradient
@@ -690,8 +694,8 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
     auto* dlog = reinterpret_cast<__nv_bfloat16*>(ws + w.dlog);
     float* dx = reinterpret_cast<float*>(ws + w.dx);
     float* lnp = reinterpret_cast<float*>(ws + w.lnp);
-    auto* dxb = reinterpret_cast<__nv_bfloat16*>(ws + w.dxb);
-    auto* dpre = reinterpret_cast<__nv_bfloat16*>(ws + w.dpre);
+    auto DXF = [&](int l) { return reinterpret_cast<__nv_bfloat16*>(ws + w.dxf) + (size_t)l * Td; };
+    auto DPRE = [&](int l) { return reinterpret_cast<__nv_bfloat16*>(ws + w.dpre) + (size_t)l * Th; };
     auto* dh = reinterpret_cast<__nv_bfloat16*>(ws + w.dh);
     auto bf = [](const void* q, size_t off) {
         return static_cast<const __nv_bfloat16*>(q) + off;
@@ -757,17 +761,17 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
     // each LayerNorm backward that writes the gradient of x_{l+1} (LNf, then
     // LN1 of layer l + 1) also sums its bf16 copy's columns: db2 of layer l
     int nk = 0;
-    cudaError_t le = launch_ln_bwd(st, U, nullptr, X(L), sf, p.lnf_g, nullptr, dx, dxb, lnp,
-                                   gr.lnf_g, gr.lnf_b, gr.b2 + (size_t)(L - 1) * d, T, d, &nk);
+    cudaError_t le = launch_ln_bwd(st, U, nullptr, X(L), sf, p.lnf_g, nullptr, dx, DXF(L - 1),
+                                   lnp, gr.lnf_g, gr.lnf_b, gr.b2 + (size_t)(L - 1) * d, T, d,
+                                   &nk);
     HCW_TRY(count_launch(le, nk));
     for (int l = L - 1; l >= 0; --l) {
-        // FFN sublayer: dxb = bf16(dx) is the gradient of its output
-        HCW_GEMM(d, h, T, dxb, true, A(l), false, gr.W2 + (size_t)l * d * h);
-        // dpre = (a > 0) * (dxb W2), and db1 = its column sums
-        HCW_TRY(gemm_ffn(st, T, h, d, dxb, bf(p.W2, (size_t)l * d * h), false, nullptr, A(l),
-                         dpre, gr.b1 + (size_t)l * h));
-        HCW_GEMM(h, d, T, dpre, true, G(l), false, gr.W1 + (size_t)l * h * d);
-        HCW_GEMM(T, d, h, dpre, false, bf(p.W1, (size_t)l * h * d), false, U);  // dg
+        // FFN sublayer: DXF(l) = bf16(dx) is the gradient of its output;
+        // dpre = (a > 0) * (DXF(l) W2), and db1 = its column sums.  Its weight
+        // gradients W2 (DXF(l)^T a) and W1 (dpre^T g) come after the loop.
+        HCW_TRY(gemm_ffn(st, T, h, d, DXF(l), bf(p.W2, (size_t)l * d * h), false, nullptr, A(l),
+                         DPRE(l), gr.b1 + (size_t)l * h));
+        HCW_GEMM(T, d, h, DPRE(l), false, bf(p.W1, (size_t)l * h * d), false, U);  // dg
         le = launch_ln_bwd(st, U, nullptr, XM(l), S2(l), p.ln2_g + (size_t)l * d, dx, dx,
                            DZM(l), lnp, gr.ln2_g + (size_t)l * d, gr.ln2_b + (size_t)l * d,
                            nullptr, T, d, &nk);
@@ -778,10 +782,21 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
         HCW_TRY(hcw_layer_bwd_data(DZM(l), nullptr, bf(p.W_self, (size_t)l * d * d),
                                    bf(p.W_nbr, (size_t)l * d * d), l, -1, B, n, d, HCW_BF16,
                                    HCW_CAUSAL, dh, st));
-        le = launch_ln_bwd(st, nullptr, dh, X(l), S1(l), p.ln1_g + (size_t)l * d, dx, dx, dxb,
-                           lnp, gr.ln1_g + (size_t)l * d, gr.ln1_b + (size_t)l * d,
-                           l > 0 ? gr.b2 + (size_t)(l - 1) * d : nullptr, T, d, &nk);
+        le = launch_ln_bwd(st, nullptr, dh, X(l), S1(l), p.ln1_g + (size_t)l * d, dx, dx,
+                           l > 0 ? DXF(l - 1) : nullptr, lnp, gr.ln1_g + (size_t)l * d,
+                           gr.ln1_b + (size_t)l * d, l > 0 ? gr.b2 + (size_t)(l - 1) * d : nullptr,
+                           T, d, &nk);
         HCW_TRY(count_launch(le, nk));
+    }
+    // the FFN weight gradients of all layers, two batched launches (every
+    // output tile over the whole token range, no partial sums):
+    // dW2_l = DXF(l)^T a_l [d][h], dW1_l = dpre_l^T g_l [h][d]
+    {
+        int nl = 0;
+        HCW_CU(gemm_bf16_f32_batched(d, h, T, DXF(0), Td * 2, A(0), Th * 2, gr.W2, L, st, &nl));
+        HCW_TRY(count_launch(cudaSuccess, nl));
+        HCW_CU(gemm_bf16_f32_batched(h, d, T, DPRE(0), Th * 2, G(0), Td * 2, gr.W1, L, st, &nl));
+        HCW_TRY(count_launch(cudaSuccess, nl));
     }
     // the mixing layers' weight gradients, all layers in one batched launch: x_l =
     // H1(l) (contiguous over l), dz_l = DZM(l)

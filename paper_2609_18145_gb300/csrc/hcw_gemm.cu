@@ -85,6 +85,10 @@ struct GemmArgs {
     int M, N, K;
     int mt, nt;                 // tile counts (256-row tiles, 256-column tiles)
     int splits, kps;            // K splits and K steps per split
+    // batched (both operands MN-major, EPI_F32): `splits` counts independent
+    // products instead of K splits; mA / mB carry the batch as a 4th dimension
+    // and each unit takes the whole K range of product s into C[s]
+    int batched;
     uint32_t stage_tx;          // bytes one CTA's two copies of a stage land
     int vec;                    // rows of the output start 16-byte aligned
     unsigned long long timeout_ns;
@@ -140,8 +144,8 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_pair_kernel(const __grid_co
     // running together share their A rows (and B, the weights, is small)
     auto unit_k = [&](int u, int& kb0, int& kb1) {
         const int s = u / tiles;
-        kb0 = s * a.kps;
-        kb1 = kb0 + a.kps < nkb ? kb0 + a.kps : nkb;
+        kb0 = a.batched ? 0 : s * a.kps;
+        kb1 = a.batched ? nkb : (kb0 + a.kps < nkb ? kb0 + a.kps : nkb);
     };
 
     if (warp == 0) {
@@ -169,14 +173,20 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_pair_kernel(const __grid_co
                     // blocks of an MN-major operand, or 128 rows of a K-major one
                     const int a_row = 2 * mi * kGM + (int)rank * kGM;
                     const int b_row = ni * kGN + (int)rank * (kGN / 2);
-                    if (A_MN)
-                        tma_load_3d_pair(sA, &a.mA, fb, 0, kb * kGK, a_row / 64);
-                    else
-                        tma_load_2d_pair(sA, &a.mA, fb, kb * kGK, a_row);
-                    if (B_MN)
-                        tma_load_3d_pair(sB, &a.mB, fb, 0, kb * kGK, b_row / 64);
-                    else
-                        tma_load_2d_pair(sB, &a.mB, fb, kb * kGK, b_row);
+                    if (A_MN && B_MN && a.batched) {
+                        const int bi = u / tiles;   // the product
+                        tma_load_4d_pair(sA, &a.mA, fb, 0, kb * kGK, a_row / 64, bi);
+                        tma_load_4d_pair(sB, &a.mB, fb, 0, kb * kGK, b_row / 64, bi);
+                    } else {
+                        if (A_MN)
+                            tma_load_3d_pair(sA, &a.mA, fb, 0, kb * kGK, a_row / 64);
+                        else
+                            tma_load_2d_pair(sA, &a.mA, fb, kb * kGK, a_row);
+                        if (B_MN)
+                            tma_load_3d_pair(sB, &a.mB, fb, 0, kb * kGK, b_row / 64);
+                        else
+                            tma_load_2d_pair(sB, &a.mB, fb, kb * kGK, b_row);
+                    }
                     if (++stage == kGStages) {
                         stage = 0;
                         phase ^= 1;
@@ -649,6 +659,22 @@ bool map_mnmajor(CUtensorMap* m, const void* base, int K, int cols, int nblk) {
                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// A batch of MN-major operands, product b at base + b * batch_bytes, each the
+// row-major [K][cols] matrix: (64 columns, K rows, cols / 64 blocks, batch),
+// box (64, 64, nblk, 1).
+bool map_mnmajor_batched(CUtensorMap* m, const void* base, int K, int cols, int nblk, int batch,
+                         size_t batch_bytes) {
+    GemmEncodeFn enc = gemm_encode_fn();
+    if (!enc || batch_bytes % 16) return false;
+    cuuint64_t dims[4] = {64, (cuuint64_t)K, (cuuint64_t)(cols / 64), (cuuint64_t)batch};
+    cuuint64_t strides[3] = {(cuuint64_t)cols * 2, 128, (cuuint64_t)batch_bytes};
+    cuuint32_t box[4] = {64, 64, (cuuint32_t)nblk, 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box,
+               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // fp32 output [splits][M][N] as (N, M, splits), box (32, 32, 1): 32 x 32
 // patches clipped at each split's M rows; 128-byte swizzle.
 bool map_out_f32(CUtensorMap* m, void* base, int M, int N, int splits) {
@@ -865,6 +891,56 @@ cudaError_t gemm_bf16_f32(int M, int N, int K, const void* A, bool ta, const voi
     return gemm_bf16(M, N, K, A, ta, B, tb, C, epi, split_ws, split_ws_bytes, st, launches);
 }
 
+cudaError_t gemm_bf16_f32_batched(int M, int N, int K, const void* A, size_t a_batch_bytes,
+                                  const void* B, size_t b_batch_bytes, float* C, int batch,
+                                  cudaStream_t st, int* launches) {
+    *launches = 0;
+    if (M <= 0 || N <= 0 || K <= 0 || batch <= 0 || !A || !B || !C) return cudaErrorInvalidValue;
+    const auto aligned = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
+    const bool tc = aligned(A) && aligned(B) && aligned(C) && M % 64 == 0 && N % 64 == 0 &&
+                    a_batch_bytes % 16 == 0 && b_batch_bytes % 16 == 0 &&
+                    gemm_encode_fn() != nullptr;
+    if (!tc) {
+        // shapes TMA cannot read: one product after another
+        for (int b = 0; b < batch; ++b) {
+            int nl = 0;
+            const cudaError_t e =
+                gemm_bf16_f32(M, N, K, static_cast<const uint8_t*>(A) + b * a_batch_bytes, true,
+                              static_cast<const uint8_t*>(B) + b * b_batch_bytes, false,
+                              C + (size_t)b * M * N, nullptr, 0, st, &nl);
+            if (e != cudaSuccess) return e;
+            *launches += nl;
+        }
+        return cudaSuccess;
+    }
+    const int a_box = M / 64 < kGM / 64 ? M / 64 : kGM / 64;
+    const int b_box = N / 64 < kGN / 128 ? N / 64 : kGN / 128;
+    GemmArgs a;
+    memset(&a, 0, sizeof(a));
+    if (!map_mnmajor_batched(&a.mA, A, K, M, a_box, batch, a_batch_bytes) ||
+        !map_mnmajor_batched(&a.mB, B, K, N, b_box, batch, b_batch_bytes))
+        return cudaErrorInvalidValue;
+    a.stage_tx = (uint32_t)(kGK * 2) * (uint32_t)(64 * a_box + 64 * b_box);
+    a.M = M;
+    a.N = N;
+    a.K = K;
+    a.mt = (M + 2 * kGM - 1) / (2 * kGM);
+    a.nt = (N + kGN - 1) / kGN;
+    a.batched = 1;
+    a.splits = batch;
+    a.kps = (K + kGK - 1) / kGK;
+    a.C = C;
+    a.vec = N % 4 == 0;
+    a.tma_out = map_out_f32(&a.mOut, C, M, N, batch);
+    a.timeout_ns = kGemmTimeoutNs;
+    const int sms = gemm_sms();
+    const int units = a.mt * a.nt * batch;
+    const int pairs = units < sms / 2 ? units : sms / 2;
+    const cudaError_t e = launch_gemm_any(true, true, EPI_F32, a, 2 * pairs, st);
+    if (e == cudaSuccess) *launches = 1;
+    return e;
+}
+
 cudaError_t gemm_error_word_read_clear(int* word) {
     const int zero = 0;
     cudaError_t e = cudaMemcpyFromSymbol(word, g_error_word, sizeof(int));
@@ -905,6 +981,29 @@ int hcw_gemm_bf16(int M, int N, int K, const void* A, int ta, const void* B, int
                                              static_cast<float*>(workspace),
                                              workspace ? ws_bytes : 0, (cudaStream_t)stream,
                                              &launches);
+    return hcw::count_launch(e, launches);
+}
+
+int hcw_gemm_bf16_batched(int M, int N, int K, const void* A, long long a_stride, const void* B,
+                          long long b_stride, float* C, int batch, void* stream) {
+    if (M < 1 || N < 1 || K < 1 || batch < 1 || a_stride < 0 || b_stride < 0 || !A || !B || !C)
+        return HCW_ERR_INVALID_ARG;
+    const auto span = [](const void* p, size_t bytes) {
+        return std::make_pair(reinterpret_cast<uintptr_t>(p),
+                              reinterpret_cast<uintptr_t>(p) + bytes);
+    };
+    const auto overlap = [](std::pair<uintptr_t, uintptr_t> x, std::pair<uintptr_t, uintptr_t> y) {
+        return x.first < y.second && y.first < x.second;
+    };
+    const size_t nb = (size_t)batch - 1;
+    const auto c = span(C, (size_t)batch * M * N * sizeof(float));
+    if (overlap(c, span(A, (nb * (size_t)a_stride + (size_t)K * M) * 2)) ||
+        overlap(c, span(B, (nb * (size_t)b_stride + (size_t)K * N) * 2)))
+        return HCW_ERR_ALIASING;
+    int launches = 0;
+    const cudaError_t e = hcw::gemm_bf16_f32_batched(M, N, K, A, (size_t)a_stride * 2, B,
+                                                     (size_t)b_stride * 2, C, batch,
+                                                     (cudaStream_t)stream, &launches);
     return hcw::count_launch(e, launches);
 }
 

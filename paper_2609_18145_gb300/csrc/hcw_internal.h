@@ -276,6 +276,14 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
 cudaError_t gemm_bf16_f32(int M, int N, int K, const void* A, bool ta, const void* B, bool tb,
                           float* C, float* split_ws, size_t split_ws_bytes, cudaStream_t st,
                           int* launches);
+// `batch` independent products contracted over their rows, in one launch:
+// C[b] (fp32 [M][N]) = A_b^T B_b with A_b the row-major [K][M] bf16 matrix at
+// A + b * a_batch_bytes and B_b the row-major [K][N] at B + b * b_batch_bytes
+// (the weight gradients of a run of layers); C[b] at C + b * M * N.  Each
+// output tile takes the whole K range (no partial sums).
+cudaError_t gemm_bf16_f32_batched(int M, int N, int K, const void* A, size_t a_batch_bytes,
+                                  const void* B, size_t b_batch_bytes, float* C, int batch,
+                                  cudaStream_t st, int* launches);
 // Epilogues of the GEMM: fp32 C; out = bf16(relu(C + bias[col])); or
 // out = bf16(aux[row][col] > 0 ? C : 0), with colsum[col] (if given) += the
 // column sums of out.  out and aux are [M][N] bf16.

@@ -91,6 +91,8 @@ _SIGNATURES = {
     "hcw_block_step": ([_P, _P, _P, _I, _I, _I, _I, _I, _I, _P, _P, _SZ, _P], _I),
     "hcw_gemm_workspace_bytes": ([_I, _I, _I], _SZ),
     "hcw_gemm_bf16": ([_I, _I, _I, _P, _I, _P, _I, _P, _P, _SZ, _P], _I),
+    "hcw_gemm_bf16_batched": ([_I, _I, _I, _P, ctypes.c_longlong, _P, ctypes.c_longlong, _P, _I,
+                               _P], _I),
     "hcw_set_stack_kernels": ([_I], _I),
     "hcw_set_decode_kernel": ([_I], _I),
     "hcw_stack_kernels_used": ([_I, _I, _I, _I], _I),
@@ -352,6 +354,29 @@ def hcw_gemm_bf16(A, B, ta: bool = False, tb: bool = False, C=None, workspace=No
         wp, wn = None, 0
     _check(lib().hcw_gemm_bf16(M, N, K, _ptr(A), int(bool(ta)), _ptr(B), int(bool(tb)), _ptr(C),
                                wp, wn, _stream(stream)), "hcw_gemm_bf16")
+    return C
+
+
+def hcw_gemm_bf16_batched(A, B, C=None, stream=None):
+    """fp32 C[b] = A[b]^T B[b] from bf16 A [batch, K, M] and B [batch, K, N]
+    (each product contracted over its rows, whole K per output tile).  The
+    batch dimension may have any stride (in elements); the rows are
+    contiguous.  Returns C [batch, M, N]."""
+    _dev(C)
+    if not (A.is_cuda and B.is_cuda):
+        raise ValueError("all tensors must be CUDA tensors")
+    if A.dtype != torch.bfloat16 or B.dtype != torch.bfloat16 or A.dim() != 3 or B.dim() != 3:
+        raise ValueError("hcw_gemm_bf16_batched: A and B must be 3-D bf16 tensors")
+    batch, K, M = A.shape
+    if B.shape[0] != batch or B.shape[1] != K:
+        raise ValueError("hcw_gemm_bf16_batched: A %s and B %s do not match"
+                         % (tuple(A.shape), tuple(B.shape)))
+    N = B.shape[2]
+    if A.stride(2) != 1 or A.stride(1) != M or B.stride(2) != 1 or B.stride(1) != N:
+        raise ValueError("hcw_gemm_bf16_batched: each product's rows must be contiguous")
+    C = torch.empty(batch, M, N, dtype=torch.float32, device=A.device) if C is None else C
+    _check(lib().hcw_gemm_bf16_batched(M, N, K, _ptr(A), A.stride(0), _ptr(B), B.stride(0),
+                                       _ptr(C), batch, _stream(stream)), "hcw_gemm_bf16_batched")
     return C
 
 

@@ -368,6 +368,27 @@ def test_gemm_validation_codes(hcw):
     assert call(w=C + 256, wsb=1 << 20) == hcw.HCW_ERR_ALIASING   # workspace inside C
 
 
+def test_batched_gemm_validation_codes(hcw):
+    """hcw_gemm_bf16_batched rejects bad sizes, strides and a C that overlaps
+    an operand's span before anything launches."""
+    P = ctypes.c_void_p
+    L = hcw.lib()
+    M, N, K, nb = 256, 512, 128, 3
+    A, B, C = (0x10000000 * k for k in range(1, 4))
+
+    def call(M=M, N=N, K=K, a=A, sa=M * K, b=B, sb=N * K, c=C, batch=nb):
+        return L.hcw_gemm_bf16_batched(M, N, K, P(a), sa, P(b), sb, P(c), batch, None)
+
+    before = hcw.hcw_launch_count()
+    assert call(batch=0) == hcw.HCW_ERR_INVALID_ARG
+    assert call(N=0) == hcw.HCW_ERR_INVALID_ARG
+    assert call(sa=-1) == hcw.HCW_ERR_INVALID_ARG
+    assert call(b=0) == hcw.HCW_ERR_INVALID_ARG
+    assert call(c=A + (nb - 1) * M * K * 2) == hcw.HCW_ERR_ALIASING   # C inside A's last product
+    assert call(c=B - 64) == hcw.HCW_ERR_ALIASING                      # C's end inside B
+    assert hcw.hcw_launch_count() == before
+
+
 def test_gemm_workspace_sizes(hcw):
     """A weight-gradient shape (few output tiles, long K) asks for a K split;
     a short K or a wide output asks for none."""

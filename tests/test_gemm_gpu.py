@@ -105,3 +105,31 @@ def test_misaligned_operands_take_the_plain_kernel(H):
     torch.cuda.synchronize()
     assert H.hcw_sync_status() == H.HCW_OK
     check(C.cpu(), A[:, 1:].contiguous(), B[:, 1:].contiguous(), False, True)
+
+
+BATCHED = [
+    # batch, M, N, K
+    (3, 512, 1024, 2000),   # the FFN's dW2 shape, ragged K
+    (4, 1024, 512, 640),    # dW1 shape
+    (2, 192, 320, 1000),    # a half tile past a whole one in M
+    (2, 100, 64, 96),       # M not a multiple of 64: one product at a time
+]
+
+
+@pytest.mark.parametrize("case", BATCHED, ids=lambda c: "b%d_M%d_N%d_K%d" % c)
+def test_batched_products_match_each_product(H, case):
+    """hcw_gemm_bf16_batched: C[b] = A[b]^T B[b] for every b, each against its
+    own fp64 product, with a batch stride larger than one product (padding
+    between them) for A."""
+    nb, M, N, K = case
+    g = torch.Generator().manual_seed(nb * 7 + M)
+    A = torch.randn(nb, K + 3, M, generator=g).to(torch.bfloat16)[:, :K, :]
+    B = torch.randn(nb, K, N, generator=g).to(torch.bfloat16)
+    Ad = torch.empty(nb, K + 3, M, dtype=torch.bfloat16, device="cuda")
+    Ad[:, :K, :] = A.cuda()
+    Ad = Ad[:, :K, :]
+    assert Ad.stride(0) == (K + 3) * M
+    C = H.hcw_gemm_bf16_batched(Ad, B.cuda())
+    torch.cuda.synchronize()
+    for b in range(nb):
+        check(C[b], A[b].contiguous(), B[b].contiguous(), True, False)
