@@ -19,6 +19,7 @@
 // hf, dlogits, bf16(dx), the FFN pre-activation gradient); the other GEMM
 // outputs are fp32.
 #include <mutex>
+#include <vector>
 
 #include "hcw.h"
 #include "hcw_internal.h"
@@ -404,6 +405,55 @@ __global__ void __launch_bounds__(kReduceWarps * 32)
     }
 }
 
+// The same sums for a list of LayerNorm backward passes at once: job
+// blockIdx.y adds up its own partial rows (in row order, as above).
+constexpr int kMaxLnJobs = 64;
+struct LnJob {
+    const float* part;
+    int nblk, ncol;
+    float* dgam;
+    float* dbet;
+    float* dcol;
+};
+struct LnJobs {
+    LnJob job[kMaxLnJobs];
+    int d;
+};
+__global__ void __launch_bounds__(kReduceWarps * 32)
+    ln_part_reduce_batched_kernel(const __grid_constant__ LnJobs J) {
+    pdl_wait();   // until the kernel before it in the stream has finished
+    pdl_trigger();
+    __shared__ float acc[kReduceWarps][33];
+    const LnJob& jb = J.job[blockIdx.y];
+    const int d = J.d;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int width = jb.ncol * d;
+    const int c = blockIdx.x * 32 + lane;
+    if (blockIdx.x * 32 >= width) return;   // block-uniform: this job is narrower
+    float s = 0.f;
+    if (c < width) {
+        for (int b0 = warp; b0 < jb.nblk; b0 += 16 * kReduceWarps) {
+            float v[16];
+#pragma unroll
+            for (int k = 0; k < 16; ++k) {
+                const int b = b0 + k * kReduceWarps;
+                v[k] = b < jb.nblk ? jb.part[(size_t)b * width + c] : 0.f;
+            }
+#pragma unroll
+            for (int k = 0; k < 16; ++k) s += v[k];
+        }
+    }
+    acc[warp][lane] = s;
+    __syncthreads();
+    if (warp == 0 && c < width) {
+        float t = 0.f;
+#pragma unroll
+        for (int w = 0; w < kReduceWarps; ++w) t += acc[w][lane];
+        const int seg = c / d, cc = c - seg * d;
+        (seg == 0 ? jb.dgam : (seg == 1 ? jb.dbet : jb.dcol))[cc] = t;
+    }
+}
+
 // dE[ids[b][t]] += dx[b n + t]   (dE zeroed before the launch)
 __global__ void embed_bwd_kernel(const int* ids, const float* dx, float* dE, int B, int n, int d,
                                  int V) {
@@ -525,7 +575,9 @@ BlockWs block_ws(int B, int n, int d, int h, int V, int L) {
     w.dxf = take((size_t)L * T * d * 2);
     w.dpre = take((size_t)L * T * h * 2);
     w.dh = take(T * d * 2);
-    w.lnp = take((size_t)kLnBwdMaxGrid * 3 * d * 4);   // LayerNorm backward partial sums
+    // LayerNorm backward partial sums, one slice per pass (2 L + 1 of them),
+    // added up together after the backward loop
+    w.lnp = take((2 * (size_t)L + 1) * kLnBwdMaxGrid * 3 * d * 4);
     // every mixing layer's output gradient, kept for one batched weight-gradient
     // launch at the end of the backward, and that launch's scratch
     w.dzm = take((size_t)L * T * d * 2);
@@ -652,7 +704,7 @@ cudaError_t launch_ln_bwd_rows(cudaStream_t st, int grid, const DY* dy, const fl
 cudaError_t launch_ln_bwd(cudaStream_t st, const float* dyf, const __nv_bfloat16* dyb,
                           const float* x, const float2* stats, const float* g, const float* dres,
                           float* dx_out, __nv_bfloat16* dxb, float* part, float* dgam, float* dbet,
-                          float* dcol, int T, int d, int* nk) {
+                          float* dcol, int T, int d, int* nk, LnJob* defer = nullptr) {
     *nk = 0;
     if (dcol && !dxb) return cudaErrorInvalidValue;
     const int ncol = dcol ? 3 : 2;
@@ -667,6 +719,11 @@ cudaError_t launch_ln_bwd(cudaStream_t st, const float* dyf, const __nv_bfloat16
                                                             dx_out, dxb, T, d, ncol, part);
     if (e != cudaSuccess) return e;
     *nk = 1;
+    if (defer) {
+        // the sums are added up later, with other passes' (part stays untouched)
+        *defer = LnJob{part, grid, ncol, dgam, dbet, dcol};
+        return cudaSuccess;
+    }
     e = launch_pdl(ln_part_reduce_kernel, dim3((ncol * d + 31) / 32), dim3(kReduceWarps * 32), 0,
                    st, static_cast<const float*>(part), grid, d, ncol, dgam, dbet, dcol);
     if (e == cudaSuccess) *nk = 2;
@@ -761,9 +818,16 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
     // each LayerNorm backward that writes the gradient of x_{l+1} (LNf, then
     // LN1 of layer l + 1) also sums its bf16 copy's columns: db2 of layer l
     int nk = 0;
+    // every LayerNorm backward pass leaves its partial sums in its own slice;
+    // one launch adds them all up after the loop
+    static thread_local std::vector<LnJob> jobs;
+    jobs.assign(2 * (size_t)L + 1, LnJob{});
+    int njobs = 0;
+    auto lnp_slice = [&](int i) { return lnp + (size_t)i * kLnBwdMaxGrid * 3 * d; };
     cudaError_t le = launch_ln_bwd(st, U, nullptr, X(L), sf, p.lnf_g, nullptr, dx, DXF(L - 1),
-                                   lnp, gr.lnf_g, gr.lnf_b, gr.b2 + (size_t)(L - 1) * d, T, d,
-                                   &nk);
+                                   lnp_slice(njobs), gr.lnf_g, gr.lnf_b,
+                                   gr.b2 + (size_t)(L - 1) * d, T, d, &nk, &jobs[njobs]);
+    ++njobs;
     HCW_TRY(count_launch(le, nk));
     for (int l = L - 1; l >= 0; --l) {
         // FFN sublayer: DXF(l) = bf16(dx) is the gradient of its output;
@@ -773,8 +837,9 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
                          DPRE(l), gr.b1 + (size_t)l * h));
         HCW_GEMM(T, d, h, DPRE(l), false, bf(p.W1, (size_t)l * h * d), false, U);  // dg
         le = launch_ln_bwd(st, U, nullptr, XM(l), S2(l), p.ln2_g + (size_t)l * d, dx, dx,
-                           DZM(l), lnp, gr.ln2_g + (size_t)l * d, gr.ln2_b + (size_t)l * d,
-                           nullptr, T, d, &nk);
+                           DZM(l), lnp_slice(njobs), gr.ln2_g + (size_t)l * d,
+                           gr.ln2_b + (size_t)l * d, nullptr, T, d, &nk, &jobs[njobs]);
+        ++njobs;
         HCW_TRY(count_launch(le, nk));
         // mixing sublayer: DZM(l) = bf16(dx) is the gradient of M_l(h) (its dz: no
         // activation); its input gradient now, its weight gradient with the other
@@ -783,10 +848,24 @@ int block_step(const int* ids, const hcw_block_params& p, const hcw_block_grads&
                                    bf(p.W_nbr, (size_t)l * d * d), l, -1, B, n, d, HCW_BF16,
                                    HCW_CAUSAL, dh, st));
         le = launch_ln_bwd(st, nullptr, dh, X(l), S1(l), p.ln1_g + (size_t)l * d, dx, dx,
-                           l > 0 ? DXF(l - 1) : nullptr, lnp, gr.ln1_g + (size_t)l * d,
-                           gr.ln1_b + (size_t)l * d, l > 0 ? gr.b2 + (size_t)(l - 1) * d : nullptr,
-                           T, d, &nk);
+                           l > 0 ? DXF(l - 1) : nullptr, lnp_slice(njobs),
+                           gr.ln1_g + (size_t)l * d, gr.ln1_b + (size_t)l * d,
+                           l > 0 ? gr.b2 + (size_t)(l - 1) * d : nullptr, T, d, &nk,
+                           &jobs[njobs]);
+        ++njobs;
         HCW_TRY(count_launch(le, nk));
+    }
+    // the LayerNorm parameter gradients (and db2) of every pass, in launches of
+    // up to kMaxLnJobs passes
+    for (int j0 = 0; j0 < njobs; j0 += kMaxLnJobs) {
+        const int cnt = njobs - j0 < kMaxLnJobs ? njobs - j0 : kMaxLnJobs;
+        static thread_local LnJobs part;
+        part.d = d;
+        for (int j = 0; j < cnt; ++j) part.job[j] = jobs[j0 + j];
+        HCW_TRY(count_launch(launch_pdl(ln_part_reduce_batched_kernel,
+                                        dim3((3 * d + 31) / 32, cnt), dim3(kReduceWarps * 32), 0,
+                                        st, part),
+                             1));
     }
     // the FFN weight gradients of all layers, two batched launches (every
     // output tile over the whole token range, no partial sums):
