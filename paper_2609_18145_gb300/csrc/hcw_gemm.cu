@@ -265,12 +265,28 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_pair_kernel(const __grid_co
         };
         for (int u = pair; u < n_units; u += n_pairs) {
             const int s = u / tiles, rem = u % tiles, mi = rem / a.nt, ni = rem - mi * a.nt;
-            const bool okw = mbar_wait(&bars->tfull[acc], acc_phase, abort, tmo);
-            if (!__all_sync(0xffffffffu, okw)) break;
-            tc_fence_after();
             const int row0 = 2 * mi * kGM + (int)rank * kGM + quarter * 32;   // the warp's rows
             const int row = row0 + lane;
             const int colw = ni * kGN + chalf * 128;                          // and columns
+            // EPI_RELU_GRAD: the aux patches of the tile's two 64-column halves go
+            // into the warp's two buffers before the accumulator is ready (the
+            // stores of the tile before have read them by then); the second half
+            // is stored only if the first is, so half hh lands in buffer nbuf ^ hh
+            int n_aux = 0;
+            if (EPI == EPI_RELU_GRAD && a.tma_out) {
+                n_aux = (row0 < a.M && colw < a.N) + (row0 < a.M && colw + 64 < a.N);
+                if (lane == 0 && n_aux > 0) {
+                    bulk_wait_read<0>();
+                    mbar_arrive_expect_tx(&bars->aux[e], (uint32_t)(n_aux * kGPatch));
+                    tma_load_2d(patch_buf(nbuf), &a.mAux, &bars->aux[e], colw, row0);
+                    if (n_aux > 1)
+                        tma_load_2d(patch_buf(nbuf ^ 1), &a.mAux, &bars->aux[e], colw + 64, row0);
+                    aux_pending = true;
+                }
+            }
+            const bool okw = mbar_wait(&bars->tfull[acc], acc_phase, abort, tmo);
+            if (!__all_sync(0xffffffffu, okw)) break;
+            tc_fence_after();
             const uint32_t tbase = tmem_base + ((uint32_t)(quarter * 32) << 16) +
                                    (uint32_t)(acc * kGN + chalf * 128);
             const uint32_t tempty_leader = mapa_shared(&bars->tempty[acc], 0);
@@ -325,14 +341,7 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_pair_kernel(const __grid_co
                         }
                         uint8_t* buf = patch_buf(nbuf);
                         nbuf ^= 1;
-                        if (lane == 0) {
-                            bulk_wait_read<1>();
-                            if (EPI == EPI_RELU_GRAD) {
-                                mbar_arrive_expect_tx(&bars->aux[e], kGPatch);
-                                tma_load_2d(buf, &a.mAux, &bars->aux[e], c0, row0);
-                                aux_pending = true;
-                            }
-                        }
+                        if (lane == 0 && EPI != EPI_RELU_GRAD) bulk_wait_read<1>();
                         uint32_t r0[32], r1[32];
                         __syncwarp();
                         tmem_ld_32x32b_x32(tbase + (uint32_t)(hh * 64), r0);
@@ -344,7 +353,8 @@ __global__ void __launch_bounds__(kGThreads, 1) gemm_pair_kernel(const __grid_co
                             __syncwarp();
                             if (lane == 0) mbar_arrive_remote_tmem(tempty_leader);
                         }
-                        if (EPI == EPI_RELU_GRAD) {
+                        if (EPI == EPI_RELU_GRAD && hh == 0) {
+                            // both halves' aux patches (one barrier phase per tile)
                             const bool okx = mbar_wait(&bars->aux[e], aux_phase, abort, tmo);
                             if (!__all_sync(0xffffffffu, okx)) {
                                 okp = false;
