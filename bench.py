@@ -362,17 +362,12 @@ def run_ours(args):
 
     def step_calls(xin, dyin, outs=None):
         oWs, oWn, ob = outs if outs is not None else (gWs, gWn, gb)
-        if dims is None:
-            # one training-step call: the forward and the input gradient in one
-            # launch where the shape allows it, then the weight gradients
-            H.hcw_stack_train_step(xin, Ws, Wn, bias, dyin, 0, -1, flags, y=y, acts=acts,
-                                   masks=masks, dx=dx, dW_self=oWs, dW_nbr=oWn, dbias=ob,
-                                   workspace=tws)
-            return
-        H.hcw_stack_fwd(xin, Ws, Wn, bias, 0, -1, flags, y=y, acts=acts, masks=masks,
-                        workspace=fws, dims=dims)
-        H.hcw_stack_bwd(xin, acts, masks, dyin, Ws, Wn, 0, -1, flags, dx=dx, dW_self=oWs,
-                        dW_nbr=oWn, dbias=ob, workspace=ws, dims=dims)
+        # one training-step call (on the schedule dims if given): the forward and
+        # the input gradient in one launch where the shape allows it, then the
+        # weight gradients
+        H.hcw_stack_train_step(xin, Ws, Wn, bias, dyin, 0, -1, flags, y=y, acts=acts,
+                               masks=masks, dx=dx, dW_self=oWs, dW_nbr=oWn, dbias=ob,
+                               workspace=tws, dims=dims)
 
     def capture(xin, dyin, outs=None):
         # the step's launches, recorded once and replayed: no host work per step
@@ -452,9 +447,13 @@ def run_ours(args):
                                                                     L)),
                       dtype=torch.uint8, device=dev)
     reps = 5
-    if dims is not None:
-        # a schedule with shift layers: time its forward and its backward (input
-        # and weight gradients) as two launch sequences
+    family = H.hcw_stack_kernels_used(B, n, d)
+    has_shift = dims is not None and any(v < 0 for v in dims)
+    fused = (family == H.HCW_STACK_STREAMING and d % 256 == 0 and L <= 16 and
+             (not has_shift or (n >= 128 and (B * n) % 256 == 0)))
+    if dims is not None and not fused:
+        # a schedule the one-launch step does not take: time its forward and its
+        # backward (input and weight gradients) as two launch sequences
         f_ms = time_calls(lambda i: H.hcw_stack_fwd(x, Ws, Wn, bias, 0, -1, flags, y=y,
                                                     acts=acts, masks=masks, workspace=fws,
                                                     dims=dims), reps)
@@ -467,8 +466,6 @@ def run_ours(args):
                   % args.schedule: 2.0 * f_flops}
         kernels = dict(zip(kflops, (f_ms, b_ms)))
         dwb_ms = dw_ms = 0.0
-    family = H.hcw_stack_kernels_used(B, n, d)
-    fused = dims is None and family == H.HCW_STACK_STREAMING and d % 256 == 0 and L <= 16
     if dims is None and not fused:
         kflops = None
         fwd_ms = time_calls(lambda i: H.hcw_stack_fwd(x, Ws, Wn, bias, 0, -1, flags, y=y,
@@ -480,22 +477,25 @@ def run_ours(args):
         # weight gradient (bias off), each timed alone on the same inputs
         fdx_ms = time_calls(lambda i: H.hcw_stack_train_step(x, Ws, Wn, bias, dy, 0, -1, flags,
                                                              y=y, acts=acts, masks=masks, dx=dx,
-                                                             want_dw=False, workspace=tws),
+                                                             want_dw=False, workspace=tws,
+                                                             dims=dims),
                             reps)
         dz_step = tws[:L * x.numel() * 2].view(torch.bfloat16).view(L, B, n, d)
         dw_ms = time_calls(lambda i: H.hcw_stack_bwd_weight(x, acts, dz_step, 0, -1, flags,
                                                             dW_self=gWs, dW_nbr=gWn,
-                                                            want_dbias=False, workspace=wws),
+                                                            want_dbias=False, workspace=wws,
+                                                            dims=dims),
                            reps)
         dwb_ms = time_calls(lambda i: H.hcw_stack_bwd_weight(x, acts, dz_step, 0, -1, flags,
                                                              dW_self=gWs, dW_nbr=gWn, dbias=gb,
-                                                             workspace=wws), reps)
-        fdx_name = ("hcw_tc_kernel<FDX,256,32> (stacked forward and input gradient in one "
-                    "launch on SM pairs, top dz written by the last forward layer)")
+                                                             workspace=wws, dims=dims), reps)
+        fdx_name = ("hcw_tc_kernel<FDX,256,%d> (stacked forward and input gradient in one "
+                    "launch on SM pairs, top dz written by the last forward layer)" % (2 * L))
         dw_name = ("hcw_dwp_kernel<256> (weight and bias gradients on SM pairs, a unit per "
                    "layer and 256 x 256 output tile)")
         kernels = {fdx_name: fdx_ms, dw_name: dw_ms}
-        kflops = {fdx_name: 2 * 3.0 * d * d * tokens * L, dw_name: 3.0 * d * d * tokens * L}
+        third = step_flops(B, n, d, L, dims) / 3.0   # one of forward, input and weight gradient
+        kflops = {fdx_name: 2.0 * third, dw_name: third}
     elif dims is None:
         dx_ms = time_calls(lambda i: H.hcw_stack_bwd_data(masks, dy, Ws, Wn, 0, -1, flags,
                                                           dx=dx, dz=dz_all, workspace=dws), reps)
@@ -619,7 +619,8 @@ def run_ours(args):
                        "act": "relu", "bias": True,
                        "l2": "flushed before every timed step (256 MiB write, untimed)",
                        "parallelism": "replicas" if world > 1 else "single",
-                       "stack_kernels": ("shift schedule" if dims is not None else
+                       "stack_kernels": ("one-launch forward + input gradient" if fused else
+                                         "schedule: forward and backward calls" if dims is not None else
                                          "resident" if family == H.HCW_STACK_RESIDENT
                                          else "streaming"),
                        "schedule": args.schedule,

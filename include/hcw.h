@@ -249,7 +249,7 @@ size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags,
  *   dW_self = dW_nbr = dbias = NULL: the forward and the input gradient only
  *   (no weight gradients); dW_self and dW_nbr are given together or not at all.
  * The results equal those of the two separate calls bit for bit.  bf16 on
- * pairs of SMs with up to 16 layers and no shift layers: the forward and the
+ * pairs of SMs with up to 16 layers: the forward and the
  * input gradient run as one persistent launch (the input gradient of a
  * 512-token window starts as soon as its forward is done, and the last
  * forward layer writes the top layer's dz = dy * act'(z) itself), then one
@@ -263,6 +263,21 @@ int hcw_stack_train_step(const void* x, const void* W_self, const void* W_nbr, c
                          size_t ws_bytes, void* stream);
 size_t hcw_stack_train_step_workspace_bytes(int B, int n, int d, int dtype, unsigned flags,
                                             int L);
+
+/*
+ * hcw_stack_train_step on the schedule dims (host array of L layers, as for
+ * hcw_stack_fwd_dims: dims[l] >= 0 a hypercube dimension, -k a shift of Eq. (1)
+ * by k positions).  The results equal those of hcw_stack_fwd_dims followed by
+ * hcw_stack_bwd_dims bit for bit.  The one-launch forward + input gradient
+ * also takes shift layers when n >= 128 and B n is a multiple of 256.  The
+ * workspace is hcw_stack_train_step_workspace_bytes(...).  Errors as for those
+ * two calls.
+ */
+int hcw_stack_train_step_dims(const void* x, const void* W_self, const void* W_nbr,
+                              const float* bias, const void* dy, const int* dims, int L, int B,
+                              int n, int d, int dtype, unsigned flags, void* y, void* acts,
+                              void* masks, void* dx, float* dW_self, float* dW_nbr, float* dbias,
+                              void* workspace, size_t ws_bytes, void* stream);
 
 /*
  * The two halves of hcw_stack_bwd, for callers that want them apart (frozen
@@ -299,6 +314,12 @@ int hcw_stack_bwd_weight(const void* x, const void* acts, const void* dz, int la
                          size_t ws_bytes, void* stream);
 size_t hcw_stack_bwd_weight_workspace_bytes(int B, int n, int d, int dtype, unsigned flags,
                                             int L);
+/* hcw_stack_bwd_weight on the schedule dims (host array of L layers, as for
+ * hcw_stack_fwd_dims); same workspace, results and errors. */
+int hcw_stack_bwd_weight_dims(const void* x, const void* acts, const void* dz, const int* dims,
+                              int L, int B, int n, int d, int dtype, unsigned flags,
+                              float* dW_self, float* dW_nbr, float* dbias, void* workspace,
+                              size_t ws_bytes, void* stream);
 
 /*
  * hcw_layer_bwd_weight for callers that cannot allocate device memory (a

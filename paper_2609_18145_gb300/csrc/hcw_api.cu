@@ -1516,8 +1516,8 @@ size_t step_counter_bytes(long long tokens, int L) {
 // bf16, the rotated or fixed schedule (no shift layers), the streaming kernels
 // on SM pairs, and up to kMaxStackLayers layers.
 bool step_fused(const Shape& sh, int dtype, const Sched& sc, int L) {
-    return dtype == HCW_BF16 && !sc.has_shift(L) && !use_resident(sh) && use_pairs(sh) &&
-           L <= kMaxStackLayers && sh.tokens > 0;
+    return dtype == HCW_BF16 && (!sc.has_shift(L) || shift_stackable(sh)) && !use_resident(sh) &&
+           use_pairs(sh) && L <= kMaxStackLayers && sh.tokens > 0;
 }
 
 size_t step_fwd_region(const Shape& sh, int dtype, unsigned flags, int L) {
@@ -1557,19 +1557,24 @@ int step_fused_launch(const Shape& sh, const void* x, const uint8_t* Ws, const u
     static thread_local TcLaunch<kMaxStepLayers> T;
     memset(&T, 0, sizeof(T));
     for (int l = 0; l < L; ++l) {
-        const int s = sc.dim(sh, l);
+        const int sl = sc.dim(sh, l);
+        // a shift layer: rows in runs of 128 positions, its input as positions
+        const int s = sl >= 0 ? sl : kShiftStackDim;
         CUtensorMap* m = T.maps[l];
-        if (!fwd_maps(m, sh, s, in_ptr(l), Ws + l * wb, Wn + l * wb, out_ptr(l), true))
+        if (!fwd_maps(m, sh, s, in_ptr(l), Ws + l * wb, Wn + l * wb, out_ptr(l), true) ||
+            (sl < 0 && !map_positions(&m[0], in_ptr(l), sh.tokens, sh.n, d, 128)))
             return HCW_ERR_CUDA;
         // the last forward layer also stores the top layer's dz (map 5)
         if (l == L - 1 && !map_rows(&m[5], dzp(L - 1), sh.tokens, d, 1 << s, 32, pw))
             return HCW_ERR_CUDA;
         T.layer[l] = {s, 1 << s, bias ? bias + (size_t)l * d : nullptr, mask(l), nullptr, true,
                       nullptr, false};
+        T.layer[l].shift = sl < 0 ? -sl : 0;
     }
     for (int i = 0; i < L; ++i) {
         const int l = L - 1 - i;   // input-gradient layers from the top down
-        const int s = sc.dim(sh, l);
+        const int sl = sc.dim(sh, l);
+        const int s = sl >= 0 ? sl : kShiftStackDim;
         const int k = 1 << s;
         // stores: g_{l-1} (map 4) and dz_{l-1} (map 5); at l = 0 the stack's dx
         void* out = l == 0 ? dx : (relu ? (resid ? gbuf(l - 1) : nullptr) : dzp(l - 1));
@@ -1583,14 +1588,18 @@ int step_fused_launch(const Shape& sh, const void* x, const uint8_t* Ws, const u
             !map_rows(&m[4], out ? out : dzo, sh.tokens, d, k, 32, pw) ||
             !map_rows(&m[5], dzo ? dzo : out, sh.tokens, d, k, 32, pw))
             return HCW_ERR_CUDA;
+        if (sl < 0 && !map_positions(&m[0], dzp(l), sh.tokens, sh.n, d, 128))
+            return HCW_ERR_CUDA;
         T.layer[L + i] = {s, k, nullptr, nullptr, nullptr, out != nullptr,
                           dzo ? mask(l - 1) : nullptr, dzo != nullptr};
+        T.layer[L + i].shift = sl < 0 ? -sl : 0;
         // the g buffers written by this launch (not dy)
         if (keep_g && i > 0) T.layer[L + i].g_discard = static_cast<const __nv_bfloat16*>(res);
     }
     row_unit_params(T.p, sh, BN, flags, false);
     pair_units(T.p);
     T.p.flags = flags;
+    T.p.seq_n = sh.n;
     T.n_layers = 2 * L;
     T.n_fwd = L;
     const int n_chunks = (int)((sh.tokens + 127) / 128);
@@ -1936,6 +1945,25 @@ int hcw_stack_bwd_data(const void* masks, const void* dy, const void* W_self, co
                              : stack_data_f32(sh, a, (cudaStream_t)stream);
 }
 
+int stack_bwd_weight_impl(const Shape& sh, const void* x, const void* acts, const void* dz,
+                          const Sched& sc, int L, int dtype, unsigned flags, float* dW_self,
+                          float* dW_nbr, float* dbias, void* workspace, size_t ws_bytes,
+                          void* stream);
+
+int hcw_stack_bwd_weight_dims(const void* x, const void* acts, const void* dz, const int* dims,
+                              int L, int B, int n, int d, int dtype, unsigned flags,
+                              float* dW_self, float* dW_nbr, float* dbias, void* workspace,
+                              size_t ws_bytes, void* stream) {
+    Shape sh;
+    if (L < 1) return HCW_ERR_INVALID_ARG;
+    int rc = check_shape(0, -1, B, n, d, dtype, flags, &sh);
+    if (rc) return rc;
+    rc = check_dims(sh, dims, L);
+    if (rc) return rc;
+    return stack_bwd_weight_impl(sh, x, acts, dz, Sched{dims, 0, -1}, L, dtype, flags, dW_self,
+                                 dW_nbr, dbias, workspace, ws_bytes, stream);
+}
+
 int hcw_stack_bwd_weight(const void* x, const void* acts, const void* dz, int layer0, int L,
                          int dim_override, int B, int n, int d, int dtype, unsigned flags,
                          float* dW_self, float* dW_nbr, float* dbias, void* workspace,
@@ -1944,6 +1972,16 @@ int hcw_stack_bwd_weight(const void* x, const void* acts, const void* dz, int la
     if (L < 1) return HCW_ERR_INVALID_ARG;
     int rc = check_shape(layer0, dim_override, B, n, d, dtype, flags, &sh);
     if (rc) return rc;
+    return stack_bwd_weight_impl(sh, x, acts, dz, Sched{nullptr, layer0, dim_override}, L, dtype,
+                                 flags, dW_self, dW_nbr, dbias, workspace, ws_bytes, stream);
+}
+
+int stack_bwd_weight_impl(const Shape& sh, const void* x, const void* acts, const void* dz,
+                          const Sched& sc, int L, int dtype, unsigned flags, float* dW_self,
+                          float* dW_nbr, float* dbias, void* workspace, size_t ws_bytes,
+                          void* stream) {
+    const int d = sh.d;
+    int rc;
     if (sh.tokens == 0) {
         if (!dW_self || !dW_nbr) return HCW_ERR_INVALID_ARG;
         return zero_weight_grads(L, d, dW_self, dW_nbr, dbias, (cudaStream_t)stream);
@@ -1951,7 +1989,7 @@ int hcw_stack_bwd_weight(const void* x, const void* acts, const void* dz, int la
     rc = check_stack_weight(sh, dtype, flags, L, x, acts, dz, dW_self, dW_nbr, dbias, workspace,
                             ws_bytes);
     if (rc) return rc;
-    StackWeight a{x, acts, static_cast<const uint8_t*>(dz), Sched{nullptr, layer0, dim_override}, L,
+    StackWeight a{x, acts, static_cast<const uint8_t*>(dz), sc, L,
                   flags, dW_self, dW_nbr, dbias, static_cast<uint8_t*>(workspace)};
     return dtype == HCW_BF16 ? stack_weight_bf16(sh, a, (cudaStream_t)stream)
                              : stack_weight_f32(sh, a, (cudaStream_t)stream);
@@ -1978,6 +2016,21 @@ int hcw_stack_train_step(const void* x, const void* W_self, const void* W_nbr, c
     return train_step_impl(sh, x, W_self, W_nbr, bias, dy, Sched{nullptr, layer0, dim_override}, L,
                            dtype, flags, y, acts, masks, dx, dW_self, dW_nbr, dbias, workspace,
                            ws_bytes, stream);
+}
+
+int hcw_stack_train_step_dims(const void* x, const void* W_self, const void* W_nbr,
+                              const float* bias, const void* dy, const int* dims, int L, int B,
+                              int n, int d, int dtype, unsigned flags, void* y, void* acts,
+                              void* masks, void* dx, float* dW_self, float* dW_nbr, float* dbias,
+                              void* workspace, size_t ws_bytes, void* stream) {
+    Shape sh;
+    if (L < 1) return HCW_ERR_INVALID_ARG;
+    int rc = check_shape(0, -1, B, n, d, dtype, flags, &sh);
+    if (rc) return rc;
+    rc = check_dims(sh, dims, L);
+    if (rc) return rc;
+    return train_step_impl(sh, x, W_self, W_nbr, bias, dy, Sched{dims, 0, -1}, L, dtype, flags, y,
+                           acts, masks, dx, dW_self, dW_nbr, dbias, workspace, ws_bytes, stream);
 }
 
 int hcw_stack_bwd(const void* x, const void* acts, const void* masks, const void* dy,

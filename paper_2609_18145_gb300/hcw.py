@@ -84,6 +84,10 @@ _SIGNATURES = {
     "hcw_stack_train_step": ([_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P,
                               _P, _P, _P, _P, _P, _SZ, _P], _I),
     "hcw_stack_train_step_workspace_bytes": ([_I, _I, _I, _I, _U, _I], _SZ),
+    "hcw_stack_bwd_weight_dims": ([_P, _P, _P, _P, _I, _I, _I, _I, _I, _U, _P, _P, _P, _P, _SZ,
+                                   _P], _I),
+    "hcw_stack_train_step_dims": ([_P, _P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _U, _P, _P, _P,
+                                   _P, _P, _P, _P, _P, _SZ, _P], _I),
     "hcw_decode_step": ([_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _I, _U, _P, _P, _P],
                         _I),
     "hcw_decode_cache_bytes": ([_P, _I, _I, _I, _I, _I], _SZ),
@@ -503,10 +507,13 @@ def hcw_stack_train_step_workspace_bytes(B: int, n: int, d: int, dtype: int, fla
 def hcw_stack_train_step(x, W_self, W_nbr, bias, dy, layer0: int = 0, dim_override: int = -1,
                          flags: int = 0, y=None, acts=None, masks=None, dx=None, dW_self=None,
                          dW_nbr=None, dbias=None, want_dbias: bool = True,
-                         want_dw: bool = True, workspace=None, stream=None):
+                         want_dw: bool = True, workspace=None, stream=None, dims=None):
     """Forward and backward of a stack in one call; returns (y, acts, masks,
     dx, dW_self[L], dW_nbr[L], dbias[L]).  want_dw=False: the forward and the
-    input gradient only (the weight-gradient outputs are None)."""
+    input gradient only (the weight-gradient outputs are None).  dims (a
+    sequence of L layer links, as for hcw_stack_fwd) calls
+    hcw_stack_train_step_dims instead; layer0 and dim_override are then
+    ignored."""
     _dev(x, W_self, W_nbr, bias, dy, y, acts, masks, dx, dW_self, dW_nbr, dbias, workspace)
     B, n, d = x.shape
     L = W_self.shape[0]
@@ -525,6 +532,15 @@ def hcw_stack_train_step(x, W_self, W_nbr, bias, dy, layer0: int = 0, dim_overri
             dbias = torch.empty(L, d, **f32)
     ws = _workspace(hcw_stack_train_step_workspace_bytes(B, n, d, dt, flags, L), x.device,
                     workspace)
+    if dims is not None:
+        arr = _dims_array(dims, L)
+        _check(lib().hcw_stack_train_step_dims(_ptr(x), _ptr(W_self), _ptr(W_nbr), _ptr(bias),
+                                               _ptr(dy), arr, L, B, n, d, dt, flags, _ptr(y),
+                                               _ptr(acts), _ptr(masks), _ptr(dx),
+                                               _ptr(dW_self), _ptr(dW_nbr), _ptr(dbias),
+                                               _ptr(ws), ws.numel(), _stream(stream)),
+               "hcw_stack_train_step_dims")
+        return y, acts, masks, dx, dW_self, dW_nbr, dbias
     _check(lib().hcw_stack_train_step(_ptr(x), _ptr(W_self), _ptr(W_nbr), _ptr(bias), _ptr(dy),
                                       layer0, L, dim_override, B, n, d, dt, flags, _ptr(y),
                                       _ptr(acts), _ptr(masks), _ptr(dx),
@@ -567,9 +583,10 @@ def hcw_stack_bwd_data(masks, dy, W_self, W_nbr, layer0: int = 0, dim_override: 
 
 def hcw_stack_bwd_weight(x, acts, dz, layer0: int = 0, dim_override: int = -1, flags: int = 0,
                          dW_self=None, dW_nbr=None, dbias=None, want_dbias: bool = True,
-                         workspace=None, stream=None):
+                         workspace=None, stream=None, dims=None):
     """Weight gradients of every layer from its input and dz; returns
-    (dW_self[L], dW_nbr[L], dbias[L] or None)."""
+    (dW_self[L], dW_nbr[L], dbias[L] or None).  dims (L layer links) calls
+    hcw_stack_bwd_weight_dims instead."""
     _dev(x, acts, dz, dW_self, dW_nbr, dbias, workspace)
     B, n, d = x.shape
     L = dz.shape[0]
@@ -581,6 +598,12 @@ def hcw_stack_bwd_weight(x, acts, dz, layer0: int = 0, dim_override: int = -1, f
         dbias = torch.empty(L, d, **f32)
     need = hcw_stack_bwd_weight_workspace_bytes(B, n, d, dt, flags, L)
     ws = _workspace(need, x.device, workspace)
+    if dims is not None:
+        _check(lib().hcw_stack_bwd_weight_dims(_ptr(x), _ptr(acts), _ptr(dz), _dims_array(dims, L),
+                                               L, B, n, d, dt, flags, _ptr(dW_self),
+                                               _ptr(dW_nbr), _ptr(dbias), _ptr(ws), ws.numel(),
+                                               _stream(stream)), "hcw_stack_bwd_weight_dims")
+        return dW_self, dW_nbr, dbias
     _check(lib().hcw_stack_bwd_weight(_ptr(x), _ptr(acts), _ptr(dz), layer0, L, dim_override,
                                       B, n, d, dt, flags, _ptr(dW_self), _ptr(dW_nbr),
                                       _ptr(dbias), _ptr(ws), ws.numel(), _stream(stream)),

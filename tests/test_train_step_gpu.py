@@ -95,3 +95,40 @@ def test_train_step_rejects_overlapping_dy(H):
     with pytest.raises(H.HcwError) as e:
         H.hcw_stack_train_step(x, Ws, Wn, bias, y, 0, -1, flags, y=y)
     assert e.value.status == H.HCW_ERR_ALIASING
+
+
+DIMS_CASES = [
+    # B, n, d, flags, dims (-k: a shift of Eq. (1) by k)
+    (4, 256, 512, CAUSAL | RESIDUAL | RELU, [-1, 7, -1, -1, 5, -1, 4, -1, -1, 2, -1, 1, -1, 0]),
+    (2, 256, 512, RESIDUAL, [-3, -64, 2, -127, -1, 5, -200, 0, -1, 7, -2, 3, -130, -255]),
+    (4, 128, 512, CAUSAL | RESIDUAL | RELU, [-1, 6, -2, 3, -127, 0, 5, -64, 1, -1, 4, 2]),
+    (3, 128, 512, CAUSAL | RESIDUAL | RELU, [-1, 6, -2, 3]),   # 384 tokens: the two calls
+    (8, 64, 128, CAUSAL | RESIDUAL | RELU, [-1, 5, -1, 4]),    # n = 64: the two calls
+]
+
+
+@pytest.mark.parametrize("case", DIMS_CASES, ids=lambda c: "B%d_n%d_d%d_f%d_L%d" % (
+    c[0], c[1], c[2], c[3], len(c[4])))
+def test_train_step_with_a_schedule_equals_the_two_calls(H, case):
+    """hcw_stack_train_step_dims (shift layers in the one-launch forward +
+    input gradient where the shape allows it) against hcw_stack_fwd_dims then
+    hcw_stack_bwd_dims, bit for bit, and its forward against the oracle."""
+    B, n, d, flags, dims = case
+    L = len(dims)
+    pr, x, Ws, Wn, dy, bias = problem(B, n, d, L, seed=13)
+    got = H.hcw_stack_train_step(x, Ws, Wn, bias, dy, flags=flags, dims=dims)
+    y, acts, masks = H.hcw_stack_fwd_dims(x, Ws, Wn, bias, dims, flags)
+    ref = (y, acts, masks) + tuple(H.hcw_stack_bwd_dims(x, acts, masks, dy, Ws, Wn, dims, flags))
+    torch.cuda.synchronize()
+    assert H.hcw_sync_status() == H.HCW_OK
+    for name, a, b in zip(("y", "acts", "masks", "dx", "dW_self", "dW_nbr", "dbias"), got, ref):
+        if a is None or b is None:
+            assert a is None and b is None, name
+            continue
+        assert torch.equal(a, b), name
+    x64 = x.double().cpu().numpy()
+    ry, _, _ = O.stack_fwd(x64, Ws.double().cpu().numpy(), Wn.double().cpu().numpy(),
+                           pr.bias.astype(np.float64), 0, L, -1, flags, round_bf16=True,
+                           dims=dims)
+    err = np.abs(got[0].double().cpu().numpy() - ry).max() / max(np.abs(ry).max(), 1e-30)
+    assert err <= TOL_BF16, err
