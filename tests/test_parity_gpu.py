@@ -870,6 +870,41 @@ def test_batched_weight_gradient_against_fp64_sums(H):
         assert rel(host(gWn[l]), host(gr.T @ xp)) <= 1e-5, l
 
 
+def test_batched_weight_gradient_with_shift_layers_against_fp64_sums(H):
+    """hcw_stack_bwd_weight_dims on a schedule of shift layers and hypercube
+    jumps (the batched launch on SM pairs, shift layers reading their partner
+    rows at p - k): every layer's dW_self, dW_nbr and dbias against fp64 sums
+    of the same bf16 tensors.  A shift layer by k gives every position p >= k
+    of a sequence the partner p - k (Eq. (1)); a jump along dimension s gives
+    the positions with bit s set the partner p - 2^s (causal)."""
+    B, n, d = 4, 256, 512
+    dims = [-1, 7, -1, -3, 5, -1, 4, -64, -1, 2, -255, 1, -1, 0]
+    L = len(dims)
+    flags = CAUSAL | RESIDUAL | RELU
+    pr = synth.problem(B, n, d, L=L, seed=37, w_std=(1 / (2 * d)) ** 0.5)
+    x, _ = dev(pr.x, torch.bfloat16)
+    Ws, _ = dev(pr.W_self, torch.bfloat16)
+    Wn, _ = dev(pr.W_nbr, torch.bfloat16)
+    bias = torch.from_numpy(pr.bias).cuda()
+    y, acts, masks = H.hcw_stack_fwd_dims(x, Ws, Wn, bias, dims, flags)
+    g = torch.Generator().manual_seed(41)
+    dz = (torch.randn(L, B, n, d, generator=g) * 0.05).to(torch.bfloat16).cuda()
+    gWs, gWn, gb = H.hcw_stack_bwd_weight(x, acts, dz, flags=flags, dims=dims)
+    torch.cuda.synchronize()
+    assert H.hcw_sync_status() == H.HCW_OK
+    for l, s in enumerate(dims):
+        inp3 = (x if l == 0 else acts[l - 1]).double()
+        g3 = dz[l].double()
+        assert rel(host(gb[l]), host(g3.reshape(-1, d).sum(0))) <= 1e-5, l
+        assert rel(host(gWs[l]), host(g3.reshape(-1, d).T @ inp3.reshape(-1, d))) <= 1e-5, l
+        k = -s if s < 0 else 1 << s
+        recv = [i for i in range(n) if (i >= k if s < 0 else (i >> s) & 1)]
+        recv = torch.tensor(recv, device="cuda")
+        gr = g3[:, recv].reshape(-1, d)
+        xp = inp3[:, recv - k].reshape(-1, d)
+        assert rel(host(gWn[l]), host(gr.T @ xp)) <= 1e-5, (l, s)
+
+
 def test_launch_counter_counts_kernels(H):
     pr = synth.problem(2, 16, 64, L=1, seed=1)
     x, _ = dev(pr.x, torch.bfloat16)
