@@ -253,8 +253,11 @@ size_t hcw_stack_workspace_bytes(int B, int n, int d, int dtype, unsigned flags,
  * input gradient run as one persistent launch (the input gradient of a
  * 512-token window starts as soon as its forward is done, and the last
  * forward layer writes the top layer's dz = dy * act'(z) itself), then one
- * launch computes the weight and bias gradients.  Other shapes run the two
- * calls.  Errors as for hcw_stack_fwd and hcw_stack_bwd.
+ * launch computes the weight and bias gradients.  That launch starts behind
+ * the first as a programmatic dependent and waits on its completion counters;
+ * when its units leave SM pairs idle, the first launch's last layer runs on
+ * those pairs alone.  Other shapes run the two calls.  Errors as for
+ * hcw_stack_fwd and hcw_stack_bwd.
  */
 int hcw_stack_train_step(const void* x, const void* W_self, const void* W_nbr, const float* bias,
                          const void* dy, int layer0, int L, int dim_override, int B, int n, int d,
