@@ -791,8 +791,8 @@ size_t stack_g_region(const Shape& sh, unsigned flags, int L) {
     const bool keep_g = (flags & HCW_ACT_RELU) && (flags & HCW_RESIDUAL);
     // two g buffers used in turn (see stack_data_bf16)
     size_t r = keep_g ? 2 * a : 0;
-    // schedules with shift layers run layer by layer: two g buffers in turn and
-    // the readers' dz of a shift layer
+    // schedules with shift layers that the stacked launches cannot take run
+    // layer by layer: two g buffers in turn and the readers' dz of a shift layer
     if (r < 3 * a) r = 3 * a;
     return r;
 }
@@ -907,7 +907,9 @@ int stack_data_resident(const Shape& sh, const StackData& a, cudaStream_t st) {
 // bf16 input gradients: the ReLU gradient of the top layer, then one stacked
 // launch per run of <= 16 layers, top down, whose kernel also applies the
 // ReLU gradient of the layer below.
-// bf16 input gradients of a schedule with shift layers, layer by layer: dz_l
+// bf16 input gradients of a schedule with shift layers that the stacked
+// launches cannot take (n < 128, or not whole 256-token row-block pairs, or
+// the resident kernels chosen), layer by layer: dz_l
 // from the ReLU gradient (or a copy of g), then the layer's input gradient --
 // a shift layer with the readers' dz, S_{-k} dz, as its row-aligned partner.
 int stack_data_layers_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
@@ -1513,8 +1515,9 @@ size_t step_counter_bytes(long long tokens, int L) {
 }
 
 // Whether a training step runs its forward and input gradient as one launch:
-// bf16, the rotated or fixed schedule (no shift layers), the streaming kernels
-// on SM pairs, and up to kMaxStackLayers layers.
+// bf16, any schedule whose shift layers the stacked launches take
+// (shift_stackable), the streaming kernels on SM pairs, and up to
+// kMaxStackLayers layers.
 bool step_fused(const Shape& sh, int dtype, const Sched& sc, int L) {
     return dtype == HCW_BF16 && (!sc.has_shift(L) || shift_stackable(sh)) && !use_resident(sh) &&
            use_pairs(sh) && L <= kMaxStackLayers && sh.tokens > 0;
