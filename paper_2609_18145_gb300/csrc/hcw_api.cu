@@ -411,8 +411,8 @@ void row_unit_params(TcParams& p, const Shape& sh, int BN, unsigned flags, bool 
 // pair: the weight boxes hold half a column tile (each CTA of a pair loads
 // its half of B)
 bool fwd_maps(CUtensorMap* m, const Shape& sh, int s, const void* x, const void* Ws,
-              const void* Wn, const void* y, bool pair = false) {
-    const int d = sh.d, BN = pick_bn(d), k = 1 << s;
+              const void* Wn, const void* y, bool pair = false, int bn = 0) {
+    const int d = sh.d, BN = bn ? bn : pick_bn(d), k = 1 << s;
     const int pw = epi_patch_cols(BN);
     const int box_o = pair ? BN / 2 : BN;
     if (!map_rows(&m[0], x, sh.tokens, d, k, 128) || !map_weight(&m[1], Ws, d, box_o) ||
@@ -1535,7 +1535,18 @@ int step_fused_launch(const Shape& sh, const void* x, const uint8_t* Ws, const u
                       const float* bias, const void* dy, const Sched& sc, int L, unsigned flags,
                       void* y, void* acts, void* masks, void* dx, uint8_t* dz, uint8_t* gws,
                       int* counters, cudaStream_t st, int dw_pairs = 0) {
-    const int d = sh.d, BN = pick_bn(d), pw = epi_patch_cols(BN);
+    // 128-column tiles when 256-column ones would leave more than half of the
+    // SM pairs without a unit of a layer (few tokens: the launch is the layer
+    // chain, and narrower units shorten each of its steps)
+    const int sms_all = sm_count();
+    int BN = pick_bn(sh.d);
+    {
+        TcParams q;
+        row_unit_params(q, sh, BN, flags, false);
+        pair_units(q);
+        if (BN == 256 && 2 * q.n_units <= sms_all / 2) BN = 128;
+    }
+    const int d = sh.d, pw = epi_patch_cols(BN);
     const size_t ab = sh.act_bytes, a256 = align256(ab), wb = (size_t)d * d * 2;
     const size_t mb = mask_bytes(sh);
     const bool relu = (flags & HCW_ACT_RELU) != 0;
@@ -1564,7 +1575,7 @@ int step_fused_launch(const Shape& sh, const void* x, const uint8_t* Ws, const u
         // a shift layer: rows in runs of 128 positions, its input as positions
         const int s = sl >= 0 ? sl : kShiftStackDim;
         CUtensorMap* m = T.maps[l];
-        if (!fwd_maps(m, sh, s, in_ptr(l), Ws + l * wb, Wn + l * wb, out_ptr(l), true) ||
+        if (!fwd_maps(m, sh, s, in_ptr(l), Ws + l * wb, Wn + l * wb, out_ptr(l), true, BN) ||
             (sl < 0 && !map_positions(&m[0], in_ptr(l), sh.tokens, sh.n, d, 128)))
             return HCW_ERR_CUDA;
         // the last forward layer also stores the top layer's dz (map 5)

@@ -156,8 +156,8 @@ cudaError_t launch_tc_stack(int mode, int BN, const TcLaunch<kMaxStackLayers>& L
 // cta_group::2; BN 256, even grid).  L.p counts pair units: row-block pairs.
 cudaError_t launch_tc_stack_pair(int mode, int BN, const TcLaunch<kMaxStackLayers>& L, int grid,
                                  cudaStream_t stream);
-// MODE_FDX on clusters of two CTAs (BN 256, even grid): L.n_fwd forward layers
-// followed by the input gradient of those layers, top down.
+// MODE_FDX on clusters of two CTAs (BN 256 or 128, even grid): L.n_fwd forward
+// layers followed by the input gradient of those layers, top down.
 cudaError_t launch_tc_step_pair(int BN, const TcLaunch<kMaxStepLayers>& L, int grid,
                                 cudaStream_t stream);
 

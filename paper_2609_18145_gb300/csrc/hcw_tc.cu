@@ -2143,8 +2143,10 @@ cudaError_t launch_tc_stack_pair(int mode, int BN, const TcLaunch<kMaxStackLayer
 
 cudaError_t launch_tc_step_pair(int BN, const TcLaunch<kMaxStepLayers>& L, int grid,
                                 cudaStream_t st) {
-    if (BN != 256 || grid % 2) return cudaErrorInvalidValue;
-    return launch_one<MODE_FDX, 256, kMaxStepLayers, true>(L, grid, st);
+    if (grid % 2) return cudaErrorInvalidValue;
+    if (BN == 256) return launch_one<MODE_FDX, 256, kMaxStepLayers, true>(L, grid, st);
+    if (BN == 128) return launch_one<MODE_FDX, 128, kMaxStepLayers, true>(L, grid, st);
+    return cudaErrorInvalidValue;
 }
 
 size_t tc_smem_bytes(int BN) {
