@@ -1516,11 +1516,14 @@ size_t step_counter_bytes(long long tokens, int L) {
 
 // Whether a training step runs its forward and input gradient as one launch:
 // bf16, any schedule whose shift layers the stacked launches take
-// (shift_stackable), the streaming kernels on SM pairs, and up to
-// kMaxStackLayers layers.
+// (shift_stackable), the streaming kernels on SM pairs (d a multiple of 128),
+// and up to kMaxStackLayers layers.
 bool step_fused(const Shape& sh, int dtype, const Sched& sc, int L) {
+    // 256- or 128-column tiles on pairs (d = 128 takes the latter), at least
+    // two row blocks
+    const bool pairs = use_pairs(sh) || (pick_bn(sh.d) == 128 && sh.tokens / 2 > 128);
     return dtype == HCW_BF16 && (!sc.has_shift(L) || shift_stackable(sh)) && !use_resident(sh) &&
-           use_pairs(sh) && L <= kMaxStackLayers && sh.tokens > 0;
+           pairs && L <= kMaxStackLayers && sh.tokens > 0;
 }
 
 size_t step_fwd_region(const Shape& sh, int dtype, unsigned flags, int L) {

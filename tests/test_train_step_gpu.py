@@ -44,7 +44,10 @@ CASES = [
     (2, 128, 256, 1, 0, CAUSAL | RESIDUAL | RELU),     # one layer
     (6, 64, 512, 7, 2, RESIDUAL | RELU),               # non-causal
     (3, 64, 512, 2, 0, CAUSAL | RESIDUAL | RELU),
-    (8, 64, 128, 6, 0, RESIDUAL | RELU),               # not on pairs: the two calls
+    (8, 64, 128, 6, 0, RESIDUAL | RELU),               # d = 128: 128-column tiles on pairs
+    (32, 64, 128, 6, 1, CAUSAL | RESIDUAL | RELU),
+    (2, 64, 128, 3, 0, RESIDUAL | RELU),               # 128 tokens: the two calls
+    (4, 64, 192, 3, 0, CAUSAL | RESIDUAL | RELU),      # 64-column tiles: the two calls
     # enough layers for the batched weight gradient on SM pairs, which then
     # starts behind the fused launch and waits on its completion counters
     (4, 256, 512, 12, 5, CAUSAL | RESIDUAL | RELU),
