@@ -294,7 +294,9 @@ struct WPlan {
         units;
 };
 
-WPlan plan_dw(long long tokens, int d, unsigned flags) {
+// The split of the token range of the weight gradient into units: one layer's,
+// or `layers` layers' sharing one launch.
+WPlan plan_dw(long long tokens, int d, unsigned flags, int layers = 1) {
     WPlan w;
     const int BN = pick_bn(d);
     const long long Mh = tokens / 2;
@@ -304,7 +306,7 @@ WPlan plan_dw(long long tokens, int d, unsigned flags) {
     w.nkb_self = 2 * w.qb;
     w.nkb_nbr = (flags & HCW_CAUSAL) ? w.qb : 2 * w.qb;
     const int tiles = w.n_ot * w.n_nt;
-    const long long total_kb = (long long)tiles * (w.nkb_self + w.nkb_nbr);
+    const long long total_kb = (long long)layers * tiles * (w.nkb_self + w.nkb_nbr);
     const int sms = sm_count();
     // the fewest token blocks per unit (at least 4, i.e. 256 tokens) whose
     // units still fit in one wave of persistent CTAs: makespan = kpu blocks
@@ -314,7 +316,8 @@ WPlan plan_dw(long long tokens, int d, unsigned flags) {
     // the count cannot drop further, even if the tiles alone exceed the SMs)
     const long long kpu_max = w.nkb_self > w.nkb_nbr ? w.nkb_self : w.nkb_nbr;
     while (kpu < kpu_max &&
-           tiles * ((w.nkb_self + kpu - 1) / kpu + (w.nkb_nbr + kpu - 1) / kpu) > sms)
+           (long long)layers * tiles *
+                   ((w.nkb_self + kpu - 1) / kpu + (w.nkb_nbr + kpu - 1) / kpu) > sms)
         ++kpu;
     w.kb_per_unit = (int)kpu;
     w.splits_self = (int)((w.nkb_self + kpu - 1) / kpu);
@@ -805,10 +808,36 @@ size_t stack_data_ws(const Shape& sh, int dtype, unsigned flags, int L) {
 
 // bf16: [unit counter (256 B)][weight-gradient workspace][the readers' dz of a
 // shift layer (one activation buffer)]
+// True when `cnt` layers' whole-range weight-gradient units (one per output
+// tile) would leave most SMs idle: their launch then splits the token range
+// of every layer (split_dw_ws).
+bool split_dw_layers(const Shape& sh, unsigned flags, int cnt) {
+    const WPlan w = plan_dw(sh.tokens, sh.d, flags);
+    return cnt * w.n_ot * w.n_nt * 2 < sm_count();
+}
+
+// Workspace of the split launch over `cnt` layers: the fp32 partials
+// [cnt][2][splits][d][d] (when the token range is split) and the column-sum
+// partials of the cnt dbias rows.
+size_t split_dw_ws(const Shape& sh, unsigned flags, int cnt) {
+    const WPlan w = plan_dw(sh.tokens, sh.d, flags, cnt);
+    const size_t dd = (size_t)sh.d * sh.d * 4;
+    const size_t part = w.splits_max > 1 ? align256((size_t)cnt * 2 * w.splits_max * dd) : 0;
+    return part + align256((size_t)cnt * colsum_workspace_bytes(sh.tokens, sh.d));
+}
+
 size_t stack_weight_ws(const Shape& sh, int dtype, unsigned flags, int L) {
     const WsLayout w = ws_layout(sh.tokens, sh.d, dtype, flags);
-    if (dtype == HCW_BF16) return 256 + align256(w.w_bytes) + align256(sh.act_bytes);
-    return w.w_bytes;
+    if (dtype != HCW_BF16) return w.w_bytes;
+    size_t body = align256(w.w_bytes) + align256(sh.act_bytes);
+    // the launches of kMaxStackLayers layers and the last, shorter one
+    const int counts[2] = {L < kMaxStackLayers ? L : kMaxStackLayers, L % kMaxStackLayers};
+    for (int cnt : counts)
+        if (cnt > 0 && split_dw_layers(sh, flags, cnt)) {
+            const size_t need = split_dw_ws(sh, flags, cnt);
+            if (need > body) body = need;
+        }
+    return 256 + body;
 }
 
 size_t stack_dz_bytes(const Shape& sh, int L) { return align256((size_t)L * sh.act_bytes); }
@@ -1050,6 +1079,80 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
 // (whole token range per tile, units handed out longest first; the kernel
 // also sums dz's columns into dbias), or layer by layer when their tiles
 // cannot fill the GPU.
+// The weight gradients of layers l0 .. l0 + cnt - 1 when each has few output
+// tiles (small d): one launch whose units split every layer's token range
+// (units of one size over all the layers, claimed dynamically), then one
+// reduction launch over all the layers' partials and one batched column sum
+// for dbias -- three launches in place of four per layer.  Hypercube layers
+// only (a shift layer takes the launches of stack_weight_bf16).
+int split_dw_launch(const Shape& sh, const StackWeight& a, int l0, int cnt, uint8_t* wws,
+                    int* sched, cudaStream_t st) {
+    const int d = sh.d, BN = pick_bn(d);
+    const size_t ab = sh.act_bytes, dd = (size_t)d * d;
+    const WPlan w = plan_dw(sh.tokens, d, a.flags, cnt);
+    const bool split = w.splits_max > 1;
+    const size_t part_floats = (size_t)2 * w.splits_max * dd;   // one layer's partials
+    float* part = reinterpret_cast<float*>(wws);
+    float* colp = reinterpret_cast<float*>(wws + (split ? align256(cnt * part_floats * 4) : 0));
+    static thread_local TcLaunch<kMaxStackLayers> T;
+    memset(&T, 0, sizeof(T));
+    for (int i = 0; i < cnt; ++i) {
+        const int l = l0 + i;
+        const int s = a.sc.dim(sh, l);
+        if (s < 0) return HCW_ERR_UNSUPPORTED;
+        const int k = 1 << s;
+        const void* x = l == 0 ? a.x : static_cast<const uint8_t*>(a.acts) + (size_t)(l - 1) * ab;
+        float* gs = a.dWs + (size_t)l * dd;
+        CUtensorMap* m = T.maps[i];
+        if (!map_rows_blocks(&m[0], a.dz + (size_t)l * ab, sh.tokens, d, k, 64, 2) ||
+            !map_rows_blocks(&m[1], x, sh.tokens, d, k, 64, BN / 64) ||
+            !map_f32_patches(&m[3], split ? (const void*)(part + i * part_floats) : (const void*)gs,
+                             split ? 2ll * w.splits_max * d : d, d) ||
+            !map_f32_patches(&m[4], gs, d, d) ||
+            !map_f32_patches(&m[5], a.dWn + (size_t)l * dd, d, d))
+            return HCW_ERR_CUDA;
+        m[2] = m[1];   // unused by the weight gradient
+        T.layer[i] = {s, k, nullptr, nullptr, nullptr, false, nullptr, false};
+        // a unit over the whole token range sums dbias on the way (helper warps)
+        T.layer[i].colsum = (a.dbias && w.splits_self == 1) ? a.dbias + (size_t)l * d : nullptr;
+    }
+    TcParams& p = T.p;
+    p.d = d;
+    p.Mh = (int)(sh.tokens / 2);
+    p.n_nt = w.n_nt;
+    p.n_ot = w.n_ot;
+    p.qb = w.qb;
+    p.nkb_self = w.nkb_self;
+    p.nkb_nbr = w.nkb_nbr;
+    p.kb_per_unit = w.kb_per_unit;
+    p.splits_self = w.splits_self;
+    p.splits_nbr = w.splits_nbr;
+    p.splits_max = w.splits_max;
+    p.causal = (a.flags & HCW_CAUSAL) ? 1 : 0;
+    p.n_units = w.units;
+    p.seq_n = sh.n;
+    p.timeout_ns = g_timeout_ns;
+    T.n_layers = cnt;
+    T.sched = sched;
+    if (cudaMemsetAsync(sched, 0, sizeof(int), st) != cudaSuccess) return HCW_ERR_CUDA;
+    const int sms = sm_count(), total = w.units * cnt;
+    int rc = launched(launch_tc_stack(MODE_DW, BN, T, total < sms ? total : sms, st), 1);
+    if (rc) return rc;
+    if (split) {
+        rc = launched(launch_splitk_reduce(part, w.splits_max, w.splits_self, w.splits_nbr, d,
+                                           a.dWs + (size_t)l0 * dd, a.dWn + (size_t)l0 * dd, st,
+                                           cnt, part_floats, dd),
+                      1);
+        if (rc) return rc;
+    }
+    if (a.dbias && w.splits_self > 1)
+        rc = launched(launch_colsum_bf16_batched(
+                          reinterpret_cast<const __nv_bfloat16*>(a.dz + (size_t)l0 * ab), cnt,
+                          sh.tokens, d, colp, a.dbias + (size_t)l0 * d, st),
+                      2);
+    return rc;
+}
+
 int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
     const int d = sh.d, BN = pick_bn(d), L = a.L;
     const size_t ab = sh.act_bytes;
@@ -1116,15 +1219,9 @@ int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
     int rc;
     for (int l0 = 0; l0 < L; l0 += kMaxStackLayers) {
         const int cnt = L - l0 < kMaxStackLayers ? L - l0 : kMaxStackLayers;
-        if (cnt * tiles * 2 < sms) {
-            for (int l = l0; l < l0 + cnt; ++l) {
-                Shape shl = sh;
-                shl.s = a.sc.dim(sh, l);
-                rc = dw_bf16(shl, act(l), dz(l), a.flags, a.dWs + (size_t)l * d * d,
-                             a.dWn + (size_t)l * d * d, a.dbias ? a.dbias + (size_t)l * d : nullptr,
-                             wws, st);
-                if (rc) return rc;
-            }
+        if (split_dw_layers(sh, a.flags, cnt)) {
+            rc = split_dw_launch(sh, a, l0, cnt, wws, sched, st);
+            if (rc) return rc;
             continue;
         }
         memset(&T, 0, sizeof(T));

@@ -344,10 +344,13 @@ cudaError_t launch_colsum_bf16(const __nv_bfloat16* dz, long long rows, int d, f
 // batch * colsum_workspace_bytes(rows, d).
 cudaError_t launch_colsum_bf16_batched(const __nv_bfloat16* dz, int batch, long long rows, int d,
                                        float* partial, float* out, cudaStream_t st);
-// out_w[o][k] = sum_{s < splits_w} partial[w][s][o][k] for w in {self, nbr}
+// out_w[o][k] = sum_{s < splits_w} partial[w][s][o][k] for w in {self, nbr};
+// `layers` such problems, partials part_stride floats apart, outputs
+// out_stride floats apart
 cudaError_t launch_splitk_reduce(const float* partial, int splits_max, int splits_self,
                                  int splits_nbr, int d, float* dWs, float* dWn,
-                                 cudaStream_t st);
+                                 cudaStream_t st, int layers = 1, size_t part_stride = 0,
+                                 size_t out_stride = 0);
 cudaError_t launch_partner_table(int s, int n, unsigned flags, int* out, cudaStream_t st);
 // out[b][i] = in[b][i - k] where 0 <= i - k < n, else 0 (bf16 [rows][d], k of
 // either sign): the row-aligned partner operand of a shift layer.

@@ -343,27 +343,43 @@ __global__ void __launch_bounds__(1024) colsum_final_kernel(const float* __restr
     }
 }
 
-__global__ void splitk_reduce_kernel(const float* __restrict__ partial, int splits_max,
-                                     int splits_self, int splits_nbr, int d,
-                                     float* __restrict__ dWs, float* __restrict__ dWn) {
-    const size_t dd = (size_t)d * d;
-    const size_t total4 = dd / 4;
-    for (size_t t = (size_t)blockIdx.x * blockDim.x + threadIdx.x; t < 2 * total4;
-         t += (size_t)gridDim.x * blockDim.x) {
-        const int which = t >= total4;
-        const size_t e4 = t - which * total4;
-        const int S = which ? splits_nbr : splits_self;
-        if (S <= 1) continue;   // written directly by the GEMM
-        const float4* src = reinterpret_cast<const float4*>(partial + (size_t)which * splits_max * dd);
-        float4 a = src[e4];
-        for (int sp = 1; sp < S; ++sp) {
-            float4 b = src[(size_t)sp * total4 + e4];
+// out_w[l][o][k] = sum over the splits s of partial[l][w][s][o][k], w in {self,
+// partner}.  Block: 64 float4 columns x 8 split lanes; lane y adds the splits
+// y, y + 8, ... in order, then the 8 lane sums meet in shared memory in lane
+// order (deterministic).  grid.y = the part, grid.z = the layer.
+__global__ void __launch_bounds__(512) splitk_reduce_kernel(
+    const float* __restrict__ partial, int splits_max, int splits_self, int splits_nbr, int d,
+    size_t part_stride, float* __restrict__ dWs, float* __restrict__ dWn, size_t out_stride) {
+    __shared__ float4 red[8][64];
+    const int which = blockIdx.y;
+    const int S = which ? splits_nbr : splits_self;
+    if (S <= 1) return;   // written directly by the GEMM
+    const size_t total4 = (size_t)d * d / 4;
+    const size_t e4 = (size_t)blockIdx.x * 64 + threadIdx.x;
+    const float4* src = reinterpret_cast<const float4*>(
+        partial + blockIdx.z * part_stride + (size_t)which * splits_max * d * d);
+    float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (e4 < total4) {
+        for (int sp = threadIdx.y; sp < S; sp += 8) {
+            const float4 b = src[(size_t)sp * total4 + e4];
             a.x += b.x;
             a.y += b.y;
             a.z += b.z;
             a.w += b.w;
         }
-        reinterpret_cast<float4*>(which ? dWn : dWs)[e4] = a;
+    }
+    red[threadIdx.y][threadIdx.x] = a;
+    __syncthreads();
+    if (threadIdx.y == 0 && e4 < total4) {
+#pragma unroll
+        for (int y = 1; y < 8; ++y) {
+            const float4 b = red[y][threadIdx.x];
+            a.x += b.x;
+            a.y += b.y;
+            a.z += b.z;
+            a.w += b.w;
+        }
+        reinterpret_cast<float4*>((which ? dWn : dWs) + blockIdx.z * out_stride)[e4] = a;
     }
 }
 
@@ -492,10 +508,13 @@ cudaError_t launch_colsum_bf16(const __nv_bfloat16* dz, long long rows, int d, f
 
 cudaError_t launch_splitk_reduce(const float* partial, int splits_max, int splits_self,
                                  int splits_nbr, int d, float* dWs, float* dWn,
-                                 cudaStream_t st) {
+                                 cudaStream_t st, int layers, size_t part_stride,
+                                 size_t out_stride) {
     const size_t total4 = (size_t)d * d / 4;
-    splitk_reduce_kernel<<<blocks_for(2 * total4, 256), 256, 0, st>>>(
-        partial, splits_max, splits_self, splits_nbr, d, dWs, dWn);
+    if (layers < 1) return cudaSuccess;
+    splitk_reduce_kernel<<<dim3((unsigned)((total4 + 63) / 64), 2, (unsigned)layers),
+                           dim3(64, 8), 0, st>>>(partial, splits_max, splits_self, splits_nbr, d,
+                                                 part_stride, dWs, dWn, out_stride);
     return cudaGetLastError();
 }
 
