@@ -817,13 +817,15 @@ bool split_dw_layers(const Shape& sh, unsigned flags, int cnt) {
 }
 
 // Workspace of the split launch over `cnt` layers: the fp32 partials
-// [cnt][2][splits][d][d] (when the token range is split) and the column-sum
-// partials of the cnt dbias rows.
+// [cnt][2][splits][d][d] and the dbias partials [cnt][splits of the self
+// part][d] (when the token range is split).
 size_t split_dw_ws(const Shape& sh, unsigned flags, int cnt) {
     const WPlan w = plan_dw(sh.tokens, sh.d, flags, cnt);
     const size_t dd = (size_t)sh.d * sh.d * 4;
     const size_t part = w.splits_max > 1 ? align256((size_t)cnt * 2 * w.splits_max * dd) : 0;
-    return part + align256((size_t)cnt * colsum_workspace_bytes(sh.tokens, sh.d));
+    const size_t bpart =
+        w.splits_self > 1 ? align256((size_t)cnt * w.splits_self * sh.d * 4) : 0;
+    return part + bpart;
 }
 
 size_t stack_weight_ws(const Shape& sh, int dtype, unsigned flags, int L) {
@@ -1081,10 +1083,11 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
 // cannot fill the GPU.
 // The weight gradients of layers l0 .. l0 + cnt - 1 when each has few output
 // tiles (small d): one launch whose units split every layer's token range
-// (units of one size over all the layers, claimed dynamically), then one
-// reduction launch over all the layers' partials and one batched column sum
-// for dbias -- three launches in place of four per layer.  Hypercube layers
-// only (a shift layer takes the launches of stack_weight_bf16).
+// (units of one size over all the layers, claimed dynamically; the self
+// part's units also sum their dz columns, the dbias of their split), then
+// one reduction launch over all the layers' partials -- two launches in place
+// of four per layer.  Hypercube layers only (a shift layer takes the launches
+// of stack_weight_bf16).
 int split_dw_launch(const Shape& sh, const StackWeight& a, int l0, int cnt, uint8_t* wws,
                     int* sched, cudaStream_t st) {
     const int d = sh.d, BN = pick_bn(d);
@@ -1093,7 +1096,7 @@ int split_dw_launch(const Shape& sh, const StackWeight& a, int l0, int cnt, uint
     const bool split = w.splits_max > 1;
     const size_t part_floats = (size_t)2 * w.splits_max * dd;   // one layer's partials
     float* part = reinterpret_cast<float*>(wws);
-    float* colp = reinterpret_cast<float*>(wws + (split ? align256(cnt * part_floats * 4) : 0));
+    float* bpart = reinterpret_cast<float*>(wws + (split ? align256(cnt * part_floats * 4) : 0));
     static thread_local TcLaunch<kMaxStackLayers> T;
     memset(&T, 0, sizeof(T));
     for (int i = 0; i < cnt; ++i) {
@@ -1113,8 +1116,12 @@ int split_dw_launch(const Shape& sh, const StackWeight& a, int l0, int cnt, uint
             return HCW_ERR_CUDA;
         m[2] = m[1];   // unused by the weight gradient
         T.layer[i] = {s, k, nullptr, nullptr, nullptr, false, nullptr, false};
-        // a unit over the whole token range sums dbias on the way (helper warps)
-        T.layer[i].colsum = (a.dbias && w.splits_self == 1) ? a.dbias + (size_t)l * d : nullptr;
+        // the self part's units sum dz's columns on the way (helper warps):
+        // dbias itself for units over the whole token range, else the split's
+        // partial sums
+        if (a.dbias)
+            T.layer[i].colsum = w.splits_self == 1 ? a.dbias + (size_t)l * d
+                                                   : bpart + (size_t)i * w.splits_self * d;
     }
     TcParams& p = T.p;
     p.d = d;
@@ -1138,18 +1145,12 @@ int split_dw_launch(const Shape& sh, const StackWeight& a, int l0, int cnt, uint
     const int sms = sm_count(), total = w.units * cnt;
     int rc = launched(launch_tc_stack(MODE_DW, BN, T, total < sms ? total : sms, st), 1);
     if (rc) return rc;
-    if (split) {
+    if (split)
         rc = launched(launch_splitk_reduce(part, w.splits_max, w.splits_self, w.splits_nbr, d,
                                            a.dWs + (size_t)l0 * dd, a.dWn + (size_t)l0 * dd, st,
-                                           cnt, part_floats, dd),
+                                           cnt, part_floats, dd, a.dbias ? bpart : nullptr,
+                                           a.dbias ? a.dbias + (size_t)l0 * d : nullptr),
                       1);
-        if (rc) return rc;
-    }
-    if (a.dbias && w.splits_self > 1)
-        rc = launched(launch_colsum_bf16_batched(
-                          reinterpret_cast<const __nv_bfloat16*>(a.dz + (size_t)l0 * ab), cnt,
-                          sh.tokens, d, colp, a.dbias + (size_t)l0 * d, st),
-                      2);
     return rc;
 }
 

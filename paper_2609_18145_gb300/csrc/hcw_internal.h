@@ -62,7 +62,8 @@ struct TcLayer {
     bool out;                     // DX: the input gradient dx is stored (map 4)
     const uint32_t* mprev;        // DX: ReLU mask words of the layer below (fused ReLU grad)
     bool dz_out;                  // DX: dz of the layer below = dx * mask is stored (map 5)
-    float* colsum;                // DW, whole token range per unit: dbias = column sums of dz
+    float* colsum;                // DW: dbias = column sums of dz; with the self part split,
+                                  // the sums of each split, [split][d]
     float* dws;                   // MODE_DWF: dW_self, dW_nbr [d][d] fp32 (stored directly)
     float* dwn;
     // FWD / DX of one layer: the partner part reads the same rows of a second
@@ -346,11 +347,13 @@ cudaError_t launch_colsum_bf16_batched(const __nv_bfloat16* dz, int batch, long 
                                        float* partial, float* out, cudaStream_t st);
 // out_w[o][k] = sum_{s < splits_w} partial[w][s][o][k] for w in {self, nbr};
 // `layers` such problems, partials part_stride floats apart, outputs
-// out_stride floats apart
+// out_stride floats apart; with bpart, also dbias[l][o] = sum over the
+// splits_self splits of bpart[l][s][o]
 cudaError_t launch_splitk_reduce(const float* partial, int splits_max, int splits_self,
                                  int splits_nbr, int d, float* dWs, float* dWn,
                                  cudaStream_t st, int layers = 1, size_t part_stride = 0,
-                                 size_t out_stride = 0);
+                                 size_t out_stride = 0, const float* bpart = nullptr,
+                                 float* dbias = nullptr);
 cudaError_t launch_partner_table(int s, int n, unsigned flags, int* out, cudaStream_t st);
 // out[b][i] = in[b][i - k] where 0 <= i - k < n, else 0 (bf16 [rows][d], k of
 // either sign): the row-aligned partner operand of a shift layer.

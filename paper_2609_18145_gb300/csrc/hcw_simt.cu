@@ -344,20 +344,24 @@ __global__ void __launch_bounds__(1024) colsum_final_kernel(const float* __restr
 }
 
 // out_w[l][o][k] = sum over the splits s of partial[l][w][s][o][k], w in {self,
-// partner}.  Block: 64 float4 columns x 8 split lanes; lane y adds the splits
-// y, y + 8, ... in order, then the 8 lane sums meet in shared memory in lane
-// order (deterministic).  grid.y = the part, grid.z = the layer.
+// partner}; grid.y = 3 adds dbias[l][o] = sum over the self part's splits of
+// bpart[l][s][o].  Block: 64 float4 columns x 8 split lanes; lane y adds the
+// splits y, y + 8, ... in order, then the 8 lane sums meet in shared memory
+// in lane order (deterministic).  grid.y = the part, grid.z = the layer.
 __global__ void __launch_bounds__(512) splitk_reduce_kernel(
     const float* __restrict__ partial, int splits_max, int splits_self, int splits_nbr, int d,
-    size_t part_stride, float* __restrict__ dWs, float* __restrict__ dWn, size_t out_stride) {
+    size_t part_stride, float* __restrict__ dWs, float* __restrict__ dWn, size_t out_stride,
+    const float* __restrict__ bpart, float* __restrict__ dbias) {
     __shared__ float4 red[8][64];
     const int which = blockIdx.y;
-    const int S = which ? splits_nbr : splits_self;
+    const int S = which == 1 ? splits_nbr : splits_self;
     if (S <= 1) return;   // written directly by the GEMM
-    const size_t total4 = (size_t)d * d / 4;
+    const size_t total4 = which == 2 ? (size_t)d / 4 : (size_t)d * d / 4;
     const size_t e4 = (size_t)blockIdx.x * 64 + threadIdx.x;
+    if ((size_t)blockIdx.x * 64 >= total4) return;   // (the dbias rows are short)
     const float4* src = reinterpret_cast<const float4*>(
-        partial + blockIdx.z * part_stride + (size_t)which * splits_max * d * d);
+        which == 2 ? bpart + (size_t)blockIdx.z * splits_self * d
+                   : partial + blockIdx.z * part_stride + (size_t)which * splits_max * d * d);
     float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
     if (e4 < total4) {
         for (int sp = threadIdx.y; sp < S; sp += 8) {
@@ -379,7 +383,9 @@ __global__ void __launch_bounds__(512) splitk_reduce_kernel(
             a.z += b.z;
             a.w += b.w;
         }
-        reinterpret_cast<float4*>((which ? dWn : dWs) + blockIdx.z * out_stride)[e4] = a;
+        float* out = which == 2 ? dbias + (size_t)blockIdx.z * d
+                                : (which ? dWn : dWs) + blockIdx.z * out_stride;
+        reinterpret_cast<float4*>(out)[e4] = a;
     }
 }
 
@@ -509,12 +515,13 @@ cudaError_t launch_colsum_bf16(const __nv_bfloat16* dz, long long rows, int d, f
 cudaError_t launch_splitk_reduce(const float* partial, int splits_max, int splits_self,
                                  int splits_nbr, int d, float* dWs, float* dWn,
                                  cudaStream_t st, int layers, size_t part_stride,
-                                 size_t out_stride) {
+                                 size_t out_stride, const float* bpart, float* dbias) {
     const size_t total4 = (size_t)d * d / 4;
     if (layers < 1) return cudaSuccess;
-    splitk_reduce_kernel<<<dim3((unsigned)((total4 + 63) / 64), 2, (unsigned)layers),
+    const unsigned parts = (bpart && dbias) ? 3 : 2;
+    splitk_reduce_kernel<<<dim3((unsigned)((total4 + 63) / 64), parts, (unsigned)layers),
                            dim3(64, 8), 0, st>>>(partial, splits_max, splits_self, splits_nbr, d,
-                                                 part_stride, dWs, dWn, out_stride);
+                                                 part_stride, dWs, dWn, out_stride, bpart, dbias);
     return cudaGetLastError();
 }
 

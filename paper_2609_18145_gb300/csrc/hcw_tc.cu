@@ -1551,9 +1551,9 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                 const WUnit& w = wu;
                 if (e < kDwHelpers &&
                     !helper_pass(w.kb1 - w.kb0,
-                                 ly.colsum != nullptr && w.which == 0 && w.nt == 0 &&
-                                     p.splits_self == 1,
-                                 ly.colsum, w.ot * kBlockM)) {
+                                 ly.colsum != nullptr && w.which == 0 && w.nt == 0,
+                                 ly.colsum + (p.splits_self > 1 ? (size_t)w.split * p.d : 0),
+                                 w.ot * kBlockM)) {
                     alive = false;
                     break;
                 }
