@@ -790,31 +790,74 @@ def run_workload(args):
 
     # end to end through the public API with host buffers: every step copies
     # x and dy in from pinned memory and its result out (the weight and bias
-    # gradients, or y for the forward), serially
+    # gradients, or y for the forward), pipelined as a training loop runs
+    # them: step i + 1's inputs come in on one copy stream and step i's result
+    # goes out on another while the steps compute (double-buffered inputs and
+    # results); the span runs from the first input copy to the last result
+    # copy, and each step still flushes L2 inside it
     x_h = torch.empty(x.shape, dtype=x.dtype, pin_memory=True)
     dy_h = torch.empty(dy.shape, dtype=dy.dtype, pin_memory=True)
     x_h.copy_(x)
     dy_h.copy_(dy)
     outs = (y,) if fwd_only else (gWs, gWn, gb)
     outs_h = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
-    x_d, dy_d = torch.empty_like(x), torch.empty_like(dy)
     h2d = x_h.numel() * 2 + (0 if fwd_only else dy_h.numel() * 2)
     d2h = sum(t.numel() * t.element_size() for t in outs_h)
-    e_steps = max(2, min(args.steps, 10))
+    e_steps = max(4, min(args.steps, 20))
+    ins = [(torch.empty_like(x), torch.empty_like(dy)) for _ in range(2)]
+    res = [tuple(torch.empty_like(t) for t in outs) for _ in range(2)]
+
+    def step_into(xin, dyin, out):
+        if fwd_only:
+            H.hcw_stack_fwd(xin, Ws, Wn, bias, 0, dim_over, flags, y=out[0], acts=acts,
+                            masks=masks, workspace=ws)
+        else:
+            H.hcw_stack_train_step(xin, Ws, Wn, bias, dyin, 0, dim_over, flags, y=y, acts=acts,
+                                   masks=masks, dx=dx, dW_self=out[0], dW_nbr=out[1],
+                                   dbias=out[2], workspace=ws)
+
+    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+    ev = {k: [torch.cuda.Event() for _ in range(2)] for k in ("in", "used", "out", "sent")}
     torch.cuda.synchronize()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    a.record(stream)
+    s_in.record_event(a)
+
+    def load(i):
+        k = i % 2
+        with torch.cuda.stream(s_in):
+            if i >= 2:
+                s_in.wait_event(ev["used"][k])       # step i - 2 has read this pair
+            ins[k][0].copy_(x_h, non_blocking=True)
+            if not fwd_only:
+                ins[k][1].copy_(dy_h, non_blocking=True)
+            s_in.record_event(ev["in"][k])
+
+    load(0)
     for i in range(e_steps):
+        k = i % 2
+        if i + 1 < e_steps:
+            load(i + 1)
+        stream.wait_event(ev["in"][k])
+        if i >= 2:
+            stream.wait_event(ev["sent"][k])         # step i - 2's result has left
         flush.fill_(i & 0xFF)
-        x_d.copy_(x_h, non_blocking=True)
-        if not fwd_only:
-            dy_d.copy_(dy_h, non_blocking=True)
-        step(x_d, dy_d)
-        for th, t in zip(outs_h, outs):
-            th.copy_(t, non_blocking=True)
-    b.record(stream)
+        step_into(ins[k][0], ins[k][1], res[k])
+        stream.record_event(ev["used"][k])
+        stream.record_event(ev["out"][k])
+        with torch.cuda.stream(s_out):
+            s_out.wait_event(ev["out"][k])
+            for th, t in zip(outs_h, res[k]):
+                th.copy_(t, non_blocking=True)
+            s_out.record_event(ev["sent"][k])
+    s_out.wait_stream(s_in)
+    s_out.wait_stream(stream)
+    s_out.record_event(b)
     torch.cuda.synchronize()
     e2e_ms = a.elapsed_time(b) / e_steps
+    if H.hcw_sync_status() != H.HCW_OK:
+        raise SystemExit("device error during the end-to-end run")
+    if not all(torch.equal(th.to(dev), t) for th, t in zip(outs_h, res[(e_steps - 1) % 2])):
+        raise SystemExit("end-to-end results differ from the ones on the device")
 
     # the oracle on the host cores, a bounded sample: whole sequences of the
     # workload for n <= 256, else one layer of one n = 256 sequence (the cost
@@ -860,7 +903,9 @@ def run_workload(args):
             "e2e": {"value": world * tokens / (e2e_ms * 1e-3), "unit": "tokens/s",
                     "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                     "ms_per_step": e2e_ms,
-                    "copies": "pinned host buffers, serial: inputs in, step, result out"},
+                    "copies": "pinned host buffers; step i+1's inputs and step i's result "
+                              "copied on two streams while the steps compute "
+                              "(double-buffered); L2 flushed every step inside the span"},
             "gpu_launches": launches,
             "clocks": clocks,
         }), flush=True)
