@@ -101,18 +101,24 @@ struct __align__(8) Barriers {
     int pub_done[2][kUnitQ];
 };
 
-// Stages of the pair variant of the row kernels: this CTA's A and half of B.
-__host__ __device__ constexpr int pair_row_stage_bytes(int BN) { return kABytes + BN * kBlockK; }
-__host__ __device__ constexpr int tc_pair_stages(int BN) {
-    return (kRingBytes / pair_row_stage_bytes(BN)) > 8 ? 8 : (kRingBytes / pair_row_stage_bytes(BN));
-}
-
-// epilogue patch buffers and bias slices (MODE_DWF stores from registers)
+// epilogue patch buffers (MODE_DWF stores from registers)
 template <int MODE, int BN>
 __host__ __device__ constexpr size_t epi_smem_bytes() {
-    return MODE == MODE_DWF ? 0
-                            : (size_t)epi_warps(BN) * kEpiBufBytes +
-                                  (size_t)epi_warps(BN) * warp_cols(BN) * 4;
+    return MODE == MODE_DWF ? 0 : (size_t)epi_warps(BN) * kEpiBufBytes;
+}
+
+// Stages of the pair variant of the row kernels: this CTA's A and half of B,
+// as many as the shared memory left by the epilogue buffers holds (at most 8;
+// five at BN = 256, six at BN = 128).
+constexpr size_t kSmemBudget = 232448;
+__host__ __device__ constexpr int pair_row_stage_bytes(int BN) { return kABytes + BN * kBlockK; }
+__host__ __device__ constexpr int tc_pair_stages(int BN) {
+    return (int)((kSmemBudget - 1024 - (size_t)epi_warps(BN) * kEpiBufBytes - sizeof(Barriers)) /
+                 pair_row_stage_bytes(BN)) > 8
+               ? 8
+               : (int)((kSmemBudget - 1024 - (size_t)epi_warps(BN) * kEpiBufBytes -
+                        sizeof(Barriers)) /
+                       pair_row_stage_bytes(BN));
 }
 
 template <int MODE, int BN, bool PAIR = false>
@@ -540,8 +546,7 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
     uint8_t* smem = reinterpret_cast<uint8_t*>(
         (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     uint8_t* epi_smem = smem + (size_t)STAGES * SB;               // 1024-aligned
-    float* bias_smem = reinterpret_cast<float*>(epi_smem + (DWF ? 0 : (size_t)EW * kEpiBufBytes));
-    Barriers* bars = reinterpret_cast<Barriers*>(bias_smem + (DWF ? 0 : EW * WCOLS));
+    Barriers* bars = reinterpret_cast<Barriers*>(epi_smem + (DWF ? 0 : (size_t)EW * kEpiBufBytes));
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -999,7 +1004,6 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
         const int quarter = warp & 3;
         const int cslice = e >> 2;
         uint8_t* buf = epi_smem + (size_t)e * kEpiBufBytes;
-        float* wbias = bias_smem + e * WCOLS;
         if (STACKED && e == EW - 1)
             for (int i = kTcMaps + lane; i < L.n_layers * kTcMaps; i += 32)
                 tma_prefetch_desc(&L.maps[i / kTcMaps][i % kTcMaps]);
@@ -1278,12 +1282,13 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     mp[h] = (has_mprev && tok_row >= 0)
                                 ? __ldg(ly.mprev + (size_t)tok_row * wpr + (col0 >> 5) + h)
                                 : 0u;
-                if (fwd) {
-                    // this warp's bias slice, read back as warp-wide broadcasts
-                    for (int c = lane; c < WCOLS; c += 32)
-                        wbias[c] = ly.bias ? __ldg(ly.bias + col0 + c) : 0.f;
-                    __syncwarp();
-                }
+                // this warp's bias slice in registers, column h * 32 + lane in
+                // bias_reg[h], handed to the lanes by shuffles (no shared memory:
+                // the ring of the pair launches takes a fifth stage instead)
+                float bias_reg[SUB];
+#pragma unroll
+                for (int h = 0; h < SUB; ++h)
+                    bias_reg[h] = fwd && ly.bias ? __ldg(ly.bias + col0 + h * 32 + lane) : 0.f;
                 if (!wait_acc()) {
                     return false;
                 }
@@ -1294,21 +1299,21 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                     for (int h = 0; h < SUB; ++h) {
                         uint32_t raw[32];
                         load_acc(h * 32, raw);
-                        if (tok_row >= 0) {
-                            uint4* dst = reinterpret_cast<uint4*>(ly.zout + (size_t)tok_row * p.d +
-                                                                  col0 + h * 32);
 #pragma unroll
-                            for (int m = 0; m < 4; ++m) {
-                                uint32_t w[4];
+                        for (int m = 0; m < 4; ++m) {
+                            uint32_t w[4];
 #pragma unroll
-                                for (int i = 0; i < 4; ++i) {
-                                    const int e2 = 8 * m + 2 * i;
-                                    w[i] = pack_bf16x2(
-                                        __uint_as_float(raw[e2]) + wbias[h * 32 + e2],
-                                        __uint_as_float(raw[e2 + 1]) + wbias[h * 32 + e2 + 1]);
-                                }
-                                dst[m] = make_uint4(w[0], w[1], w[2], w[3]);
+                            for (int i = 0; i < 4; ++i) {
+                                const int e2 = 8 * m + 2 * i;
+                                w[i] = pack_bf16x2(
+                                    __uint_as_float(raw[e2]) +
+                                        __shfl_sync(0xffffffffu, bias_reg[h], e2),
+                                    __uint_as_float(raw[e2 + 1]) +
+                                        __shfl_sync(0xffffffffu, bias_reg[h], e2 + 1));
                             }
+                            if (tok_row >= 0)
+                                reinterpret_cast<uint4*>(ly.zout + (size_t)tok_row * p.d + col0 +
+                                                         h * 32)[m] = make_uint4(w[0], w[1], w[2], w[3]);
                         }
                     }
                 }
@@ -1350,20 +1355,15 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                             rw[2] = q4.z;
                             rw[3] = q4.w;
                         }
-                        float4 bb[2] = {make_float4(0.f, 0.f, 0.f, 0.f), make_float4(0.f, 0.f, 0.f, 0.f)};
-                        if (fwd) {
-                            const float4* b4 = reinterpret_cast<const float4*>(wbias + h * 32 + 8 * m);
-                            bb[0] = b4[0];
-                            bb[1] = b4[1];
-                        }
 #pragma unroll
                         for (int i = 0; i < 4; ++i) {
                             const int q = 4 * m + i;
                             uint64_t v2 = f32x2_pack(__uint_as_float(raw[2 * q]),
                                                      __uint_as_float(raw[2 * q + 1]));
                             if (fwd)
-                                v2 = f32x2_add(v2, i & 1 ? f32x2_pack(bb[i >> 1].z, bb[i >> 1].w)
-                                                         : f32x2_pack(bb[i >> 1].x, bb[i >> 1].y));
+                                v2 = f32x2_add(
+                                    v2, f32x2_pack(__shfl_sync(0xffffffffu, bias_reg[h], 2 * q),
+                                                   __shfl_sync(0xffffffffu, bias_reg[h], 2 * q + 1)));
                             const uint64_t r2 = bf16x2_to_f32x2(rw[i]);
                             if (relu) {
                                 // b = [z > 0] exactly as 1.0 / 0.0: z * 2^100 * 2^100 saturated
