@@ -806,8 +806,6 @@ size_t stack_data_ws(const Shape& sh, int dtype, unsigned flags, int L) {
     return 2 * a;
 }
 
-// bf16: [unit counter (256 B)][weight-gradient workspace][the readers' dz of a
-// shift layer (one activation buffer)]
 // True when `cnt` layers' whole-range weight-gradient units (one per output
 // tile) would leave most SMs idle: their launch then splits the token range
 // of every layer (split_dw_ws).
@@ -828,6 +826,9 @@ size_t split_dw_ws(const Shape& sh, unsigned flags, int cnt) {
     return part + bpart;
 }
 
+// bf16: [unit counter (256 B)][weight-gradient workspace][the readers' dz of a
+// shift layer (one activation buffer)], or [unit counter][the split launch's
+// partials] when that is larger
 size_t stack_weight_ws(const Shape& sh, int dtype, unsigned flags, int L) {
     const WsLayout w = ws_layout(sh.tokens, sh.d, dtype, flags);
     if (dtype != HCW_BF16) return w.w_bytes;
@@ -1077,10 +1078,6 @@ int stack_data_bf16(const Shape& sh, const StackData& a, cudaStream_t st) {
     return HCW_OK;
 }
 
-// bf16 weight gradients: runs of up to 16 independent layers in one launch
-// (whole token range per tile, units handed out longest first; the kernel
-// also sums dz's columns into dbias), or layer by layer when their tiles
-// cannot fill the GPU.
 // The weight gradients of layers l0 .. l0 + cnt - 1 when each has few output
 // tiles (small d): one launch whose units split every layer's token range
 // (units of one size over all the layers, claimed dynamically; the self
@@ -1154,6 +1151,12 @@ int split_dw_launch(const Shape& sh, const StackWeight& a, int l0, int cnt, uint
     return rc;
 }
 
+// bf16 weight gradients: runs of up to 16 independent layers in one launch
+// (whole token range per tile, units handed out longest first; the kernel
+// also sums dz's columns into dbias), or, when their tiles cannot fill the
+// GPU, one launch over token splits of every layer (split_dw_launch); a
+// schedule with shift layers that cannot take the batched launch runs layer
+// by layer.
 int stack_weight_bf16(const Shape& sh, const StackWeight& a, cudaStream_t st) {
     const int d = sh.d, BN = pick_bn(d), L = a.L;
     const size_t ab = sh.act_bytes;

@@ -1876,6 +1876,11 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
             const int ot = 2 * tp + (int)rank;
             const TcLayer& ly = L.layer[l];
             const bool last = u + n_pairs >= n_units;   // no further unit: the ring goes idle
+            // the output maps of the last unit's staged stores, fetched while it runs
+            if (last && e == EW - 1 && lane == 0) {
+                tma_prefetch_desc(&L.maps[l][4]);
+                tma_prefetch_desc(&L.maps[l][5]);
+            }
             if (e < kDwHelpers) {
                 // release this CTA's stages once the pair's MMAs have read them, and
                 // sum the dz tile's columns on the way (dbias, output rows of tile ot)
