@@ -309,7 +309,11 @@ size_t hcw_stack_bwd_data_workspace_bytes(int B, int n, int d, int dtype, unsign
  *   dbias[l] = sum_i dz_l,i (dbias may be NULL).  fp32 outputs [L][d][d], [L][d].
  *   workspace: at least hcw_stack_bwd_weight_workspace_bytes(...) bytes.
  * bf16: up to 16 layers per launch, whole token range per tile (no split
- * reduction, deterministic); the same kernel sums dz's columns into dbias.
+ * reduction); the same kernel sums dz's columns into dbias.  Layers with few
+ * output tiles (small d, few layers: fewer than 76 tiles in the launch)
+ * instead split every layer's token range over one launch and add the fp32
+ * partials of weights and dbias in a second one, in split order.  Either way
+ * deterministic: the same inputs give the same bits.
  */
 int hcw_stack_bwd_weight(const void* x, const void* acts, const void* dz, int layer0, int L,
                          int dim_override, int B, int n, int d, int dtype, unsigned flags,

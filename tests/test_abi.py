@@ -278,9 +278,34 @@ def test_schedule_entry_points_reject_bad_dims_before_any_launch(hcw):
         rc = lib.hcw_stack_bwd_dims(fake, fake, None, fake, fake, fake, ptr, L, B, n, d,
                                     hcw.HCW_BF16, 0, fake, fake, fake, None, None, 0, None)
         assert rc == hcw.HCW_ERR_INVALID_ARG, dims
+        rc = lib.hcw_stack_bwd_weight_dims(fake, fake, fake, ptr, L, B, n, d, hcw.HCW_BF16, 0,
+                                           fake, fake, None, None, 0, None)
+        assert rc == hcw.HCW_ERR_INVALID_ARG, dims
+        rc = lib.hcw_stack_train_step_dims(fake, fake, fake, None, fake, ptr, L, B, n, d,
+                                           hcw.HCW_BF16, 0, fake, fake, fake, fake, fake, fake,
+                                           None, None, 0, None)
+        assert rc == hcw.HCW_ERR_INVALID_ARG, dims
     assert hcw.hcw_launch_count() == before
     with pytest.raises(ValueError):
         hcw._dims_array([0, 1, 2], 4)
+
+
+def test_small_d_weight_gradient_workspace_holds_the_split_partials(hcw):
+    """Few output tiles (d = 128 or 256): the layers' weight gradients split the
+    token range over one launch, so the workspace holds fp32 partial weight
+    tiles and dbias partials of every layer of the launch; it grows with the
+    layer count (up to 16 a launch), and the training step's workspace holds
+    it."""
+    B, n = 256, 64
+    for d in (128, 256):
+        one = hcw.hcw_stack_bwd_weight_workspace_bytes(B, n, d, hcw.HCW_BF16, 7, 1)
+        six = hcw.hcw_stack_bwd_weight_workspace_bytes(B, n, d, hcw.HCW_BF16, 7, 6)
+        sixteen = hcw.hcw_stack_bwd_weight_workspace_bytes(B, n, d, hcw.HCW_BF16, 7, 16)
+        assert 0 < one <= six <= sixteen
+        # at least two splits of two d x d fp32 parts per layer
+        assert six >= 6 * 2 * 2 * d * d * 4
+        step = hcw.hcw_stack_train_step_workspace_bytes(B, n, d, hcw.HCW_BF16, 7, 6)
+        assert step >= six
 
 
 def test_decode_cache_is_bounded_by_the_link_distances(hcw):
