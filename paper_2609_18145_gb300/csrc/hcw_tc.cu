@@ -1674,7 +1674,13 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
     constexpr int EW = epi_warps(BN);
     constexpr int WCOLS = warp_cols(BN);
     static_assert(STAGES % 2 == 0 && STAGES >= 2, "pairs of stages");
-    static_assert(EW * 2 * kEpiBufBytes <= STAGES * SB, "patch buffers inside the ring");
+    // the last unit's staging buffers per epilogue warp: as many 4 KB patches as
+    // the idle ring holds, up to the warp's four stores
+    constexpr int NBUF = (STAGES * SB) / (EW * kEpiBufBytes) >= 4
+                             ? 4
+                             : (STAGES * SB) / (EW * kEpiBufBytes);
+    static_assert(NBUF >= 2 && EW * NBUF * kEpiBufBytes <= STAGES * SB,
+                  "patch buffers inside the ring");
     const TcParams& p = L.p;
     const uint32_t rank = cluster_ctarank();
     const int pair = (int)blockIdx.x >> 1, n_pairs = (int)gridDim.x >> 1;
@@ -1690,9 +1696,14 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
     const int lane = threadIdx.x & 31;
 
     if (threadIdx.x == 0) {
-        for (int l = 0; l < L.n_layers; ++l) {
+        // the operand maps of this pair's own units only (one unit a pair in
+        // the training step), in the order the units come
+        for (int u = pair; u < n_units; u += n_pairs) {
+            const int lu = u / upl;
+            const int l = L.dep_counters != nullptr ? L.n_layers - 1 - lu : lu;
             tma_prefetch_desc(&L.maps[l][0]);
             tma_prefetch_desc(&L.maps[l][1]);
+            if (SHIFT && L.layer[l].shift > 0) tma_prefetch_desc(&L.maps[l][2]);
         }
         for (int s = 0; s < STAGES; ++s) {
             mbar_init(&bars->full[s], 1);
@@ -1944,14 +1955,14 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
             }
             tc_fence_after();
             // The CTA's last unit: the ring is idle once the helper warps are done
-            // with it, so the tiles go out through shared memory by TMA (two 4 KB
+            // with it, so the tiles go out through shared memory by TMA (NBUF 4 KB
             // patch buffers per warp, whole 128-byte rows): per-lane row stores at
             // the end of the launch, all SMs at once, took ~13 us to drain.
             // Earlier units store from registers while the next unit's operands
             // stream into the ring.
             const bool staged =
                 last && __all_sync(0xffffffffu, mbar_wait(&bars->ring_idle, 0, abort, tmo));
-            uint8_t* sbuf = smem + (size_t)e * 2 * kEpiBufBytes;
+            uint8_t* sbuf = smem + (size_t)e * NBUF * kEpiBufBytes;
             int nbuf = 0;
             // this CTA's 128 rows of the tile: one row per lane, 32 fp32 columns per load
             const int row = ot * kBlockM + quarter * 32 + lane;
@@ -1972,9 +1983,9 @@ __global__ void __launch_bounds__(cta_threads(BN), 1)
                         if (lane == 0) mbar_arrive_remote_tmem(tempty_leader);
                     }
                     if (staged) {
-                        uint8_t* buf = sbuf + (nbuf & 1) * kEpiBufBytes;
+                        uint8_t* buf = sbuf + (nbuf % NBUF) * kEpiBufBytes;
                         // the buffer's store before last has been read
-                        if (lane == 0 && nbuf >= 2) bulk_wait_read<1>();
+                        if (lane == 0 && nbuf >= NBUF) bulk_wait_read<NBUF - 1>();
                         __syncwarp();
 #pragma unroll
                         for (int m = 0; m < 8; ++m)
