@@ -237,6 +237,10 @@ STACK_CASES = [
      CAUSAL | RESIDUAL | RELU, (1 / 512) ** 0.5),
     ("n64_d256_bf16_odd_row_blocks_noncausal", torch.bfloat16, 10, 64, 256, 6,
      RESIDUAL, (1 / 512) ** 0.5),
+    # d = 192: 64-column tiles and a ragged 128-row o tile in the weight
+    # gradient, whose few tiles take the launch over token splits of every layer
+    ("n64_d192_bf16_split_weight_gradient", torch.bfloat16, 4, 64, 192, 5,
+     CAUSAL | RESIDUAL | RELU, (1 / 384) ** 0.5),
 ]
 
 
