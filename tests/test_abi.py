@@ -435,3 +435,20 @@ def test_decode_kernel_switch(hcw):
         assert L.hcw_set_decode_kernel(hcw.HCW_DECODE_WARP_MMA) == hcw.HCW_DECODE_TCGEN05
     finally:
         L.hcw_set_decode_kernel(prev)
+
+
+def test_compute_calls_take_device_tensors_only(hcw):
+    """No CPU fallback: the compute entry points of the binding reject host
+    tensors before anything reaches the library."""
+    import torch
+    x = torch.zeros(2, 16, 64, dtype=torch.bfloat16)
+    W = torch.zeros(1, 64, 64, dtype=torch.bfloat16)
+    before = hcw.hcw_launch_count()
+    calls = (lambda: hcw.hcw_layer_fwd(x, W[0], W[0]),
+             lambda: hcw.hcw_stack_fwd(x, W, W),
+             lambda: hcw.hcw_stack_train_step(x, W, W, None, x),
+             lambda: hcw.hcw_stack_bwd_weight(x, None, W.reshape(1, 1, 64, 64)))
+    for call in calls:
+        with pytest.raises(ValueError, match="CUDA tensors"):
+            call()
+    assert hcw.hcw_launch_count() == before
